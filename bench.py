@@ -1,0 +1,427 @@
+"""Benchmark of the SAO loss head on GB300: one step = one pass of the whole
+hot path over one packed batch:
+
+    sao_advantages -> sao_value_loss -> sao_token_logprobs_fwd ->
+    sao_policy_loss_fwd -> sao_policy_loss_bwd -> sao_token_logprobs_bwd
+
+on the MoE-policy head shape (hidden 2048, vocabulary 151936, bf16, 65536
+packed tokens of single-rollout agentic trajectories). Prints one JSON line.
+
+    python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+
+Under torchrun each rank processes its own batch (weak scaling, trajectories
+sharded across ranks, no collective on the data path); rank 0 prints the
+whole-job tokens/s over the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "loss-head tokens/s (fwd+bwd) at h=2048,V=151936 bf16; % bf16 tensor peak"
+UNIT = "tokens/s"
+WORKLOAD = "moe"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ---------------------------------------------------------------------------
+# clocks sampled with nvidia-smi during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, mx, power, reasons = [], [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+                power.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[4:8]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "power_w_max": max(power) if power else None, "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------------------
+# the step
+# ---------------------------------------------------------------------------
+class LossHeadStep:
+    """Device buffers and the six ABI calls of one loss-head step."""
+
+    def __init__(self, wl, device, torch):
+        from paper_2607_07508_gb300 import sao
+        self.sao = sao
+        self.torch = torch
+        self.wl = wl
+        N, h, V = wl.N, wl.h, wl.V
+        f32 = torch.float32
+        dev = device
+        self.H = wl.H
+        self.W = wl.W
+        self.y = torch.as_tensor(wl.y).to(dev)
+        self.mask = torch.as_tensor(wl.loss_mask).to(dev)
+        self.values = torch.as_tensor(wl.values).to(dev)
+        self.rewards = torch.as_tensor(wl.rewards).to(dev)
+        self.cu = torch.as_tensor(wl.cu_seqlens).to(dev)
+        self.adv = torch.empty(N, dtype=f32, device=dev)
+        self.ret = torch.empty(N, dtype=f32, device=dev)
+        self.logp = torch.empty(N, dtype=f32, device=dev)
+        self.lse = torch.empty(N, dtype=f32, device=dev)
+        self.coef = torch.empty(N, dtype=f32, device=dev)
+        self.flags = torch.empty(N, dtype=torch.uint8, device=dev)
+        self.G = torch.empty(N, dtype=f32, device=dev)
+        self.dV = torch.empty(N, dtype=f32, device=dev)
+        self.loss = torch.empty(1, dtype=f32, device=dev)
+        self.vloss = torch.empty(1, dtype=f32, device=dev)
+        self.counts = torch.empty(4, dtype=torch.int64, device=dev)
+        self.ev = torch.empty(4, dtype=torch.float64, device=dev)
+        self.one = torch.ones(1, dtype=f32, device=dev)
+        self.dH = torch.empty_like(self.H)
+        self.dW = torch.empty(V, h, dtype=f32, device=dev)
+        self.ws = sao.workspace(N, h, V, self.H.dtype, device=dev)
+        # The rollout policy's log-probs: the current policy's, perturbed by the
+        # workload's staleness noise (prepared once, outside any timing).
+        sao.sao_token_logprobs_fwd(self.H, self.W, self.y, self.logp, self.lse, self.ws)
+        self.old = (self.logp + torch.as_tensor(wl.xi).to(dev)).contiguous()
+
+    def run(self):
+        s, wl = self.sao, self.wl
+        s.sao_advantages(self.values, self.rewards, self.mask, self.cu, wl.gamma, wl.lam, wl.lam_critic, wl.alpha,
+                         self.adv, self.ret, self.ws)
+        s.sao_value_loss(self.values, self.ret, self.mask, self.vloss, self.dV, self.ws, ev_sums=self.ev)
+        s.sao_token_logprobs_fwd(self.H, self.W, self.y, self.logp, self.lse, self.ws)
+        s.sao_policy_loss_fwd(self.logp, self.old, self.adv, self.mask, wl.eps_low, wl.eps_high, self.loss,
+                              self.counts, self.ws, coef=self.coef, flags=self.flags)
+        s.sao_policy_loss_bwd(self.logp, self.old, self.adv, self.mask, wl.eps_low, wl.eps_high, self.one, self.G,
+                              self.ws)
+        s.sao_token_logprobs_bwd(self.H, self.W, self.y, self.lse, self.G, self.dH, self.dW, self.ws)
+
+
+# Algorithmic work per launch of each tensor-core kernel, in flops, for N rows.
+def kernel_flops(name, N, h, V, rows_g):
+    if name == "tc_logits_lse_fwd":
+        return 2.0 * N * h * V
+    if name in ("tc_dlogits", "tc_dH_gemm", "tc_dW_gemm"):
+        return 2.0 * N * h * V
+    return None
+
+
+# ---------------------------------------------------------------------------
+# CPU baseline: the fp64 oracle on a bounded sample of the same workload
+# ---------------------------------------------------------------------------
+def cpu_baseline(wl, rows: int, H_cpu=None, W_cpu=None):
+    """Times the oracle on `rows` sampled tokens (all three GEMMs over the full
+    vocabulary) and on all N tokens for the O(N) parts; returns tokens/s
+    extrapolated to the N-token step."""
+    from oracle import sao_oracle as O
+    rng = np.random.default_rng(0)
+    idx = np.sort(rng.choice(wl.N, size=rows, replace=False))
+    Hs = (H_cpu if H_cpu is not None else wl.H.cpu())[idx]
+    Wc = W_cpu if W_cpu is not None else wl.W.cpu()
+    ys = wl.y[idx]
+    t0 = time.perf_counter()
+    adv, ret = O.advantages(wl.values, wl.rewards, wl.loss_mask, wl.cu_seqlens, wl.gamma, wl.lam, wl.lam_critic,
+                            wl.alpha)
+    O.value_loss(wl.values, ret, wl.loss_mask)
+    t_on = time.perf_counter() - t0
+    t1 = time.perf_counter()
+    logp, lse = O.token_logprobs(Hs, Wc, ys)
+    old = logp + wl.xi[idx]
+    pl = O.policy_loss(logp, old, adv[idx], wl.loss_mask[idx], wl.eps_low, wl.eps_high)
+    G = O.policy_loss_bwd(logp, old, adv[idx], wl.loss_mask[idx], wl.eps_low, wl.eps_high, 0, 1.0)
+    O.token_logprobs_bwd(Hs, Wc, ys, lse, G)
+    t_gemm = time.perf_counter() - t1
+    t_step = t_on + t_gemm * (wl.N / rows)
+    cores = os.cpu_count() or 1
+    return {"value": wl.N / t_step, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": (f"fp64 numpy oracle: advantages + value loss on all {wl.N} tokens ({t_on:.2f} s), "
+                       f"log-prob fwd + policy loss + log-prob bwd on {rows} sampled tokens over the full "
+                       f"vocabulary ({t_gemm:.2f} s), extrapolated linearly to {wl.N} tokens; BLAS threads = "
+                       f"host cores"),
+            "measured_s": t_on + t_gemm, "_pl": pl["loss"]}
+
+
+def choose_rows(wl, H_cpu, W_cpu, budget_s=15.0):
+    from oracle import sao_oracle as O
+    r = 8
+    t0 = time.perf_counter()
+    lp, lse = O.token_logprobs(H_cpu[:r], W_cpu, wl.y[:r])
+    O.token_logprobs_bwd(H_cpu[:r], W_cpu, wl.y[:r], lse, np.ones(r))
+    dt = time.perf_counter() - t0
+    rows = int(max(8, min(512, r * budget_s / max(dt, 1e-3))))
+    return rows
+
+
+# ---------------------------------------------------------------------------
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    from paper_2607_07508_gb300 import synthetic as S
+    import torch
+    wl = S.make_workload(WORKLOAD, device="cpu")
+    H_cpu, W_cpu = wl.H, wl.W
+    rows = max(8, choose_rows(wl, H_cpu, W_cpu, budget_s=8.0) // 2)
+    for _ in range(args.warmup if args.warmup < 1 else 1):
+        cpu_baseline(wl, 8, H_cpu, W_cpu)
+    vals = []
+    cb = None
+    for _ in range(args.steps):
+        cb = cpu_baseline(wl, rows, H_cpu, W_cpu)
+        vals.append(cb["value"])
+    value = statistics.median(vals)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * wl.N / value,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": workload_config(wl),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cb["cores"], "kind": "oracle",
+                             "sample": cb["sample"]},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+def workload_config(wl):
+    return {"workload": f"{wl.name}: MoE-policy head, {wl.N} packed tokens in {wl.B} single-rollout agentic "
+                        f"trajectories (lognormal lengths, median 4k, max 32k), 25% observation tokens",
+            "tokens": wl.N, "trajectories": wl.B, "hidden": wl.h, "vocab": wl.V, "dtype": wl.dtype,
+            "gamma": wl.gamma, "lambda": wl.lam, "eps_low": wl.eps_low, "eps_high": wl.eps_high,
+            "l2": "inputs larger than L2 (H 268 MB + W 622 MB per step, L2 126 MB); no flush"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    from paper_2607_07508_gb300 import sao, synthetic as S
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    sao.load()
+    peaks, peak_src = load_peaks()
+
+    wl = S.make_workload(WORKLOAD, device=dev, seed=S.SEED_BASE + S.CONFIG_NAMES.index(WORKLOAD) + 97 * rank)
+    step = LossHeadStep(wl, dev, torch)
+    stream = torch.cuda.current_stream()
+    for _ in range(max(3, args.warmup)):
+        step.run()
+    torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    # ---- timed region (device-resident inputs) --------------------------------
+    sao.sao_profile_enable(True)
+    sao.sao_profile_reset()
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step.run()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    prof = sao.sao_profile_read()
+    sao.sao_profile_enable(False)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    total_tokens = wl.N * world
+    value = total_tokens / (ms / 1000.0)
+
+    # ---- roofline of the dominant kernel --------------------------------------
+    launches = sum(n for n, _ in prof.values())
+    dom = max(prof.items(), key=lambda kv: kv[1][1])
+    dom_name, (dom_n, dom_ms) = dom
+    avg_ms = dom_ms / dom_n
+    fl = kernel_flops(dom_name, wl.N, wl.h, wl.V, None)
+    peak_t = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    if fl is not None:
+        achieved = fl / (avg_ms / 1000.0) / 1e12
+        roofline = {"bound": "tensor", "kernel": dom_name, "achieved": achieved, "peak": peak_t,
+                    "unit": "TFLOP/s", "frac": achieved / peak_t, "traffic": None,
+                    "algorithmic_per_launch": f"2*N*h*V = {fl:.4g} flop", "avg_launch_ms": avg_ms,
+                    "peak_source": f"{peak_src} bf16_tflops_sustained (kernel timed inside a long step)"}
+    else:
+        roofline = {"bound": "hbm", "kernel": dom_name, "achieved": None, "peak": peaks.get("hbm_gbs"),
+                    "unit": "GB/s", "frac": None, "traffic": None}
+    step_alg = 6.0 * wl.N * wl.h * wl.V
+    step_exec = 8.0 * wl.N * wl.h * wl.V
+    burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+    step_roof = {"algorithmic_tflops": step_alg / (ms / 1000) / 1e12,
+                 "frac_of_burst_peak": step_alg / (ms / 1000) / 1e12 / burst,
+                 "executed_tflops": step_exec / (ms / 1000) / 1e12,
+                 "executed_frac_of_sustained_peak": step_exec / (ms / 1000) / 1e12 / peak_t,
+                 "algorithmic_flops_per_step": "6*N*h*V (2hV fwd + 4hV bwd per token)",
+                 "executed_flops_per_step": "8*N*h*V (the backward recomputes the logits)",
+                 "peak_source": peak_src}
+    kernels = {k: {"launches": n, "avg_ms": t / n} for k, (n, t) in sorted(prof.items(), key=lambda kv: -kv[1][1])}
+
+    # ---- end to end through the ABI with host buffers ---------------------------
+    e2e = None
+    if not args.no_e2e:
+        host = {
+            "H": torch.empty(step.H.shape, dtype=step.H.dtype, pin_memory=True),
+            "y": torch.empty(wl.N, dtype=torch.int32, pin_memory=True),
+            "old": torch.empty(wl.N, dtype=torch.float32, pin_memory=True),
+            "values": torch.empty(wl.N, dtype=torch.float32, pin_memory=True),
+            "rewards": torch.empty(wl.B, dtype=torch.float32, pin_memory=True),
+            "mask": torch.empty(wl.N, dtype=torch.uint8, pin_memory=True),
+            "cu": torch.empty(wl.B + 1, dtype=torch.int32, pin_memory=True),
+        }
+        host["H"].copy_(step.H)
+        host["y"].copy_(step.y)
+        host["old"].copy_(step.old)
+        host["values"].copy_(step.values)
+        host["rewards"].copy_(step.rewards)
+        host["mask"].copy_(step.mask)
+        host["cu"].copy_(step.cu)
+        out = torch.empty(1 + 1 + 4 * 2, dtype=torch.float32, pin_memory=True)
+        dst = {"H": step.H, "y": step.y, "old": step.old, "values": step.values, "rewards": step.rewards,
+               "mask": step.mask, "cu": step.cu}
+        h2d = sum(t.numel() * t.element_size() for t in host.values())
+        d2h = out.numel() * out.element_size()
+        res = torch.empty(10, dtype=torch.float32, device=dev)
+        torch.cuda.synchronize()
+        barrier()
+        e2 = torch.cuda.Event(enable_timing=True)
+        e3 = torch.cuda.Event(enable_timing=True)
+        t_wall = time.perf_counter()
+        e2.record(stream)
+        for _ in range(args.steps):
+            for k, t in host.items():
+                dst[k].copy_(t, non_blocking=True)
+            step.run()
+            res[0:1].copy_(step.loss)
+            res[1:2].copy_(step.vloss)
+            res[2:10].copy_(step.counts.view(torch.float32))
+            out.copy_(res, non_blocking=True)
+        e3.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        ms_e2e = e2.elapsed_time(e3) / args.steps
+        if world > 1:
+            t = torch.tensor([ms_e2e], device=dev)
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            ms_e2e = float(t.item())
+        e2e = {"value": total_tokens / (ms_e2e / 1000.0), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e,
+               "note": "pinned host H, token ids, rollout log-probs, values, rewards, mask and cu_seqlens copied in, "
+                       "loss, value loss and counts copied out, every step; W stays resident (model weight)"}
+
+    # ---- CPU baseline (rank 0, single GPU only) ---------------------------------
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        H_cpu, W_cpu = step.H.cpu(), step.W.cpu()
+        rows = choose_rows(wl, H_cpu, W_cpu)
+        cpu = cpu_baseline(wl, rows, H_cpu, W_cpu)
+        cpu.pop("_pl", None)
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+                "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": workload_config(wl),
+                "roofline": roofline, "step_roofline": step_roof, "cpu_baseline": cpu, "e2e": e2e,
+                "clocks": clk, "gpu_launches": launches * 1, "gpu_launches_per_step": launches / args.steps,
+                "kernels": kernels}
+        print(json.dumps(line))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,209 @@
+/*
+ * sao.h -- C ABI of the SAO per-token RL loss head on one GB300 (sm_103a).
+ *
+ * The operations follow "Single-Rollout Asynchronous Optimization for Agentic
+ * Reinforcement Learning" (arxiv 2607.07508):
+ *   - sao_token_logprobs_fwd/bwd : log pi_theta(a_t|s_t) of Eq. 1-2 from the
+ *     LM head (logits H W^T, log-softmax, gather), vocabulary-chunked so the
+ *     [N, V] logits are never stored, and its gradient;
+ *   - sao_policy_loss_fwd/bwd    : the DIS ratio of Eq. 2 against the rollout
+ *     log-probs, the strict double-sided calibration f of Eq. 3 and the token
+ *     objective of Eq. 1 (§3.1), with the clip-ratio counts of §4.4;
+ *   - sao_advantages             : token-level GAE (Preliminaries) with the
+ *     skip-observation link of Eq. 4-5 (§3.2) and the length-adaptive lambda
+ *     of §4.1, as a reverse scan over packed trajectories;
+ *   - sao_value_loss             : the value error (V - R)^2 (Preliminaries)
+ *     and the explained-variance sums of §4.4.
+ *
+ * Conventions shared by every entry point:
+ *   - Every array argument is a DEVICE pointer owned by the caller; the
+ *     library never allocates, frees or keeps a pointer past the call.
+ *   - Scratch space comes from the caller's workspace `ws` of `ws_bytes`
+ *     bytes, 256-byte aligned, of at least sao_workspace_bytes(...) bytes.
+ *     Its contents on entry do not matter; one workspace must not be used by
+ *     two calls that overlap on the GPU.
+ *   - Each call only enqueues kernels on `stream` (a cudaStream_t; NULL is
+ *     the legacy default stream) and returns without waiting, unless checked
+ *     mode is on (sao_set_checked), in which case it synchronises the stream
+ *     and reports device-side validation failures as SAO_ERR_DEVICE_CHECK.
+ *   - Errors are returned as sao_status; no exception crosses the ABI; the
+ *     last error message is available from sao_last_error_string().
+ *   - N is the number of packed tokens; row t of H predicts token y[t] (the
+ *     caller does the shift). Per-token floating point arrays are fp32;
+ *     token ids and cu_seqlens are int32; counts are int64.
+ *   - Arrays are contiguous (row-major for matrices). Vectorised paths need
+ *     16-byte aligned pointers; other alignments take a scalar path.
+ */
+#ifndef SAO_H_
+#define SAO_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SAO_API __attribute__((visibility("default")))
+#else
+#define SAO_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *sao_stream_t; /* a cudaStream_t */
+
+typedef enum sao_status {
+  SAO_OK = 0,
+  SAO_ERR_INVALID_ARG = 1,  /* null pointer, bad scalar, misaligned workspace */
+  SAO_ERR_SHAPE = 2,        /* inconsistent or unsupported sizes */
+  SAO_ERR_WORKSPACE = 3,    /* ws_bytes smaller than required */
+  SAO_ERR_UNSUPPORTED = 4,  /* dtype, or a device that is not sm_103 */
+  SAO_ERR_CUDA = 5,         /* a CUDA runtime or driver call failed */
+  SAO_ERR_DEVICE_CHECK = 6  /* checked mode: the device flagged bad input */
+} sao_status;
+
+typedef enum sao_dtype {
+  SAO_F32 = 0,   /* fp32 H, W, dH (fp32 FMA path) */
+  SAO_BF16 = 1   /* bf16 H, W, dH (tcgen05 tensor-core path, fp32 accumulate) */
+} sao_dtype;
+
+/* Per-token flag values written by sao_policy_loss_fwd (Eq. 3). */
+#define SAO_FLAG_IN 0        /* 1 - eps_low < r < 1 + eps_high: kept, f(r) = r */
+#define SAO_FLAG_LOW 1       /* r <= 1 - eps_low: masked, f(r) = 0 */
+#define SAO_FLAG_HIGH 2      /* r >= 1 + eps_high: masked, f(r) = 0 */
+#define SAO_FLAG_NONFINITE 3 /* log-ratio or advantage not finite: masked */
+#define SAO_FLAG_NOT_ACTION 4/* loss_mask == 0 (prompt / observation token) */
+
+/* Device-side error bits (checked mode), OR-ed into one word. */
+#define SAO_DEVERR_TOKEN_ID 0x1u     /* some y[t] outside [0, V) */
+#define SAO_DEVERR_CU_SEQLENS 0x2u   /* cu_seqlens not 0..N non-decreasing */
+#define SAO_DEVERR_SCAN_TIMEOUT 0x4u /* advantage scan gave up waiting for a carry */
+#define SAO_DEVERR_PIPE_TIMEOUT 0x8u /* a GEMM pipeline wait gave up */
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+SAO_API int sao_version(void);
+
+/* Message for the most recent non-OK status on the calling host thread. */
+SAO_API const char *sao_last_error_string(void);
+
+/* Checked mode (off by default): every call synchronises its stream, reads
+ * and clears the device error word, and returns SAO_ERR_DEVICE_CHECK if it is
+ * non-zero. Process-wide setting. */
+SAO_API void sao_set_checked(int on);
+SAO_API int sao_get_checked(void);
+
+/* Upper bound on the bf16 dZ chunk buffer of sao_token_logprobs_bwd
+ * (default 24 GiB). Smaller budgets split the vocabulary into more chunks and
+ * add an fp32 dH accumulator. Affects sao_workspace_bytes. Process-wide. */
+SAO_API void sao_set_dz_budget_bytes(size_t bytes);
+
+/* Workspace bytes that every entry point needs for N tokens, hidden size h,
+ * vocabulary V and dtype dt (pass h = V = 0 when only the O(N) calls are
+ * used). Returns 0 for invalid sizes. */
+SAO_API size_t sao_workspace_bytes(int64_t N, int32_t h, int32_t V, sao_dtype dt);
+
+/*
+ * Eq. 1-2: logp[t] = z[t, y[t]] - lse[t], z = H W^T, lse[t] = log sum_v e^z[t,v].
+ *   H        [N, h] dt, row-major          W  [V, h] dt, row-major
+ *   y        [N] int32 in [0, V)           row_mask [N] uint8 or NULL: rows
+ *            with row_mask[t] == 0 are not computed and get logp = lse = 0
+ *   logp,lse [N] fp32 outputs (lse is kept for the backward)
+ * Sizes: N >= 0; 1 <= V; h >= 1; for bf16, h % 8 == 0 (TMA row pitch).
+ * A token id outside [0, V) yields logp = NaN (and SAO_DEVERR_TOKEN_ID).
+ */
+SAO_API sao_status sao_token_logprobs_fwd(const void *H, const void *W, sao_dtype dt, const int32_t *y,
+                                  const uint8_t *row_mask, int64_t N, int32_t h, int32_t V,
+                                  float *logp, float *lse, void *ws, size_t ws_bytes,
+                                  sao_stream_t stream);
+
+/*
+ * Gradient of sum_t G[t] * logp[t] (G = grad_logp): with p = e^(z - lse),
+ * dZ[t, v] = G[t] * (1[v == y[t]] - p[t, v]); dH = dZ W; dW = dZ^T H.
+ *   lse       [N] fp32 from sao_token_logprobs_fwd on the same H, W, y
+ *   grad_logp [N] fp32; rows with grad_logp == 0 contribute nothing
+ *   dH        [N, h] dt output (overwritten)
+ *   dW        [V, h] fp32 output; overwritten if accumulate_dW == 0, else
+ *             the gradient is added to its contents
+ */
+SAO_API sao_status sao_token_logprobs_bwd(const void *H, const void *W, sao_dtype dt, const int32_t *y,
+                                  const float *lse, const float *grad_logp, int64_t N, int32_t h,
+                                  int32_t V, void *dH, float *dW, int accumulate_dW, void *ws,
+                                  size_t ws_bytes, sao_stream_t stream);
+
+/*
+ * Skip-observation GAE (Preliminaries; §3.2 Eq. 4-5; §4.1). For trajectory b
+ * (tokens cu_seqlens[b] .. cu_seqlens[b+1]-1) only action tokens
+ * (loss_mask == 1) take part; the Bellman successor of an action token is the
+ * next action token of the same trajectory, skipping observation tokens; the
+ * value after the last action token is 0 and rewards[b] is the reward of the
+ * last action token. delta_j = r_j + gamma V_next - V_j,
+ * A_j = delta_j + gamma lambda_b A_next, ret_j = GAE(lambda_critic)_j + V_j.
+ * lambda_b = lambda_policy, or 1 - 1/(alpha * L_b) clamped to [0,1] when
+ * len_adaptive_alpha = alpha > 0 (L_b = number of action tokens of b).
+ * Non-action tokens get adv = ret = 0. Computed in double-float (about 48
+ * significant bits) and rounded to fp32.
+ *   values [N] fp32, rewards [B] fp32, loss_mask [N] uint8,
+ *   cu_seqlens [B+1] int32 with 0 = cu[0] <= ... <= cu[B] = N
+ *   adv, ret [N] fp32 outputs
+ * Scalars: 0 <= gamma, lambda_policy, lambda_critic <= 1.
+ */
+SAO_API sao_status sao_advantages(const float *values, const float *rewards, const uint8_t *loss_mask,
+                          const int32_t *cu_seqlens, int32_t B, int64_t N, float gamma,
+                          float lambda_policy, float lambda_critic, float len_adaptive_alpha,
+                          float *adv, float *ret, void *ws, size_t ws_bytes, sao_stream_t stream);
+
+/*
+ * Eq. 1-3 (§3.1). r_t = exp(logp_t - old_logp_t); a token is kept iff it is an
+ * action token, its log-ratio and advantage are finite and
+ * 1 - eps_low < r_t < 1 + eps_high (strict; decided in fp32). With n = n_norm
+ * if n_norm > 0, else the number of action tokens:
+ *   loss    = -(1/n) sum_{kept t} r_t adv_t            [1] fp32 output
+ *   coef[t] = d loss / d logp_t = -r_t adv_t / n (kept), 0 otherwise (f(r) is
+ *             a detached coefficient)                   [N] fp32 output
+ *   flags[t]  SAO_FLAG_* value                          [N] uint8 output
+ *   counts  = {n_action, n_low, n_high, n_nonfinite}    [4] int64 output
+ * coef and flags may be NULL. The reductions are deterministic.
+ * Scalars: eps_low >= 0 (eps_low >= 1 disables the lower bound), eps_high >= 0.
+ */
+SAO_API sao_status sao_policy_loss_fwd(const float *logp, const float *old_logp, const float *adv,
+                               const uint8_t *loss_mask, int64_t N, float eps_low, float eps_high,
+                               int64_t n_norm, float *loss, float *coef, uint8_t *flags,
+                               int64_t *counts, void *ws, size_t ws_bytes, sao_stream_t stream);
+
+/*
+ * grad_logp[t] = grad_loss[0] * coef[t], with coef recomputed from the same
+ * inputs as sao_policy_loss_fwd (stateless). grad_loss is a device scalar.
+ */
+SAO_API sao_status sao_policy_loss_bwd(const float *logp, const float *old_logp, const float *adv,
+                               const uint8_t *loss_mask, int64_t N, float eps_low, float eps_high,
+                               int64_t n_norm, const float *grad_loss, float *grad_logp, void *ws,
+                               size_t ws_bytes, sao_stream_t stream);
+
+/*
+ * Value loss (Preliminaries, PPO): over the n action tokens,
+ *   loss = (1/n) sum_t (V_t - ret_t)^2           [1] fp32 output
+ *   grad_values[t] = 2 (V_t - ret_t) / n, 0 on non-action tokens   [N] fp32
+ *   ev_sums = {sum (R-V), sum (R-V)^2, sum R, sum R^2} over action tokens
+ *             ([4] fp64, may be NULL), from which explained variance
+ *             EV = 1 - Var(R - V) / Var(R) (§4.4) follows.
+ */
+SAO_API sao_status sao_value_loss(const float *values, const float *ret, const uint8_t *loss_mask,
+                          int64_t N, float *loss, float *grad_values, double *ev_sums, void *ws,
+                          size_t ws_bytes, sao_stream_t stream);
+
+/*
+ * Kernel timing for profiling. When enabled, every kernel the library
+ * launches is bracketed by CUDA events on its stream; sao_profile_read
+ * synchronises those events and returns, for up to `cap` kernel kinds, the
+ * name (static string), the number of launches and the summed device
+ * milliseconds since the last reset. Returns the number of kinds written.
+ */
+SAO_API void sao_profile_enable(int on);
+SAO_API void sao_profile_reset(void);
+SAO_API int sao_profile_read(const char **names, int64_t *launches, double *total_ms, int cap);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SAO_H_ */

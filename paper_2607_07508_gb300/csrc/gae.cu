@@ -1,0 +1,731 @@
+// Skip-observation token-level GAE (Preliminaries; §3.2 Eq. 4-5; §4.1) as a
+// single-pass reverse scan over packed trajectories.
+//
+// Formulation. Over the action tokens of one trajectory (observation tokens
+// are skipped, Eq. 4-5) write B_j = A_j + V_j, the lambda-return. The GAE
+// recursion A_j = r_j + gamma V_{j+1} - V_j + a A_{j+1} (a = gamma lambda)
+// becomes
+//     B_j = a B_{j+1} + (gamma - a) V_{j+1} + r_j ,   A_j = B_j - V_j ,
+// with B = V = 0 after the last action token and r_j = R only on it. The
+// return of the critic (lambda_critic) is the same recursion's B itself. This
+// form keeps every intermediate O(1) and lets A come out of one final
+// subtraction. All of it runs in double-float arithmetic (an fp32 pair, ~48
+// significant bits) so long trajectories do not accumulate fp32 rounding.
+//
+// The state carried right-to-left is S = (B_p, B_c, Vn, P): the two
+// lambda-returns of the next action token, its value, and the reward still
+// waiting for its action token. Each action token maps S affinely
+// (B' = a B + g Vn + P, Vn' = V, P' = 0); the last token of a trajectory
+// resets S to (0, 0, 0, R_b). Maps compose associatively, so:
+//   * each thread folds its 16 tokens into one map,
+//   * a warp-shuffle suffix scan and a per-CTA pass combine them,
+//   * CTAs (4096-token chunks) chain their maps right-to-left by decoupled
+//     look-back: each CTA takes a ticket, works on chunk nchunks-1-ticket, so
+//     it only ever waits on chunks whose CTAs started before it; every wait
+//     is bounded and a time-out raises SAO_DEVERR_SCAN_TIMEOUT,
+//   * each thread then replays its tokens from its incoming state.
+// Traffic: values 4 B + mask 1 B read, adv 4 B + ret 4 B written per token.
+#include <stdint.h>
+
+#include "sao_common.cuh"
+#include "sao_internal.h"
+
+namespace sao {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kItems = 16;
+constexpr int kChunk = kThreads * kItems;
+constexpr int kWarps = kThreads / 32;
+
+// ---------------------------------------------------------------------------
+// double-float arithmetic (Dekker / Knuth error-free transformations)
+// ---------------------------------------------------------------------------
+struct df {
+  float hi, lo;
+};
+__device__ __forceinline__ df quick_two_sum(float a, float b) {  // |a| >= |b|
+  const float s = __fadd_rn(a, b);
+  return {s, __fsub_rn(b, __fsub_rn(s, a))};
+}
+__device__ __forceinline__ df two_sum(float a, float b) {
+  const float s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  return {s, __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb))};
+}
+__device__ __forceinline__ df df_add(df x, df y) {
+  const df s = two_sum(x.hi, y.hi);
+  return quick_two_sum(s.hi, __fadd_rn(s.lo, __fadd_rn(x.lo, y.lo)));
+}
+__device__ __forceinline__ df df_add_f(df x, float y) {
+  const df s = two_sum(x.hi, y);
+  return quick_two_sum(s.hi, __fadd_rn(s.lo, x.lo));
+}
+__device__ __forceinline__ df df_mul(df x, df y) {
+  const float p = __fmul_rn(x.hi, y.hi);
+  float e = __fmaf_rn(x.hi, y.hi, -p);
+  e = __fmaf_rn(x.hi, y.lo, e);
+  e = __fmaf_rn(x.lo, y.hi, e);
+  return quick_two_sum(p, e);
+}
+__device__ __forceinline__ df df_mul_f(df x, float y) {
+  const float p = __fmul_rn(x.hi, y);
+  float e = __fmaf_rn(x.hi, y, -p);
+  e = __fmaf_rn(x.lo, y, e);
+  return quick_two_sum(p, e);
+}
+__device__ __forceinline__ float df_round(df x) { return __fadd_rn(x.hi, x.lo); }
+__device__ __forceinline__ df df_from_double(double x) {
+  const float hi = float(x);
+  return {hi, float(x - double(hi))};
+}
+
+// Per-trajectory coefficients: a = gamma*lambda and g = gamma - a for the
+// policy (lambda_b) and the critic (lambda_critic).
+struct TCoef {
+  df ap, gp, ac, gc;
+};
+__device__ __forceinline__ TCoef load_coef(const float4 *tab, int b) {
+  const float4 u = __ldg(tab + 2 * b), w = __ldg(tab + 2 * b + 1);
+  return {{u.x, u.y}, {u.z, u.w}, {w.x, w.y}, {w.z, w.w}};
+}
+
+// The affine map of a token segment, from the state at its right edge to the
+// state at its left edge. fl bit 0: the segment holds the last token of a
+// trajectory (the map ignores the incoming state); bit 1: the segment (left of
+// any reset) holds an action token. Identity when fl == 0.
+//   reset:          B = c,                        Vn = act ? v : 0, P = act ? 0 : p0
+//   act, no reset:  B = ap (a B + g Vn + P) + c,  Vn = v,           P = 0
+// b is the trajectory of the segment's leftmost token.
+struct GMap {
+  int b, fl;
+  df ap, cp, ac, cc;
+  float v, p0;
+};
+struct GState {
+  df Bp, Bc;
+  float Vn, P;
+};
+
+__device__ __forceinline__ GMap identity_map() {
+  GMap m;
+  m.b = 0;
+  m.fl = 0;
+  m.ap = m.ac = {1.f, 0.f};
+  m.cp = m.cc = {0.f, 0.f};
+  m.v = m.p0 = 0.f;
+  return m;
+}
+
+// x o y: x is the left segment, y the one immediately to its right.
+template <bool kCrit>
+__device__ GMap compose(const GMap &x, const GMap &y, const float4 *tab) {
+  if (x.fl & 1) return x;
+  if (!(x.fl & 2)) return y;
+  if (!(y.fl & 3)) return x;
+  const TCoef c = load_coef(tab, x.b);
+  const bool yact = (y.fl & 2) != 0;
+  const float Yv = yact ? y.v : 0.f, Yp = yact ? 0.f : y.p0;
+  GMap r;
+  r.b = x.b;
+  r.v = x.v;
+  r.p0 = 0.f;
+  df tp = df_add_f(df_add(df_mul(c.ap, y.cp), df_mul_f(c.gp, Yv)), Yp);
+  r.cp = df_add(df_mul(x.ap, tp), x.cp);
+  if (kCrit) {
+    df tc = df_add_f(df_add(df_mul(c.ac, y.cc), df_mul_f(c.gc, Yv)), Yp);
+    r.cc = df_add(df_mul(x.ac, tc), x.cc);
+  } else {
+    r.cc = {0.f, 0.f};
+  }
+  if (y.fl & 1) {
+    r.fl = 3;
+    r.ap = r.ac = {0.f, 0.f};
+  } else {
+    r.fl = 2;
+    r.ap = df_mul(df_mul(x.ap, c.ap), y.ap);
+    r.ac = kCrit ? df_mul(df_mul(x.ac, c.ac), y.ac) : df{1.f, 0.f};
+  }
+  return r;
+}
+
+template <bool kCrit>
+__device__ GState apply(const GMap &m, const GState &s, const float4 *tab) {
+  if (m.fl & 1) {
+    const bool act = (m.fl & 2) != 0;
+    return {m.cp, m.cc, act ? m.v : 0.f, act ? 0.f : m.p0};
+  }
+  if (!(m.fl & 2)) return s;
+  const TCoef c = load_coef(tab, m.b);
+  GState r;
+  const df tp = df_add_f(df_add(df_mul(c.ap, s.Bp), df_mul_f(c.gp, s.Vn)), s.P);
+  r.Bp = df_add(df_mul(m.ap, tp), m.cp);
+  if (kCrit) {
+    const df tc = df_add_f(df_add(df_mul(c.ac, s.Bc), df_mul_f(c.gc, s.Vn)), s.P);
+    r.Bc = df_add(df_mul(m.ac, tc), m.cc);
+  } else {
+    r.Bc = {0.f, 0.f};
+  }
+  r.Vn = m.v;
+  r.P = 0.f;
+  return r;
+}
+
+__device__ __forceinline__ GMap shfl_down_map(const GMap &m, int d) {
+  GMap r;
+  r.b = __shfl_down_sync(0xffffffffu, m.b, d);
+  r.fl = __shfl_down_sync(0xffffffffu, m.fl, d);
+  r.ap.hi = __shfl_down_sync(0xffffffffu, m.ap.hi, d);
+  r.ap.lo = __shfl_down_sync(0xffffffffu, m.ap.lo, d);
+  r.cp.hi = __shfl_down_sync(0xffffffffu, m.cp.hi, d);
+  r.cp.lo = __shfl_down_sync(0xffffffffu, m.cp.lo, d);
+  r.ac.hi = __shfl_down_sync(0xffffffffu, m.ac.hi, d);
+  r.ac.lo = __shfl_down_sync(0xffffffffu, m.ac.lo, d);
+  r.cc.hi = __shfl_down_sync(0xffffffffu, m.cc.hi, d);
+  r.cc.lo = __shfl_down_sync(0xffffffffu, m.cc.lo, d);
+  r.v = __shfl_down_sync(0xffffffffu, m.v, d);
+  r.p0 = __shfl_down_sync(0xffffffffu, m.p0, d);
+  return r;
+}
+
+// ---------------------------------------------------------------------------
+// cross-CTA publication (decoupled look-back)
+// ---------------------------------------------------------------------------
+struct __align__(16) ChunkPub {
+  GMap agg;     // map of the whole chunk (status >= 1)
+  GState incl;  // state at the chunk's left edge (status == 2)
+};
+
+__device__ __forceinline__ int ld_acquire(const int *p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release(int *p, int v) {
+  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Published maps and states go through L2 only (st.cg / ld.cg), so a reader on
+// another SM never sees a stale L1 line.
+__device__ __forceinline__ void st_df(df *p, df x) {
+  __stcg(&p->hi, x.hi);
+  __stcg(&p->lo, x.lo);
+}
+__device__ __forceinline__ df ld_df(const df *p) { return {__ldcg(&p->hi), __ldcg(&p->lo)}; }
+__device__ void store_map(GMap *p, const GMap &m) {
+  __stcg(&p->b, m.b);
+  __stcg(&p->fl, m.fl);
+  st_df(&p->ap, m.ap);
+  st_df(&p->cp, m.cp);
+  st_df(&p->ac, m.ac);
+  st_df(&p->cc, m.cc);
+  __stcg(&p->v, m.v);
+  __stcg(&p->p0, m.p0);
+}
+__device__ GMap load_map(const GMap *p) {
+  GMap m;
+  m.b = __ldcg(&p->b);
+  m.fl = __ldcg(&p->fl);
+  m.ap = ld_df(&p->ap);
+  m.cp = ld_df(&p->cp);
+  m.ac = ld_df(&p->ac);
+  m.cc = ld_df(&p->cc);
+  m.v = __ldcg(&p->v);
+  m.p0 = __ldcg(&p->p0);
+  return m;
+}
+__device__ void store_state(GState *p, const GState &s) {
+  st_df(&p->Bp, s.Bp);
+  st_df(&p->Bc, s.Bc);
+  __stcg(&p->Vn, s.Vn);
+  __stcg(&p->P, s.P);
+}
+__device__ GState load_state(const GState *p) {
+  GState s;
+  s.Bp = ld_df(&p->Bp);
+  s.Bc = ld_df(&p->Bc);
+  s.Vn = __ldcg(&p->Vn);
+  s.P = __ldcg(&p->P);
+  return s;
+}
+
+// Waits until *p != 0; returns it, or 0 after kWaitLimitNs / kSpinLimit polls.
+__device__ int wait_nonzero(const int *p) {
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t n = 0; n < kSpinLimit; ++n) {
+    const int s = ld_acquire(p);
+    if (s != 0) return s;
+    if ((n & 63u) == 63u && globaltimer_ns() - t0 > kWaitLimitNs) return 0;
+    __nanosleep(64);
+  }
+  return 0;
+}
+
+struct GaeArgs {
+  const float *values, *rewards;
+  const uint8_t *m;
+  const int32_t *cu;
+  int B;
+  int64_t N;
+  int nchunks;
+  const float4 *coef;  // [B][2]
+  const int *chunk_first;  // [nchunks] trajectory of each chunk's first token
+  int *ticket;
+  int *status;         // [nchunks]
+  ChunkPub *pub;       // [nchunks]
+  float *adv, *ret;
+  unsigned int *err;
+};
+
+constexpr int kCuCap = 1024;
+
+// cu_seqlens entries [blo, blo + n) of one chunk, read from shared memory
+// when the slice fits there, else from global memory.
+struct CuView {
+  const int32_t *g;
+  const int32_t *s;
+  int blo;
+  bool in_smem;
+  __device__ __forceinline__ int64_t operator[](int b) const { return in_smem ? s[b - blo] : __ldg(g + b); }
+  // largest b in [lo, hi] with cu[b] <= t
+  __device__ __forceinline__ int find(int lo, int hi, int64_t t) const {
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if ((*this)[mid] <= t) lo = mid;
+      else hi = mid - 1;
+    }
+    return lo;
+  }
+};
+
+__device__ __forceinline__ int find_traj(const int32_t *cu, int B, int64_t t) {
+  int lo = 0, hi = B - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (int64_t(__ldg(cu + mid)) <= t) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
+template <bool kCrit>
+__global__ void __launch_bounds__(kThreads, 2) gae_scan_kernel(GaeArgs a) {
+  __shared__ int s_q, s_blo, s_ncu;
+  __shared__ GMap s_warp[kWarps];
+  __shared__ GState s_wstate[kWarps];
+  __shared__ int32_t s_cu[kCuCap];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) {
+    const int q = a.nchunks - 1 - atomicAdd(a.ticket, 1);
+    const int blo = a.chunk_first[q];
+    const int bhi = q + 1 < a.nchunks ? a.chunk_first[q + 1] : a.B - 1;
+    s_q = q;
+    s_blo = blo;
+    s_ncu = bhi - blo + 2;  // cu[blo .. bhi + 1]
+  }
+  __syncthreads();
+  const int q = s_q;
+  const int64_t t0 = int64_t(q) * kChunk + int64_t(threadIdx.x) * kItems;
+  const int64_t N = a.N;
+  // This chunk's slice of cu_seqlens, in shared memory when it fits.
+  const CuView cu{a.cu, s_cu, s_blo, s_ncu <= kCuCap};
+  if (cu.in_smem)
+    for (int i = threadIdx.x; i < s_ncu; i += kThreads) s_cu[i] = __ldg(a.cu + s_blo + i);
+  __syncthreads();
+
+  // ---- load 16 tokens -------------------------------------------------------
+  float v[kItems];
+  uint32_t act = 0;
+  const bool full = t0 + kItems <= N;
+  if (full && aligned16_dev(a.values) && aligned16_dev(a.m)) {
+    const float4 *v4 = reinterpret_cast<const float4 *>(a.values + t0);
+#pragma unroll
+    for (int k = 0; k < kItems / 4; ++k) {
+      const float4 x = __ldcs(v4 + k);
+      v[4 * k] = x.x;
+      v[4 * k + 1] = x.y;
+      v[4 * k + 2] = x.z;
+      v[4 * k + 3] = x.w;
+    }
+    const uint4 mq = __ldcs(reinterpret_cast<const uint4 *>(a.m + t0));
+    const uint32_t w[4] = {mq.x, mq.y, mq.z, mq.w};
+#pragma unroll
+    for (int k = 0; k < kItems; ++k) act |= uint32_t(((w[k >> 2] >> (8 * (k & 3))) & 0xffu) != 0u) << k;
+  } else {
+#pragma unroll
+    for (int k = 0; k < kItems; ++k) {
+      const int64_t t = t0 + k;
+      v[k] = t < N ? a.values[t] : 0.f;
+      act |= uint32_t(t < N && a.m[t] != 0) << k;
+    }
+  }
+
+  // ---- trajectory ends among the 16 tokens (forward walk) ----------------------
+  // The walk is repeated backwards in the two right-to-left passes below, so no
+  // per-token trajectory id is kept in registers.
+  uint32_t endbits = 0;
+  int b_last;
+  {
+    const int bhi = s_blo + s_ncu - 2;
+    int b = cu.find(s_blo, bhi, t0 < N ? t0 : N - 1);
+    int64_t next_end = cu[b + 1];
+    bool bad = false;
+#pragma unroll
+    for (int k = 0; k < kItems; ++k) {
+      const int64_t t = t0 + k;
+      if (t < N) {
+        while (b < bhi && t >= next_end) {
+          ++b;
+          next_end = cu[b + 1];
+        }
+        if (t >= next_end) bad = true;  // cu_seqlens[B] < N
+        endbits |= uint32_t(t == next_end - 1) << k;
+      }
+    }
+    b_last = b;
+    if (bad) {
+      raise_device_error(a.err, SAO_DEVERR_CU_SEQLENS);
+      act = 0;
+    }
+  }
+
+  // ---- fold the thread's tokens into one map (right to left) ------------------
+  GMap M = identity_map();
+  {
+    int b = b_last;
+    int64_t b_start = cu[b];
+    TCoef c = load_coef(a.coef, b);
+#pragma unroll
+    for (int k = kItems - 1; k >= 0; --k) {
+      const int64_t t = t0 + k;
+      if (t >= N) continue;
+      if (t < b_start) {
+        while (b > s_blo && t < b_start) {
+          --b;
+          b_start = cu[b];
+        }
+        c = load_coef(a.coef, b);
+      }
+      const bool is_act = (act >> k) & 1u, is_end = (endbits >> k) & 1u;
+      if (is_end) {
+        const float R = __ldg(a.rewards + b);
+        M.b = b;
+        M.ap = M.ac = {0.f, 0.f};
+        if (is_act) {
+          M.fl = 3;
+          M.cp = M.cc = {R, 0.f};
+          M.v = v[k];
+          M.p0 = 0.f;
+        } else {
+          M.fl = 1;
+          M.cp = M.cc = {0.f, 0.f};
+          M.v = 0.f;
+          M.p0 = R;
+        }
+      } else if (is_act) {
+        if (M.fl == 0) {
+          M.fl = 2;
+          M.ap = M.ac = {1.f, 0.f};
+          M.cp = M.cc = {0.f, 0.f};
+        } else {
+          const bool mact = (M.fl & 2) != 0;
+          const float Yv = mact ? M.v : 0.f, Yp = mact ? 0.f : M.p0;
+          M.cp = df_add_f(df_add(df_mul(c.ap, M.cp), df_mul_f(c.gp, Yv)), Yp);
+          if (kCrit) M.cc = df_add_f(df_add(df_mul(c.ac, M.cc), df_mul_f(c.gc, Yv)), Yp);
+          if (!(M.fl & 1)) {
+            M.ap = df_mul(c.ap, M.ap);
+            if (kCrit) M.ac = df_mul(c.ac, M.ac);
+          }
+          M.fl |= 2;
+        }
+        M.b = b;
+        M.v = v[k];
+        M.p0 = 0.f;
+      } else if (M.fl != 0) {
+        M.b = b;
+      }
+    }
+  }
+
+  // ---- suffix scan within the warp, then across warps ---------------------------
+  GMap S = M;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const GMap o = shfl_down_map(S, d);
+    if (lane + d < 32) S = compose<kCrit>(S, o, a.coef);
+  }
+  GMap E = shfl_down_map(S, 1);  // lanes to my right within the warp
+  if (lane == 31) E = identity_map();
+  if (lane == 0) s_warp[warp] = S;
+  __syncthreads();
+
+  if (warp == 0) {
+    // Lanes 0..7 scan the warp maps: W = map of warp `lane` .. last (inclusive),
+    // T = map of warps lane+1 .. last (exclusive); lane 0 holds the chunk map.
+    GMap W = lane < kWarps ? s_warp[lane] : identity_map();
+#pragma unroll
+    for (int d = 1; d < kWarps; d <<= 1) {
+      const GMap o = shfl_down_map(W, d);
+      if (lane + d < kWarps) W = compose<kCrit>(W, o, a.coef);
+    }
+    GMap T = shfl_down_map(W, 1);
+    if (lane >= kWarps - 1) T = identity_map();
+    GState zero;
+    zero.Bp = zero.Bc = {0.f, 0.f};
+    zero.Vn = zero.P = 0.f;
+    GState right = zero;
+    if (lane == 0) {
+      const GMap &agg = W;
+      ChunkPub *me = a.pub + q;
+      const bool last = (q == a.nchunks - 1);
+      const bool reset = (agg.fl & 1) != 0;
+      // A chunk whose map ignores its right neighbour publishes its left-edge
+      // state at once; the others publish their map first.
+      if (last || reset) {
+        store_state(&me->incl, apply<kCrit>(agg, zero, a.coef));
+        __threadfence();
+        st_release(a.status + q, 2);
+      } else {
+        store_map(&me->agg, agg);
+        __threadfence();
+        st_release(a.status + q, 1);
+      }
+      if (!last) {
+        // look back to the right for the state at this chunk's right edge
+        GMap acc = identity_map();
+        for (int j = q + 1;; ++j) {
+          if (j >= a.nchunks) {
+            right = apply<kCrit>(acc, zero, a.coef);
+            break;
+          }
+          const int st = wait_nonzero(a.status + j);
+          if (st == 0) {
+            raise_device_error(a.err, SAO_DEVERR_SCAN_TIMEOUT);
+            right = apply<kCrit>(acc, zero, a.coef);
+            break;
+          }
+          if (st == 2) {
+            right = apply<kCrit>(acc, load_state(&a.pub[j].incl), a.coef);
+            break;
+          }
+          acc = compose<kCrit>(acc, load_map(&a.pub[j].agg), a.coef);
+          if (acc.fl & 1) {
+            right = apply<kCrit>(acc, zero, a.coef);
+            break;
+          }
+        }
+        if (!reset) {
+          store_state(&me->incl, apply<kCrit>(agg, right, a.coef));
+          __threadfence();
+          st_release(a.status + q, 2);
+        }
+      }
+    }
+    // broadcast the right-edge state and give every warp its incoming state
+    right.Bp.hi = __shfl_sync(0xffffffffu, right.Bp.hi, 0);
+    right.Bp.lo = __shfl_sync(0xffffffffu, right.Bp.lo, 0);
+    right.Bc.hi = __shfl_sync(0xffffffffu, right.Bc.hi, 0);
+    right.Bc.lo = __shfl_sync(0xffffffffu, right.Bc.lo, 0);
+    right.Vn = __shfl_sync(0xffffffffu, right.Vn, 0);
+    right.P = __shfl_sync(0xffffffffu, right.P, 0);
+    if (lane < kWarps) s_wstate[lane] = apply<kCrit>(T, right, a.coef);
+  }
+  __syncthreads();
+
+  // ---- replay the tokens from the incoming state, store 4 at a time --------------
+  GState st = apply<kCrit>(E, s_wstate[warp], a.coef);
+  const bool vec_out = full && aligned16_dev(a.adv) && aligned16_dev(a.ret);
+  {
+    int b = b_last;
+    int64_t b_start = cu[b];
+    TCoef c = load_coef(a.coef, b);
+    float R = __ldg(a.rewards + b);
+#pragma unroll
+    for (int g = kItems / 4 - 1; g >= 0; --g) {
+      float ov[4], orr[4];
+#pragma unroll
+      for (int i = 3; i >= 0; --i) {
+        const int k = 4 * g + i;
+        const int64_t t = t0 + k;
+        ov[i] = 0.f;
+        orr[i] = 0.f;
+        if (t >= N) continue;
+        if (t < b_start) {
+          while (b > s_blo && t < b_start) {
+            --b;
+            b_start = cu[b];
+          }
+          c = load_coef(a.coef, b);
+          R = __ldg(a.rewards + b);
+        }
+        if ((endbits >> k) & 1u) {
+          st.Bp = st.Bc = {0.f, 0.f};
+          st.Vn = 0.f;
+          st.P = R;
+        }
+        if ((act >> k) & 1u) {
+          st.Bp = df_add_f(df_add(df_mul(c.ap, st.Bp), df_mul_f(c.gp, st.Vn)), st.P);
+          if (kCrit) {
+            st.Bc = df_add_f(df_add(df_mul(c.ac, st.Bc), df_mul_f(c.gc, st.Vn)), st.P);
+            orr[i] = df_round(st.Bc);
+          } else {
+            orr[i] = R;  // gamma = lambda_critic = 1: the return is the reward
+          }
+          ov[i] = df_round(df_add_f(st.Bp, -v[k]));
+          st.Vn = v[k];
+          st.P = 0.f;
+        }
+      }
+      if (vec_out) {
+        __stcs(reinterpret_cast<float4 *>(a.adv + t0) + g, make_float4(ov[0], ov[1], ov[2], ov[3]));
+        __stcs(reinterpret_cast<float4 *>(a.ret + t0) + g, make_float4(orr[0], orr[1], orr[2], orr[3]));
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (t0 + 4 * g + i < N) {
+            a.adv[t0 + 4 * g + i] = ov[i];
+            a.ret[t0 + 4 * g + i] = orr[i];
+          }
+      }
+    }
+  }
+}
+
+// Number of action tokens per trajectory (only for the length-adaptive lambda).
+// One CTA per 4096-token chunk, like the scan, with the chunk's cu_seqlens
+// slice in shared memory.
+__global__ void __launch_bounds__(kThreads) gae_count_kernel(const uint8_t *m, const int32_t *cu_g, int B,
+                                                             int64_t N, int nchunks, const int *chunk_first,
+                                                             int *nact) {
+  __shared__ int32_t s_cu[kCuCap];
+  const int q = blockIdx.x;
+  const int blo = chunk_first[q];
+  const int bhi = q + 1 < nchunks ? chunk_first[q + 1] : B - 1;
+  const int ncu = bhi - blo + 2;
+  const CuView cu{cu_g, s_cu, blo, ncu <= kCuCap};
+  if (cu.in_smem)
+    for (int i = threadIdx.x; i < ncu; i += kThreads) s_cu[i] = __ldg(cu_g + blo + i);
+  __syncthreads();
+  const int64_t t0 = int64_t(q) * kChunk + int64_t(threadIdx.x) * kItems;
+  int b = cu.find(blo, bhi, t0 < N ? t0 : N - 1);
+  int64_t next_end = cu[b + 1];
+  int cnt = 0;
+#pragma unroll
+  for (int k = 0; k < kItems; ++k) {
+    const int64_t t = t0 + k;
+    if (t >= N) break;
+    if (t >= next_end) {
+      const int nb0 = b;
+      while (b < bhi && t >= next_end) {
+        ++b;
+        next_end = cu[b + 1];
+      }
+      if (b != nb0 && cnt) {
+        atomicAdd(nact + nb0, cnt);
+        cnt = 0;
+      }
+    }
+    cnt += (m[t] != 0);
+  }
+  const unsigned peers = __match_any_sync(0xffffffffu, b);
+  const int tot = __reduce_add_sync(peers, cnt);
+  if ((threadIdx.x & 31) == __ffs(peers) - 1 && tot) atomicAdd(nact + b, tot);
+}
+
+// First trajectory of every chunk (one binary search per chunk, all in parallel).
+__global__ void gae_chunk_first_kernel(const int32_t *cu, int B, int64_t N, int nchunks, int *chunk_first) {
+  const int q = blockIdx.x * blockDim.x + threadIdx.x;
+  if (q >= nchunks) return;
+  const int64_t t = int64_t(q) * kChunk;
+  chunk_first[q] = find_traj(cu, B, t < N ? t : N - 1);
+}
+
+// Per-trajectory coefficients (fp64 then split to double-float) and a check of
+// cu_seqlens: 0 = cu[0] <= cu[1] <= ... <= cu[B] = N.
+__global__ void gae_coef_kernel(const int32_t *cu, int B, int64_t N, float gamma, float lam, float lam_c,
+                                float alpha, const int *nact, float4 *coef, unsigned int *err) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  if ((b == 0 && cu[0] != 0) || cu[b + 1] < cu[b] || (b == B - 1 && int64_t(cu[B]) != N))
+    raise_device_error(err, SAO_DEVERR_CU_SEQLENS);
+  double lb = lam;
+  if (alpha > 0.f) {
+    const int L = nact[b];
+    lb = L > 0 ? 1.0 - 1.0 / (double(alpha) * double(L)) : 0.0;
+    lb = lb < 0.0 ? 0.0 : (lb > 1.0 ? 1.0 : lb);
+  }
+  const double g = gamma;
+  const double ap = g * lb, ac = g * double(lam_c);
+  const df Ap = df_from_double(ap), Gp = df_from_double(g - ap);
+  const df Ac = df_from_double(ac), Gc = df_from_double(g - ac);
+  coef[2 * b] = make_float4(Ap.hi, Ap.lo, Gp.hi, Gp.lo);
+  coef[2 * b + 1] = make_float4(Ac.hi, Ac.lo, Gc.hi, Gc.lo);
+}
+
+}  // namespace
+
+size_t gae_ws_bytes(int64_t N, int64_t B) {
+  const int64_t nchunks = (N + kChunk - 1) / kChunk;
+  return round256(sizeof(int)) + round256(sizeof(int) * (B + 1)) + round256(sizeof(int) * nchunks) +
+         round256(sizeof(float4) * 2 * (B + 1)) + round256(sizeof(ChunkPub) * nchunks) +
+         round256(sizeof(int) * (nchunks + 1));
+}
+
+sao_status gae_launch(const float *values, const float *rewards, const uint8_t *m, const int32_t *cu,
+                      int32_t B, int64_t N, float gamma, float lam, float lam_c, float alpha, float *adv,
+                      float *ret, unsigned int *err, void *ws_body, size_t body_bytes, cudaStream_t s) {
+  if (N == 0) return SAO_OK;
+  const int64_t nchunks = (N + kChunk - 1) / kChunk;
+  if (nchunks > (int64_t(1) << 30)) return fail(SAO_ERR_SHAPE, "too many tokens for the advantage scan");
+  Carver c(ws_body, body_bytes);
+  char *zero_begin = c.base + c.off;
+  int *ticket = c.take<int>(1);
+  int *nact = c.take<int>(size_t(B) + 1);
+  int *status = c.take<int>(size_t(nchunks));
+  char *zero_end = c.base + c.off;
+  float4 *coef = c.take<float4>(2 * (size_t(B) + 1));
+  ChunkPub *pub = c.take<ChunkPub>(size_t(nchunks));
+  int *chunk_first = c.take<int>(size_t(nchunks) + 1);
+  if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the advantage scan");
+  SAO_CUDA_TRY(cudaMemsetAsync(zero_begin, 0, size_t(zero_end - zero_begin), s));
+  {
+    int slot = launch_begin("gae_chunk_first", s);
+    gae_chunk_first_kernel<<<unsigned((nchunks + 255) / 256), 256, 0, s>>>(cu, B, N, int(nchunks), chunk_first);
+    SAO_TRY(launch_end(slot, s));
+  }
+  if (alpha > 0.f) {
+    int slot = launch_begin("gae_count", s);
+    gae_count_kernel<<<unsigned(nchunks), kThreads, 0, s>>>(m, cu, B, N, int(nchunks), chunk_first, nact);
+    SAO_TRY(launch_end(slot, s));
+  }
+  {
+    int slot = launch_begin("gae_coef", s);
+    gae_coef_kernel<<<(B + 127) / 128, 128, 0, s>>>(cu, B, N, gamma, lam, lam_c, alpha, nact, coef, err);
+    SAO_TRY(launch_end(slot, s));
+  }
+  GaeArgs a;
+  a.values = values;
+  a.rewards = rewards;
+  a.m = m;
+  a.cu = cu;
+  a.B = B;
+  a.N = N;
+  a.nchunks = int(nchunks);
+  a.coef = coef;
+  a.chunk_first = chunk_first;
+  a.ticket = ticket;
+  a.status = status;
+  a.pub = pub;
+  a.adv = adv;
+  a.ret = ret;
+  a.err = err;
+  const bool crit_trivial = (gamma == 1.0f && lam_c == 1.0f);
+  int slot = launch_begin("gae_scan", s);
+  if (crit_trivial)
+    gae_scan_kernel<false><<<int(nchunks), kThreads, 0, s>>>(a);
+  else
+    gae_scan_kernel<true><<<int(nchunks), kThreads, 0, s>>>(a);
+  return launch_end(slot, s);
+}
+
+}  // namespace sao

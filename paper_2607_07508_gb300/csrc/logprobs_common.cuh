@@ -1,0 +1,35 @@
+// Pieces shared by the fp32 and tensor-core log-prob paths.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/sao.h"
+
+namespace sao {
+
+// Merges per-(vocab tile, row) partials part[j * N + row] = (max_j, sumexp_j)
+// into lse[row] = log sum_v e^z and logp[row] = zy[row] - lse[row]. Rows with
+// row_mask == 0 get logp = lse = 0; rows whose token id is outside [0, V) get
+// logp = NaN.
+sao_status lse_merge_launch(const float2 *part, int nvt, const float *zy, const int32_t *y,
+                            const uint8_t *row_mask, int64_t N, int32_t V, float *logp, float *lse,
+                            unsigned int *err, cudaStream_t s);
+
+size_t simt_ws_bytes(int64_t N, int32_t h, int32_t V);
+sao_status simt_fwd(const float *H, const float *W, const int32_t *y, const uint8_t *row_mask, int64_t N,
+                    int32_t h, int32_t V, float *logp, float *lse, unsigned int *err, void *ws, size_t ws_bytes,
+                    cudaStream_t s);
+sao_status simt_bwd(const float *H, const float *W, const int32_t *y, const float *lse, const float *G,
+                    int64_t N, int32_t h, int32_t V, float *dH, float *dW, int accumulate, void *ws,
+                    size_t ws_bytes, cudaStream_t s);
+
+size_t tc_ws_bytes(int64_t N, int32_t h, int32_t V);
+sao_status tc_fwd(const void *H, const void *W, const int32_t *y, const uint8_t *row_mask, int64_t N,
+                  int32_t h, int32_t V, float *logp, float *lse, unsigned int *err, void *ws, size_t ws_bytes,
+                  cudaStream_t s);
+sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *lse, const float *G,
+                  int64_t N, int32_t h, int32_t V, void *dH, float *dW, int accumulate, unsigned int *err,
+                  void *ws, size_t ws_bytes, cudaStream_t s);
+
+}  // namespace sao

@@ -1,0 +1,599 @@
+// bf16 tensor-core path of the LM-head log-probs (Eq. 1-2) and their gradient.
+//
+// One persistent, warp-specialised GEMM kernel on the 5th-generation tensor
+// cores serves all four contractions, with the per-element work fused into
+// the epilogue so the [N, V] logits never reach memory:
+//
+//   forward   Z = H W^T          -> online (max, sum-exp) per row over each
+//                                   256-wide vocabulary tile + gather of z[y]
+//   backward  Z = H W^T (again)  -> dZ = G (1[v == y] - exp(z - lse)), bf16,
+//                                   into a [N, Vc] chunk buffer
+//             dH (+)= dZ W_chunk    (A K-major, B = W MN-major)
+//             dW_chunk = dZ^T H     (A = dZ MN-major, B = H MN-major)
+//
+// CTA layout (192 threads): warp 0 issues TMA loads of 128x64 A and 256x64 B
+// bf16 tiles (128-byte swizzle) into a 4-stage shared-memory ring; warp 1
+// owns 512 TMEM columns (two 128x256 fp32 accumulators) and issues
+// tcgen05.mma (M=128, N=256, K=16) from one thread; warps 2-5 drain the
+// accumulator through tcgen05.ld, one TMEM lane (= output row) per thread,
+// while the MMA warp already fills the other accumulator. Every wait is
+// bounded; a time-out raises SAO_DEVERR_PIPE_TIMEOUT and all roles wind down.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cudaTypedefs.h>
+#include <math.h>
+#include <stdint.h>
+
+#include <mutex>
+
+#include "logprobs_common.cuh"
+#include "sao_common.cuh"
+#include "sao_internal.h"
+#include "tc_ptx.cuh"
+
+namespace sao {
+namespace {
+
+using namespace tc;
+
+constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr uint32_t A_BYTES = BM * BK * 2;
+constexpr uint32_t B_BYTES = BN * BK * 2;
+constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int NUM_THREADS = 192;
+constexpr uint32_t TMEM_COLS = 2 * BN;
+constexpr uint32_t MN_ATOM_BYTES = 64 * BK * 2;   // one 64(MN) x 64(K) box
+constexpr size_t SMEM_BYTES = 1024 + size_t(STAGES) * STAGE_BYTES + 256;
+constexpr float kLog2e = 1.4426950408889634f;
+
+enum EpiKind : int { kSoftmax = 0, kDLogits = 1, kStoreF32 = 2, kStoreBF16 = 3 };
+
+struct GemmParams {
+  int nM, nN, nK;      // tiles along M, N and 64-wide K blocks
+  int group_m;         // tile raster: group_m M-tiles per group, M fastest inside
+  int a_row_off;       // A K-major: row offset; A MN-major: column (M) offset
+  int b_row_off;       // B K-major: row offset of N; B MN-major: K offset
+  // epilogue
+  int64_t rows;        // valid output rows (M extent)
+  int cols;            // valid output columns (N extent)
+  const int32_t *y;
+  int vocab;           // V (softmax / dlogits)
+  int v0;              // vocabulary index of GEMM column 0 (dlogits)
+  float2 *part;        // softmax partials [nN][rows]
+  float *zy;           // gathered logit of the sampled token
+  const float *lse, *G;
+  __nv_bfloat16 *dz;   // dlogits output [rows][ldz]
+  int64_t ldz;
+  float *cf;           // store f32 output (row-major, ldc)
+  __nv_bfloat16 *cb;   // store bf16 output
+  int64_t ldc;
+  int64_t c_row_off;   // output row offset
+  int accumulate;
+  unsigned int *err;
+};
+
+struct __align__(8) SmemCtl {
+  uint64_t full[STAGES], empty[STAGES], acc_full[2], acc_empty[2];
+  uint32_t tmem_base;
+  int abort;
+};
+
+__device__ __forceinline__ void tile_coords(int L, const GemmParams &p, int &m, int &n) {
+  const int per_group = p.group_m * p.nN;
+  const int g = L / per_group;
+  const int within = L - g * per_group;
+  const int m0 = g * p.group_m;
+  const int gm = min(p.group_m, p.nM - m0);
+  m = m0 + within % gm;
+  n = within / gm;
+}
+
+template <int kEpi, bool kAMN, bool kBMN>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
+                   const GemmParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t *gbase = smem_raw + (base - raw);
+  SmemCtl *ctl = reinterpret_cast<SmemCtl *>(gbase + size_t(STAGES) * STAGE_BYTES);
+  volatile int *abort = &ctl->abort;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int num_tiles = p.nM * p.nN;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(smem_u32(&ctl->full[s]), 1);
+      mbar_init(smem_u32(&ctl->empty[s]), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(smem_u32(&ctl->acc_full[a]), 1);
+      mbar_init(smem_u32(&ctl->acc_empty[a]), 4 * 32);
+    }
+    ctl->abort = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&ctl->tmem_base), TMEM_COLS);
+    tmem_relinquish();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_map(&map_a);
+    tma_prefetch_map(&map_b);
+  }
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tmem_base = ctl->tmem_base;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      uint32_t issued = 0;  // bit s: stage s has a load whose full-barrier phase is phase_of(s)
+      uint32_t issued_phase = 0;
+      for (int L = blockIdx.x; L < num_tiles && ok; L += gridDim.x) {
+        int m, n;
+        tile_coords(L, p, m, n);
+        for (int kb = 0; kb < p.nK; ++kb) {
+          if (!mbar_wait(smem_u32(&ctl->empty[stage]), phase ^ 1u, abort, p.err)) {
+            ok = false;
+            break;
+          }
+          const uint32_t fb = smem_u32(&ctl->full[stage]);
+          issued |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          mbar_arrive_expect_tx(fb, STAGE_BYTES);
+          const uint32_t sa = base + uint32_t(stage) * STAGE_BYTES;
+          const uint32_t sb = sa + A_BYTES;
+          const int k0 = kb * BK;
+          if (!kAMN) {
+            tma_load_2d(sa, &map_a, fb, k0, p.a_row_off + m * BM);
+          } else {
+#pragma unroll
+            for (int j = 0; j < BM / 64; ++j)
+              tma_load_2d(sa + j * MN_ATOM_BYTES, &map_a, fb, p.a_row_off + m * BM + 64 * j, k0);
+          }
+          if (!kBMN) {
+            tma_load_2d(sb, &map_b, fb, k0, p.b_row_off + n * BN);
+          } else {
+#pragma unroll
+            for (int j = 0; j < BN / 64; ++j)
+              tma_load_2d(sb + j * MN_ATOM_BYTES, &map_b, fb, n * BN + 64 * j, p.b_row_off + k0);
+          }
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        // let the copies already in flight land before the CTA can exit
+        for (int s = 0; s < STAGES; ++s) {
+          if (!((issued >> s) & 1u)) continue;
+          const uint32_t par = (issued_phase >> s) & 1u;
+          const uint64_t t0 = globaltimer_ns();
+          while (!mbar_try_wait(smem_u32(&ctl->full[s]), par) && globaltimer_ns() - t0 < kWaitLimitNs) {
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16(BM, BN, kAMN, kBMN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int local = 0;
+      bool ok = true;
+      for (int L = blockIdx.x; L < num_tiles && ok; L += gridDim.x, ++local) {
+        const int acc = local & 1;
+        const uint32_t acc_phase = uint32_t(local >> 1) & 1u;
+        if (!mbar_wait(smem_u32(&ctl->acc_empty[acc]), acc_phase ^ 1u, abort, p.err)) break;
+        fence_after_sync();
+        const uint32_t d_tmem = tmem_base + uint32_t(acc) * BN;
+        for (int kb = 0; kb < p.nK; ++kb) {
+          if (!mbar_wait(smem_u32(&ctl->full[stage]), phase, abort, p.err)) {
+            ok = false;
+            break;
+          }
+          fence_after_sync();
+          const uint32_t sa = base + uint32_t(stage) * STAGE_BYTES;
+          const uint32_t sb = sa + A_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            const uint64_t ad = kAMN ? sdesc_sw128(sa + kk * 2048u, MN_ATOM_BYTES, 1024u)
+                                     : sdesc_sw128(sa + kk * 32u, 16u, 1024u);
+            const uint64_t bd = kBMN ? sdesc_sw128(sb + kk * 2048u, MN_ATOM_BYTES, 1024u)
+                                     : sdesc_sw128(sb + kk * 32u, 16u, 1024u);
+            mma_bf16(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+          }
+          mma_commit(smem_u32(&ctl->empty[stage]));
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        mma_commit(smem_u32(&ctl->acc_full[acc]));
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int quad = warp & 3;  // TMEM lane quadrant this warp may access
+    const int r = quad * 32 + lane;
+    int local = 0;
+    for (int L = blockIdx.x; L < num_tiles; L += gridDim.x, ++local) {
+      int m, n;
+      tile_coords(L, p, m, n);
+      const int acc = local & 1;
+      const uint32_t acc_phase = uint32_t(local >> 1) & 1u;
+      if (!mbar_wait(smem_u32(&ctl->acc_full[acc]), acc_phase, abort, p.err)) break;
+      fence_after_sync();
+      const uint32_t taddr = tmem_base + (uint32_t(quad * 32) << 16) + uint32_t(acc) * BN;
+      const int64_t row = int64_t(m) * BM + r;
+      const bool row_ok = row < p.rows;
+
+      if constexpr (kEpi == kSoftmax) {
+        const int col0 = n * BN;
+        const int yy = row_ok ? __ldg(p.y + row) : -1;
+        float mx = -INFINITY, sm = 0.f, zsel = 0.f;
+        bool have = false;
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t u[32];
+          tmem_ld32(taddr + c * 32, u);
+          tmem_wait_ld();
+          const int cbase = col0 + c * 32;
+          const int valid = p.vocab - cbase;
+          float v[32];
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] = (j < valid) ? __uint_as_float(u[j]) : -INFINITY;
+          float cm = v[0];
+#pragma unroll
+          for (int j = 1; j < 32; ++j) cm = fmaxf(cm, v[j]);
+          const float mn = fmaxf(mx, cm);
+          const float off = -mn * kLog2e;
+          float s = 0.f;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) s += ex2_approx(fmaf(v[j], kLog2e, off));
+          sm = fmaf(sm, ex2_approx((mx - mn) * kLog2e), s);
+          mx = mn;
+          const unsigned rel = unsigned(yy - cbase);
+          if (rel < 32u) {
+            float z = v[0];
+#pragma unroll
+            for (int j = 1; j < 32; ++j) z = (unsigned(j) == rel) ? v[j] : z;
+            zsel = z;
+            have = true;
+          }
+        }
+        fence_before_sync();
+        mbar_arrive(smem_u32(&ctl->acc_empty[acc]));
+        if (row_ok) {
+          p.part[int64_t(n) * p.rows + row] = make_float2(mx, sm);
+          if (have) p.zy[row] = zsel;
+        }
+      } else if constexpr (kEpi == kDLogits) {
+        const int lc0 = n * BN;  // column inside the chunk
+        int yy = -1;
+        float g = 0.f, l2 = 0.f;
+        if (row_ok) {
+          yy = __ldg(p.y + row) - p.v0;
+          g = __ldg(p.G + row);
+          l2 = __ldg(p.lse + row) * kLog2e;
+        }
+        __nv_bfloat16 *out = p.dz + (row_ok ? row : 0) * p.ldz;
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t u[32];
+          tmem_ld32(taddr + c * 32, u);
+          tmem_wait_ld();
+          const int lc = lc0 + c * 32;
+          if (!row_ok || lc >= p.cols) continue;
+          uint32_t pk[16];
+#pragma unroll
+          for (int j = 0; j < 32; j += 2) {
+            float d0 = 0.f, d1 = 0.f;
+            if (g != 0.f) {
+              d0 = -g * ex2_approx(fmaf(__uint_as_float(u[j]), kLog2e, -l2));
+              d1 = -g * ex2_approx(fmaf(__uint_as_float(u[j + 1]), kLog2e, -l2));
+              if (lc + j == yy) d0 += g;
+              if (lc + j + 1 == yy) d1 += g;
+            }
+            const __nv_bfloat162 b2 = __floats2bfloat162_rn(d0, d1);
+            pk[j / 2] = *reinterpret_cast<const uint32_t *>(&b2);
+          }
+          if (lc + 32 <= p.cols) {
+            uint4 *dst = reinterpret_cast<uint4 *>(out + lc);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) dst[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+          } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+              if (lc + j < p.cols) {
+                const uint32_t w = pk[j / 2];
+                const uint16_t hbits = (j & 1) ? uint16_t(w >> 16) : uint16_t(w & 0xffffu);
+                reinterpret_cast<uint16_t *>(out)[lc + j] = hbits;
+              }
+            }
+          }
+        }
+        fence_before_sync();
+        mbar_arrive(smem_u32(&ctl->acc_empty[acc]));
+      } else {
+        // kStoreF32 / kStoreBF16: plain tile store (optionally accumulating)
+        const int64_t orow = p.c_row_off + row;
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t u[32];
+          tmem_ld32(taddr + c * 32, u);
+          tmem_wait_ld();
+          const int col = n * BN + c * 32;
+          if (!row_ok || col >= p.cols) continue;
+          const bool full = col + 32 <= p.cols;
+          if constexpr (kEpi == kStoreF32) {
+            float *dst = p.cf + orow * p.ldc + col;
+            if (full) {
+              float4 *d4 = reinterpret_cast<float4 *>(dst);
+#pragma unroll
+              for (int q = 0; q < 8; ++q) {
+                float4 w = make_float4(__uint_as_float(u[4 * q]), __uint_as_float(u[4 * q + 1]),
+                                       __uint_as_float(u[4 * q + 2]), __uint_as_float(u[4 * q + 3]));
+                if (p.accumulate) {
+                  const float4 o = d4[q];
+                  w.x += o.x;
+                  w.y += o.y;
+                  w.z += o.z;
+                  w.w += o.w;
+                }
+                d4[q] = w;
+              }
+            } else {
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (col + j < p.cols) dst[j] = p.accumulate ? dst[j] + __uint_as_float(u[j]) : __uint_as_float(u[j]);
+            }
+          } else {
+            __nv_bfloat16 *dst = p.cb + orow * p.ldc + col;
+            if (full) {
+              uint32_t pk[16];
+#pragma unroll
+              for (int j = 0; j < 32; j += 2) {
+                const __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(u[j]), __uint_as_float(u[j + 1]));
+                pk[j / 2] = *reinterpret_cast<const uint32_t *>(&b2);
+              }
+              uint4 *d4 = reinterpret_cast<uint4 *>(dst);
+#pragma unroll
+              for (int q = 0; q < 4; ++q) d4[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+            } else {
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (col + j < p.cols) dst[j] = __float2bfloat16_rn(__uint_as_float(u[j]));
+            }
+          }
+        }
+        fence_before_sync();
+        mbar_arrive(smem_u32(&ctl->acc_empty[acc]));
+      }
+    }
+  }
+
+  fence_before_sync();
+  __syncthreads();
+  if (warp == 1) {
+    fence_after_sync();
+    tmem_dealloc(tmem_base, TMEM_COLS);
+  }
+}
+
+// fp32 dH accumulator -> bf16 dH (multi-chunk backward only)
+__global__ void f32_to_bf16_kernel(const float *src, __nv_bfloat16 *dst, int64_t n) {
+  const int64_t i = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) * 4;
+  if (i + 4 <= n) {
+    const float4 v = *reinterpret_cast<const float4 *>(src + i);
+    const __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+    uint2 w;
+    w.x = *reinterpret_cast<const uint32_t *>(&a);
+    w.y = *reinterpret_cast<const uint32_t *>(&b);
+    *reinterpret_cast<uint2 *>(dst + i) = w;
+  } else {
+    for (int64_t j = i; j < n; ++j) dst[j] = __float2bfloat16_rn(src[j]);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// host side: tensor maps and launches
+// ---------------------------------------------------------------------------
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor map over a row-major [outer][inner] array with row pitch
+// `pitch_elems`, box {box_inner (64 = 128 bytes), box_outer}, 128-byte swizzle,
+// zero fill outside the array.
+sao_status make_map(CUtensorMap *m, const void *ptr, uint64_t inner, uint64_t outer, uint64_t pitch_elems,
+                    uint32_t box_inner, uint32_t box_outer) {
+  auto fn = encode_fn();
+  if (!fn) return fail(SAO_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+  if ((reinterpret_cast<uintptr_t>(ptr) & 15u) != 0) return fail(SAO_ERR_INVALID_ARG, "bf16 operand not 16-byte aligned");
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {pitch_elems * 2};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(SAO_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", int(r));
+  return SAO_OK;
+}
+
+template <int kEpi, bool kAMN, bool kBMN>
+sao_status launch_gemm(const char *name, const CUtensorMap &ma, const CUtensorMap &mb, const GemmParams &p,
+                       cudaStream_t s) {
+  auto kern = tc_gemm_kernel<kEpi, kAMN, kBMN>;
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [&] {
+    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(SMEM_BYTES));
+  });
+  if (attr_err != cudaSuccess) return fail(SAO_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(attr_err));
+  DeviceInfo di;
+  SAO_TRY(device_info(&di));
+  const int tiles = p.nM * p.nN;
+  if (tiles == 0 || p.nK == 0) return SAO_OK;
+  const int grid = tiles < di.sm_count ? tiles : di.sm_count;
+  int slot = launch_begin(name, s);
+  kern<<<grid, NUM_THREADS, SMEM_BYTES, s>>>(ma, mb, p);
+  return launch_end(slot, s);
+}
+
+int vocab_chunk(int64_t N, int V) {
+  const int64_t vpad = (int64_t(V) + BN - 1) / BN * BN;
+  int64_t vc = int64_t(dz_budget() / (size_t(N > 0 ? N : 1) * 2));
+  vc = vc / BN * BN;
+  if (vc < BN) vc = BN;
+  if (vc > vpad) vc = vpad;
+  return int(vc);
+}
+
+}  // namespace
+
+size_t tc_ws_bytes(int64_t N, int32_t h, int32_t V) {
+  const int64_t nvt = (int64_t(V) + BN - 1) / BN;
+  const size_t fwd = round256(sizeof(float2) * size_t(nvt) * size_t(N)) + round256(sizeof(float) * size_t(N));
+  const int vc = vocab_chunk(N, V);
+  size_t bwd = round256(size_t(N) * size_t(vc) * 2);
+  if (vc < V) bwd += round256(size_t(N) * size_t(h) * sizeof(float));
+  return fwd > bwd ? fwd : bwd;
+}
+
+sao_status tc_fwd(const void *H, const void *W, const int32_t *y, const uint8_t *row_mask, int64_t N, int32_t h,
+                  int32_t V, float *logp, float *lse, unsigned int *err, void *ws, size_t ws_bytes,
+                  cudaStream_t s) {
+  const int nvt = (V + BN - 1) / BN;
+  Carver c(ws, ws_bytes);
+  float2 *part = c.take<float2>(size_t(nvt) * size_t(N));
+  float *zy = c.take<float>(size_t(N));
+  if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the log-prob forward");
+  CUtensorMap ma, mb;
+  SAO_TRY(make_map(&ma, H, uint64_t(h), uint64_t(N), uint64_t(h), 64, BM));
+  SAO_TRY(make_map(&mb, W, uint64_t(h), uint64_t(V), uint64_t(h), 64, BN));
+  GemmParams p{};
+  p.nM = int((N + BM - 1) / BM);
+  p.nN = nvt;
+  p.nK = (h + BK - 1) / BK;
+  p.group_m = 16;
+  p.rows = N;
+  p.cols = V;
+  p.y = y;
+  p.vocab = V;
+  p.part = part;
+  p.zy = zy;
+  p.err = err;
+  SAO_TRY((launch_gemm<kSoftmax, false, false>("tc_logits_lse_fwd", ma, mb, p, s)));
+  return lse_merge_launch(part, nvt, zy, y, row_mask, N, V, logp, lse, err, s);
+}
+
+sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *lse, const float *G, int64_t N,
+                  int32_t h, int32_t V, void *dH, float *dW, int accumulate, unsigned int *err, void *ws,
+                  size_t ws_bytes, cudaStream_t s) {
+  const int Vc = vocab_chunk(N, V);
+  const bool multi = Vc < V;
+  Carver c(ws, ws_bytes);
+  __nv_bfloat16 *dz = c.take<__nv_bfloat16>(size_t(N) * size_t(Vc));
+  float *dh_acc = multi ? c.take<float>(size_t(N) * size_t(h)) : nullptr;
+  if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the log-prob backward");
+
+  CUtensorMap mH_K, mW_K, mH_MN, mW_MN;
+  SAO_TRY(make_map(&mH_K, H, uint64_t(h), uint64_t(N), uint64_t(h), 64, BM));
+  SAO_TRY(make_map(&mW_K, W, uint64_t(h), uint64_t(V), uint64_t(h), 64, BN));
+  SAO_TRY(make_map(&mH_MN, H, uint64_t(h), uint64_t(N), uint64_t(h), 64, 64));
+  SAO_TRY(make_map(&mW_MN, W, uint64_t(h), uint64_t(V), uint64_t(h), 64, 64));
+  const int nMt = int((N + BM - 1) / BM);
+
+  for (int v0 = 0; v0 < V; v0 += Vc) {
+    const int vc = (V - v0) < Vc ? (V - v0) : Vc;
+    const bool first = (v0 == 0), last = (v0 + Vc >= V);
+    CUtensorMap mZ_K, mZ_MN;
+    SAO_TRY(make_map(&mZ_K, dz, uint64_t(vc), uint64_t(N), uint64_t(Vc), 64, BM));
+    SAO_TRY(make_map(&mZ_MN, dz, uint64_t(vc), uint64_t(N), uint64_t(Vc), 64, 64));
+    {  // dZ for vocabulary [v0, v0 + vc)
+      GemmParams p{};
+      p.nM = nMt;
+      p.nN = (vc + BN - 1) / BN;
+      p.nK = (h + BK - 1) / BK;
+      p.group_m = 16;
+      p.b_row_off = v0;
+      p.rows = N;
+      p.cols = vc;
+      p.y = y;
+      p.vocab = V;
+      p.v0 = v0;
+      p.lse = lse;
+      p.G = G;
+      p.dz = dz;
+      p.ldz = Vc;
+      p.err = err;
+      SAO_TRY((launch_gemm<kDLogits, false, false>("tc_dlogits", mH_K, mW_K, p, s)));
+    }
+    {  // dH (+)= dZ W[v0:v0+vc]
+      GemmParams p{};
+      p.nM = nMt;
+      p.nN = (h + BN - 1) / BN;
+      p.nK = (vc + BK - 1) / BK;
+      p.group_m = 1;
+      p.b_row_off = v0;
+      p.rows = N;
+      p.cols = h;
+      p.ldc = h;
+      p.err = err;
+      if (multi) {
+        p.cf = dh_acc;
+        p.accumulate = first ? 0 : 1;
+        SAO_TRY((launch_gemm<kStoreF32, false, true>("tc_dH_gemm", mZ_K, mW_MN, p, s)));
+      } else {
+        p.cb = static_cast<__nv_bfloat16 *>(dH);
+        SAO_TRY((launch_gemm<kStoreBF16, false, true>("tc_dH_gemm", mZ_K, mW_MN, p, s)));
+      }
+    }
+    {  // dW[v0:v0+vc] (+)= dZ^T H
+      GemmParams p{};
+      p.nM = (vc + BM - 1) / BM;
+      p.nN = (h + BN - 1) / BN;
+      p.nK = int((N + BK - 1) / BK);
+      p.group_m = 1;
+      p.rows = vc;
+      p.cols = h;
+      p.cf = dW;
+      p.ldc = h;
+      p.c_row_off = v0;
+      p.accumulate = accumulate;
+      p.err = err;
+      SAO_TRY((launch_gemm<kStoreF32, true, true>("tc_dW_gemm", mZ_MN, mH_MN, p, s)));
+    }
+    if (multi && last) {
+      const int64_t n = N * int64_t(h);
+      const int64_t threads = (n + 3) / 4;
+      int slot = launch_begin("dH_to_bf16", s);
+      f32_to_bf16_kernel<<<unsigned((threads + 255) / 256), 256, 0, s>>>(dh_acc, static_cast<__nv_bfloat16 *>(dH), n);
+      SAO_TRY(launch_end(slot, s));
+    }
+  }
+  return SAO_OK;
+}
+
+}  // namespace sao

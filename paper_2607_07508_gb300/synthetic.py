@@ -114,6 +114,12 @@ def lognormal_lengths(rng, total: int, median: int, max_len: int, min_len: int =
     return _fit_total(np.array(draws), total, min_len, max_len)
 
 
+def lognormal_lengths_n(rng, n: int, total: int, median: int, max_len: int, min_len: int = 16,
+                        sigma: float = 1.0) -> np.ndarray:
+    raw = np.clip(rng.lognormal(math.log(median), sigma, size=n), min_len, max_len)
+    return _fit_total(raw, total, min_len, max_len)
+
+
 def pareto_lengths(rng, n: int, total: int, lo: int, hi: int, shape: float = 1.5) -> np.ndarray:
     raw = lo * (1.0 + rng.pareto(shape, size=n))
     return _fit_total(np.clip(raw, lo, hi), total, lo, hi)
@@ -206,13 +212,13 @@ def make_workload(name: str, *, dense: bool = True, device="cpu", seed: Optional
     elif name == "small":
         h, V, dtype = 1024, 32000, "bf16"
         N = 98304 if N_override is None else N_override
-        lengths = lognormal_lengths(rng, N, 1024, 8192)
+        lengths = lognormal_lengths_n(rng, 64, N, 1024, 8192)
         mask = np.ones(N, np.uint8)
         stale = rng.random(N) < 0.3
         xi = np.where(stale, rng.normal(0.0, 0.1, size=N), 0.0)
         gamma, lam, lam_c, alpha, el, eh = 1.0, 1.0, 1.0, 0.0, 0.2, 0.28
         vm, vs, pr = 0.4, 0.2, 0.4
-        recipe = "lognormal(median 1k, sigma 1) clamp [16,8k] to 98304 tokens; xi~N(0,0.1) on 30%"
+        recipe = "64 lognormal(median 1k, sigma 1) lengths clamp [16,8k] fit to 98304 tokens; xi~N(0,0.1) on 30%"
     elif name == "moe":
         h, V, dtype = 2048, 151936, "bf16"
         N = 65536 if N_override is None else N_override
@@ -245,7 +251,7 @@ def make_workload(name: str, *, dense: bool = True, device="cpu", seed: Optional
     elif name == "large":
         h, V, dtype = 6144, 154880, "bf16"
         N = 262144 if N_override is None else N_override
-        lengths = lognormal_lengths(rng, N, 2048, 65536)
+        lengths = lognormal_lengths_n(rng, 128, N, 2048, 65536)
         mask = np.ones(N, np.uint8)
         el, eh = PAPER_EPS_REASONING
         xi = rng.normal(0.0, 0.05, size=N)
@@ -257,7 +263,7 @@ def make_workload(name: str, *, dense: bool = True, device="cpu", seed: Optional
         xi = np.where(push, -np.log(r_target), xi)
         gamma, lam, lam_c, alpha = 1.0, 1.0, 1.0, 0.0
         vm, vs, pr = 0.4, 0.2, 0.4
-        recipe = ("lognormal(median 2k, sigma 1) clamp [16,64k] to 262144 tokens; 10% of tokens "
+        recipe = ("128 lognormal(median 2k, sigma 1) lengths clamp [16,64k] fit to 262144 tokens; 10% of tokens "
                   "with a target ratio outside the clip bounds, the rest xi~N(0,0.05)")
     else:
         raise KeyError(name)

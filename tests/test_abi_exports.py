@@ -1,0 +1,85 @@
+"""libsao builds for sm_103a, loads, and exports every entry point include/sao.h
+declares; argument checks that return before any CUDA call work without a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "sao.h")
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(sao_[a-z0-9_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2607_07508_gb300 import build, sao
+    build.build()
+    return sao.load()
+
+
+def test_header_declares_the_six_operations():
+    names = _declared()
+    for op in ("sao_token_logprobs_fwd", "sao_token_logprobs_bwd", "sao_advantages", "sao_policy_loss_fwd",
+               "sao_policy_loss_bwd", "sao_value_loss", "sao_workspace_bytes"):
+        assert op in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    missing = [n for n in _declared() if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def test_binding_covers_every_export(lib):
+    from paper_2607_07508_gb300 import sao
+    assert sorted(sao.EXPORTS) == _declared()
+
+
+def test_library_needs_no_cuda_shared_libraries():
+    """The static CUDA runtime is linked in and the driver is found at run time,
+    so the library loads on a machine without a GPU driver."""
+    import shutil
+    import subprocess
+    from paper_2607_07508_gb300 import build
+    if shutil.which("readelf") is None:
+        pytest.skip("readelf not available")
+    out = subprocess.run(["readelf", "-d", build.build()], capture_output=True, text=True).stdout
+    needed = [l for l in out.splitlines() if "NEEDED" in l]
+    assert needed and not any("libcuda" in l for l in needed), needed
+
+
+def test_workspace_sizes(lib):
+    from paper_2607_07508_gb300 import sao
+    small = sao.sao_workspace_bytes(1024)
+    big = sao.sao_workspace_bytes(65536, 2048, 151936)
+    assert small >= 256 and big > small
+    assert sao.sao_workspace_bytes(-1) == 0
+
+
+def test_argument_errors_without_gpu(lib):
+    P = ctypes.c_void_p
+    # NULL loss pointer: rejected before any CUDA call
+    st = lib.sao_policy_loss_fwd(None, None, None, None, 0, 0.2, 0.28, 0, None, None, None, None, None, 0, None)
+    assert st == 1
+    # negative clip bound
+    st = lib.sao_policy_loss_fwd(None, None, None, None, 0, -0.1, 0.28, 0, P(8), None, None, P(8), None, 0, None)
+    assert st == 1
+    # bf16 needs h % 8 == 0
+    st = lib.sao_token_logprobs_fwd(P(8), P(8), 1, P(8), None, 16, 12, 100, P(8), P(8), None, 0, None)
+    assert st == 2
+    # unknown dtype
+    st = lib.sao_token_logprobs_fwd(P(8), P(8), 7, P(8), None, 16, 16, 100, P(8), P(8), None, 0, None)
+    assert st == 4
+    # gamma outside [0, 1]
+    st = lib.sao_advantages(P(8), P(8), P(8), P(8), 1, 16, 1.5, 1.0, 1.0, 0.0, P(8), P(8), P(8), 1 << 20, None)
+    assert st == 1
+    # tokens without trajectories
+    st = lib.sao_advantages(P(8), P(8), P(8), P(8), 0, 16, 1.0, 1.0, 1.0, 0.0, P(8), P(8), P(8), 1 << 20, None)
+    assert st == 2
+    msg = lib.sao_last_error_string().decode()
+    assert "trajectory" in msg
