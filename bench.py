@@ -260,6 +260,67 @@ def workload_config(wl):
             "l2": "inputs larger than L2 (H 268 MB + W 622 MB per step, L2 126 MB); no flush"}
 
 
+# Algorithmic bytes per token of each O(N) kernel (reads + writes).
+ON_BYTES = {"gae_scan": 13, "policy_loss_fwd": 18, "policy_loss_bwd": 17, "value_loss": 13, "count_mask": 1,
+            "gae_count": 1}
+
+
+def bandwidth_study(args):
+    """HBM study of the O(N) kernels on the 2^27-token workload (inputs far
+    above L2): achieved algorithmic GB/s per kernel from the library's own
+    CUDA-event timing, against the measured HBM copy bandwidth."""
+    import torch
+    from paper_2607_07508_gb300 import sao, synthetic as S
+    torch.cuda.set_device(0)
+    sao.load()
+    peaks, src = load_peaks()
+    N = args.tokens or (1 << 27)
+    wl = S.bandwidth_workload(N=N, B=max(1, N >> 13))
+    dev = "cuda"
+    t = lambda a: torch.as_tensor(a).to(dev)
+    v, m, cu, R = t(wl.values), t(wl.loss_mask), t(wl.cu_seqlens), t(wl.rewards)
+    lp, old = t(wl.logp_syn), t(wl.old_logp_syn)
+    f = lambda: torch.empty(N, dtype=torch.float32, device=dev)
+    adv, ret, coef, grad, dV = f(), f(), f(), f(), f()
+    flags = torch.empty(N, dtype=torch.uint8, device=dev)
+    loss = torch.empty(1, device=dev)
+    counts = torch.empty(4, dtype=torch.int64, device=dev)
+    ev = torch.empty(4, dtype=torch.float64, device=dev)
+    one = torch.ones(1, device=dev)
+    ws = sao.workspace(N)
+
+    def calls():
+        sao.sao_advantages(v, R, m, cu, wl.gamma, wl.lam, wl.lam_critic, 0.0, adv, ret, ws)
+        sao.sao_advantages(v, R, m, cu, 1.0, 1.0, 1.0, 1.5, adv, ret, ws)
+        sao.sao_policy_loss_fwd(lp, old, adv, m, wl.eps_low, wl.eps_high, loss, counts, ws, coef=coef, flags=flags)
+        sao.sao_policy_loss_bwd(lp, old, adv, m, wl.eps_low, wl.eps_high, one, grad, ws)
+        sao.sao_value_loss(v, ret, m, loss, dV, ws, ev_sums=ev)
+
+    for _ in range(max(3, args.warmup)):
+        calls()
+    torch.cuda.synchronize()
+    sao.sao_profile_enable(True)
+    sao.sao_profile_reset()
+    for _ in range(args.steps):
+        calls()
+    torch.cuda.synchronize()
+    prof = sao.sao_profile_read()
+    sao.sao_profile_enable(False)
+    out = {}
+    names = {"policy_loss_fwd": "policy_loss_fwd", "policy_loss_bwd": "policy_loss_bwd"}
+    for k, (n, ms) in prof.items():
+        b = ON_BYTES.get(names.get(k, k))
+        avg = ms / n
+        row = {"launches": n, "avg_us": 1000 * avg}
+        if b is not None:
+            gbs = b * N / (avg / 1000) / 1e9
+            row.update({"bytes_per_token": b, "achieved_gbs": gbs, "frac_of_hbm": gbs / peaks["hbm_gbs"]})
+        out[k] = row
+    print(json.dumps({"study": "O(N) kernels, HBM", "tokens": N, "trajectories": wl.B,
+                      "peak_hbm_gbs": peaks["hbm_gbs"], "peak_source": src, "kernels": out}))
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -268,9 +329,15 @@ def main():
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--tokens", type=int, default=None,
+                    help="override the packed token count (smaller cases for profiling captures)")
+    ap.add_argument("--bandwidth-study", action="store_true",
+                    help="time the O(N) kernels alone on the 2^27-token bandwidth workload")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.bandwidth_study:
+        return bandwidth_study(args)
 
     import torch
     from paper_2607_07508_gb300 import sao, synthetic as S
@@ -284,7 +351,8 @@ def main():
     sao.load()
     peaks, peak_src = load_peaks()
 
-    wl = S.make_workload(WORKLOAD, device=dev, seed=S.SEED_BASE + S.CONFIG_NAMES.index(WORKLOAD) + 97 * rank)
+    wl = S.make_workload(WORKLOAD, device=dev, seed=S.SEED_BASE + S.CONFIG_NAMES.index(WORKLOAD) + 97 * rank,
+                         N_override=args.tokens)
     step = LossHeadStep(wl, dev, torch)
     stream = torch.cuda.current_stream()
     for _ in range(max(3, args.warmup)):

@@ -1,0 +1,127 @@
+"""Full-size parity of the tensor-core log-prob path, in the launch
+configuration bench.py times (persistent grid, many tiles per CTA).
+
+The oracle cannot redo 2*N*h*V fp64 flops at these sizes, so:
+  * logp and lse are checked on a seeded sample of rows, each over the whole
+    vocabulary (the oracle's own forward on those rows);
+  * with the incoming gradient non-zero only on sampled rows, dH is checked on
+    those rows (and must be exactly zero elsewhere) and dW on a seeded sample
+    of vocabulary rows that includes the sampled tokens (the oracle's own lse);
+  * with a dense gradient, dH is checked on sampled rows, and dW against the
+    linearity property dW(G) = dW(G on S) + dW(G off S) plus the column sums
+    sum_v dW[v, :] = 0 that every softmax gradient satisfies.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import sao_oracle as O
+from paper_2607_07508_gb300 import sao, synthetic as S
+from tests._util import rel_l2
+
+pytestmark = pytest.mark.gpu
+
+LOGP_TOL = 2e-3
+GRAD_TOL = 2e-2
+
+
+def _run(wl, G=None, ws=None):
+    N, h, V = wl.N, wl.h, wl.V
+    y = torch.as_tensor(wl.y).cuda()
+    ws = ws if ws is not None else sao.workspace(N, h, V, wl.H.dtype)
+    logp = torch.empty(N, device="cuda")
+    lse = torch.empty(N, device="cuda")
+    sao.sao_token_logprobs_fwd(wl.H, wl.W, y, logp, lse, ws)
+    if G is None:
+        return logp, lse, None, None, ws
+    dH = torch.empty_like(wl.H)
+    dW = torch.empty(V, h, device="cuda")
+    sao.sao_token_logprobs_bwd(wl.H, wl.W, y, lse, G, dH, dW, ws)
+    return logp, lse, dH, dW, ws
+
+
+def _oracle_dW_rows(Hs, W_cpu, ys, lse_s, Gs, vrows):
+    """dW restricted to vocabulary rows `vrows` for the sampled token rows."""
+    Wsub = W_cpu[torch.as_tensor(vrows)]
+    pos = {int(v): i for i, v in enumerate(vrows)}
+    ysub = np.array([pos.get(int(t), -1) for t in ys])
+    Hd = O._f64(Hs)
+    Z = Hd @ O._f64(Wsub).T
+    dZ = -Gs[:, None] * np.exp(Z - lse_s[:, None])
+    for i, j in enumerate(ysub):
+        if j >= 0:
+            dZ[i, j] += Gs[i]
+    return dZ.T @ Hd
+
+
+@pytest.mark.parametrize("name", ["small", "moe", "long", "large"])
+def test_full_size_sampled_rows(name):
+    torch.manual_seed(0)
+    wl = S.make_workload(name, device="cuda")
+    rng = np.random.default_rng(11)
+    rows = np.sort(rng.choice(wl.N, size=32, replace=False))
+    G = np.zeros(wl.N, np.float32)
+    G[rows] = rng.normal(size=len(rows)).astype(np.float32)
+    logp, lse, dH, dW, ws = _run(wl, torch.as_tensor(G).cuda())
+    torch.cuda.synchronize()
+    H_cpu, W_cpu = wl.H[torch.as_tensor(rows).cuda()].cpu(), wl.W.cpu()
+    want_lp, want_lse = O.token_logprobs(H_cpu, W_cpu, wl.y[rows])
+    assert np.abs(logp.cpu().numpy()[rows] - want_lp).max() <= LOGP_TOL
+    assert np.abs(lse.cpu().numpy()[rows] - want_lse).max() <= LOGP_TOL
+    # dH on the sampled rows, exact zeros elsewhere
+    want_dH, _ = O.token_logprobs_bwd(H_cpu, W_cpu, wl.y[rows], want_lse, G[rows])
+    got_dH = dH.float().cpu().numpy()
+    assert rel_l2(got_dH[rows], want_dH) <= GRAD_TOL
+    others = np.ones(wl.N, bool)
+    others[rows] = False
+    assert not np.any(got_dH[others])
+    # dW on a vocabulary sample that includes the sampled tokens
+    vrows = np.unique(np.concatenate([rng.choice(wl.V, size=512, replace=False), wl.y[rows], [wl.V - 1]]))
+    want_dW = _oracle_dW_rows(H_cpu, W_cpu, wl.y[rows], want_lse, G[rows].astype(np.float64), vrows)
+    got_dW = dW[torch.as_tensor(vrows).cuda()].cpu().numpy()
+    assert rel_l2(got_dW, want_dW) <= GRAD_TOL
+
+
+@pytest.mark.parametrize("name", ["moe", "large"])
+def test_full_size_dense_gradient(name):
+    wl = S.make_workload(name, device="cuda")
+    rng = np.random.default_rng(12)
+    G = (rng.normal(size=wl.N) * 1e-4).astype(np.float32)
+    G[wl.loss_mask == 0] = 0.0
+    rows = np.sort(rng.choice(np.flatnonzero(G), size=24, replace=False))
+    Gt = torch.as_tensor(G).cuda()
+    logp, lse, dH, dW, ws = _run(wl, Gt)
+    torch.cuda.synchronize()
+    H_cpu, W_cpu = wl.H[torch.as_tensor(rows).cuda()].cpu(), wl.W.cpu()
+    _, want_lse = O.token_logprobs(H_cpu, W_cpu, wl.y[rows])
+    want_dH, _ = O.token_logprobs_bwd(H_cpu, W_cpu, wl.y[rows], want_lse, G[rows])
+    assert rel_l2(dH.float().cpu().numpy()[rows], want_dH) <= GRAD_TOL
+    # linearity in G: split the rows into two disjoint sets
+    part = rng.random(wl.N) < 0.5
+    G1 = torch.as_tensor(np.where(part, G, 0).astype(np.float32)).cuda()
+    G2 = torch.as_tensor(np.where(part, 0, G).astype(np.float32)).cuda()
+    y = torch.as_tensor(wl.y).cuda()
+    dH1 = torch.empty_like(wl.H)
+    dW12 = torch.empty_like(dW)
+    sao.sao_token_logprobs_bwd(wl.H, wl.W, y, lse, G1, dH1, dW12, ws)
+    sao.sao_token_logprobs_bwd(wl.H, wl.W, y, lse, G2, dH1, dW12, ws, accumulate_dW=True)
+    torch.cuda.synchronize()
+    diff = torch.linalg.vector_norm(dW12 - dW).item() / torch.linalg.vector_norm(dW).item()
+    assert diff <= 1e-2
+    colsum = dW.sum(dim=0).abs().max().item()
+    assert colsum <= 1e-2 * dW.abs().sum(dim=0).max().item()
+
+
+def test_many_tiles_per_cta_full_oracle():
+    """2048 x 20000 logits = 1264 tiles, about 8 per CTA: the persistent loop,
+    both TMEM accumulators and the ring phases across tiles, checked fully."""
+    wl = S.make_custom([2048], 256, 20000, "bf16", seed=77, device="cuda")
+    G = np.random.default_rng(5).normal(size=wl.N).astype(np.float32)
+    logp, lse, dH, dW, _ = _run(wl, torch.as_tensor(G).cuda())
+    torch.cuda.synchronize()
+    H_cpu, W_cpu = wl.H.cpu(), wl.W.cpu()
+    want_lp, want_lse = O.token_logprobs(H_cpu, W_cpu, wl.y)
+    assert np.abs(logp.cpu().numpy() - want_lp).max() <= LOGP_TOL
+    want_dH, want_dW = O.token_logprobs_bwd(H_cpu, W_cpu, wl.y, want_lse, G)
+    assert rel_l2(dH.float().cpu().numpy(), want_dH) <= GRAD_TOL
+    assert rel_l2(dW.cpu().numpy(), want_dW) <= GRAD_TOL
