@@ -153,6 +153,33 @@ SAO_API sao_status sao_advantages(const float *values, const float *rewards, con
                           float *adv, float *ret, void *ws, size_t ws_bytes, sao_stream_t stream);
 
 /*
+ * sao_advantages without a workspace argument, for callers that cannot
+ * allocate device memory: a host library that is handed only data pointers
+ * and a stream by another framework and has no allocator of its own, or a
+ * process that reserves all device memory at start-up and forbids later
+ * allocations (cudaMalloc also synchronises the whole device, which a
+ * latency-critical caller cannot afford). The paper has no counterpart to
+ * this entry point; it computes exactly what sao_advantages computes.
+ *
+ * Scratch: a fixed 8 MiB array inside this library's device image, present on
+ * every GPU that loads the library until the process exits. It bounds the
+ * sizes: 256 + gae scratch(N, B) bytes must fit, about 88 bytes per 4096
+ * tokens plus 36 bytes per trajectory (for example 2^27 tokens with up to
+ * 131,072 trajectories); larger inputs return SAO_ERR_SHAPE with the bytes
+ * needed. Nothing is allocated and nothing is freed.
+ * The first call on each device looks up the array's device address (with
+ * that device current) and caches it; make that first call before any stream
+ * capture. Every call on a device shares the one array, so calls that overlap
+ * on the GPU (two streams, or two threads) race and corrupt each other's
+ * results; serialise them. Each call clears the parts of the array that must
+ * start at zero, so stale contents from a previous call do no harm.
+ */
+SAO_API sao_status sao_advantages_noalloc(const float *values, const float *rewards, const uint8_t *loss_mask,
+                                          const int32_t *cu_seqlens, int32_t B, int64_t N, float gamma,
+                                          float lambda_policy, float lambda_critic, float len_adaptive_alpha,
+                                          float *adv, float *ret, sao_stream_t stream);
+
+/*
  * Eq. 1-3 (§3.1). r_t = exp(logp_t - old_logp_t); a token is kept iff it is an
  * action token, its log-ratio and advantage are finite and
  * 1 - eps_low < r_t < 1 + eps_high (strict; decided in fp32). With n = n_norm

@@ -24,7 +24,8 @@ FLAG_IN, FLAG_LOW, FLAG_HIGH, FLAG_NONFINITE, FLAG_NOT_ACTION = 0, 1, 2, 3, 4
 
 EXPORTS = ("sao_version", "sao_last_error_string", "sao_set_checked", "sao_get_checked",
            "sao_set_dz_budget_bytes", "sao_workspace_bytes", "sao_token_logprobs_fwd",
-           "sao_token_logprobs_bwd", "sao_advantages", "sao_policy_loss_fwd", "sao_policy_loss_bwd",
+           "sao_token_logprobs_bwd", "sao_advantages", "sao_advantages_noalloc", "sao_policy_loss_fwd",
+           "sao_policy_loss_bwd",
            "sao_value_loss", "sao_profile_enable", "sao_profile_reset", "sao_profile_read")
 
 
@@ -59,6 +60,7 @@ def load(path: Optional[str] = None):
         "sao_token_logprobs_bwd": (ctypes.c_int, [P, P, ctypes.c_int, P, P, P, I64, I32, I32, P, P,
                                                   ctypes.c_int, P, SZ, P]),
         "sao_advantages": (ctypes.c_int, [P, P, P, P, I32, I64, F, F, F, F, P, P, P, SZ, P]),
+        "sao_advantages_noalloc": (ctypes.c_int, [P, P, P, P, I32, I64, F, F, F, F, P, P, P]),
         "sao_policy_loss_fwd": (ctypes.c_int, [P, P, P, P, I64, F, F, I64, P, P, P, P, P, SZ, P]),
         "sao_policy_loss_bwd": (ctypes.c_int, [P, P, P, P, I64, F, F, I64, P, P, P, SZ, P]),
         "sao_value_loss": (ctypes.c_int, [P, P, P, I64, P, P, P, P, SZ, P]),
@@ -189,6 +191,23 @@ def sao_advantages(values, rewards, loss_mask, cu_seqlens, gamma, lambda_policy,
                                  float(gamma), float(lambda_policy), float(lambda_critic),
                                  float(len_adaptive_alpha), _ptr(adv), _ptr(ret), _ptr(ws), ws.numel(),
                                  _stream(stream)))
+
+
+def sao_advantages_noalloc(values, rewards, loss_mask, cu_seqlens, gamma, lambda_policy, lambda_critic,
+                           len_adaptive_alpha, adv, ret, stream=None):
+    """sao_advantages with the library's fixed device scratch instead of a
+    workspace, for callers that cannot allocate device memory."""
+    N = values.numel()
+    B = cu_seqlens.numel() - 1
+    _expect(values, torch.float32, N, "values")
+    _expect(rewards, torch.float32, B, "rewards")
+    _expect(loss_mask, torch.uint8, N, "loss_mask")
+    _expect(cu_seqlens, torch.int32, B + 1, "cu_seqlens")
+    _expect(adv, torch.float32, N, "adv")
+    _expect(ret, torch.float32, N, "ret")
+    _check(load().sao_advantages_noalloc(_ptr(values), _ptr(rewards), _ptr(loss_mask), _ptr(cu_seqlens), B, N,
+                                         float(gamma), float(lambda_policy), float(lambda_critic),
+                                         float(len_adaptive_alpha), _ptr(adv), _ptr(ret), _stream(stream)))
 
 
 def sao_policy_loss_fwd(logp, old_logp, adv, loss_mask, eps_low, eps_high, loss, counts, ws, coef=None,
