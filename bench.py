@@ -153,7 +153,8 @@ class LossHeadStep:
         s.sao_advantages(self.values, self.rewards, self.mask, self.cu, wl.gamma, wl.lam, wl.lam_critic, wl.alpha,
                          self.adv, self.ret, self.ws)
         s.sao_value_loss(self.values, self.ret, self.mask, self.vloss, self.dV, self.ws, ev_sums=self.ev)
-        s.sao_token_logprobs_fwd(self.H, self.W, self.y, self.logp, self.lse, self.ws)
+        # log-probs of observation tokens are never read: skip those rows
+        s.sao_token_logprobs_fwd(self.H, self.W, self.y, self.logp, self.lse, self.ws, row_mask=self.mask)
         s.sao_policy_loss_fwd(self.logp, self.old, self.adv, self.mask, wl.eps_low, wl.eps_high, self.loss,
                               self.counts, self.ws, coef=self.coef, flags=self.flags)
         s.sao_policy_loss_bwd(self.logp, self.old, self.adv, self.mask, wl.eps_low, wl.eps_high, self.one, self.G,
@@ -161,12 +162,14 @@ class LossHeadStep:
         s.sao_token_logprobs_bwd(self.H, self.W, self.y, self.lse, self.G, self.dH, self.dW, self.ws)
 
 
-# Algorithmic work per launch of each tensor-core kernel, in flops, for N rows.
-def kernel_flops(name, N, h, V, rows_g):
+# Algorithmic work per launch of each tensor-core kernel, in flops: the
+# forward computes the rows with loss_mask = 1, the backward kernels the rows
+# with a non-zero incoming gradient.
+def kernel_flops(name, h, V, rows_fwd, rows_bwd):
     if name == "tc_logits_lse_fwd":
-        return 2.0 * N * h * V
+        return 2.0 * rows_fwd * h * V
     if name in ("tc_dlogits", "tc_dH_gemm", "tc_dW_gemm"):
-        return 2.0 * N * h * V
+        return 2.0 * rows_bwd * h * V
     return None
 
 
@@ -391,30 +394,35 @@ def main():
     value = total_tokens / (ms / 1000.0)
 
     # ---- roofline of the dominant kernel --------------------------------------
+    rows_fwd = int(step.mask.sum().item())
+    rows_bwd = int((step.G != 0).sum().item())
     launches = sum(n for n, _ in prof.values())
     dom = max(prof.items(), key=lambda kv: kv[1][1])
     dom_name, (dom_n, dom_ms) = dom
     avg_ms = dom_ms / dom_n
-    fl = kernel_flops(dom_name, wl.N, wl.h, wl.V, None)
+    fl = kernel_flops(dom_name, wl.h, wl.V, rows_fwd, rows_bwd)
     peak_t = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
     if fl is not None:
         achieved = fl / (avg_ms / 1000.0) / 1e12
         roofline = {"bound": "tensor", "kernel": dom_name, "achieved": achieved, "peak": peak_t,
                     "unit": "TFLOP/s", "frac": achieved / peak_t, "traffic": None,
-                    "algorithmic_per_launch": f"2*N*h*V = {fl:.4g} flop", "avg_launch_ms": avg_ms,
+                    "algorithmic_per_launch": f"2*rows*h*V = {fl:.4g} flop", "avg_launch_ms": avg_ms,
                     "peak_source": f"{peak_src} bf16_tflops_sustained (kernel timed inside a long step)"}
     else:
         roofline = {"bound": "hbm", "kernel": dom_name, "achieved": None, "peak": peaks.get("hbm_gbs"),
                     "unit": "GB/s", "frac": None, "traffic": None}
-    step_alg = 6.0 * wl.N * wl.h * wl.V
-    step_exec = 8.0 * wl.N * wl.h * wl.V
+    step_alg = 2.0 * wl.h * wl.V * (rows_fwd + 2 * rows_bwd)
+    step_exec = 2.0 * wl.h * wl.V * (rows_fwd + 3 * rows_bwd)
     burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
     step_roof = {"algorithmic_tflops": step_alg / (ms / 1000) / 1e12,
                  "frac_of_burst_peak": step_alg / (ms / 1000) / 1e12 / burst,
                  "executed_tflops": step_exec / (ms / 1000) / 1e12,
                  "executed_frac_of_sustained_peak": step_exec / (ms / 1000) / 1e12 / peak_t,
-                 "algorithmic_flops_per_step": "6*N*h*V (2hV fwd + 4hV bwd per token)",
-                 "executed_flops_per_step": "8*N*h*V (the backward recomputes the logits)",
+                 "algorithmic_flops_per_step": f"2hV per forward row ({rows_fwd} action tokens) + 4hV per row "
+                                               f"with a non-zero gradient ({rows_bwd}); 6*N*h*V = "
+                                               f"{6.0 * wl.N * wl.h * wl.V:.4g} if no row were skipped",
+                 "executed_flops_per_step": "algorithmic + 2hV per backward row (the logits are recomputed)",
+                 "rows_forward": rows_fwd, "rows_backward": rows_bwd,
                  "peak_source": peak_src}
     kernels = {k: {"launches": n, "avg_ms": t / n} for k, (n, t) in sorted(prof.items(), key=lambda kv: -kv[1][1])}
 

@@ -8,12 +8,13 @@
 
 namespace sao {
 
-// Merges per-(vocab tile, row) partials part[j * N + row] = (max_j, sumexp_j)
-// into lse[row] = log sum_v e^z and logp[row] = zy[row] - lse[row]. Rows with
-// row_mask == 0 get logp = lse = 0; rows whose token id is outside [0, V) get
-// logp = NaN.
+// Merges per-(vocab tile, row) partials part[j * N + i] = (max_j, sumexp_j)
+// into lse[row] = log sum_v e^z and logp[row] = zy[i] - lse[row], where i is
+// the row itself, or pos[row] when the forward ran on compacted rows (pos < 0:
+// a skipped row, logp = lse = 0). Rows with row_mask == 0 also get zeros.
+// Token ids outside [0, V) give logp = NaN.
 sao_status lse_merge_launch(const float2 *part, int nvt, const float *zy, const int32_t *y,
-                            const uint8_t *row_mask, int64_t N, int32_t V, float *logp, float *lse,
+                            const uint8_t *row_mask, const int *pos, int64_t N, int32_t V, float *logp, float *lse,
                             unsigned int *err, cudaStream_t s);
 
 size_t simt_ws_bytes(int64_t N, int32_t h, int32_t V);

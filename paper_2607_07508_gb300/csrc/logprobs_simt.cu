@@ -193,7 +193,7 @@ sao_status simt_fwd(const float *H, const float *W, const int32_t *y, const uint
   int slot = launch_begin("simt_logits_fwd", s);
   simt_fwd_kernel<<<grid, 256, 0, s>>>(H, W, y, row_mask, N, h, V, part, zy, err);
   SAO_TRY(launch_end(slot, s));
-  return lse_merge_launch(part, nvt, zy, y, row_mask, N, V, logp, lse, err, s);
+  return lse_merge_launch(part, nvt, zy, y, row_mask, nullptr, N, V, logp, lse, err, s);
 }
 
 sao_status simt_bwd(const float *H, const float *W, const int32_t *y, const float *lse, const float *G,

@@ -27,6 +27,7 @@
 #include <mutex>
 
 #include "logprobs_common.cuh"
+#include "rows.cuh"
 #include "sao_common.cuh"
 #include "sao_internal.h"
 #include "tc_ptx.cuh"
@@ -43,7 +44,9 @@ constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int NUM_THREADS = 192;
 constexpr uint32_t TMEM_COLS = 2 * BN;
 constexpr uint32_t MN_ATOM_BYTES = 64 * BK * 2;   // one 64(MN) x 64(K) box
-constexpr size_t SMEM_BYTES = 1024 + size_t(STAGES) * STAGE_BYTES + 256;
+constexpr uint32_t STAGE_OUT_BYTES = BM * 64 * 2; // one 128-row x 64-column bf16 output box
+constexpr size_t SMEM_BYTES = 1024 + size_t(STAGES) * STAGE_BYTES + 2 * STAGE_OUT_BYTES + 256;
+constexpr int EPI_BARRIER = 1;                    // named barrier of the 4 epilogue warps
 constexpr float kLog2e = 1.4426950408889634f;
 
 enum EpiKind : int { kSoftmax = 0, kDLogits = 1, kStoreF32 = 2, kStoreBF16 = 3 };
@@ -70,6 +73,11 @@ struct GemmParams {
   int64_t c_row_off;   // output row offset
   int accumulate;
   unsigned int *err;
+  // row compaction (all optional): M extent and K extent read from the
+  // device at start-up, and the original row of each compacted GEMM row
+  const int *m_count;
+  const int *k_count;
+  const int *row_idx;
 };
 
 struct __align__(8) SmemCtl {
@@ -78,12 +86,12 @@ struct __align__(8) SmemCtl {
   int abort;
 };
 
-__device__ __forceinline__ void tile_coords(int L, const GemmParams &p, int &m, int &n) {
+__device__ __forceinline__ void tile_coords(int L, const GemmParams &p, int nM, int &m, int &n) {
   const int per_group = p.group_m * p.nN;
   const int g = L / per_group;
   const int within = L - g * per_group;
   const int m0 = g * p.group_m;
-  const int gm = min(p.group_m, p.nM - m0);
+  const int gm = min(p.group_m, nM - m0);
   m = m0 + within % gm;
   n = within / gm;
 }
@@ -91,16 +99,26 @@ __device__ __forceinline__ void tile_coords(int L, const GemmParams &p, int &m, 
 template <int kEpi, bool kAMN, bool kBMN>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
-                   const GemmParams p) {
+                   const __grid_constant__ CUtensorMap map_c, const GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t *gbase = smem_raw + (base - raw);
-  SmemCtl *ctl = reinterpret_cast<SmemCtl *>(gbase + size_t(STAGES) * STAGE_BYTES);
+  const uint32_t out_base = base + uint32_t(STAGES) * STAGE_BYTES;  // 2 output staging boxes
+  SmemCtl *ctl = reinterpret_cast<SmemCtl *>(gbase + size_t(STAGES) * STAGE_BYTES + 2 * STAGE_OUT_BYTES);
   volatile int *abort = &ctl->abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int num_tiles = p.nM * p.nN;
+  int nM = p.nM, nK = p.nK;
+  int64_t rows = p.rows;
+  if (p.m_count) {
+    const int c = *p.m_count;
+    rows = c;
+    nM = (c + BM - 1) / BM;
+  }
+  if (p.k_count) nK = (*p.k_count + BK - 1) / BK;
+  const int num_tiles = nM * p.nN;
+  const bool kzero = (nK == 0);  // empty contraction: the tile is all zeros
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -137,8 +155,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       uint32_t issued_phase = 0;
       for (int L = blockIdx.x; L < num_tiles && ok; L += gridDim.x) {
         int m, n;
-        tile_coords(L, p, m, n);
-        for (int kb = 0; kb < p.nK; ++kb) {
+        tile_coords(L, p, nM, m, n);
+        for (int kb = 0; kb < nK; ++kb) {
           if (!mbar_wait(smem_u32(&ctl->empty[stage]), phase ^ 1u, abort, p.err)) {
             ok = false;
             break;
@@ -195,7 +213,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         if (!mbar_wait(smem_u32(&ctl->acc_empty[acc]), acc_phase ^ 1u, abort, p.err)) break;
         fence_after_sync();
         const uint32_t d_tmem = tmem_base + uint32_t(acc) * BN;
-        for (int kb = 0; kb < p.nK; ++kb) {
+        for (int kb = 0; kb < nK; ++kb) {
           if (!mbar_wait(smem_u32(&ctl->full[stage]), phase, abort, p.err)) {
             ok = false;
             break;
@@ -228,18 +246,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     int local = 0;
     for (int L = blockIdx.x; L < num_tiles; L += gridDim.x, ++local) {
       int m, n;
-      tile_coords(L, p, m, n);
+      tile_coords(L, p, nM, m, n);
       const int acc = local & 1;
       const uint32_t acc_phase = uint32_t(local >> 1) & 1u;
-      if (!mbar_wait(smem_u32(&ctl->acc_full[acc]), acc_phase, abort, p.err)) break;
+      bool ok = mbar_wait(smem_u32(&ctl->acc_full[acc]), acc_phase, abort, p.err);
+      // The dlogits epilogue synchronises its 4 warps with named barriers, so
+      // they must agree on whether this tile goes ahead.
+      if constexpr (kEpi == kDLogits) ok = named_barrier_and(EPI_BARRIER, 128, ok);
+      if (!ok) break;
       fence_after_sync();
       const uint32_t taddr = tmem_base + (uint32_t(quad * 32) << 16) + uint32_t(acc) * BN;
       const int64_t row = int64_t(m) * BM + r;
-      const bool row_ok = row < p.rows;
+      const bool row_ok = row < rows;
+      const int64_t orig = (row_ok && p.row_idx) ? int64_t(__ldg(p.row_idx + row)) : row;
 
       if constexpr (kEpi == kSoftmax) {
         const int col0 = n * BN;
-        const int yy = row_ok ? __ldg(p.y + row) : -1;
+        const int yy = row_ok ? __ldg(p.y + orig) : -1;
         float mx = -INFINITY, sm = 0.f, zsel = 0.f;
         bool have = false;
 #pragma unroll 1
@@ -274,64 +297,79 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         fence_before_sync();
         mbar_arrive(smem_u32(&ctl->acc_empty[acc]));
         if (row_ok) {
-          p.part[int64_t(n) * p.rows + row] = make_float2(mx, sm);
+          p.part[int64_t(n) * p.rows + row] = make_float2(mx, sm);  // compacted row, stride N
           if (have) p.zy[row] = zsel;
         }
       } else if constexpr (kEpi == kDLogits) {
+        // dZ goes out through two swizzled 128x64 staging boxes and TMA
+        // stores; one epilogue thread issues the stores and tracks them.
+        const bool issuer = (warp == 2 && lane == 0);
         const int lc0 = n * BN;  // column inside the chunk
         int yy = -1;
         float g = 0.f, l2 = 0.f;
         if (row_ok) {
-          yy = __ldg(p.y + row) - p.v0;
-          g = __ldg(p.G + row);
-          l2 = __ldg(p.lse + row) * kLog2e;
+          yy = __ldg(p.y + orig) - p.v0;
+          g = __ldg(p.G + orig);
+          l2 = __ldg(p.lse + orig) * kLog2e;
         }
-        __nv_bfloat16 *out = p.dz + (row_ok ? row : 0) * p.ldz;
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
-          uint32_t u[32];
-          tmem_ld32(taddr + c * 32, u);
-          tmem_wait_ld();
-          const int lc = lc0 + c * 32;
-          if (!row_ok || lc >= p.cols) continue;
-          uint32_t pk[16];
+        for (int box = 0; box < BN / 64; ++box) {
+          const uint32_t buf = out_base + uint32_t(box & 1) * STAGE_OUT_BYTES;
+          if (issuer) bulk_wait_group_read<1>();  // the store that last read `buf` is done
+          named_barrier(EPI_BARRIER, 128);
 #pragma unroll
-          for (int j = 0; j < 32; j += 2) {
-            float d0 = 0.f, d1 = 0.f;
-            if (g != 0.f) {
-              d0 = -g * ex2_approx(fmaf(__uint_as_float(u[j]), kLog2e, -l2));
-              d1 = -g * ex2_approx(fmaf(__uint_as_float(u[j + 1]), kLog2e, -l2));
-              if (lc + j == yy) d0 += g;
-              if (lc + j + 1 == yy) d1 += g;
+          for (int half = 0; half < 2; ++half) {
+            const int c = box * 2 + half;
+            uint32_t u[32];
+            tmem_ld32(taddr + c * 32, u);
+            tmem_wait_ld();
+            if (c == BN / 32 - 1) {
+              fence_before_sync();
+              mbar_arrive(smem_u32(&ctl->acc_empty[acc]));
             }
-            const __nv_bfloat162 b2 = __floats2bfloat162_rn(d0, d1);
-            pk[j / 2] = *reinterpret_cast<const uint32_t *>(&b2);
-          }
-          if (lc + 32 <= p.cols) {
-            uint4 *dst = reinterpret_cast<uint4 *>(out + lc);
+            const int lc = lc0 + c * 32;
+            uint32_t pk[16];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) dst[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
-          } else {
-#pragma unroll
-            for (int j = 0; j < 32; ++j) {
-              if (lc + j < p.cols) {
-                const uint32_t w = pk[j / 2];
-                const uint16_t hbits = (j & 1) ? uint16_t(w >> 16) : uint16_t(w & 0xffffu);
-                reinterpret_cast<uint16_t *>(out)[lc + j] = hbits;
+            for (int j = 0; j < 32; j += 2) {
+              float d0 = 0.f, d1 = 0.f;
+              if (g != 0.f) {
+                d0 = -g * ex2_approx(fmaf(__uint_as_float(u[j]), kLog2e, -l2));
+                d1 = -g * ex2_approx(fmaf(__uint_as_float(u[j + 1]), kLog2e, -l2));
+                if (lc + j == yy) d0 += g;
+                if (lc + j + 1 == yy) d1 += g;
               }
+              const __nv_bfloat162 b2 = __floats2bfloat162_rn(d0, d1);
+              pk[j / 2] = *reinterpret_cast<const uint32_t *>(&b2);
             }
+            // 128-byte swizzle: 16-byte chunk j of row r sits at chunk j ^ (r % 8)
+            const uint32_t row_addr = buf + uint32_t(r) * 128u;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const uint32_t chunk = uint32_t(half * 4 + q) ^ uint32_t(r & 7);
+              asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(row_addr + chunk * 16u),
+                           "r"(pk[4 * q]), "r"(pk[4 * q + 1]), "r"(pk[4 * q + 2]), "r"(pk[4 * q + 3])
+                           : "memory");
+            }
+          }
+          fence_proxy_async_smem();
+          named_barrier(EPI_BARRIER, 128);
+          if (issuer) {
+            tma_store_2d(&map_c, buf, lc0 + box * 64, m * BM);
+            bulk_commit_group();
           }
         }
-        fence_before_sync();
-        mbar_arrive(smem_u32(&ctl->acc_empty[acc]));
       } else {
         // kStoreF32 / kStoreBF16: plain tile store (optionally accumulating)
-        const int64_t orow = p.c_row_off + row;
+        const int64_t orow = p.c_row_off + orig;
 #pragma unroll 1
         for (int c = 0; c < BN / 32; ++c) {
           uint32_t u[32];
           tmem_ld32(taddr + c * 32, u);
           tmem_wait_ld();
+          if (kzero) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) u[j] = 0u;
+          }
           const int col = n * BN + c * 32;
           if (!row_ok || col >= p.cols) continue;
           const bool full = col + 32 <= p.cols;
@@ -382,26 +420,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   }
 
+  if constexpr (kEpi == kDLogits) {
+    if (warp == 2 && lane == 0) bulk_wait_group<0>();
+  }
   fence_before_sync();
   __syncthreads();
   if (warp == 1) {
     fence_after_sync();
     tmem_dealloc(tmem_base, TMEM_COLS);
-  }
-}
-
-// fp32 dH accumulator -> bf16 dH (multi-chunk backward only)
-__global__ void f32_to_bf16_kernel(const float *src, __nv_bfloat16 *dst, int64_t n) {
-  const int64_t i = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) * 4;
-  if (i + 4 <= n) {
-    const float4 v = *reinterpret_cast<const float4 *>(src + i);
-    const __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
-    uint2 w;
-    w.x = *reinterpret_cast<const uint32_t *>(&a);
-    w.y = *reinterpret_cast<const uint32_t *>(&b);
-    *reinterpret_cast<uint2 *>(dst + i) = w;
-  } else {
-    for (int64_t j = i; j < n; ++j) dst[j] = __float2bfloat16_rn(src[j]);
   }
 }
 
@@ -442,8 +468,8 @@ sao_status make_map(CUtensorMap *m, const void *ptr, uint64_t inner, uint64_t ou
 }
 
 template <int kEpi, bool kAMN, bool kBMN>
-sao_status launch_gemm(const char *name, const CUtensorMap &ma, const CUtensorMap &mb, const GemmParams &p,
-                       cudaStream_t s) {
+sao_status launch_gemm(const char *name, const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &mc,
+                       const GemmParams &p, cudaStream_t s) {
   auto kern = tc_gemm_kernel<kEpi, kAMN, kBMN>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
@@ -457,7 +483,7 @@ sao_status launch_gemm(const char *name, const CUtensorMap &ma, const CUtensorMa
   if (tiles == 0 || p.nK == 0) return SAO_OK;
   const int grid = tiles < di.sm_count ? tiles : di.sm_count;
   int slot = launch_begin(name, s);
-  kern<<<grid, NUM_THREADS, SMEM_BYTES, s>>>(ma, mb, p);
+  kern<<<grid, NUM_THREADS, SMEM_BYTES, s>>>(ma, mb, mc, p);
   return launch_end(slot, s);
 }
 
@@ -478,7 +504,7 @@ size_t tc_ws_bytes(int64_t N, int32_t h, int32_t V) {
   const int vc = vocab_chunk(N, V);
   size_t bwd = round256(size_t(N) * size_t(vc) * 2);
   if (vc < V) bwd += round256(size_t(N) * size_t(h) * sizeof(float));
-  return fwd > bwd ? fwd : bwd;
+  return compact_ws_bytes(N, h) + (fwd > bwd ? fwd : bwd);
 }
 
 sao_status tc_fwd(const void *H, const void *W, const int32_t *y, const uint8_t *row_mask, int64_t N, int32_t h,
@@ -486,11 +512,17 @@ sao_status tc_fwd(const void *H, const void *W, const int32_t *y, const uint8_t 
                   cudaStream_t s) {
   const int nvt = (V + BN - 1) / BN;
   Carver c(ws, ws_bytes);
+  // Rows with row_mask == 0 are skipped: the GEMM runs on the compacted rows.
+  CompactRows cr{};
+  if (row_mask) SAO_TRY(compact_rows(row_mask, nullptr, N, static_cast<const __nv_bfloat16 *>(H), h, &cr, c, s));
   float2 *part = c.take<float2>(size_t(nvt) * size_t(N));
   float *zy = c.take<float>(size_t(N));
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the log-prob forward");
   CUtensorMap ma, mb;
-  SAO_TRY(make_map(&ma, H, uint64_t(h), uint64_t(N), uint64_t(h), 64, BM));
+  if (row_mask)
+    SAO_TRY(make_map(&ma, cr.Hc, uint64_t(h), uint64_t(cr.cap), uint64_t(h), 64, BM));
+  else
+    SAO_TRY(make_map(&ma, H, uint64_t(h), uint64_t(N), uint64_t(h), 64, BM));
   SAO_TRY(make_map(&mb, W, uint64_t(h), uint64_t(V), uint64_t(h), 64, BN));
   GemmParams p{};
   p.nM = int((N + BM - 1) / BM);
@@ -504,8 +536,12 @@ sao_status tc_fwd(const void *H, const void *W, const int32_t *y, const uint8_t 
   p.part = part;
   p.zy = zy;
   p.err = err;
-  SAO_TRY((launch_gemm<kSoftmax, false, false>("tc_logits_lse_fwd", ma, mb, p, s)));
-  return lse_merge_launch(part, nvt, zy, y, row_mask, N, V, logp, lse, err, s);
+  if (row_mask) {
+    p.m_count = cr.count;
+    p.row_idx = cr.idx;
+  }
+  SAO_TRY((launch_gemm<kSoftmax, false, false>("tc_logits_lse_fwd", ma, mb, ma, p, s)));
+  return lse_merge_launch(part, nvt, zy, y, nullptr, row_mask ? cr.pos : nullptr, N, V, logp, lse, err, s);
 }
 
 sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *lse, const float *G, int64_t N,
@@ -514,14 +550,18 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
   const int Vc = vocab_chunk(N, V);
   const bool multi = Vc < V;
   Carver c(ws, ws_bytes);
+  // Rows whose incoming gradient is zero contribute nothing: compact the rest.
+  CompactRows cr{};
+  SAO_TRY(compact_rows(nullptr, G, N, static_cast<const __nv_bfloat16 *>(H), h, &cr, c, s));
   __nv_bfloat16 *dz = c.take<__nv_bfloat16>(size_t(N) * size_t(Vc));
   float *dh_acc = multi ? c.take<float>(size_t(N) * size_t(h)) : nullptr;
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the log-prob backward");
+  if (!multi) SAO_CUDA_TRY(cudaMemsetAsync(dH, 0, size_t(N) * size_t(h) * 2, s));
 
-  CUtensorMap mH_K, mW_K, mH_MN, mW_MN;
-  SAO_TRY(make_map(&mH_K, H, uint64_t(h), uint64_t(N), uint64_t(h), 64, BM));
+  CUtensorMap mHc_K, mW_K, mHc_MN, mW_MN;
+  SAO_TRY(make_map(&mHc_K, cr.Hc, uint64_t(h), uint64_t(cr.cap), uint64_t(h), 64, BM));
   SAO_TRY(make_map(&mW_K, W, uint64_t(h), uint64_t(V), uint64_t(h), 64, BN));
-  SAO_TRY(make_map(&mH_MN, H, uint64_t(h), uint64_t(N), uint64_t(h), 64, 64));
+  SAO_TRY(make_map(&mHc_MN, cr.Hc, uint64_t(h), uint64_t(cr.cap), uint64_t(h), 64, 64));
   SAO_TRY(make_map(&mW_MN, W, uint64_t(h), uint64_t(V), uint64_t(h), 64, 64));
   const int nMt = int((N + BM - 1) / BM);
 
@@ -531,7 +571,7 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
     CUtensorMap mZ_K, mZ_MN;
     SAO_TRY(make_map(&mZ_K, dz, uint64_t(vc), uint64_t(N), uint64_t(Vc), 64, BM));
     SAO_TRY(make_map(&mZ_MN, dz, uint64_t(vc), uint64_t(N), uint64_t(Vc), 64, 64));
-    {  // dZ for vocabulary [v0, v0 + vc)
+    {  // dZ for vocabulary [v0, v0 + vc), compacted rows
       GemmParams p{};
       p.nM = nMt;
       p.nN = (vc + BN - 1) / BN;
@@ -548,7 +588,9 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
       p.dz = dz;
       p.ldz = Vc;
       p.err = err;
-      SAO_TRY((launch_gemm<kDLogits, false, false>("tc_dlogits", mH_K, mW_K, p, s)));
+      p.m_count = cr.count;
+      p.row_idx = cr.idx;
+      SAO_TRY((launch_gemm<kDLogits, false, false>("tc_dlogits", mHc_K, mW_K, mZ_K, p, s)));
     }
     {  // dH (+)= dZ W[v0:v0+vc]
       GemmParams p{};
@@ -561,16 +603,18 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
       p.cols = h;
       p.ldc = h;
       p.err = err;
+      p.m_count = cr.count;
       if (multi) {
-        p.cf = dh_acc;
+        p.cf = dh_acc;  // compacted rows
         p.accumulate = first ? 0 : 1;
-        SAO_TRY((launch_gemm<kStoreF32, false, true>("tc_dH_gemm", mZ_K, mW_MN, p, s)));
+        SAO_TRY((launch_gemm<kStoreF32, false, true>("tc_dH_gemm", mZ_K, mW_MN, mZ_K, p, s)));
       } else {
         p.cb = static_cast<__nv_bfloat16 *>(dH);
-        SAO_TRY((launch_gemm<kStoreBF16, false, true>("tc_dH_gemm", mZ_K, mW_MN, p, s)));
+        p.row_idx = cr.idx;  // scatter to the original rows
+        SAO_TRY((launch_gemm<kStoreBF16, false, true>("tc_dH_gemm", mZ_K, mW_MN, mZ_K, p, s)));
       }
     }
-    {  // dW[v0:v0+vc] (+)= dZ^T H
+    {  // dW[v0:v0+vc] (+)= dZ^T H over the compacted tokens
       GemmParams p{};
       p.nM = (vc + BM - 1) / BM;
       p.nN = (h + BN - 1) / BN;
@@ -583,15 +627,11 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
       p.c_row_off = v0;
       p.accumulate = accumulate;
       p.err = err;
-      SAO_TRY((launch_gemm<kStoreF32, true, true>("tc_dW_gemm", mZ_MN, mH_MN, p, s)));
+      p.k_count = cr.count;
+      SAO_TRY((launch_gemm<kStoreF32, true, true>("tc_dW_gemm", mZ_MN, mHc_MN, mZ_MN, p, s)));
     }
-    if (multi && last) {
-      const int64_t n = N * int64_t(h);
-      const int64_t threads = (n + 3) / 4;
-      int slot = launch_begin("dH_to_bf16", s);
-      f32_to_bf16_kernel<<<unsigned((threads + 255) / 256), 256, 0, s>>>(dh_acc, static_cast<__nv_bfloat16 *>(dH), n);
-      SAO_TRY(launch_end(slot, s));
-    }
+    if (multi && last)
+      SAO_TRY(scatter_rows_to_bf16(dh_acc, h, cr.pos, N, static_cast<__nv_bfloat16 *>(dH), s));
   }
   return SAO_OK;
 }

@@ -9,7 +9,8 @@ namespace {
 
 __global__ void __launch_bounds__(256) lse_merge_kernel(const float2 *__restrict__ part, int nvt,
                                                         const float *__restrict__ zy, const int32_t *__restrict__ y,
-                                                        const uint8_t *__restrict__ row_mask, int64_t N, int V,
+                                                        const uint8_t *__restrict__ row_mask,
+                                                        const int *__restrict__ pos, int64_t N, int V,
                                                         float *logp, float *lse, unsigned int *err) {
   const int64_t row = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
   if (row >= N) return;
@@ -18,18 +19,29 @@ __global__ void __launch_bounds__(256) lse_merge_kernel(const float2 *__restrict
     lse[row] = 0.f;
     return;
   }
+  // partials of a compacted forward are stored at the row's compact index
+  int64_t src = row;
+  if (pos != nullptr) {
+    const int i = pos[row];
+    if (i < 0) {
+      logp[row] = 0.f;
+      lse[row] = 0.f;
+      return;
+    }
+    src = i;
+  }
   float m = -INFINITY;
-  for (int j = 0; j < nvt; ++j) m = fmaxf(m, __ldcs(&part[int64_t(j) * N + row].x));
+  for (int j = 0; j < nvt; ++j) m = fmaxf(m, __ldcs(&part[int64_t(j) * N + src].x));
   float s = 0.f;
   for (int j = 0; j < nvt; ++j) {
-    const float2 p = __ldcs(part + int64_t(j) * N + row);
+    const float2 p = __ldcs(part + int64_t(j) * N + src);
     s = fmaf(p.y, expf(p.x - m), s);
   }
   const float l = m + logf(s);
   lse[row] = l;
   const int yy = y[row];
   if (yy >= 0 && yy < V) {
-    logp[row] = zy[row] - l;
+    logp[row] = zy[src] - l;
   } else {
     logp[row] = __int_as_float(0x7fc00000);
     raise_device_error(err, SAO_DEVERR_TOKEN_ID);
@@ -39,11 +51,11 @@ __global__ void __launch_bounds__(256) lse_merge_kernel(const float2 *__restrict
 }  // namespace
 
 sao_status lse_merge_launch(const float2 *part, int nvt, const float *zy, const int32_t *y,
-                            const uint8_t *row_mask, int64_t N, int32_t V, float *logp, float *lse,
+                            const uint8_t *row_mask, const int *pos, int64_t N, int32_t V, float *logp, float *lse,
                             unsigned int *err, cudaStream_t s) {
   const int64_t grid = (N + 255) / 256;
   int slot = launch_begin("lse_merge", s);
-  lse_merge_kernel<<<unsigned(grid), 256, 0, s>>>(part, nvt, zy, y, row_mask, N, V, logp, lse, err);
+  lse_merge_kernel<<<unsigned(grid), 256, 0, s>>>(part, nvt, zy, y, row_mask, pos, N, V, logp, lse, err);
   return launch_end(slot, s);
 }
 

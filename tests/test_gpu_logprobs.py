@@ -128,3 +128,17 @@ def test_tiny_config_full_oracle():
     want_dH, want_dW = O.token_logprobs_bwd(wl.H.cpu(), wl.W.cpu(), wl.y, want_lse, G)
     assert rel_l2(dH.cpu().numpy(), want_dH) <= GRAD_TOL
     assert rel_l2(dW.cpu().numpy(), want_dW) <= GRAD_TOL
+
+
+@pytest.mark.parametrize("dt", ["bf16", "f32"])
+def test_logprobs_backward_all_zero_gradient(dt):
+    """No active row: dH = 0, dW = 0 (or unchanged when accumulating)."""
+    wl, H, W, y = _case(300, 64, 700, dt, seed=2)
+    logp, lse = _fwd(H, W, y)
+    G = torch.zeros(300, device="cuda")
+    dH, dW = _bwd(H, W, y, lse, G)
+    prev = torch.randn(700, 64, device="cuda")
+    _, dW2 = _bwd(H, W, y, lse, G, accumulate=prev)
+    torch.cuda.synchronize()
+    assert not dH.float().abs().max().item() and not dW.abs().max().item()
+    assert torch.equal(dW2, prev)

@@ -125,3 +125,27 @@ def test_many_tiles_per_cta_full_oracle():
     want_dH, want_dW = O.token_logprobs_bwd(H_cpu, W_cpu, wl.y, want_lse, G)
     assert rel_l2(dH.float().cpu().numpy(), want_dH) <= GRAD_TOL
     assert rel_l2(dW.cpu().numpy(), want_dW) <= GRAD_TOL
+
+
+def test_full_size_row_mask_forward():
+    """moe with row_mask = loss_mask: the forward runs on the compacted action
+    rows only; skipped rows return 0, active rows match the oracle."""
+    wl = S.make_workload("moe", device="cuda")
+    N, h, V = wl.N, wl.h, wl.V
+    y = torch.as_tensor(wl.y).cuda()
+    mask = torch.as_tensor(wl.loss_mask).cuda()
+    ws = sao.workspace(N, h, V, wl.H.dtype)
+    logp = torch.empty(N, device="cuda")
+    lse = torch.empty(N, device="cuda")
+    sao.sao_token_logprobs_fwd(wl.H, wl.W, y, logp, lse, ws, row_mask=mask)
+    full_lp = torch.empty(N, device="cuda")
+    full_lse = torch.empty(N, device="cuda")
+    sao.sao_token_logprobs_fwd(wl.H, wl.W, y, full_lp, full_lse, ws)
+    torch.cuda.synchronize()
+    m = wl.loss_mask.astype(bool)
+    got = logp.cpu().numpy()
+    assert np.all(got[~m] == 0) and np.all(lse.cpu().numpy()[~m] == 0)
+    assert np.array_equal(got[m], full_lp.cpu().numpy()[m])
+    rows = np.sort(np.random.default_rng(13).choice(np.flatnonzero(m), size=16, replace=False))
+    want, _ = O.token_logprobs(wl.H[torch.as_tensor(rows).cuda()].cpu(), wl.W.cpu(), wl.y[rows])
+    assert np.abs(got[rows] - want).max() <= LOGP_TOL
