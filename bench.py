@@ -50,7 +50,7 @@ def load_peaks():
 # clocks sampled with nvidia-smi during the timed region
 # ---------------------------------------------------------------------------
 class ClockSampler:
-    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
@@ -75,7 +75,10 @@ class ClockSampler:
         for line in self.proc.stdout:
             self.lines.append(line.strip())
 
-    def stop(self):
+    def stop(self, t_begin=None, t_end=None):
+        """Median clocks over the samples taken between t_begin and t_end
+        (host wall-clock seconds); all samples if none falls inside."""
+        import datetime
         if self.proc is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
         self.proc.terminate()
@@ -85,25 +88,32 @@ class ClockSampler:
             self.proc.kill()
         if self.thread:
             self.thread.join(timeout=2)
-        sm, mx, power, reasons = [], [], [], set()
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        samples = []
         for line in self.lines:
             parts = [p.strip() for p in line.split(",")]
-            if len(parts) < 8:
+            if len(parts) < 9:
                 continue
             try:
-                sm.append(float(parts[0]))
-                mx.append(float(parts[1]))
-                power.append(float(parts[2]))
+                ts = datetime.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                samples.append((ts, float(parts[1]), float(parts[2]), float(parts[3]), parts[5:9]))
             except ValueError:
                 continue
-            for name, val in zip(names, parts[4:8]):
+        inside = [x for x in samples if t_begin is not None and t_begin <= x[0] <= t_end]
+        used = inside or samples
+        sm = [x[1] for x in used]
+        mx = [x[2] for x in used]
+        power = [x[3] for x in used]
+        reasons = set()
+        for x in used:
+            for name, val in zip(names, x[4]):
                 if val.lower().startswith("active"):
                     reasons.add(name)
         if not sm:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
-                "power_w_max": max(power) if power else None, "reasons": sorted(reasons)}
+                "samples_in_timed_region": len(inside), "power_w_max": max(power) if power else None,
+                "reasons": sorted(reasons)}
 
 
 # ---------------------------------------------------------------------------
@@ -327,7 +337,7 @@ def bandwidth_study(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -376,13 +386,15 @@ def main():
     torch.cuda.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
+    t_begin = time.time()
     e0.record(stream)
     for _ in range(args.steps):
         step.run()
     e1.record(stream)
     torch.cuda.synchronize()
+    t_end = time.time()
     barrier()
-    clk = clocks.stop()
+    clk = clocks.stop(t_begin, t_end)
     ms = e0.elapsed_time(e1) / args.steps
     prof = sao.sao_profile_read()
     sao.sao_profile_enable(False)

@@ -163,10 +163,10 @@ SAO_API sao_status sao_advantages(const float *values, const float *rewards, con
  *
  * Scratch: a fixed 8 MiB array inside this library's device image, present on
  * every GPU that loads the library until the process exits. It bounds the
- * sizes: 256 + gae scratch(N, B) bytes must fit, about 88 bytes per 4096
- * tokens plus 36 bytes per trajectory (for example 2^27 tokens with up to
- * 131,072 trajectories); larger inputs return SAO_ERR_SHAPE with the bytes
- * needed. Nothing is allocated and nothing is freed.
+ * sizes: about 88 bytes per 512 tokens plus 36 bytes per trajectory must
+ * fit (for example 2^25 tokens with up to 65,536 trajectories); larger
+ * inputs return SAO_ERR_SHAPE with the bytes needed. Nothing is allocated
+ * and nothing is freed.
  * The first call on each device looks up the array's device address (with
  * that device current) and caches it; make that first call before any stream
  * capture. Every call on a device shares the one array, so calls that overlap

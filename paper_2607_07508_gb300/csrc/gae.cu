@@ -17,12 +17,15 @@
 // waiting for its action token. Each action token maps S affinely
 // (B' = a B + g Vn + P, Vn' = V, P' = 0); the last token of a trajectory
 // resets S to (0, 0, 0, R_b). Maps compose associatively, so:
-//   * each thread folds its 16 tokens into one map,
-//   * a warp-shuffle suffix scan and a per-CTA pass combine them,
-//   * CTAs (4096-token chunks) chain their maps right-to-left by decoupled
-//     look-back: each CTA takes a ticket, works on chunk nchunks-1-ticket, so
-//     it only ever waits on chunks whose CTAs started before it; every wait
-//     is bounded and a time-out raises SAO_DEVERR_SCAN_TIMEOUT,
+//   * each thread folds its 32 tokens into one map,
+//   * a warp-shuffle suffix scan combines the 32 maps of a warp's 1024-token
+//     chunk,
+//   * warps chain their chunks right-to-left by decoupled look-back: each
+//     warp takes a ticket and works on chunk nchunks-1-ticket, so it only
+//     ever waits on chunks whose warps started before it; no CTA-wide barrier
+//     exists, so a waiting warp never holds up the others; the look-back
+//     inspects 32 predecessors at once and composes their maps in log depth;
+//     every wait is bounded and a time-out raises SAO_DEVERR_SCAN_TIMEOUT,
 //   * each thread then replays its tokens from its incoming state.
 // Traffic: values 4 B + mask 1 B read, adv 4 B + ret 4 B written per token.
 #include <stdint.h>
@@ -34,8 +37,8 @@ namespace sao {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kItems = 16;
-constexpr int kChunk = kThreads * kItems;
+constexpr int kItems = 32;           // tokens per lane (at most 32: one bit each)
+constexpr int kChunk = 32 * kItems;  // tokens per warp chunk
 constexpr int kWarps = kThreads / 32;
 
 // ---------------------------------------------------------------------------
@@ -277,7 +280,7 @@ struct GaeArgs {
   unsigned int *err;
 };
 
-constexpr int kCuCap = 1024;
+constexpr int kCuCap = 128;  // cu_seqlens entries staged per warp
 
 // cu_seqlens entries [blo, blo + n) of one chunk, read from shared memory
 // when the slice fits there, else from global memory.
@@ -308,69 +311,128 @@ __device__ __forceinline__ int find_traj(const int32_t *cu, int B, int64_t t) {
   return lo;
 }
 
+// State at the right edge of chunk q, from the chunks to its right. The warp
+// inspects 32 successors (q+1 .. q+32) per round: each lane polls one status
+// word; the first chunk whose left-edge state is known (published inclusive
+// state, a map that ignores its right neighbour, or the end of the input) ends
+// the walk, and the maps of the chunks before it are composed by a log-depth
+// shuffle scan. A round waits (bounded) only for chunks before that point.
 template <bool kCrit>
-__global__ void __launch_bounds__(kThreads, 2) gae_scan_kernel(GaeArgs a) {
-  __shared__ int s_q, s_blo, s_ncu;
-  __shared__ GMap s_warp[kWarps];
-  __shared__ GState s_wstate[kWarps];
-  __shared__ int32_t s_cu[kCuCap];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (threadIdx.x == 0) {
-    const int q = a.nchunks - 1 - atomicAdd(a.ticket, 1);
-    const int blo = a.chunk_first[q];
-    const int bhi = q + 1 < a.nchunks ? a.chunk_first[q + 1] : a.B - 1;
-    s_q = q;
-    s_blo = blo;
-    s_ncu = bhi - blo + 2;  // cu[blo .. bhi + 1]
-  }
-  __syncthreads();
-  const int q = s_q;
-  const int64_t t0 = int64_t(q) * kChunk + int64_t(threadIdx.x) * kItems;
-  const int64_t N = a.N;
-  // This chunk's slice of cu_seqlens, in shared memory when it fits.
-  const CuView cu{a.cu, s_cu, s_blo, s_ncu <= kCuCap};
-  if (cu.in_smem)
-    for (int i = threadIdx.x; i < s_ncu; i += kThreads) s_cu[i] = __ldg(a.cu + s_blo + i);
-  __syncthreads();
-
-  // ---- load 16 tokens -------------------------------------------------------
-  float v[kItems];
-  uint32_t act = 0;
-  const bool full = t0 + kItems <= N;
-  if (full && aligned16_dev(a.values) && aligned16_dev(a.m)) {
-    const float4 *v4 = reinterpret_cast<const float4 *>(a.values + t0);
-#pragma unroll
-    for (int k = 0; k < kItems / 4; ++k) {
-      const float4 x = __ldcs(v4 + k);
-      v[4 * k] = x.x;
-      v[4 * k + 1] = x.y;
-      v[4 * k + 2] = x.z;
-      v[4 * k + 3] = x.w;
+__device__ GState look_back(const GaeArgs &a, int q, int lane) {
+  GState zero;
+  zero.Bp = zero.Bc = {0.f, 0.f};
+  zero.Vn = zero.P = 0.f;
+  GMap acc = identity_map();  // maps of the chunks already walked (lane 0)
+  const uint64_t t_start = globaltimer_ns();
+  for (int base = q + 1;; base += 32) {
+    const int j = base + lane;
+    int st = 0;
+    GMap mj = identity_map();
+    bool term = false;
+    uint32_t polls = 0;
+    for (;;) {
+      st = j < a.nchunks ? ld_acquire(a.status + j) : 2;
+      term = (st == 2);
+      if (st == 1) {
+        mj = load_map(&a.pub[j].agg);
+        term = (mj.fl & 1) != 0;
+      }
+      const unsigned bt = __ballot_sync(0xffffffffu, term);
+      const unsigned bn = __ballot_sync(0xffffffffu, st == 0);
+      const int first_term = bt ? __ffs(bt) - 1 : 32;
+      const int first_nr = bn ? __ffs(bn) - 1 : 32;
+      if (first_nr >= first_term) break;  // everything up to the first terminal chunk is known
+      if ((++polls & 31u) == 0u && globaltimer_ns() - t_start > kWaitLimitNs) {
+        if (lane == 0) raise_device_error(a.err, SAO_DEVERR_SCAN_TIMEOUT);
+        return zero;
+      }
+      __nanosleep(128);
     }
-    const uint4 mq = __ldcs(reinterpret_cast<const uint4 *>(a.m + t0));
-    const uint32_t w[4] = {mq.x, mq.y, mq.z, mq.w};
-#pragma unroll
-    for (int k = 0; k < kItems; ++k) act |= uint32_t(((w[k >> 2] >> (8 * (k & 3))) & 0xffu) != 0u) << k;
+    const unsigned bt = __ballot_sync(0xffffffffu, term);
+    const int stop = bt ? __ffs(bt) - 1 : 32;
+    // state at the left edge of the terminal chunk (if any in this round)
+    GState tstate = zero;
+    if (lane == stop && j < a.nchunks) tstate = (st == 2) ? load_state(&a.pub[j].incl) : apply<kCrit>(mj, zero, a.coef);
+    // compose maps of lanes [0, stop): suffix scan, lane 0 ends with m_0 o ... o m_{stop-1}
+    GMap m = lane < stop ? mj : identity_map();
+#pragma unroll 1
+    for (int d = 1; d < 32; d <<= 1) {
+      const GMap o = shfl_down_map(m, d);
+      if (lane + d < 32) m = compose<kCrit>(m, o, a.coef);
+    }
+    if (lane == 0) acc = compose<kCrit>(acc, m, a.coef);
+    if (stop < 32) {
+      tstate.Bp.hi = __shfl_sync(0xffffffffu, tstate.Bp.hi, stop);
+      tstate.Bp.lo = __shfl_sync(0xffffffffu, tstate.Bp.lo, stop);
+      tstate.Bc.hi = __shfl_sync(0xffffffffu, tstate.Bc.hi, stop);
+      tstate.Bc.lo = __shfl_sync(0xffffffffu, tstate.Bc.lo, stop);
+      tstate.Vn = __shfl_sync(0xffffffffu, tstate.Vn, stop);
+      tstate.P = __shfl_sync(0xffffffffu, tstate.P, stop);
+      GState r = apply<kCrit>(acc, tstate, a.coef);  // meaningful in lane 0
+      r.Bp.hi = __shfl_sync(0xffffffffu, r.Bp.hi, 0);
+      r.Bp.lo = __shfl_sync(0xffffffffu, r.Bp.lo, 0);
+      r.Bc.hi = __shfl_sync(0xffffffffu, r.Bc.hi, 0);
+      r.Bc.lo = __shfl_sync(0xffffffffu, r.Bc.lo, 0);
+      r.Vn = __shfl_sync(0xffffffffu, r.Vn, 0);
+      r.P = __shfl_sync(0xffffffffu, r.P, 0);
+      return r;
+    }
+  }
+}
+
+// Loads 4 consecutive tokens (value, action bit) starting at t; tokens at or
+// beyond N read as observation tokens with value 0.
+__device__ __forceinline__ void load4(const GaeArgs &a, int64_t t, bool vec, float (&v)[4], uint32_t &act4) {
+  if (vec) {
+    const float4 x = __ldg(reinterpret_cast<const float4 *>(a.values + t));
+    const uint32_t w = __ldg(reinterpret_cast<const unsigned int *>(a.m + t));
+    v[0] = x.x;
+    v[1] = x.y;
+    v[2] = x.z;
+    v[3] = x.w;
+    act4 = ((w & 0xffu) != 0u) | (((w >> 8) & 0xffu) != 0u) << 1 | (((w >> 16) & 0xffu) != 0u) << 2 |
+           (((w >> 24) & 0xffu) != 0u) << 3;
   } else {
+    act4 = 0;
 #pragma unroll
-    for (int k = 0; k < kItems; ++k) {
-      const int64_t t = t0 + k;
-      v[k] = t < N ? a.values[t] : 0.f;
-      act |= uint32_t(t < N && a.m[t] != 0) << k;
+    for (int i = 0; i < 4; ++i) {
+      const bool in = t + i < a.N;
+      v[i] = in ? a.values[t + i] : 0.f;
+      act4 |= uint32_t(in && a.m[t + i] != 0) << i;
     }
   }
+}
 
-  // ---- trajectory ends among the 16 tokens (forward walk) ----------------------
-  // The walk is repeated backwards in the two right-to-left passes below, so no
-  // per-token trajectory id is kept in registers.
+template <bool kCrit>
+__global__ void __launch_bounds__(kThreads, 3) gae_scan_kernel(GaeArgs a) {
+  __shared__ int32_t s_cu_all[kWarps][kCuCap];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int q = 0;
+  if (lane == 0) q = a.nchunks - 1 - atomicAdd(a.ticket, 1);
+  q = __shfl_sync(0xffffffffu, q, 0);
+  if (q < 0) return;  // the grid rounds the warp count up to whole CTAs
+  const int64_t t0 = int64_t(q) * kChunk + int64_t(lane) * kItems;
+  const int64_t N = a.N;
+
+  // This chunk's slice of cu_seqlens, in shared memory when it fits.
+  const int blo = __ldg(a.chunk_first + q);
+  const int bhi = q + 1 < a.nchunks ? __ldg(a.chunk_first + q + 1) : a.B - 1;
+  const int ncu = bhi - blo + 2;  // cu[blo .. bhi + 1]
+  int32_t *s_cu = s_cu_all[warp];
+  const CuView cu{a.cu, s_cu, blo, ncu <= kCuCap};
+  if (cu.in_smem)
+    for (int i = lane; i < ncu; i += 32) s_cu[i] = __ldg(a.cu + blo + i);
+  __syncwarp();
+  const bool vec = (t0 + kItems <= N) && aligned16_dev(a.values) && aligned16_dev(a.m);
+
+  // ---- trajectory ends among the 16 tokens (forward walk over cu_seqlens) -------
   uint32_t endbits = 0;
   int b_last;
   {
-    const int bhi = s_blo + s_ncu - 2;
-    int b = cu.find(s_blo, bhi, t0 < N ? t0 : N - 1);
+    int b = cu.find(blo, bhi, t0 < N ? t0 : N - 1);
     int64_t next_end = cu[b + 1];
     bool bad = false;
-#pragma unroll
+#pragma unroll 4
     for (int k = 0; k < kItems; ++k) {
       const int64_t t = t0 + k;
       if (t < N) {
@@ -378,15 +440,12 @@ __global__ void __launch_bounds__(kThreads, 2) gae_scan_kernel(GaeArgs a) {
           ++b;
           next_end = cu[b + 1];
         }
-        if (t >= next_end) bad = true;  // cu_seqlens[B] < N
+        bad |= (t >= next_end);  // cu_seqlens[B] < N
         endbits |= uint32_t(t == next_end - 1) << k;
       }
     }
     b_last = b;
-    if (bad) {
-      raise_device_error(a.err, SAO_DEVERR_CU_SEQLENS);
-      act = 0;
-    }
+    if (bad) raise_device_error(a.err, SAO_DEVERR_CU_SEQLENS);
   }
 
   // ---- fold the thread's tokens into one map (right to left) ------------------
@@ -395,163 +454,119 @@ __global__ void __launch_bounds__(kThreads, 2) gae_scan_kernel(GaeArgs a) {
     int b = b_last;
     int64_t b_start = cu[b];
     TCoef c = load_coef(a.coef, b);
+#pragma unroll 1
+    for (int g = kItems / 4 - 1; g >= 0; --g) {
+      float v[4];
+      uint32_t act4;
+      load4(a, t0 + 4 * g, vec, v, act4);
 #pragma unroll
-    for (int k = kItems - 1; k >= 0; --k) {
-      const int64_t t = t0 + k;
-      if (t >= N) continue;
-      if (t < b_start) {
-        while (b > s_blo && t < b_start) {
-          --b;
-          b_start = cu[b];
-        }
-        c = load_coef(a.coef, b);
-      }
-      const bool is_act = (act >> k) & 1u, is_end = (endbits >> k) & 1u;
-      if (is_end) {
-        const float R = __ldg(a.rewards + b);
-        M.b = b;
-        M.ap = M.ac = {0.f, 0.f};
-        if (is_act) {
-          M.fl = 3;
-          M.cp = M.cc = {R, 0.f};
-          M.v = v[k];
-          M.p0 = 0.f;
-        } else {
-          M.fl = 1;
-          M.cp = M.cc = {0.f, 0.f};
-          M.v = 0.f;
-          M.p0 = R;
-        }
-      } else if (is_act) {
-        if (M.fl == 0) {
-          M.fl = 2;
-          M.ap = M.ac = {1.f, 0.f};
-          M.cp = M.cc = {0.f, 0.f};
-        } else {
-          const bool mact = (M.fl & 2) != 0;
-          const float Yv = mact ? M.v : 0.f, Yp = mact ? 0.f : M.p0;
-          M.cp = df_add_f(df_add(df_mul(c.ap, M.cp), df_mul_f(c.gp, Yv)), Yp);
-          if (kCrit) M.cc = df_add_f(df_add(df_mul(c.ac, M.cc), df_mul_f(c.gc, Yv)), Yp);
-          if (!(M.fl & 1)) {
-            M.ap = df_mul(c.ap, M.ap);
-            if (kCrit) M.ac = df_mul(c.ac, M.ac);
+      for (int i = 3; i >= 0; --i) {
+        const int k = 4 * g + i;
+        const int64_t t = t0 + k;
+        if (t < b_start && t < N) {
+          while (b > blo && t < b_start) {
+            --b;
+            b_start = cu[b];
           }
-          M.fl |= 2;
+          c = load_coef(a.coef, b);
         }
-        M.b = b;
-        M.v = v[k];
-        M.p0 = 0.f;
-      } else if (M.fl != 0) {
-        M.b = b;
+        const bool is_act = (act4 >> i) & 1u, is_end = (endbits >> k) & 1u;
+        if (is_end) {
+          const float R = __ldg(a.rewards + b);
+          M.b = b;
+          M.ap = M.ac = {0.f, 0.f};
+          M.fl = is_act ? 3 : 1;
+          M.cp = M.cc = {is_act ? R : 0.f, 0.f};
+          M.v = is_act ? v[i] : 0.f;
+          M.p0 = is_act ? 0.f : R;
+        } else if (is_act) {
+          if (M.fl == 0) {
+            M.fl = 2;
+            M.ap = M.ac = {1.f, 0.f};
+            M.cp = M.cc = {0.f, 0.f};
+          } else {
+            const bool mact = (M.fl & 2) != 0;
+            const float Yv = mact ? M.v : 0.f, Yp = mact ? 0.f : M.p0;
+            M.cp = df_add(df_mul(c.ap, M.cp), df_mul_f(c.gp, Yv));
+            if (kCrit) M.cc = df_add(df_mul(c.ac, M.cc), df_mul_f(c.gc, Yv));
+            if (Yp != 0.f) {  // only right after a trajectory that ends on observations
+              M.cp = df_add_f(M.cp, Yp);
+              if (kCrit) M.cc = df_add_f(M.cc, Yp);
+            }
+            if (!(M.fl & 1)) {
+              M.ap = df_mul(c.ap, M.ap);
+              if (kCrit) M.ac = df_mul(c.ac, M.ac);
+            }
+            M.fl |= 2;
+          }
+          M.b = b;
+          M.v = v[i];
+          M.p0 = 0.f;
+        } else if (M.fl != 0) {
+          M.b = b;
+        }
       }
     }
   }
 
-  // ---- suffix scan within the warp, then across warps ---------------------------
+  // ---- suffix scan of the 32 maps of this warp ------------------------------------
   GMap S = M;
-#pragma unroll
+#pragma unroll 1
   for (int d = 1; d < 32; d <<= 1) {
     const GMap o = shfl_down_map(S, d);
     if (lane + d < 32) S = compose<kCrit>(S, o, a.coef);
   }
-  GMap E = shfl_down_map(S, 1);  // lanes to my right within the warp
+  GMap E = shfl_down_map(S, 1);  // lanes to my right within the chunk
   if (lane == 31) E = identity_map();
-  if (lane == 0) s_warp[warp] = S;
-  __syncthreads();
 
-  if (warp == 0) {
-    // Lanes 0..7 scan the warp maps: W = map of warp `lane` .. last (inclusive),
-    // T = map of warps lane+1 .. last (exclusive); lane 0 holds the chunk map.
-    GMap W = lane < kWarps ? s_warp[lane] : identity_map();
-#pragma unroll
-    for (int d = 1; d < kWarps; d <<= 1) {
-      const GMap o = shfl_down_map(W, d);
-      if (lane + d < kWarps) W = compose<kCrit>(W, o, a.coef);
+  // ---- publish this chunk and look back for the state at its right edge ------------
+  // Release stores of the status word order the published map/state before it;
+  // readers acquire the status before reading them.
+  GState zero;
+  zero.Bp = zero.Bc = {0.f, 0.f};
+  zero.Vn = zero.P = 0.f;
+  const bool last = (q == a.nchunks - 1);
+  const bool reset = (S.fl & 1) != 0;  // lane 0 holds the chunk's map
+  ChunkPub *me = a.pub + q;
+  if (lane == 0) {
+    // A chunk whose map ignores its right neighbour publishes its left-edge
+    // state at once; the others publish their map first.
+    if (last || reset) {
+      store_state(&me->incl, apply<kCrit>(S, zero, a.coef));
+      st_release(a.status + q, 2);
+    } else {
+      store_map(&me->agg, S);
+      st_release(a.status + q, 1);
     }
-    GMap T = shfl_down_map(W, 1);
-    if (lane >= kWarps - 1) T = identity_map();
-    GState zero;
-    zero.Bp = zero.Bc = {0.f, 0.f};
-    zero.Vn = zero.P = 0.f;
-    GState right = zero;
-    if (lane == 0) {
-      const GMap &agg = W;
-      ChunkPub *me = a.pub + q;
-      const bool last = (q == a.nchunks - 1);
-      const bool reset = (agg.fl & 1) != 0;
-      // A chunk whose map ignores its right neighbour publishes its left-edge
-      // state at once; the others publish their map first.
-      if (last || reset) {
-        store_state(&me->incl, apply<kCrit>(agg, zero, a.coef));
-        __threadfence();
-        st_release(a.status + q, 2);
-      } else {
-        store_map(&me->agg, agg);
-        __threadfence();
-        st_release(a.status + q, 1);
-      }
-      if (!last) {
-        // look back to the right for the state at this chunk's right edge
-        GMap acc = identity_map();
-        for (int j = q + 1;; ++j) {
-          if (j >= a.nchunks) {
-            right = apply<kCrit>(acc, zero, a.coef);
-            break;
-          }
-          const int st = wait_nonzero(a.status + j);
-          if (st == 0) {
-            raise_device_error(a.err, SAO_DEVERR_SCAN_TIMEOUT);
-            right = apply<kCrit>(acc, zero, a.coef);
-            break;
-          }
-          if (st == 2) {
-            right = apply<kCrit>(acc, load_state(&a.pub[j].incl), a.coef);
-            break;
-          }
-          acc = compose<kCrit>(acc, load_map(&a.pub[j].agg), a.coef);
-          if (acc.fl & 1) {
-            right = apply<kCrit>(acc, zero, a.coef);
-            break;
-          }
-        }
-        if (!reset) {
-          store_state(&me->incl, apply<kCrit>(agg, right, a.coef));
-          __threadfence();
-          st_release(a.status + q, 2);
-        }
-      }
-    }
-    // broadcast the right-edge state and give every warp its incoming state
-    right.Bp.hi = __shfl_sync(0xffffffffu, right.Bp.hi, 0);
-    right.Bp.lo = __shfl_sync(0xffffffffu, right.Bp.lo, 0);
-    right.Bc.hi = __shfl_sync(0xffffffffu, right.Bc.hi, 0);
-    right.Bc.lo = __shfl_sync(0xffffffffu, right.Bc.lo, 0);
-    right.Vn = __shfl_sync(0xffffffffu, right.Vn, 0);
-    right.P = __shfl_sync(0xffffffffu, right.P, 0);
-    if (lane < kWarps) s_wstate[lane] = apply<kCrit>(T, right, a.coef);
   }
-  __syncthreads();
+  GState right = zero;
+  if (!__shfl_sync(0xffffffffu, int(last), 0)) right = look_back<kCrit>(a, q, lane);
+  if (lane == 0 && !reset && !last) {
+    store_state(&me->incl, apply<kCrit>(S, right, a.coef));
+    st_release(a.status + q, 2);
+  }
 
-  // ---- replay the tokens from the incoming state, store 4 at a time --------------
-  GState st = apply<kCrit>(E, s_wstate[warp], a.coef);
-  const bool vec_out = full && aligned16_dev(a.adv) && aligned16_dev(a.ret);
+  // ---- replay the tokens from the incoming state, 4 at a time ---------------------
+  GState st = apply<kCrit>(E, right, a.coef);
+  const bool vec_out = vec && aligned16_dev(a.adv) && aligned16_dev(a.ret);
   {
     int b = b_last;
     int64_t b_start = cu[b];
     TCoef c = load_coef(a.coef, b);
     float R = __ldg(a.rewards + b);
-#pragma unroll
+#pragma unroll 1
     for (int g = kItems / 4 - 1; g >= 0; --g) {
-      float ov[4], orr[4];
+      float v[4], ov[4], orr[4];
+      uint32_t act4;
+      load4(a, t0 + 4 * g, vec, v, act4);
 #pragma unroll
       for (int i = 3; i >= 0; --i) {
         const int k = 4 * g + i;
         const int64_t t = t0 + k;
         ov[i] = 0.f;
         orr[i] = 0.f;
-        if (t >= N) continue;
-        if (t < b_start) {
-          while (b > s_blo && t < b_start) {
+        if (t < b_start && t < N) {
+          while (b > blo && t < b_start) {
             --b;
             b_start = cu[b];
           }
@@ -563,28 +578,29 @@ __global__ void __launch_bounds__(kThreads, 2) gae_scan_kernel(GaeArgs a) {
           st.Vn = 0.f;
           st.P = R;
         }
-        if ((act >> k) & 1u) {
-          st.Bp = df_add_f(df_add(df_mul(c.ap, st.Bp), df_mul_f(c.gp, st.Vn)), st.P);
-          if (kCrit) {
-            st.Bc = df_add_f(df_add(df_mul(c.ac, st.Bc), df_mul_f(c.gc, st.Vn)), st.P);
-            orr[i] = df_round(st.Bc);
-          } else {
-            orr[i] = R;  // gamma = lambda_critic = 1: the return is the reward
+        if ((act4 >> i) & 1u) {
+          st.Bp = df_add(df_mul(c.ap, st.Bp), df_mul_f(c.gp, st.Vn));
+          if (kCrit) st.Bc = df_add(df_mul(c.ac, st.Bc), df_mul_f(c.gc, st.Vn));
+          if (st.P != 0.f) {
+            st.Bp = df_add_f(st.Bp, st.P);
+            if (kCrit) st.Bc = df_add_f(st.Bc, st.P);
           }
-          ov[i] = df_round(df_add_f(st.Bp, -v[k]));
-          st.Vn = v[k];
+          orr[i] = kCrit ? df_round(st.Bc) : R;  // gamma = lambda_critic = 1: the return is R
+          ov[i] = df_round(df_add_f(st.Bp, -v[i]));
+          st.Vn = v[i];
           st.P = 0.f;
         }
       }
+      const int64_t tg = t0 + 4 * g;
       if (vec_out) {
-        __stcs(reinterpret_cast<float4 *>(a.adv + t0) + g, make_float4(ov[0], ov[1], ov[2], ov[3]));
-        __stcs(reinterpret_cast<float4 *>(a.ret + t0) + g, make_float4(orr[0], orr[1], orr[2], orr[3]));
+        __stcs(reinterpret_cast<float4 *>(a.adv + tg), make_float4(ov[0], ov[1], ov[2], ov[3]));
+        __stcs(reinterpret_cast<float4 *>(a.ret + tg), make_float4(orr[0], orr[1], orr[2], orr[3]));
       } else {
 #pragma unroll
         for (int i = 0; i < 4; ++i)
-          if (t0 + 4 * g + i < N) {
-            a.adv[t0 + 4 * g + i] = ov[i];
-            a.ret[t0 + 4 * g + i] = orr[i];
+          if (tg + i < N) {
+            a.adv[tg + i] = ov[i];
+            a.ret[tg + i] = orr[i];
           }
       }
     }
@@ -592,44 +608,63 @@ __global__ void __launch_bounds__(kThreads, 2) gae_scan_kernel(GaeArgs a) {
 }
 
 // Number of action tokens per trajectory (only for the length-adaptive lambda).
-// One CTA per 4096-token chunk, like the scan, with the chunk's cu_seqlens
-// slice in shared memory.
+// One warp per 512-token chunk, like the scan.
 __global__ void __launch_bounds__(kThreads) gae_count_kernel(const uint8_t *m, const int32_t *cu_g, int B,
                                                              int64_t N, int nchunks, const int *chunk_first,
                                                              int *nact) {
-  __shared__ int32_t s_cu[kCuCap];
-  const int q = blockIdx.x;
+  __shared__ int32_t s_cu_all[kWarps][kCuCap];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int q = blockIdx.x * kWarps + warp;
+  if (q >= nchunks) return;
   const int blo = chunk_first[q];
   const int bhi = q + 1 < nchunks ? chunk_first[q + 1] : B - 1;
   const int ncu = bhi - blo + 2;
+  int32_t *s_cu = s_cu_all[warp];
   const CuView cu{cu_g, s_cu, blo, ncu <= kCuCap};
   if (cu.in_smem)
-    for (int i = threadIdx.x; i < ncu; i += kThreads) s_cu[i] = __ldg(cu_g + blo + i);
-  __syncthreads();
-  const int64_t t0 = int64_t(q) * kChunk + int64_t(threadIdx.x) * kItems;
+    for (int i = lane; i < ncu; i += 32) s_cu[i] = __ldg(cu_g + blo + i);
+  __syncwarp();
+  const int64_t t0 = int64_t(q) * kChunk + int64_t(lane) * kItems;
   int b = cu.find(blo, bhi, t0 < N ? t0 : N - 1);
   int64_t next_end = cu[b + 1];
   int cnt = 0;
-#pragma unroll
-  for (int k = 0; k < kItems; ++k) {
-    const int64_t t = t0 + k;
-    if (t >= N) break;
-    if (t >= next_end) {
-      const int nb0 = b;
-      while (b < bhi && t >= next_end) {
-        ++b;
-        next_end = cu[b + 1];
-      }
-      if (b != nb0 && cnt) {
-        atomicAdd(nact + nb0, cnt);
-        cnt = 0;
+  const bool vec = (t0 + kItems <= N) && ((reinterpret_cast<uintptr_t>(m) & 15u) == 0);
+#pragma unroll 1
+  for (int g = 0; g < kItems / 16; ++g) {
+    uint32_t w[4] = {0u, 0u, 0u, 0u};
+    if (vec) {
+      const uint4 x = __ldg(reinterpret_cast<const uint4 *>(m + t0) + g);
+      w[0] = x.x;
+      w[1] = x.y;
+      w[2] = x.z;
+      w[3] = x.w;
+    } else {
+      for (int k = 0; k < 16; ++k) {
+        const int64_t t = t0 + 16 * g + k;
+        if (t < N && m[t] != 0) w[k >> 2] |= 1u << (8 * (k & 3));
       }
     }
-    cnt += (m[t] != 0);
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      const int64_t t = t0 + 16 * g + k;
+      if (t >= N) break;
+      if (t >= next_end) {
+        const int nb0 = b;
+        while (b < bhi && t >= next_end) {
+          ++b;
+          next_end = cu[b + 1];
+        }
+        if (b != nb0 && cnt) {
+          atomicAdd(nact + nb0, cnt);
+          cnt = 0;
+        }
+      }
+      cnt += ((w[k >> 2] >> (8 * (k & 3))) & 0xffu) != 0u;
+    }
   }
   const unsigned peers = __match_any_sync(0xffffffffu, b);
   const int tot = __reduce_add_sync(peers, cnt);
-  if ((threadIdx.x & 31) == __ffs(peers) - 1 && tot) atomicAdd(nact + b, tot);
+  if (lane == __ffs(peers) - 1 && tot) atomicAdd(nact + b, tot);
 }
 
 // First trajectory of every chunk (one binary search per chunk, all in parallel).
@@ -695,7 +730,8 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   }
   if (alpha > 0.f) {
     int slot = launch_begin("gae_count", s);
-    gae_count_kernel<<<unsigned(nchunks), kThreads, 0, s>>>(m, cu, B, N, int(nchunks), chunk_first, nact);
+    gae_count_kernel<<<unsigned((nchunks + kWarps - 1) / kWarps), kThreads, 0, s>>>(m, cu, B, N, int(nchunks),
+                                                                                    chunk_first, nact);
     SAO_TRY(launch_end(slot, s));
   }
   {
@@ -720,11 +756,12 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   a.ret = ret;
   a.err = err;
   const bool crit_trivial = (gamma == 1.0f && lam_c == 1.0f);
+  const unsigned grid = unsigned((nchunks + kWarps - 1) / kWarps);
   int slot = launch_begin("gae_scan", s);
   if (crit_trivial)
-    gae_scan_kernel<false><<<int(nchunks), kThreads, 0, s>>>(a);
+    gae_scan_kernel<false><<<grid, kThreads, 0, s>>>(a);
   else
-    gae_scan_kernel<true><<<int(nchunks), kThreads, 0, s>>>(a);
+    gae_scan_kernel<true><<<grid, kThreads, 0, s>>>(a);
   return launch_end(slot, s);
 }
 

@@ -51,3 +51,24 @@ def test_no_alloc_rejects_sizes_beyond_its_scratch():
     st = lib.sao_advantages_noalloc(P, P, P, P, 1 << 22, (1 << 31) - 1, 1.0, 1.0, 1.0, 0.0, P, P, None)
     assert st == 2
     assert "scratch" in lib.sao_last_error_string().decode()
+
+
+def test_no_alloc_documented_example_fits():
+    """The size the header quotes (2^25 tokens in 65,536 trajectories) fits
+    the fixed scratch and matches the workspace entry point."""
+    N, B = 1 << 25, 1 << 16
+    rng = np.random.default_rng(21)
+    cu = np.arange(0, N + 1, N // B, dtype=np.int32)
+    values = rng.standard_normal(N, dtype=np.float32)
+    mask = (rng.random(N) < 0.75).astype(np.uint8)
+    rewards = (rng.random(B) < 0.4).astype(np.float32)
+    args = [torch.as_tensor(a).cuda() for a in (values, rewards, mask, cu)] + [1.0, 0.95, 1.0, 0.0]
+
+    class _Shape:
+        pass
+    wl = _Shape()
+    wl.N = N
+    a0, r0 = _with_workspace(wl, args)
+    a1, r1 = _no_alloc(wl, args)
+    torch.cuda.synchronize()
+    assert torch.equal(a0, a1) and torch.equal(r0, r1)
