@@ -152,6 +152,30 @@ SAO_API sao_status sao_advantages(const float *values, const float *rewards, con
                           float lambda_policy, float lambda_critic, float len_adaptive_alpha,
                           float *adv, float *ret, void *ws, size_t ws_bytes, sao_stream_t stream);
 
+/* Step value definitions of sao_step_advantages (App. A.1). */
+#define SAO_STEP_AVERAGE 0 /* V(S) = mean of the step's token values; every step token is a value-loss token */
+#define SAO_STEP_LAST 1    /* V(S) = value of the step's last token; only that token is a value-loss token */
+
+/*
+ * Step-level GAE (App. A.1, "RL with Agentic Step as Action"). A step is one
+ * conversation turn: a maximal run of action tokens (loss_mask == 1) inside a
+ * trajectory. With V(S_i) per `mode`, the terminal reward on the last step and
+ * the step value after the last step 0: delta_i = r_i + gamma V(S_{i+1}) -
+ * V(S_i), A_i = delta_i + gamma lambda A_{i+1} where lambda = lambda_policy,
+ * or 1 - 1/(alpha * number of steps) clamped to [0,1] when
+ * len_adaptive_alpha = alpha > 0 (the length-adaptive rule counted in steps).
+ * Every token of step i receives adv = A_i and ret = GAE(lambda_critic)_i +
+ * V(S_i); other tokens get 0. value_mask (nullable, [N] uint8) marks the
+ * tokens the value loss keeps: all step tokens (SAO_STEP_AVERAGE) or the last
+ * token of each step (SAO_STEP_LAST). Per-step arithmetic is fp64.
+ * Arguments otherwise as sao_advantages; workspace from sao_workspace_bytes.
+ */
+SAO_API sao_status sao_step_advantages(const float *values, const float *rewards, const uint8_t *loss_mask,
+                                       const int32_t *cu_seqlens, int32_t B, int64_t N, float gamma,
+                                       float lambda_policy, float lambda_critic, float len_adaptive_alpha, int mode,
+                                       float *adv, float *ret, uint8_t *value_mask, void *ws, size_t ws_bytes,
+                                       sao_stream_t stream);
+
 /*
  * sao_advantages without a workspace argument, for callers that cannot
  * allocate device memory: a host library that is handed only data pointers

@@ -22,6 +22,12 @@ Optimization for Agentic Reinforcement Learning" (arxiv 2607.07508):
                           lambda of §4.1
 * ``value_loss``          the value error (V - R)^2 of the Preliminaries (PPO),
                           with the explained-variance sums of §4.4
+* ``step_advantages``     the step-level GAE variants of App. A.1 ("step
+                          average" and "last-token prediction")
+* ``clip_loss``           the clipped surrogate of the Preliminaries' unified
+                          objective with asymmetric ("clip-higher") bounds, the
+                          loss of the paper's GRPO / GRPO (w/ DIS) arms (§4.2)
+* ``group_advantages``    GRPO's group-normalised advantage (Preliminaries)
 
 Readings taken where the paper is silent or ambiguous (each one is listed with
 its reason in the design notes):
@@ -47,6 +53,24 @@ R6  Length-adaptive lambda: l is the trajectory's number of action tokens,
     lambda_b = 1 - 1/(alpha*l), clamped to [0, 1]; alpha <= 0 disables it.
 R7  Returns are GAE with lambda_critic plus V; the value loss is the plain mean
     over action tokens of (V - ret)^2, no 1/2 factor and no clipping.
+R13 Step-level GAE (App. A.1): a step is one conversation turn, i.e. a maximal
+    run of action tokens inside a trajectory; the terminal reward is the
+    reward of the last step; the step value after the last step is 0; every
+    token of a step receives the step's advantage and the step's value target
+    GAE(lambda_critic) + V(S); with "step average" every token of the step is
+    a value-loss token, with "last-token" only the step's last token is.
+R14 Clipped surrogate (Preliminaries): loss = -sum_t w_t min(r_t A_t,
+    clip(r_t, 1-eps_low, 1+eps_high) A_t) with w_t = 1/(number of action
+    tokens) ("token" normalisation) or 1/(|y_b| * number of trajectories with
+    an action token) ("sequence": the per-sequence 1/|y| mean, then the batch
+    mean). The ratio is taken against whatever log-probs the caller passes
+    (pi_old for PPO/GRPO, pi_rollout for GRPO w/ DIS). A token is clipped when
+    the min picks the clipped term strictly (A > 0 and r > 1+eps_high, or A < 0
+    and r < 1-eps_low), decided in fp32; clipped tokens have zero gradient;
+    non-finite tokens are masked as in R4.
+R15 GRPO advantage: A_b = (R_b - mean_g) / sqrt(var_g + eps_stab) over the
+    trajectories of b's group g (population variance), broadcast to b's action
+    tokens; other tokens get 0.
 """
 from __future__ import annotations
 
@@ -278,3 +302,161 @@ def explained_variance(ev_sums, n: int) -> float:
     var_e = s2 / n - (s1 / n) ** 2
     var_r = r2 / n - (r1 / n) ** 2
     return 1.0 - var_e / var_r if var_r > 0 else float("nan")
+
+
+# ---------------------------------------------------------------------------
+# step-level GAE variants (App. A.1)
+# ---------------------------------------------------------------------------
+
+STEP_AVERAGE = 0
+STEP_LAST = 1
+
+
+def step_spans(loss_mask, start: int, end: int):
+    """Steps of the trajectory occupying tokens [start, end): maximal runs of
+    action tokens, as (first, last + 1) pairs in order (reading R13)."""
+    m = np.asarray(loss_mask).astype(bool)
+    spans = []
+    t = start
+    while t < end:
+        if m[t]:
+            u = t
+            while u < end and m[u]:
+                u += 1
+            spans.append((t, u))
+            t = u
+        else:
+            t += 1
+    return spans
+
+
+def step_advantages(values, rewards, loss_mask, cu_seqlens, gamma: float, lam: float, lam_critic: float,
+                    alpha: float = 0.0, mode: int = STEP_AVERAGE):
+    """Step-wise GAE of App. A.1.
+
+    V(S_i) = mean of the step's token values (STEP_AVERAGE) or the value of its
+    last token (STEP_LAST); delta_i = r_i + gamma V(S_{i+1}) - V(S_i) with the
+    terminal reward on the last step; A_i = sum_l (gamma lambda)^l delta_{i+l}
+    with lambda = 1 - 1/(alpha * number of steps) when alpha > 0 (the
+    length-adaptive rule counted in steps). Returns (adv, ret, value_mask)
+    over all tokens: adv and ret broadcast to the step's tokens, value_mask =
+    the tokens the value loss keeps (R13).
+    """
+    v_all = _f64(values)
+    R = _f64(rewards)
+    cu = np.asarray(cu_seqlens, np.int64)
+    N = len(v_all)
+    adv = np.zeros(N, F64)
+    ret = np.zeros(N, F64)
+    vmask = np.zeros(N, np.uint8)
+    for b in range(len(cu) - 1):
+        spans = step_spans(loss_mask, cu[b], cu[b + 1])
+        n = len(spans)
+        if n == 0:
+            continue
+        if mode == STEP_AVERAGE:
+            vs = np.array([v_all[a:e].mean() for a, e in spans])
+        else:
+            vs = np.array([v_all[e - 1] for a, e in spans])
+        r = np.zeros(n, F64)
+        r[-1] = R[b]
+        lam_b = trajectory_lambda(lam, alpha, n)
+        A = _gae_backward(vs, r, gamma, lam_b)
+        T = _gae_backward(vs, r, gamma, lam_critic) + vs
+        for i, (a, e) in enumerate(spans):
+            adv[a:e] = A[i]
+            ret[a:e] = T[i]
+            if mode == STEP_AVERAGE:
+                vmask[a:e] = 1
+            else:
+                vmask[e - 1] = 1
+    return adv, ret, vmask
+
+
+# ---------------------------------------------------------------------------
+# clipped surrogate of the PPO / GRPO arms (Preliminaries; §4.2 baselines)
+# ---------------------------------------------------------------------------
+
+NORM_TOKEN = 0
+NORM_SEQUENCE = 1
+CLIP_NONE = 0
+CLIP_LOW = 1
+CLIP_HIGH = 2
+
+
+def clip_flags(logp, old_logp, adv, loss_mask, eps_low: float, eps_high: float) -> np.ndarray:
+    """0: the unclipped term r*A is the min; 1: clipped at 1-eps_low (A < 0);
+    2: clipped at 1+eps_high (A > 0); 3: non-finite; 4: not an action token.
+    Decided in fp32 (R14)."""
+    lp32 = np.asarray(logp, np.float32)
+    old32 = np.asarray(old_logp, np.float32)
+    adv32 = np.asarray(adv, np.float32)
+    m = np.asarray(loss_mask).astype(bool)
+    with np.errstate(all="ignore"):
+        d32 = (lp32 - old32).astype(np.float32)
+        r32 = np.exp(d32).astype(np.float32)
+        lo = np.float32(1.0) - np.float32(eps_low)
+        hi = np.float32(1.0) + np.float32(eps_high)
+        flags = np.zeros(m.shape, np.uint8)
+        flags[(adv32 > 0) & (r32 > hi)] = CLIP_HIGH
+        flags[(adv32 < 0) & (r32 < lo)] = CLIP_LOW
+        finite = np.isfinite(d32) & np.isfinite(adv32)
+    flags[~finite] = FLAG_NONFINITE
+    flags[~m] = FLAG_MASKED
+    return flags
+
+
+def clip_loss(logp, old_logp, adv, loss_mask, cu_seqlens, eps_low: float, eps_high: float,
+              norm: int = NORM_TOKEN) -> Dict[str, object]:
+    """Clipped surrogate with clip-higher bounds (R14).
+
+    loss = -sum_t w_t min(r_t A_t, clip(r_t, 1-eps_low, 1+eps_high) A_t);
+    coef_t = d loss / d logp_t = -w_t r_t A_t on unclipped tokens, else 0.
+    counts = [n_action, n_clip_low, n_clip_high, n_nonfinite].
+    """
+    flags = clip_flags(logp, old_logp, adv, loss_mask, eps_low, eps_high)
+    m = np.asarray(loss_mask).astype(bool)
+    cu = np.asarray(cu_seqlens, np.int64)
+    N = len(m)
+    w = np.zeros(N, F64)
+    if norm == NORM_TOKEN:
+        n = int(m.sum())
+        if n > 0:
+            w[m] = 1.0 / n
+    else:
+        lens = [int(m[cu[b]:cu[b + 1]].sum()) for b in range(len(cu) - 1)]
+        nseq = sum(1 for L in lens if L > 0)
+        for b, L in enumerate(lens):
+            if L > 0:
+                sl = slice(cu[b], cu[b + 1])
+                w[sl] = np.where(m[sl], 1.0 / (L * nseq), 0.0)
+    with np.errstate(all="ignore"):
+        r = np.exp(_f64(logp) - _f64(old_logp))
+        A = _f64(adv)
+        lo = float(np.float32(1.0) - np.float32(eps_low))
+        hi = float(np.float32(1.0) + np.float32(eps_high))
+        term = np.where(flags == CLIP_NONE, r * A,
+                        np.where(flags == CLIP_LOW, lo * A, np.where(flags == CLIP_HIGH, hi * A, 0.0)))
+        term = np.where(flags <= CLIP_HIGH, term, 0.0)
+        coef = np.where(flags == CLIP_NONE, -w * r * A, 0.0)
+    loss = -float((w * term).sum())
+    counts = np.array([int(m.sum()), int((flags == CLIP_LOW).sum()), int((flags == CLIP_HIGH).sum()),
+                       int((flags == FLAG_NONFINITE).sum())], np.int64)
+    return {"loss": loss, "coef": coef, "flags": flags, "counts": counts}
+
+
+def group_advantages(rewards, group_ids, loss_mask, cu_seqlens, eps_stab: float) -> np.ndarray:
+    """GRPO advantage (R15): (R_b - mean_g) / sqrt(var_g + eps_stab)."""
+    R = _f64(rewards)
+    g = np.asarray(group_ids, np.int64)
+    m = np.asarray(loss_mask).astype(bool)
+    cu = np.asarray(cu_seqlens, np.int64)
+    adv = np.zeros(len(m), F64)
+    for b in range(len(R)):
+        members = R[g == g[b]]
+        mu = members.mean()
+        var = ((members - mu) ** 2).mean()
+        a = (R[b] - mu) / np.sqrt(var + eps_stab)
+        sl = slice(cu[b], cu[b + 1])
+        adv[sl] = np.where(m[sl], a, 0.0)
+    return adv

@@ -17,9 +17,12 @@ size_t dz_budget() { return g_dz_budget.load(); }
 
 // O(N) kernels size their grids from N alone (deterministic on any device).
 size_t on_ws_bytes(int64_t N) {
-  const size_t e = elementwise_ws_bytes(N, 0);
+  size_t w = elementwise_ws_bytes(N, 0);
   const size_t g = gae_ws_bytes(N, N + 1);
-  return e > g ? e : g;
+  const size_t st = step_gae_ws_bytes(N, N + 1);
+  if (g > w) w = g;
+  if (st > w) w = st;
+  return w;
 }
 
 size_t logprobs_ws_bytes(int64_t N, int32_t h, int32_t V, sao_dtype dt) {
@@ -153,6 +156,29 @@ sao_status sao_advantages(const float *values, const float *rewards, const uint8
   SAO_TRY(begin_call(ws, s));
   SAO_TRY(gae_launch(values, rewards, loss_mask, cu_seqlens, B, N, gamma, lambda_policy, lambda_critic,
                      len_adaptive_alpha, adv, ret, w.err, w.body, w.body_bytes, s));
+  return finish_call(ws, s);
+}
+
+sao_status sao_step_advantages(const float *values, const float *rewards, const uint8_t *loss_mask,
+                               const int32_t *cu_seqlens, int32_t B, int64_t N, float gamma, float lambda_policy,
+                               float lambda_critic, float len_adaptive_alpha, int mode, float *adv, float *ret,
+                               uint8_t *value_mask, void *ws, size_t ws_bytes, sao_stream_t stream) {
+  if (N < 0 || N >= (int64_t(1) << 31)) return fail(SAO_ERR_SHAPE, "N = %lld out of range", (long long)N);
+  if (B < 0) return fail(SAO_ERR_SHAPE, "B = %d < 0", B);
+  if (N > 0 && B == 0) return fail(SAO_ERR_SHAPE, "N > 0 tokens need at least one trajectory");
+  if (mode != SAO_STEP_AVERAGE && mode != SAO_STEP_LAST) return fail(SAO_ERR_INVALID_ARG, "unknown step mode %d", mode);
+  if (!(gamma >= 0.f && gamma <= 1.f) || !(lambda_policy >= 0.f && lambda_policy <= 1.f) ||
+      !(lambda_critic >= 0.f && lambda_critic <= 1.f) || !isfinite(len_adaptive_alpha))
+    return fail(SAO_ERR_INVALID_ARG, "gamma and lambdas must lie in [0, 1] and alpha be finite");
+  if (N == 0) return SAO_OK;
+  if (!values || !rewards || !loss_mask || !cu_seqlens || !adv || !ret)
+    return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
+  Ws w;
+  SAO_TRY(take_ws(ws, ws_bytes, step_gae_ws_bytes(N, B), &w));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  SAO_TRY(begin_call(ws, s));
+  SAO_TRY(step_gae_launch(values, rewards, loss_mask, cu_seqlens, B, N, gamma, lambda_policy, lambda_critic,
+                          len_adaptive_alpha, mode, adv, ret, value_mask, w.body, w.body_bytes, s));
   return finish_call(ws, s);
 }
 

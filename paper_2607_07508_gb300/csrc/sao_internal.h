@@ -27,6 +27,12 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
                       int32_t B, int64_t N, float gamma, float lam, float lam_c, float alpha, float *adv,
                       float *ret, unsigned int *err, void *ws_body, size_t body_bytes, cudaStream_t s);
 
+// step_gae.cu -----------------------------------------------------------------
+size_t step_gae_ws_bytes(int64_t N, int64_t B);
+sao_status step_gae_launch(const float *values, const float *rewards, const uint8_t *m, const int32_t *cu, int32_t B,
+                           int64_t N, float gamma, float lam, float lam_c, float alpha, int mode, float *adv,
+                           float *ret, uint8_t *vmask, void *ws_body, size_t body_bytes, cudaStream_t s);
+
 // logprobs (tensor-core and fp32 paths) ----------------------------------------
 size_t logprobs_ws_bytes(int64_t N, int32_t h, int32_t V, sao_dtype dt);
 sao_status logprobs_fwd_launch(const void *H, const void *W, sao_dtype dt, const int32_t *y,

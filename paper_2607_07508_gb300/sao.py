@@ -18,14 +18,15 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libsao.so")
 
 SAO_F32, SAO_BF16 = 0, 1
+SAO_STEP_AVERAGE, SAO_STEP_LAST = 0, 1
 STATUS = {0: "SAO_OK", 1: "SAO_ERR_INVALID_ARG", 2: "SAO_ERR_SHAPE", 3: "SAO_ERR_WORKSPACE",
           4: "SAO_ERR_UNSUPPORTED", 5: "SAO_ERR_CUDA", 6: "SAO_ERR_DEVICE_CHECK"}
 FLAG_IN, FLAG_LOW, FLAG_HIGH, FLAG_NONFINITE, FLAG_NOT_ACTION = 0, 1, 2, 3, 4
 
 EXPORTS = ("sao_version", "sao_last_error_string", "sao_set_checked", "sao_get_checked",
            "sao_set_dz_budget_bytes", "sao_workspace_bytes", "sao_token_logprobs_fwd",
-           "sao_token_logprobs_bwd", "sao_advantages", "sao_advantages_noalloc", "sao_policy_loss_fwd",
-           "sao_policy_loss_bwd",
+           "sao_token_logprobs_bwd", "sao_advantages", "sao_advantages_noalloc", "sao_step_advantages",
+           "sao_policy_loss_fwd", "sao_policy_loss_bwd",
            "sao_value_loss", "sao_profile_enable", "sao_profile_reset", "sao_profile_read")
 
 
@@ -61,6 +62,7 @@ def load(path: Optional[str] = None):
                                                   ctypes.c_int, P, SZ, P]),
         "sao_advantages": (ctypes.c_int, [P, P, P, P, I32, I64, F, F, F, F, P, P, P, SZ, P]),
         "sao_advantages_noalloc": (ctypes.c_int, [P, P, P, P, I32, I64, F, F, F, F, P, P, P]),
+        "sao_step_advantages": (ctypes.c_int, [P, P, P, P, I32, I64, F, F, F, F, ctypes.c_int, P, P, P, P, SZ, P]),
         "sao_policy_loss_fwd": (ctypes.c_int, [P, P, P, P, I64, F, F, I64, P, P, P, P, P, SZ, P]),
         "sao_policy_loss_bwd": (ctypes.c_int, [P, P, P, P, I64, F, F, I64, P, P, P, SZ, P]),
         "sao_value_loss": (ctypes.c_int, [P, P, P, I64, P, P, P, P, SZ, P]),
@@ -191,6 +193,23 @@ def sao_advantages(values, rewards, loss_mask, cu_seqlens, gamma, lambda_policy,
                                  float(gamma), float(lambda_policy), float(lambda_critic),
                                  float(len_adaptive_alpha), _ptr(adv), _ptr(ret), _ptr(ws), ws.numel(),
                                  _stream(stream)))
+
+
+def sao_step_advantages(values, rewards, loss_mask, cu_seqlens, gamma, lambda_policy, lambda_critic,
+                        len_adaptive_alpha, mode, adv, ret, ws, value_mask=None, stream=None):
+    N = values.numel()
+    B = cu_seqlens.numel() - 1
+    _expect(values, torch.float32, N, "values")
+    _expect(rewards, torch.float32, B, "rewards")
+    _expect(loss_mask, torch.uint8, N, "loss_mask")
+    _expect(cu_seqlens, torch.int32, B + 1, "cu_seqlens")
+    _expect(adv, torch.float32, N, "adv")
+    _expect(ret, torch.float32, N, "ret")
+    _expect(value_mask, torch.uint8, N, "value_mask")
+    _check(load().sao_step_advantages(_ptr(values), _ptr(rewards), _ptr(loss_mask), _ptr(cu_seqlens), B, N,
+                                      float(gamma), float(lambda_policy), float(lambda_critic),
+                                      float(len_adaptive_alpha), int(mode), _ptr(adv), _ptr(ret), _ptr(value_mask),
+                                      _ptr(ws), ws.numel(), _stream(stream)))
 
 
 def sao_advantages_noalloc(values, rewards, loss_mask, cu_seqlens, gamma, lambda_policy, lambda_critic,

@@ -456,3 +456,136 @@ def test_explained_variance_matches_numpy_var():
     mb = m.astype(bool)
     want = 1.0 - np.var(R[mb] - v[mb]) / np.var(R[mb])
     assert abs(O.explained_variance(ev, int(mb.sum())) - want) < 1e-12
+
+
+# ---------------------------------------------------------------------------
+# step-level GAE (App. A.1)
+# ---------------------------------------------------------------------------
+
+def test_step_gae_single_token_steps_equal_token_gae():
+    """When every step is one action token (observations between them), both
+    step values are the token value and step GAE is token GAE."""
+    r = _rng(60)
+    L = 41
+    m = np.zeros(L, np.uint8)
+    m[::2] = 1
+    v = r.normal(0.4, 0.2, size=L)
+    for mode in (O.STEP_AVERAGE, O.STEP_LAST):
+        a_s, r_s, vm = O.step_advantages(v, np.array([1.0]), m, np.array([0, L]), 0.97, 0.9, 1.0, 1.5, mode)
+        a_t, r_t = O.advantages(v, np.array([1.0]), m, np.array([0, L]), 0.97, 0.9, 1.0, 1.5)
+        assert np.allclose(a_s, a_t, atol=1e-14) and np.allclose(r_s, r_t, atol=1e-14)
+        assert np.array_equal(vm, m)
+
+
+def test_step_gae_telescopes_and_broadcasts():
+    """gamma = lambda = 1: every token of step i gets R - V(S_i); mean vs last."""
+    m = np.array([0, 1, 1, 1, 0, 0, 1, 1, 0, 1], np.uint8)
+    v = np.array([9.0, 0.1, 0.2, 0.6, 9.0, 9.0, 0.3, 0.5, 9.0, 0.7])
+    R = 1.0
+    a_avg, r_avg, vm_avg = O.step_advantages(v, np.array([R]), m, np.array([0, 10]), 1.0, 1.0, 1.0, 0.0,
+                                             O.STEP_AVERAGE)
+    assert np.allclose(a_avg[[1, 2, 3]], R - 0.3) and np.allclose(a_avg[[6, 7]], R - 0.4)
+    assert np.allclose(a_avg[9], R - 0.7) and np.all(a_avg[m == 0] == 0)
+    assert np.allclose(r_avg[m == 1], R) and np.array_equal(vm_avg, m)
+    a_last, _, vm_last = O.step_advantages(v, np.array([R]), m, np.array([0, 10]), 1.0, 1.0, 1.0, 0.0,
+                                           O.STEP_LAST)
+    assert np.allclose(a_last[[1, 2, 3]], R - 0.6) and np.allclose(a_last[[6, 7]], R - 0.5)
+    assert list(np.flatnonzero(vm_last)) == [3, 7, 9]
+
+
+def test_step_gae_explicit_sum_and_step_count_lambda():
+    """Step advantages follow the explicit GAE sum over steps, with the
+    length-adaptive lambda counted in steps (App. A.1)."""
+    r = _rng(61)
+    m = np.array([1, 1, 0, 1, 1, 1, 0, 0, 1, 0, 1, 1], np.uint8)
+    v = r.normal(0.4, 0.2, size=len(m))
+    a, _, _ = O.step_advantages(v, np.array([1.0]), m, np.array([0, len(m)]), 0.9, 0.5, 1.0, 1.5,
+                                O.STEP_AVERAGE)
+    vs = np.array([v[0:2].mean(), v[3:6].mean(), v[8], v[10:12].mean()])
+    lam = 1.0 - 1.0 / (1.5 * 4)
+    want = _explicit_sum_gae(vs, 1.0, 0.9, lam)
+    assert np.allclose(a[[0, 3, 8, 10]], want, atol=1e-14)
+
+
+# ---------------------------------------------------------------------------
+# clipped surrogate (PPO / GRPO arms) and GRPO advantages
+# ---------------------------------------------------------------------------
+
+def test_clip_loss_no_bounds_equals_dis_without_bounds():
+    logp, old, adv, m = _loss_inputs(70)
+    cu = np.array([0, len(m)])
+    a = O.clip_loss(logp, old, adv, m, cu, 1e30, 1e30, O.NORM_TOKEN)
+    b = O.policy_loss(logp, old, adv, m, 1e30, 1e30)
+    assert abs(a["loss"] - b["loss"]) < 1e-12 and np.allclose(a["coef"], b["coef"], atol=1e-15)
+
+
+def test_clip_loss_hand_example():
+    """A > 0 above 1+eps_high and A < 0 below 1-eps_low are clipped (value at the
+    bound, zero gradient); A > 0 below 1-eps_low and A < 0 above 1+eps_high are
+    not (the min keeps r*A)."""
+    logp = np.log(np.array([1.5, 0.5, 0.5, 1.5, 1.0])).astype(np.float32)
+    old = np.zeros(5, np.float32)
+    adv = np.array([2.0, -1.0, 1.0, -0.5, 0.25], np.float32)
+    m = np.ones(5, np.uint8)
+    out = O.clip_loss(logp, old, adv, m, np.array([0, 5]), 0.2, 0.28, O.NORM_TOKEN)
+    assert list(out["flags"]) == [2, 1, 0, 0, 0]
+    r = np.exp(logp.astype(np.float64))
+    lo, hi = float(np.float32(0.8)), float(np.float32(1.0) + np.float32(0.28))
+    want = -(hi * 2.0 + lo * -1.0 + r[2] * 1.0 + r[3] * -0.5 + r[4] * 0.25) / 5
+    assert abs(out["loss"] - want) < 1e-12
+    assert out["coef"][0] == 0 and out["coef"][1] == 0
+    assert abs(out["coef"][3] - (-(r[3] * -0.5) / 5)) < 1e-15
+
+
+def test_clip_loss_sequence_normalisation():
+    """Sequence mode: each trajectory's tokens average first, so a 1-token
+    trajectory weighs as much as a 3-token one; old = new gives minus the mean
+    over trajectories of the per-trajectory mean advantage."""
+    adv = np.array([1.0, 2.0, 3.0, 10.0], np.float32)
+    lp = np.full(4, -1.0, np.float32)
+    m = np.ones(4, np.uint8)
+    cu = np.array([0, 3, 4])
+    out = O.clip_loss(lp, lp, adv, m, cu, 0.2, 0.28, O.NORM_SEQUENCE)
+    assert abs(out["loss"] - (-(2.0 + 10.0) / 2)) < 1e-12
+    tok = O.clip_loss(lp, lp, adv, m, cu, 0.2, 0.28, O.NORM_TOKEN)
+    assert abs(tok["loss"] - (-16.0 / 4)) < 1e-12
+
+
+def test_clip_loss_finite_differences():
+    logp, old, adv, m = _loss_inputs(71, N=20)
+    cu = np.array([0, 7, 7, 20])
+    for norm in (O.NORM_TOKEN, O.NORM_SEQUENCE):
+        out = O.clip_loss(logp, old, adv, m, cu, 0.2, 0.28, norm)
+        lp = logp.astype(np.float64)
+        for t in range(20):
+            r = math.exp(lp[t] - float(old[t]))
+            if abs(r - 0.8) < 1e-4 or abs(r - 1.28) < 1e-4:
+                continue
+            a, b = lp.copy(), lp.copy()
+            a[t] += 1e-7
+            b[t] -= 1e-7
+            num = (O.clip_loss(a, old, adv, m, cu, 0.2, 0.28, norm)["loss"] -
+                   O.clip_loss(b, old, adv, m, cu, 0.2, 0.28, norm)["loss"]) / 2e-7
+            assert abs(num - out["coef"][t]) < 1e-7
+
+
+def test_group_advantages_are_standardised():
+    r = _rng(72)
+    B = 24
+    gid = np.repeat(np.arange(3), 8)
+    R = (r.random(B) < 0.5).astype(np.float32)
+    R[16:] = 1.0                                       # a constant group
+    lens = r.integers(1, 9, size=B)
+    cu = np.concatenate([[0], np.cumsum(lens)])
+    m = np.ones(cu[-1], np.uint8)
+    adv = O.group_advantages(R, gid, m, cu, 1e-6)
+    per_traj = adv[cu[:-1]]
+    for g in range(2):
+        a = per_traj[gid == g]
+        var = np.var(R[gid == g].astype(np.float64))
+        assert abs(a.mean()) < 1e-12
+        assert abs(np.mean(a ** 2) - var / (var + 1e-6)) < 1e-9
+    assert np.all(per_traj[gid == 2] == 0)
+    single = O.group_advantages(np.array([1.0], np.float32), np.array([0]), np.ones(3, np.uint8),
+                                np.array([0, 3]), 1e-6)
+    assert np.all(single == 0)
