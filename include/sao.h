@@ -176,6 +176,65 @@ SAO_API sao_status sao_step_advantages(const float *values, const float *rewards
                                        float *adv, float *ret, uint8_t *value_mask, void *ws, size_t ws_bytes,
                                        sao_stream_t stream);
 
+/* Normalisation of sao_clip_loss_fwd/bwd (Preliminaries, unified objective). */
+#define SAO_NORM_TOKEN 0    /* mean over all action tokens of the batch */
+#define SAO_NORM_SEQUENCE 1 /* 1/|y| mean inside each trajectory, then the mean over trajectories */
+
+/*
+ * Clipped surrogate of the Preliminaries' unified objective with asymmetric
+ * ("clip-higher") bounds: the loss of the paper's PPO/GRPO comparison arms
+ * (§4.2; "GRPO w/ DIS" passes rollout log-probs as old_logp). With
+ * r_t = exp(logp_t - old_logp_t):
+ *   loss = -sum_t w_t min(r_t adv_t, clip(r_t, 1 - eps_low, 1 + eps_high) adv_t)
+ * over action tokens, w_t = 1/(action tokens) for SAO_NORM_TOKEN, or
+ * 1/(|y_b| * trajectories with an action token) for SAO_NORM_SEQUENCE. A token
+ * is clipped when the min takes the clipped term strictly (adv > 0 and
+ * r > 1 + eps_high: flag 2; adv < 0 and r < 1 - eps_low: flag 1), decided in
+ * fp32; clipped tokens have coef = 0, others coef = d loss / d logp =
+ * -w_t r_t adv_t. Non-finite tokens: flag 3, masked. counts = {n_action,
+ * n_clip_low, n_clip_high, n_nonfinite}. coef and flags may be NULL.
+ * cu_seqlens [B+1] as for sao_advantages (used by both normalisations).
+ */
+SAO_API sao_status sao_clip_loss_fwd(const float *logp, const float *old_logp, const float *adv,
+                                     const uint8_t *loss_mask, const int32_t *cu_seqlens, int32_t B, int64_t N,
+                                     float eps_low, float eps_high, int norm, float *loss, float *coef,
+                                     uint8_t *flags, int64_t *counts, void *ws, size_t ws_bytes, sao_stream_t stream);
+
+/* grad_logp[t] = grad_loss[0] * coef[t] of sao_clip_loss_fwd, recomputed. */
+SAO_API sao_status sao_clip_loss_bwd(const float *logp, const float *old_logp, const float *adv,
+                                     const uint8_t *loss_mask, const int32_t *cu_seqlens, int32_t B, int64_t N,
+                                     float eps_low, float eps_high, int norm, const float *grad_loss,
+                                     float *grad_logp, void *ws, size_t ws_bytes, sao_stream_t stream);
+
+/*
+ * GRPO's group-normalised advantage (Preliminaries): for trajectory b in
+ * group g = group_ids[b], A_b = (R_b - mean_g R) / sqrt(var_g R + eps_stab)
+ * (population variance over the group's trajectories, fp64), broadcast to b's
+ * action tokens; every other token gets 0. Cost O(B^2 / SMs) for the group
+ * statistics (deterministic), then O(N).
+ */
+SAO_API sao_status sao_group_advantages(const float *rewards, const int32_t *group_ids, int32_t B,
+                                        const uint8_t *loss_mask, const int32_t *cu_seqlens, int64_t N,
+                                        float eps_stab, float *adv, void *ws, size_t ws_bytes, sao_stream_t stream);
+
+/*
+ * Running-mean reward baseline, the single-rollout alternative to a value
+ * model in the ablations (§4.3: window of the 8 most recent rewards of each
+ * prompt; §4.5: one window of the 128 most recent rewards, i.e. one prompt
+ * id for all). Trajectories are taken in batch order: the baseline of b is
+ * the mean of the at most `window` most recent rewards recorded for prompt
+ * prompt_ids[b] before b (0 if none), A_b = R_b - baseline is written to b's
+ * action tokens (0 elsewhere), then R_b enters that prompt's window.
+ *   history [num_prompts, window] fp32 and seen [num_prompts] int64: the
+ *   windows (ring buffers indexed by seen % window) and the number of rewards
+ *   recorded per prompt; caller-owned device state, updated in place (zero
+ *   both before the first batch). prompt_ids in [0, num_prompts).
+ */
+SAO_API sao_status sao_running_mean_advantages(const float *rewards, const int32_t *prompt_ids, int32_t B,
+                                               int32_t num_prompts, float *history, int64_t *seen, int32_t window,
+                                               const uint8_t *loss_mask, const int32_t *cu_seqlens, int64_t N,
+                                               float *adv, void *ws, size_t ws_bytes, sao_stream_t stream);
+
 /*
  * sao_advantages without a workspace argument, for callers that cannot
  * allocate device memory: a host library that is handed only data pointers

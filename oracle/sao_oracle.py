@@ -28,6 +28,9 @@ Optimization for Agentic Reinforcement Learning" (arxiv 2607.07508):
                           objective with asymmetric ("clip-higher") bounds, the
                           loss of the paper's GRPO / GRPO (w/ DIS) arms (§4.2)
 * ``group_advantages``    GRPO's group-normalised advantage (Preliminaries)
+* ``running_mean_advantages``  the running-mean reward baseline of the
+                          single-rollout ablation (§4.3) and the online writing
+                          comparison (§4.5)
 
 Readings taken where the paper is silent or ambiguous (each one is listed with
 its reason in the design notes):
@@ -71,6 +74,11 @@ R14 Clipped surrogate (Preliminaries): loss = -sum_t w_t min(r_t A_t,
 R15 GRPO advantage: A_b = (R_b - mean_g) / sqrt(var_g + eps_stab) over the
     trajectories of b's group g (population variance), broadcast to b's action
     tokens; other tokens get 0.
+R16 Running-mean baseline: trajectories are taken in batch order; the baseline
+    of trajectory b is the mean of the (at most `window`) most recent rewards
+    recorded for its prompt before b, 0 when there are none; A_b = R_b -
+    baseline is broadcast to b's action tokens; then R_b enters the prompt's
+    window. One shared prompt id gives the single global window of §4.5.
 """
 from __future__ import annotations
 
@@ -460,3 +468,30 @@ def group_advantages(rewards, group_ids, loss_mask, cu_seqlens, eps_stab: float)
         sl = slice(cu[b], cu[b + 1])
         adv[sl] = np.where(m[sl], a, 0.0)
     return adv
+
+
+# ---------------------------------------------------------------------------
+# running-mean reward baseline (§4.3 ablation, §4.5 comparison)
+# ---------------------------------------------------------------------------
+
+def running_mean_advantages(rewards, prompt_ids, loss_mask, cu_seqlens, history, seen, window: int):
+    """A_b = R_b - mean(recent rewards of b's prompt) (R16). `history`
+    [P, window] and `seen` [P] are the per-prompt windows (ring buffers) and
+    reward counts; copies are updated and returned with the advantages."""
+    R = _f64(rewards)
+    pid = np.asarray(prompt_ids, np.int64)
+    m = np.asarray(loss_mask).astype(bool)
+    cu = np.asarray(cu_seqlens, np.int64)
+    hist = np.array(history, dtype=np.float64, copy=True)
+    cnt = np.array(seen, dtype=np.int64, copy=True)
+    adv = np.zeros(len(m), F64)
+    for b in range(len(R)):
+        p = pid[b]
+        n = int(min(cnt[p], window))
+        base = hist[p, :n].mean() if n > 0 else 0.0
+        a = R[b] - base
+        sl = slice(cu[b], cu[b + 1])
+        adv[sl] = np.where(m[sl], a, 0.0)
+        hist[p, cnt[p] % window] = R[b]
+        cnt[p] += 1
+    return adv, hist, cnt

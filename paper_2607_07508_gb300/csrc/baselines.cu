@@ -1,0 +1,404 @@
+// The paper's comparison arms (§4.2): the clipped surrogate of the
+// Preliminaries' unified objective with asymmetric ("clip-higher") bounds and
+// token or per-sequence normalisation, and GRPO's group-normalised advantage.
+//
+// The surrogate walks the packed trajectories in 1024-token warp chunks (like
+// the advantage scan) so every token knows its trajectory's action count for
+// the per-sequence weight; per-warp partial sums are added in a fixed order by
+// a one-CTA finaliser, so results are deterministic.
+#include <math.h>
+#include <stdint.h>
+
+#include "sao_common.cuh"
+#include "sao_internal.h"
+#include "segments.cuh"
+
+namespace sao {
+namespace {
+
+using seg::CuView;
+using seg::kCuCap;
+using seg::kItems;
+using seg::kSegChunk;
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+
+struct Norms {
+  long long n_action;  // action tokens
+  long long n_seq;     // trajectories with at least one action token
+};
+
+// Sums the per-trajectory action counts (one CTA, fixed order).
+__global__ void __launch_bounds__(256) norms_kernel(const int *nact, int B, Norms *out) {
+  long long n = 0, s = 0;
+  for (int b = threadIdx.x; b < B; b += 256) {
+    n += nact[b];
+    s += nact[b] > 0;
+  }
+  __shared__ long long sh[2][8];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    n += __shfl_xor_sync(0xffffffffu, n, o);
+    s += __shfl_xor_sync(0xffffffffu, s, o);
+  }
+  if ((threadIdx.x & 31) == 0) {
+    sh[0][threadIdx.x >> 5] = n;
+    sh[1][threadIdx.x >> 5] = s;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    Norms r{0, 0};
+    for (int w = 0; w < 8; ++w) {
+      r.n_action += sh[0][w];
+      r.n_seq += sh[1][w];
+    }
+    *out = r;
+  }
+}
+
+struct ClipArgs {
+  const float *logp, *old, *adv;
+  const uint8_t *m;
+  const int32_t *cu;
+  int B;
+  int64_t N;
+  int nchunks;
+  const int *chunk_first;
+  const int *nact;
+  const Norms *norms;
+  float lo, hi;
+  int seq;             // per-sequence normalisation
+  float *coef;         // may be null
+  uint8_t *flags;      // may be null
+  const float *grad_scale;
+  double *part_loss;   // [warps]
+  int *part_cnt;       // [3][warps]
+};
+
+// One token of the clipped surrogate: returns the weighted value term and
+// writes the coefficient d loss / d logp (before the sign) and the flag.
+__device__ __forceinline__ float clip_token(float lp, float old, float a, bool act, float lo, float hi, float w,
+                                            float &coef, uint8_t &flag, int &nl, int &nh, int &nf) {
+  coef = 0.f;
+  if (!act) {
+    flag = SAO_FLAG_NOT_ACTION;
+    return 0.f;
+  }
+  const float d = lp - old;
+  if (!isfinite(d) || !isfinite(a)) {
+    flag = SAO_FLAG_NONFINITE;
+    nf++;
+    return 0.f;
+  }
+  const float r = expf(d);
+  if (a > 0.f && r > hi) {
+    flag = 2;
+    nh++;
+    return w * hi * a;
+  }
+  if (a < 0.f && r < lo) {
+    flag = 1;
+    nl++;
+    return w * lo * a;
+  }
+  flag = 0;
+  const float t = w * r * a;
+  coef = -t;
+  return t;
+}
+
+template <bool kBwd>
+__global__ void __launch_bounds__(kThreads) clip_loss_kernel(ClipArgs a) {
+  __shared__ int32_t s_cu_all[kWarps][kCuCap];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int q = blockIdx.x * kWarps + warp;
+  const int gw = q;  // partial slot
+  if (q >= a.nchunks) return;
+  int blo, bhi;
+  const CuView cu = seg::stage_chunk(a.cu, a.B, a.nchunks, a.chunk_first, q, lane, s_cu_all[warp], blo, bhi);
+  const Norms nm = *a.norms;
+  const float w_tok = nm.n_action > 0 ? float(1.0 / double(nm.n_action)) : 0.f;
+  const double inv_seq = nm.n_seq > 0 ? 1.0 / double(nm.n_seq) : 0.0;
+  const float gscale = kBwd ? __ldg(a.grad_scale) : 1.f;
+  const int64_t t0 = int64_t(q) * kSegChunk + int64_t(lane) * kItems;
+  const int64_t N = a.N;
+  int b = cu.find(blo, bhi, t0 < N ? t0 : N - 1);
+  int64_t next_end = cu[b + 1];
+  auto weight = [&](int bb) {
+    if (!a.seq) return w_tok;
+    const int L = __ldg(a.nact + bb);
+    return L > 0 ? float(inv_seq / double(L)) : 0.f;
+  };
+  float w = weight(b);
+  float acc_hi = 0.f, acc_lo = 0.f;  // compensated sum of the value terms
+  int nl = 0, nh = 0, nf = 0;
+  const bool vec = (t0 + kItems <= N) && aligned16_dev(a.logp) && aligned16_dev(a.old) && aligned16_dev(a.adv) &&
+                   ((reinterpret_cast<uintptr_t>(a.m) & 3u) == 0) && (a.coef == nullptr || aligned16_dev(a.coef)) &&
+                   (a.flags == nullptr || (reinterpret_cast<uintptr_t>(a.flags) & 3u) == 0);
+#pragma unroll 1
+  for (int g = 0; g < kItems / 4; ++g) {
+    const int64_t tg = t0 + 4 * g;
+    float lp[4], od[4], ad[4];
+    bool act[4];
+    if (vec) {
+      const float4 x = __ldg(reinterpret_cast<const float4 *>(a.logp + tg));
+      const float4 y = __ldg(reinterpret_cast<const float4 *>(a.old + tg));
+      const float4 z = __ldg(reinterpret_cast<const float4 *>(a.adv + tg));
+      const uint32_t mw = __ldg(reinterpret_cast<const unsigned int *>(a.m + tg));
+      lp[0] = x.x; lp[1] = x.y; lp[2] = x.z; lp[3] = x.w;
+      od[0] = y.x; od[1] = y.y; od[2] = y.z; od[3] = y.w;
+      ad[0] = z.x; ad[1] = z.y; ad[2] = z.z; ad[3] = z.w;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) act[i] = ((mw >> (8 * i)) & 0xffu) != 0u;
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const bool in = tg + i < N;
+        lp[i] = in ? a.logp[tg + i] : 0.f;
+        od[i] = in ? a.old[tg + i] : 0.f;
+        ad[i] = in ? a.adv[tg + i] : 0.f;
+        act[i] = in && a.m[tg + i] != 0;
+      }
+    }
+    float cf[4];
+    uint8_t fl[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int64_t t = tg + i;
+      if (a.seq && t < N && t >= next_end) {
+        while (b < bhi && t >= next_end) {
+          ++b;
+          next_end = cu[b + 1];
+        }
+        w = weight(b);
+      }
+      const float term = clip_token(lp[i], od[i], ad[i], act[i], a.lo, a.hi, w, cf[i], fl[i], nl, nh, nf);
+      // compensated accumulation (Knuth two-sum)
+      const float s = __fadd_rn(acc_hi, term);
+      const float bb = __fsub_rn(s, acc_hi);
+      acc_lo = __fadd_rn(acc_lo, __fadd_rn(__fsub_rn(acc_hi, __fsub_rn(s, bb)), __fsub_rn(term, bb)));
+      acc_hi = s;
+      cf[i] *= gscale;
+    }
+    if (vec) {
+      if (a.coef) *reinterpret_cast<float4 *>(a.coef + tg) = make_float4(cf[0], cf[1], cf[2], cf[3]);
+      if (a.flags && !kBwd) *reinterpret_cast<uchar4 *>(a.flags + tg) = make_uchar4(fl[0], fl[1], fl[2], fl[3]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (tg + i < N) {
+          if (a.coef) a.coef[tg + i] = cf[i];
+          if (a.flags && !kBwd) a.flags[tg + i] = fl[i];
+        }
+    }
+  }
+  if (kBwd) return;
+  double sum = double(acc_hi) + double(acc_lo);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    nl += __shfl_xor_sync(0xffffffffu, nl, o);
+    nh += __shfl_xor_sync(0xffffffffu, nh, o);
+    nf += __shfl_xor_sync(0xffffffffu, nf, o);
+  }
+  if (lane == 0) {
+    a.part_loss[gw] = sum;
+    a.part_cnt[gw] = nl;
+    a.part_cnt[a.nchunks + gw] = nh;
+    a.part_cnt[2 * a.nchunks + gw] = nf;
+  }
+}
+
+__global__ void __launch_bounds__(256) clip_finalize_kernel(const double *part_loss, const int *part_cnt, int n,
+                                                            const Norms *norms, float *loss, int64_t *counts) {
+  double s = 0.0;
+  long long l = 0, h = 0, f = 0;
+  for (int i = threadIdx.x; i < n; i += 256) {
+    s += part_loss[i];
+    l += part_cnt[i];
+    h += part_cnt[n + i];
+    f += part_cnt[2 * n + i];
+  }
+  __shared__ double sd[8];
+  __shared__ long long sl[3][8];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    s += __shfl_xor_sync(0xffffffffu, s, o);
+    l += __shfl_xor_sync(0xffffffffu, l, o);
+    h += __shfl_xor_sync(0xffffffffu, h, o);
+    f += __shfl_xor_sync(0xffffffffu, f, o);
+  }
+  const int w = threadIdx.x >> 5;
+  if ((threadIdx.x & 31) == 0) {
+    sd[w] = s;
+    sl[0][w] = l;
+    sl[1][w] = h;
+    sl[2][w] = f;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double S = 0.0;
+    long long L = 0, Hh = 0, F = 0;
+    for (int k = 0; k < 8; ++k) {
+      S += sd[k];
+      L += sl[0][k];
+      Hh += sl[1][k];
+      F += sl[2][k];
+    }
+    *loss = float(-S);
+    counts[0] = norms->n_action;
+    counts[1] = L;
+    counts[2] = Hh;
+    counts[3] = F;
+  }
+}
+
+// GRPO: per-trajectory standardised reward within its group (fp64).
+__global__ void group_norm_kernel(const float *R, const int32_t *gid, int B, float eps, float *a_traj) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  const int g = gid[b];
+  double s = 0.0, s2 = 0.0;
+  long long n = 0;
+  for (int j = 0; j < B; ++j)
+    if (gid[j] == g) {
+      const double r = R[j];
+      s += r;
+      n++;
+    }
+  const double mu = s / double(n);
+  for (int j = 0; j < B; ++j)
+    if (gid[j] == g) {
+      const double d = double(R[j]) - mu;
+      s2 += d * d;
+    }
+  const double var = s2 / double(n);
+  a_traj[b] = float((double(R[b]) - mu) / sqrt(var + double(eps)));
+}
+
+// One warp per trajectory: broadcast to its action tokens.
+__global__ void __launch_bounds__(256) group_broadcast_kernel(const float *a_traj, const uint8_t *m,
+                                                              const int32_t *cu, int B, int64_t N, float *adv) {
+  const int lane = threadIdx.x & 31;
+  for (int b = (blockIdx.x * 256 + threadIdx.x) >> 5; b < B; b += (gridDim.x * 256) >> 5) {
+    const int64_t lo = cu[b], hi = cu[b + 1] < N ? cu[b + 1] : N;
+    const float v = a_traj[b];
+    for (int64_t t = lo + lane; t < hi; t += 32) adv[t] = m[t] ? v : 0.f;
+  }
+}
+
+// Running-mean baseline: trajectories in batch order against per-prompt
+// windows of recent rewards (one thread: the windows make it sequential).
+__global__ void running_mean_kernel(const float *R, const int32_t *pid, int B, float *history, long long *seen,
+                                    int window, float *a_traj) {
+  if (blockIdx.x != 0 || threadIdx.x != 0) return;
+  for (int b = 0; b < B; ++b) {
+    const int p = pid[b];
+    const long long c = seen[p];
+    const int n = int(c < window ? c : window);
+    float *h = history + int64_t(p) * window;
+    double s = 0.0;
+    for (int i = 0; i < n; ++i) s += h[i];
+    const double base = n > 0 ? s / double(n) : 0.0;
+    a_traj[b] = float(double(R[b]) - base);
+    h[c % window] = R[b];
+    seen[p] = c + 1;
+  }
+}
+
+}  // namespace
+
+size_t baselines_ws_bytes(int64_t N, int64_t B) {
+  const int64_t nchunks = (N + kSegChunk - 1) / kSegChunk;
+  return round256(sizeof(int) * (nchunks + 1)) + round256(sizeof(int) * (B + 1)) + round256(sizeof(Norms)) +
+         round256(sizeof(double) * nchunks) + round256(sizeof(int) * 3 * nchunks) + round256(sizeof(float) * (B + 1));
+}
+
+sao_status clip_loss_launch(const float *logp, const float *old, const float *adv, const uint8_t *m, const int32_t *cu,
+                            int32_t B, int64_t N, float eps_low, float eps_high, int norm, float *loss, float *coef,
+                            uint8_t *flags, int64_t *counts, const float *grad_loss, void *ws_body,
+                            size_t body_bytes, cudaStream_t s) {
+  const int64_t nchunks = (N + kSegChunk - 1) / kSegChunk;
+  Carver c(ws_body, body_bytes);
+  int *chunk_first = c.take<int>(size_t(nchunks) + 1);
+  int *nact = c.take<int>(size_t(B) + 1);
+  Norms *norms = c.take<Norms>(1);
+  double *part_loss = c.take<double>(size_t(nchunks));
+  int *part_cnt = c.take<int>(3 * size_t(nchunks));
+  if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the clipped surrogate");
+  if (N == 0) {
+    if (loss) SAO_CUDA_TRY(cudaMemsetAsync(loss, 0, sizeof(float), s));
+    if (counts) SAO_CUDA_TRY(cudaMemsetAsync(counts, 0, 4 * sizeof(int64_t), s));
+    return SAO_OK;
+  }
+  SAO_CUDA_TRY(cudaMemsetAsync(nact, 0, sizeof(int) * size_t(B), s));
+  const unsigned grid = unsigned((nchunks + kWarps - 1) / kWarps);
+  int slot = launch_begin("clip_loss_counts", s);
+  seg::chunk_first_kernel<<<unsigned((nchunks + 255) / 256), 256, 0, s>>>(cu, B, N, int(nchunks), chunk_first);
+  seg::action_count_kernel<<<grid, kThreads, 0, s>>>(m, cu, B, N, int(nchunks), chunk_first, nact);
+  norms_kernel<<<1, 256, 0, s>>>(nact, B, norms);
+  SAO_TRY(launch_end(slot, s));
+  ClipArgs a;
+  a.logp = logp;
+  a.old = old;
+  a.adv = adv;
+  a.m = m;
+  a.cu = cu;
+  a.B = B;
+  a.N = N;
+  a.nchunks = int(nchunks);
+  a.chunk_first = chunk_first;
+  a.nact = nact;
+  a.norms = norms;
+  a.lo = 1.0f - eps_low;
+  a.hi = 1.0f + eps_high;
+  a.seq = norm == SAO_NORM_SEQUENCE;
+  a.coef = coef;
+  a.flags = flags;
+  a.grad_scale = grad_loss;
+  a.part_loss = part_loss;
+  a.part_cnt = part_cnt;
+  if (grad_loss) {
+    slot = launch_begin("clip_loss_bwd", s);
+    clip_loss_kernel<true><<<grid, kThreads, 0, s>>>(a);
+    return launch_end(slot, s);
+  }
+  slot = launch_begin("clip_loss_fwd", s);
+  clip_loss_kernel<false><<<grid, kThreads, 0, s>>>(a);
+  clip_finalize_kernel<<<1, 256, 0, s>>>(part_loss, part_cnt, int(nchunks), norms, loss, counts);
+  return launch_end(slot, s);
+}
+
+sao_status group_adv_launch(const float *rewards, const int32_t *gid, int32_t B, const uint8_t *m, const int32_t *cu,
+                            int64_t N, float eps, float *adv, void *ws_body, size_t body_bytes, cudaStream_t s) {
+  Carver c(ws_body, body_bytes);
+  float *a_traj = c.take<float>(size_t(B) + 1);
+  if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the group advantages");
+  SAO_CUDA_TRY(cudaMemsetAsync(adv, 0, sizeof(float) * size_t(N), s));
+  if (B == 0) return SAO_OK;
+  DeviceInfo di;
+  SAO_TRY(device_info(&di));
+  int slot = launch_begin("group_advantages", s);
+  group_norm_kernel<<<unsigned((B + 127) / 128), 128, 0, s>>>(rewards, gid, B, eps, a_traj);
+  group_broadcast_kernel<<<unsigned(di.sm_count * 4), 256, 0, s>>>(a_traj, m, cu, B, N, adv);
+  return launch_end(slot, s);
+}
+
+sao_status running_mean_launch(const float *rewards, const int32_t *pid, int32_t B, float *history, int64_t *seen,
+                               int32_t window, const uint8_t *m, const int32_t *cu, int64_t N, float *adv,
+                               void *ws_body, size_t body_bytes, cudaStream_t s) {
+  Carver c(ws_body, body_bytes);
+  float *a_traj = c.take<float>(size_t(B) + 1);
+  if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the running-mean baseline");
+  if (N > 0) SAO_CUDA_TRY(cudaMemsetAsync(adv, 0, sizeof(float) * size_t(N), s));
+  if (B == 0) return SAO_OK;
+  DeviceInfo di;
+  SAO_TRY(device_info(&di));
+  int slot = launch_begin("running_mean_advantages", s);
+  running_mean_kernel<<<1, 32, 0, s>>>(rewards, pid, B, history, reinterpret_cast<long long *>(seen), window, a_traj);
+  if (N > 0) group_broadcast_kernel<<<unsigned(di.sm_count * 4), 256, 0, s>>>(a_traj, m, cu, B, N, adv);
+  return launch_end(slot, s);
+}
+
+}  // namespace sao

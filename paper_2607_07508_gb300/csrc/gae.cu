@@ -32,13 +32,14 @@
 
 #include "sao_common.cuh"
 #include "sao_internal.h"
+#include "segments.cuh"
 
 namespace sao {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kItems = 32;           // tokens per lane (at most 32: one bit each)
-constexpr int kChunk = 32 * kItems;  // tokens per warp chunk
+constexpr int kItems = seg::kItems;       // tokens per lane (at most 32: one bit each)
+constexpr int kChunk = seg::kSegChunk;    // tokens per warp chunk
 constexpr int kWarps = kThreads / 32;
 
 // ---------------------------------------------------------------------------
@@ -280,36 +281,9 @@ struct GaeArgs {
   unsigned int *err;
 };
 
-constexpr int kCuCap = 128;  // cu_seqlens entries staged per warp
-
-// cu_seqlens entries [blo, blo + n) of one chunk, read from shared memory
-// when the slice fits there, else from global memory.
-struct CuView {
-  const int32_t *g;
-  const int32_t *s;
-  int blo;
-  bool in_smem;
-  __device__ __forceinline__ int64_t operator[](int b) const { return in_smem ? s[b - blo] : __ldg(g + b); }
-  // largest b in [lo, hi] with cu[b] <= t
-  __device__ __forceinline__ int find(int lo, int hi, int64_t t) const {
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if ((*this)[mid] <= t) lo = mid;
-      else hi = mid - 1;
-    }
-    return lo;
-  }
-};
-
-__device__ __forceinline__ int find_traj(const int32_t *cu, int B, int64_t t) {
-  int lo = 0, hi = B - 1;
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (int64_t(__ldg(cu + mid)) <= t) lo = mid;
-    else hi = mid - 1;
-  }
-  return lo;
-}
+using seg::CuView;
+using seg::find_traj;
+using seg::kCuCap;
 
 // State at the right edge of chunk q, from the chunks to its right. The warp
 // inspects 32 successors (q+1 .. q+32) per round: each lane polls one status
@@ -607,74 +581,6 @@ __global__ void __launch_bounds__(kThreads, 3) gae_scan_kernel(GaeArgs a) {
   }
 }
 
-// Number of action tokens per trajectory (only for the length-adaptive lambda).
-// One warp per 512-token chunk, like the scan.
-__global__ void __launch_bounds__(kThreads) gae_count_kernel(const uint8_t *m, const int32_t *cu_g, int B,
-                                                             int64_t N, int nchunks, const int *chunk_first,
-                                                             int *nact) {
-  __shared__ int32_t s_cu_all[kWarps][kCuCap];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int q = blockIdx.x * kWarps + warp;
-  if (q >= nchunks) return;
-  const int blo = chunk_first[q];
-  const int bhi = q + 1 < nchunks ? chunk_first[q + 1] : B - 1;
-  const int ncu = bhi - blo + 2;
-  int32_t *s_cu = s_cu_all[warp];
-  const CuView cu{cu_g, s_cu, blo, ncu <= kCuCap};
-  if (cu.in_smem)
-    for (int i = lane; i < ncu; i += 32) s_cu[i] = __ldg(cu_g + blo + i);
-  __syncwarp();
-  const int64_t t0 = int64_t(q) * kChunk + int64_t(lane) * kItems;
-  int b = cu.find(blo, bhi, t0 < N ? t0 : N - 1);
-  int64_t next_end = cu[b + 1];
-  int cnt = 0;
-  const bool vec = (t0 + kItems <= N) && ((reinterpret_cast<uintptr_t>(m) & 15u) == 0);
-#pragma unroll 1
-  for (int g = 0; g < kItems / 16; ++g) {
-    uint32_t w[4] = {0u, 0u, 0u, 0u};
-    if (vec) {
-      const uint4 x = __ldg(reinterpret_cast<const uint4 *>(m + t0) + g);
-      w[0] = x.x;
-      w[1] = x.y;
-      w[2] = x.z;
-      w[3] = x.w;
-    } else {
-      for (int k = 0; k < 16; ++k) {
-        const int64_t t = t0 + 16 * g + k;
-        if (t < N && m[t] != 0) w[k >> 2] |= 1u << (8 * (k & 3));
-      }
-    }
-#pragma unroll
-    for (int k = 0; k < 16; ++k) {
-      const int64_t t = t0 + 16 * g + k;
-      if (t >= N) break;
-      if (t >= next_end) {
-        const int nb0 = b;
-        while (b < bhi && t >= next_end) {
-          ++b;
-          next_end = cu[b + 1];
-        }
-        if (b != nb0 && cnt) {
-          atomicAdd(nact + nb0, cnt);
-          cnt = 0;
-        }
-      }
-      cnt += ((w[k >> 2] >> (8 * (k & 3))) & 0xffu) != 0u;
-    }
-  }
-  const unsigned peers = __match_any_sync(0xffffffffu, b);
-  const int tot = __reduce_add_sync(peers, cnt);
-  if (lane == __ffs(peers) - 1 && tot) atomicAdd(nact + b, tot);
-}
-
-// First trajectory of every chunk (one binary search per chunk, all in parallel).
-__global__ void gae_chunk_first_kernel(const int32_t *cu, int B, int64_t N, int nchunks, int *chunk_first) {
-  const int q = blockIdx.x * blockDim.x + threadIdx.x;
-  if (q >= nchunks) return;
-  const int64_t t = int64_t(q) * kChunk;
-  chunk_first[q] = find_traj(cu, B, t < N ? t : N - 1);
-}
-
 // Per-trajectory coefficients (fp64 then split to double-float) and a check of
 // cu_seqlens: 0 = cu[0] <= cu[1] <= ... <= cu[B] = N.
 __global__ void gae_coef_kernel(const int32_t *cu, int B, int64_t N, float gamma, float lam, float lam_c,
@@ -725,12 +631,12 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   SAO_CUDA_TRY(cudaMemsetAsync(zero_begin, 0, size_t(zero_end - zero_begin), s));
   {
     int slot = launch_begin("gae_chunk_first", s);
-    gae_chunk_first_kernel<<<unsigned((nchunks + 255) / 256), 256, 0, s>>>(cu, B, N, int(nchunks), chunk_first);
+    seg::chunk_first_kernel<<<unsigned((nchunks + 255) / 256), 256, 0, s>>>(cu, B, N, int(nchunks), chunk_first);
     SAO_TRY(launch_end(slot, s));
   }
   if (alpha > 0.f) {
     int slot = launch_begin("gae_count", s);
-    gae_count_kernel<<<unsigned((nchunks + kWarps - 1) / kWarps), kThreads, 0, s>>>(m, cu, B, N, int(nchunks),
+    seg::action_count_kernel<<<unsigned((nchunks + kWarps - 1) / kWarps), kThreads, 0, s>>>(m, cu, B, N, int(nchunks),
                                                                                     chunk_first, nact);
     SAO_TRY(launch_end(slot, s));
   }

@@ -20,8 +20,10 @@ size_t on_ws_bytes(int64_t N) {
   size_t w = elementwise_ws_bytes(N, 0);
   const size_t g = gae_ws_bytes(N, N + 1);
   const size_t st = step_gae_ws_bytes(N, N + 1);
+  const size_t bl = baselines_ws_bytes(N, N + 1);
   if (g > w) w = g;
   if (st > w) w = st;
+  if (bl > w) w = bl;
   return w;
 }
 
@@ -233,6 +235,82 @@ sao_status sao_value_loss(const float *values, const float *ret, const uint8_t *
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   SAO_TRY(begin_call(ws, s));
   SAO_TRY(value_loss_launch(values, ret, loss_mask, N, loss, grad_values, ev_sums, w.body, w.body_bytes, s));
+  return finish_call(ws, s);
+}
+
+static sao_status check_traj(int32_t B, int64_t N, const int32_t *cu) {
+  if (N < 0 || N >= (int64_t(1) << 31)) return fail(SAO_ERR_SHAPE, "N = %lld out of range", (long long)N);
+  if (B < 0) return fail(SAO_ERR_SHAPE, "B = %d < 0", B);
+  if (N > 0 && (B == 0 || !cu)) return fail(SAO_ERR_SHAPE, "N > 0 tokens need at least one trajectory");
+  return SAO_OK;
+}
+
+sao_status sao_clip_loss_fwd(const float *logp, const float *old_logp, const float *adv, const uint8_t *loss_mask,
+                             const int32_t *cu_seqlens, int32_t B, int64_t N, float eps_low, float eps_high, int norm,
+                             float *loss, float *coef, uint8_t *flags, int64_t *counts, void *ws, size_t ws_bytes,
+                             sao_stream_t stream) {
+  SAO_TRY(check_traj(B, N, cu_seqlens));
+  SAO_TRY(check_eps(eps_low, eps_high));
+  if (norm != SAO_NORM_TOKEN && norm != SAO_NORM_SEQUENCE) return fail(SAO_ERR_INVALID_ARG, "unknown norm %d", norm);
+  if (!loss || !counts) return fail(SAO_ERR_INVALID_ARG, "NULL loss or counts");
+  if (N > 0 && (!logp || !old_logp || !adv || !loss_mask)) return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
+  Ws w;
+  SAO_TRY(take_ws(ws, ws_bytes, baselines_ws_bytes(N, B), &w));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  SAO_TRY(begin_call(ws, s));
+  SAO_TRY(clip_loss_launch(logp, old_logp, adv, loss_mask, cu_seqlens, B, N, eps_low, eps_high, norm, loss, coef,
+                           flags, counts, nullptr, w.body, w.body_bytes, s));
+  return finish_call(ws, s);
+}
+
+sao_status sao_clip_loss_bwd(const float *logp, const float *old_logp, const float *adv, const uint8_t *loss_mask,
+                             const int32_t *cu_seqlens, int32_t B, int64_t N, float eps_low, float eps_high, int norm,
+                             const float *grad_loss, float *grad_logp, void *ws, size_t ws_bytes,
+                             sao_stream_t stream) {
+  SAO_TRY(check_traj(B, N, cu_seqlens));
+  SAO_TRY(check_eps(eps_low, eps_high));
+  if (norm != SAO_NORM_TOKEN && norm != SAO_NORM_SEQUENCE) return fail(SAO_ERR_INVALID_ARG, "unknown norm %d", norm);
+  if (N == 0) return SAO_OK;
+  if (!logp || !old_logp || !adv || !loss_mask || !grad_loss || !grad_logp)
+    return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
+  Ws w;
+  SAO_TRY(take_ws(ws, ws_bytes, baselines_ws_bytes(N, B), &w));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  SAO_TRY(begin_call(ws, s));
+  SAO_TRY(clip_loss_launch(logp, old_logp, adv, loss_mask, cu_seqlens, B, N, eps_low, eps_high, norm, nullptr,
+                           grad_logp, nullptr, nullptr, grad_loss, w.body, w.body_bytes, s));
+  return finish_call(ws, s);
+}
+
+sao_status sao_group_advantages(const float *rewards, const int32_t *group_ids, int32_t B, const uint8_t *loss_mask,
+                                const int32_t *cu_seqlens, int64_t N, float eps_stab, float *adv, void *ws,
+                                size_t ws_bytes, sao_stream_t stream) {
+  SAO_TRY(check_traj(B, N, cu_seqlens));
+  if (!(eps_stab >= 0.f) || !isfinite(eps_stab)) return fail(SAO_ERR_INVALID_ARG, "eps_stab must be >= 0");
+  if (N == 0) return SAO_OK;
+  if (!rewards || !group_ids || !loss_mask || !adv) return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
+  Ws w;
+  SAO_TRY(take_ws(ws, ws_bytes, baselines_ws_bytes(N, B), &w));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  SAO_TRY(begin_call(ws, s));
+  SAO_TRY(group_adv_launch(rewards, group_ids, B, loss_mask, cu_seqlens, N, eps_stab, adv, w.body, w.body_bytes, s));
+  return finish_call(ws, s);
+}
+
+sao_status sao_running_mean_advantages(const float *rewards, const int32_t *prompt_ids, int32_t B,
+                                       int32_t num_prompts, float *history, int64_t *seen, int32_t window,
+                                       const uint8_t *loss_mask, const int32_t *cu_seqlens, int64_t N, float *adv,
+                                       void *ws, size_t ws_bytes, sao_stream_t stream) {
+  SAO_TRY(check_traj(B, N, cu_seqlens));
+  if (window < 1 || num_prompts < 1) return fail(SAO_ERR_INVALID_ARG, "window and num_prompts must be >= 1");
+  if (B > 0 && (!rewards || !prompt_ids || !history || !seen)) return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
+  if (N > 0 && (!loss_mask || !adv)) return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
+  Ws w;
+  SAO_TRY(take_ws(ws, ws_bytes, baselines_ws_bytes(N, B), &w));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  SAO_TRY(begin_call(ws, s));
+  SAO_TRY(running_mean_launch(rewards, prompt_ids, B, history, seen, window, loss_mask, cu_seqlens, N, adv, w.body,
+                              w.body_bytes, s));
   return finish_call(ws, s);
 }
 

@@ -33,6 +33,18 @@ sao_status step_gae_launch(const float *values, const float *rewards, const uint
                            int64_t N, float gamma, float lam, float lam_c, float alpha, int mode, float *adv,
                            float *ret, uint8_t *vmask, void *ws_body, size_t body_bytes, cudaStream_t s);
 
+// baselines.cu ----------------------------------------------------------------
+size_t baselines_ws_bytes(int64_t N, int64_t B);
+sao_status clip_loss_launch(const float *logp, const float *old, const float *adv, const uint8_t *m, const int32_t *cu,
+                            int32_t B, int64_t N, float eps_low, float eps_high, int norm, float *loss, float *coef,
+                            uint8_t *flags, int64_t *counts, const float *grad_loss, void *ws_body,
+                            size_t body_bytes, cudaStream_t s);
+sao_status running_mean_launch(const float *rewards, const int32_t *pid, int32_t B, float *history, int64_t *seen,
+                               int32_t window, const uint8_t *m, const int32_t *cu, int64_t N, float *adv,
+                               void *ws_body, size_t body_bytes, cudaStream_t s);
+sao_status group_adv_launch(const float *rewards, const int32_t *gid, int32_t B, const uint8_t *m, const int32_t *cu,
+                            int64_t N, float eps, float *adv, void *ws_body, size_t body_bytes, cudaStream_t s);
+
 // logprobs (tensor-core and fp32 paths) ----------------------------------------
 size_t logprobs_ws_bytes(int64_t N, int32_t h, int32_t V, sao_dtype dt);
 sao_status logprobs_fwd_launch(const void *H, const void *W, sao_dtype dt, const int32_t *y,

@@ -19,6 +19,7 @@ LIB_PATH = os.path.join(_HERE, "libsao.so")
 
 SAO_F32, SAO_BF16 = 0, 1
 SAO_STEP_AVERAGE, SAO_STEP_LAST = 0, 1
+SAO_NORM_TOKEN, SAO_NORM_SEQUENCE = 0, 1
 STATUS = {0: "SAO_OK", 1: "SAO_ERR_INVALID_ARG", 2: "SAO_ERR_SHAPE", 3: "SAO_ERR_WORKSPACE",
           4: "SAO_ERR_UNSUPPORTED", 5: "SAO_ERR_CUDA", 6: "SAO_ERR_DEVICE_CHECK"}
 FLAG_IN, FLAG_LOW, FLAG_HIGH, FLAG_NONFINITE, FLAG_NOT_ACTION = 0, 1, 2, 3, 4
@@ -26,7 +27,8 @@ FLAG_IN, FLAG_LOW, FLAG_HIGH, FLAG_NONFINITE, FLAG_NOT_ACTION = 0, 1, 2, 3, 4
 EXPORTS = ("sao_version", "sao_last_error_string", "sao_set_checked", "sao_get_checked",
            "sao_set_dz_budget_bytes", "sao_workspace_bytes", "sao_token_logprobs_fwd",
            "sao_token_logprobs_bwd", "sao_advantages", "sao_advantages_noalloc", "sao_step_advantages",
-           "sao_policy_loss_fwd", "sao_policy_loss_bwd",
+           "sao_policy_loss_fwd", "sao_policy_loss_bwd", "sao_clip_loss_fwd", "sao_clip_loss_bwd",
+           "sao_group_advantages", "sao_running_mean_advantages",
            "sao_value_loss", "sao_profile_enable", "sao_profile_reset", "sao_profile_read")
 
 
@@ -66,6 +68,10 @@ def load(path: Optional[str] = None):
         "sao_policy_loss_fwd": (ctypes.c_int, [P, P, P, P, I64, F, F, I64, P, P, P, P, P, SZ, P]),
         "sao_policy_loss_bwd": (ctypes.c_int, [P, P, P, P, I64, F, F, I64, P, P, P, SZ, P]),
         "sao_value_loss": (ctypes.c_int, [P, P, P, I64, P, P, P, P, SZ, P]),
+        "sao_clip_loss_fwd": (ctypes.c_int, [P, P, P, P, P, I32, I64, F, F, ctypes.c_int, P, P, P, P, P, SZ, P]),
+        "sao_clip_loss_bwd": (ctypes.c_int, [P, P, P, P, P, I32, I64, F, F, ctypes.c_int, P, P, P, SZ, P]),
+        "sao_group_advantages": (ctypes.c_int, [P, P, I32, P, P, I64, F, P, P, SZ, P]),
+        "sao_running_mean_advantages": (ctypes.c_int, [P, P, I32, I32, P, P, I32, P, P, I64, P, P, SZ, P]),
         "sao_profile_enable": (None, [ctypes.c_int]),
         "sao_profile_reset": (None, []),
         "sao_profile_read": (ctypes.c_int, [P, P, P, ctypes.c_int]),
@@ -266,6 +272,67 @@ def sao_value_loss(values, ret, loss_mask, loss, grad_values, ws, ev_sums=None, 
     _expect(ev_sums, torch.float64, 4, "ev_sums")
     _check(load().sao_value_loss(_ptr(values), _ptr(ret), _ptr(loss_mask), N, _ptr(loss), _ptr(grad_values),
                                  _ptr(ev_sums), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def sao_clip_loss_fwd(logp, old_logp, adv, loss_mask, cu_seqlens, eps_low, eps_high, norm, loss, counts, ws,
+                      coef=None, flags=None, stream=None):
+    N = logp.numel()
+    B = cu_seqlens.numel() - 1
+    for t, name in ((logp, "logp"), (old_logp, "old_logp"), (adv, "adv")):
+        _expect(t, torch.float32, N, name)
+    _expect(loss_mask, torch.uint8, N, "loss_mask")
+    _expect(cu_seqlens, torch.int32, B + 1, "cu_seqlens")
+    _expect(coef, torch.float32, N, "coef")
+    _expect(flags, torch.uint8, N, "flags")
+    _expect(loss, torch.float32, 1, "loss")
+    _expect(counts, torch.int64, 4, "counts")
+    _check(load().sao_clip_loss_fwd(_ptr(logp), _ptr(old_logp), _ptr(adv), _ptr(loss_mask), _ptr(cu_seqlens), B, N,
+                                    float(eps_low), float(eps_high), int(norm), _ptr(loss), _ptr(coef), _ptr(flags),
+                                    _ptr(counts), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def sao_clip_loss_bwd(logp, old_logp, adv, loss_mask, cu_seqlens, eps_low, eps_high, norm, grad_loss, grad_logp, ws,
+                      stream=None):
+    N = logp.numel()
+    B = cu_seqlens.numel() - 1
+    for t, name in ((logp, "logp"), (old_logp, "old_logp"), (adv, "adv"), (grad_logp, "grad_logp")):
+        _expect(t, torch.float32, N, name)
+    _expect(loss_mask, torch.uint8, N, "loss_mask")
+    _expect(cu_seqlens, torch.int32, B + 1, "cu_seqlens")
+    _expect(grad_loss, torch.float32, 1, "grad_loss")
+    _check(load().sao_clip_loss_bwd(_ptr(logp), _ptr(old_logp), _ptr(adv), _ptr(loss_mask), _ptr(cu_seqlens), B, N,
+                                    float(eps_low), float(eps_high), int(norm), _ptr(grad_loss), _ptr(grad_logp),
+                                    _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def sao_group_advantages(rewards, group_ids, loss_mask, cu_seqlens, eps_stab, adv, ws, stream=None):
+    N = loss_mask.numel()
+    B = cu_seqlens.numel() - 1
+    _expect(rewards, torch.float32, B, "rewards")
+    _expect(group_ids, torch.int32, B, "group_ids")
+    _expect(loss_mask, torch.uint8, N, "loss_mask")
+    _expect(cu_seqlens, torch.int32, B + 1, "cu_seqlens")
+    _expect(adv, torch.float32, N, "adv")
+    _check(load().sao_group_advantages(_ptr(rewards), _ptr(group_ids), B, _ptr(loss_mask), _ptr(cu_seqlens), N,
+                                       float(eps_stab), _ptr(adv), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def sao_running_mean_advantages(rewards, prompt_ids, history, seen, loss_mask, cu_seqlens, adv, ws, stream=None):
+    """history [P, window] fp32 and seen [P] int64 are updated in place."""
+    N = loss_mask.numel()
+    B = cu_seqlens.numel() - 1
+    P, window = history.shape
+    _expect(rewards, torch.float32, B, "rewards")
+    _expect(prompt_ids, torch.int32, B, "prompt_ids")
+    _expect(seen, torch.int64, P, "seen")
+    _expect(loss_mask, torch.uint8, N, "loss_mask")
+    _expect(cu_seqlens, torch.int32, B + 1, "cu_seqlens")
+    _expect(adv, torch.float32, N, "adv")
+    if history.dtype != torch.float32:
+        raise ValueError("history must be fp32")
+    _check(load().sao_running_mean_advantages(_ptr(rewards), _ptr(prompt_ids), B, P, _ptr(history), _ptr(seen),
+                                              window, _ptr(loss_mask), _ptr(cu_seqlens), N, _ptr(adv), _ptr(ws),
+                                              ws.numel(), _stream(stream)))
 
 
 # ---------------------------------------------------------------------------

@@ -59,3 +59,96 @@ def test_step_advantages_no_action_tokens():
     wl.loss_mask[:] = 0
     adv, ret, vm = _step_gpu(wl, 1.0, 1.0, 1.0, 0.0, sao.SAO_STEP_AVERAGE)
     assert not adv.any() and not ret.any() and not vm.any()
+
+
+# ---------------------------------------------------------------------------
+# clipped surrogate (PPO / GRPO arms) and GRPO advantages
+# ---------------------------------------------------------------------------
+
+def _clip_gpu(logp, old, adv, mask, cu, el, eh, norm):
+    N = len(logp)
+    loss = torch.empty(1, device="cuda")
+    counts = torch.empty(4, dtype=torch.int64, device="cuda")
+    coef = torch.empty(N, device="cuda")
+    flags = torch.empty(N, dtype=torch.uint8, device="cuda")
+    grad = torch.empty(N, device="cuda")
+    ws = sao.workspace(N)
+    args = [cuda(x) for x in (logp, old, adv, mask, cu)]
+    sao.sao_clip_loss_fwd(*args, el, eh, norm, loss, counts, ws, coef=coef, flags=flags)
+    sao.sao_clip_loss_bwd(*args, el, eh, norm, torch.tensor([0.5], device="cuda"), grad, ws)
+    torch.cuda.synchronize()
+    return float(loss.item()), counts.cpu().numpy(), coef.cpu().numpy(), flags.cpu().numpy(), grad.cpu().numpy()
+
+
+def _near_clip_bound(logp, old, el, eh, tol=1e-6):
+    r = np.exp(np.asarray(logp, np.float64) - np.asarray(old, np.float64))
+    with np.errstate(invalid="ignore"):
+        return (np.abs(r - (1 - el)) <= tol) | (np.abs(r - (1 + eh)) <= tol)
+
+
+@pytest.mark.parametrize("norm", [sao.SAO_NORM_TOKEN, sao.SAO_NORM_SEQUENCE])
+@pytest.mark.parametrize("name", S.CONFIG_NAMES)
+def test_clip_loss_match_oracle(name, norm):
+    wl = S.make_workload(name, dense=False)
+    adv = np.random.default_rng(5).normal(size=wl.N).astype(np.float32)
+    el, eh = 0.2, 0.28
+    loss, counts, coef, flags, grad = _clip_gpu(wl.logp_syn, wl.old_logp_syn, adv, wl.loss_mask, wl.cu_seqlens,
+                                                el, eh, norm)
+    want = O.clip_loss(wl.logp_syn, wl.old_logp_syn, adv, wl.loss_mask, wl.cu_seqlens, el, eh, norm)
+    skip = _near_clip_bound(wl.logp_syn, wl.old_logp_syn, el, eh)
+    assert np.array_equal(flags[~skip], want["flags"][~skip])
+    if not skip.any():
+        assert np.array_equal(counts, want["counts"])
+    assert abs(loss - want["loss"]) <= 1e-4 * max(abs(want["loss"]), 1e-6)
+    keep = ~skip
+    assert rel_err_floor(coef[keep], want["coef"][keep], 1e-12).max() <= 1e-5
+    assert rel_err_floor(grad[keep], 0.5 * want["coef"][keep], 1e-12).max() <= 1e-5
+
+
+@pytest.mark.parametrize("norm", [sao.SAO_NORM_TOKEN, sao.SAO_NORM_SEQUENCE])
+def test_clip_loss_edge_layouts(norm):
+    wl = S.make_custom([0, 1, 1023, 0, 2049, 5], 8, 16, "f32", seed=8, dense=False, obs_frac=0.3)
+    rng = np.random.default_rng(6)
+    adv = rng.normal(size=wl.N).astype(np.float32)
+    old = (wl.logp_syn + rng.normal(0, 0.5, wl.N)).astype(np.float32)
+    old[::50] = -np.inf
+    loss, counts, coef, flags, grad = _clip_gpu(wl.logp_syn, old, adv, wl.loss_mask, wl.cu_seqlens, 0.3, 5.0, norm)
+    want = O.clip_loss(wl.logp_syn, old, adv, wl.loss_mask, wl.cu_seqlens, 0.3, 5.0, norm)
+    assert np.array_equal(flags, want["flags"]) and np.array_equal(counts, want["counts"])
+    assert abs(loss - want["loss"]) <= 1e-4 * max(abs(want["loss"]), 1e-6)
+    assert rel_err_floor(coef, want["coef"], 1e-12).max() <= 1e-5
+
+
+def test_group_advantages_match_oracle():
+    for name in ("small", "large"):
+        wl = S.make_workload(name, dense=False)
+        gid = (np.arange(wl.B) // 8).astype(np.int32)            # 8 rollouts per prompt
+        rng = np.random.default_rng(3)
+        rng.shuffle(gid)
+        adv = torch.empty(wl.N, device="cuda")
+        sao.sao_group_advantages(cuda(wl.rewards), cuda(gid), cuda(wl.loss_mask), cuda(wl.cu_seqlens), 1e-6, adv,
+                                 sao.workspace(wl.N))
+        torch.cuda.synchronize()
+        want = O.group_advantages(wl.rewards, gid, wl.loss_mask, wl.cu_seqlens, f32(1e-6))
+        assert rel_err_floor(adv.cpu().numpy(), want, 1e-3).max() <= 1e-5
+
+
+def test_running_mean_advantages_match_oracle():
+    """Two batches in a row with per-prompt windows of 8 (§4.3) and one global
+    window of 128 (§4.5); the windows persist between calls."""
+    for P, window in ((16, 8), (1, 128)):
+        hist_d = torch.zeros(P, window, device="cuda")
+        seen_d = torch.zeros(P, dtype=torch.int64, device="cuda")
+        hist_o, seen_o = np.zeros((P, window)), np.zeros(P, np.int64)
+        for seed in (1, 2):
+            wl = S.make_workload("large", dense=False, seed=S.SEED_BASE + 40 + seed)
+            pid = np.random.default_rng(seed).integers(0, P, size=wl.B).astype(np.int32)
+            adv = torch.empty(wl.N, device="cuda")
+            sao.sao_running_mean_advantages(cuda(wl.rewards), cuda(pid), hist_d, seen_d, cuda(wl.loss_mask),
+                                            cuda(wl.cu_seqlens), adv, sao.workspace(wl.N))
+            torch.cuda.synchronize()
+            want, hist_o, seen_o = O.running_mean_advantages(wl.rewards, pid, wl.loss_mask, wl.cu_seqlens, hist_o,
+                                                             seen_o, window)
+            assert rel_err_floor(adv.cpu().numpy(), want, 1e-3).max() <= 1e-5
+            assert np.array_equal(seen_d.cpu().numpy(), seen_o)
+            assert np.allclose(hist_d.cpu().numpy(), hist_o)

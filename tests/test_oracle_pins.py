@@ -589,3 +589,19 @@ def test_group_advantages_are_standardised():
     single = O.group_advantages(np.array([1.0], np.float32), np.array([0]), np.ones(3, np.uint8),
                                 np.array([0, 3]), 1e-6)
     assert np.all(single == 0)
+
+
+def test_running_mean_baseline_window():
+    """Window 2 for prompt 0 over rewards 1, 0, 1, 1: baselines 0 (empty), 1,
+    mean(1, 0), mean(0, 1); prompt 1 keeps its own window."""
+    R = np.array([1.0, 0.0, 1.0, 5.0, 1.0], np.float32)
+    pid = np.array([0, 0, 0, 1, 0])
+    cu = np.arange(6)
+    m = np.ones(5, np.uint8)
+    adv, hist, cnt = O.running_mean_advantages(R, pid, m, cu, np.zeros((2, 2)), np.zeros(2, np.int64), 2)
+    assert np.allclose(adv, [1.0, -1.0, 0.5, 5.0, 0.5])
+    assert list(cnt) == [4, 1] and sorted(hist[0]) == [1.0, 1.0] and hist[1, 0] == 5.0
+    # the state carries over to the next batch
+    adv2, _, _ = O.running_mean_advantages(np.array([0.0], np.float32), np.array([0]), np.ones(1, np.uint8),
+                                           np.array([0, 1]), hist, cnt, 2)
+    assert np.allclose(adv2, [-1.0])
