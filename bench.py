@@ -36,6 +36,24 @@ WORKLOAD = "moe"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
+def stored_traffic(kernel: str, rows: int):
+    """DRAM bytes per launch of `kernel` from the committed ncu capture
+    (profiles/dram_traffic_moe.txt), scaled to `rows` active rows, or None if
+    the capture is missing or the kernel sources changed since it was taken."""
+    from paper_2607_07508_gb300.build import kernel_source_hash
+    path = os.path.join(ROOT, "profiles", "dram_traffic_moe.txt")
+    try:
+        lines = [l.split() for l in open(path) if l.strip() and not l.startswith("#")]
+    except OSError:
+        return None
+    src = kernel_source_hash()
+    for f in lines:
+        if len(f) == 5 and f[0] == kernel and f[1] == src:
+            cap_rows, rd, wr = int(f[2]), float(f[3]), float(f[4])
+            return (rd + wr) * rows / cap_rows
+    return None
+
+
 def load_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -416,8 +434,10 @@ def main():
     peak_t = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
     if fl is not None:
         achieved = fl / (avg_ms / 1000.0) / 1e12
+        dom_rows = rows_fwd if dom_name == "tc_logits_lse_fwd" else rows_bwd
         roofline = {"bound": "tensor", "kernel": dom_name, "achieved": achieved, "peak": peak_t,
-                    "unit": "TFLOP/s", "frac": achieved / peak_t, "traffic": None,
+                    "unit": "TFLOP/s", "frac": achieved / peak_t, "traffic": stored_traffic(dom_name, dom_rows),
+                    "traffic_unit": "bytes per launch (dram read + write, ncu, scaled by active rows)",
                     "algorithmic_per_launch": f"2*rows*h*V = {fl:.4g} flop", "avg_launch_ms": avg_ms,
                     "peak_source": f"{peak_src} bf16_tflops_sustained (kernel timed inside a long step)"}
     else:

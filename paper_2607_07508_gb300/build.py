@@ -45,6 +45,16 @@ def _stamp(srcs) -> str:
     return h.hexdigest()
 
 
+def kernel_source_hash(names=("logprobs_tc.cu", "tc_ptx.cuh", "rows.cu", "rows.cuh")) -> str:
+    """Short hash of the sources that define the tensor-core kernels, used to
+    tell whether stored profiler counters still describe the current kernels."""
+    h = hashlib.sha256()
+    for n in names:
+        with open(os.path.join(CSRC, n), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
 def build(force: bool = False, verbose: bool = False) -> str:
     """Compile (if sources changed) and return the path of libsao.so."""
     srcs = _sources()
