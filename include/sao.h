@@ -246,7 +246,7 @@ SAO_API sao_status sao_running_mean_advantages(const float *rewards, const int32
  *
  * Scratch: a fixed 8 MiB array inside this library's device image, present on
  * every GPU that loads the library until the process exits. It bounds the
- * sizes: about 88 bytes per 512 tokens plus 36 bytes per trajectory must
+ * sizes: about 120 bytes per 1024 tokens plus 36 bytes per trajectory must
  * fit (for example 2^25 tokens with up to 65,536 trajectories); larger
  * inputs return SAO_ERR_SHAPE with the bytes needed. Nothing is allocated
  * and nothing is freed.

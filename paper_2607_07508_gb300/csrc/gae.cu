@@ -37,7 +37,7 @@
 namespace sao {
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 128;
 constexpr int kItems = seg::kItems;       // tokens per lane (at most 32: one bit each)
 constexpr int kChunk = seg::kSegChunk;    // tokens per warp chunk
 constexpr int kWarps = kThreads / 32;
@@ -105,6 +105,7 @@ struct GMap {
   int b, fl;
   df ap, cp, ac, cc;
   float v, p0;
+  TCoef k;  // coefficients of trajectory b (used when the map is the left operand)
 };
 struct GState {
   df Bp, Bc;
@@ -118,20 +119,22 @@ __device__ __forceinline__ GMap identity_map() {
   m.ap = m.ac = {1.f, 0.f};
   m.cp = m.cc = {0.f, 0.f};
   m.v = m.p0 = 0.f;
+  m.k = TCoef{};
   return m;
 }
 
 // x o y: x is the left segment, y the one immediately to its right.
 template <bool kCrit>
-__device__ GMap compose(const GMap &x, const GMap &y, const float4 *tab) {
+__device__ GMap compose(const GMap &x, const GMap &y, const float4 *) {
   if (x.fl & 1) return x;
   if (!(x.fl & 2)) return y;
   if (!(y.fl & 3)) return x;
-  const TCoef c = load_coef(tab, x.b);
+  const TCoef &c = x.k;
   const bool yact = (y.fl & 2) != 0;
   const float Yv = yact ? y.v : 0.f, Yp = yact ? 0.f : y.p0;
   GMap r;
   r.b = x.b;
+  r.k = x.k;
   r.v = x.v;
   r.p0 = 0.f;
   df tp = df_add_f(df_add(df_mul(c.ap, y.cp), df_mul_f(c.gp, Yv)), Yp);
@@ -154,13 +157,13 @@ __device__ GMap compose(const GMap &x, const GMap &y, const float4 *tab) {
 }
 
 template <bool kCrit>
-__device__ GState apply(const GMap &m, const GState &s, const float4 *tab) {
+__device__ GState apply(const GMap &m, const GState &s, const float4 *) {
   if (m.fl & 1) {
     const bool act = (m.fl & 2) != 0;
     return {m.cp, m.cc, act ? m.v : 0.f, act ? 0.f : m.p0};
   }
   if (!(m.fl & 2)) return s;
-  const TCoef c = load_coef(tab, m.b);
+  const TCoef &c = m.k;
   GState r;
   const df tp = df_add_f(df_add(df_mul(c.ap, s.Bp), df_mul_f(c.gp, s.Vn)), s.P);
   r.Bp = df_add(df_mul(m.ap, tp), m.cp);
@@ -189,6 +192,14 @@ __device__ __forceinline__ GMap shfl_down_map(const GMap &m, int d) {
   r.cc.lo = __shfl_down_sync(0xffffffffu, m.cc.lo, d);
   r.v = __shfl_down_sync(0xffffffffu, m.v, d);
   r.p0 = __shfl_down_sync(0xffffffffu, m.p0, d);
+  r.k.ap.hi = __shfl_down_sync(0xffffffffu, m.k.ap.hi, d);
+  r.k.ap.lo = __shfl_down_sync(0xffffffffu, m.k.ap.lo, d);
+  r.k.gp.hi = __shfl_down_sync(0xffffffffu, m.k.gp.hi, d);
+  r.k.gp.lo = __shfl_down_sync(0xffffffffu, m.k.gp.lo, d);
+  r.k.ac.hi = __shfl_down_sync(0xffffffffu, m.k.ac.hi, d);
+  r.k.ac.lo = __shfl_down_sync(0xffffffffu, m.k.ac.lo, d);
+  r.k.gc.hi = __shfl_down_sync(0xffffffffu, m.k.gc.hi, d);
+  r.k.gc.lo = __shfl_down_sync(0xffffffffu, m.k.gc.lo, d);
   return r;
 }
 
@@ -225,6 +236,10 @@ __device__ void store_map(GMap *p, const GMap &m) {
   st_df(&p->cc, m.cc);
   __stcg(&p->v, m.v);
   __stcg(&p->p0, m.p0);
+  st_df(&p->k.ap, m.k.ap);
+  st_df(&p->k.gp, m.k.gp);
+  st_df(&p->k.ac, m.k.ac);
+  st_df(&p->k.gc, m.k.gc);
 }
 __device__ GMap load_map(const GMap *p) {
   GMap m;
@@ -236,6 +251,10 @@ __device__ GMap load_map(const GMap *p) {
   m.cc = ld_df(&p->cc);
   m.v = __ldcg(&p->v);
   m.p0 = __ldcg(&p->p0);
+  m.k.ap = ld_df(&p->k.ap);
+  m.k.gp = ld_df(&p->k.gp);
+  m.k.ac = ld_df(&p->k.ac);
+  m.k.gc = ld_df(&p->k.gc);
   return m;
 }
 __device__ void store_state(GState *p, const GState &s) {
@@ -354,36 +373,87 @@ __device__ GState look_back(const GaeArgs &a, int q, int lane) {
   }
 }
 
-// Loads 4 consecutive tokens (value, action bit) starting at t; tokens at or
-// beyond N read as observation tokens with value 0.
-__device__ __forceinline__ void load4(const GaeArgs &a, int64_t t, bool vec, float (&v)[4], uint32_t &act4) {
-  if (vec) {
-    const float4 x = __ldg(reinterpret_cast<const float4 *>(a.values + t));
-    const uint32_t w = __ldg(reinterpret_cast<const unsigned int *>(a.m + t));
-    v[0] = x.x;
-    v[1] = x.y;
-    v[2] = x.z;
-    v[3] = x.w;
-    act4 = ((w & 0xffu) != 0u) | (((w >> 8) & 0xffu) != 0u) << 1 | (((w >> 16) & 0xffu) != 0u) << 2 |
-           (((w >> 24) & 0xffu) != 0u) << 3;
-  } else {
-    act4 = 0;
+// Per-warp staging of a 1024-token chunk in shared memory: global memory is
+// read and written with fully coalesced 16-byte accesses, while each lane
+// works on its own run of 32 consecutive tokens. Rows are padded (33 floats,
+// 36 bytes) so lane-major reads hit 32 different banks.
+constexpr int kPadF = kItems + 1;
+constexpr int kPadB = kItems + 4;
+struct WarpStage {
+  float val[32][kPadF];   // values in, advantages out
+  float ret[32][kPadF];   // returns out
+  uint8_t msk[32][kPadB]; // action flags
+};
+
+__device__ __forceinline__ void stage_in(const GaeArgs &a, int64_t c0, int lane, WarpStage &ws) {
+  const int64_t N = a.N;
+  const bool full = c0 + kChunk <= N && aligned16_dev(a.values) && aligned16_dev(a.m);
+  if (full) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const bool in = t + i < a.N;
-      v[i] = in ? a.values[t + i] : 0.f;
-      act4 |= uint32_t(in && a.m[t + i] != 0) << i;
+    for (int it = 0; it < kChunk / 128; ++it) {
+      const int i = it * 128 + lane * 4;
+      const float4 x = __ldcs(reinterpret_cast<const float4 *>(a.values + c0 + i));
+      float *d = &ws.val[i / kItems][i % kItems];
+      d[0] = x.x;
+      d[1] = x.y;
+      d[2] = x.z;
+      d[3] = x.w;
+    }
+#pragma unroll
+    for (int it = 0; it < kChunk / 512; ++it) {
+      const int i = it * 512 + lane * 16;
+      const uint4 x = __ldcs(reinterpret_cast<const uint4 *>(a.m + c0 + i));
+      uint32_t *d = reinterpret_cast<uint32_t *>(&ws.msk[i / kItems][i % kItems]);
+      d[0] = x.x;
+      d[1] = x.y;
+      d[2] = x.z;
+      d[3] = x.w;
+    }
+  } else {
+    for (int i = lane; i < kChunk; i += 32) {
+      const int64_t t = c0 + i;
+      ws.val[i / kItems][i % kItems] = t < N ? a.values[t] : 0.f;
+      ws.msk[i / kItems][i % kItems] = (t < N && a.m[t] != 0) ? 1 : 0;
+    }
+  }
+  __syncwarp();
+}
+
+__device__ __forceinline__ void stage_out(const GaeArgs &a, int64_t c0, int lane, const WarpStage &ws) {
+  __syncwarp();
+  const int64_t N = a.N;
+  const bool full = c0 + kChunk <= N && aligned16_dev(a.adv) && aligned16_dev(a.ret);
+  if (full) {
+#pragma unroll
+    for (int it = 0; it < kChunk / 128; ++it) {
+      const int i = it * 128 + lane * 4;
+      const float *v = &ws.val[i / kItems][i % kItems];
+      const float *r = &ws.ret[i / kItems][i % kItems];
+      __stcs(reinterpret_cast<float4 *>(a.adv + c0 + i), make_float4(v[0], v[1], v[2], v[3]));
+      __stcs(reinterpret_cast<float4 *>(a.ret + c0 + i), make_float4(r[0], r[1], r[2], r[3]));
+    }
+  } else {
+    for (int i = lane; i < kChunk; i += 32) {
+      const int64_t t = c0 + i;
+      if (t < N) {
+        a.adv[t] = ws.val[i / kItems][i % kItems];
+        a.ret[t] = ws.ret[i / kItems][i % kItems];
+      }
     }
   }
 }
 
 template <bool kCrit>
-__global__ void __launch_bounds__(kThreads, 3) gae_scan_kernel(GaeArgs a) {
+__global__ void __launch_bounds__(kThreads, 4) gae_scan_kernel(GaeArgs a) {
   __shared__ int32_t s_cu_all[kWarps][kCuCap];
+  __shared__ WarpStage s_stage[kWarps];
+  __shared__ int s_ticket;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  int q = 0;
-  if (lane == 0) q = a.nchunks - 1 - atomicAdd(a.ticket, 1);
-  q = __shfl_sync(0xffffffffu, q, 0);
+  // One ticket per CTA: its warps take consecutive chunks, highest first, so
+  // every chunk a warp waits on belongs to a CTA (or a warp) already running.
+  if (threadIdx.x == 0) s_ticket = atomicAdd(a.ticket, kWarps);
+  __syncthreads();
+  const int q = a.nchunks - 1 - (s_ticket + warp);
   if (q < 0) return;  // the grid rounds the warp count up to whole CTAs
   const int64_t t0 = int64_t(q) * kChunk + int64_t(lane) * kItems;
   const int64_t N = a.N;
@@ -397,7 +467,10 @@ __global__ void __launch_bounds__(kThreads, 3) gae_scan_kernel(GaeArgs a) {
   if (cu.in_smem)
     for (int i = lane; i < ncu; i += 32) s_cu[i] = __ldg(a.cu + blo + i);
   __syncwarp();
-  const bool vec = (t0 + kItems <= N) && aligned16_dev(a.values) && aligned16_dev(a.m);
+  WarpStage &stg = s_stage[warp];
+  stage_in(a, int64_t(q) * kChunk, lane, stg);
+  const float *vrow = stg.val[lane];
+  const uint8_t *mrow = stg.msk[lane];
 
   // ---- trajectory ends among the 16 tokens (forward walk over cu_seqlens) -------
   uint32_t endbits = 0;
@@ -431,8 +504,12 @@ __global__ void __launch_bounds__(kThreads, 3) gae_scan_kernel(GaeArgs a) {
 #pragma unroll 1
     for (int g = kItems / 4 - 1; g >= 0; --g) {
       float v[4];
-      uint32_t act4;
-      load4(a, t0 + 4 * g, vec, v, act4);
+      uint32_t act4 = 0;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        v[i] = vrow[4 * g + i];
+        act4 |= uint32_t(mrow[4 * g + i] != 0) << i;
+      }
 #pragma unroll
       for (int i = 3; i >= 0; --i) {
         const int k = 4 * g + i;
@@ -481,6 +558,7 @@ __global__ void __launch_bounds__(kThreads, 3) gae_scan_kernel(GaeArgs a) {
         }
       }
     }
+    M.k = c;  // M.b, when the map is not the identity, is the trajectory of the leftmost token: b
   }
 
   // ---- suffix scan of the 32 maps of this warp ------------------------------------
@@ -520,26 +598,32 @@ __global__ void __launch_bounds__(kThreads, 3) gae_scan_kernel(GaeArgs a) {
     st_release(a.status + q, 2);
   }
 
-  // ---- replay the tokens from the incoming state, 4 at a time ---------------------
+  // ---- replay the tokens from the incoming state ----------------------------------
   GState st = apply<kCrit>(E, right, a.coef);
-  const bool vec_out = vec && aligned16_dev(a.adv) && aligned16_dev(a.ret);
   {
     int b = b_last;
     int64_t b_start = cu[b];
     TCoef c = load_coef(a.coef, b);
     float R = __ldg(a.rewards + b);
+    float *orow = stg.val[lane];
+    float *rrow = stg.ret[lane];
 #pragma unroll 1
     for (int g = kItems / 4 - 1; g >= 0; --g) {
       float v[4], ov[4], orr[4];
-      uint32_t act4;
-      load4(a, t0 + 4 * g, vec, v, act4);
+      uint32_t act4 = 0;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        v[i] = vrow[4 * g + i];
+        act4 |= uint32_t(mrow[4 * g + i] != 0) << i;
+      }
 #pragma unroll
       for (int i = 3; i >= 0; --i) {
         const int k = 4 * g + i;
         const int64_t t = t0 + k;
         ov[i] = 0.f;
         orr[i] = 0.f;
-        if (t < b_start && t < N) {
+        if (t >= N) continue;
+        if (t < b_start) {
           while (b > blo && t < b_start) {
             --b;
             b_start = cu[b];
@@ -565,20 +649,14 @@ __global__ void __launch_bounds__(kThreads, 3) gae_scan_kernel(GaeArgs a) {
           st.P = 0.f;
         }
       }
-      const int64_t tg = t0 + 4 * g;
-      if (vec_out) {
-        __stcs(reinterpret_cast<float4 *>(a.adv + tg), make_float4(ov[0], ov[1], ov[2], ov[3]));
-        __stcs(reinterpret_cast<float4 *>(a.ret + tg), make_float4(orr[0], orr[1], orr[2], orr[3]));
-      } else {
 #pragma unroll
-        for (int i = 0; i < 4; ++i)
-          if (tg + i < N) {
-            a.adv[tg + i] = ov[i];
-            a.ret[tg + i] = orr[i];
-          }
+      for (int i = 0; i < 4; ++i) {
+        orow[4 * g + i] = ov[i];
+        rrow[4 * g + i] = orr[i];
       }
     }
   }
+  stage_out(a, int64_t(q) * kChunk, lane, stg);
 }
 
 // Per-trajectory coefficients (fp64 then split to double-float) and a check of
@@ -636,7 +714,7 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   }
   if (alpha > 0.f) {
     int slot = launch_begin("gae_count", s);
-    seg::action_count_kernel<<<unsigned((nchunks + kWarps - 1) / kWarps), kThreads, 0, s>>>(m, cu, B, N, int(nchunks),
+    seg::action_count_kernel<<<unsigned((nchunks + 7) / 8), 256, 0, s>>>(m, cu, B, N, int(nchunks),
                                                                                     chunk_first, nact);
     SAO_TRY(launch_end(slot, s));
   }
