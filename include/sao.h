@@ -244,9 +244,9 @@ SAO_API sao_status sao_running_mean_advantages(const float *rewards, const int32
  * latency-critical caller cannot afford). The paper has no counterpart to
  * this entry point; it computes exactly what sao_advantages computes.
  *
- * Scratch: a fixed 8 MiB array inside this library's device image, present on
+ * Scratch: a fixed 16 MiB array inside this library's device image, present on
  * every GPU that loads the library until the process exits. It bounds the
- * sizes: about 120 bytes per 1024 tokens plus 36 bytes per trajectory must
+ * sizes: about 200 bytes per 1024 tokens plus 36 bytes per trajectory must
  * fit (for example 2^25 tokens with up to 65,536 trajectories); larger
  * inputs return SAO_ERR_SHAPE with the bytes needed. Nothing is allocated
  * and nothing is freed.

@@ -14,21 +14,30 @@
 //
 // The state carried right-to-left is S = (B_p, B_c, Vn, P): the two
 // lambda-returns of the next action token, its value, and the reward still
-// waiting for its action token. Each action token maps S affinely
+// waiting for its action token (P != 0 only in the state a trajectory end
+// leaves, where B = Vn = 0). Each action token maps S affinely
 // (B' = a B + g Vn + P, Vn' = V, P' = 0); the last token of a trajectory
 // resets S to (0, 0, 0, R_b). Maps compose associatively, so:
-//   * each thread folds its 32 tokens into one map,
-//   * a warp-shuffle suffix scan combines the 32 maps of a warp's 1024-token
-//     chunk,
-//   * warps chain their chunks right-to-left by decoupled look-back: each
-//     warp takes a ticket and works on chunk nchunks-1-ticket, so it only
-//     ever waits on chunks whose warps started before it; no CTA-wide barrier
-//     exists, so a waiting warp never holds up the others; the look-back
-//     inspects 32 predecessors at once and composes their maps in log depth;
-//     every wait is bounded and a time-out raises SAO_DEVERR_SCAN_TIMEOUT,
-//   * each thread then replays its tokens from its incoming state.
+//   * a warp owns a 1024-token chunk, each lane 32 consecutive tokens; the
+//     chunk is copied into shared memory with cp.async (16-byte granules,
+//     rows XOR-swizzled so that both the coalesced copies and the lane-major
+//     row reads are free of bank conflicts),
+//   * each lane folds its 32 tokens into one map, driven by two bit masks
+//     (action tokens, trajectory ends) so the common token costs one fused
+//     double-float a*B + g*V and no index arithmetic,
+//   * a warp-shuffle suffix scan combines the 32 maps of the chunk,
+//   * warps chain their chunks right-to-left by decoupled look-back: each CTA
+//     takes one ticket and its warps work on the chunks below it, so a warp
+//     only ever waits on chunks whose warps started before it; the look-back
+//     inspects 32 predecessors at once; maps and states are published as
+//     tagged 8-byte words, so neither side needs a fence; every wait is
+//     bounded and a time-out raises SAO_DEVERR_SCAN_TIMEOUT,
+//   * each lane then replays its tokens from its incoming state, writing A
+//     and the return into shared memory, and the warp stores both coalesced.
 // Traffic: values 4 B + mask 1 B read, adv 4 B + ret 4 B written per token.
 #include <stdint.h>
+
+#include <mutex>
 
 #include "sao_common.cuh"
 #include "sao_internal.h"
@@ -38,9 +47,11 @@ namespace sao {
 namespace {
 
 constexpr int kThreads = 128;
-constexpr int kItems = seg::kItems;       // tokens per lane (at most 32: one bit each)
-constexpr int kChunk = seg::kSegChunk;    // tokens per warp chunk
 constexpr int kWarps = kThreads / 32;
+constexpr int kMinBlocks = 4;             // 16 warps per SM (shared memory bound)
+constexpr int kItems = seg::kItems;       // tokens per lane (one bit each)
+constexpr int kChunk = seg::kSegChunk;    // tokens per warp chunk
+static_assert(kItems == 32 && kChunk == 1024, "the staging layout assumes 32 x 32 tokens per warp");
 
 // ---------------------------------------------------------------------------
 // double-float arithmetic (Dekker / Knuth error-free transformations)
@@ -61,10 +72,6 @@ __device__ __forceinline__ df df_add(df x, df y) {
   const df s = two_sum(x.hi, y.hi);
   return quick_two_sum(s.hi, __fadd_rn(s.lo, __fadd_rn(x.lo, y.lo)));
 }
-__device__ __forceinline__ df df_add_f(df x, float y) {
-  const df s = two_sum(x.hi, y);
-  return quick_two_sum(s.hi, __fadd_rn(s.lo, x.lo));
-}
 __device__ __forceinline__ df df_mul(df x, df y) {
   const float p = __fmul_rn(x.hi, y.hi);
   float e = __fmaf_rn(x.hi, y.hi, -p);
@@ -72,216 +79,265 @@ __device__ __forceinline__ df df_mul(df x, df y) {
   e = __fmaf_rn(x.lo, y.hi, e);
   return quick_two_sum(p, e);
 }
-__device__ __forceinline__ df df_mul_f(df x, float y) {
-  const float p = __fmul_rn(x.hi, y);
-  float e = __fmaf_rn(x.hi, y, -p);
-  e = __fmaf_rn(x.lo, y, e);
-  return quick_two_sum(p, e);
+// a*x + g*v for double-float a, x, g and a float v: both products split
+// exactly (FMA), their high parts added exactly (two-sum), the low-order terms
+// gathered in one float and renormalised once. a.lo*x.lo and g.lo*v's
+// rounding are below the format's precision.
+__device__ __forceinline__ df df_axpby(df a, df x, df g, float v) {
+  const float p1 = __fmul_rn(a.hi, x.hi);
+  const float e1 = __fmaf_rn(a.hi, x.hi, -p1);
+  const float p2 = __fmul_rn(g.hi, v);
+  const float e2 = __fmaf_rn(g.hi, v, -p2);
+  const df s = two_sum(p1, p2);
+  float lo = __fmaf_rn(a.hi, x.lo, e1);
+  lo = __fmaf_rn(a.lo, x.hi, lo);
+  lo = __fmaf_rn(g.lo, v, lo);
+  lo = __fadd_rn(lo, e2);
+  lo = __fadd_rn(lo, s.lo);
+  return quick_two_sum(s.hi, lo);
+}
+// x^e for 0 <= e < 32 by squaring.
+__device__ df df_pow(df x, int e) {
+  df r = {1.f, 0.f};
+  while (e) {
+    if (e & 1) r = df_mul(r, x);
+    e >>= 1;
+    if (e) x = df_mul(x, x);
+  }
+  return r;
 }
 __device__ __forceinline__ float df_round(df x) { return __fadd_rn(x.hi, x.lo); }
+// round(x - v) to float
+__device__ __forceinline__ float df_sub_round(df x, float v) {
+  const df s = two_sum(x.hi, -v);
+  return __fadd_rn(s.hi, __fadd_rn(s.lo, x.lo));
+}
 __device__ __forceinline__ df df_from_double(double x) {
   const float hi = float(x);
   return {hi, float(x - double(hi))};
 }
+__device__ __forceinline__ df df_shfl_down(df x, int d) {
+  return {__shfl_down_sync(0xffffffffu, x.hi, d), __shfl_down_sync(0xffffffffu, x.lo, d)};
+}
+__device__ __forceinline__ df df_shfl(df x, int src) {
+  return {__shfl_sync(0xffffffffu, x.hi, src), __shfl_sync(0xffffffffu, x.lo, src)};
+}
 
-// Per-trajectory coefficients: a = gamma*lambda and g = gamma - a for the
-// policy (lambda_b) and the critic (lambda_critic).
-struct TCoef {
-  df ap, gp, ac, gc;
+// Coefficients of one recursion: a = gamma*lambda and g = gamma - a.
+struct TC {
+  df a, g;
 };
-__device__ __forceinline__ TCoef load_coef(const float4 *tab, int b) {
-  const float4 u = __ldg(tab + 2 * b), w = __ldg(tab + 2 * b + 1);
-  return {{u.x, u.y}, {u.z, u.w}, {w.x, w.y}, {w.z, w.w}};
+// Per trajectory: the policy's (lambda_b) and, when the critic's recursion is
+// not trivial, the critic's (lambda_critic). Table layout: [B][2] float4.
+template <bool kCrit>
+struct Coefs {
+  TC p, c;
+};
+template <bool kCrit>
+__device__ __forceinline__ Coefs<kCrit> load_coefs(const float4 *tab, int b) {
+  Coefs<kCrit> k;
+  const float4 u = __ldg(tab + 2 * b);
+  k.p = {{u.x, u.y}, {u.z, u.w}};
+  if constexpr (kCrit) {
+    const float4 w = __ldg(tab + 2 * b + 1);
+    k.c = {{w.x, w.y}, {w.z, w.w}};
+  }
+  return k;
 }
 
 // The affine map of a token segment, from the state at its right edge to the
 // state at its left edge. fl bit 0: the segment holds the last token of a
-// trajectory (the map ignores the incoming state); bit 1: the segment (left of
-// any reset) holds an action token. Identity when fl == 0.
-//   reset:          B = c,                        Vn = act ? v : 0, P = act ? 0 : p0
-//   act, no reset:  B = ap (a B + g Vn + P) + c,  Vn = v,           P = 0
-// b is the trajectory of the segment's leftmost token.
-struct GMap {
-  int b, fl;
-  df ap, cp, ac, cc;
-  float v, p0;
-  TCoef k;  // coefficients of trajectory b (used when the map is the left operand)
+// trajectory (the map ignores the incoming state); bit 1: the segment, left of
+// any such end, holds an action token. Identity when fl == 0.
+//   fl 1 (end, no action after it):  S' = (0, 0, 0, vp)          vp = reward waiting
+//   fl 3 (end, then actions):         S' = (cp, cc, vp, 0)        vp = leftmost action value
+//   fl 2 (actions, no end):           B' = ap (a B + g Vn + P) + cp,  Vn' = vp,  P' = 0
+// with (a, g) = kp, the coefficients of the segment's trajectory.
+template <bool kCrit>
+struct CritMap {
+  df ac, cc;
+  TC kc;
+};
+template <>
+struct CritMap<false> {};
+template <bool kCrit>
+struct GMap : CritMap<kCrit> {
+  int fl;
+  float vp;
+  df ap, cp;
+  TC kp;
 };
 struct GState {
   df Bp, Bc;
   float Vn, P;
 };
 
-__device__ __forceinline__ GMap identity_map() {
-  GMap m;
-  m.b = 0;
+template <bool kCrit>
+__device__ __forceinline__ GMap<kCrit> identity_map() {
+  GMap<kCrit> m;
   m.fl = 0;
-  m.ap = m.ac = {1.f, 0.f};
-  m.cp = m.cc = {0.f, 0.f};
-  m.v = m.p0 = 0.f;
-  m.k = TCoef{};
+  m.vp = 0.f;
+  m.ap = m.cp = {0.f, 0.f};
+  m.kp = {{0.f, 0.f}, {0.f, 0.f}};
+  if constexpr (kCrit) {
+    m.ac = m.cc = {0.f, 0.f};
+    m.kc = {{0.f, 0.f}, {0.f, 0.f}};
+  }
   return m;
+}
+__device__ __forceinline__ GState zero_state() {
+  GState s;
+  s.Bp = s.Bc = {0.f, 0.f};
+  s.Vn = s.P = 0.f;
+  return s;
+}
+
+// One action token's update of a lambda-return: a B + g Vn, or the waiting
+// reward right after a trajectory end (where B = Vn = 0).
+__device__ __forceinline__ df step_return(const TC &k, df B, float Vn, float P) {
+  const df n = df_axpby(k.a, B, k.g, Vn);
+  return P != 0.f ? df{P, 0.f} : n;
 }
 
 // x o y: x is the left segment, y the one immediately to its right.
 template <bool kCrit>
-__device__ GMap compose(const GMap &x, const GMap &y, const float4 *) {
+__device__ GMap<kCrit> compose(const GMap<kCrit> &x, const GMap<kCrit> &y) {
   if (x.fl & 1) return x;
   if (!(x.fl & 2)) return y;
   if (!(y.fl & 3)) return x;
-  const TCoef &c = x.k;
   const bool yact = (y.fl & 2) != 0;
-  const float Yv = yact ? y.v : 0.f, Yp = yact ? 0.f : y.p0;
-  GMap r;
-  r.b = x.b;
-  r.k = x.k;
-  r.v = x.v;
-  r.p0 = 0.f;
-  df tp = df_add_f(df_add(df_mul(c.ap, y.cp), df_mul_f(c.gp, Yv)), Yp);
-  r.cp = df_add(df_mul(x.ap, tp), x.cp);
-  if (kCrit) {
-    df tc = df_add_f(df_add(df_mul(c.ac, y.cc), df_mul_f(c.gc, Yv)), Yp);
-    r.cc = df_add(df_mul(x.ac, tc), x.cc);
-  } else {
-    r.cc = {0.f, 0.f};
-  }
+  const float Yv = yact ? y.vp : 0.f, Yp = yact ? 0.f : y.vp;
+  GMap<kCrit> r = x;
+  r.cp = df_add(df_mul(x.ap, step_return(x.kp, y.cp, Yv, Yp)), x.cp);
+  if constexpr (kCrit) r.cc = df_add(df_mul(x.ac, step_return(x.kc, y.cc, Yv, Yp)), x.cc);
   if (y.fl & 1) {
     r.fl = 3;
-    r.ap = r.ac = {0.f, 0.f};
-  } else {
-    r.fl = 2;
-    r.ap = df_mul(df_mul(x.ap, c.ap), y.ap);
-    r.ac = kCrit ? df_mul(df_mul(x.ac, c.ac), y.ac) : df{1.f, 0.f};
+    r.ap = {0.f, 0.f};
+    if constexpr (kCrit) r.ac = {0.f, 0.f};
+  } else {  // same trajectory on both sides
+    r.ap = df_mul(df_mul(x.ap, x.kp.a), y.ap);
+    if constexpr (kCrit) r.ac = df_mul(df_mul(x.ac, x.kc.a), y.ac);
   }
   return r;
 }
 
 template <bool kCrit>
-__device__ GState apply(const GMap &m, const GState &s, const float4 *) {
+__device__ GState apply(const GMap<kCrit> &m, const GState &s) {
+  GState r = zero_state();
   if (m.fl & 1) {
     const bool act = (m.fl & 2) != 0;
-    return {m.cp, m.cc, act ? m.v : 0.f, act ? 0.f : m.p0};
+    r.Bp = m.cp;
+    if constexpr (kCrit) r.Bc = m.cc;
+    r.Vn = act ? m.vp : 0.f;
+    r.P = act ? 0.f : m.vp;
+    return r;
   }
   if (!(m.fl & 2)) return s;
-  const TCoef &c = m.k;
-  GState r;
-  const df tp = df_add_f(df_add(df_mul(c.ap, s.Bp), df_mul_f(c.gp, s.Vn)), s.P);
-  r.Bp = df_add(df_mul(m.ap, tp), m.cp);
-  if (kCrit) {
-    const df tc = df_add_f(df_add(df_mul(c.ac, s.Bc), df_mul_f(c.gc, s.Vn)), s.P);
-    r.Bc = df_add(df_mul(m.ac, tc), m.cc);
-  } else {
-    r.Bc = {0.f, 0.f};
-  }
-  r.Vn = m.v;
-  r.P = 0.f;
+  r.Bp = df_add(df_mul(m.ap, step_return(m.kp, s.Bp, s.Vn, s.P)), m.cp);
+  if constexpr (kCrit) r.Bc = df_add(df_mul(m.ac, step_return(m.kc, s.Bc, s.Vn, s.P)), m.cc);
+  r.Vn = m.vp;
   return r;
 }
 
-__device__ __forceinline__ GMap shfl_down_map(const GMap &m, int d) {
-  GMap r;
-  r.b = __shfl_down_sync(0xffffffffu, m.b, d);
+template <bool kCrit>
+__device__ __forceinline__ GMap<kCrit> shfl_down_map(const GMap<kCrit> &m, int d) {
+  GMap<kCrit> r;
   r.fl = __shfl_down_sync(0xffffffffu, m.fl, d);
-  r.ap.hi = __shfl_down_sync(0xffffffffu, m.ap.hi, d);
-  r.ap.lo = __shfl_down_sync(0xffffffffu, m.ap.lo, d);
-  r.cp.hi = __shfl_down_sync(0xffffffffu, m.cp.hi, d);
-  r.cp.lo = __shfl_down_sync(0xffffffffu, m.cp.lo, d);
-  r.ac.hi = __shfl_down_sync(0xffffffffu, m.ac.hi, d);
-  r.ac.lo = __shfl_down_sync(0xffffffffu, m.ac.lo, d);
-  r.cc.hi = __shfl_down_sync(0xffffffffu, m.cc.hi, d);
-  r.cc.lo = __shfl_down_sync(0xffffffffu, m.cc.lo, d);
-  r.v = __shfl_down_sync(0xffffffffu, m.v, d);
-  r.p0 = __shfl_down_sync(0xffffffffu, m.p0, d);
-  r.k.ap.hi = __shfl_down_sync(0xffffffffu, m.k.ap.hi, d);
-  r.k.ap.lo = __shfl_down_sync(0xffffffffu, m.k.ap.lo, d);
-  r.k.gp.hi = __shfl_down_sync(0xffffffffu, m.k.gp.hi, d);
-  r.k.gp.lo = __shfl_down_sync(0xffffffffu, m.k.gp.lo, d);
-  r.k.ac.hi = __shfl_down_sync(0xffffffffu, m.k.ac.hi, d);
-  r.k.ac.lo = __shfl_down_sync(0xffffffffu, m.k.ac.lo, d);
-  r.k.gc.hi = __shfl_down_sync(0xffffffffu, m.k.gc.hi, d);
-  r.k.gc.lo = __shfl_down_sync(0xffffffffu, m.k.gc.lo, d);
+  r.vp = __shfl_down_sync(0xffffffffu, m.vp, d);
+  r.ap = df_shfl_down(m.ap, d);
+  r.cp = df_shfl_down(m.cp, d);
+  r.kp.a = df_shfl_down(m.kp.a, d);
+  r.kp.g = df_shfl_down(m.kp.g, d);
+  if constexpr (kCrit) {
+    r.ac = df_shfl_down(m.ac, d);
+    r.cc = df_shfl_down(m.cc, d);
+    r.kc.a = df_shfl_down(m.kc.a, d);
+    r.kc.g = df_shfl_down(m.kc.g, d);
+  }
+  return r;
+}
+__device__ __forceinline__ GState shfl_state(const GState &s, int src) {
+  GState r;
+  r.Bp = df_shfl(s.Bp, src);
+  r.Bc = df_shfl(s.Bc, src);
+  r.Vn = __shfl_sync(0xffffffffu, s.Vn, src);
+  r.P = __shfl_sync(0xffffffffu, s.P, src);
   return r;
 }
 
 // ---------------------------------------------------------------------------
-// cross-CTA publication (decoupled look-back)
+// cross-warp publication (decoupled look-back)
 // ---------------------------------------------------------------------------
-struct __align__(16) ChunkPub {
-  GMap agg;     // map of the whole chunk (status >= 1)
-  GState incl;  // state at the chunk's left edge (status == 2)
-};
+// Every published field is one naturally aligned 8-byte word: the field's 32
+// bits and a tag (1) in the high half. An 8-byte access is single-copy atomic,
+// so a reader that sees the tags of all words of a record has read the whole
+// record, with no fence on either side and no separate status word: a poll is
+// one round trip to L2. The arrays are zeroed before the scan, so an unwritten
+// word reads as untagged.
+constexpr uint64_t kTag = uint64_t(1) << 32;
+template <bool kCrit>
+constexpr int kMapWords = kCrit ? 18 : 10;  // GMap fields
+template <bool kCrit>
+constexpr int kStateWords = kCrit ? 6 : 4;  // GState fields
 
-__device__ __forceinline__ int ld_acquire(const int *p) {
-  int v;
-  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
+__device__ __forceinline__ void st_pair(uint64_t *p, float x, float y) {
+  const uint64_t u = kTag | __float_as_uint(x), v = kTag | __float_as_uint(y);
+  asm volatile("st.relaxed.gpu.global.v2.b64 [%0], {%1, %2};" ::"l"(p), "l"(u), "l"(v) : "memory");
 }
-__device__ __forceinline__ void st_release(int *p, int v) {
-  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+// True when both words carry the tag.
+__device__ __forceinline__ bool ld_pair(const uint64_t *p, float &x, float &y) {
+  uint64_t u, v;
+  asm volatile("ld.relaxed.gpu.global.v2.b64 {%0, %1}, [%2];" : "=l"(u), "=l"(v) : "l"(p) : "memory");
+  x = __uint_as_float(uint32_t(u));
+  y = __uint_as_float(uint32_t(v));
+  return ((u & v) >> 32) != 0;
 }
+__device__ __forceinline__ bool ld_pair(const uint64_t *p, df &x) { return ld_pair(p, x.hi, x.lo); }
 
-// Published maps and states go through L2 only (st.cg / ld.cg), so a reader on
-// another SM never sees a stale L1 line.
-__device__ __forceinline__ void st_df(df *p, df x) {
-  __stcg(&p->hi, x.hi);
-  __stcg(&p->lo, x.lo);
-}
-__device__ __forceinline__ df ld_df(const df *p) { return {__ldcg(&p->hi), __ldcg(&p->lo)}; }
-__device__ void store_map(GMap *p, const GMap &m) {
-  __stcg(&p->b, m.b);
-  __stcg(&p->fl, m.fl);
-  st_df(&p->ap, m.ap);
-  st_df(&p->cp, m.cp);
-  st_df(&p->ac, m.ac);
-  st_df(&p->cc, m.cc);
-  __stcg(&p->v, m.v);
-  __stcg(&p->p0, m.p0);
-  st_df(&p->k.ap, m.k.ap);
-  st_df(&p->k.gp, m.k.gp);
-  st_df(&p->k.ac, m.k.ac);
-  st_df(&p->k.gc, m.k.gc);
-}
-__device__ GMap load_map(const GMap *p) {
-  GMap m;
-  m.b = __ldcg(&p->b);
-  m.fl = __ldcg(&p->fl);
-  m.ap = ld_df(&p->ap);
-  m.cp = ld_df(&p->cp);
-  m.ac = ld_df(&p->ac);
-  m.cc = ld_df(&p->cc);
-  m.v = __ldcg(&p->v);
-  m.p0 = __ldcg(&p->p0);
-  m.k.ap = ld_df(&p->k.ap);
-  m.k.gp = ld_df(&p->k.gp);
-  m.k.ac = ld_df(&p->k.ac);
-  m.k.gc = ld_df(&p->k.gc);
-  return m;
-}
-__device__ void store_state(GState *p, const GState &s) {
-  st_df(&p->Bp, s.Bp);
-  st_df(&p->Bc, s.Bc);
-  __stcg(&p->Vn, s.Vn);
-  __stcg(&p->P, s.P);
-}
-__device__ GState load_state(const GState *p) {
-  GState s;
-  s.Bp = ld_df(&p->Bp);
-  s.Bc = ld_df(&p->Bc);
-  s.Vn = __ldcg(&p->Vn);
-  s.P = __ldcg(&p->P);
-  return s;
-}
-
-// Waits until *p != 0; returns it, or 0 after kWaitLimitNs / kSpinLimit polls.
-__device__ int wait_nonzero(const int *p) {
-  const uint64_t t0 = globaltimer_ns();
-  for (uint32_t n = 0; n < kSpinLimit; ++n) {
-    const int s = ld_acquire(p);
-    if (s != 0) return s;
-    if ((n & 63u) == 63u && globaltimer_ns() - t0 > kWaitLimitNs) return 0;
-    __nanosleep(64);
+template <bool kCrit>
+__device__ void publish_map(uint64_t *p, const GMap<kCrit> &m) {
+  st_pair(p + 0, __int_as_float(m.fl), m.vp);
+  st_pair(p + 2, m.ap.hi, m.ap.lo);
+  st_pair(p + 4, m.cp.hi, m.cp.lo);
+  st_pair(p + 6, m.kp.a.hi, m.kp.a.lo);
+  st_pair(p + 8, m.kp.g.hi, m.kp.g.lo);
+  if constexpr (kCrit) {
+    st_pair(p + 10, m.ac.hi, m.ac.lo);
+    st_pair(p + 12, m.cc.hi, m.cc.lo);
+    st_pair(p + 14, m.kc.a.hi, m.kc.a.lo);
+    st_pair(p + 16, m.kc.g.hi, m.kc.g.lo);
   }
-  return 0;
+}
+template <bool kCrit>
+__device__ bool fetch_map(const uint64_t *p, GMap<kCrit> &m) {
+  float f;
+  bool ok = ld_pair(p + 0, f, m.vp);
+  m.fl = __float_as_int(f);
+  ok &= ld_pair(p + 2, m.ap);
+  ok &= ld_pair(p + 4, m.cp);
+  ok &= ld_pair(p + 6, m.kp.a);
+  ok &= ld_pair(p + 8, m.kp.g);
+  if constexpr (kCrit) {
+    ok &= ld_pair(p + 10, m.ac);
+    ok &= ld_pair(p + 12, m.cc);
+    ok &= ld_pair(p + 14, m.kc.a);
+    ok &= ld_pair(p + 16, m.kc.g);
+  }
+  return ok;
+}
+template <bool kCrit>
+__device__ void publish_state(uint64_t *p, const GState &s) {
+  st_pair(p + 0, s.Bp.hi, s.Bp.lo);
+  st_pair(p + 2, s.Vn, s.P);
+  if constexpr (kCrit) st_pair(p + 4, s.Bc.hi, s.Bc.lo);
+}
+template <bool kCrit>
+__device__ bool fetch_state(const uint64_t *p, GState &s) {
+  bool ok = ld_pair(p + 0, s.Bp);
+  ok &= ld_pair(p + 2, s.Vn, s.P);
+  if constexpr (kCrit) ok &= ld_pair(p + 4, s.Bc);
+  else s.Bc = {0.f, 0.f};
+  return ok;
 }
 
 struct GaeArgs {
@@ -291,372 +347,461 @@ struct GaeArgs {
   int B;
   int64_t N;
   int nchunks;
-  const float4 *coef;  // [B][2]
+  const float4 *coef;      // [B][2]
   const int *chunk_first;  // [nchunks] trajectory of each chunk's first token
   int *ticket;
-  int *status;         // [nchunks]
-  ChunkPub *pub;       // [nchunks]
+  uint64_t *agg;           // [nchunks][kMapWords]: map of the whole chunk
+  uint64_t *incl;          // [nchunks][kStateWords]: state at the chunk's left edge
   float *adv, *ret;
   unsigned int *err;
 };
 
 using seg::CuView;
-using seg::find_traj;
 using seg::kCuCap;
 
+// A look-back round whose first known chunk is at most this many chunks away
+// applies the maps one by one instead of composing them in log depth.
+constexpr int kSerialWalk = 6;
+
 // State at the right edge of chunk q, from the chunks to its right. The warp
-// inspects 32 successors (q+1 .. q+32) per round: each lane polls one status
-// word; the first chunk whose left-edge state is known (published inclusive
-// state, a map that ignores its right neighbour, or the end of the input) ends
-// the walk, and the maps of the chunks before it are composed by a log-depth
-// shuffle scan. A round waits (bounded) only for chunks before that point.
+// inspects 32 successors (q+1 .. q+32) per round: each lane polls one chunk's
+// published state and map; the first chunk whose left-edge state is known
+// (published state, a map that ignores its right neighbour, or the end of the
+// input) ends the walk, and the maps of the chunks before it are applied one
+// by one when there are few of them, else composed by a log-depth shuffle
+// scan. A round waits (bounded) only for chunks before that point.
 template <bool kCrit>
 __device__ GState look_back(const GaeArgs &a, int q, int lane) {
-  GState zero;
-  zero.Bp = zero.Bc = {0.f, 0.f};
-  zero.Vn = zero.P = 0.f;
-  GMap acc = identity_map();  // maps of the chunks already walked (lane 0)
+  GMap<kCrit> acc = identity_map<kCrit>();  // maps of the chunks already walked (lane 0)
   const uint64_t t_start = globaltimer_ns();
   for (int base = q + 1;; base += 32) {
     const int j = base + lane;
-    int st = 0;
-    GMap mj = identity_map();
-    bool term = false;
+    GMap<kCrit> mj = identity_map<kCrit>();
+    GState sj = zero_state();
+    int kind = 2;  // 0: nothing published yet, 1: map, 2: left-edge state known
     uint32_t polls = 0;
     for (;;) {
-      st = j < a.nchunks ? ld_acquire(a.status + j) : 2;
-      term = (st == 2);
-      if (st == 1) {
-        mj = load_map(&a.pub[j].agg);
-        term = (mj.fl & 1) != 0;
+      if (j < a.nchunks) {
+        const bool has_s = fetch_state<kCrit>(a.incl + size_t(j) * kStateWords<kCrit>, sj);
+        const bool has_m = fetch_map<kCrit>(a.agg + size_t(j) * kMapWords<kCrit>, mj);
+        kind = has_s ? 2 : (has_m ? 1 : 0);
+        if (kind == 1 && (mj.fl & 1)) {  // the map ignores its right neighbour
+          sj = apply<kCrit>(mj, zero_state());
+          kind = 2;
+        }
       }
-      const unsigned bt = __ballot_sync(0xffffffffu, term);
-      const unsigned bn = __ballot_sync(0xffffffffu, st == 0);
+      const unsigned bt = __ballot_sync(0xffffffffu, kind == 2);
+      const unsigned bn = __ballot_sync(0xffffffffu, kind == 0);
       const int first_term = bt ? __ffs(bt) - 1 : 32;
       const int first_nr = bn ? __ffs(bn) - 1 : 32;
       if (first_nr >= first_term) break;  // everything up to the first terminal chunk is known
       if ((++polls & 31u) == 0u && globaltimer_ns() - t_start > kWaitLimitNs) {
         if (lane == 0) raise_device_error(a.err, SAO_DEVERR_SCAN_TIMEOUT);
-        return zero;
+        return zero_state();
       }
-      __nanosleep(128);
+      __nanosleep(64);
     }
-    const unsigned bt = __ballot_sync(0xffffffffu, term);
+    const unsigned bt = __ballot_sync(0xffffffffu, kind == 2);
     const int stop = bt ? __ffs(bt) - 1 : 32;
-    // state at the left edge of the terminal chunk (if any in this round)
-    GState tstate = zero;
-    if (lane == stop && j < a.nchunks) tstate = (st == 2) ? load_state(&a.pub[j].incl) : apply<kCrit>(mj, zero, a.coef);
+    if (stop <= kSerialWalk) {
+      // near terminal: carry its state through the maps of lanes stop-1 .. 0
+      GState cur = shfl_state(sj, stop);
+      for (int i = stop - 1; i >= 0; --i) cur = shfl_state(apply<kCrit>(mj, cur), i);
+      return shfl_state(apply<kCrit>(acc, cur), 0);  // acc is meaningful in lane 0
+    }
     // compose maps of lanes [0, stop): suffix scan, lane 0 ends with m_0 o ... o m_{stop-1}
-    GMap m = lane < stop ? mj : identity_map();
+    GMap<kCrit> m = lane < stop ? mj : identity_map<kCrit>();
 #pragma unroll 1
     for (int d = 1; d < 32; d <<= 1) {
-      const GMap o = shfl_down_map(m, d);
-      if (lane + d < 32) m = compose<kCrit>(m, o, a.coef);
+      const GMap<kCrit> o = shfl_down_map<kCrit>(m, d);
+      if (lane + d < 32) m = compose<kCrit>(m, o);
     }
-    if (lane == 0) acc = compose<kCrit>(acc, m, a.coef);
+    if (lane == 0) acc = compose<kCrit>(acc, m);
     if (stop < 32) {
-      tstate.Bp.hi = __shfl_sync(0xffffffffu, tstate.Bp.hi, stop);
-      tstate.Bp.lo = __shfl_sync(0xffffffffu, tstate.Bp.lo, stop);
-      tstate.Bc.hi = __shfl_sync(0xffffffffu, tstate.Bc.hi, stop);
-      tstate.Bc.lo = __shfl_sync(0xffffffffu, tstate.Bc.lo, stop);
-      tstate.Vn = __shfl_sync(0xffffffffu, tstate.Vn, stop);
-      tstate.P = __shfl_sync(0xffffffffu, tstate.P, stop);
-      GState r = apply<kCrit>(acc, tstate, a.coef);  // meaningful in lane 0
-      r.Bp.hi = __shfl_sync(0xffffffffu, r.Bp.hi, 0);
-      r.Bp.lo = __shfl_sync(0xffffffffu, r.Bp.lo, 0);
-      r.Bc.hi = __shfl_sync(0xffffffffu, r.Bc.hi, 0);
-      r.Bc.lo = __shfl_sync(0xffffffffu, r.Bc.lo, 0);
-      r.Vn = __shfl_sync(0xffffffffu, r.Vn, 0);
-      r.P = __shfl_sync(0xffffffffu, r.P, 0);
-      return r;
+      const GState tstate = shfl_state(sj, stop);
+      return shfl_state(apply<kCrit>(acc, tstate), 0);  // meaningful in lane 0
     }
   }
 }
 
-// Per-warp staging of a 1024-token chunk in shared memory: global memory is
-// read and written with fully coalesced 16-byte accesses, while each lane
-// works on its own run of 32 consecutive tokens. Rows are padded (33 floats,
-// 36 bytes) so lane-major reads hit 32 different banks.
-constexpr int kPadF = kItems + 1;
-constexpr int kPadB = kItems + 4;
-struct WarpStage {
-  float val[32][kPadF];   // values in, advantages out
-  float ret[32][kPadF];   // returns out
-  uint8_t msk[32][kPadB]; // action flags
+// ---------------------------------------------------------------------------
+// per-warp staging in shared memory
+// ---------------------------------------------------------------------------
+// Row r holds lane r's 32 tokens. val/ret rows are 8 granules of 16 bytes,
+// granule j stored at 8r + (j ^ (r & 7)); msk rows are 2 granules, granule j
+// at 2r + (j ^ ((r >> 2) & 1)). A quarter-warp (8 lanes) then touches 8
+// distinct bank groups both when it copies 8 consecutive granules of the chunk
+// and when 8 lanes read the same granule of their own rows.
+// A warp keeps two chunks: the one it folds and the one waiting for its
+// look-back; values arrive in val[buf] and leave as advantages.
+struct __align__(16) WarpBuf {
+  float val[2][kChunk];  // values in, advantages out
+  float ret[kChunk];     // returns of the chunk being replayed
+  uint8_t msk[kChunk];   // action flags of the chunk being folded
+  int32_t cu[kCuCap];    // cu_seqlens slice of the chunk being folded
 };
+__device__ __forceinline__ int fgran(int r, int j) { return 8 * r + (j ^ (r & 7)); }
+__device__ __forceinline__ int mgran(int r, int j) { return 2 * r + (j ^ ((r >> 2) & 1)); }
 
-__device__ __forceinline__ void stage_in(const GaeArgs &a, int64_t c0, int lane, WarpStage &ws) {
+__device__ __forceinline__ void cp_async16(void *smem, const void *gmem) {
+  const unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(s), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
+// Starts the copy of the chunk's values and flags (asynchronous for a full,
+// aligned chunk; element by element, zero-filled past N, otherwise).
+__device__ __forceinline__ void stage_in(const GaeArgs &a, int64_t c0, int lane, float *val, uint8_t *msk) {
   const int64_t N = a.N;
-  const bool full = c0 + kChunk <= N && aligned16_dev(a.values) && aligned16_dev(a.m);
-  if (full) {
+  if (c0 + kChunk <= N && aligned16_dev(a.values) && aligned16_dev(a.m)) {
 #pragma unroll
-    for (int it = 0; it < kChunk / 128; ++it) {
-      const int i = it * 128 + lane * 4;
-      const float4 x = __ldcs(reinterpret_cast<const float4 *>(a.values + c0 + i));
-      float *d = &ws.val[i / kItems][i % kItems];
-      d[0] = x.x;
-      d[1] = x.y;
-      d[2] = x.z;
-      d[3] = x.w;
+    for (int it = 0; it < 8; ++it) {
+      const int G = it * 32 + lane;
+      cp_async16(&val[4 * fgran(G >> 3, G & 7)], a.values + c0 + 4 * G);
     }
 #pragma unroll
-    for (int it = 0; it < kChunk / 512; ++it) {
-      const int i = it * 512 + lane * 16;
-      const uint4 x = __ldcs(reinterpret_cast<const uint4 *>(a.m + c0 + i));
-      uint32_t *d = reinterpret_cast<uint32_t *>(&ws.msk[i / kItems][i % kItems]);
-      d[0] = x.x;
-      d[1] = x.y;
-      d[2] = x.z;
-      d[3] = x.w;
+    for (int it = 0; it < 2; ++it) {
+      const int G = it * 32 + lane;
+      cp_async16(&msk[16 * mgran(G >> 1, G & 1)], a.m + c0 + 16 * G);
     }
   } else {
     for (int i = lane; i < kChunk; i += 32) {
       const int64_t t = c0 + i;
-      ws.val[i / kItems][i % kItems] = t < N ? a.values[t] : 0.f;
-      ws.msk[i / kItems][i % kItems] = (t < N && a.m[t] != 0) ? 1 : 0;
+      const int r = i >> 5, k = i & 31;
+      val[4 * fgran(r, k >> 2) + (k & 3)] = t < N ? a.values[t] : 0.f;
+      msk[16 * mgran(r, k >> 4) + (k & 15)] = (t < N && a.m[t] != 0) ? 1 : 0;
     }
   }
-  __syncwarp();
 }
 
-__device__ __forceinline__ void stage_out(const GaeArgs &a, int64_t c0, int lane, const WarpStage &ws) {
-  __syncwarp();
+__device__ __forceinline__ void stage_out(const GaeArgs &a, int64_t c0, int lane, const float *val,
+                                          const float *ret) {
   const int64_t N = a.N;
-  const bool full = c0 + kChunk <= N && aligned16_dev(a.adv) && aligned16_dev(a.ret);
-  if (full) {
+  if (c0 + kChunk <= N && aligned16_dev(a.adv) && aligned16_dev(a.ret)) {
 #pragma unroll
-    for (int it = 0; it < kChunk / 128; ++it) {
-      const int i = it * 128 + lane * 4;
-      const float *v = &ws.val[i / kItems][i % kItems];
-      const float *r = &ws.ret[i / kItems][i % kItems];
-      __stcs(reinterpret_cast<float4 *>(a.adv + c0 + i), make_float4(v[0], v[1], v[2], v[3]));
-      __stcs(reinterpret_cast<float4 *>(a.ret + c0 + i), make_float4(r[0], r[1], r[2], r[3]));
+    for (int it = 0; it < 8; ++it) {
+      const int G = it * 32 + lane;
+      const int p = 4 * fgran(G >> 3, G & 7);
+      __stcs(reinterpret_cast<float4 *>(a.adv + c0) + G, *reinterpret_cast<const float4 *>(&val[p]));
+      __stcs(reinterpret_cast<float4 *>(a.ret + c0) + G, *reinterpret_cast<const float4 *>(&ret[p]));
     }
   } else {
     for (int i = lane; i < kChunk; i += 32) {
       const int64_t t = c0 + i;
+      const int r = i >> 5, k = i & 31;
       if (t < N) {
-        a.adv[t] = ws.val[i / kItems][i % kItems];
-        a.ret[t] = ws.ret[i / kItems][i % kItems];
+        a.adv[t] = val[4 * fgran(r, k >> 2) + (k & 3)];
+        a.ret[t] = ret[4 * fgran(r, k >> 2) + (k & 3)];
       }
     }
   }
 }
 
+// Bit i set when byte i of x is non-zero (i = 0..3).
+__device__ __forceinline__ uint32_t nonzero_bytes(uint32_t x) {
+  const uint32_t h = (((x & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | x) & 0x80808080u;
+  return (h * 0x00204081u) >> 28;
+}
+
+// ---------------------------------------------------------------------------
+// per-lane fold and replay
+// ---------------------------------------------------------------------------
+// The lane's tokens are t0 .. t0+31; bit k of `act` / `ends`: token t0+k is an
+// action token / the last token of its trajectory; b_last is the trajectory of
+// the lane's last token below N.
+
+// Map of the lane's 32 tokens. kEnds: some lane of the warp holds a trajectory
+// end (the warp-uniform choice between the general loop and the branch-free
+// one for runs inside a single trajectory).
+template <bool kCrit, bool kEnds>
+__device__ GMap<kCrit> fold_lane(const GaeArgs &a, const float *val, int lane, uint32_t act, uint32_t ends,
+                                 int64_t t0, const CuView &cu, int blo, int b_last) {
+  Coefs<kCrit> k = load_coefs<kCrit>(a.coef, b_last);
+  df Bp = {0.f, 0.f}, Bc = {0.f, 0.f};
+  float Vn = 0.f, P = 0.f;
+  int fl = 0, n = 0;
+  const int sw = lane & 7;
+  if constexpr (!kEnds) {
+#pragma unroll 1
+    for (int g = 7; g >= 0; --g) {
+      const float4 v4 = *reinterpret_cast<const float4 *>(&val[4 * (8 * lane + (g ^ sw))]);
+      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
+      const uint32_t a4 = (act >> (4 * g)) & 15u;
+#pragma unroll
+      for (int i = 3; i >= 0; --i) {
+        const bool on = (a4 >> i) & 1u;
+        const df np = df_axpby(k.p.a, Bp, k.p.g, Vn);
+        Bp = on ? np : Bp;
+        if constexpr (kCrit) {
+          const df nc = df_axpby(k.c.a, Bc, k.c.g, Vn);
+          Bc = on ? nc : Bc;
+        }
+        Vn = on ? vv[i] : Vn;
+      }
+      n += __popc(a4);
+    }
+    fl = n > 0 ? 2 : 0;
+  } else {
+#pragma unroll 1
+  for (int g = 7; g >= 0; --g) {
+    const float4 v4 = *reinterpret_cast<const float4 *>(&val[4 * (8 * lane + (g ^ sw))]);
+    const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
+    const uint32_t a4 = act >> (4 * g), e4 = ends >> (4 * g);
+#pragma unroll
+    for (int i = 3; i >= 0; --i) {
+      if ((e4 >> i) & 1u) {  // last token of a trajectory: reset
+        const int b = cu.find(blo, b_last, t0 + 4 * g + i);
+        k = load_coefs<kCrit>(a.coef, b);
+        P = __ldg(a.rewards + b);
+        Bp = Bc = {0.f, 0.f};
+        Vn = 0.f;
+        fl = 1;
+      }
+      if ((a4 >> i) & 1u) {
+        Bp = step_return(k.p, Bp, Vn, P);
+        if constexpr (kCrit) Bc = step_return(k.c, Bc, Vn, P);
+        Vn = vv[i];
+        P = 0.f;
+        fl |= 2;
+        ++n;
+      }
+    }
+  }
+  }
+  GMap<kCrit> m;
+  m.fl = fl;
+  m.vp = (fl & 2) ? Vn : P;
+  m.cp = Bp;
+  m.kp = k.p;
+  m.ap = fl == 2 ? df_pow(k.p.a, n - 1) : df{0.f, 0.f};
+  if constexpr (kCrit) {
+    m.cc = Bc;
+    m.kc = k.c;
+    m.ac = fl == 2 ? df_pow(k.c.a, n - 1) : df{0.f, 0.f};
+  }
+  return m;
+}
+
+// Replays the lane's tokens from the state at its right edge; advantages
+// overwrite the values in the lane's row, returns go to the ret row.
+template <bool kCrit, bool kEnds>
+__device__ void replay_lane(const GaeArgs &a, float *val, float *ret, int lane, uint32_t act, uint32_t ends, int64_t t0,
+                            const CuView &cu, int blo, int b_last, GState st) {
+  Coefs<kCrit> k = load_coefs<kCrit>(a.coef, b_last);
+  float R = __ldg(a.rewards + b_last);
+  const int sw = lane & 7;
+  if constexpr (!kEnds) {
+#pragma unroll 1
+    for (int g = 7; g >= 0; --g) {
+      float4 *vp = reinterpret_cast<float4 *>(&val[4 * (8 * lane + (g ^ sw))]);
+      float4 *rp = reinterpret_cast<float4 *>(&ret[4 * (8 * lane + (g ^ sw))]);
+      const float4 v4 = *vp;
+      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
+      float ov[4], orr[4];
+      const uint32_t a4 = (act >> (4 * g)) & 15u;
+#pragma unroll
+      for (int i = 3; i >= 0; --i) {
+        const bool on = (a4 >> i) & 1u;
+        const df np = step_return(k.p, st.Bp, st.Vn, st.P);
+        ov[i] = on ? df_sub_round(np, vv[i]) : 0.f;
+        st.Bp = on ? np : st.Bp;
+        if constexpr (kCrit) {
+          const df nc = step_return(k.c, st.Bc, st.Vn, st.P);
+          orr[i] = on ? df_round(nc) : 0.f;
+          st.Bc = on ? nc : st.Bc;
+        } else {
+          orr[i] = on ? R : 0.f;
+        }
+        st.Vn = on ? vv[i] : st.Vn;
+        st.P = on ? 0.f : st.P;
+      }
+      *vp = make_float4(ov[0], ov[1], ov[2], ov[3]);
+      *rp = make_float4(orr[0], orr[1], orr[2], orr[3]);
+    }
+    return;
+  } else {
+#pragma unroll 1
+  for (int g = 7; g >= 0; --g) {
+    float4 *vp = reinterpret_cast<float4 *>(&val[4 * (8 * lane + (g ^ sw))]);
+    float4 *rp = reinterpret_cast<float4 *>(&ret[4 * (8 * lane + (g ^ sw))]);
+    const float4 v4 = *vp;
+    const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
+    float ov[4] = {0.f, 0.f, 0.f, 0.f}, orr[4] = {0.f, 0.f, 0.f, 0.f};
+    const uint32_t a4 = act >> (4 * g), e4 = ends >> (4 * g);
+#pragma unroll
+    for (int i = 3; i >= 0; --i) {
+      if ((e4 >> i) & 1u) {
+        const int b = cu.find(blo, b_last, t0 + 4 * g + i);
+        k = load_coefs<kCrit>(a.coef, b);
+        R = __ldg(a.rewards + b);
+        st.Bp = st.Bc = {0.f, 0.f};
+        st.Vn = 0.f;
+        st.P = R;
+      }
+      if ((a4 >> i) & 1u) {
+        st.Bp = step_return(k.p, st.Bp, st.Vn, st.P);
+        if constexpr (kCrit) st.Bc = step_return(k.c, st.Bc, st.Vn, st.P);
+        ov[i] = df_sub_round(st.Bp, vv[i]);
+        // gamma = lambda_critic = 1: the critic's return is the trajectory's reward
+        orr[i] = kCrit ? df_round(st.Bc) : R;
+        st.Vn = vv[i];
+        st.P = 0.f;
+      }
+    }
+    *vp = make_float4(ov[0], ov[1], ov[2], ov[3]);
+    *rp = make_float4(orr[0], orr[1], orr[2], orr[3]);
+  }
+  }
+}
+
+// What a lane keeps about a folded chunk until its look-back is done.
 template <bool kCrit>
-__global__ void __launch_bounds__(kThreads, 4) gae_scan_kernel(GaeArgs a) {
-  __shared__ int32_t s_cu_all[kWarps][kCuCap];
-  __shared__ WarpStage s_stage[kWarps];
-  __shared__ int s_ticket;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  // One ticket per CTA: its warps take consecutive chunks, highest first, so
-  // every chunk a warp waits on belongs to a CTA (or a warp) already running.
-  if (threadIdx.x == 0) s_ticket = atomicAdd(a.ticket, kWarps);
-  __syncthreads();
-  const int q = a.nchunks - 1 - (s_ticket + warp);
-  if (q < 0) return;  // the grid rounds the warp count up to whole CTAs
-  const int64_t t0 = int64_t(q) * kChunk + int64_t(lane) * kItems;
+struct Pending {
+  int q;           // chunk index
+  int buf;         // val buffer holding the chunk
+  bool active;     // the lane's first token is below N
+  bool any_end;    // some lane of the chunk holds a trajectory end
+  uint32_t act, ends;
+  int blo, b_last;
+  GMap<kCrit> E;   // maps of the lanes to the right within the chunk
+  GMap<kCrit> S;   // lane 0: map of the whole chunk
+};
+
+__device__ __forceinline__ int take_chunk(const GaeArgs &a, int lane) {
+  int t = 0;
+  if (lane == 0) t = atomicAdd(a.ticket, 1);
+  return a.nchunks - 1 - __shfl_sync(0xffffffffu, t, 0);
+}
+
+// Copies chunk q into val[buf], folds each lane's tokens, scans the lane maps
+// and publishes the chunk's map (or, when it ignores its right neighbour, its
+// left-edge state). Nothing here waits on another warp.
+template <bool kCrit>
+__device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, int lane, int q, int buf, Pending<kCrit> &p) {
+  const int64_t c0 = int64_t(q) * kChunk;
+  const int64_t t0 = c0 + int64_t(lane) * kItems;
   const int64_t N = a.N;
+  stage_in(a, c0, lane, w.val[buf], w.msk);
 
   // This chunk's slice of cu_seqlens, in shared memory when it fits.
   const int blo = __ldg(a.chunk_first + q);
   const int bhi = q + 1 < a.nchunks ? __ldg(a.chunk_first + q + 1) : a.B - 1;
   const int ncu = bhi - blo + 2;  // cu[blo .. bhi + 1]
-  int32_t *s_cu = s_cu_all[warp];
-  const CuView cu{a.cu, s_cu, blo, ncu <= kCuCap};
+  const CuView cu{a.cu, w.cu, blo, ncu <= kCuCap};
   if (cu.in_smem)
-    for (int i = lane; i < ncu; i += 32) s_cu[i] = __ldg(a.cu + blo + i);
+    for (int i = lane; i < ncu; i += 32) w.cu[i] = __ldg(a.cu + blo + i);
   __syncwarp();
-  WarpStage &stg = s_stage[warp];
-  stage_in(a, int64_t(q) * kChunk, lane, stg);
-  const float *vrow = stg.val[lane];
-  const uint8_t *mrow = stg.msk[lane];
 
-  // ---- trajectory ends among the 16 tokens (forward walk over cu_seqlens) -------
-  uint32_t endbits = 0;
-  int b_last;
-  {
-    int b = cu.find(blo, bhi, t0 < N ? t0 : N - 1);
-    int64_t next_end = cu[b + 1];
-    bool bad = false;
-#pragma unroll 4
-    for (int k = 0; k < kItems; ++k) {
-      const int64_t t = t0 + k;
-      if (t < N) {
-        while (b < bhi && t >= next_end) {
-          ++b;
-          next_end = cu[b + 1];
-        }
-        bad |= (t >= next_end);  // cu_seqlens[B] < N
-        endbits |= uint32_t(t == next_end - 1) << k;
-      }
+  // trajectory ends among the lane's tokens (forward walk over cu_seqlens)
+  const bool active = t0 < N;
+  uint32_t ends = 0;
+  int b_last = blo;
+  if (active) {
+    const int64_t tl = (t0 + kItems <= N ? int64_t(kItems) : N - t0) - 1;  // last token, relative to t0
+    int b = cu.find(blo, bhi, t0);
+    for (;;) {
+      const int64_t e = cu[b + 1] - 1 - t0;  // last token of trajectory b, relative to t0
+      if (e >= 0 && e <= tl) ends |= 1u << e;
+      if (e >= tl || b >= bhi) break;  // b holds the lane's last token (or cu_seqlens is malformed)
+      ++b;
     }
     b_last = b;
-    if (bad) raise_device_error(a.err, SAO_DEVERR_CU_SEQLENS);
   }
 
-  // ---- fold the thread's tokens into one map (right to left) ------------------
-  GMap M = identity_map();
+  cp_async_wait_all();
+  __syncwarp();
+  uint32_t act;
   {
-    int b = b_last;
-    int64_t b_start = cu[b];
-    TCoef c = load_coef(a.coef, b);
-#pragma unroll 1
-    for (int g = kItems / 4 - 1; g >= 0; --g) {
-      float v[4];
-      uint32_t act4 = 0;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        v[i] = vrow[4 * g + i];
-        act4 |= uint32_t(mrow[4 * g + i] != 0) << i;
-      }
-#pragma unroll
-      for (int i = 3; i >= 0; --i) {
-        const int k = 4 * g + i;
-        const int64_t t = t0 + k;
-        if (t < b_start && t < N) {
-          while (b > blo && t < b_start) {
-            --b;
-            b_start = cu[b];
-          }
-          c = load_coef(a.coef, b);
-        }
-        const bool is_act = (act4 >> i) & 1u, is_end = (endbits >> k) & 1u;
-        if (is_end) {
-          const float R = __ldg(a.rewards + b);
-          M.b = b;
-          M.ap = M.ac = {0.f, 0.f};
-          M.fl = is_act ? 3 : 1;
-          M.cp = M.cc = {is_act ? R : 0.f, 0.f};
-          M.v = is_act ? v[i] : 0.f;
-          M.p0 = is_act ? 0.f : R;
-        } else if (is_act) {
-          if (M.fl == 0) {
-            M.fl = 2;
-            M.ap = M.ac = {1.f, 0.f};
-            M.cp = M.cc = {0.f, 0.f};
-          } else {
-            const bool mact = (M.fl & 2) != 0;
-            const float Yv = mact ? M.v : 0.f, Yp = mact ? 0.f : M.p0;
-            M.cp = df_add(df_mul(c.ap, M.cp), df_mul_f(c.gp, Yv));
-            if (kCrit) M.cc = df_add(df_mul(c.ac, M.cc), df_mul_f(c.gc, Yv));
-            if (Yp != 0.f) {  // only right after a trajectory that ends on observations
-              M.cp = df_add_f(M.cp, Yp);
-              if (kCrit) M.cc = df_add_f(M.cc, Yp);
-            }
-            if (!(M.fl & 1)) {
-              M.ap = df_mul(c.ap, M.ap);
-              if (kCrit) M.ac = df_mul(c.ac, M.ac);
-            }
-            M.fl |= 2;
-          }
-          M.b = b;
-          M.v = v[i];
-          M.p0 = 0.f;
-        } else if (M.fl != 0) {
-          M.b = b;
-        }
-      }
-    }
-    M.k = c;  // M.b, when the map is not the identity, is the trajectory of the leftmost token: b
+    const uint4 m0 = *reinterpret_cast<const uint4 *>(&w.msk[16 * mgran(lane, 0)]);
+    const uint4 m1 = *reinterpret_cast<const uint4 *>(&w.msk[16 * mgran(lane, 1)]);
+    act = nonzero_bytes(m0.x) | nonzero_bytes(m0.y) << 4 | nonzero_bytes(m0.z) << 8 | nonzero_bytes(m0.w) << 12 |
+          nonzero_bytes(m1.x) << 16 | nonzero_bytes(m1.y) << 20 | nonzero_bytes(m1.z) << 24 |
+          nonzero_bytes(m1.w) << 28;
   }
 
-  // ---- suffix scan of the 32 maps of this warp ------------------------------------
-  GMap S = M;
+  // fold the lane's tokens, then the suffix scan of the warp's 32 maps
+  const bool any_end = __any_sync(0xffffffffu, ends != 0u);
+  GMap<kCrit> S = identity_map<kCrit>();
+  if (active)
+    S = any_end ? fold_lane<kCrit, true>(a, w.val[buf], lane, act, ends, t0, cu, blo, b_last)
+                : fold_lane<kCrit, false>(a, w.val[buf], lane, act, ends, t0, cu, blo, b_last);
 #pragma unroll 1
   for (int d = 1; d < 32; d <<= 1) {
-    const GMap o = shfl_down_map(S, d);
-    if (lane + d < 32) S = compose<kCrit>(S, o, a.coef);
+    const GMap<kCrit> o = shfl_down_map<kCrit>(S, d);
+    if (lane + d < 32) S = compose<kCrit>(S, o);
   }
-  GMap E = shfl_down_map(S, 1);  // lanes to my right within the chunk
-  if (lane == 31) E = identity_map();
+  GMap<kCrit> E = shfl_down_map<kCrit>(S, 1);  // lanes to my right within the chunk
+  if (lane == 31) E = identity_map<kCrit>();
 
-  // ---- publish this chunk and look back for the state at its right edge ------------
-  // Release stores of the status word order the published map/state before it;
-  // readers acquire the status before reading them.
-  GState zero;
-  zero.Bp = zero.Bc = {0.f, 0.f};
-  zero.Vn = zero.P = 0.f;
-  const bool last = (q == a.nchunks - 1);
-  const bool reset = (S.fl & 1) != 0;  // lane 0 holds the chunk's map
-  ChunkPub *me = a.pub + q;
+  // A chunk whose map ignores its right neighbour publishes its left-edge
+  // state at once; the others publish their map.
   if (lane == 0) {
-    // A chunk whose map ignores its right neighbour publishes its left-edge
-    // state at once; the others publish their map first.
-    if (last || reset) {
-      store_state(&me->incl, apply<kCrit>(S, zero, a.coef));
-      st_release(a.status + q, 2);
-    } else {
-      store_map(&me->agg, S);
-      st_release(a.status + q, 1);
-    }
+    if (q == a.nchunks - 1 || (S.fl & 1))
+      publish_state<kCrit>(a.incl + size_t(q) * kStateWords<kCrit>, apply<kCrit>(S, zero_state()));
+    else
+      publish_map<kCrit>(a.agg + size_t(q) * kMapWords<kCrit>, S);
   }
-  GState right = zero;
-  if (!__shfl_sync(0xffffffffu, int(last), 0)) right = look_back<kCrit>(a, q, lane);
-  if (lane == 0 && !reset && !last) {
-    store_state(&me->incl, apply<kCrit>(S, right, a.coef));
-    st_release(a.status + q, 2);
-  }
+  p.q = q;
+  p.buf = buf;
+  p.active = active;
+  p.any_end = any_end;
+  p.act = act;
+  p.ends = ends;
+  p.blo = blo;
+  p.b_last = b_last;
+  p.E = E;
+  p.S = S;
+}
 
-  // ---- replay the tokens from the incoming state ----------------------------------
-  GState st = apply<kCrit>(E, right, a.coef);
-  {
-    int b = b_last;
-    int64_t b_start = cu[b];
-    TCoef c = load_coef(a.coef, b);
-    float R = __ldg(a.rewards + b);
-    float *orow = stg.val[lane];
-    float *rrow = stg.ret[lane];
-#pragma unroll 1
-    for (int g = kItems / 4 - 1; g >= 0; --g) {
-      float v[4], ov[4], orr[4];
-      uint32_t act4 = 0;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        v[i] = vrow[4 * g + i];
-        act4 |= uint32_t(mrow[4 * g + i] != 0) << i;
-      }
-#pragma unroll
-      for (int i = 3; i >= 0; --i) {
-        const int k = 4 * g + i;
-        const int64_t t = t0 + k;
-        ov[i] = 0.f;
-        orr[i] = 0.f;
-        if (t >= N) continue;
-        if (t < b_start) {
-          while (b > blo && t < b_start) {
-            --b;
-            b_start = cu[b];
-          }
-          c = load_coef(a.coef, b);
-          R = __ldg(a.rewards + b);
-        }
-        if ((endbits >> k) & 1u) {
-          st.Bp = st.Bc = {0.f, 0.f};
-          st.Vn = 0.f;
-          st.P = R;
-        }
-        if ((act4 >> i) & 1u) {
-          st.Bp = df_add(df_mul(c.ap, st.Bp), df_mul_f(c.gp, st.Vn));
-          if (kCrit) st.Bc = df_add(df_mul(c.ac, st.Bc), df_mul_f(c.gc, st.Vn));
-          if (st.P != 0.f) {
-            st.Bp = df_add_f(st.Bp, st.P);
-            if (kCrit) st.Bc = df_add_f(st.Bc, st.P);
-          }
-          orr[i] = kCrit ? df_round(st.Bc) : R;  // gamma = lambda_critic = 1: the return is R
-          ov[i] = df_round(df_add_f(st.Bp, -v[i]));
-          st.Vn = v[i];
-          st.P = 0.f;
-        }
-      }
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        orow[4 * g + i] = ov[i];
-        rrow[4 * g + i] = orr[i];
-      }
-    }
+// Looks back for the state at the chunk's right edge, publishes its left-edge
+// state, replays the tokens and stores advantages and returns.
+template <bool kCrit>
+__device__ void finish_chunk(const GaeArgs &a, WarpBuf &w, int lane, const Pending<kCrit> &p) {
+  const bool last = (p.q == a.nchunks - 1);
+  const bool reset = __shfl_sync(0xffffffffu, p.S.fl & 1, 0) != 0;  // lane 0 holds the chunk's map
+  GState right = zero_state();
+  if (!last) right = look_back<kCrit>(a, p.q, lane);
+  if (lane == 0 && !reset && !last)
+    publish_state<kCrit>(a.incl + size_t(p.q) * kStateWords<kCrit>, apply<kCrit>(p.S, right));
+  const int64_t c0 = int64_t(p.q) * kChunk;
+  if (p.active) {
+    const GState in = apply<kCrit>(p.E, right);
+    const CuView cu{a.cu, nullptr, p.blo, false};  // ends are rare: read cu_seqlens from global memory
+    const int64_t t0 = c0 + int64_t(lane) * kItems;
+    if (p.any_end)
+      replay_lane<kCrit, true>(a, w.val[p.buf], w.ret, lane, p.act, p.ends, t0, cu, p.blo, p.b_last, in);
+    else
+      replay_lane<kCrit, false>(a, w.val[p.buf], w.ret, lane, p.act, p.ends, t0, cu, p.blo, p.b_last, in);
   }
-  stage_out(a, int64_t(q) * kChunk, lane, stg);
+  __syncwarp();
+  stage_out(a, c0, lane, w.val[p.buf], w.ret);
+  __syncwarp();
+}
+
+// Persistent warps, software-pipelined: a warp takes a chunk (ticket), folds
+// and publishes it, and only then looks back for the chunk it took before, so
+// the chunks it waits on have had a whole fold to publish. Tickets keep the
+// decoupled look-back safe: a warp waits only on chunks taken before its own,
+// and every taken chunk is published before its warp waits on anything.
+template <bool kCrit>
+__global__ void __launch_bounds__(kThreads, kMinBlocks) gae_scan_kernel(GaeArgs a) {
+  extern __shared__ __align__(16) unsigned char s_raw[];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  WarpBuf &w = reinterpret_cast<WarpBuf *>(s_raw)[warp];
+  int q = take_chunk(a, lane);
+  if (q < 0) return;
+  Pending<kCrit> p;
+  int buf = 0;
+  fold_chunk<kCrit>(a, w, lane, q, buf, p);
+  for (;;) {
+    const int qn = take_chunk(a, lane);
+    Pending<kCrit> n;
+    if (qn >= 0) fold_chunk<kCrit>(a, w, lane, qn, buf ^ 1, n);
+    finish_chunk<kCrit>(a, w, lane, p);
+    if (qn < 0) break;
+    p = n;
+    buf ^= 1;
+  }
 }
 
 // Per-trajectory coefficients (fp64 then split to double-float) and a check of
@@ -681,12 +826,30 @@ __global__ void gae_coef_kernel(const int32_t *cu, int B, int64_t N, float gamma
   coef[2 * b + 1] = make_float4(Ac.hi, Ac.lo, Gc.hi, Gc.lo);
 }
 
+constexpr size_t kScanSmem = sizeof(WarpBuf) * kWarps;
+
+// The scan's shared memory exceeds the default 48 KB: opt in once per kernel
+// and device.
+sao_status set_scan_smem(void (*kern)(GaeArgs), int which, int device) {
+  constexpr int kMaxDevices = 64;
+  static std::once_flag once[2][kMaxDevices];
+  static cudaError_t err[2][kMaxDevices];
+  if (device < 0 || device >= kMaxDevices) return fail(SAO_ERR_CUDA, "device %d out of range", device);
+  std::call_once(once[which][device], [&] {
+    err[which][device] = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kScanSmem));
+  });
+  if (err[which][device] != cudaSuccess)
+    return fail(SAO_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(err[which][device]));
+  return SAO_OK;
+}
+
 }  // namespace
 
 size_t gae_ws_bytes(int64_t N, int64_t B) {
   const int64_t nchunks = (N + kChunk - 1) / kChunk;
-  return round256(sizeof(int)) + round256(sizeof(int) * (B + 1)) + round256(sizeof(int) * nchunks) +
-         round256(sizeof(float4) * 2 * (B + 1)) + round256(sizeof(ChunkPub) * nchunks) +
+  return round256(sizeof(int)) + round256(sizeof(int) * (B + 1)) +
+         round256(sizeof(uint64_t) * kMapWords<true> * nchunks) +
+         round256(sizeof(uint64_t) * kStateWords<true> * nchunks) + round256(sizeof(float4) * 2 * (B + 1)) +
          round256(sizeof(int) * (nchunks + 1));
 }
 
@@ -696,14 +859,18 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   if (N == 0) return SAO_OK;
   const int64_t nchunks = (N + kChunk - 1) / kChunk;
   if (nchunks > (int64_t(1) << 30)) return fail(SAO_ERR_SHAPE, "too many tokens for the advantage scan");
+  const bool crit_trivial = (gamma == 1.0f && lam_c == 1.0f);
+  const size_t map_words = crit_trivial ? kMapWords<false> : kMapWords<true>;
+  const size_t state_words = crit_trivial ? kStateWords<false> : kStateWords<true>;
   Carver c(ws_body, body_bytes);
+  // ticket, action counts and the publication arrays start at zero
   char *zero_begin = c.base + c.off;
   int *ticket = c.take<int>(1);
   int *nact = c.take<int>(size_t(B) + 1);
-  int *status = c.take<int>(size_t(nchunks));
+  uint64_t *agg = c.take<uint64_t>(map_words * size_t(nchunks));
+  uint64_t *incl = c.take<uint64_t>(state_words * size_t(nchunks));
   char *zero_end = c.base + c.off;
   float4 *coef = c.take<float4>(2 * (size_t(B) + 1));
-  ChunkPub *pub = c.take<ChunkPub>(size_t(nchunks));
   int *chunk_first = c.take<int>(size_t(nchunks) + 1);
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the advantage scan");
   SAO_CUDA_TRY(cudaMemsetAsync(zero_begin, 0, size_t(zero_end - zero_begin), s));
@@ -734,18 +901,21 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   a.coef = coef;
   a.chunk_first = chunk_first;
   a.ticket = ticket;
-  a.status = status;
-  a.pub = pub;
+  a.agg = agg;
+  a.incl = incl;
   a.adv = adv;
   a.ret = ret;
   a.err = err;
-  const bool crit_trivial = (gamma == 1.0f && lam_c == 1.0f);
-  const unsigned grid = unsigned((nchunks + kWarps - 1) / kWarps);
+  DeviceInfo di;
+  SAO_TRY(device_info(&di));
+  auto kern = crit_trivial ? gae_scan_kernel<false> : gae_scan_kernel<true>;
+  SAO_TRY(set_scan_smem(kern, crit_trivial ? 0 : 1, di.device));
+  // persistent: as many warps as fit on the GPU, never more than chunks
+  const int64_t ctas = (nchunks + kWarps - 1) / kWarps;
+  const int64_t resident = int64_t(di.sm_count) * kMinBlocks;
+  const unsigned grid = unsigned(ctas < resident ? ctas : resident);
   int slot = launch_begin("gae_scan", s);
-  if (crit_trivial)
-    gae_scan_kernel<false><<<grid, kThreads, 0, s>>>(a);
-  else
-    gae_scan_kernel<true><<<grid, kThreads, 0, s>>>(a);
+  kern<<<grid, kThreads, kScanSmem, s>>>(a);
   return launch_end(slot, s);
 }
 

@@ -12,7 +12,7 @@
 namespace sao {
 namespace {
 
-constexpr size_t kNoAllocScratchBytes = size_t(8) << 20;  // 8 MiB
+constexpr size_t kNoAllocScratchBytes = size_t(16) << 20;  // 16 MiB
 
 // Shared by every call on a device; held until the process exits.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
