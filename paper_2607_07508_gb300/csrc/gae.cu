@@ -24,7 +24,7 @@
 //     row reads are free of bank conflicts),
 //   * each lane folds its 32 tokens into one map, driven by two bit masks
 //     (action tokens, trajectory ends) so the common token costs one fused
-//     double-float a*B + g*V and no index arithmetic,
+//     double-float a*B + g*V, a few selects and no index arithmetic,
 //   * a warp-shuffle suffix scan combines the 32 maps of the chunk,
 //   * warps chain their chunks right-to-left by decoupled look-back: each CTA
 //     takes one ticket and its warps work on the chunks below it, so a warp
@@ -107,11 +107,6 @@ __device__ df df_pow(df x, int e) {
   return r;
 }
 __device__ __forceinline__ float df_round(df x) { return __fadd_rn(x.hi, x.lo); }
-// round(x - v) to float
-__device__ __forceinline__ float df_sub_round(df x, float v) {
-  const df s = two_sum(x.hi, -v);
-  return __fadd_rn(s.hi, __fadd_rn(s.lo, x.lo));
-}
 __device__ __forceinline__ df df_from_double(double x) {
   const float hi = float(x);
   return {hi, float(x - double(hi))};
@@ -510,10 +505,14 @@ __device__ __forceinline__ uint32_t nonzero_bytes(uint32_t x) {
 // action token / the last token of its trajectory; b_last is the trajectory of
 // the lane's last token below N.
 
-// Map of the lane's 32 tokens. kEnds: some lane of the warp holds a trajectory
-// end (the warp-uniform choice between the general loop and the branch-free
-// one for runs inside a single trajectory).
-template <bool kCrit, bool kEnds>
+// The token loops below take 4 tokens at a time. A group in which no lane of
+// the warp holds a trajectory end or a waiting reward (the common case: turns
+// and trajectories span hundreds of tokens) runs branch-free, one fused
+// double-float a*B + g*V per token with the action flag applied by selects;
+// otherwise the warp takes the general path for that group.
+
+// Map of the lane's 32 tokens.
+template <bool kCrit>
 __device__ GMap<kCrit> fold_lane(const GaeArgs &a, const float *val, int lane, uint32_t act, uint32_t ends,
                                  int64_t t0, const CuView &cu, int blo, int b_last) {
   Coefs<kCrit> k = load_coefs<kCrit>(a.coef, b_last);
@@ -521,12 +520,31 @@ __device__ GMap<kCrit> fold_lane(const GaeArgs &a, const float *val, int lane, u
   float Vn = 0.f, P = 0.f;
   int fl = 0, n = 0;
   const int sw = lane & 7;
-  if constexpr (!kEnds) {
 #pragma unroll 1
-    for (int g = 7; g >= 0; --g) {
-      const float4 v4 = *reinterpret_cast<const float4 *>(&val[4 * (8 * lane + (g ^ sw))]);
-      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
-      const uint32_t a4 = (act >> (4 * g)) & 15u;
+  for (int g = 7; g >= 0; --g) {
+    const float4 v4 = *reinterpret_cast<const float4 *>(&val[4 * (8 * lane + (g ^ sw))]);
+    const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
+    const uint32_t a4 = (act >> (4 * g)) & 15u, e4 = (ends >> (4 * g)) & 15u;
+    if (__any_sync(0xffffffffu, e4 != 0u || P != 0.f)) {
+#pragma unroll
+      for (int i = 3; i >= 0; --i) {
+        if ((e4 >> i) & 1u) {  // last token of a trajectory: reset
+          const int b = cu.find(blo, b_last, t0 + 4 * g + i);
+          k = load_coefs<kCrit>(a.coef, b);
+          P = __ldg(a.rewards + b);
+          Bp = Bc = {0.f, 0.f};
+          Vn = 0.f;
+          fl = 1;
+        }
+        if ((a4 >> i) & 1u) {
+          Bp = step_return(k.p, Bp, Vn, P);
+          if constexpr (kCrit) Bc = step_return(k.c, Bc, Vn, P);
+          Vn = vv[i];
+          P = 0.f;
+          fl |= 2;
+        }
+      }
+    } else {
 #pragma unroll
       for (int i = 3; i >= 0; --i) {
         const bool on = (a4 >> i) & 1u;
@@ -538,36 +556,12 @@ __device__ GMap<kCrit> fold_lane(const GaeArgs &a, const float *val, int lane, u
         }
         Vn = on ? vv[i] : Vn;
       }
-      n += __popc(a4);
-    }
-    fl = n > 0 ? 2 : 0;
-  } else {
-#pragma unroll 1
-  for (int g = 7; g >= 0; --g) {
-    const float4 v4 = *reinterpret_cast<const float4 *>(&val[4 * (8 * lane + (g ^ sw))]);
-    const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
-    const uint32_t a4 = act >> (4 * g), e4 = ends >> (4 * g);
-#pragma unroll
-    for (int i = 3; i >= 0; --i) {
-      if ((e4 >> i) & 1u) {  // last token of a trajectory: reset
-        const int b = cu.find(blo, b_last, t0 + 4 * g + i);
-        k = load_coefs<kCrit>(a.coef, b);
-        P = __ldg(a.rewards + b);
-        Bp = Bc = {0.f, 0.f};
-        Vn = 0.f;
-        fl = 1;
-      }
-      if ((a4 >> i) & 1u) {
-        Bp = step_return(k.p, Bp, Vn, P);
-        if constexpr (kCrit) Bc = step_return(k.c, Bc, Vn, P);
-        Vn = vv[i];
-        P = 0.f;
-        fl |= 2;
-        ++n;
-      }
+      fl |= a4 ? 2 : 0;
     }
   }
-  }
+  // act tokens left of the leftmost end (all of them when there is none)
+  const int lead = ends ? __clz(__brev(ends)) : 32;  // index of the lowest end bit
+  n = __popc(act & (lead >= 32 ? 0xffffffffu : ((1u << lead) - 1u)));
   GMap<kCrit> m;
   m.fl = fl;
   m.vp = (fl & 2) ? Vn : P;
@@ -582,75 +576,68 @@ __device__ GMap<kCrit> fold_lane(const GaeArgs &a, const float *val, int lane, u
   return m;
 }
 
+// A - V rounded to float, from the double-float lambda-return B: B.hi - V is
+// exact when the two are within a factor of two of each other (the case where
+// A is small against V), and otherwise already within half an ulp of A.
+__device__ __forceinline__ float adv_round(df B, float v) { return __fadd_rn(__fsub_rn(B.hi, v), B.lo); }
+
 // Replays the lane's tokens from the state at its right edge; advantages
 // overwrite the values in the lane's row, returns go to the ret row.
-template <bool kCrit, bool kEnds>
-__device__ void replay_lane(const GaeArgs &a, float *val, float *ret, int lane, uint32_t act, uint32_t ends, int64_t t0,
-                            const CuView &cu, int blo, int b_last, GState st) {
+template <bool kCrit>
+__device__ void replay_lane(const GaeArgs &a, float *val, float *ret, int lane, uint32_t act, uint32_t ends,
+                            int64_t t0, const CuView &cu, int blo, int b_last, GState st) {
   Coefs<kCrit> k = load_coefs<kCrit>(a.coef, b_last);
   float R = __ldg(a.rewards + b_last);
   const int sw = lane & 7;
-  if constexpr (!kEnds) {
-#pragma unroll 1
-    for (int g = 7; g >= 0; --g) {
-      float4 *vp = reinterpret_cast<float4 *>(&val[4 * (8 * lane + (g ^ sw))]);
-      float4 *rp = reinterpret_cast<float4 *>(&ret[4 * (8 * lane + (g ^ sw))]);
-      const float4 v4 = *vp;
-      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
-      float ov[4], orr[4];
-      const uint32_t a4 = (act >> (4 * g)) & 15u;
-#pragma unroll
-      for (int i = 3; i >= 0; --i) {
-        const bool on = (a4 >> i) & 1u;
-        const df np = step_return(k.p, st.Bp, st.Vn, st.P);
-        ov[i] = on ? df_sub_round(np, vv[i]) : 0.f;
-        st.Bp = on ? np : st.Bp;
-        if constexpr (kCrit) {
-          const df nc = step_return(k.c, st.Bc, st.Vn, st.P);
-          orr[i] = on ? df_round(nc) : 0.f;
-          st.Bc = on ? nc : st.Bc;
-        } else {
-          orr[i] = on ? R : 0.f;
-        }
-        st.Vn = on ? vv[i] : st.Vn;
-        st.P = on ? 0.f : st.P;
-      }
-      *vp = make_float4(ov[0], ov[1], ov[2], ov[3]);
-      *rp = make_float4(orr[0], orr[1], orr[2], orr[3]);
-    }
-    return;
-  } else {
 #pragma unroll 1
   for (int g = 7; g >= 0; --g) {
     float4 *vp = reinterpret_cast<float4 *>(&val[4 * (8 * lane + (g ^ sw))]);
     float4 *rp = reinterpret_cast<float4 *>(&ret[4 * (8 * lane + (g ^ sw))]);
     const float4 v4 = *vp;
     const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
-    float ov[4] = {0.f, 0.f, 0.f, 0.f}, orr[4] = {0.f, 0.f, 0.f, 0.f};
-    const uint32_t a4 = act >> (4 * g), e4 = ends >> (4 * g);
+    float ov[4], orr[4];
+    const uint32_t a4 = (act >> (4 * g)) & 15u, e4 = (ends >> (4 * g)) & 15u;
+    if (__any_sync(0xffffffffu, e4 != 0u || st.P != 0.f)) {
 #pragma unroll
-    for (int i = 3; i >= 0; --i) {
-      if ((e4 >> i) & 1u) {
-        const int b = cu.find(blo, b_last, t0 + 4 * g + i);
-        k = load_coefs<kCrit>(a.coef, b);
-        R = __ldg(a.rewards + b);
-        st.Bp = st.Bc = {0.f, 0.f};
-        st.Vn = 0.f;
-        st.P = R;
+      for (int i = 3; i >= 0; --i) {
+        ov[i] = orr[i] = 0.f;
+        if ((e4 >> i) & 1u) {
+          const int b = cu.find(blo, b_last, t0 + 4 * g + i);
+          k = load_coefs<kCrit>(a.coef, b);
+          R = __ldg(a.rewards + b);
+          st.Bp = st.Bc = {0.f, 0.f};
+          st.Vn = 0.f;
+          st.P = R;
+        }
+        if ((a4 >> i) & 1u) {
+          st.Bp = step_return(k.p, st.Bp, st.Vn, st.P);
+          if constexpr (kCrit) st.Bc = step_return(k.c, st.Bc, st.Vn, st.P);
+          ov[i] = adv_round(st.Bp, vv[i]);
+          // gamma = lambda_critic = 1: the critic's return is the trajectory's reward
+          orr[i] = kCrit ? df_round(st.Bc) : R;
+          st.Vn = vv[i];
+          st.P = 0.f;
+        }
       }
-      if ((a4 >> i) & 1u) {
-        st.Bp = step_return(k.p, st.Bp, st.Vn, st.P);
-        if constexpr (kCrit) st.Bc = step_return(k.c, st.Bc, st.Vn, st.P);
-        ov[i] = df_sub_round(st.Bp, vv[i]);
-        // gamma = lambda_critic = 1: the critic's return is the trajectory's reward
-        orr[i] = kCrit ? df_round(st.Bc) : R;
-        st.Vn = vv[i];
-        st.P = 0.f;
+    } else {
+#pragma unroll
+      for (int i = 3; i >= 0; --i) {
+        const bool on = (a4 >> i) & 1u;
+        const df np = df_axpby(k.p.a, st.Bp, k.p.g, st.Vn);
+        ov[i] = on ? adv_round(np, vv[i]) : 0.f;
+        st.Bp = on ? np : st.Bp;
+        if constexpr (kCrit) {
+          const df nc = df_axpby(k.c.a, st.Bc, k.c.g, st.Vn);
+          orr[i] = on ? df_round(nc) : 0.f;
+          st.Bc = on ? nc : st.Bc;
+        } else {
+          orr[i] = on ? R : 0.f;
+        }
+        st.Vn = on ? vv[i] : st.Vn;
       }
     }
     *vp = make_float4(ov[0], ov[1], ov[2], ov[3]);
     *rp = make_float4(orr[0], orr[1], orr[2], orr[3]);
-  }
   }
 }
 
@@ -660,7 +647,6 @@ struct Pending {
   int q;           // chunk index
   int buf;         // val buffer holding the chunk
   bool active;     // the lane's first token is below N
-  bool any_end;    // some lane of the chunk holds a trajectory end
   uint32_t act, ends;
   int blo, b_last;
   GMap<kCrit> E;   // maps of the lanes to the right within the chunk
@@ -720,11 +706,9 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, int lane, int q, int bu
   }
 
   // fold the lane's tokens, then the suffix scan of the warp's 32 maps
-  const bool any_end = __any_sync(0xffffffffu, ends != 0u);
-  GMap<kCrit> S = identity_map<kCrit>();
-  if (active)
-    S = any_end ? fold_lane<kCrit, true>(a, w.val[buf], lane, act, ends, t0, cu, blo, b_last)
-                : fold_lane<kCrit, false>(a, w.val[buf], lane, act, ends, t0, cu, blo, b_last);
+  // every lane folds (the token loops vote across the warp); a lane past N
+  // has no flags and yields the identity map
+  GMap<kCrit> S = fold_lane<kCrit>(a, w.val[buf], lane, act, ends, t0, cu, blo, b_last);
 #pragma unroll 1
   for (int d = 1; d < 32; d <<= 1) {
     const GMap<kCrit> o = shfl_down_map<kCrit>(S, d);
@@ -744,7 +728,6 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, int lane, int q, int bu
   p.q = q;
   p.buf = buf;
   p.active = active;
-  p.any_end = any_end;
   p.act = act;
   p.ends = ends;
   p.blo = blo;
@@ -764,14 +747,13 @@ __device__ void finish_chunk(const GaeArgs &a, WarpBuf &w, int lane, const Pendi
   if (lane == 0 && !reset && !last)
     publish_state<kCrit>(a.incl + size_t(p.q) * kStateWords<kCrit>, apply<kCrit>(p.S, right));
   const int64_t c0 = int64_t(p.q) * kChunk;
-  if (p.active) {
+  {
+    // every lane replays (the token loops vote across the warp); rows past N
+    // are never stored
     const GState in = apply<kCrit>(p.E, right);
     const CuView cu{a.cu, nullptr, p.blo, false};  // ends are rare: read cu_seqlens from global memory
     const int64_t t0 = c0 + int64_t(lane) * kItems;
-    if (p.any_end)
-      replay_lane<kCrit, true>(a, w.val[p.buf], w.ret, lane, p.act, p.ends, t0, cu, p.blo, p.b_last, in);
-    else
-      replay_lane<kCrit, false>(a, w.val[p.buf], w.ret, lane, p.act, p.ends, t0, cu, p.blo, p.b_last, in);
+    replay_lane<kCrit>(a, w.val[p.buf], w.ret, lane, p.act, p.ends, t0, cu, p.blo, p.b_last, in);
   }
   __syncwarp();
   stage_out(a, c0, lane, w.val[p.buf], w.ret);
