@@ -31,6 +31,10 @@ Optimization for Agentic Reinforcement Learning" (arxiv 2607.07508):
 * ``running_mean_advantages``  the running-mean reward baseline of the
                           single-rollout ablation (§4.3) and the online writing
                           comparison (§4.5)
+* ``decoupled_loss``      the decoupled three-policy objective that DIS
+                          simplifies (§3.1): a clipped ratio against the old
+                          policy, weighted by the old/rollout ratio, with a
+                          double-sided mask on that weight
 
 Readings taken where the paper is silent or ambiguous (each one is listed with
 its reason in the design notes):
@@ -79,6 +83,15 @@ R16 Running-mean baseline: trajectories are taken in batch order; the baseline
     recorded for its prompt before b, 0 when there are none; A_b = R_b -
     baseline is broadcast to b's action tokens; then R_b enters the prompt's
     window. One shared prompt id gives the single global window of §4.5.
+R17 Decoupled three-policy objective (§3.1 names its parts but writes no
+    formula): r_t = pi_theta/pi_old corrects staleness and is clipped as in
+    R14; w_t = pi_old/pi_rollout corrects the training/rollout mismatch and is
+    kept only inside a strict band (w_low < w < w_high, the double-sided
+    masking that §3.1 likens DIS to), else the token is masked. loss =
+    -(1/n) sum_t w_t min(r_t A_t, clip(r_t, 1-eps_low, 1+eps_high) A_t) over
+    kept action tokens, n as in R2; w is a detached coefficient, so
+    d loss / d logp_t = -(1/n) w_t r_t A_t on unclipped kept tokens, else 0.
+    All decisions in fp32, the mismatch test before the clip test.
 """
 from __future__ import annotations
 
@@ -495,3 +508,65 @@ def running_mean_advantages(rewards, prompt_ids, loss_mask, cu_seqlens, history,
         hist[p, cnt[p] % window] = R[b]
         cnt[p] += 1
     return adv, hist, cnt
+
+
+# ---------------------------------------------------------------------------
+# Decoupled three-policy objective (§3.1), reading R17
+# ---------------------------------------------------------------------------
+
+MIS_LOW = 5
+MIS_HIGH = 6
+
+
+def decoupled_flags(logp, prox_logp, rollout_logp, adv, loss_mask, eps_low: float, eps_high: float,
+                    w_low: float, w_high: float) -> np.ndarray:
+    """0 kept, unclipped; 1 / 2 clipped at 1-eps_low / 1+eps_high (as R14);
+    3 non-finite; 4 not an action token; 5 w <= w_low; 6 w >= w_high.
+    Decided in fp32 (R17)."""
+    lp = np.asarray(logp, np.float32)
+    px = np.asarray(prox_logp, np.float32)
+    ro = np.asarray(rollout_logp, np.float32)
+    a = np.asarray(adv, np.float32)
+    m = np.asarray(loss_mask).astype(bool)
+    with np.errstate(all="ignore"):
+        d = (lp - px).astype(np.float32)        # log pi_theta/pi_old
+        e = (px - ro).astype(np.float32)        # log pi_old/pi_rollout
+        r = np.exp(d).astype(np.float32)
+        w = np.exp(e).astype(np.float32)
+        lo = np.float32(1.0) - np.float32(eps_low)
+        hi = np.float32(1.0) + np.float32(eps_high)
+        flags = np.zeros(m.shape, np.uint8)
+        flags[(a > 0) & (r > hi)] = CLIP_HIGH
+        flags[(a < 0) & (r < lo)] = CLIP_LOW
+        flags[w >= np.float32(w_high)] = MIS_HIGH
+        flags[w <= np.float32(w_low)] = MIS_LOW
+        finite = np.isfinite(d) & np.isfinite(e) & np.isfinite(a)
+    flags[~finite] = FLAG_NONFINITE
+    flags[~m] = FLAG_MASKED
+    return flags
+
+
+def decoupled_loss(logp, prox_logp, rollout_logp, adv, loss_mask, eps_low: float, eps_high: float,
+                   w_low: float, w_high: float, n_norm: int = 0) -> Dict[str, object]:
+    """Decoupled PPO objective with the mismatch weight masked outside
+    (w_low, w_high) (R17). counts = [n_action, n_clip_low, n_clip_high,
+    n_nonfinite, n_mismatch_low, n_mismatch_high]."""
+    flags = decoupled_flags(logp, prox_logp, rollout_logp, adv, loss_mask, eps_low, eps_high, w_low, w_high)
+    m = np.asarray(loss_mask).astype(bool)
+    n_action = int(m.sum())
+    n = int(n_norm) if n_norm > 0 else n_action
+    with np.errstate(all="ignore"):
+        r = np.exp(_f64(logp) - _f64(prox_logp))
+        w = np.exp(_f64(prox_logp) - _f64(rollout_logp))
+        A = _f64(adv)
+        lo = float(np.float32(1.0) - np.float32(eps_low))
+        hi = float(np.float32(1.0) + np.float32(eps_high))
+        term = np.where(flags == CLIP_NONE, r * A,
+                        np.where(flags == CLIP_LOW, lo * A, np.where(flags == CLIP_HIGH, hi * A, 0.0)))
+        contrib = np.where(flags <= CLIP_HIGH, w * term, 0.0)
+        coef = np.where(flags == CLIP_NONE, -w * r * A / n, 0.0) if n > 0 else np.zeros(len(m))
+    loss = -float(contrib.sum()) / n if n > 0 else 0.0
+    counts = np.array([n_action, int((flags == CLIP_LOW).sum()), int((flags == CLIP_HIGH).sum()),
+                       int((flags == FLAG_NONFINITE).sum()), int((flags == MIS_LOW).sum()),
+                       int((flags == MIS_HIGH).sum())], np.int64)
+    return {"loss": loss, "coef": coef, "flags": flags, "counts": counts}

@@ -605,3 +605,98 @@ def test_running_mean_baseline_window():
     adv2, _, _ = O.running_mean_advantages(np.array([0.0], np.float32), np.array([0]), np.ones(1, np.uint8),
                                            np.array([0, 1]), hist, cnt, 2)
     assert np.allclose(adv2, [-1.0])
+
+
+# ---------------------------------------------------------------------------
+# decoupled three-policy objective (§3.1), reading R17
+# ---------------------------------------------------------------------------
+
+def _three_policies(seed, N=200):
+    r = _rng(seed)
+    logp = (-r.exponential(2.0, N)).astype(np.float32)
+    prox = (logp + r.normal(0, 0.2, N)).astype(np.float32)
+    roll = (prox + r.normal(0, 0.3, N)).astype(np.float32)
+    adv = r.normal(size=N).astype(np.float32)
+    m = (r.random(N) < 0.8).astype(np.uint8)
+    return logp, prox, roll, adv, m
+
+
+def test_decoupled_loss_equal_old_and_rollout_is_the_clipped_surrogate():
+    """pi_old = pi_rollout makes the mismatch weight 1 (inside the band): the
+    objective is the token-mean clipped surrogate against pi_old."""
+    logp, prox, _, adv, m = _three_policies(80)
+    d = O.decoupled_loss(logp, prox, prox, adv, m, 0.2, 0.28, 0.5, 2.0)
+    c = O.clip_loss(logp, prox, adv, m, np.array([0, len(m)]), 0.2, 0.28, O.NORM_TOKEN)
+    assert abs(d["loss"] - c["loss"]) < 1e-12
+    assert np.allclose(d["coef"], c["coef"], atol=1e-15) and np.array_equal(d["flags"], c["flags"])
+    assert list(d["counts"][:4]) == list(c["counts"]) and d["counts"][4] == d["counts"][5] == 0
+
+
+def test_decoupled_loss_without_bounds_telescopes_to_eq1():
+    """With every bound off, w*r = pi_theta/pi_rollout: the loss is Eq. 1 with
+    f = identity against the rollout log-probs, -(1/n) sum exp(logp - rollout) A."""
+    logp, prox, roll, adv, m = _three_policies(81)
+    d = O.decoupled_loss(logp, prox, roll, adv, m, 1e30, 1e30, 0.0, np.inf)
+    k = m.astype(bool)
+    lp, ro, a = (x.astype(np.float64) for x in (logp, roll, adv))
+    want = -math.fsum(np.exp(lp[k] - ro[k]) * a[k]) / k.sum()
+    assert abs(d["loss"] - want) < 1e-12
+    dis = O.policy_loss(logp, roll, adv, m, 1e30, 1e30)
+    assert np.allclose(d["coef"], dis["coef"], atol=1e-15)
+
+
+def test_decoupled_loss_hand_example():
+    """Token 0: w = 2.5 >= 2 (masked high); 1: w = 0.25 <= 0.5 (masked low);
+    2: w = 1.25 kept, r = 1.5 > 1.28 with A > 0 (clipped: w*(1+eps_high)*A, no
+    gradient); 3: w = 1, r = 0.9 with A < 0 above 1-eps_low (unclipped: w*r*A);
+    4: not an action token."""
+    logp = np.log(np.array([1.0, 1.0, 1.5, 0.9, 1.0])).astype(np.float32)
+    prox = np.zeros(5, np.float32)
+    roll = np.log(np.array([0.4, 4.0, 0.8, 1.0, 1.0])).astype(np.float32)
+    adv = np.array([1.0, 1.0, 2.0, -1.0, 3.0], np.float32)
+    m = np.array([1, 1, 1, 1, 0], np.uint8)
+    out = O.decoupled_loss(logp, prox, roll, adv, m, 0.2, 0.28, 0.5, 2.0)
+    assert list(out["flags"]) == [O.MIS_HIGH, O.MIS_LOW, O.CLIP_HIGH, O.CLIP_NONE, O.FLAG_MASKED]
+    assert list(out["counts"]) == [4, 0, 1, 0, 1, 1]
+    w2 = math.exp(-float(roll[2]))
+    r3 = math.exp(float(logp[3]))
+    hi = float(np.float32(1.0) + np.float32(0.28))
+    assert abs(out["loss"] - (-(w2 * hi * 2.0 + 1.0 * r3 * -1.0) / 4)) < 1e-12
+    assert out["coef"][2] == 0 and abs(out["coef"][3] - (r3 / 4)) < 1e-15
+
+
+def test_decoupled_loss_band_is_strict():
+    """w = 1 exactly (pi_old = pi_rollout): masked when a band edge equals 1."""
+    lp = np.zeros(3, np.float32)
+    adv = np.ones(3, np.float32)
+    m = np.ones(3, np.uint8)
+    assert set(O.decoupled_loss(lp, lp, lp, adv, m, 0.2, 0.28, 1.0, 2.0)["flags"]) == {O.MIS_LOW}
+    assert set(O.decoupled_loss(lp, lp, lp, adv, m, 0.2, 0.28, 0.5, 1.0)["flags"]) == {O.MIS_HIGH}
+    assert set(O.decoupled_loss(lp, lp, lp, adv, m, 0.2, 0.28, 0.5, 2.0)["flags"]) == {O.CLIP_NONE}
+
+
+def test_decoupled_loss_finite_differences_and_normaliser():
+    logp, prox, roll, adv, m = _three_policies(82, N=24)
+    out = O.decoupled_loss(logp, prox, roll, adv, m, 0.2, 0.28, 0.5, 2.0, n_norm=7)
+    lp = logp.astype(np.float64)
+    for t in range(24):
+        r = math.exp(lp[t] - float(prox[t]))
+        if abs(r - 0.8) < 1e-4 or abs(r - 1.28) < 1e-4:
+            continue
+        a, b = lp.copy(), lp.copy()
+        a[t] += 1e-7
+        b[t] -= 1e-7
+        num = (O.decoupled_loss(a, prox, roll, adv, m, 0.2, 0.28, 0.5, 2.0, n_norm=7)["loss"] -
+               O.decoupled_loss(b, prox, roll, adv, m, 0.2, 0.28, 0.5, 2.0, n_norm=7)["loss"]) / 2e-7
+        assert abs(num - out["coef"][t]) < 1e-7
+
+
+def test_decoupled_loss_nonfinite_tokens_are_masked():
+    logp, prox, roll, adv, m = _three_policies(83, N=30)
+    m[:] = 1
+    roll[3] = -np.inf
+    prox[5] = np.nan
+    adv[7] = np.inf
+    out = O.decoupled_loss(logp, prox, roll, adv, m, 0.2, 0.28, 0.5, 2.0)
+    assert all(out["flags"][t] == O.FLAG_NONFINITE for t in (3, 5, 7))
+    assert out["counts"][3] == 3 and out["counts"][0] == 30 and np.isfinite(out["loss"])
