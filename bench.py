@@ -293,7 +293,7 @@ def workload_config(wl):
 
 # Algorithmic bytes per token of each O(N) kernel (reads + writes).
 ON_BYTES = {"gae_scan": 13, "policy_loss_fwd": 18, "policy_loss_bwd": 17, "value_loss": 13, "count_mask": 1,
-            "gae_count": 1}
+            "gae_count": 1, "decoupled_loss_fwd": 22, "decoupled_loss_bwd": 21}
 
 
 def bandwidth_study(args):
@@ -320,12 +320,20 @@ def bandwidth_study(args):
     one = torch.ones(1, device=dev)
     ws = sao.workspace(N)
 
+    # decoupled three-policy objective: pi_old = the stale log-probs, pi_rollout
+    # = pi_old with an engine mismatch (the generator's xi)
+    roll = t((wl.old_logp_syn + wl.xi).astype("float32"))
+    counts6 = torch.empty(6, dtype=torch.int64, device=dev)
+
     def calls():
         sao.sao_advantages(v, R, m, cu, wl.gamma, wl.lam, wl.lam_critic, 0.0, adv, ret, ws)
         sao.sao_advantages(v, R, m, cu, 1.0, 1.0, 1.0, 1.5, adv, ret, ws)
         sao.sao_policy_loss_fwd(lp, old, adv, m, wl.eps_low, wl.eps_high, loss, counts, ws, coef=coef, flags=flags)
         sao.sao_policy_loss_bwd(lp, old, adv, m, wl.eps_low, wl.eps_high, one, grad, ws)
         sao.sao_value_loss(v, ret, m, loss, dV, ws, ev_sums=ev)
+        sao.sao_decoupled_loss_fwd(lp, old, roll, adv, m, 0.2, 0.28, 0.5, 2.0, loss, counts6, ws, coef=coef,
+                                   flags=flags)
+        sao.sao_decoupled_loss_bwd(lp, old, roll, adv, m, 0.2, 0.28, 0.5, 2.0, one, grad, ws)
 
     for _ in range(max(3, args.warmup)):
         calls()

@@ -235,6 +235,45 @@ SAO_API sao_status sao_running_mean_advantages(const float *rewards, const int32
                                                const uint8_t *loss_mask, const int32_t *cu_seqlens, int64_t N,
                                                float *adv, void *ws, size_t ws_bytes, sao_stream_t stream);
 
+/* Extra per-token flag values written by sao_decoupled_loss_fwd. */
+#define SAO_FLAG_MISMATCH_LOW 5  /* w = pi_old / pi_rollout <= w_low: masked */
+#define SAO_FLAG_MISMATCH_HIGH 6 /* w >= w_high: masked */
+
+/*
+ * Decoupled three-policy objective, the mechanism that DIS simplifies (§3.1:
+ * pi_theta / pi_old corrects staleness, pi_old / pi_rollout the training /
+ * rollout mismatch, and tokens whose mismatch leaves a band are masked). With
+ *   r_t = exp(logp_t - prox_logp_t)          (pi_theta / pi_old)
+ *   w_t = exp(prox_logp_t - rollout_logp_t)  (pi_old / pi_rollout)
+ * a token is kept when it is an action token, both log-ratios and adv_t are
+ * finite and w_low < w_t < w_high (strict); then
+ *   loss = -(1/n) sum_t w_t min(r_t adv_t, clip(r_t, 1 - eps_low, 1 + eps_high) adv_t)
+ * with n = n_norm if n_norm > 0, else the number of action tokens. w is a
+ * detached coefficient: coef_t = d loss / d logp_t = -w_t r_t adv_t / n when
+ * the min keeps r_t adv_t (flag 0), and 0 when it is clipped (flag 1: adv < 0
+ * and r < 1 - eps_low; flag 2: adv > 0 and r > 1 + eps_high) or the token is
+ * masked (flags 3-6). Decisions are taken in fp32, the band before the clip.
+ *   logp, prox_logp, rollout_logp, adv [N] fp32; loss_mask [N] uint8
+ *   loss [1] fp32, coef [N] fp32 (nullable), flags [N] uint8 (nullable)
+ *   counts [6] int64 = {n_action, n_clip_low, n_clip_high, n_nonfinite,
+ *                       n_mismatch_low, n_mismatch_high}
+ * Scalars: eps_low, eps_high >= 0; 0 <= w_low < w_high (w_high may be +inf).
+ * Workspace from sao_workspace_bytes. Deterministic (fixed-order reductions).
+ */
+SAO_API sao_status sao_decoupled_loss_fwd(const float *logp, const float *prox_logp, const float *rollout_logp,
+                                          const float *adv, const uint8_t *loss_mask, int64_t N, float eps_low,
+                                          float eps_high, float w_low, float w_high, int64_t n_norm, float *loss,
+                                          float *coef, uint8_t *flags, int64_t *counts, void *ws, size_t ws_bytes,
+                                          sao_stream_t stream);
+
+/* grad_logp[t] = grad_loss[0] * coef[t] of sao_decoupled_loss_fwd, recomputed
+ * from the inputs (stateless); grad_loss is a device scalar. */
+SAO_API sao_status sao_decoupled_loss_bwd(const float *logp, const float *prox_logp, const float *rollout_logp,
+                                          const float *adv, const uint8_t *loss_mask, int64_t N, float eps_low,
+                                          float eps_high, float w_low, float w_high, int64_t n_norm,
+                                          const float *grad_loss, float *grad_logp, void *ws, size_t ws_bytes,
+                                          sao_stream_t stream);
+
 /*
  * sao_advantages without a workspace argument, for callers that cannot
  * allocate device memory: a host library that is handed only data pointers

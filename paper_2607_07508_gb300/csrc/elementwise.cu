@@ -1,4 +1,5 @@
-// Policy loss (Eq. 1-3, §3.1) and value loss (Preliminaries, §4.4) kernels.
+// Policy loss (Eq. 1-3, §3.1), the decoupled three-policy objective that DIS
+// simplifies (§3.1) and value loss (Preliminaries, §4.4) kernels.
 //
 // Both are HBM-bound streams over the packed tokens: 16-byte vector loads of
 // four tokens at a time, a grid of a few CTAs per SM striding over the input,
@@ -225,6 +226,154 @@ __global__ void __launch_bounds__(kThreads) policy_loss_finalize(
 }
 
 // ---------------------------------------------------------------------------
+// decoupled three-policy objective (§3.1)
+// ---------------------------------------------------------------------------
+struct DLArgs {
+  const float *logp, *prox, *roll, *adv;
+  const uint8_t *m;
+  int64_t N;
+  float lo, hi, wlo, whi;
+  int64_t n_norm;
+  const long long *cnt_partial;
+  int n_cnt;
+  float *coef;              // may be null
+  uint8_t *flags;           // may be null
+  const float *grad_scale;  // bwd: device scalar; fwd: null
+  double *loss_partial;
+  long long *cnt5_partial;  // [5][grid]
+};
+
+struct DLCounts {
+  int low = 0, high = 0, nonfin = 0, wlow = 0, whigh = 0;
+};
+
+// One token: the mismatch weight w = pi_old/pi_rollout must lie strictly
+// inside (wlo, whi); then the clipped surrogate of r = pi_theta/pi_old, scaled
+// by w. Adds the token's -loss contribution to `contrib`.
+__device__ __forceinline__ PLToken dl_token(float lp, float px, float ro, float a, uint8_t m, const DLArgs &A,
+                                            float inv_n, float &contrib, DLCounts &c) {
+  PLToken t{0.f, SAO_FLAG_NOT_ACTION};
+  if (!m) return t;
+  const float d = lp - px, e = px - ro;
+  if (!isfinite(d) || !isfinite(e) || !isfinite(a)) {
+    t.flag = SAO_FLAG_NONFINITE;
+    c.nonfin++;
+    return t;
+  }
+  const float w = expf(e);
+  if (w <= A.wlo) {
+    t.flag = SAO_FLAG_MISMATCH_LOW;
+    c.wlow++;
+    return t;
+  }
+  if (w >= A.whi) {
+    t.flag = SAO_FLAG_MISMATCH_HIGH;
+    c.whigh++;
+    return t;
+  }
+  const float r = expf(d);
+  if (a > 0.f && r > A.hi) {
+    t.flag = SAO_FLAG_HIGH;
+    c.high++;
+    contrib += w * (A.hi * a);
+  } else if (a < 0.f && r < A.lo) {
+    t.flag = SAO_FLAG_LOW;
+    c.low++;
+    contrib += w * (A.lo * a);
+  } else {
+    const float v = w * (r * a);
+    contrib += v;
+    t.flag = SAO_FLAG_IN;
+    t.coef = -v * inv_n;
+  }
+  return t;
+}
+
+template <bool kBwd>
+__global__ void __launch_bounds__(kThreads) decoupled_loss_kernel(DLArgs a) {
+  int64_t n = a.n_norm;
+  if (n <= 0) n = total_of(a.cnt_partial, a.n_cnt);
+  const float inv_n = n > 0 ? float(1.0 / double(n)) : 0.f;
+  const float gscale = kBwd ? __ldg(a.grad_scale) : 1.f;
+  double acc = 0.0;
+  DLCounts c;
+  const int64_t tid = int64_t(blockIdx.x) * kThreads + threadIdx.x;
+  const int64_t stride = int64_t(gridDim.x) * kThreads;
+  const bool vec = aligned16_dev(a.logp) && aligned16_dev(a.prox) && aligned16_dev(a.roll) &&
+                   aligned16_dev(a.adv) && ((reinterpret_cast<uintptr_t>(a.m) & 3u) == 0) &&
+                   (a.coef == nullptr || aligned16_dev(a.coef)) &&
+                   (a.flags == nullptr || (reinterpret_cast<uintptr_t>(a.flags) & 3u) == 0);
+  int64_t done = 0;
+  if (vec) {
+    const int64_t n4 = a.N / 4;
+    for (int64_t i = tid; i < n4; i += stride) {
+      const float4 lp = __ldcs(reinterpret_cast<const float4 *>(a.logp) + i);
+      const float4 px = __ldcs(reinterpret_cast<const float4 *>(a.prox) + i);
+      const float4 ro = __ldcs(reinterpret_cast<const float4 *>(a.roll) + i);
+      const float4 ad = __ldcs(reinterpret_cast<const float4 *>(a.adv) + i);
+      const uchar4 mk = __ldcs(reinterpret_cast<const uchar4 *>(a.m) + i);
+      float contrib = 0.f;
+      const PLToken t0 = dl_token(lp.x, px.x, ro.x, ad.x, mk.x, a, inv_n, contrib, c);
+      const PLToken t1 = dl_token(lp.y, px.y, ro.y, ad.y, mk.y, a, inv_n, contrib, c);
+      const PLToken t2 = dl_token(lp.z, px.z, ro.z, ad.z, mk.z, a, inv_n, contrib, c);
+      const PLToken t3 = dl_token(lp.w, px.w, ro.w, ad.w, mk.w, a, inv_n, contrib, c);
+      acc += double(contrib);
+      if (a.coef)
+        __stcs(reinterpret_cast<float4 *>(a.coef) + i,
+               make_float4(t0.coef * gscale, t1.coef * gscale, t2.coef * gscale, t3.coef * gscale));
+      if (a.flags) reinterpret_cast<uchar4 *>(a.flags)[i] = make_uchar4(t0.flag, t1.flag, t2.flag, t3.flag);
+    }
+    done = n4 * 4;
+  }
+  for (int64_t i = done + tid; i < a.N; i += stride) {
+    float contrib = 0.f;
+    const PLToken t = dl_token(__ldg(a.logp + i), __ldg(a.prox + i), __ldg(a.roll + i), __ldg(a.adv + i),
+                               __ldg(a.m + i), a, inv_n, contrib, c);
+    acc += double(contrib);
+    if (a.coef) a.coef[i] = t.coef * gscale;
+    if (a.flags) a.flags[i] = t.flag;
+  }
+  if (kBwd) return;
+  acc = block_sum(acc);
+  const long long k0 = block_sum((long long)c.low), k1 = block_sum((long long)c.high);
+  const long long k2 = block_sum((long long)c.nonfin), k3 = block_sum((long long)c.wlow);
+  const long long k4 = block_sum((long long)c.whigh);
+  if (threadIdx.x == 0) {
+    const int g = gridDim.x, b = blockIdx.x;
+    a.loss_partial[b] = acc;
+    a.cnt5_partial[b] = k0;
+    a.cnt5_partial[g + b] = k1;
+    a.cnt5_partial[2 * g + b] = k2;
+    a.cnt5_partial[3 * g + b] = k3;
+    a.cnt5_partial[4 * g + b] = k4;
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) decoupled_loss_finalize(const double *loss_partial,
+                                                                    const long long *cnt5_partial, int grid,
+                                                                    const long long *cnt_partial, int n_cnt,
+                                                                    int64_t n_norm, float *loss, int64_t *counts) {
+  const long long n_action = total_of(cnt_partial, n_cnt);
+  double s = 0.0;
+  long long k[5] = {0, 0, 0, 0, 0};
+  for (int i = threadIdx.x; i < grid; i += kThreads) {
+    s += loss_partial[i];
+#pragma unroll
+    for (int j = 0; j < 5; ++j) k[j] += cnt5_partial[j * grid + i];
+  }
+  s = block_sum(s);
+#pragma unroll
+  for (int j = 0; j < 5; ++j) k[j] = block_sum(k[j]);
+  if (threadIdx.x == 0) {
+    const long long n = n_norm > 0 ? n_norm : n_action;
+    *loss = n > 0 ? float(-s / double(n)) : 0.f;
+    counts[0] = n_action;
+#pragma unroll
+    for (int j = 0; j < 5; ++j) counts[1 + j] = k[j];
+  }
+}
+
+// ---------------------------------------------------------------------------
 // value loss
 // ---------------------------------------------------------------------------
 // Compensated fp32 accumulator (Knuth two-sum): sums millions of terms with
@@ -415,6 +564,52 @@ sao_status policy_loss_launch(const float *logp, const float *old, const float *
   SAO_TRY(launch_end(slot, s));
   slot = launch_begin("policy_loss_finalize", s);
   policy_loss_finalize<<<1, kThreads, 0, s>>>(lossp, cnt3, grid, cnt, grid, n_norm, loss, counts);
+  return launch_end(slot, s);
+}
+
+sao_status decoupled_loss_launch(const float *logp, const float *prox, const float *roll, const float *adv,
+                                 const uint8_t *m, int64_t N, float eps_low, float eps_high, float w_low,
+                                 float w_high, int64_t n_norm, float *loss, float *coef, uint8_t *flags,
+                                 int64_t *counts, const float *grad_loss, void *ws_body, size_t body_bytes,
+                                 cudaStream_t s) {
+  const int grid =
+      grad_loss ? stream_grid(N, decoupled_loss_kernel<true>) : stream_grid(N, decoupled_loss_kernel<false>);
+  Carver c(ws_body, body_bytes);
+  long long *cnt = c.take<long long>(grid);
+  double *lossp = c.take<double>(grid);
+  long long *cnt5 = c.take<long long>(5 * size_t(grid));
+  if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the decoupled loss");
+  const bool need_count = (n_norm <= 0) || (grad_loss == nullptr);
+  if (need_count) SAO_TRY(launch_count(m, N, cnt, grid, s));
+  DLArgs a;
+  a.logp = logp;
+  a.prox = prox;
+  a.roll = roll;
+  a.adv = adv;
+  a.m = m;
+  a.N = N;
+  a.lo = 1.0f - eps_low;
+  a.hi = 1.0f + eps_high;
+  a.wlo = w_low;
+  a.whi = w_high;
+  a.n_norm = n_norm;
+  a.cnt_partial = cnt;
+  a.n_cnt = need_count ? grid : 0;
+  a.coef = coef;
+  a.flags = flags;
+  a.grad_scale = grad_loss;
+  a.loss_partial = lossp;
+  a.cnt5_partial = cnt5;
+  if (grad_loss) {
+    int slot = launch_begin("decoupled_loss_bwd", s);
+    decoupled_loss_kernel<true><<<grid, kThreads, 0, s>>>(a);
+    return launch_end(slot, s);
+  }
+  int slot = launch_begin("decoupled_loss_fwd", s);
+  decoupled_loss_kernel<false><<<grid, kThreads, 0, s>>>(a);
+  SAO_TRY(launch_end(slot, s));
+  slot = launch_begin("decoupled_loss_finalize", s);
+  decoupled_loss_finalize<<<1, kThreads, 0, s>>>(lossp, cnt5, grid, cnt, grid, n_norm, loss, counts);
   return launch_end(slot, s);
 }
 

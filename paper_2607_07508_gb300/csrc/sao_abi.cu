@@ -225,6 +225,52 @@ sao_status sao_policy_loss_bwd(const float *logp, const float *old_logp, const f
   return finish_call(ws, s);
 }
 
+static sao_status check_band(float w_low, float w_high) {
+  if (!(w_low >= 0.f) || !(w_high > w_low) || isnan(w_low) || isnan(w_high))
+    return fail(SAO_ERR_INVALID_ARG, "mismatch band needs 0 <= w_low < w_high (w_low = %g, w_high = %g)", w_low,
+                w_high);
+  return SAO_OK;
+}
+
+sao_status sao_decoupled_loss_fwd(const float *logp, const float *prox_logp, const float *rollout_logp,
+                                  const float *adv, const uint8_t *loss_mask, int64_t N, float eps_low,
+                                  float eps_high, float w_low, float w_high, int64_t n_norm, float *loss,
+                                  float *coef, uint8_t *flags, int64_t *counts, void *ws, size_t ws_bytes,
+                                  sao_stream_t stream) {
+  if (N < 0) return fail(SAO_ERR_SHAPE, "N < 0");
+  SAO_TRY(check_eps(eps_low, eps_high));
+  SAO_TRY(check_band(w_low, w_high));
+  if (!loss || !counts) return fail(SAO_ERR_INVALID_ARG, "NULL loss or counts");
+  if (N > 0 && (!logp || !prox_logp || !rollout_logp || !adv || !loss_mask))
+    return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
+  Ws w;
+  SAO_TRY(take_ws(ws, ws_bytes, elementwise_ws_bytes(N, 0), &w));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  SAO_TRY(begin_call(ws, s));
+  SAO_TRY(decoupled_loss_launch(logp, prox_logp, rollout_logp, adv, loss_mask, N, eps_low, eps_high, w_low, w_high,
+                                n_norm, loss, coef, flags, counts, nullptr, w.body, w.body_bytes, s));
+  return finish_call(ws, s);
+}
+
+sao_status sao_decoupled_loss_bwd(const float *logp, const float *prox_logp, const float *rollout_logp,
+                                  const float *adv, const uint8_t *loss_mask, int64_t N, float eps_low,
+                                  float eps_high, float w_low, float w_high, int64_t n_norm, const float *grad_loss,
+                                  float *grad_logp, void *ws, size_t ws_bytes, sao_stream_t stream) {
+  if (N < 0) return fail(SAO_ERR_SHAPE, "N < 0");
+  SAO_TRY(check_eps(eps_low, eps_high));
+  SAO_TRY(check_band(w_low, w_high));
+  if (N == 0) return SAO_OK;
+  if (!logp || !prox_logp || !rollout_logp || !adv || !loss_mask || !grad_loss || !grad_logp)
+    return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
+  Ws w;
+  SAO_TRY(take_ws(ws, ws_bytes, elementwise_ws_bytes(N, 0), &w));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  SAO_TRY(begin_call(ws, s));
+  SAO_TRY(decoupled_loss_launch(logp, prox_logp, rollout_logp, adv, loss_mask, N, eps_low, eps_high, w_low, w_high,
+                                n_norm, nullptr, grad_logp, nullptr, nullptr, grad_loss, w.body, w.body_bytes, s));
+  return finish_call(ws, s);
+}
+
 sao_status sao_value_loss(const float *values, const float *ret, const uint8_t *loss_mask, int64_t N, float *loss,
                           float *grad_values, double *ev_sums, void *ws, size_t ws_bytes, sao_stream_t stream) {
   if (N < 0) return fail(SAO_ERR_SHAPE, "N < 0");

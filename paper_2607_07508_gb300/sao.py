@@ -23,12 +23,14 @@ SAO_NORM_TOKEN, SAO_NORM_SEQUENCE = 0, 1
 STATUS = {0: "SAO_OK", 1: "SAO_ERR_INVALID_ARG", 2: "SAO_ERR_SHAPE", 3: "SAO_ERR_WORKSPACE",
           4: "SAO_ERR_UNSUPPORTED", 5: "SAO_ERR_CUDA", 6: "SAO_ERR_DEVICE_CHECK"}
 FLAG_IN, FLAG_LOW, FLAG_HIGH, FLAG_NONFINITE, FLAG_NOT_ACTION = 0, 1, 2, 3, 4
+FLAG_MISMATCH_LOW, FLAG_MISMATCH_HIGH = 5, 6
 
 EXPORTS = ("sao_version", "sao_last_error_string", "sao_set_checked", "sao_get_checked",
            "sao_set_dz_budget_bytes", "sao_workspace_bytes", "sao_token_logprobs_fwd",
            "sao_token_logprobs_bwd", "sao_advantages", "sao_advantages_noalloc", "sao_step_advantages",
            "sao_policy_loss_fwd", "sao_policy_loss_bwd", "sao_clip_loss_fwd", "sao_clip_loss_bwd",
-           "sao_group_advantages", "sao_running_mean_advantages",
+           "sao_group_advantages", "sao_running_mean_advantages", "sao_decoupled_loss_fwd",
+           "sao_decoupled_loss_bwd",
            "sao_value_loss", "sao_profile_enable", "sao_profile_reset", "sao_profile_read")
 
 
@@ -67,6 +69,8 @@ def load(path: Optional[str] = None):
         "sao_step_advantages": (ctypes.c_int, [P, P, P, P, I32, I64, F, F, F, F, ctypes.c_int, P, P, P, P, SZ, P]),
         "sao_policy_loss_fwd": (ctypes.c_int, [P, P, P, P, I64, F, F, I64, P, P, P, P, P, SZ, P]),
         "sao_policy_loss_bwd": (ctypes.c_int, [P, P, P, P, I64, F, F, I64, P, P, P, SZ, P]),
+        "sao_decoupled_loss_fwd": (ctypes.c_int, [P, P, P, P, P, I64, F, F, F, F, I64, P, P, P, P, P, SZ, P]),
+        "sao_decoupled_loss_bwd": (ctypes.c_int, [P, P, P, P, P, I64, F, F, F, F, I64, P, P, P, SZ, P]),
         "sao_value_loss": (ctypes.c_int, [P, P, P, I64, P, P, P, P, SZ, P]),
         "sao_clip_loss_fwd": (ctypes.c_int, [P, P, P, P, P, I32, I64, F, F, ctypes.c_int, P, P, P, P, P, SZ, P]),
         "sao_clip_loss_bwd": (ctypes.c_int, [P, P, P, P, P, I32, I64, F, F, ctypes.c_int, P, P, P, SZ, P]),
@@ -260,6 +264,36 @@ def sao_policy_loss_bwd(logp, old_logp, adv, loss_mask, eps_low, eps_high, grad_
     _check(load().sao_policy_loss_bwd(_ptr(logp), _ptr(old_logp), _ptr(adv), _ptr(loss_mask), N, float(eps_low),
                                       float(eps_high), int(n_norm), _ptr(grad_loss), _ptr(grad_logp), _ptr(ws),
                                       ws.numel(), _stream(stream)))
+
+
+def sao_decoupled_loss_fwd(logp, prox_logp, rollout_logp, adv, loss_mask, eps_low, eps_high, w_low, w_high, loss,
+                           counts, ws, coef=None, flags=None, n_norm=0, stream=None):
+    N = logp.numel()
+    for t, name in ((logp, "logp"), (prox_logp, "prox_logp"), (rollout_logp, "rollout_logp"), (adv, "adv")):
+        _expect(t, torch.float32, N, name)
+    _expect(loss_mask, torch.uint8, N, "loss_mask")
+    _expect(coef, torch.float32, N, "coef")
+    _expect(flags, torch.uint8, N, "flags")
+    _expect(loss, torch.float32, 1, "loss")
+    _expect(counts, torch.int64, 6, "counts")
+    _check(load().sao_decoupled_loss_fwd(_ptr(logp), _ptr(prox_logp), _ptr(rollout_logp), _ptr(adv),
+                                         _ptr(loss_mask), N, float(eps_low), float(eps_high), float(w_low),
+                                         float(w_high), int(n_norm), _ptr(loss), _ptr(coef), _ptr(flags),
+                                         _ptr(counts), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def sao_decoupled_loss_bwd(logp, prox_logp, rollout_logp, adv, loss_mask, eps_low, eps_high, w_low, w_high,
+                           grad_loss, grad_logp, ws, n_norm=0, stream=None):
+    N = logp.numel()
+    for t, name in ((logp, "logp"), (prox_logp, "prox_logp"), (rollout_logp, "rollout_logp"), (adv, "adv"),
+                    (grad_logp, "grad_logp")):
+        _expect(t, torch.float32, N, name)
+    _expect(loss_mask, torch.uint8, N, "loss_mask")
+    _expect(grad_loss, torch.float32, 1, "grad_loss")
+    _check(load().sao_decoupled_loss_bwd(_ptr(logp), _ptr(prox_logp), _ptr(rollout_logp), _ptr(adv),
+                                         _ptr(loss_mask), N, float(eps_low), float(eps_high), float(w_low),
+                                         float(w_high), int(n_norm), _ptr(grad_loss), _ptr(grad_logp), _ptr(ws),
+                                         ws.numel(), _stream(stream)))
 
 
 def sao_value_loss(values, ret, loss_mask, loss, grad_values, ws, ev_sums=None, stream=None):

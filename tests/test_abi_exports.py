@@ -83,3 +83,16 @@ def test_argument_errors_without_gpu(lib):
     assert st == 2
     msg = lib.sao_last_error_string().decode()
     assert "trajectory" in msg
+
+
+def test_decoupled_loss_argument_errors_without_gpu(lib):
+    P = ctypes.c_void_p
+    # mismatch band must satisfy 0 <= w_low < w_high
+    for wl_, wh in ((2.0, 0.5), (1.0, 1.0), (-0.1, 2.0), (float("nan"), 2.0)):
+        st = lib.sao_decoupled_loss_fwd(None, None, None, None, None, 0, 0.2, 0.28, wl_, wh, 0, P(8), None, None,
+                                        P(8), None, 0, None)
+        assert st == 1
+        assert "band" in lib.sao_last_error_string().decode()
+    st = lib.sao_decoupled_loss_bwd(None, None, None, None, None, 0, -1.0, 0.28, 0.5, 2.0, 0, None, None, None, 0,
+                                    None)
+    assert st == 1

@@ -152,3 +152,93 @@ def test_running_mean_advantages_match_oracle():
             assert rel_err_floor(adv.cpu().numpy(), want, 1e-3).max() <= 1e-5
             assert np.array_equal(seen_d.cpu().numpy(), seen_o)
             assert np.allclose(hist_d.cpu().numpy(), hist_o)
+
+
+# ---------------------------------------------------------------------------
+# decoupled three-policy objective (§3.1)
+# ---------------------------------------------------------------------------
+
+def _three_policy_inputs(wl, seed):
+    """pi_theta = the synthetic log-probs, pi_old = the stale ones, pi_rollout =
+    pi_old with an engine mismatch of N(0, 0.3) in log space."""
+    rng = np.random.default_rng(seed)
+    prox = wl.old_logp_syn.astype(np.float32)
+    roll = (prox + rng.normal(0, 0.3, wl.N)).astype(np.float32)
+    adv = rng.normal(size=wl.N).astype(np.float32)
+    return wl.logp_syn.astype(np.float32), prox, roll, adv
+
+
+def _decoupled_gpu(logp, prox, roll, adv, mask, el, eh, wl_, wh, n_norm=0):
+    N = len(logp)
+    loss = torch.empty(1, device="cuda")
+    counts = torch.empty(6, dtype=torch.int64, device="cuda")
+    coef = torch.full((N,), float("nan"), device="cuda")
+    flags = torch.full((N,), 9, dtype=torch.uint8, device="cuda")
+    grad = torch.full((N,), float("nan"), device="cuda")
+    ws = sao.workspace(N)
+    args = [cuda(x) for x in (logp, prox, roll, adv, mask)]
+    sao.sao_decoupled_loss_fwd(*args, el, eh, wl_, wh, loss, counts, ws, coef=coef, flags=flags, n_norm=n_norm)
+    sao.sao_decoupled_loss_bwd(*args, el, eh, wl_, wh, torch.tensor([0.5], device="cuda"), grad, ws, n_norm=n_norm)
+    torch.cuda.synchronize()
+    return float(loss.item()), counts.cpu().numpy(), coef.cpu().numpy(), flags.cpu().numpy(), grad.cpu().numpy()
+
+
+def _near_decoupled_bound(logp, prox, roll, el, eh, wl_, wh, tol=1e-6):
+    f64 = lambda x: np.asarray(x, np.float64)
+    with np.errstate(all="ignore"):
+        r = np.exp(f64(logp) - f64(prox))
+        w = np.exp(f64(prox) - f64(roll))
+        return ((np.abs(r - (1 - el)) <= tol) | (np.abs(r - (1 + eh)) <= tol) | (np.abs(w - wl_) <= tol) |
+                (np.abs(w - wh) <= tol))
+
+
+def _check_decoupled(logp, prox, roll, adv, mask, el, eh, wl_, wh, n_norm=0):
+    loss, counts, coef, flags, grad = _decoupled_gpu(logp, prox, roll, adv, mask, el, eh, wl_, wh, n_norm)
+    want = O.decoupled_loss(logp, prox, roll, adv, mask, el, eh, wl_, wh, n_norm)
+    skip = _near_decoupled_bound(logp, prox, roll, el, eh, wl_, wh)
+    keep = ~skip
+    assert np.array_equal(flags[keep], want["flags"][keep])
+    if not skip.any():
+        assert np.array_equal(counts, want["counts"])
+    assert abs(loss - want["loss"]) <= 1e-4 * max(abs(want["loss"]), 1e-6)
+    assert rel_err_floor(coef[keep], want["coef"][keep], 1e-12).max() <= 1e-5
+    assert rel_err_floor(grad[keep], 0.5 * want["coef"][keep], 1e-12).max() <= 1e-5
+    return want
+
+
+@pytest.mark.parametrize("name", S.CONFIG_NAMES)
+def test_decoupled_loss_match_oracle(name):
+    wl = S.make_workload(name, dense=False)
+    logp, prox, roll, adv = _three_policy_inputs(wl, 11)
+    want = _check_decoupled(logp, prox, roll, adv, wl.loss_mask, 0.2, 0.28, 0.5, 2.0)
+    assert want["counts"][4] + want["counts"][5] > 0      # the band masks some tokens
+
+
+def test_decoupled_loss_edge_layouts():
+    """Ragged length (not a multiple of 4), non-finite log-probs and advantages,
+    masked tokens, an external normaliser and an open upper band."""
+    rng = np.random.default_rng(12)
+    N = 4099
+    logp = (-rng.exponential(2.0, N)).astype(np.float32)
+    prox = (logp + rng.normal(0, 0.4, N)).astype(np.float32)
+    roll = (prox + rng.normal(0, 0.6, N)).astype(np.float32)
+    adv = rng.normal(size=N).astype(np.float32)
+    mask = (rng.random(N) < 0.7).astype(np.uint8)
+    roll[::97] = -np.inf
+    prox[5::101] = np.nan
+    adv[7::89] = np.inf
+    _check_decoupled(logp, prox, roll, adv, mask, 0.3, 5.0, 0.25, 4.0)
+    _check_decoupled(logp, prox, roll, adv, mask, 0.3, 5.0, 0.0, float("inf"), n_norm=1000)
+    _check_decoupled(logp[:3], prox[:3], roll[:3], adv[:3], mask[:3], 0.2, 0.28, 0.5, 2.0)
+
+
+def test_decoupled_loss_equal_old_and_rollout_matches_clip_loss_kernel():
+    """pi_old = pi_rollout: the decoupled kernel and the clipped-surrogate
+    kernel agree token by token (two independent kernels)."""
+    wl = S.make_workload("moe", dense=False)
+    logp, prox, _, adv = _three_policy_inputs(wl, 13)
+    d = _decoupled_gpu(logp, prox, prox, adv, wl.loss_mask, 0.2, 0.28, 0.5, 2.0)
+    c = _clip_gpu(logp, prox, adv, wl.loss_mask, wl.cu_seqlens, 0.2, 0.28, sao.SAO_NORM_TOKEN)
+    assert np.array_equal(d[3], c[3]) and np.array_equal(d[1][:4], c[1])
+    assert abs(d[0] - c[0]) <= 1e-5 * max(abs(c[0]), 1e-6)
+    assert rel_err_floor(d[2], c[2], 1e-12).max() <= 1e-6
