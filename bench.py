@@ -140,7 +140,7 @@ class ClockSampler:
 class LossHeadStep:
     """Device buffers and the six ABI calls of one loss-head step."""
 
-    def __init__(self, wl, device, torch):
+    def __init__(self, wl, device, torch, cached=True):
         from paper_2607_07508_gb300 import sao
         self.sao = sao
         self.torch = torch
@@ -175,6 +175,15 @@ class LossHeadStep:
         # workload's staleness noise (prepared once, outside any timing).
         sao.sao_token_logprobs_fwd(self.H, self.W, self.y, self.logp, self.lse, self.ws)
         self.old = (self.logp + torch.as_tensor(wl.xi).to(dev)).contiguous()
+        # The forward keeps its probabilities (bf16, about 2*N*V bytes) for the
+        # backward when they fit next to everything else; else the backward
+        # recomputes the logits.
+        self.cache = None
+        if cached and self.H.dtype == torch.bfloat16:
+            need = sao.sao_logprob_cache_bytes(N, V)
+            free, _ = torch.cuda.mem_get_info(dev)
+            if need + (4 << 30) < free:
+                self.cache = sao.logprob_cache(N, V, device=dev)
 
     def run(self):
         s, wl = self.sao, self.wl
@@ -182,12 +191,20 @@ class LossHeadStep:
                          self.adv, self.ret, self.ws)
         s.sao_value_loss(self.values, self.ret, self.mask, self.vloss, self.dV, self.ws, ev_sums=self.ev)
         # log-probs of observation tokens are never read: skip those rows
-        s.sao_token_logprobs_fwd(self.H, self.W, self.y, self.logp, self.lse, self.ws, row_mask=self.mask)
+        if self.cache is not None:
+            s.sao_token_logprobs_fwd_cached(self.H, self.W, self.y, self.logp, self.lse, self.cache, self.ws,
+                                            row_mask=self.mask)
+        else:
+            s.sao_token_logprobs_fwd(self.H, self.W, self.y, self.logp, self.lse, self.ws, row_mask=self.mask)
         s.sao_policy_loss_fwd(self.logp, self.old, self.adv, self.mask, wl.eps_low, wl.eps_high, self.loss,
                               self.counts, self.ws, coef=self.coef, flags=self.flags)
         s.sao_policy_loss_bwd(self.logp, self.old, self.adv, self.mask, wl.eps_low, wl.eps_high, self.one, self.G,
                               self.ws)
-        s.sao_token_logprobs_bwd(self.H, self.W, self.y, self.lse, self.G, self.dH, self.dW, self.ws)
+        if self.cache is not None:
+            s.sao_token_logprobs_bwd_cached(self.H, self.W, self.y, self.lse, self.G, self.dH, self.dW, self.cache,
+                                            self.ws)
+        else:
+            s.sao_token_logprobs_bwd(self.H, self.W, self.y, self.lse, self.G, self.dH, self.dW, self.ws)
 
 
 # Algorithmic work per launch of each tensor-core kernel, in flops: the
@@ -370,6 +387,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--tokens", type=int, default=None,
                     help="override the packed token count (smaller cases for profiling captures)")
+    ap.add_argument("--recompute", action="store_true",
+                    help="backward recomputes the logits instead of reading the forward's stored probabilities")
     ap.add_argument("--bandwidth-study", action="store_true",
                     help="time the O(N) kernels alone on the 2^27-token bandwidth workload")
     args = ap.parse_args()
@@ -392,7 +411,7 @@ def main():
 
     wl = S.make_workload(WORKLOAD, device=dev, seed=S.SEED_BASE + S.CONFIG_NAMES.index(WORKLOAD) + 97 * rank,
                          N_override=args.tokens)
-    step = LossHeadStep(wl, dev, torch)
+    step = LossHeadStep(wl, dev, torch, cached=not args.recompute)
     stream = torch.cuda.current_stream()
     for _ in range(max(3, args.warmup)):
         step.run()
@@ -451,8 +470,9 @@ def main():
     else:
         roofline = {"bound": "hbm", "kernel": dom_name, "achieved": None, "peak": peaks.get("hbm_gbs"),
                     "unit": "GB/s", "frac": None, "traffic": None}
+    cached = step.cache is not None
     step_alg = 2.0 * wl.h * wl.V * (rows_fwd + 2 * rows_bwd)
-    step_exec = 2.0 * wl.h * wl.V * (rows_fwd + 3 * rows_bwd)
+    step_exec = 2.0 * wl.h * wl.V * (rows_fwd + (2 if cached else 3) * rows_bwd)
     burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
     step_roof = {"algorithmic_tflops": step_alg / (ms / 1000) / 1e12,
                  "frac_of_burst_peak": step_alg / (ms / 1000) / 1e12 / burst,
@@ -461,7 +481,10 @@ def main():
                  "algorithmic_flops_per_step": f"2hV per forward row ({rows_fwd} action tokens) + 4hV per row "
                                                f"with a non-zero gradient ({rows_bwd}); 6*N*h*V = "
                                                f"{6.0 * wl.N * wl.h * wl.V:.4g} if no row were skipped",
-                 "executed_flops_per_step": "algorithmic + 2hV per backward row (the logits are recomputed)",
+                 "executed_flops_per_step": ("algorithmic (the backward reads the forward's stored bf16 "
+                                             "probabilities: no logit recompute)" if cached else
+                                             "algorithmic + 2hV per backward row (the logits are recomputed)"),
+                 "logprob_path": "cached" if cached else "recompute",
                  "rows_forward": rows_fwd, "rows_backward": rows_bwd,
                  "peak_source": peak_src}
     kernels = {k: {"launches": n, "avg_ms": t / n} for k, (n, t) in sorted(prof.items(), key=lambda kv: -kv[1][1])}

@@ -79,6 +79,7 @@ typedef enum sao_dtype {
 #define SAO_DEVERR_CU_SEQLENS 0x2u   /* cu_seqlens not 0..N non-decreasing */
 #define SAO_DEVERR_SCAN_TIMEOUT 0x4u /* advantage scan gave up waiting for a carry */
 #define SAO_DEVERR_PIPE_TIMEOUT 0x8u /* a GEMM pipeline wait gave up */
+#define SAO_DEVERR_CACHE_ROW 0x10u   /* cached backward: a row with grad != 0 the forward skipped */
 
 /* Library version, major * 10000 + minor * 100 + patch. */
 SAO_API int sao_version(void);
@@ -129,6 +130,34 @@ SAO_API sao_status sao_token_logprobs_bwd(const void *H, const void *W, sao_dtyp
                                   const float *lse, const float *grad_logp, int64_t N, int32_t h,
                                   int32_t V, void *dH, float *dW, int accumulate_dW, void *ws,
                                   size_t ws_bytes, sao_stream_t stream);
+
+/*
+ * The same two calls with the forward's probabilities kept for the backward
+ * (bf16 only). The forward additionally stores, for every row it computes,
+ * e[t, v] = exp(z[t, v] - m) in bf16, m being the maximum of z[t, .] over the
+ * 256-wide vocabulary tile holding v, with those maxima; the backward forms
+ * p[t, v] = e[t, v] exp(m - lse[t]) from them, so dZ costs one pass over the
+ * stored rows instead of recomputing the logits (2 h V flops per row). The
+ * results match sao_token_logprobs_fwd / _bwd within the bf16 rounding of e.
+ *   cache        caller-owned device buffer of sao_logprob_cache_bytes(N, V)
+ *                bytes (about 2 N V bytes), 256-byte aligned; written by the
+ *                forward, read (not modified) by the backward, which must get
+ *                the same H, W, y, N, V and the forward's lse
+ * A backward row with grad_logp != 0 that the forward skipped (row_mask 0)
+ * has no stored probabilities: it contributes nothing and raises
+ * SAO_DEVERR_CACHE_ROW. Other arguments as the uncached calls; SAO_F32 gives
+ * SAO_ERR_UNSUPPORTED.
+ */
+SAO_API size_t sao_logprob_cache_bytes(int64_t N, int32_t V);
+SAO_API sao_status sao_token_logprobs_fwd_cached(const void *H, const void *W, sao_dtype dt, const int32_t *y,
+                                                 const uint8_t *row_mask, int64_t N, int32_t h, int32_t V,
+                                                 float *logp, float *lse, void *cache, size_t cache_bytes, void *ws,
+                                                 size_t ws_bytes, sao_stream_t stream);
+SAO_API sao_status sao_token_logprobs_bwd_cached(const void *H, const void *W, sao_dtype dt, const int32_t *y,
+                                                 const float *lse, const float *grad_logp, int64_t N, int32_t h,
+                                                 int32_t V, void *dH, float *dW, int accumulate_dW,
+                                                 const void *cache, size_t cache_bytes, void *ws, size_t ws_bytes,
+                                                 sao_stream_t stream);
 
 /*
  * Skip-observation GAE (Preliminaries; §3.2 Eq. 4-5; §4.1). For trajectory b

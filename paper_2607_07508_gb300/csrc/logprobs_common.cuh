@@ -1,6 +1,7 @@
 // Pieces shared by the fp32 and tensor-core log-prob paths.
 #pragma once
 
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -25,12 +26,24 @@ sao_status simt_bwd(const float *H, const float *W, const int32_t *y, const floa
                     int64_t N, int32_t h, int32_t V, float *dH, float *dW, int accumulate, void *ws,
                     size_t ws_bytes, cudaStream_t s);
 
+// The forward's stored probabilities (tensor-core path): e[f, v] =
+// exp(z - max_tile) in bf16 for forward row f, the per-(tile, row) partials
+// (max_tile, sum-exp) and the forward row of every token (-1: not computed).
+struct LogprobCache {
+  __nv_bfloat16 *e;   // [rows, lde]
+  int64_t lde, rows;
+  float2 *part;       // [ceil(V/256), N]
+  int *pos;           // [N]
+  size_t bytes;       // total size of the cache buffer
+};
+LogprobCache logprob_cache_view(void *base, int64_t N, int32_t V);
+
 size_t tc_ws_bytes(int64_t N, int32_t h, int32_t V);
 sao_status tc_fwd(const void *H, const void *W, const int32_t *y, const uint8_t *row_mask, int64_t N,
                   int32_t h, int32_t V, float *logp, float *lse, unsigned int *err, void *ws, size_t ws_bytes,
-                  cudaStream_t s);
+                  const LogprobCache *cache, cudaStream_t s);
 sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *lse, const float *G,
                   int64_t N, int32_t h, int32_t V, void *dH, float *dW, int accumulate, unsigned int *err,
-                  void *ws, size_t ws_bytes, cudaStream_t s);
+                  void *ws, size_t ws_bytes, const LogprobCache *cache, cudaStream_t s);
 
 }  // namespace sao

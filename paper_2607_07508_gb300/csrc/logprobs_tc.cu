@@ -49,7 +49,12 @@ constexpr size_t SMEM_BYTES = 1024 + size_t(STAGES) * STAGE_BYTES + 2 * STAGE_OU
 constexpr int EPI_BARRIER = 1;                    // named barrier of the 4 epilogue warps
 constexpr float kLog2e = 1.4426950408889634f;
 
-enum EpiKind : int { kSoftmax = 0, kDLogits = 1, kStoreF32 = 2, kStoreBF16 = 3 };
+enum EpiKind : int { kSoftmax = 0, kDLogits = 1, kStoreF32 = 2, kStoreBF16 = 3, kSoftmaxStore = 4 };
+
+// Epilogues that stage bf16 boxes in shared memory and write them with TMA
+// stores; their 4 warps synchronise with named barriers.
+template <int kEpi>
+constexpr bool kTmaStoreEpi = (kEpi == kDLogits || kEpi == kSoftmaxStore);
 
 struct GemmParams {
   int nM, nN, nK;      // tiles along M, N and 64-wide K blocks
@@ -252,7 +257,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       bool ok = mbar_wait(smem_u32(&ctl->acc_full[acc]), acc_phase, abort, p.err);
       // The dlogits epilogue synchronises its 4 warps with named barriers, so
       // they must agree on whether this tile goes ahead.
-      if constexpr (kEpi == kDLogits) ok = named_barrier_and(EPI_BARRIER, 128, ok);
+      if constexpr (kTmaStoreEpi<kEpi>) ok = named_barrier_and(EPI_BARRIER, 128, ok);
       if (!ok) break;
       fence_after_sync();
       const uint32_t taddr = tmem_base + (uint32_t(quad * 32) << 16) + uint32_t(acc) * BN;
@@ -296,6 +301,82 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         fence_before_sync();
         mbar_arrive(smem_u32(&ctl->acc_empty[acc]));
+        if (row_ok) {
+          p.part[int64_t(n) * p.rows + row] = make_float2(mx, sm);  // compacted row, stride N
+          if (have) p.zy[row] = zsel;
+        }
+      } else if constexpr (kEpi == kSoftmaxStore) {
+        // As kSoftmax, but the tile's maximum is taken first (one pass over
+        // TMEM), so the second pass can also store e = exp(z - max_tile) as
+        // bf16: the backward then forms p = e * exp(max_tile - lse) instead of
+        // recomputing the logits. Boxes of 128 rows x 64 columns go out through
+        // two swizzled staging buffers and TMA stores issued by one thread.
+        const bool issuer = (warp == 2 && lane == 0);
+        const int col0 = n * BN;
+        const int yy = row_ok ? __ldg(p.y + orig) : -1;
+        float mx = -INFINITY;
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t u[32];
+          tmem_ld32(taddr + c * 32, u);
+          tmem_wait_ld();
+          const int valid = p.vocab - (col0 + c * 32);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) mx = (j < valid) ? fmaxf(mx, __uint_as_float(u[j])) : mx;
+        }
+        const float off = -mx * kLog2e;
+        float sm = 0.f, zsel = 0.f;
+        bool have = false;
+#pragma unroll 1
+        for (int box = 0; box < BN / 64; ++box) {
+          const uint32_t buf = out_base + uint32_t(box & 1) * STAGE_OUT_BYTES;
+          if (issuer) bulk_wait_group_read<1>();  // the store that last read `buf` is done
+          named_barrier(EPI_BARRIER, 128);
+#pragma unroll
+          for (int half = 0; half < 2; ++half) {
+            const int c = box * 2 + half;
+            uint32_t u[32];
+            tmem_ld32(taddr + c * 32, u);
+            tmem_wait_ld();
+            if (c == BN / 32 - 1) {
+              fence_before_sync();
+              mbar_arrive(smem_u32(&ctl->acc_empty[acc]));
+            }
+            const int cbase = col0 + c * 32;
+            const int valid = p.vocab - cbase;
+            uint32_t pk[16];
+#pragma unroll
+            for (int j = 0; j < 32; j += 2) {
+              const float e0 = (j < valid) ? ex2_approx(fmaf(__uint_as_float(u[j]), kLog2e, off)) : 0.f;
+              const float e1 = (j + 1 < valid) ? ex2_approx(fmaf(__uint_as_float(u[j + 1]), kLog2e, off)) : 0.f;
+              sm += e0 + e1;
+              const __nv_bfloat162 b2 = __floats2bfloat162_rn(e0, e1);
+              pk[j / 2] = *reinterpret_cast<const uint32_t *>(&b2);
+            }
+            const unsigned rel = unsigned(yy - cbase);
+            if (rel < 32u) {
+              float z = __uint_as_float(u[0]);
+#pragma unroll
+              for (int j = 1; j < 32; ++j) z = (unsigned(j) == rel) ? __uint_as_float(u[j]) : z;
+              zsel = z;
+              have = true;
+            }
+            const uint32_t row_addr = buf + uint32_t(r) * 128u;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const uint32_t chunk = uint32_t(half * 4 + q) ^ uint32_t(r & 7);
+              asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(row_addr + chunk * 16u),
+                           "r"(pk[4 * q]), "r"(pk[4 * q + 1]), "r"(pk[4 * q + 2]), "r"(pk[4 * q + 3])
+                           : "memory");
+            }
+          }
+          fence_proxy_async_smem();
+          named_barrier(EPI_BARRIER, 128);
+          if (issuer) {
+            tma_store_2d(&map_c, buf, col0 + box * 64, m * BM);
+            bulk_commit_group();
+          }
+        }
         if (row_ok) {
           p.part[int64_t(n) * p.rows + row] = make_float2(mx, sm);  // compacted row, stride N
           if (have) p.zy[row] = zsel;
@@ -420,7 +501,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   }
 
-  if constexpr (kEpi == kDLogits) {
+  if constexpr (kTmaStoreEpi<kEpi>) {
     if (warp == 2 && lane == 0) bulk_wait_group<0>();
   }
   fence_before_sync();
@@ -429,6 +510,79 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     fence_after_sync();
     tmem_dealloc(tmem_base, TMEM_COLS);
   }
+}
+
+// ---------------------------------------------------------------------------
+// backward from the forward's stored probabilities
+// ---------------------------------------------------------------------------
+// dZ[i, v - v0] = G_t (1[v == y_t] - e[f, v] exp(max[tile(v), f] - lse_t)) for
+// the compacted backward row i (token t = idx[i], forward row f = pos[t]) and
+// v in [v0, v0 + vc): one CTA per row, 16-byte loads and stores of 8 bf16.
+// Rows from the active count up to the next multiple of 128 are zeroed (the
+// GEMMs read whole 128-row tiles); a token whose forward row was skipped has
+// no stored probabilities: its row is zeroed and SAO_DEVERR_CACHE_ROW raised.
+constexpr int kDzThreads = 256;
+
+__global__ void __launch_bounds__(kDzThreads) dz_from_cache_kernel(
+    const __nv_bfloat16 *__restrict__ e, int64_t lde, const float2 *__restrict__ part, int64_t N,
+    const int *__restrict__ pos, const int *__restrict__ idx, const int *__restrict__ count,
+    const int32_t *__restrict__ y, const float *__restrict__ lse, const float *__restrict__ G, int v0, int vc,
+    __nv_bfloat16 *__restrict__ dz, int64_t ldz, unsigned int *err) {
+  const int64_t i = blockIdx.x;
+  const int64_t cnt = *count;
+  if (i >= (cnt + BM - 1) / BM * BM) return;
+  __nv_bfloat16 *out = dz + i * ldz;
+  int f = -1;
+  int64_t t = 0;
+  if (i < cnt) {
+    t = __ldg(idx + i);
+    f = __ldg(pos + t);
+    if (f < 0 && threadIdx.x == 0) raise_device_error(err, SAO_DEVERR_CACHE_ROW);
+  }
+  if (f < 0) {
+    for (int k = threadIdx.x * 8; k < vc; k += kDzThreads * 8) {
+      if (k + 8 <= vc)
+        *reinterpret_cast<uint4 *>(out + k) = make_uint4(0u, 0u, 0u, 0u);
+      else
+        for (int j = k; j < vc; ++j) out[j] = __float2bfloat16_rn(0.f);
+    }
+    return;
+  }
+  const float g = __ldg(G + t);
+  const float l2 = __ldg(lse + t) * kLog2e;
+  const int yy = __ldg(y + t) - v0;
+  const __nv_bfloat16 *src = e + int64_t(f) * lde + v0;
+  for (int k = threadIdx.x * 8; k < vc; k += kDzThreads * 8) {
+    // the 8 columns share one 256-wide tile (v0 and k are multiples of 8)
+    const float s = ex2_approx(fmaf(__ldg(&part[int64_t((v0 + k) / BN) * N + f].x), kLog2e, -l2));
+    const float gs = g * s;
+    if (k + 8 <= vc) {
+      const uint4 q = __ldcs(reinterpret_cast<const uint4 *>(src + k));
+      const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+      uint32_t o[4];
+#pragma unroll
+      for (int h2 = 0; h2 < 4; ++h2) {
+        const float2 ev = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[h2]));
+        float d0 = -gs * ev.x, d1 = -gs * ev.y;
+        if (k + 2 * h2 == yy) d0 += g;
+        if (k + 2 * h2 + 1 == yy) d1 += g;
+        const __nv_bfloat162 b2 = __floats2bfloat162_rn(d0, d1);
+        o[h2] = *reinterpret_cast<const uint32_t *>(&b2);
+      }
+      __stcs(reinterpret_cast<uint4 *>(out + k), make_uint4(o[0], o[1], o[2], o[3]));
+    } else {
+      for (int j = k; j < vc; ++j) {
+        float d = -gs * __bfloat162float(src[j]);
+        if (j == yy) d += g;
+        out[j] = __float2bfloat16_rn(d);
+      }
+    }
+  }
+}
+
+__global__ void iota_kernel(int *pos, int64_t N) {
+  const int64_t t = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (t < N) pos[t] = int(t);
 }
 
 // ---------------------------------------------------------------------------
@@ -507,15 +661,28 @@ size_t tc_ws_bytes(int64_t N, int32_t h, int32_t V) {
   return compact_ws_bytes(N, h) + (fwd > bwd ? fwd : bwd);
 }
 
+LogprobCache logprob_cache_view(void *base, int64_t N, int32_t V) {
+  const int64_t nvt = (int64_t(V) + BN - 1) / BN;
+  LogprobCache k;
+  k.rows = (N + BM - 1) / BM * BM;
+  k.lde = (int64_t(V) + 63) / 64 * 64;
+  Carver c(base, ~size_t(0));
+  k.e = c.take<__nv_bfloat16>(size_t(k.rows) * size_t(k.lde));
+  k.part = c.take<float2>(size_t(nvt) * size_t(N));
+  k.pos = c.take<int>(size_t(N));
+  k.bytes = c.off;
+  return k;
+}
+
 sao_status tc_fwd(const void *H, const void *W, const int32_t *y, const uint8_t *row_mask, int64_t N, int32_t h,
                   int32_t V, float *logp, float *lse, unsigned int *err, void *ws, size_t ws_bytes,
-                  cudaStream_t s) {
+                  const LogprobCache *cache, cudaStream_t s) {
   const int nvt = (V + BN - 1) / BN;
   Carver c(ws, ws_bytes);
   // Rows with row_mask == 0 are skipped: the GEMM runs on the compacted rows.
   CompactRows cr{};
   if (row_mask) SAO_TRY(compact_rows(row_mask, nullptr, N, static_cast<const __nv_bfloat16 *>(H), h, &cr, c, s));
-  float2 *part = c.take<float2>(size_t(nvt) * size_t(N));
+  float2 *part = cache ? cache->part : c.take<float2>(size_t(nvt) * size_t(N));
   float *zy = c.take<float>(size_t(N));
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the log-prob forward");
   CUtensorMap ma, mb;
@@ -540,13 +707,27 @@ sao_status tc_fwd(const void *H, const void *W, const int32_t *y, const uint8_t 
     p.m_count = cr.count;
     p.row_idx = cr.idx;
   }
-  SAO_TRY((launch_gemm<kSoftmax, false, false>("tc_logits_lse_fwd", ma, mb, ma, p, s)));
+  if (cache) {
+    // also store e = exp(z - max_tile) and every token's forward row
+    CUtensorMap me;
+    SAO_TRY(make_map(&me, cache->e, uint64_t(V), uint64_t(cache->rows), uint64_t(cache->lde), 64, BM));
+    SAO_TRY((launch_gemm<kSoftmaxStore, false, false>("tc_logits_lse_fwd", ma, mb, me, p, s)));
+    if (row_mask) {
+      SAO_CUDA_TRY(cudaMemcpyAsync(cache->pos, cr.pos, sizeof(int) * size_t(N), cudaMemcpyDeviceToDevice, s));
+    } else {
+      int slot = launch_begin("iota_pos", s);
+      iota_kernel<<<unsigned((N + 255) / 256), 256, 0, s>>>(cache->pos, N);
+      SAO_TRY(launch_end(slot, s));
+    }
+  } else {
+    SAO_TRY((launch_gemm<kSoftmax, false, false>("tc_logits_lse_fwd", ma, mb, ma, p, s)));
+  }
   return lse_merge_launch(part, nvt, zy, y, nullptr, row_mask ? cr.pos : nullptr, N, V, logp, lse, err, s);
 }
 
 sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *lse, const float *G, int64_t N,
                   int32_t h, int32_t V, void *dH, float *dW, int accumulate, unsigned int *err, void *ws,
-                  size_t ws_bytes, cudaStream_t s) {
+                  size_t ws_bytes, const LogprobCache *cache, cudaStream_t s) {
   const int Vc = vocab_chunk(N, V);
   const bool multi = Vc < V;
   Carver c(ws, ws_bytes);
@@ -571,7 +752,12 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
     CUtensorMap mZ_K, mZ_MN;
     SAO_TRY(make_map(&mZ_K, dz, uint64_t(vc), uint64_t(N), uint64_t(Vc), 64, BM));
     SAO_TRY(make_map(&mZ_MN, dz, uint64_t(vc), uint64_t(N), uint64_t(Vc), 64, 64));
-    {  // dZ for vocabulary [v0, v0 + vc), compacted rows
+    if (cache) {  // dZ from the stored probabilities, compacted rows
+      int slot = launch_begin("dz_from_cache", s);
+      dz_from_cache_kernel<<<unsigned(N), kDzThreads, 0, s>>>(cache->e, cache->lde, cache->part, N, cache->pos,
+                                                               cr.idx, cr.count, y, lse, G, v0, vc, dz, Vc, err);
+      SAO_TRY(launch_end(slot, s));
+    } else {  // dZ for vocabulary [v0, v0 + vc), compacted rows: recompute the logits
       GemmParams p{};
       p.nM = nMt;
       p.nN = (vc + BN - 1) / BN;

@@ -108,7 +108,7 @@ sao_status sao_token_logprobs_fwd(const void *H, const void *W, sao_dtype dt, co
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   SAO_TRY(begin_call(ws, s));
   if (dt == SAO_BF16)
-    SAO_TRY(tc_fwd(H, W, y, row_mask, N, h, V, logp, lse, w.err, w.body, w.body_bytes, s));
+    SAO_TRY(tc_fwd(H, W, y, row_mask, N, h, V, logp, lse, w.err, w.body, w.body_bytes, nullptr, s));
   else
     SAO_TRY(simt_fwd(static_cast<const float *>(H), static_cast<const float *>(W), y, row_mask, N, h, V, logp,
                      lse, w.err, w.body, w.body_bytes, s));
@@ -132,10 +132,70 @@ sao_status sao_token_logprobs_bwd(const void *H, const void *W, sao_dtype dt, co
   SAO_TRY(take_ws(ws, ws_bytes, logprobs_ws_bytes(N, h, V, dt), &w));
   SAO_TRY(begin_call(ws, s));
   if (dt == SAO_BF16)
-    SAO_TRY(tc_bwd(H, W, y, lse, grad_logp, N, h, V, dH, dW, accumulate_dW, w.err, w.body, w.body_bytes, s));
+    SAO_TRY(tc_bwd(H, W, y, lse, grad_logp, N, h, V, dH, dW, accumulate_dW, w.err, w.body, w.body_bytes, nullptr,
+                   s));
   else
     SAO_TRY(simt_bwd(static_cast<const float *>(H), static_cast<const float *>(W), y, lse, grad_logp, N, h, V,
                      static_cast<float *>(dH), dW, accumulate_dW, w.body, w.body_bytes, s));
+  return finish_call(ws, s);
+}
+
+size_t sao_logprob_cache_bytes(int64_t N, int32_t V) {
+  if (N <= 0 || V <= 0) return 0;
+  return logprob_cache_view(nullptr, N, V).bytes;
+}
+
+// The cache must hold sao_logprob_cache_bytes(N, V) bytes at a 256-byte
+// aligned address (its parts are TMA operands and 16-byte vector streams).
+static sao_status take_cache(const void *cache, size_t cache_bytes, int64_t N, int32_t V, LogprobCache *out) {
+  if (!cache) return fail(SAO_ERR_INVALID_ARG, "NULL probability cache");
+  if ((reinterpret_cast<uintptr_t>(cache) & 255u) != 0)
+    return fail(SAO_ERR_INVALID_ARG, "probability cache not 256-byte aligned");
+  *out = logprob_cache_view(const_cast<void *>(cache), N, V);
+  if (cache_bytes < out->bytes)
+    return fail(SAO_ERR_WORKSPACE, "probability cache too small: %zu bytes, need %zu", cache_bytes, out->bytes);
+  return SAO_OK;
+}
+
+sao_status sao_token_logprobs_fwd_cached(const void *H, const void *W, sao_dtype dt, const int32_t *y,
+                                         const uint8_t *row_mask, int64_t N, int32_t h, int32_t V, float *logp,
+                                         float *lse, void *cache, size_t cache_bytes, void *ws, size_t ws_bytes,
+                                         sao_stream_t stream) {
+  SAO_TRY(check_logprob_shapes(dt, N, h, V));
+  if (dt != SAO_BF16) return fail(SAO_ERR_UNSUPPORTED, "the probability cache is for bf16 only");
+  if (N == 0) return SAO_OK;
+  if (!H || !W || !y || !logp || !lse) return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
+  SAO_TRY(check_tc_device(dt));
+  LogprobCache k;
+  SAO_TRY(take_cache(cache, cache_bytes, N, V, &k));
+  Ws w;
+  SAO_TRY(take_ws(ws, ws_bytes, logprobs_ws_bytes(N, h, V, dt), &w));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  SAO_TRY(begin_call(ws, s));
+  SAO_TRY(tc_fwd(H, W, y, row_mask, N, h, V, logp, lse, w.err, w.body, w.body_bytes, &k, s));
+  return finish_call(ws, s);
+}
+
+sao_status sao_token_logprobs_bwd_cached(const void *H, const void *W, sao_dtype dt, const int32_t *y,
+                                         const float *lse, const float *grad_logp, int64_t N, int32_t h, int32_t V,
+                                         void *dH, float *dW, int accumulate_dW, const void *cache,
+                                         size_t cache_bytes, void *ws, size_t ws_bytes, sao_stream_t stream) {
+  SAO_TRY(check_logprob_shapes(dt, N, h, V));
+  if (dt != SAO_BF16) return fail(SAO_ERR_UNSUPPORTED, "the probability cache is for bf16 only");
+  if (!W || !dW) return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (N == 0) {
+    if (!accumulate_dW) SAO_CUDA_TRY(cudaMemsetAsync(dW, 0, sizeof(float) * size_t(V) * size_t(h), s));
+    return SAO_OK;
+  }
+  if (!H || !y || !lse || !grad_logp || !dH) return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
+  SAO_TRY(check_tc_device(dt));
+  LogprobCache k;
+  SAO_TRY(take_cache(cache, cache_bytes, N, V, &k));
+  Ws w;
+  SAO_TRY(take_ws(ws, ws_bytes, logprobs_ws_bytes(N, h, V, dt), &w));
+  SAO_TRY(begin_call(ws, s));
+  SAO_TRY(tc_bwd(H, W, y, lse, grad_logp, N, h, V, dH, dW, accumulate_dW, w.err, w.body, w.body_bytes, &k, s));
   return finish_call(ws, s);
 }
 

@@ -30,7 +30,8 @@ EXPORTS = ("sao_version", "sao_last_error_string", "sao_set_checked", "sao_get_c
            "sao_token_logprobs_bwd", "sao_advantages", "sao_advantages_noalloc", "sao_step_advantages",
            "sao_policy_loss_fwd", "sao_policy_loss_bwd", "sao_clip_loss_fwd", "sao_clip_loss_bwd",
            "sao_group_advantages", "sao_running_mean_advantages", "sao_decoupled_loss_fwd",
-           "sao_decoupled_loss_bwd",
+           "sao_decoupled_loss_bwd", "sao_logprob_cache_bytes", "sao_token_logprobs_fwd_cached",
+           "sao_token_logprobs_bwd_cached",
            "sao_value_loss", "sao_profile_enable", "sao_profile_reset", "sao_profile_read")
 
 
@@ -61,6 +62,11 @@ def load(path: Optional[str] = None):
         "sao_get_checked": (ctypes.c_int, []),
         "sao_set_dz_budget_bytes": (None, [SZ]),
         "sao_workspace_bytes": (SZ, [I64, I32, I32, ctypes.c_int]),
+        "sao_logprob_cache_bytes": (SZ, [I64, I32]),
+        "sao_token_logprobs_fwd_cached": (ctypes.c_int, [P, P, ctypes.c_int, P, P, I64, I32, I32, P, P, P, SZ, P,
+                                                         SZ, P]),
+        "sao_token_logprobs_bwd_cached": (ctypes.c_int, [P, P, ctypes.c_int, P, P, P, I64, I32, I32, P, P,
+                                                         ctypes.c_int, P, SZ, P, SZ, P]),
         "sao_token_logprobs_fwd": (ctypes.c_int, [P, P, ctypes.c_int, P, P, I64, I32, I32, P, P, P, SZ, P]),
         "sao_token_logprobs_bwd": (ctypes.c_int, [P, P, ctypes.c_int, P, P, P, I64, I32, I32, P, P,
                                                   ctypes.c_int, P, SZ, P]),
@@ -187,6 +193,45 @@ def sao_token_logprobs_bwd(H, W, y, lse, grad_logp, dH, dW, ws, accumulate_dW=Fa
     _check(load().sao_token_logprobs_bwd(_ptr(H), _ptr(W), _dtype_code(H), _ptr(y), _ptr(lse), _ptr(grad_logp),
                                          N, h, V, _ptr(dH), _ptr(dW), 1 if accumulate_dW else 0, _ptr(ws),
                                          ws.numel(), _stream(stream)))
+
+
+def sao_logprob_cache_bytes(N: int, V: int) -> int:
+    return int(load().sao_logprob_cache_bytes(int(N), int(V)))
+
+
+def logprob_cache(N: int, V: int, device=None) -> torch.Tensor:
+    """Allocate the forward's probability cache (about 2*N*V bytes)."""
+    return torch.empty(max(sao_logprob_cache_bytes(N, V), 256), dtype=torch.uint8, device=device or "cuda")
+
+
+def sao_token_logprobs_fwd_cached(H, W, y, logp, lse, cache, ws, row_mask=None, stream=None):
+    N, h = H.shape
+    V = W.shape[0]
+    if W.shape[1] != h or W.dtype != H.dtype:
+        raise ValueError("W must be [V, h] with the dtype of H")
+    _expect(y, torch.int32, N, "y")
+    _expect(logp, torch.float32, N, "logp")
+    _expect(lse, torch.float32, N, "lse")
+    _expect(row_mask, torch.uint8, N, "row_mask")
+    _check(load().sao_token_logprobs_fwd_cached(_ptr(H), _ptr(W), _dtype_code(H), _ptr(y), _ptr(row_mask), N, h, V,
+                                                _ptr(logp), _ptr(lse), _ptr(cache), cache.numel(), _ptr(ws),
+                                                ws.numel(), _stream(stream)))
+
+
+def sao_token_logprobs_bwd_cached(H, W, y, lse, grad_logp, dH, dW, cache, ws, accumulate_dW=False, stream=None):
+    N, h = H.shape
+    V = W.shape[0]
+    if W.shape[1] != h or W.dtype != H.dtype or dH.dtype != H.dtype or tuple(dH.shape) != (N, h):
+        raise ValueError("W [V,h] and dH [N,h] must share the dtype of H")
+    if dW.dtype != torch.float32 or tuple(dW.shape) != (V, h):
+        raise ValueError("dW must be fp32 [V, h]")
+    _expect(y, torch.int32, N, "y")
+    _expect(lse, torch.float32, N, "lse")
+    _expect(grad_logp, torch.float32, N, "grad_logp")
+    _check(load().sao_token_logprobs_bwd_cached(_ptr(H), _ptr(W), _dtype_code(H), _ptr(y), _ptr(lse),
+                                                _ptr(grad_logp), N, h, V, _ptr(dH), _ptr(dW),
+                                                1 if accumulate_dW else 0, _ptr(cache), cache.numel(), _ptr(ws),
+                                                ws.numel(), _stream(stream)))
 
 
 def sao_advantages(values, rewards, loss_mask, cu_seqlens, gamma, lambda_policy, lambda_critic,

@@ -96,3 +96,16 @@ def test_decoupled_loss_argument_errors_without_gpu(lib):
     st = lib.sao_decoupled_loss_bwd(None, None, None, None, None, 0, -1.0, 0.28, 0.5, 2.0, 0, None, None, None, 0,
                                     None)
     assert st == 1
+
+
+def test_cached_logprobs_argument_errors_without_gpu(lib):
+    P = ctypes.c_void_p
+    assert lib.sao_logprob_cache_bytes(0, 100) == 0
+    assert lib.sao_logprob_cache_bytes(1000, 151936) >= 1024 * 151936 * 2
+    # fp32 has no cached path
+    st = lib.sao_token_logprobs_fwd_cached(P(16), P(16), 0, P(16), None, 8, 8, 10, P(16), P(16), P(256), 1 << 20,
+                                           None, 0, None)
+    assert st == 4
+    st = lib.sao_token_logprobs_bwd_cached(P(16), P(16), 0, P(16), P(16), P(16), 8, 8, 10, P(16), P(16), 0,
+                                           P(256), 1 << 20, None, 0, None)
+    assert st == 4
