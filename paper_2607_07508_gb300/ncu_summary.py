@@ -21,6 +21,7 @@ def summarize(path, only=None):
         if "sao::" in short:
             short = short.split("::")[-1]
         short = short.replace("tc_gemm_kernel<0, 0, 0>", "tc_gemm<softmax> (logits lse fwd)")
+        short = short.replace("tc_gemm_kernel<4, 0, 0>", "tc_gemm<softmax+store> (logits lse fwd, stores bf16 e)")
         short = short.replace("tc_gemm_kernel<1, 0, 0>", "tc_gemm<dlogits> (bwd recompute + dZ)")
         short = short.replace("tc_gemm_kernel<3, 0, 1>", "tc_gemm<store bf16> (dH = dZ W)")
         short = short.replace("tc_gemm_kernel<2, 0, 1>", "tc_gemm<store f32> (dH accumulate)")
