@@ -352,8 +352,41 @@ def bandwidth_study(args):
                                    flags=flags)
         sao.sao_decoupled_loss_bwd(lp, old, roll, adv, m, 0.2, 0.28, 0.5, 2.0, one, grad, ws)
 
+    # the follow-on rows (App. A.1 step GAE, clipped surrogate, GRPO and running-mean advantages)
+    vm = torch.empty(N, dtype=torch.uint8, device=dev)
+    B = wl.B
+    gid = t((np.arange(B) // 8).astype(np.int32))              # groups of 8 trajectories
+    pid = t((np.arange(B) % 64).astype(np.int32))              # 64 prompts
+    hist = torch.zeros(64, 8, dtype=torch.float32, device=dev)
+    seen = torch.zeros(64, dtype=torch.int64, device=dev)
+
+    # whole calls with their algorithmic bytes per token (reads + writes)
+    whole = {
+        "sao_advantages": (13, lambda: sao.sao_advantages(v, R, m, cu, wl.gamma, wl.lam, wl.lam_critic, 0.0,
+                                                          adv, ret, ws)),
+        "sao_step_advantages": (14, lambda: sao.sao_step_advantages(v, R, m, cu, wl.gamma, wl.lam, wl.lam_critic,
+                                                                    0.0, sao.SAO_STEP_AVERAGE, adv, ret, ws,
+                                                                    value_mask=vm)),
+        "sao_policy_loss_fwd": (18, lambda: sao.sao_policy_loss_fwd(lp, old, adv, m, wl.eps_low, wl.eps_high, loss,
+                                                                    counts, ws, coef=coef, flags=flags)),
+        "sao_value_loss": (13, lambda: sao.sao_value_loss(v, ret, m, loss, dV, ws, ev_sums=ev)),
+        "sao_clip_loss_fwd": (18, lambda: sao.sao_clip_loss_fwd(lp, old, adv, m, cu, 0.2, 0.28,
+                                                                sao.SAO_NORM_SEQUENCE, loss, counts, ws, coef=coef,
+                                                                flags=flags)),
+        "sao_clip_loss_bwd": (17, lambda: sao.sao_clip_loss_bwd(lp, old, adv, m, cu, 0.2, 0.28,
+                                                                sao.SAO_NORM_SEQUENCE, one, grad, ws)),
+        "sao_decoupled_loss_fwd": (22, lambda: sao.sao_decoupled_loss_fwd(lp, old, roll, adv, m, 0.2, 0.28, 0.5,
+                                                                          2.0, loss, counts6, ws, coef=coef,
+                                                                          flags=flags)),
+        "sao_group_advantages": (5, lambda: sao.sao_group_advantages(R, gid, m, cu, 1e-6, adv, ws)),
+        "sao_running_mean_advantages": (5, lambda: sao.sao_running_mean_advantages(R, pid, hist, seen, m, cu, adv,
+                                                                                   ws)),
+    }
+
     for _ in range(max(3, args.warmup)):
         calls()
+        for _, fn in whole.values():
+            fn()
     torch.cuda.synchronize()
     sao.sao_profile_enable(True)
     sao.sao_profile_reset()
@@ -362,6 +395,27 @@ def bandwidth_study(args):
     torch.cuda.synchronize()
     prof = sao.sao_profile_read()
     sao.sao_profile_enable(False)
+    per_call = {}
+    stream = torch.cuda.current_stream()
+    for name, (b, fn) in whole.items():
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        us = 1000 * e0.elapsed_time(e1) / args.steps
+        gbs = b * N / (us / 1e6) / 1e9
+        # the call's kernels, timed separately by the library (one more round)
+        sao.sao_profile_enable(True)
+        sao.sao_profile_reset()
+        fn()
+        torch.cuda.synchronize()
+        ks = {k: round(1000 * t / n, 1) for k, (n, t) in sao.sao_profile_read().items()}
+        sao.sao_profile_enable(False)
+        per_call[name] = {"avg_us": us, "bytes_per_token": b, "achieved_gbs": gbs,
+                          "frac_of_hbm": gbs / peaks["hbm_gbs"], "kernels_us": ks}
     out = {}
     names = {"policy_loss_fwd": "policy_loss_fwd", "policy_loss_bwd": "policy_loss_bwd"}
     for k, (n, ms) in prof.items():
@@ -373,7 +427,8 @@ def bandwidth_study(args):
             row.update({"bytes_per_token": b, "achieved_gbs": gbs, "frac_of_hbm": gbs / peaks["hbm_gbs"]})
         out[k] = row
     print(json.dumps({"study": "O(N) kernels, HBM", "tokens": N, "trajectories": wl.B,
-                      "peak_hbm_gbs": peaks["hbm_gbs"], "peak_source": src, "kernels": out}))
+                      "peak_hbm_gbs": peaks["hbm_gbs"], "peak_source": src, "kernels": out,
+                      "calls": per_call}))
     return 0
 
 

@@ -3,15 +3,18 @@
 // broadcast to the step's tokens.
 //
 //   1. flag trajectory starts, then step starts (an action token that opens a
-//      trajectory or follows a non-action token), and compact the step starts
-//      into an ordered step list (count on the device);
-//   2. one warp per step finds the step's end and reduces its token values
-//      (fp64 sum for the step average, or the last value);
-//   3. one thread per trajectory runs the backward GAE over its steps in fp64
-//      (steps are few, so fp64 costs nothing here), with the length-adaptive
-//      lambda counted in steps;
-//   4. one warp per step writes the step's advantage, value target and
-//      value-loss mask to its tokens (everything else was zeroed).
+//      trajectory or follows a non-action token); a block-level scan gives the
+//      ordered step list (count on the device) and every action token's step;
+//   2. a warp takes 32 consecutive steps, one per lane: a lane walks its own
+//      step when it is short (most turns), the warp walks the long ones
+//      together; sums are compensated fp32 pairs (~48 bits), so GB300's slow
+//      fp64 pipe is not on this path;
+//   3. one warp per trajectory runs the backward GAE over its steps: each
+//      lane folds a contiguous block of steps into an affine map, a shuffle
+//      scan combines the maps, each lane replays its block (fp64; the
+//      length-adaptive lambda is counted in steps);
+//   4. every token reads its step's advantage, value target and value-loss
+//      flag (coalesced, one pass; non-action tokens get zeros).
 #include <stdint.h>
 
 #include "sao_common.cuh"
@@ -22,6 +25,7 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kRowsPerBlock = 4096;
+constexpr int kShortStep = 64;  // a step this close to the next step start is walked by one lane
 
 __global__ void mark_traj_starts(const int32_t *cu, int B, int64_t N, uint8_t *traj_start) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
@@ -80,7 +84,8 @@ __global__ void __launch_bounds__(1024) step_scan_kernel(int *block_count, int n
 }
 
 __global__ void __launch_bounds__(kThreads) step_scatter_kernel(const uint8_t *m, const uint8_t *ts, int64_t N,
-                                                                const int *block_offset, int *step_first) {
+                                                                const int *block_offset, int *step_first,
+                                                                int *step_id) {
   const int64_t r0 = int64_t(blockIdx.x) * kRowsPerBlock;
   __shared__ int sh[kThreads / 32];
   __shared__ int base;
@@ -99,70 +104,138 @@ __global__ void __launch_bounds__(kThreads) step_scatter_kernel(const uint8_t *m
       total += sh[w];
     }
     if (a) step_first[base + before + __popc(bal & ((1u << lane) - 1u))] = int(t);
+    if (t < N) {
+      // step of an action token: step starts at or before it, minus one
+      const unsigned upto = lane == 31 ? 0xffffffffu : ((2u << lane) - 1u);
+      step_id[t] = m[t] != 0 ? base + before + __popc(bal & upto) - 1 : -1;
+    }
     __syncthreads();
     if (threadIdx.x == 0) base += total;
     __syncthreads();
   }
 }
 
-__device__ __forceinline__ int traj_of(const int32_t *cu, int B, int64_t t) {
-  int lo = 0, hi = B - 1;
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (int64_t(cu[mid]) <= t) lo = mid;
-    else hi = mid - 1;
+// Compensated fp32 accumulator (Knuth two-sum).
+struct Acc2 {
+  float hi = 0.f, lo = 0.f;
+  __device__ __forceinline__ void add(float x) {
+    const float s = __fadd_rn(hi, x);
+    const float bb = __fsub_rn(s, hi);
+    lo = __fadd_rn(lo, __fadd_rn(__fsub_rn(hi, __fsub_rn(s, bb)), __fsub_rn(x, bb)));
+    hi = s;
   }
-  return lo;
-}
+  __device__ __forceinline__ void add(const Acc2 &o) {
+    add(o.hi);
+    lo = __fadd_rn(lo, o.lo);
+  }
+};
 
 struct StepInfo {
   double v;    // step value V(S)
   int end;     // one past the step's last token
-  int traj;    // trajectory of the step
+  int pad;
 };
 
-// One warp per step: end of the run of action tokens and the step value.
+// Mean of a compensated sum over n tokens, to about 48 bits.
+__device__ __forceinline__ double acc_mean(const Acc2 &a, int n) {
+  const float fn = float(n);
+  const float q = __fdiv_rn(a.hi, fn);
+  const float r = __fadd_rn(__fmaf_rn(-q, fn, a.hi), a.lo);
+  return double(q) + double(__fdiv_rn(r, fn));
+}
+
+// A token continues the step that starts at `first` while it is an action
+// token that does not open a new trajectory.
+__device__ __forceinline__ bool in_step(const uint8_t *m, const uint8_t *ts, int64_t first, int64_t t, int64_t N) {
+  return t < N && m[t] != 0 && (t == first || ts[t] == 0);
+}
+
+// A warp takes 32 consecutive steps, one per lane.
 __global__ void __launch_bounds__(kThreads) step_reduce_kernel(const float *values, const uint8_t *m,
-                                                               const uint8_t *ts, const int32_t *cu, int B,
-                                                               int64_t N, const int *step_first,
+                                                               const uint8_t *ts, int64_t N, const int *step_first,
                                                                const int *nsteps, int mode, StepInfo *info) {
   const int lane = threadIdx.x & 31;
   const int S = *nsteps;
-  for (int s = (blockIdx.x * kThreads + threadIdx.x) >> 5; s < S; s += (gridDim.x * kThreads) >> 5) {
-    const int64_t first = step_first[s];
-    double sum = 0.0;
-    int64_t end = -1;
-    for (int64_t t0 = first;; t0 += 32) {
-      const int64_t t = t0 + lane;
-      const bool in = t < N && m[t] != 0 && (t == first || ts[t] == 0);
-      const unsigned bal = __ballot_sync(0xffffffffu, in);
-      const unsigned run = ~bal ? (__ffs(~bal) - 1) : 32;  // tokens of this step in the 32-window
-      if (lane < int(run)) sum += double(values[t]);
-      if (run < 32) {
-        end = t0 + run;
-        break;
+  const int nwarps = (gridDim.x * kThreads) >> 5;
+  for (int g = (blockIdx.x * kThreads + threadIdx.x) >> 5; g * 32 < S; g += nwarps) {
+    const int s = g * 32 + lane;
+    const bool own = s < S;
+    int64_t first = 0, bound = 0;
+    if (own) {
+      first = step_first[s];
+      bound = s + 1 < S ? int64_t(step_first[s + 1]) : N;
+    }
+    const bool shortstep = own && bound - first <= kShortStep;
+    Acc2 acc;
+    int64_t end = first;
+    if (shortstep) {
+      while (end < bound && in_step(m, ts, first, end, N)) {
+        acc.add(values[end]);
+        ++end;
       }
     }
+    // the long steps of this group, walked by the whole warp, 32 tokens at a time
+    unsigned longs = __ballot_sync(0xffffffffu, own && !shortstep);
+    while (longs) {
+      const int src = __ffs(longs) - 1;
+      longs &= longs - 1;
+      const int64_t f = __shfl_sync(0xffffffffu, first, src);
+      Acc2 part;
+      int64_t e = -1;
+      for (int64_t t0 = f;; t0 += 32) {
+        const int64_t t = t0 + lane;
+        const bool in = in_step(m, ts, f, t, N);
+        const unsigned bal = __ballot_sync(0xffffffffu, in);
+        const unsigned run = ~bal ? (__ffs(~bal) - 1) : 32;  // tokens of this step in the window
+        if (lane < int(run)) part.add(values[t]);
+        if (run < 32) {
+          e = t0 + run;
+          break;
+        }
+      }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    if (lane == 0) {
+      for (int o = 16; o > 0; o >>= 1) {
+        Acc2 other;
+        other.hi = __shfl_xor_sync(0xffffffffu, part.hi, o);
+        other.lo = __shfl_xor_sync(0xffffffffu, part.lo, o);
+        part.add(other);
+      }
+      if (lane == src) {
+        acc = part;
+        end = e;
+      }
+    }
+    if (own) {
       StepInfo si;
       si.end = int(end);
-      si.v = mode == SAO_STEP_LAST ? double(values[end - 1]) : sum / double(end - first);
-      si.traj = traj_of(cu, B, first);
+      si.pad = 0;
+      si.v = mode == SAO_STEP_LAST ? double(values[end - 1]) : acc_mean(acc, int(end - first));
       info[s] = si;
     }
   }
 }
 
-// One thread per trajectory: backward GAE over its steps, in fp64.
-__global__ void step_gae_kernel(const float *rewards, const int32_t *cu, int B, const int *step_first,
-                                const int *nsteps, StepInfo *info, float gamma, float lam, float lam_c,
-                                float alpha, float2 *out /*[S] (adv, ret)*/) {
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+// Affine map of a block of steps: A_left = p * A_right + c.
+struct StepMap {
+  double p, c;
+};
+__device__ __forceinline__ StepMap compose_steps(const StepMap &x, const StepMap &y) {  // x left of y
+  return {x.p * y.p, fma(x.p, y.c, x.c)};
+}
+
+// One warp per trajectory: lane l folds steps [s0 + l*c, s0 + (l+1)*c) into
+// maps for the policy (a = gamma*lambda_b) and the critic (a = gamma*lambda_c),
+// a shuffle scan gives each lane the advantages to the right of its block, and
+// the lane replays its block.
+__global__ void __launch_bounds__(128) step_gae_kernel(const float *rewards, const int32_t *cu, int B,
+                                                       const int *step_first, const int *nsteps,
+                                                       const StepInfo *info, float gamma, float lam, float lam_c,
+                                                       float alpha, float2 *out /*[S] (adv, ret)*/) {
+  const int lane = threadIdx.x & 31;
+  const int b = (blockIdx.x * 128 + threadIdx.x) >> 5;
   if (b >= B) return;
   const int S = *nsteps;
-  // steps of trajectory b: first steps whose first token lies in [cu[b], cu[b+1])
+  // steps of trajectory b: those whose first token lies in [cu[b], cu[b+1])
   auto lower = [&](int64_t t) {
     int lo = 0, hi = S;
     while (lo < hi) {
@@ -172,7 +245,13 @@ __global__ void step_gae_kernel(const float *rewards, const int32_t *cu, int B, 
     }
     return lo;
   };
-  const int s0 = lower(cu[b]), s1 = lower(cu[b + 1]);
+  int s0 = 0, s1 = 0;
+  if (lane == 0) {
+    s0 = lower(cu[b]);
+    s1 = lower(cu[b + 1]);
+  }
+  s0 = __shfl_sync(0xffffffffu, s0, 0);
+  s1 = __shfl_sync(0xffffffffu, s1, 0);
   const int n = s1 - s0;
   if (n <= 0) return;
   double lb = lam;
@@ -181,34 +260,70 @@ __global__ void step_gae_kernel(const float *rewards, const int32_t *cu, int B, 
     lb = lb < 0.0 ? 0.0 : (lb > 1.0 ? 1.0 : lb);
   }
   const double g = gamma, ap = g * lb, ac = g * double(lam_c);
-  double Ap = 0.0, Ac = 0.0, v_next = 0.0;
-  double r = rewards[b];
-  for (int s = s1 - 1; s >= s0; --s) {
-    const double v = info[s].v;
-    const double delta = r + g * v_next - v;
-    Ap = delta + ap * Ap;
-    Ac = delta + ac * Ac;
-    out[s] = make_float2(float(Ap), float(Ac + v));
+  const double R = rewards[b];
+  const int c = (n + 31) / 32;
+  const int a0 = s0 + lane * c, a1 = min(a0 + c, s1);  // this lane's steps [a0, a1)
+  // value of the step right after the block (0 after the last step)
+  const double v_after = a1 < s1 ? info[a1].v : 0.0;
+  // fold: A_i = delta_i + a A_{i+1}, delta_i = r_i + g v_{i+1} - v_i
+  StepMap mp{1.0, 0.0}, mc{1.0, 0.0};
+  {
+    double v_next = v_after;
+    for (int i = a1 - 1; i >= a0; --i) {
+      const double v = info[i].v;
+      const double delta = (i == s1 - 1 ? R : 0.0) + g * v_next - v;
+      mp = {ap * mp.p, fma(ap, mp.c, delta)};
+      mc = {ac * mc.p, fma(ac, mc.c, delta)};
+      v_next = v;
+    }
+  }
+  // suffix scan over lanes: the maps of lanes l+1 .. 31 applied to A = 0
+  StepMap sp = mp, sc = mc;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    StepMap op, oc;
+    op.p = __shfl_down_sync(0xffffffffu, sp.p, d);
+    op.c = __shfl_down_sync(0xffffffffu, sp.c, d);
+    oc.p = __shfl_down_sync(0xffffffffu, sc.p, d);
+    oc.c = __shfl_down_sync(0xffffffffu, sc.c, d);
+    if (lane + d < 32) {
+      sp = compose_steps(sp, op);
+      sc = compose_steps(sc, oc);
+    }
+  }
+  double Ap = __shfl_down_sync(0xffffffffu, sp.c, 1);  // advantage of the step right of the block
+  double Ac = __shfl_down_sync(0xffffffffu, sc.c, 1);
+  if (lane == 31) Ap = Ac = 0.0;
+  // replay
+  double v_next = v_after;
+  for (int i = a1 - 1; i >= a0; --i) {
+    const double v = info[i].v;
+    const double delta = (i == s1 - 1 ? R : 0.0) + g * v_next - v;
+    Ap = fma(ap, Ap, delta);
+    Ac = fma(ac, Ac, delta);
+    out[i] = make_float2(float(Ap), float(Ac + v));
     v_next = v;
-    r = 0.0;
   }
 }
 
-// One warp per step: broadcast to the step's tokens.
-__global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const int *step_first, const int *nsteps,
-                                                                  const StepInfo *info, const float2 *out,
-                                                                  int mode, float *adv, float *ret,
-                                                                  uint8_t *vmask) {
-  const int lane = threadIdx.x & 31;
-  const int S = *nsteps;
-  for (int s = (blockIdx.x * kThreads + threadIdx.x) >> 5; s < S; s += (gridDim.x * kThreads) >> 5) {
-    const int first = step_first[s], end = info[s].end;
-    const float2 o = out[s];
-    for (int t = first + lane; t < end; t += 32) {
-      adv[t] = o.x;
-      ret[t] = o.y;
-      if (vmask) vmask[t] = (mode == SAO_STEP_AVERAGE || t == end - 1) ? 1 : 0;
+// Every token reads its step's results (non-action tokens get zeros).
+__global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const int *step_id, const StepInfo *info,
+                                                                  const float2 *out, int64_t N, int mode,
+                                                                  float *adv, float *ret, uint8_t *vmask) {
+  const int64_t stride = int64_t(gridDim.x) * kThreads;
+  for (int64_t t = int64_t(blockIdx.x) * kThreads + threadIdx.x; t < N; t += stride) {
+    const int s = step_id[t];
+    float a = 0.f, r = 0.f;
+    uint8_t k = 0;
+    if (s >= 0) {
+      const float2 o = out[s];
+      a = o.x;
+      r = o.y;
+      k = (mode == SAO_STEP_AVERAGE || t == int64_t(info[s].end) - 1) ? 1 : 0;
     }
+    adv[t] = a;
+    ret[t] = r;
+    if (vmask) vmask[t] = k;
   }
 }
 
@@ -218,7 +333,8 @@ size_t step_gae_ws_bytes(int64_t N, int64_t B) {
   (void)B;
   const int64_t nblocks = (N + kRowsPerBlock - 1) / kRowsPerBlock;
   return round256(size_t(N)) + round256(sizeof(int) * (nblocks + 1)) + round256(sizeof(int) * 4) +
-         round256(sizeof(int) * N) + round256(sizeof(StepInfo) * N) + round256(sizeof(float2) * N);
+         round256(sizeof(int) * N) + round256(sizeof(int) * N) + round256(sizeof(StepInfo) * N) +
+         round256(sizeof(float2) * N);
 }
 
 sao_status step_gae_launch(const float *values, const float *rewards, const uint8_t *m, const int32_t *cu, int32_t B,
@@ -231,31 +347,29 @@ sao_status step_gae_launch(const float *values, const float *rewards, const uint
   int *block = c.take<int>(size_t(nblocks) + 1);
   int *nsteps = c.take<int>(4);
   int *step_first = c.take<int>(size_t(N));
+  int *step_id = c.take<int>(size_t(N));
   StepInfo *info = c.take<StepInfo>(size_t(N));
   float2 *out = c.take<float2>(size_t(N));
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the step-level advantages");
   DeviceInfo di;
   SAO_TRY(device_info(&di));
   SAO_CUDA_TRY(cudaMemsetAsync(ts, 0, size_t(N), s));
-  SAO_CUDA_TRY(cudaMemsetAsync(adv, 0, sizeof(float) * size_t(N), s));
-  SAO_CUDA_TRY(cudaMemsetAsync(ret, 0, sizeof(float) * size_t(N), s));
-  if (vmask) SAO_CUDA_TRY(cudaMemsetAsync(vmask, 0, size_t(N), s));
   int slot = launch_begin("step_gae_segments", s);
   mark_traj_starts<<<unsigned((B + 255) / 256), 256, 0, s>>>(cu, B, N, ts);
   step_count_kernel<<<unsigned(nblocks), kThreads, 0, s>>>(m, ts, N, block);
   step_scan_kernel<<<1, 1024, 0, s>>>(block, int(nblocks), nsteps);
-  step_scatter_kernel<<<unsigned(nblocks), kThreads, 0, s>>>(m, ts, N, block, step_first);
+  step_scatter_kernel<<<unsigned(nblocks), kThreads, 0, s>>>(m, ts, N, block, step_first, step_id);
   SAO_TRY(launch_end(slot, s));
   const unsigned warps_grid = unsigned(di.sm_count * 8);
   slot = launch_begin("step_gae_reduce", s);
-  step_reduce_kernel<<<warps_grid, kThreads, 0, s>>>(values, m, ts, cu, B, N, step_first, nsteps, mode, info);
+  step_reduce_kernel<<<warps_grid, kThreads, 0, s>>>(values, m, ts, N, step_first, nsteps, mode, info);
   SAO_TRY(launch_end(slot, s));
   slot = launch_begin("step_gae_scan", s);
-  step_gae_kernel<<<unsigned((B + 127) / 128), 128, 0, s>>>(rewards, cu, B, step_first, nsteps, info, gamma, lam,
-                                                           lam_c, alpha, out);
+  step_gae_kernel<<<unsigned((int64_t(B) * 32 + 127) / 128), 128, 0, s>>>(rewards, cu, B, step_first, nsteps, info,
+                                                                          gamma, lam, lam_c, alpha, out);
   SAO_TRY(launch_end(slot, s));
   slot = launch_begin("step_gae_broadcast", s);
-  step_broadcast_kernel<<<warps_grid, kThreads, 0, s>>>(step_first, nsteps, info, out, mode, adv, ret, vmask);
+  step_broadcast_kernel<<<warps_grid, kThreads, 0, s>>>(step_id, info, out, N, mode, adv, ret, vmask);
   return launch_end(slot, s);
 }
 
