@@ -254,27 +254,64 @@ __global__ void __launch_bounds__(256) clip_finalize_kernel(const double *part_l
   }
 }
 
-// GRPO: per-trajectory standardised reward within its group (fp64).
-__global__ void group_norm_kernel(const float *R, const int32_t *gid, int B, float eps, float *a_traj) {
+// Compensated fp32 sum (Knuth two-sum): about 48 bits without the fp64 pipe.
+struct Sum2 {
+  float hi = 0.f, lo = 0.f;
+  __device__ __forceinline__ void add(float x) {
+    const float s = __fadd_rn(hi, x);
+    const float bb = __fsub_rn(s, hi);
+    lo = __fadd_rn(lo, __fadd_rn(__fsub_rn(hi, __fsub_rn(s, bb)), __fsub_rn(x, bb)));
+    hi = s;
+  }
+  __device__ __forceinline__ double value() const { return double(hi) + double(lo); }
+};
+
+// GRPO: per-trajectory standardised reward within its group. Every thread
+// scans all trajectories for its group's members, through shared-memory tiles
+// of the group ids and rewards (members summed in batch order, compensated
+// fp32; the final moments in fp64).
+constexpr int kTile = 2048;
+
+__global__ void __launch_bounds__(256) group_norm_kernel(const float *R, const int32_t *gid, int B, float eps,
+                                                         float *a_traj) {
+  __shared__ int32_t sg[kTile];
+  __shared__ float sr[kTile];
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b >= B) return;
-  const int g = gid[b];
-  double s = 0.0, s2 = 0.0;
-  long long n = 0;
-  for (int j = 0; j < B; ++j)
-    if (gid[j] == g) {
-      const double r = R[j];
-      s += r;
-      n++;
+  const int g = b < B ? gid[b] : 0;
+  Sum2 s, s2;
+  int n = 0;
+  float mu = 0.f;
+  for (int pass = 0; pass < 2; ++pass) {
+    if (pass) mu = float(s.value() / double(n > 0 ? n : 1));
+    for (int t0 = 0; t0 < B; t0 += kTile) {
+      const int len = min(kTile, B - t0);
+      __syncthreads();
+      for (int k = threadIdx.x; k < len; k += blockDim.x) {
+        sg[k] = gid[t0 + k];
+        sr[k] = R[t0 + k];
+      }
+      __syncthreads();
+      if (b >= B) continue;
+#pragma unroll 8
+      for (int k = 0; k < len; ++k) {
+        if (sg[k] != g) continue;
+        if (pass == 0) {
+          s.add(sr[k]);
+          ++n;
+        } else {
+          const float d = __fsub_rn(sr[k], mu);
+          s2.add(__fmul_rn(d, d));
+        }
+      }
     }
-  const double mu = s / double(n);
-  for (int j = 0; j < B; ++j)
-    if (gid[j] == g) {
-      const double d = double(R[j]) - mu;
-      s2 += d * d;
-    }
-  const double var = s2 / double(n);
-  a_traj[b] = float((double(R[b]) - mu) / sqrt(var + double(eps)));
+  }
+  if (b < B) {
+    // exact mean correction for the rounded mu: var = E[(r - mu)^2] - (mean - mu)^2
+    const double mean = s.value() / double(n);
+    const double dm = mean - double(mu);
+    const double var = s2.value() / double(n) - dm * dm;
+    a_traj[b] = float((double(R[b]) - mean) / sqrt((var > 0.0 ? var : 0.0) + double(eps)));
+  }
 }
 
 // One warp per trajectory: broadcast to its action tokens.
@@ -288,23 +325,76 @@ __global__ void __launch_bounds__(256) group_broadcast_kernel(const float *a_tra
   }
 }
 
-// Running-mean baseline: trajectories in batch order against per-prompt
-// windows of recent rewards (one thread: the windows make it sequential).
-__global__ void running_mean_kernel(const float *R, const int32_t *pid, int B, float *history, long long *seen,
-                                    int window, float *a_traj) {
-  if (blockIdx.x != 0 || threadIdx.x != 0) return;
-  for (int b = 0; b < B; ++b) {
-    const int p = pid[b];
-    const long long c = seen[p];
-    const int n = int(c < window ? c : window);
-    float *h = history + int64_t(p) * window;
-    double s = 0.0;
-    for (int i = 0; i < n; ++i) s += h[i];
-    const double base = n > 0 ? s / double(n) : 0.0;
-    a_traj[b] = float(double(R[b]) - base);
-    h[c % window] = R[b];
-    seen[p] = c + 1;
+// Running-mean baseline. Trajectory b of prompt p sees the window as it stands
+// after the k in-batch trajectories of p before it have been recorded: their
+// last min(k, window) rewards, plus the slots of the caller's ring buffer that
+// those k writes have not overwritten. So every trajectory is independent:
+// one thread walks the batch backwards from b (most recent first), then the
+// ring buffers are updated in a second pass.
+__global__ void __launch_bounds__(256) running_mean_kernel(const float *R, const int32_t *pid, int B,
+                                                           const float *history, const long long *seen, int window,
+                                                           float *a_traj, long long *rec) {
+  __shared__ int32_t sp[kTile];
+  __shared__ float sR[kTile];
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  const int p = b < B ? pid[b] : -1;
+  double sum = 0.0;
+  int k = 0;  // in-batch trajectories of p before b
+  // tiles of the batch, newest first, down from the block's last trajectory
+  const int bend = min(B, int(blockIdx.x + 1) * int(blockDim.x));
+  for (int t1 = bend; t1 > 0; t1 -= kTile) {
+    const int t0 = max(0, t1 - kTile), len = t1 - t0;
+    __syncthreads();
+    for (int i = threadIdx.x; i < len; i += blockDim.x) {
+      sp[i] = pid[t0 + i];
+      sR[i] = R[t0 + i];
+    }
+    __syncthreads();
+    if (b >= B) continue;
+    for (int i = min(len, b - t0) - 1; i >= 0; --i)
+      if (sp[i] == p) {
+        if (k < window) sum += double(sR[i]);
+        ++k;
+      }
   }
+  if (b >= B) return;
+  const long long c = seen[p];
+  // old slots still holding rewards: the first min(c, window) slots, except the
+  // k (cyclic) slots c % window, ..., (c + k - 1) % window written since
+  const int valid_old = int(c < window ? c : window);
+  if (k < window) {
+    const float *h = history + int64_t(p) * window;
+    for (int q = 0; q < valid_old; ++q) {
+      const int since = int(((long long)q - c % window + window) % window);  // write order of slot q after c
+      if (since >= k) sum += double(h[q]);
+    }
+  }
+  const long long n = (c + k) < window ? (c + k) : window;
+  a_traj[b] = float(double(R[b]) - (n > 0 ? sum / double(n) : 0.0));
+  rec[b] = c + k;  // b's position in its prompt's reward sequence
+}
+
+// Records the batch: the last `window` rewards of each prompt go to their ring
+// slots (distinct slots), and the prompt's last trajectory advances its count.
+// Positions come from the first pass, so this pass never reads `seen`.
+__global__ void __launch_bounds__(256) running_mean_record_kernel(const float *R, const int32_t *pid, int B,
+                                                                  const long long *rec, float *history,
+                                                                  long long *seen, int window) {
+  __shared__ int32_t sp[kTile];
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  const int p = b < B ? pid[b] : -1;
+  int after = 0;
+  for (int t0 = int(blockIdx.x) * int(blockDim.x) + 1; t0 < B; t0 += kTile) {
+    const int len = min(kTile, B - t0);
+    __syncthreads();
+    for (int i = threadIdx.x; i < len; i += blockDim.x) sp[i] = pid[t0 + i];
+    __syncthreads();
+    if (b >= B) continue;
+    for (int i = max(0, b + 1 - t0); i < len; ++i) after += (sp[i] == p);
+  }
+  if (b >= B) return;
+  if (after < window) history[int64_t(p) * window + int(rec[b] % window)] = R[b];
+  if (after == 0) seen[p] = rec[b] + 1;
 }
 
 }  // namespace
@@ -312,7 +402,8 @@ __global__ void running_mean_kernel(const float *R, const int32_t *pid, int B, f
 size_t baselines_ws_bytes(int64_t N, int64_t B) {
   const int64_t nchunks = (N + kSegChunk - 1) / kSegChunk;
   return round256(sizeof(int) * (nchunks + 1)) + round256(sizeof(int) * (B + 1)) + round256(sizeof(Norms)) +
-         round256(sizeof(double) * nchunks) + round256(sizeof(int) * 3 * nchunks) + round256(sizeof(float) * (B + 1));
+         round256(sizeof(double) * nchunks) + round256(sizeof(int) * 3 * nchunks) + round256(sizeof(float) * (B + 1)) +
+         round256(sizeof(long long) * (B + 1));
 }
 
 sao_status clip_loss_launch(const float *logp, const float *old, const float *adv, const uint8_t *m, const int32_t *cu,
@@ -380,7 +471,7 @@ sao_status group_adv_launch(const float *rewards, const int32_t *gid, int32_t B,
   DeviceInfo di;
   SAO_TRY(device_info(&di));
   int slot = launch_begin("group_advantages", s);
-  group_norm_kernel<<<unsigned((B + 127) / 128), 128, 0, s>>>(rewards, gid, B, eps, a_traj);
+  group_norm_kernel<<<unsigned((B + 255) / 256), 256, 0, s>>>(rewards, gid, B, eps, a_traj);
   group_broadcast_kernel<<<unsigned(di.sm_count * 4), 256, 0, s>>>(a_traj, m, cu, B, N, adv);
   return launch_end(slot, s);
 }
@@ -390,13 +481,18 @@ sao_status running_mean_launch(const float *rewards, const int32_t *pid, int32_t
                                void *ws_body, size_t body_bytes, cudaStream_t s) {
   Carver c(ws_body, body_bytes);
   float *a_traj = c.take<float>(size_t(B) + 1);
+  long long *rec = c.take<long long>(size_t(B) + 1);
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the running-mean baseline");
   if (N > 0) SAO_CUDA_TRY(cudaMemsetAsync(adv, 0, sizeof(float) * size_t(N), s));
   if (B == 0) return SAO_OK;
   DeviceInfo di;
   SAO_TRY(device_info(&di));
   int slot = launch_begin("running_mean_advantages", s);
-  running_mean_kernel<<<1, 32, 0, s>>>(rewards, pid, B, history, reinterpret_cast<long long *>(seen), window, a_traj);
+  const unsigned g = unsigned((B + 255) / 256);
+  running_mean_kernel<<<g, 256, 0, s>>>(rewards, pid, B, history, reinterpret_cast<const long long *>(seen), window,
+                                        a_traj, rec);
+  running_mean_record_kernel<<<g, 256, 0, s>>>(rewards, pid, B, rec, history, reinterpret_cast<long long *>(seen),
+                                               window);
   if (N > 0) group_broadcast_kernel<<<unsigned(di.sm_count * 4), 256, 0, s>>>(a_traj, m, cu, B, N, adv);
   return launch_end(slot, s);
 }
