@@ -121,9 +121,12 @@ __global__ void __launch_bounds__(kThreads) clip_loss_kernel(ClipArgs a) {
   const float w_tok = nm.n_action > 0 ? float(1.0 / double(nm.n_action)) : 0.f;
   const double inv_seq = nm.n_seq > 0 ? 1.0 / double(nm.n_seq) : 0.0;
   const float gscale = kBwd ? __ldg(a.grad_scale) : 1.f;
-  const int64_t t0 = int64_t(q) * kSegChunk + int64_t(lane) * kItems;
+  // window-major: in each 128-token window of the chunk, lane l takes tokens
+  // 4l .. 4l+3, so every warp load and store is one contiguous 512 (or 128)
+  // byte access; each lane's trajectory walk still only moves forward
+  const int64_t c0 = int64_t(q) * kSegChunk;
   const int64_t N = a.N;
-  int b = cu.find(blo, bhi, t0 < N ? t0 : N - 1);
+  int b = blo;
   int64_t next_end = cu[b + 1];
   auto weight = [&](int bb) {
     if (!a.seq) return w_tok;
@@ -133,12 +136,13 @@ __global__ void __launch_bounds__(kThreads) clip_loss_kernel(ClipArgs a) {
   float w = weight(b);
   float acc_hi = 0.f, acc_lo = 0.f;  // compensated sum of the value terms
   int nl = 0, nh = 0, nf = 0;
-  const bool vec = (t0 + kItems <= N) && aligned16_dev(a.logp) && aligned16_dev(a.old) && aligned16_dev(a.adv) &&
-                   ((reinterpret_cast<uintptr_t>(a.m) & 3u) == 0) && (a.coef == nullptr || aligned16_dev(a.coef)) &&
-                   (a.flags == nullptr || (reinterpret_cast<uintptr_t>(a.flags) & 3u) == 0);
+  const bool aligned = aligned16_dev(a.logp) && aligned16_dev(a.old) && aligned16_dev(a.adv) &&
+                       ((reinterpret_cast<uintptr_t>(a.m) & 3u) == 0) && (a.coef == nullptr || aligned16_dev(a.coef)) &&
+                       (a.flags == nullptr || (reinterpret_cast<uintptr_t>(a.flags) & 3u) == 0);
 #pragma unroll 1
-  for (int g = 0; g < kItems / 4; ++g) {
-    const int64_t tg = t0 + 4 * g;
+  for (int g = 0; g < kSegChunk / 128; ++g) {
+    const int64_t tg = c0 + int64_t(g) * 128 + int64_t(lane) * 4;
+    const bool vec = aligned && tg + 4 <= N;
     float lp[4], od[4], ad[4];
     bool act[4];
     if (vec) {
