@@ -34,18 +34,42 @@ __global__ void mark_traj_starts(const int32_t *cu, int B, int64_t N, uint8_t *t
   if (t >= 0 && t < N && cu[b + 1] > t) traj_start[t] = 1;
 }
 
-__device__ __forceinline__ bool step_start(const uint8_t *m, const uint8_t *traj_start, int64_t t) {
-  return m[t] != 0 && (t == 0 || traj_start[t] != 0 || m[t - 1] == 0);
+// Bit i set when byte i of x is non-zero (i = 0..3).
+__device__ __forceinline__ uint32_t nz4(uint32_t x) {
+  const uint32_t h = (((x & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | x) & 0x80808080u;
+  return (h * 0x00204081u) >> 28;
 }
 
+// Step starts among the 16 tokens t0 .. t0+15 (bit i: token t0+i opens a
+// step: an action token that opens a trajectory or follows a non-action
+// token), and their action flags. 16-byte loads when the run is in range and
+// aligned, byte loads otherwise.
+__device__ __forceinline__ uint32_t step_starts16(const uint8_t *m, const uint8_t *ts, int64_t N, int64_t t0,
+                                                  uint32_t &act) {
+  uint32_t M = 0, T = 0;
+  if (t0 + 16 <= N && ((reinterpret_cast<uintptr_t>(m) | reinterpret_cast<uintptr_t>(ts)) & 15u) == 0) {
+    const uint4 mv = __ldg(reinterpret_cast<const uint4 *>(m + t0));
+    const uint4 tv = __ldg(reinterpret_cast<const uint4 *>(ts + t0));
+    M = nz4(mv.x) | nz4(mv.y) << 4 | nz4(mv.z) << 8 | nz4(mv.w) << 12;
+    T = nz4(tv.x) | nz4(tv.y) << 4 | nz4(tv.z) << 8 | nz4(tv.w) << 12;
+  } else {
+    for (int i = 0; i < 16; ++i)
+      if (t0 + i < N) {
+        M |= uint32_t(m[t0 + i] != 0) << i;
+        T |= uint32_t(ts[t0 + i] != 0) << i;
+      }
+  }
+  const uint32_t prev = (M << 1) | uint32_t(t0 > 0 && t0 - 1 < N && m[t0 - 1] != 0);  // bit i: token t0+i-1 acts
+  act = M;
+  return M & (T | ~prev) & 0xFFFFu;
+}
+
+// Step starts per 4096-token block (each thread 16 consecutive tokens).
 __global__ void __launch_bounds__(kThreads) step_count_kernel(const uint8_t *m, const uint8_t *ts, int64_t N,
                                                               int *block_count) {
-  const int64_t r0 = int64_t(blockIdx.x) * kRowsPerBlock;
-  int c = 0;
-  for (int i = threadIdx.x; i < kRowsPerBlock; i += kThreads) {
-    const int64_t t = r0 + i;
-    if (t < N) c += step_start(m, ts, t);
-  }
+  const int64_t t0 = int64_t(blockIdx.x) * kRowsPerBlock + int64_t(threadIdx.x) * 16;
+  uint32_t act;
+  int c = t0 < N ? __popc(step_starts16(m, ts, N, t0, act)) : 0;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
   __shared__ int sh[kThreads / 32];
@@ -57,6 +81,7 @@ __global__ void __launch_bounds__(kThreads) step_count_kernel(const uint8_t *m, 
     block_count[blockIdx.x] = s;
   }
 }
+static_assert(kRowsPerBlock == kThreads * 16, "16 tokens per thread");
 
 __global__ void __launch_bounds__(1024) step_scan_kernel(int *block_count, int nblocks, int *total) {
   __shared__ int sh[1024];
@@ -83,35 +108,43 @@ __global__ void __launch_bounds__(1024) step_scan_kernel(int *block_count, int n
   if (threadIdx.x == 1023) *total = sh[1023];
 }
 
+// Ordered step list and every token's step (-1 for non-action tokens).
 __global__ void __launch_bounds__(kThreads) step_scatter_kernel(const uint8_t *m, const uint8_t *ts, int64_t N,
                                                                 const int *block_offset, int *step_first,
                                                                 int *step_id) {
-  const int64_t r0 = int64_t(blockIdx.x) * kRowsPerBlock;
-  __shared__ int sh[kThreads / 32];
-  __shared__ int base;
-  if (threadIdx.x == 0) base = block_offset[blockIdx.x];
-  __syncthreads();
+  const int64_t t0 = int64_t(blockIdx.x) * kRowsPerBlock + int64_t(threadIdx.x) * 16;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (int i0 = 0; i0 < kRowsPerBlock; i0 += kThreads) {
-    const int64_t t = r0 + i0 + threadIdx.x;
-    const bool a = t < N && step_start(m, ts, t);
-    const unsigned bal = __ballot_sync(0xffffffffu, a);
-    if (lane == 0) sh[warp] = __popc(bal);
-    __syncthreads();
-    int before = 0, total = 0;
-    for (int w = 0; w < kThreads / 32; ++w) {
-      before += (w < warp) ? sh[w] : 0;
-      total += sh[w];
-    }
-    if (a) step_first[base + before + __popc(bal & ((1u << lane) - 1u))] = int(t);
-    if (t < N) {
-      // step of an action token: step starts at or before it, minus one
-      const unsigned upto = lane == 31 ? 0xffffffffu : ((2u << lane) - 1u);
-      step_id[t] = m[t] != 0 ? base + before + __popc(bal & upto) - 1 : -1;
-    }
-    __syncthreads();
-    if (threadIdx.x == 0) base += total;
-    __syncthreads();
+  uint32_t act = 0, st = 0;
+  if (t0 < N) st = step_starts16(m, ts, N, t0, act);
+  const int c = __popc(st);
+  // exclusive prefix of the counts over the block
+  int x = c;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  __shared__ int sh[kThreads / 32];
+  if (lane == 31) sh[warp] = x;
+  __syncthreads();
+  int before = 0;
+  for (int w = 0; w < warp; ++w) before += sh[w];
+  const int base = block_offset[blockIdx.x] + before + x - c;  // steps opened before token t0
+  if (t0 >= N) return;
+  int k = base;
+  int ids[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    if ((st >> i) & 1u) step_first[k++] = int(t0 + i);
+    ids[i] = ((act >> i) & 1u) ? k - 1 : -1;
+  }
+  if (t0 + 16 <= N && (reinterpret_cast<uintptr_t>(step_id) & 15u) == 0) {
+    int4 *d = reinterpret_cast<int4 *>(step_id + t0);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) d[q] = make_int4(ids[4 * q], ids[4 * q + 1], ids[4 * q + 2], ids[4 * q + 3]);
+  } else {
+    for (int i = 0; i < 16; ++i)
+      if (t0 + i < N) step_id[t0 + i] = ids[i];
   }
 }
 
@@ -235,23 +268,24 @@ __global__ void __launch_bounds__(128) step_gae_kernel(const float *rewards, con
   const int b = (blockIdx.x * 128 + threadIdx.x) >> 5;
   if (b >= B) return;
   const int S = *nsteps;
-  // steps of trajectory b: those whose first token lies in [cu[b], cu[b+1])
+  // steps of trajectory b: those whose first token lies in [cu[b], cu[b+1]);
+  // first step index with step_first >= t by a 33-way warp search
   auto lower = [&](int64_t t) {
-    int lo = 0, hi = S;
-    while (lo < hi) {
-      const int mid = (lo + hi) >> 1;
-      if (int64_t(step_first[mid]) < t) lo = mid + 1;
-      else hi = mid;
+    int lo = 0, hi = S;  // the answer lies in [lo, hi]
+    while (hi - lo > 32) {
+      const int p = lo + int(int64_t(hi - lo) * (lane + 1) / 33);  // 32 rising pivots in [lo, hi)
+      const unsigned below = __ballot_sync(0xffffffffu, int64_t(step_first[p]) < t);
+      const int c = __popc(below);  // pivots below t: lanes 0 .. c-1
+      const int nlo = c > 0 ? __shfl_sync(0xffffffffu, p, c - 1) + 1 : lo;
+      const int nhi = c < 32 ? __shfl_sync(0xffffffffu, p, c & 31) : hi;
+      lo = nlo;
+      hi = nhi;
     }
-    return lo;
+    const bool below = lo + lane < hi && int64_t(step_first[lo + lane]) < t;
+    return lo + __popc(__ballot_sync(0xffffffffu, below));
   };
-  int s0 = 0, s1 = 0;
-  if (lane == 0) {
-    s0 = lower(cu[b]);
-    s1 = lower(cu[b + 1]);
-  }
-  s0 = __shfl_sync(0xffffffffu, s0, 0);
-  s1 = __shfl_sync(0xffffffffu, s1, 0);
+  const int s0 = lower(cu[b]);
+  const int s1 = lower(cu[b + 1]);
   const int n = s1 - s0;
   if (n <= 0) return;
   double lb = lam;
@@ -306,24 +340,48 @@ __global__ void __launch_bounds__(128) step_gae_kernel(const float *rewards, con
   }
 }
 
-// Every token reads its step's results (non-action tokens get zeros).
+// Every token reads its step's results (non-action tokens get zeros); four
+// consecutive tokens per thread.
+__device__ __forceinline__ void step_result(int s, int64_t t, const StepInfo *info, const float2 *out, int mode,
+                                            float &a, float &r, uint8_t &k) {
+  a = r = 0.f;
+  k = 0;
+  if (s >= 0) {
+    const float2 o = out[s];
+    a = o.x;
+    r = o.y;
+    k = (mode == SAO_STEP_AVERAGE || t == int64_t(info[s].end) - 1) ? 1 : 0;
+  }
+}
+
 __global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const int *step_id, const StepInfo *info,
                                                                   const float2 *out, int64_t N, int mode,
                                                                   float *adv, float *ret, uint8_t *vmask) {
-  const int64_t stride = int64_t(gridDim.x) * kThreads;
-  for (int64_t t = int64_t(blockIdx.x) * kThreads + threadIdx.x; t < N; t += stride) {
-    const int s = step_id[t];
-    float a = 0.f, r = 0.f;
-    uint8_t k = 0;
-    if (s >= 0) {
-      const float2 o = out[s];
-      a = o.x;
-      r = o.y;
-      k = (mode == SAO_STEP_AVERAGE || t == int64_t(info[s].end) - 1) ? 1 : 0;
+  const int64_t stride = int64_t(gridDim.x) * kThreads * 4;
+  const bool vec = ((reinterpret_cast<uintptr_t>(step_id) | reinterpret_cast<uintptr_t>(adv) |
+                     reinterpret_cast<uintptr_t>(ret)) & 15u) == 0 &&
+                   (reinterpret_cast<uintptr_t>(vmask) & 3u) == 0;
+  for (int64_t t = (int64_t(blockIdx.x) * kThreads + threadIdx.x) * 4; t < N; t += stride) {
+    if (vec && t + 4 <= N) {
+      const int4 s4 = *reinterpret_cast<const int4 *>(step_id + t);
+      const int sv[4] = {s4.x, s4.y, s4.z, s4.w};
+      float a[4], r[4];
+      uint8_t k[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) step_result(sv[i], t + i, info, out, mode, a[i], r[i], k[i]);
+      *reinterpret_cast<float4 *>(adv + t) = make_float4(a[0], a[1], a[2], a[3]);
+      *reinterpret_cast<float4 *>(ret + t) = make_float4(r[0], r[1], r[2], r[3]);
+      if (vmask) *reinterpret_cast<uchar4 *>(vmask + t) = make_uchar4(k[0], k[1], k[2], k[3]);
+    } else {
+      for (int64_t u = t; u < t + 4 && u < N; ++u) {
+        float a, r;
+        uint8_t k;
+        step_result(step_id[u], u, info, out, mode, a, r, k);
+        adv[u] = a;
+        ret[u] = r;
+        if (vmask) vmask[u] = k;
+      }
     }
-    adv[t] = a;
-    ret[t] = r;
-    if (vmask) vmask[t] = k;
   }
 }
 
