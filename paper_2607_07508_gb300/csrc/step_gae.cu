@@ -4,14 +4,15 @@
 //
 //   1. flag trajectory starts, then step starts (an action token that opens a
 //      trajectory or follows a non-action token); a block-level scan gives the
-//      ordered step list (count on the device) and every action token's step;
-//   2. a warp takes 32 consecutive steps, one per lane: a lane walks its own
-//      step when it is short (most turns), the warp walks the long ones
+//      ordered step list with each step's token range (count on the device)
+//      and every action token's step;
+//   2. a warp takes 32 consecutive steps, one per lane: a lane sums its own
+//      step when it is short (most turns), the warp sums the long ones
 //      together; sums are compensated fp32 pairs (~48 bits), so GB300's slow
 //      fp64 pipe is not on this path;
 //   3. one warp per trajectory runs the backward GAE over its steps: each
 //      lane folds a contiguous block of steps into an affine map, a shuffle
-//      scan combines the maps, each lane replays its block (fp64; the
+//      scan combines the maps, each lane replays its block (double-float; the
 //      length-adaptive lambda is counted in steps);
 //   4. every token reads its step's advantage, value target and value-loss
 //      flag (coalesced, one pass; non-action tokens get zeros).
@@ -25,7 +26,7 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kRowsPerBlock = 4096;
-constexpr int kShortStep = 64;  // a step this close to the next step start is walked by one lane
+constexpr int kShortStep = 32;  // a step this long or shorter is summed by one lane
 
 __global__ void mark_traj_starts(const int32_t *cu, int B, int64_t N, uint8_t *traj_start) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
@@ -45,7 +46,7 @@ __device__ __forceinline__ uint32_t nz4(uint32_t x) {
 // token), and their action flags. 16-byte loads when the run is in range and
 // aligned, byte loads otherwise.
 __device__ __forceinline__ uint32_t step_starts16(const uint8_t *m, const uint8_t *ts, int64_t N, int64_t t0,
-                                                  uint32_t &act) {
+                                                  uint32_t &act, uint32_t &tstart) {
   uint32_t M = 0, T = 0;
   if (t0 + 16 <= N && ((reinterpret_cast<uintptr_t>(m) | reinterpret_cast<uintptr_t>(ts)) & 15u) == 0) {
     const uint4 mv = __ldg(reinterpret_cast<const uint4 *>(m + t0));
@@ -61,6 +62,7 @@ __device__ __forceinline__ uint32_t step_starts16(const uint8_t *m, const uint8_
   }
   const uint32_t prev = (M << 1) | uint32_t(t0 > 0 && t0 - 1 < N && m[t0 - 1] != 0);  // bit i: token t0+i-1 acts
   act = M;
+  tstart = T;
   return M & (T | ~prev) & 0xFFFFu;
 }
 
@@ -68,8 +70,8 @@ __device__ __forceinline__ uint32_t step_starts16(const uint8_t *m, const uint8_
 __global__ void __launch_bounds__(kThreads) step_count_kernel(const uint8_t *m, const uint8_t *ts, int64_t N,
                                                               int *block_count) {
   const int64_t t0 = int64_t(blockIdx.x) * kRowsPerBlock + int64_t(threadIdx.x) * 16;
-  uint32_t act;
-  int c = t0 < N ? __popc(step_starts16(m, ts, N, t0, act)) : 0;
+  uint32_t act, tst;
+  int c = t0 < N ? __popc(step_starts16(m, ts, N, t0, act, tst)) : 0;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
   __shared__ int sh[kThreads / 32];
@@ -108,14 +110,26 @@ __global__ void __launch_bounds__(1024) step_scan_kernel(int *block_count, int n
   if (threadIdx.x == 1023) *total = sh[1023];
 }
 
-// Ordered step list and every token's step (-1 for non-action tokens).
+// Ordered step list with each step's first and one-past-last token, and every
+// token's step (-1 for non-action tokens).
 __global__ void __launch_bounds__(kThreads) step_scatter_kernel(const uint8_t *m, const uint8_t *ts, int64_t N,
                                                                 const int *block_offset, int *step_first,
-                                                                int *step_id) {
+                                                                int *step_end, int *step_id) {
   const int64_t t0 = int64_t(blockIdx.x) * kRowsPerBlock + int64_t(threadIdx.x) * 16;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  uint32_t act = 0, st = 0;
-  if (t0 < N) st = step_starts16(m, ts, N, t0, act);
+  uint32_t act = 0, st = 0, tst = 0;
+  if (t0 < N) st = step_starts16(m, ts, N, t0, act, tst);
+  // does token t0+16 continue a step? (an action token that opens no trajectory)
+  uint32_t nact = __shfl_down_sync(0xffffffffu, act, 1), ntst = __shfl_down_sync(0xffffffffu, tst, 1);
+  if (lane == 31) {
+    const int64_t u = t0 + 16;
+    nact = (u < N && m[u] != 0) ? 1u : 0u;
+    ntst = (u < N && ts[u] != 0) ? 1u : 0u;
+  }
+  const uint32_t cont_next = (nact & ~ntst) & 1u;
+  // bit i: token t0+i+1 continues the step; last: token t0+i is a step's last token
+  const uint32_t cont = ((act & ~tst) >> 1) | (cont_next << 15);
+  const uint32_t last = act & ~cont & 0xFFFFu;
   const int c = __popc(st);
   // exclusive prefix of the counts over the block
   int x = c;
@@ -137,6 +151,7 @@ __global__ void __launch_bounds__(kThreads) step_scatter_kernel(const uint8_t *m
   for (int i = 0; i < 16; ++i) {
     if ((st >> i) & 1u) step_first[k++] = int(t0 + i);
     ids[i] = ((act >> i) & 1u) ? k - 1 : -1;
+    if ((last >> i) & 1u) step_end[k - 1] = int(t0 + i + 1);
   }
   if (t0 + 16 <= N && (reinterpret_cast<uintptr_t>(step_id) & 15u) == 0) {
     int4 *d = reinterpret_cast<int4 *>(step_id + t0);
@@ -163,69 +178,88 @@ struct Acc2 {
   }
 };
 
-struct StepInfo {
-  double v;    // step value V(S)
-  int end;     // one past the step's last token
-  int pad;
+// ---------------------------------------------------------------------------
+// double-float arithmetic (fp32 pairs, ~48 bits): GB300's fp64 pipe is far
+// slower than its fp32 one, and these recurrences run over millions of steps
+// ---------------------------------------------------------------------------
+struct dd {
+  float hi, lo;
 };
+__device__ __forceinline__ dd dd_quick(float a, float b) {  // |a| >= |b|
+  const float s = __fadd_rn(a, b);
+  return {s, __fsub_rn(b, __fsub_rn(s, a))};
+}
+__device__ __forceinline__ dd dd_two_sum(float a, float b) {
+  const float s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  return {s, __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb))};
+}
+__device__ __forceinline__ dd dd_add(dd x, dd y) {
+  const dd s = dd_two_sum(x.hi, y.hi);
+  return dd_quick(s.hi, __fadd_rn(s.lo, __fadd_rn(x.lo, y.lo)));
+}
+__device__ __forceinline__ dd dd_mul(dd x, dd y) {
+  const float p = __fmul_rn(x.hi, y.hi);
+  float e = __fmaf_rn(x.hi, y.hi, -p);
+  e = __fmaf_rn(x.hi, y.lo, e);
+  e = __fmaf_rn(x.lo, y.hi, e);
+  return dd_quick(p, e);
+}
+__device__ __forceinline__ dd dd_neg(dd x) { return {-x.hi, -x.lo}; }
+__device__ __forceinline__ dd dd_from_double(double x) {
+  const float hi = float(x);
+  return {hi, float(x - double(hi))};
+}
+__device__ __forceinline__ float dd_round(dd x) { return __fadd_rn(x.hi, x.lo); }
 
-// Mean of a compensated sum over n tokens, to about 48 bits.
-__device__ __forceinline__ double acc_mean(const Acc2 &a, int n) {
+// Step value V(S) as a double-float: the mean of a compensated sum over n tokens.
+__device__ __forceinline__ float2 acc_mean(const Acc2 &a, int n) {
   const float fn = float(n);
   const float q = __fdiv_rn(a.hi, fn);
   const float r = __fadd_rn(__fmaf_rn(-q, fn, a.hi), a.lo);
-  return double(q) + double(__fdiv_rn(r, fn));
+  const dd m = dd_quick(q, __fdiv_rn(r, fn));
+  return make_float2(m.hi, m.lo);
 }
 
-// A token continues the step that starts at `first` while it is an action
-// token that does not open a new trajectory.
-__device__ __forceinline__ bool in_step(const uint8_t *m, const uint8_t *ts, int64_t first, int64_t t, int64_t N) {
-  return t < N && m[t] != 0 && (t == first || ts[t] == 0);
-}
-
-// A warp takes 32 consecutive steps, one per lane.
-__global__ void __launch_bounds__(kThreads) step_reduce_kernel(const float *values, const uint8_t *m,
-                                                               const uint8_t *ts, int64_t N, const int *step_first,
-                                                               const int *nsteps, int mode, StepInfo *info) {
+// A warp takes 32 consecutive steps, one per lane: a lane sums its own step
+// when it is short (4 independent loads at a time), the warp sums the long
+// ones together. Step ranges come from the scatter pass, so no load waits on
+// another.
+__global__ void __launch_bounds__(kThreads) step_reduce_kernel(const float *values, const int *step_first,
+                                                               const int *step_end, const int *nsteps, int mode,
+                                                               float2 *sv) {
   const int lane = threadIdx.x & 31;
   const int S = *nsteps;
   const int nwarps = (gridDim.x * kThreads) >> 5;
   for (int g = (blockIdx.x * kThreads + threadIdx.x) >> 5; g * 32 < S; g += nwarps) {
     const int s = g * 32 + lane;
     const bool own = s < S;
-    int64_t first = 0, bound = 0;
-    if (own) {
-      first = step_first[s];
-      bound = s + 1 < S ? int64_t(step_first[s + 1]) : N;
+    const int first = own ? step_first[s] : 0;
+    const int end = own ? step_end[s] : 0;
+    if (mode == SAO_STEP_LAST) {  // the value of the step's last token
+      if (own) sv[s] = make_float2(values[end - 1], 0.f);
+      continue;
     }
-    const bool shortstep = own && bound - first <= kShortStep;
+    const bool shortstep = own && end - first <= kShortStep;
     Acc2 acc;
-    int64_t end = first;
     if (shortstep) {
-      while (end < bound && in_step(m, ts, first, end, N)) {
-        acc.add(values[end]);
-        ++end;
+      int t = first;
+      for (; t + 4 <= end; t += 4) {
+        const float a0 = values[t], a1 = values[t + 1], a2 = values[t + 2], a3 = values[t + 3];
+        acc.add(a0);
+        acc.add(a1);
+        acc.add(a2);
+        acc.add(a3);
       }
+      for (; t < end; ++t) acc.add(values[t]);
     }
-    // the long steps of this group, walked by the whole warp, 32 tokens at a time
     unsigned longs = __ballot_sync(0xffffffffu, own && !shortstep);
     while (longs) {
       const int src = __ffs(longs) - 1;
       longs &= longs - 1;
-      const int64_t f = __shfl_sync(0xffffffffu, first, src);
+      const int f = __shfl_sync(0xffffffffu, first, src), e = __shfl_sync(0xffffffffu, end, src);
       Acc2 part;
-      int64_t e = -1;
-      for (int64_t t0 = f;; t0 += 32) {
-        const int64_t t = t0 + lane;
-        const bool in = in_step(m, ts, f, t, N);
-        const unsigned bal = __ballot_sync(0xffffffffu, in);
-        const unsigned run = ~bal ? (__ffs(~bal) - 1) : 32;  // tokens of this step in the window
-        if (lane < int(run)) part.add(values[t]);
-        if (run < 32) {
-          e = t0 + run;
-          break;
-        }
-      }
+      for (int t = f + lane; t < e; t += 32) part.add(values[t]);
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
         Acc2 other;
@@ -233,27 +267,21 @@ __global__ void __launch_bounds__(kThreads) step_reduce_kernel(const float *valu
         other.lo = __shfl_xor_sync(0xffffffffu, part.lo, o);
         part.add(other);
       }
-      if (lane == src) {
-        acc = part;
-        end = e;
-      }
+      if (lane == src) acc = part;
     }
-    if (own) {
-      StepInfo si;
-      si.end = int(end);
-      si.pad = 0;
-      si.v = mode == SAO_STEP_LAST ? double(values[end - 1]) : acc_mean(acc, int(end - first));
-      info[s] = si;
-    }
+    if (own) sv[s] = acc_mean(acc, end - first);
   }
 }
 
 // Affine map of a block of steps: A_left = p * A_right + c.
 struct StepMap {
-  double p, c;
+  dd p, c;
 };
 __device__ __forceinline__ StepMap compose_steps(const StepMap &x, const StepMap &y) {  // x left of y
-  return {x.p * y.p, fma(x.p, y.c, x.c)};
+  return {dd_mul(x.p, y.p), dd_add(dd_mul(x.p, y.c), x.c)};
+}
+__device__ __forceinline__ dd dd_shfl_down(dd x, int d) {
+  return {__shfl_down_sync(0xffffffffu, x.hi, d), __shfl_down_sync(0xffffffffu, x.lo, d)};
 }
 
 // One warp per trajectory: lane l folds steps [s0 + l*c, s0 + (l+1)*c) into
@@ -261,9 +289,9 @@ __device__ __forceinline__ StepMap compose_steps(const StepMap &x, const StepMap
 // a shuffle scan gives each lane the advantages to the right of its block, and
 // the lane replays its block.
 __global__ void __launch_bounds__(128) step_gae_kernel(const float *rewards, const int32_t *cu, int B,
-                                                       const int *step_first, const int *nsteps,
-                                                       const StepInfo *info, float gamma, float lam, float lam_c,
-                                                       float alpha, float2 *out /*[S] (adv, ret)*/) {
+                                                       const int *step_first, const int *nsteps, const float2 *sv,
+                                                       float gamma, float lam, float lam_c, float alpha,
+                                                       float2 *out /*[S] (adv, ret)*/) {
   const int lane = threadIdx.x & 31;
   const int b = (blockIdx.x * 128 + threadIdx.x) >> 5;
   if (b >= B) return;
@@ -293,21 +321,31 @@ __global__ void __launch_bounds__(128) step_gae_kernel(const float *rewards, con
     lb = 1.0 - 1.0 / (double(alpha) * double(n));
     lb = lb < 0.0 ? 0.0 : (lb > 1.0 ? 1.0 : lb);
   }
-  const double g = gamma, ap = g * lb, ac = g * double(lam_c);
-  const double R = rewards[b];
+  const dd ap = dd_from_double(double(gamma) * lb), ac = dd_from_double(double(gamma) * double(lam_c));
+  const dd g = {gamma, 0.f};
+  const float R = rewards[b];
   const int c = (n + 31) / 32;
   const int a0 = s0 + lane * c, a1 = min(a0 + c, s1);  // this lane's steps [a0, a1)
-  // value of the step right after the block (0 after the last step)
-  const double v_after = a1 < s1 ? info[a1].v : 0.0;
-  // fold: A_i = delta_i + a A_{i+1}, delta_i = r_i + g v_{i+1} - v_i
-  StepMap mp{1.0, 0.0}, mc{1.0, 0.0};
+  auto value = [&](int i) {
+    const float2 v = sv[i];
+    return dd{v.x, v.y};
+  };
+  // delta_i = r_i + gamma v_{i+1} - v_i (the reward only on the trajectory's last step)
+  auto delta = [&](int i, dd v, dd v_next) {
+    dd d = dd_add(dd_mul(g, v_next), dd_neg(v));
+    if (i == s1 - 1) d = dd_add(d, dd{R, 0.f});
+    return d;
+  };
+  const dd zero = {0.f, 0.f}, one = {1.f, 0.f};
+  const dd v_after = a1 < s1 ? value(a1) : zero;  // value of the step right after the block
+  StepMap mp{one, zero}, mc{one, zero};
   {
-    double v_next = v_after;
+    dd v_next = v_after;
     for (int i = a1 - 1; i >= a0; --i) {
-      const double v = info[i].v;
-      const double delta = (i == s1 - 1 ? R : 0.0) + g * v_next - v;
-      mp = {ap * mp.p, fma(ap, mp.c, delta)};
-      mc = {ac * mc.p, fma(ac, mc.c, delta)};
+      const dd v = value(i);
+      const dd d = delta(i, v, v_next);
+      mp = {dd_mul(ap, mp.p), dd_add(dd_mul(ap, mp.c), d)};
+      mc = {dd_mul(ac, mc.p), dd_add(dd_mul(ac, mc.c), d)};
       v_next = v;
     }
   }
@@ -315,34 +353,29 @@ __global__ void __launch_bounds__(128) step_gae_kernel(const float *rewards, con
   StepMap sp = mp, sc = mc;
 #pragma unroll
   for (int d = 1; d < 32; d <<= 1) {
-    StepMap op, oc;
-    op.p = __shfl_down_sync(0xffffffffu, sp.p, d);
-    op.c = __shfl_down_sync(0xffffffffu, sp.c, d);
-    oc.p = __shfl_down_sync(0xffffffffu, sc.p, d);
-    oc.c = __shfl_down_sync(0xffffffffu, sc.c, d);
+    const StepMap op{dd_shfl_down(sp.p, d), dd_shfl_down(sp.c, d)};
+    const StepMap oc{dd_shfl_down(sc.p, d), dd_shfl_down(sc.c, d)};
     if (lane + d < 32) {
       sp = compose_steps(sp, op);
       sc = compose_steps(sc, oc);
     }
   }
-  double Ap = __shfl_down_sync(0xffffffffu, sp.c, 1);  // advantage of the step right of the block
-  double Ac = __shfl_down_sync(0xffffffffu, sc.c, 1);
-  if (lane == 31) Ap = Ac = 0.0;
-  // replay
-  double v_next = v_after;
+  dd Ap = dd_shfl_down(sp.c, 1), Ac = dd_shfl_down(sc.c, 1);  // advantages of the step right of the block
+  if (lane == 31) Ap = Ac = zero;
+  dd v_next = v_after;
   for (int i = a1 - 1; i >= a0; --i) {
-    const double v = info[i].v;
-    const double delta = (i == s1 - 1 ? R : 0.0) + g * v_next - v;
-    Ap = fma(ap, Ap, delta);
-    Ac = fma(ac, Ac, delta);
-    out[i] = make_float2(float(Ap), float(Ac + v));
+    const dd v = value(i);
+    const dd d = delta(i, v, v_next);
+    Ap = dd_add(dd_mul(ap, Ap), d);
+    Ac = dd_add(dd_mul(ac, Ac), d);
+    out[i] = make_float2(dd_round(Ap), dd_round(dd_add(Ac, v)));
     v_next = v;
   }
 }
 
 // Every token reads its step's results (non-action tokens get zeros); four
 // consecutive tokens per thread.
-__device__ __forceinline__ void step_result(int s, int64_t t, const StepInfo *info, const float2 *out, int mode,
+__device__ __forceinline__ void step_result(int s, int64_t t, const int *step_end, const float2 *out, int mode,
                                             float &a, float &r, uint8_t &k) {
   a = r = 0.f;
   k = 0;
@@ -350,11 +383,11 @@ __device__ __forceinline__ void step_result(int s, int64_t t, const StepInfo *in
     const float2 o = out[s];
     a = o.x;
     r = o.y;
-    k = (mode == SAO_STEP_AVERAGE || t == int64_t(info[s].end) - 1) ? 1 : 0;
+    k = (mode == SAO_STEP_AVERAGE || t == int64_t(step_end[s]) - 1) ? 1 : 0;
   }
 }
 
-__global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const int *step_id, const StepInfo *info,
+__global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const int *step_id, const int *step_end,
                                                                   const float2 *out, int64_t N, int mode,
                                                                   float *adv, float *ret, uint8_t *vmask) {
   const int64_t stride = int64_t(gridDim.x) * kThreads * 4;
@@ -368,7 +401,7 @@ __global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const int *ste
       float a[4], r[4];
       uint8_t k[4];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) step_result(sv[i], t + i, info, out, mode, a[i], r[i], k[i]);
+      for (int i = 0; i < 4; ++i) step_result(sv[i], t + i, step_end, out, mode, a[i], r[i], k[i]);
       *reinterpret_cast<float4 *>(adv + t) = make_float4(a[0], a[1], a[2], a[3]);
       *reinterpret_cast<float4 *>(ret + t) = make_float4(r[0], r[1], r[2], r[3]);
       if (vmask) *reinterpret_cast<uchar4 *>(vmask + t) = make_uchar4(k[0], k[1], k[2], k[3]);
@@ -376,7 +409,7 @@ __global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const int *ste
       for (int64_t u = t; u < t + 4 && u < N; ++u) {
         float a, r;
         uint8_t k;
-        step_result(step_id[u], u, info, out, mode, a, r, k);
+        step_result(step_id[u], u, step_end, out, mode, a, r, k);
         adv[u] = a;
         ret[u] = r;
         if (vmask) vmask[u] = k;
@@ -391,7 +424,7 @@ size_t step_gae_ws_bytes(int64_t N, int64_t B) {
   (void)B;
   const int64_t nblocks = (N + kRowsPerBlock - 1) / kRowsPerBlock;
   return round256(size_t(N)) + round256(sizeof(int) * (nblocks + 1)) + round256(sizeof(int) * 4) +
-         round256(sizeof(int) * N) + round256(sizeof(int) * N) + round256(sizeof(StepInfo) * N) +
+         round256(sizeof(int) * N) + round256(sizeof(int) * N) + round256(sizeof(int) * N) + round256(sizeof(float2) * N) +
          round256(sizeof(float2) * N);
 }
 
@@ -406,7 +439,8 @@ sao_status step_gae_launch(const float *values, const float *rewards, const uint
   int *nsteps = c.take<int>(4);
   int *step_first = c.take<int>(size_t(N));
   int *step_id = c.take<int>(size_t(N));
-  StepInfo *info = c.take<StepInfo>(size_t(N));
+  int *step_end = c.take<int>(size_t(N));
+  float2 *sv = c.take<float2>(size_t(N));
   float2 *out = c.take<float2>(size_t(N));
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the step-level advantages");
   DeviceInfo di;
@@ -416,18 +450,18 @@ sao_status step_gae_launch(const float *values, const float *rewards, const uint
   mark_traj_starts<<<unsigned((B + 255) / 256), 256, 0, s>>>(cu, B, N, ts);
   step_count_kernel<<<unsigned(nblocks), kThreads, 0, s>>>(m, ts, N, block);
   step_scan_kernel<<<1, 1024, 0, s>>>(block, int(nblocks), nsteps);
-  step_scatter_kernel<<<unsigned(nblocks), kThreads, 0, s>>>(m, ts, N, block, step_first, step_id);
+  step_scatter_kernel<<<unsigned(nblocks), kThreads, 0, s>>>(m, ts, N, block, step_first, step_end, step_id);
   SAO_TRY(launch_end(slot, s));
   const unsigned warps_grid = unsigned(di.sm_count * 8);
   slot = launch_begin("step_gae_reduce", s);
-  step_reduce_kernel<<<warps_grid, kThreads, 0, s>>>(values, m, ts, N, step_first, nsteps, mode, info);
+  step_reduce_kernel<<<warps_grid, kThreads, 0, s>>>(values, step_first, step_end, nsteps, mode, sv);
   SAO_TRY(launch_end(slot, s));
   slot = launch_begin("step_gae_scan", s);
-  step_gae_kernel<<<unsigned((int64_t(B) * 32 + 127) / 128), 128, 0, s>>>(rewards, cu, B, step_first, nsteps, info,
+  step_gae_kernel<<<unsigned((int64_t(B) * 32 + 127) / 128), 128, 0, s>>>(rewards, cu, B, step_first, nsteps, sv,
                                                                           gamma, lam, lam_c, alpha, out);
   SAO_TRY(launch_end(slot, s));
   slot = launch_begin("step_gae_broadcast", s);
-  step_broadcast_kernel<<<warps_grid, kThreads, 0, s>>>(step_id, info, out, N, mode, adv, ret, vmask);
+  step_broadcast_kernel<<<warps_grid, kThreads, 0, s>>>(step_id, step_end, out, N, mode, adv, ret, vmask);
   return launch_end(slot, s);
 }
 
