@@ -24,6 +24,22 @@ using seg::kSegChunk;
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 
+// Compensated fp32 sum (Knuth two-sum): about 48 bits without the fp64 pipe.
+struct Sum2 {
+  float hi = 0.f, lo = 0.f;
+  __device__ __forceinline__ void add(float x) {
+    const float s = __fadd_rn(hi, x);
+    const float bb = __fsub_rn(s, hi);
+    lo = __fadd_rn(lo, __fadd_rn(__fsub_rn(hi, __fsub_rn(s, bb)), __fsub_rn(x, bb)));
+    hi = s;
+  }
+  __device__ __forceinline__ void merge(float ohi, float olo) {
+    add(ohi);
+    lo = __fadd_rn(lo, olo);
+  }
+  __device__ __forceinline__ double value() const { return double(hi) + double(lo); }
+};
+
 struct Norms {
   long long n_action;  // action tokens
   long long n_seq;     // trajectories with at least one action token
@@ -72,8 +88,8 @@ struct ClipArgs {
   float *coef;         // may be null
   uint8_t *flags;      // may be null
   const float *grad_scale;
-  double *part_loss;   // [warps]
-  int *part_cnt;       // [3][warps]
+  float2 *part_loss;   // [CTAs] compensated (hi, lo)
+  int *part_cnt;        // [3][CTAs]
 };
 
 // One token of the clipped surrogate: returns the weighted value term and
@@ -111,164 +127,167 @@ __device__ __forceinline__ float clip_token(float lp, float old, float a, bool a
 template <bool kBwd>
 __global__ void __launch_bounds__(kThreads) clip_loss_kernel(ClipArgs a) {
   __shared__ int32_t s_cu_all[kWarps][kCuCap];
+  __shared__ float2 s_sum[kWarps];
+  __shared__ int s_cnt[3][kWarps];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int q = blockIdx.x * kWarps + warp;
-  const int gw = q;  // partial slot
-  if (q >= a.nchunks) return;
-  int blo, bhi;
-  const CuView cu = seg::stage_chunk(a.cu, a.B, a.nchunks, a.chunk_first, q, lane, s_cu_all[warp], blo, bhi);
-  const Norms nm = *a.norms;
-  const float w_tok = nm.n_action > 0 ? float(1.0 / double(nm.n_action)) : 0.f;
-  const double inv_seq = nm.n_seq > 0 ? 1.0 / double(nm.n_seq) : 0.0;
-  const float gscale = kBwd ? __ldg(a.grad_scale) : 1.f;
-  // window-major: in each 128-token window of the chunk, lane l takes tokens
-  // 4l .. 4l+3, so every warp load and store is one contiguous 512 (or 128)
-  // byte access; each lane's trajectory walk still only moves forward
-  const int64_t c0 = int64_t(q) * kSegChunk;
-  const int64_t N = a.N;
-  int b = blo;
-  int64_t next_end = cu[b + 1];
-  auto weight = [&](int bb) {
-    if (!a.seq) return w_tok;
-    const int L = __ldg(a.nact + bb);
-    return L > 0 ? float(inv_seq / double(L)) : 0.f;
-  };
-  float w = weight(b);
-  float acc_hi = 0.f, acc_lo = 0.f;  // compensated sum of the value terms
+  Sum2 acc;  // compensated sum of the value terms
   int nl = 0, nh = 0, nf = 0;
-  const bool aligned = aligned16_dev(a.logp) && aligned16_dev(a.old) && aligned16_dev(a.adv) &&
-                       ((reinterpret_cast<uintptr_t>(a.m) & 3u) == 0) && (a.coef == nullptr || aligned16_dev(a.coef)) &&
-                       (a.flags == nullptr || (reinterpret_cast<uintptr_t>(a.flags) & 3u) == 0);
-#pragma unroll 1
-  for (int g = 0; g < kSegChunk / 128; ++g) {
-    const int64_t tg = c0 + int64_t(g) * 128 + int64_t(lane) * 4;
-    const bool vec = aligned && tg + 4 <= N;
-    float lp[4], od[4], ad[4];
-    bool act[4];
-    if (vec) {
-      const float4 x = __ldg(reinterpret_cast<const float4 *>(a.logp + tg));
-      const float4 y = __ldg(reinterpret_cast<const float4 *>(a.old + tg));
-      const float4 z = __ldg(reinterpret_cast<const float4 *>(a.adv + tg));
-      const uint32_t mw = __ldg(reinterpret_cast<const unsigned int *>(a.m + tg));
-      lp[0] = x.x; lp[1] = x.y; lp[2] = x.z; lp[3] = x.w;
-      od[0] = y.x; od[1] = y.y; od[2] = y.z; od[3] = y.w;
-      ad[0] = z.x; ad[1] = z.y; ad[2] = z.z; ad[3] = z.w;
+  if (q < a.nchunks) {
+    int blo, bhi;
+    const CuView cu = seg::stage_chunk(a.cu, a.B, a.nchunks, a.chunk_first, q, lane, s_cu_all[warp], blo, bhi);
+    const Norms nm = *a.norms;
+    const float w_tok = nm.n_action > 0 ? float(1.0 / double(nm.n_action)) : 0.f;
+    const double inv_seq = nm.n_seq > 0 ? 1.0 / double(nm.n_seq) : 0.0;
+    const float gscale = kBwd ? __ldg(a.grad_scale) : 1.f;
+    // window-major: in each 128-token window of the chunk, lane l takes tokens
+    // 4l .. 4l+3, so every warp load and store is one contiguous 512 (or 128)
+    // byte access; each lane's trajectory walk still only moves forward
+    const int64_t c0 = int64_t(q) * kSegChunk;
+    const int64_t N = a.N;
+    int b = blo;
+    int64_t next_end = cu[b + 1];
+    auto weight = [&](int bb) {
+      if (!a.seq) return w_tok;
+      const int L = __ldg(a.nact + bb);
+      return L > 0 ? float(inv_seq / double(L)) : 0.f;
+    };
+    float w = weight(b);
+    const bool aligned = aligned16_dev(a.logp) && aligned16_dev(a.old) && aligned16_dev(a.adv) &&
+                         ((reinterpret_cast<uintptr_t>(a.m) & 3u) == 0) && (a.coef == nullptr || aligned16_dev(a.coef)) &&
+                         (a.flags == nullptr || (reinterpret_cast<uintptr_t>(a.flags) & 3u) == 0);
+  #pragma unroll 1
+    for (int g = 0; g < kSegChunk / 128; ++g) {
+      const int64_t tg = c0 + int64_t(g) * 128 + int64_t(lane) * 4;
+      const bool vec = aligned && tg + 4 <= N;
+      float lp[4], od[4], ad[4];
+      bool act[4];
+      if (vec) {
+        const float4 x = __ldg(reinterpret_cast<const float4 *>(a.logp + tg));
+        const float4 y = __ldg(reinterpret_cast<const float4 *>(a.old + tg));
+        const float4 z = __ldg(reinterpret_cast<const float4 *>(a.adv + tg));
+        const uint32_t mw = __ldg(reinterpret_cast<const unsigned int *>(a.m + tg));
+        lp[0] = x.x; lp[1] = x.y; lp[2] = x.z; lp[3] = x.w;
+        od[0] = y.x; od[1] = y.y; od[2] = y.z; od[3] = y.w;
+        ad[0] = z.x; ad[1] = z.y; ad[2] = z.z; ad[3] = z.w;
 #pragma unroll
-      for (int i = 0; i < 4; ++i) act[i] = ((mw >> (8 * i)) & 0xffu) != 0u;
-    } else {
+        for (int i = 0; i < 4; ++i) act[i] = ((mw >> (8 * i)) & 0xffu) != 0u;
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const bool in = tg + i < N;
+          lp[i] = in ? a.logp[tg + i] : 0.f;
+          od[i] = in ? a.old[tg + i] : 0.f;
+          ad[i] = in ? a.adv[tg + i] : 0.f;
+          act[i] = in && a.m[tg + i] != 0;
+        }
+      }
+      float cf[4];
+      uint8_t fl[4];
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        const bool in = tg + i < N;
-        lp[i] = in ? a.logp[tg + i] : 0.f;
-        od[i] = in ? a.old[tg + i] : 0.f;
-        ad[i] = in ? a.adv[tg + i] : 0.f;
-        act[i] = in && a.m[tg + i] != 0;
+        const int64_t t = tg + i;
+        if (a.seq && t < N && t >= next_end) {
+          while (b < bhi && t >= next_end) {
+            ++b;
+            next_end = cu[b + 1];
+          }
+          w = weight(b);
+        }
+        acc.add(clip_token(lp[i], od[i], ad[i], act[i], a.lo, a.hi, w, cf[i], fl[i], nl, nh, nf));
+        cf[i] *= gscale;
+      }
+      if (vec) {
+        if (a.coef) *reinterpret_cast<float4 *>(a.coef + tg) = make_float4(cf[0], cf[1], cf[2], cf[3]);
+        if (a.flags && !kBwd) *reinterpret_cast<uchar4 *>(a.flags + tg) = make_uchar4(fl[0], fl[1], fl[2], fl[3]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (tg + i < N) {
+            if (a.coef) a.coef[tg + i] = cf[i];
+            if (a.flags && !kBwd) a.flags[tg + i] = fl[i];
+          }
       }
     }
-    float cf[4];
-    uint8_t fl[4];
+  }
+  if constexpr (!kBwd) {
+    // warp, then CTA (fixed order), in compensated fp32
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int64_t t = tg + i;
-      if (a.seq && t < N && t >= next_end) {
-        while (b < bhi && t >= next_end) {
-          ++b;
-          next_end = cu[b + 1];
-        }
-        w = weight(b);
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ohi = __shfl_xor_sync(0xffffffffu, acc.hi, o), olo = __shfl_xor_sync(0xffffffffu, acc.lo, o);
+      acc.merge(ohi, olo);
+      nl += __shfl_xor_sync(0xffffffffu, nl, o);
+      nh += __shfl_xor_sync(0xffffffffu, nh, o);
+      nf += __shfl_xor_sync(0xffffffffu, nf, o);
+    }
+    if (lane == 0) {
+      s_sum[warp] = make_float2(acc.hi, acc.lo);
+      s_cnt[0][warp] = nl;
+      s_cnt[1][warp] = nh;
+      s_cnt[2][warp] = nf;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      Sum2 t;
+      int l = 0, h = 0, f = 0;
+      for (int k = 0; k < kWarps; ++k) {
+        t.merge(s_sum[k].x, s_sum[k].y);
+        l += s_cnt[0][k];
+        h += s_cnt[1][k];
+        f += s_cnt[2][k];
       }
-      const float term = clip_token(lp[i], od[i], ad[i], act[i], a.lo, a.hi, w, cf[i], fl[i], nl, nh, nf);
-      // compensated accumulation (Knuth two-sum)
-      const float s = __fadd_rn(acc_hi, term);
-      const float bb = __fsub_rn(s, acc_hi);
-      acc_lo = __fadd_rn(acc_lo, __fadd_rn(__fsub_rn(acc_hi, __fsub_rn(s, bb)), __fsub_rn(term, bb)));
-      acc_hi = s;
-      cf[i] *= gscale;
+      a.part_loss[blockIdx.x] = make_float2(t.hi, t.lo);
+      a.part_cnt[blockIdx.x] = l;
+      a.part_cnt[gridDim.x + blockIdx.x] = h;
+      a.part_cnt[2 * gridDim.x + blockIdx.x] = f;
     }
-    if (vec) {
-      if (a.coef) *reinterpret_cast<float4 *>(a.coef + tg) = make_float4(cf[0], cf[1], cf[2], cf[3]);
-      if (a.flags && !kBwd) *reinterpret_cast<uchar4 *>(a.flags + tg) = make_uchar4(fl[0], fl[1], fl[2], fl[3]);
-    } else {
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-        if (tg + i < N) {
-          if (a.coef) a.coef[tg + i] = cf[i];
-          if (a.flags && !kBwd) a.flags[tg + i] = fl[i];
-        }
-    }
-  }
-  if (kBwd) return;
-  double sum = double(acc_hi) + double(acc_lo);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    nl += __shfl_xor_sync(0xffffffffu, nl, o);
-    nh += __shfl_xor_sync(0xffffffffu, nh, o);
-    nf += __shfl_xor_sync(0xffffffffu, nf, o);
-  }
-  if (lane == 0) {
-    a.part_loss[gw] = sum;
-    a.part_cnt[gw] = nl;
-    a.part_cnt[a.nchunks + gw] = nh;
-    a.part_cnt[2 * a.nchunks + gw] = nf;
   }
 }
 
-__global__ void __launch_bounds__(256) clip_finalize_kernel(const double *part_loss, const int *part_cnt, int n,
+__global__ void __launch_bounds__(256) clip_finalize_kernel(const float2 *part_loss, const int *part_cnt, int n,
                                                             const Norms *norms, float *loss, int64_t *counts) {
-  double s = 0.0;
+  Sum2 acc;
   long long l = 0, h = 0, f = 0;
   for (int i = threadIdx.x; i < n; i += 256) {
-    s += part_loss[i];
+    acc.merge(part_loss[i].x, part_loss[i].y);
     l += part_cnt[i];
     h += part_cnt[n + i];
     f += part_cnt[2 * n + i];
   }
-  __shared__ double sd[8];
+  __shared__ float2 sd[8];
   __shared__ long long sl[3][8];
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    s += __shfl_xor_sync(0xffffffffu, s, o);
+    const float ohi = __shfl_xor_sync(0xffffffffu, acc.hi, o), olo = __shfl_xor_sync(0xffffffffu, acc.lo, o);
+    acc.merge(ohi, olo);
     l += __shfl_xor_sync(0xffffffffu, l, o);
     h += __shfl_xor_sync(0xffffffffu, h, o);
     f += __shfl_xor_sync(0xffffffffu, f, o);
   }
   const int w = threadIdx.x >> 5;
   if ((threadIdx.x & 31) == 0) {
-    sd[w] = s;
+    sd[w] = make_float2(acc.hi, acc.lo);
     sl[0][w] = l;
     sl[1][w] = h;
     sl[2][w] = f;
   }
   __syncthreads();
   if (threadIdx.x == 0) {
-    double S = 0.0;
+    Sum2 T;
     long long L = 0, Hh = 0, F = 0;
     for (int k = 0; k < 8; ++k) {
-      S += sd[k];
+      T.merge(sd[k].x, sd[k].y);
       L += sl[0][k];
       Hh += sl[1][k];
       F += sl[2][k];
     }
-    *loss = float(-S);
+    *loss = float(-T.value());
     counts[0] = norms->n_action;
     counts[1] = L;
     counts[2] = Hh;
     counts[3] = F;
   }
 }
-
-// Compensated fp32 sum (Knuth two-sum): about 48 bits without the fp64 pipe.
-struct Sum2 {
-  float hi = 0.f, lo = 0.f;
-  __device__ __forceinline__ void add(float x) {
-    const float s = __fadd_rn(hi, x);
-    const float bb = __fsub_rn(s, hi);
-    lo = __fadd_rn(lo, __fadd_rn(__fsub_rn(hi, __fsub_rn(s, bb)), __fsub_rn(x, bb)));
-    hi = s;
-  }
-  __device__ __forceinline__ double value() const { return double(hi) + double(lo); }
-};
 
 // GRPO: per-trajectory standardised reward within its group. Every thread
 // scans all trajectories for its group's members, through shared-memory tiles
@@ -419,7 +438,7 @@ sao_status clip_loss_launch(const float *logp, const float *old, const float *ad
   int *chunk_first = c.take<int>(size_t(nchunks) + 1);
   int *nact = c.take<int>(size_t(B) + 1);
   Norms *norms = c.take<Norms>(1);
-  double *part_loss = c.take<double>(size_t(nchunks));
+  float2 *part_loss = c.take<float2>(size_t(nchunks));
   int *part_cnt = c.take<int>(3 * size_t(nchunks));
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the clipped surrogate");
   if (N == 0) {
@@ -461,7 +480,9 @@ sao_status clip_loss_launch(const float *logp, const float *old, const float *ad
   }
   slot = launch_begin("clip_loss_fwd", s);
   clip_loss_kernel<false><<<grid, kThreads, 0, s>>>(a);
-  clip_finalize_kernel<<<1, 256, 0, s>>>(part_loss, part_cnt, int(nchunks), norms, loss, counts);
+  SAO_TRY(launch_end(slot, s));
+  slot = launch_begin("clip_loss_finalize", s);
+  clip_finalize_kernel<<<1, 256, 0, s>>>(part_loss, part_cnt, int(grid), norms, loss, counts);
   return launch_end(slot, s);
 }
 

@@ -70,7 +70,9 @@ __global__ void chunk_first_kernel(const int32_t *cu, int B, int64_t N, int nchu
 }
 
 // Number of action tokens per trajectory; nact must start at zero. One warp
-// per chunk, 8 warps per CTA.
+// per chunk, 8 warps per CTA; in each 512-token window of the chunk lane l
+// reads tokens 16l .. 16l+15 (one contiguous 512-byte warp load), and each
+// lane's trajectory walk only moves forward.
 __global__ void __launch_bounds__(256) action_count_kernel(const uint8_t *m, const int32_t *cu_g, int B, int64_t N,
                                                            int nchunks, const int *chunk_first, int *nact) {
   __shared__ int32_t s_cu_all[8][kCuCap];
@@ -79,29 +81,31 @@ __global__ void __launch_bounds__(256) action_count_kernel(const uint8_t *m, con
   if (q >= nchunks) return;
   int blo, bhi;
   const CuView cu = stage_chunk(cu_g, B, nchunks, chunk_first, q, lane, s_cu_all[warp], blo, bhi);
-  const int64_t t0 = int64_t(q) * kSegChunk + int64_t(lane) * kItems;
-  int b = cu.find(blo, bhi, t0 < N ? t0 : N - 1);
+  const int64_t c0 = int64_t(q) * kSegChunk;
+  int b = blo;
   int64_t next_end = cu[b + 1];
   int cnt = 0;
-  const bool vec = (t0 + kItems <= N) && ((reinterpret_cast<uintptr_t>(m) & 15u) == 0);
+  const bool aligned = (reinterpret_cast<uintptr_t>(m) & 15u) == 0;
 #pragma unroll 1
-  for (int g = 0; g < kItems / 16; ++g) {
+  for (int g = 0; g < kSegChunk / 512; ++g) {
+    const int64_t t0 = c0 + int64_t(g) * 512 + int64_t(lane) * 16;
+    if (t0 >= N) break;
     uint32_t w[4] = {0u, 0u, 0u, 0u};
-    if (vec) {
-      const uint4 x = __ldg(reinterpret_cast<const uint4 *>(m + t0) + g);
+    if (aligned && t0 + 16 <= N) {
+      const uint4 x = __ldg(reinterpret_cast<const uint4 *>(m + t0));
       w[0] = x.x;
       w[1] = x.y;
       w[2] = x.z;
       w[3] = x.w;
     } else {
       for (int k = 0; k < 16; ++k) {
-        const int64_t t = t0 + 16 * g + k;
+        const int64_t t = t0 + k;
         if (t < N && m[t] != 0) w[k >> 2] |= 1u << (8 * (k & 3));
       }
     }
 #pragma unroll
     for (int k = 0; k < 16; ++k) {
-      const int64_t t = t0 + 16 * g + k;
+      const int64_t t = t0 + k;
       if (t >= N) break;
       if (t >= next_end) {
         const int nb0 = b;
