@@ -552,24 +552,41 @@ __global__ void __launch_bounds__(kDzThreads) dz_from_cache_kernel(
   const float l2 = __ldg(lse + t) * kLog2e;
   const int yy = __ldg(y + t) - v0;
   const __nv_bfloat16 *src = e + int64_t(f) * lde + v0;
-  for (int k = threadIdx.x * 8; k < vc; k += kDzThreads * 8) {
-    // the 8 columns share one 256-wide tile (v0 and k are multiples of 8)
-    const float s = ex2_approx(fmaf(__ldg(&part[int64_t((v0 + k) / BN) * N + f].x), kLog2e, -l2));
-    const float gs = g * s;
-    if (k + 8 <= vc) {
-      const uint4 q = __ldcs(reinterpret_cast<const uint4 *>(src + k));
-      const uint32_t w[4] = {q.x, q.y, q.z, q.w};
-      uint32_t o[4];
+  // the 8 columns of a vector share one 256-wide tile (v0 and k are multiples of 8)
+  auto scale = [&](int k) { return g * ex2_approx(fmaf(__ldg(&part[int64_t((v0 + k) / BN) * N + f].x), kLog2e, -l2)); };
+  auto dz8 = [&](const uint4 q, float gs, int k) {
+    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+    uint32_t o[4];
 #pragma unroll
-      for (int h2 = 0; h2 < 4; ++h2) {
-        const float2 ev = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[h2]));
-        float d0 = -gs * ev.x, d1 = -gs * ev.y;
-        if (k + 2 * h2 == yy) d0 += g;
-        if (k + 2 * h2 + 1 == yy) d1 += g;
-        const __nv_bfloat162 b2 = __floats2bfloat162_rn(d0, d1);
-        o[h2] = *reinterpret_cast<const uint32_t *>(&b2);
-      }
-      __stcs(reinterpret_cast<uint4 *>(out + k), make_uint4(o[0], o[1], o[2], o[3]));
+    for (int h2 = 0; h2 < 4; ++h2) {
+      const float2 ev = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[h2]));
+      float d0 = -gs * ev.x, d1 = -gs * ev.y;
+      if (k + 2 * h2 == yy) d0 += g;
+      if (k + 2 * h2 + 1 == yy) d1 += g;
+      const __nv_bfloat162 b2 = __floats2bfloat162_rn(d0, d1);
+      o[h2] = *reinterpret_cast<const uint32_t *>(&b2);
+    }
+    return make_uint4(o[0], o[1], o[2], o[3]);
+  };
+  constexpr int kStep = kDzThreads * 8, kUnroll = 4;
+  int k = threadIdx.x * 8;
+  // kUnroll independent 16-byte loads in flight per thread
+  for (; k + (kUnroll - 1) * kStep + 8 <= vc; k += kUnroll * kStep) {
+    uint4 q[kUnroll];
+    float gs[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      q[u] = __ldcs(reinterpret_cast<const uint4 *>(src + k + u * kStep));
+      gs[u] = scale(k + u * kStep);
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u)
+      __stcs(reinterpret_cast<uint4 *>(out + k + u * kStep), dz8(q[u], gs[u], k + u * kStep));
+  }
+  for (; k < vc; k += kStep) {
+    const float gs = scale(k);
+    if (k + 8 <= vc) {
+      __stcs(reinterpret_cast<uint4 *>(out + k), dz8(__ldcs(reinterpret_cast<const uint4 *>(src + k)), gs, k));
     } else {
       for (int j = k; j < vc; ++j) {
         float d = -gs * __bfloat162float(src[j]);
