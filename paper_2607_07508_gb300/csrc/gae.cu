@@ -29,9 +29,11 @@
 //   * warps chain their chunks right-to-left by decoupled look-back: each CTA
 //     takes one ticket and its warps work on the chunks below it, so a warp
 //     only ever waits on chunks whose warps started before it; the look-back
-//     inspects 32 predecessors at once; maps and states are published as
-//     tagged 8-byte words, so neither side needs a fence; every wait is
-//     bounded and a time-out raises SAO_DEVERR_SCAN_TIMEOUT,
+//     polls 32 predecessors at once and carries the nearest known state
+//     through the maps before it one by one (so results do not depend on
+//     timing); maps and states are published as tagged 8-byte words, so
+//     neither side needs a fence; every wait is bounded and a time-out raises
+//     SAO_DEVERR_SCAN_TIMEOUT,
 //   * each lane then replays its tokens from its incoming state, writing A
 //     and the return into shared memory, and the warp stores both coalesced.
 // Traffic: values 4 B + mask 1 B read, adv 4 B + ret 4 B written per token.
@@ -354,69 +356,51 @@ struct GaeArgs {
 using seg::CuView;
 using seg::kCuCap;
 
-// A look-back round whose first known chunk is at most this many chunks away
-// applies the maps one by one instead of composing them in log depth.
-constexpr int kSerialWalk = 6;
 
 // State at the right edge of chunk q, from the chunks to its right. The warp
-// inspects 32 successors (q+1 .. q+32) per round: each lane polls one chunk's
-// published state and map; the first chunk whose left-edge state is known
-// (published state, a map that ignores its right neighbour, or the end of the
-// input) ends the walk, and the maps of the chunks before it are applied one
-// by one when there are few of them, else composed by a log-depth shuffle
-// scan. A round waits (bounded) only for chunks before that point.
+// polls the 32 successors q+1 .. q+32, each lane one chunk's published state
+// and map, until the first chunk whose left-edge state is known (published
+// state, a map that ignores its right neighbour, or the end of the input) lies
+// in that window with every map before it published; the state then goes
+// through the maps of the chunks before it one by one. Every state is thus
+// the same chain of map applications from the nearest trajectory end, however
+// the warps were timed, and the results are bit-identical from run to run.
+// The wait ends: the highest unfinished chunk only waits on finished ones.
+// Every wait is bounded.
 template <bool kCrit>
 __device__ GState look_back(const GaeArgs &a, int q, int lane) {
-  GMap<kCrit> acc = identity_map<kCrit>();  // maps of the chunks already walked (lane 0)
   const uint64_t t_start = globaltimer_ns();
-  for (int base = q + 1;; base += 32) {
-    const int j = base + lane;
-    GMap<kCrit> mj = identity_map<kCrit>();
-    GState sj = zero_state();
-    int kind = 2;  // 0: nothing published yet, 1: map, 2: left-edge state known
-    uint32_t polls = 0;
-    for (;;) {
-      if (j < a.nchunks) {
-        const bool has_s = fetch_state<kCrit>(a.incl + size_t(j) * kStateWords<kCrit>, sj);
-        const bool has_m = fetch_map<kCrit>(a.agg + size_t(j) * kMapWords<kCrit>, mj);
-        kind = has_s ? 2 : (has_m ? 1 : 0);
-        if (kind == 1 && (mj.fl & 1)) {  // the map ignores its right neighbour
-          sj = apply<kCrit>(mj, zero_state());
-          kind = 2;
-        }
+  const int j = q + 1 + lane;
+  GMap<kCrit> mj = identity_map<kCrit>();
+  GState sj = zero_state();
+  int kind = 2;  // 0: nothing published yet, 1: map, 2: left-edge state known
+  uint32_t polls = 0;
+  int stop;
+  for (;;) {
+    if (j < a.nchunks) {
+      const bool has_s = fetch_state<kCrit>(a.incl + size_t(j) * kStateWords<kCrit>, sj);
+      const bool has_m = fetch_map<kCrit>(a.agg + size_t(j) * kMapWords<kCrit>, mj);
+      kind = has_s ? 2 : (has_m ? 1 : 0);
+      if (kind == 1 && (mj.fl & 1)) {  // the map ignores its right neighbour
+        sj = apply<kCrit>(mj, zero_state());
+        kind = 2;
       }
-      const unsigned bt = __ballot_sync(0xffffffffu, kind == 2);
-      const unsigned bn = __ballot_sync(0xffffffffu, kind == 0);
-      const int first_term = bt ? __ffs(bt) - 1 : 32;
-      const int first_nr = bn ? __ffs(bn) - 1 : 32;
-      if (first_nr >= first_term) break;  // everything up to the first terminal chunk is known
-      if ((++polls & 31u) == 0u && globaltimer_ns() - t_start > kWaitLimitNs) {
-        if (lane == 0) raise_device_error(a.err, SAO_DEVERR_SCAN_TIMEOUT);
-        return zero_state();
-      }
-      __nanosleep(64);
     }
     const unsigned bt = __ballot_sync(0xffffffffu, kind == 2);
-    const int stop = bt ? __ffs(bt) - 1 : 32;
-    if (stop <= kSerialWalk) {
-      // near terminal: carry its state through the maps of lanes stop-1 .. 0
-      GState cur = shfl_state(sj, stop);
-      for (int i = stop - 1; i >= 0; --i) cur = shfl_state(apply<kCrit>(mj, cur), i);
-      return shfl_state(apply<kCrit>(acc, cur), 0);  // acc is meaningful in lane 0
+    const unsigned bn = __ballot_sync(0xffffffffu, kind == 0);
+    stop = bt ? __ffs(bt) - 1 : 32;
+    const int first_nr = bn ? __ffs(bn) - 1 : 32;
+    if (stop < 32 && first_nr > stop) break;  // a known state, and every map before it
+    if ((++polls & 31u) == 0u && globaltimer_ns() - t_start > kWaitLimitNs) {
+      if (lane == 0) raise_device_error(a.err, SAO_DEVERR_SCAN_TIMEOUT);
+      return zero_state();
     }
-    // compose maps of lanes [0, stop): suffix scan, lane 0 ends with m_0 o ... o m_{stop-1}
-    GMap<kCrit> m = lane < stop ? mj : identity_map<kCrit>();
-#pragma unroll 1
-    for (int d = 1; d < 32; d <<= 1) {
-      const GMap<kCrit> o = shfl_down_map<kCrit>(m, d);
-      if (lane + d < 32) m = compose<kCrit>(m, o);
-    }
-    if (lane == 0) acc = compose<kCrit>(acc, m);
-    if (stop < 32) {
-      const GState tstate = shfl_state(sj, stop);
-      return shfl_state(apply<kCrit>(acc, tstate), 0);  // meaningful in lane 0
-    }
+    __nanosleep(64);
   }
+  // carry the known state through the maps of lanes stop-1 .. 0
+  GState cur = shfl_state(sj, stop);
+  for (int i = stop - 1; i >= 0; --i) cur = shfl_state(apply<kCrit>(mj, cur), i);
+  return cur;
 }
 
 // ---------------------------------------------------------------------------
