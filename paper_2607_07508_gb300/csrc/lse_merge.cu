@@ -30,13 +30,23 @@ __global__ void __launch_bounds__(256) lse_merge_kernel(const float2 *__restrict
     }
     src = i;
   }
-  float m = -INFINITY;
-  for (int j = 0; j < nvt; ++j) m = fmaxf(m, __ldcs(&part[int64_t(j) * N + src].x));
-  float s = 0.f;
-  for (int j = 0; j < nvt; ++j) {
-    const float2 p = __ldcs(part + int64_t(j) * N + src);
-    s = fmaf(p.y, expf(p.x - m), s);
+  // one online pass: (m, s) = running maximum and sum of exp(z - m); four
+  // tiles' partials in flight per thread
+  float m = -INFINITY, s = 0.f;
+  auto merge = [&](float2 p) {
+    const float mn = fmaxf(m, p.x);
+    s = fmaf(s, expf(m - mn), p.y * expf(p.x - mn));  // every tile holds a finite maximum
+    m = mn;
+  };
+  int j = 0;
+  for (; j + 4 <= nvt; j += 4) {
+    float2 p[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) p[u] = __ldcs(part + int64_t(j + u) * N + src);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) merge(p[u]);
   }
+  for (; j < nvt; ++j) merge(__ldcs(part + int64_t(j) * N + src));
   const float l = m + logf(s);
   lse[row] = l;
   const int yy = y[row];
