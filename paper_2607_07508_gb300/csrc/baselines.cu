@@ -18,7 +18,6 @@ namespace {
 
 using seg::CuView;
 using seg::kCuCap;
-using seg::kItems;
 using seg::kSegChunk;
 
 constexpr int kThreads = 256;
