@@ -36,10 +36,13 @@ WORKLOAD = "moe"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
-def stored_traffic(kernel: str, rows: int):
+def stored_traffic(kernel: str, rows: int, workload: str = "moe"):
     """DRAM bytes per launch of `kernel` from the committed ncu capture
-    (profiles/dram_traffic_moe.txt), scaled to `rows` active rows, or None if
-    the capture is missing or the kernel sources changed since it was taken."""
+    (profiles/dram_traffic_moe.txt, taken on the moe shape), scaled to `rows`
+    active rows, or None for another shape, a missing capture, or kernel
+    sources changed since it was taken."""
+    if workload != "moe":
+        return None
     from paper_2607_07508_gb300.build import kernel_source_hash
     path = os.path.join(ROOT, "profiles", "dram_traffic_moe.txt")
     try:
@@ -278,7 +281,7 @@ def run_reference(args):
         return 0
     from paper_2607_07508_gb300 import synthetic as S
     import torch
-    wl = S.make_workload(WORKLOAD, device="cpu")
+    wl = S.make_workload(args.config, device="cpu")
     H_cpu, W_cpu = wl.H, wl.W
     rows = max(8, choose_rows(wl, H_cpu, W_cpu, budget_s=8.0) // 2)
     for _ in range(args.warmup if args.warmup < 1 else 1):
@@ -301,11 +304,16 @@ def run_reference(args):
 
 
 def workload_config(wl):
-    return {"workload": f"{wl.name}: MoE-policy head, {wl.N} packed tokens in {wl.B} single-rollout agentic "
-                        f"trajectories (lognormal lengths, median 4k, max 32k), 25% observation tokens",
+    if wl.name == "moe":
+        what = (f"moe: MoE-policy head, {wl.N} packed tokens in {wl.B} single-rollout agentic trajectories "
+                f"(lognormal lengths, median 4k, max 32k), 25% observation tokens")
+    else:
+        what = f"{wl.name}: {wl.N} packed tokens in {wl.B} trajectories; {wl.recipe}"
+    return {"workload": what,
             "tokens": wl.N, "trajectories": wl.B, "hidden": wl.h, "vocab": wl.V, "dtype": wl.dtype,
             "gamma": wl.gamma, "lambda": wl.lam, "eps_low": wl.eps_low, "eps_high": wl.eps_high,
-            "l2": "inputs larger than L2 (H 268 MB + W 622 MB per step, L2 126 MB); no flush"}
+            "l2": (f"inputs larger than L2 (H {wl.N * wl.h * 2 / 1e6:.0f} MB + W {wl.V * wl.h * 2 / 1e6:.0f} MB per step, "
+                   f"L2 126 MB); no flush")}
 
 
 # Algorithmic bytes per token of each O(N) kernel (reads + writes).
@@ -442,6 +450,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--tokens", type=int, default=None,
                     help="override the packed token count (smaller cases for profiling captures)")
+    ap.add_argument("--config", default=WORKLOAD, choices=["tiny", "small", "moe", "long", "large"],
+                    help="workload (the metric is quoted on moe; the others are the parity configurations)")
     ap.add_argument("--recompute", action="store_true",
                     help="backward recomputes the logits instead of reading the forward's stored probabilities")
     ap.add_argument("--bandwidth-study", action="store_true",
@@ -464,7 +474,7 @@ def main():
     sao.load()
     peaks, peak_src = load_peaks()
 
-    wl = S.make_workload(WORKLOAD, device=dev, seed=S.SEED_BASE + S.CONFIG_NAMES.index(WORKLOAD) + 97 * rank,
+    wl = S.make_workload(args.config, device=dev, seed=S.SEED_BASE + S.CONFIG_NAMES.index(args.config) + 97 * rank,
                          N_override=args.tokens)
     step = LossHeadStep(wl, dev, torch, cached=not args.recompute)
     stream = torch.cuda.current_stream()
@@ -518,7 +528,7 @@ def main():
         achieved = fl / (avg_ms / 1000.0) / 1e12
         dom_rows = rows_fwd if dom_name == "tc_logits_lse_fwd" else rows_bwd
         roofline = {"bound": "tensor", "kernel": dom_name, "achieved": achieved, "peak": peak_t,
-                    "unit": "TFLOP/s", "frac": achieved / peak_t, "traffic": stored_traffic(dom_name, dom_rows),
+                    "unit": "TFLOP/s", "frac": achieved / peak_t, "traffic": stored_traffic(dom_name, dom_rows, wl.name),
                     "traffic_unit": "bytes per launch (dram read + write, ncu, scaled by active rows)",
                     "algorithmic_per_launch": f"2*rows*h*V = {fl:.4g} flop", "avg_launch_ms": avg_ms,
                     "peak_source": f"{peak_src} bf16_tflops_sustained (kernel timed inside a long step)"}

@@ -98,6 +98,18 @@ SAO_API int sao_get_checked(void);
  * add an fp32 dH accumulator. Affects sao_workspace_bytes. Process-wide. */
 SAO_API void sao_set_dz_budget_bytes(size_t bytes);
 
+/*
+ * Test hooks of the advantage scan (process-wide; defaults restored by
+ * (0, 0)): every look-back wait gives up after wait_ns nanoseconds (0: the
+ * default 2 s; longer values are capped at it), and the scan's top
+ * skip_chunks 1024-token chunks are never processed, so the chunks below them
+ * wait for a carry that never comes. Failure-detection tests use them to make
+ * the bounded wait run out: the call still completes, the context stays
+ * usable, and checked mode reports SAO_DEVERR_SCAN_TIMEOUT. Not for
+ * production use (the skipped chunks' outputs are left unwritten).
+ */
+SAO_API void sao_debug_set_scan_hooks(uint64_t wait_ns, int32_t skip_chunks);
+
 /* Workspace bytes that every entry point needs for N tokens, hidden size h,
  * vocabulary V and dtype dt (pass h = V = 0 when only the O(N) calls are
  * used). Returns 0 for invalid sizes. */

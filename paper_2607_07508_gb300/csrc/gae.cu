@@ -351,6 +351,7 @@ struct GaeArgs {
   uint64_t *incl;          // [nchunks][kStateWords]: state at the chunk's left edge
   float *adv, *ret;
   unsigned int *err;
+  uint64_t wait_ns;        // bound of every look-back wait
 };
 
 using seg::CuView;
@@ -391,7 +392,7 @@ __device__ GState look_back(const GaeArgs &a, int q, int lane) {
     stop = bt ? __ffs(bt) - 1 : 32;
     const int first_nr = bn ? __ffs(bn) - 1 : 32;
     if (stop < 32 && first_nr > stop) break;  // a known state, and every map before it
-    if ((++polls & 31u) == 0u && globaltimer_ns() - t_start > kWaitLimitNs) {
+    if ((++polls & 31u) == 0u && globaltimer_ns() - t_start > a.wait_ns) {
       if (lane == 0) raise_device_error(a.err, SAO_DEVERR_SCAN_TIMEOUT);
       return zero_state();
     }
@@ -770,6 +771,11 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) gae_scan_kernel(GaeArgs 
   }
 }
 
+// Test hook: the scan's first `skip` tickets are taken before any warp runs,
+// so the top chunks are never processed and the chunks below them wait for
+// states that never come (until the bounded wait gives up).
+__global__ void preset_ticket_kernel(int *ticket, int skip) { *ticket = skip; }
+
 // Per-trajectory coefficients (fp64 then split to double-float) and a check of
 // cu_seqlens: 0 = cu[0] <= cu[1] <= ... <= cu[B] = N.
 __global__ void gae_coef_kernel(const int32_t *cu, int B, int64_t N, float gamma, float lam, float lam_c,
@@ -840,6 +846,10 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   int *chunk_first = c.take<int>(size_t(nchunks) + 1);
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the advantage scan");
   SAO_CUDA_TRY(cudaMemsetAsync(zero_begin, 0, size_t(zero_end - zero_begin), s));
+  if (const int skip = scan_skip(); skip > 0) {
+    preset_ticket_kernel<<<1, 1, 0, s>>>(ticket, skip);
+    SAO_CUDA_TRY(cudaGetLastError());
+  }
   {
     int slot = launch_begin("gae_chunk_first", s);
     seg::chunk_first_kernel<<<unsigned((nchunks + 255) / 256), 256, 0, s>>>(cu, B, N, int(nchunks), chunk_first);
@@ -872,6 +882,7 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   a.adv = adv;
   a.ret = ret;
   a.err = err;
+  a.wait_ns = scan_wait_ns();
   DeviceInfo di;
   SAO_TRY(device_info(&di));
   auto kern = crit_trivial ? gae_scan_kernel<false> : gae_scan_kernel<true>;

@@ -5,6 +5,8 @@
 
 #include <atomic>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "logprobs_common.cuh"
 #include "sao_common.cuh"
 #include "sao_internal.h"
@@ -14,6 +16,11 @@ namespace sao {
 static std::atomic<size_t> g_dz_budget{size_t(24) << 30};
 void set_dz_budget(size_t bytes) { g_dz_budget.store(bytes < (size_t(1) << 20) ? (size_t(1) << 20) : bytes); }
 size_t dz_budget() { return g_dz_budget.load(); }
+
+static std::atomic<uint64_t> g_scan_wait_ns{kWaitLimitNs};
+static std::atomic<int> g_scan_skip{0};
+uint64_t scan_wait_ns() { return g_scan_wait_ns.load(); }
+int scan_skip() { return g_scan_skip.load(); }
 
 // O(N) kernels size their grids from N alone (deterministic on any device).
 size_t on_ws_bytes(int64_t N) {
@@ -37,6 +44,16 @@ size_t logprobs_ws_bytes(int64_t N, int32_t h, int32_t V, sao_dtype dt) {
 using namespace sao;
 
 namespace {
+
+// An NVTX range around every entry point, so a profiler timeline shows the
+// ABI calls with their kernels (header-only NVTX: no cost without a tool).
+struct NvtxRange {
+  explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange &) = delete;
+  NvtxRange &operator=(const NvtxRange &) = delete;
+};
+#define SAO_RANGE() NvtxRange sao_nvtx_range_(__func__)
 
 struct Ws {
   unsigned int *err;
@@ -88,6 +105,11 @@ int sao_get_checked(void) { return checked_mode() ? 1 : 0; }
 
 void sao_set_dz_budget_bytes(size_t bytes) { set_dz_budget(bytes); }
 
+void sao_debug_set_scan_hooks(uint64_t wait_ns, int32_t skip_chunks) {
+  g_scan_wait_ns.store(wait_ns == 0 ? kWaitLimitNs : (wait_ns > kWaitLimitNs ? kWaitLimitNs : wait_ns));
+  g_scan_skip.store(skip_chunks > 0 ? skip_chunks : 0);
+}
+
 size_t sao_workspace_bytes(int64_t N, int32_t h, int32_t V, sao_dtype dt) {
   if (N < 0 || h < 0 || V < 0 || bad_dtype(dt)) return 0;
   size_t body = on_ws_bytes(N);
@@ -99,6 +121,7 @@ size_t sao_workspace_bytes(int64_t N, int32_t h, int32_t V, sao_dtype dt) {
 sao_status sao_token_logprobs_fwd(const void *H, const void *W, sao_dtype dt, const int32_t *y,
                                   const uint8_t *row_mask, int64_t N, int32_t h, int32_t V, float *logp,
                                   float *lse, void *ws, size_t ws_bytes, sao_stream_t stream) {
+  SAO_RANGE();
   SAO_TRY(check_logprob_shapes(dt, N, h, V));
   if (N == 0) return SAO_OK;
   if (!H || !W || !y || !logp || !lse) return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
@@ -119,6 +142,7 @@ sao_status sao_token_logprobs_bwd(const void *H, const void *W, sao_dtype dt, co
                                   const float *lse, const float *grad_logp, int64_t N, int32_t h, int32_t V,
                                   void *dH, float *dW, int accumulate_dW, void *ws, size_t ws_bytes,
                                   sao_stream_t stream) {
+  SAO_RANGE();
   SAO_TRY(check_logprob_shapes(dt, N, h, V));
   if (!W || !dW) return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
@@ -161,6 +185,7 @@ sao_status sao_token_logprobs_fwd_cached(const void *H, const void *W, sao_dtype
                                          const uint8_t *row_mask, int64_t N, int32_t h, int32_t V, float *logp,
                                          float *lse, void *cache, size_t cache_bytes, void *ws, size_t ws_bytes,
                                          sao_stream_t stream) {
+  SAO_RANGE();
   SAO_TRY(check_logprob_shapes(dt, N, h, V));
   if (dt != SAO_BF16) return fail(SAO_ERR_UNSUPPORTED, "the probability cache is for bf16 only");
   if (N == 0) return SAO_OK;
@@ -180,6 +205,7 @@ sao_status sao_token_logprobs_bwd_cached(const void *H, const void *W, sao_dtype
                                          const float *lse, const float *grad_logp, int64_t N, int32_t h, int32_t V,
                                          void *dH, float *dW, int accumulate_dW, const void *cache,
                                          size_t cache_bytes, void *ws, size_t ws_bytes, sao_stream_t stream) {
+  SAO_RANGE();
   SAO_TRY(check_logprob_shapes(dt, N, h, V));
   if (dt != SAO_BF16) return fail(SAO_ERR_UNSUPPORTED, "the probability cache is for bf16 only");
   if (!W || !dW) return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
@@ -203,6 +229,7 @@ sao_status sao_advantages(const float *values, const float *rewards, const uint8
                           const int32_t *cu_seqlens, int32_t B, int64_t N, float gamma, float lambda_policy,
                           float lambda_critic, float len_adaptive_alpha, float *adv, float *ret, void *ws,
                           size_t ws_bytes, sao_stream_t stream) {
+  SAO_RANGE();
   if (N < 0 || N >= (int64_t(1) << 31)) return fail(SAO_ERR_SHAPE, "N = %lld out of range", (long long)N);
   if (B < 0) return fail(SAO_ERR_SHAPE, "B = %d < 0", B);
   if (N > 0 && B == 0) return fail(SAO_ERR_SHAPE, "N > 0 tokens need at least one trajectory");
@@ -225,6 +252,7 @@ sao_status sao_step_advantages(const float *values, const float *rewards, const 
                                const int32_t *cu_seqlens, int32_t B, int64_t N, float gamma, float lambda_policy,
                                float lambda_critic, float len_adaptive_alpha, int mode, float *adv, float *ret,
                                uint8_t *value_mask, void *ws, size_t ws_bytes, sao_stream_t stream) {
+  SAO_RANGE();
   if (N < 0 || N >= (int64_t(1) << 31)) return fail(SAO_ERR_SHAPE, "N = %lld out of range", (long long)N);
   if (B < 0) return fail(SAO_ERR_SHAPE, "B = %d < 0", B);
   if (N > 0 && B == 0) return fail(SAO_ERR_SHAPE, "N > 0 tokens need at least one trajectory");
@@ -254,6 +282,7 @@ sao_status sao_policy_loss_fwd(const float *logp, const float *old_logp, const f
                                const uint8_t *loss_mask, int64_t N, float eps_low, float eps_high, int64_t n_norm,
                                float *loss, float *coef, uint8_t *flags, int64_t *counts, void *ws,
                                size_t ws_bytes, sao_stream_t stream) {
+  SAO_RANGE();
   if (N < 0) return fail(SAO_ERR_SHAPE, "N < 0");
   SAO_TRY(check_eps(eps_low, eps_high));
   if (!loss || !counts) return fail(SAO_ERR_INVALID_ARG, "NULL loss or counts");
@@ -271,6 +300,7 @@ sao_status sao_policy_loss_bwd(const float *logp, const float *old_logp, const f
                                const uint8_t *loss_mask, int64_t N, float eps_low, float eps_high, int64_t n_norm,
                                const float *grad_loss, float *grad_logp, void *ws, size_t ws_bytes,
                                sao_stream_t stream) {
+  SAO_RANGE();
   if (N < 0) return fail(SAO_ERR_SHAPE, "N < 0");
   SAO_TRY(check_eps(eps_low, eps_high));
   if (N == 0) return SAO_OK;
@@ -297,6 +327,7 @@ sao_status sao_decoupled_loss_fwd(const float *logp, const float *prox_logp, con
                                   float eps_high, float w_low, float w_high, int64_t n_norm, float *loss,
                                   float *coef, uint8_t *flags, int64_t *counts, void *ws, size_t ws_bytes,
                                   sao_stream_t stream) {
+  SAO_RANGE();
   if (N < 0) return fail(SAO_ERR_SHAPE, "N < 0");
   SAO_TRY(check_eps(eps_low, eps_high));
   SAO_TRY(check_band(w_low, w_high));
@@ -316,6 +347,7 @@ sao_status sao_decoupled_loss_bwd(const float *logp, const float *prox_logp, con
                                   const float *adv, const uint8_t *loss_mask, int64_t N, float eps_low,
                                   float eps_high, float w_low, float w_high, int64_t n_norm, const float *grad_loss,
                                   float *grad_logp, void *ws, size_t ws_bytes, sao_stream_t stream) {
+  SAO_RANGE();
   if (N < 0) return fail(SAO_ERR_SHAPE, "N < 0");
   SAO_TRY(check_eps(eps_low, eps_high));
   SAO_TRY(check_band(w_low, w_high));
@@ -333,6 +365,7 @@ sao_status sao_decoupled_loss_bwd(const float *logp, const float *prox_logp, con
 
 sao_status sao_value_loss(const float *values, const float *ret, const uint8_t *loss_mask, int64_t N, float *loss,
                           float *grad_values, double *ev_sums, void *ws, size_t ws_bytes, sao_stream_t stream) {
+  SAO_RANGE();
   if (N < 0) return fail(SAO_ERR_SHAPE, "N < 0");
   if (!loss) return fail(SAO_ERR_INVALID_ARG, "NULL loss");
   if (N > 0 && (!values || !ret || !loss_mask || !grad_values)) return fail(SAO_ERR_INVALID_ARG, "NULL array argument");
@@ -355,6 +388,7 @@ sao_status sao_clip_loss_fwd(const float *logp, const float *old_logp, const flo
                              const int32_t *cu_seqlens, int32_t B, int64_t N, float eps_low, float eps_high, int norm,
                              float *loss, float *coef, uint8_t *flags, int64_t *counts, void *ws, size_t ws_bytes,
                              sao_stream_t stream) {
+  SAO_RANGE();
   SAO_TRY(check_traj(B, N, cu_seqlens));
   SAO_TRY(check_eps(eps_low, eps_high));
   if (norm != SAO_NORM_TOKEN && norm != SAO_NORM_SEQUENCE) return fail(SAO_ERR_INVALID_ARG, "unknown norm %d", norm);
@@ -373,6 +407,7 @@ sao_status sao_clip_loss_bwd(const float *logp, const float *old_logp, const flo
                              const int32_t *cu_seqlens, int32_t B, int64_t N, float eps_low, float eps_high, int norm,
                              const float *grad_loss, float *grad_logp, void *ws, size_t ws_bytes,
                              sao_stream_t stream) {
+  SAO_RANGE();
   SAO_TRY(check_traj(B, N, cu_seqlens));
   SAO_TRY(check_eps(eps_low, eps_high));
   if (norm != SAO_NORM_TOKEN && norm != SAO_NORM_SEQUENCE) return fail(SAO_ERR_INVALID_ARG, "unknown norm %d", norm);
@@ -391,6 +426,7 @@ sao_status sao_clip_loss_bwd(const float *logp, const float *old_logp, const flo
 sao_status sao_group_advantages(const float *rewards, const int32_t *group_ids, int32_t B, const uint8_t *loss_mask,
                                 const int32_t *cu_seqlens, int64_t N, float eps_stab, float *adv, void *ws,
                                 size_t ws_bytes, sao_stream_t stream) {
+  SAO_RANGE();
   SAO_TRY(check_traj(B, N, cu_seqlens));
   if (!(eps_stab >= 0.f) || !isfinite(eps_stab)) return fail(SAO_ERR_INVALID_ARG, "eps_stab must be >= 0");
   if (N == 0) return SAO_OK;
@@ -407,6 +443,7 @@ sao_status sao_running_mean_advantages(const float *rewards, const int32_t *prom
                                        int32_t num_prompts, float *history, int64_t *seen, int32_t window,
                                        const uint8_t *loss_mask, const int32_t *cu_seqlens, int64_t N, float *adv,
                                        void *ws, size_t ws_bytes, sao_stream_t stream) {
+  SAO_RANGE();
   SAO_TRY(check_traj(B, N, cu_seqlens));
   if (window < 1 || num_prompts < 1) return fail(SAO_ERR_INVALID_ARG, "window and num_prompts must be >= 1");
   if (B > 0 && (!rewards || !prompt_ids || !history || !seen)) return fail(SAO_ERR_INVALID_ARG, "NULL array argument");

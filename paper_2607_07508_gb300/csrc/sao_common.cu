@@ -165,6 +165,7 @@ sao_status finish_call(void *ws, cudaStream_t s) {
     if (word & SAO_DEVERR_CU_SEQLENS) what += " bad-cu_seqlens";
     if (word & SAO_DEVERR_SCAN_TIMEOUT) what += " scan-carry-timeout";
     if (word & SAO_DEVERR_PIPE_TIMEOUT) what += " pipeline-wait-timeout";
+    if (word & SAO_DEVERR_CACHE_ROW) what += " cached-row-not-computed";
     return fail(SAO_ERR_DEVICE_CHECK, "device check failed (0x%x):%s", word, what.c_str());
   }
   return SAO_OK;

@@ -64,4 +64,8 @@ sao_status logprobs_bwd_launch(const void *H, const void *W, sao_dtype dt, const
 void set_dz_budget(size_t bytes);
 size_t dz_budget();
 
+// Test hooks of the advantage scan (see sao_debug_set_scan_hooks in sao.h).
+uint64_t scan_wait_ns();
+int scan_skip();
+
 }  // namespace sao
