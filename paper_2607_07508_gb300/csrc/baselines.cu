@@ -288,23 +288,40 @@ __global__ void __launch_bounds__(256) clip_finalize_kernel(const float2 *part_l
   }
 }
 
-// GRPO: per-trajectory standardised reward within its group. Every thread
-// scans all trajectories for its group's members, through shared-memory tiles
-// of the group ids and rewards (members summed in batch order, compensated
-// fp32; the final moments in fp64).
+// GRPO: per-trajectory standardised reward within its group. One warp per
+// trajectory, 8 per CTA sharing shared-memory tiles of the group ids and
+// rewards; lane l takes entries l, l + 32, ... of each tile in batch order
+// (compensated fp32), the lanes' partial sums are combined down to lane 0 in
+// a fixed order, and the final moments are taken in fp64. Two passes: the
+// mean, then the centred second moment.
 constexpr int kTile = 2048;
+
+// Lane 0's total of the 32 lanes' compensated partials (fixed tree order).
+__device__ __forceinline__ Sum2 warp_total(Sum2 s) {
+#pragma unroll
+  for (int d = 16; d >= 1; d >>= 1) {
+    const float ohi = __shfl_down_sync(0xffffffffu, s.hi, d), olo = __shfl_down_sync(0xffffffffu, s.lo, d);
+    s.merge(ohi, olo);
+  }
+  return s;
+}
 
 __global__ void __launch_bounds__(256) group_norm_kernel(const float *R, const int32_t *gid, int B, float eps,
                                                          float *a_traj) {
   __shared__ int32_t sg[kTile];
   __shared__ float sr[kTile];
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  const int lane = threadIdx.x & 31;
+  const int b = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int g = b < B ? gid[b] : 0;
   Sum2 s, s2;
   int n = 0;
   float mu = 0.f;
   for (int pass = 0; pass < 2; ++pass) {
-    if (pass) mu = float(s.value() / double(n > 0 ? n : 1));
+    if (pass) {  // the group's mean, from lane 0 to every lane
+      const Sum2 t = warp_total(s);
+      const int nt = __reduce_add_sync(0xffffffffu, n);
+      mu = __shfl_sync(0xffffffffu, float(t.value() / double(nt > 0 ? nt : 1)), 0);
+    }
     for (int t0 = 0; t0 < B; t0 += kTile) {
       const int len = min(kTile, B - t0);
       __syncthreads();
@@ -314,8 +331,7 @@ __global__ void __launch_bounds__(256) group_norm_kernel(const float *R, const i
       }
       __syncthreads();
       if (b >= B) continue;
-#pragma unroll 8
-      for (int k = 0; k < len; ++k) {
+      for (int k = lane; k < len; k += 32) {
         if (sg[k] != g) continue;
         if (pass == 0) {
           s.add(sr[k]);
@@ -327,23 +343,15 @@ __global__ void __launch_bounds__(256) group_norm_kernel(const float *R, const i
       }
     }
   }
-  if (b < B) {
+  if (b >= B) return;
+  const Sum2 t = warp_total(s), t2 = warp_total(s2);
+  const int nt = __reduce_add_sync(0xffffffffu, n);
+  if (lane == 0) {
     // exact mean correction for the rounded mu: var = E[(r - mu)^2] - (mean - mu)^2
-    const double mean = s.value() / double(n);
+    const double mean = t.value() / double(nt);
     const double dm = mean - double(mu);
-    const double var = s2.value() / double(n) - dm * dm;
+    const double var = t2.value() / double(nt) - dm * dm;
     a_traj[b] = float((double(R[b]) - mean) / sqrt((var > 0.0 ? var : 0.0) + double(eps)));
-  }
-}
-
-// One warp per trajectory: broadcast to its action tokens.
-__global__ void __launch_bounds__(256) group_broadcast_kernel(const float *a_traj, const uint8_t *m,
-                                                              const int32_t *cu, int B, int64_t N, float *adv) {
-  const int lane = threadIdx.x & 31;
-  for (int b = (blockIdx.x * 256 + threadIdx.x) >> 5; b < B; b += (gridDim.x * 256) >> 5) {
-    const int64_t lo = cu[b], hi = cu[b + 1] < N ? cu[b + 1] : N;
-    const float v = a_traj[b];
-    for (int64_t t = lo + lane; t < hi; t += 32) adv[t] = m[t] ? v : 0.f;
   }
 }
 
@@ -351,19 +359,28 @@ __global__ void __launch_bounds__(256) group_broadcast_kernel(const float *a_tra
 // after the k in-batch trajectories of p before it have been recorded: their
 // last min(k, window) rewards, plus the slots of the caller's ring buffer that
 // those k writes have not overwritten. So every trajectory is independent:
-// one thread walks the batch backwards from b (most recent first), then the
-// ring buffers are updated in a second pass.
+// one warp per trajectory walks the batch backwards from b (most recent
+// first, 32 entries per step: a ballot ranks the matches), then the ring
+// buffers are updated in a second pass. Sums are fp64, combined in a fixed
+// order.
+__device__ __forceinline__ double warp_total_f64(double x) {
+#pragma unroll
+  for (int d = 16; d >= 1; d >>= 1) x += __shfl_down_sync(0xffffffffu, x, d);
+  return x;  // lane 0
+}
+
 __global__ void __launch_bounds__(256) running_mean_kernel(const float *R, const int32_t *pid, int B,
                                                            const float *history, const long long *seen, int window,
                                                            float *a_traj, long long *rec) {
   __shared__ int32_t sp[kTile];
   __shared__ float sR[kTile];
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  const int lane = threadIdx.x & 31;
+  const int b = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int p = b < B ? pid[b] : -1;
-  double sum = 0.0;
-  int k = 0;  // in-batch trajectories of p before b
+  double sum = 0.0;  // this lane's share
+  int k = 0;         // in-batch trajectories of p before b (warp-uniform)
   // tiles of the batch, newest first, down from the block's last trajectory
-  const int bend = min(B, int(blockIdx.x + 1) * int(blockDim.x));
+  const int bend = min(B, int(blockIdx.x + 1) * 8);
   for (int t1 = bend; t1 > 0; t1 -= kTile) {
     const int t0 = max(0, t1 - kTile), len = t1 - t0;
     __syncthreads();
@@ -373,11 +390,14 @@ __global__ void __launch_bounds__(256) running_mean_kernel(const float *R, const
     }
     __syncthreads();
     if (b >= B) continue;
-    for (int i = min(len, b - t0) - 1; i >= 0; --i)
-      if (sp[i] == p) {
-        if (k < window) sum += double(sR[i]);
-        ++k;
-      }
+    // entries i = top - lane for top = min(len, b - t0) - 1, top - 32, ...
+    for (int top = min(len, b - t0) - 1; top >= 0; top -= 32) {
+      const int i = top - lane;
+      const bool hit = i >= 0 && sp[i] == p;
+      const unsigned mask = __ballot_sync(0xffffffffu, hit);
+      if (hit && k + __popc(mask & ((1u << lane) - 1u)) < window) sum += double(sR[i]);
+      k += __popc(mask);
+    }
   }
   if (b >= B) return;
   const long long c = seen[p];
@@ -386,35 +406,42 @@ __global__ void __launch_bounds__(256) running_mean_kernel(const float *R, const
   const int valid_old = int(c < window ? c : window);
   if (k < window) {
     const float *h = history + int64_t(p) * window;
-    for (int q = 0; q < valid_old; ++q) {
+    for (int q = lane; q < valid_old; q += 32) {
       const int since = int(((long long)q - c % window + window) % window);  // write order of slot q after c
       if (since >= k) sum += double(h[q]);
     }
   }
-  const long long n = (c + k) < window ? (c + k) : window;
-  a_traj[b] = float(double(R[b]) - (n > 0 ? sum / double(n) : 0.0));
-  rec[b] = c + k;  // b's position in its prompt's reward sequence
+  sum = warp_total_f64(sum);
+  if (lane == 0) {
+    const long long n = (c + k) < window ? (c + k) : window;
+    a_traj[b] = float(double(R[b]) - (n > 0 ? sum / double(n) : 0.0));
+    rec[b] = c + k;  // b's position in its prompt's reward sequence
+  }
 }
 
 // Records the batch: the last `window` rewards of each prompt go to their ring
 // slots (distinct slots), and the prompt's last trajectory advances its count.
-// Positions come from the first pass, so this pass never reads `seen`.
+// Positions come from the first pass, so this pass never reads `seen`. One
+// warp per trajectory counts the later trajectories of its prompt, stopping
+// once there are `window` of them.
 __global__ void __launch_bounds__(256) running_mean_record_kernel(const float *R, const int32_t *pid, int B,
                                                                   const long long *rec, float *history,
                                                                   long long *seen, int window) {
   __shared__ int32_t sp[kTile];
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  const int lane = threadIdx.x & 31;
+  const int b = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int p = b < B ? pid[b] : -1;
   int after = 0;
-  for (int t0 = int(blockIdx.x) * int(blockDim.x) + 1; t0 < B; t0 += kTile) {
+  for (int t0 = int(blockIdx.x) * 8 + 1; t0 < B; t0 += kTile) {
     const int len = min(kTile, B - t0);
     __syncthreads();
     for (int i = threadIdx.x; i < len; i += blockDim.x) sp[i] = pid[t0 + i];
     __syncthreads();
-    if (b >= B) continue;
-    for (int i = max(0, b + 1 - t0); i < len; ++i) after += (sp[i] == p);
+    if (b >= B || after >= window) continue;
+    for (int i = max(0, b + 1 - t0) + lane; i - lane < len && after < window; i += 32)
+      after += __popc(__ballot_sync(0xffffffffu, i < len && sp[i] == p));
   }
-  if (b >= B) return;
+  if (b >= B || lane != 0) return;
   if (after < window) history[int64_t(p) * window + int(rec[b] % window)] = R[b];
   if (after == 0) seen[p] = rec[b] + 1;
 }
@@ -449,7 +476,8 @@ sao_status clip_loss_launch(const float *logp, const float *old, const float *ad
   const unsigned grid = unsigned((nchunks + kWarps - 1) / kWarps);
   int slot = launch_begin("clip_loss_counts", s);
   seg::chunk_first_kernel<<<unsigned((nchunks + 255) / 256), 256, 0, s>>>(cu, B, N, int(nchunks), chunk_first);
-  seg::action_count_kernel<<<grid, kThreads, 0, s>>>(m, cu, B, N, int(nchunks), chunk_first, nact);
+  seg::action_count_kernel<<<seg::action_count_grid(int(nchunks)), 256, 0, s>>>(m, cu, B, N, int(nchunks),
+                                                                                chunk_first, nact);
   norms_kernel<<<1, 256, 0, s>>>(nact, B, norms);
   SAO_TRY(launch_end(slot, s));
   ClipArgs a;
@@ -485,19 +513,32 @@ sao_status clip_loss_launch(const float *logp, const float *old, const float *ad
   return launch_end(slot, s);
 }
 
+// adv[t] = a_traj[trajectory of t] on action tokens, 0 elsewhere, all N tokens.
+static sao_status broadcast_launch(const float *a_traj, const uint8_t *m, const int32_t *cu, int32_t B, int64_t N,
+                                   int *chunk_first, float *adv, cudaStream_t s) {
+  if (N == 0) return SAO_OK;
+  const int64_t nchunks = (N + kSegChunk - 1) / kSegChunk;
+  int slot = launch_begin("adv_broadcast", s);
+  seg::chunk_first_kernel<<<unsigned((nchunks + 255) / 256), 256, 0, s>>>(cu, B, N, int(nchunks), chunk_first);
+  seg::traj_broadcast_kernel<<<seg::action_count_grid(int(nchunks)), 256, 0, s>>>(a_traj, m, cu, B, N,
+                                                                                  int(nchunks), chunk_first, adv);
+  return launch_end(slot, s);
+}
+
 sao_status group_adv_launch(const float *rewards, const int32_t *gid, int32_t B, const uint8_t *m, const int32_t *cu,
                             int64_t N, float eps, float *adv, void *ws_body, size_t body_bytes, cudaStream_t s) {
   Carver c(ws_body, body_bytes);
   float *a_traj = c.take<float>(size_t(B) + 1);
+  int *chunk_first = c.take<int>(size_t((N + kSegChunk - 1) / kSegChunk) + 1);
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the group advantages");
-  SAO_CUDA_TRY(cudaMemsetAsync(adv, 0, sizeof(float) * size_t(N), s));
-  if (B == 0) return SAO_OK;
-  DeviceInfo di;
-  SAO_TRY(device_info(&di));
+  if (B == 0) {
+    if (N > 0) SAO_CUDA_TRY(cudaMemsetAsync(adv, 0, sizeof(float) * size_t(N), s));
+    return SAO_OK;
+  }
   int slot = launch_begin("group_advantages", s);
-  group_norm_kernel<<<unsigned((B + 255) / 256), 256, 0, s>>>(rewards, gid, B, eps, a_traj);
-  group_broadcast_kernel<<<unsigned(di.sm_count * 4), 256, 0, s>>>(a_traj, m, cu, B, N, adv);
-  return launch_end(slot, s);
+  group_norm_kernel<<<unsigned((B + 7) / 8), 256, 0, s>>>(rewards, gid, B, eps, a_traj);
+  SAO_TRY(launch_end(slot, s));
+  return broadcast_launch(a_traj, m, cu, B, N, chunk_first, adv, s);
 }
 
 sao_status running_mean_launch(const float *rewards, const int32_t *pid, int32_t B, float *history, int64_t *seen,
@@ -506,19 +547,20 @@ sao_status running_mean_launch(const float *rewards, const int32_t *pid, int32_t
   Carver c(ws_body, body_bytes);
   float *a_traj = c.take<float>(size_t(B) + 1);
   long long *rec = c.take<long long>(size_t(B) + 1);
+  int *chunk_first = c.take<int>(size_t((N + kSegChunk - 1) / kSegChunk) + 1);
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the running-mean baseline");
-  if (N > 0) SAO_CUDA_TRY(cudaMemsetAsync(adv, 0, sizeof(float) * size_t(N), s));
-  if (B == 0) return SAO_OK;
-  DeviceInfo di;
-  SAO_TRY(device_info(&di));
+  if (B == 0) {
+    if (N > 0) SAO_CUDA_TRY(cudaMemsetAsync(adv, 0, sizeof(float) * size_t(N), s));
+    return SAO_OK;
+  }
   int slot = launch_begin("running_mean_advantages", s);
-  const unsigned g = unsigned((B + 255) / 256);
+  const unsigned g = unsigned((B + 7) / 8);  // a warp per trajectory
   running_mean_kernel<<<g, 256, 0, s>>>(rewards, pid, B, history, reinterpret_cast<const long long *>(seen), window,
                                         a_traj, rec);
   running_mean_record_kernel<<<g, 256, 0, s>>>(rewards, pid, B, rec, history, reinterpret_cast<long long *>(seen),
                                                window);
-  if (N > 0) group_broadcast_kernel<<<unsigned(di.sm_count * 4), 256, 0, s>>>(a_traj, m, cu, B, N, adv);
-  return launch_end(slot, s);
+  SAO_TRY(launch_end(slot, s));
+  return broadcast_launch(a_traj, m, cu, B, N, chunk_first, adv, s);
 }
 
 }  // namespace sao

@@ -857,7 +857,7 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   }
   if (alpha > 0.f) {
     int slot = launch_begin("gae_count", s);
-    seg::action_count_kernel<<<unsigned((nchunks + 7) / 8), 256, 0, s>>>(m, cu, B, N, int(nchunks),
+    seg::action_count_kernel<<<seg::action_count_grid(int(nchunks)), 256, 0, s>>>(m, cu, B, N, int(nchunks),
                                                                                     chunk_first, nact);
     SAO_TRY(launch_end(slot, s));
   }

@@ -12,6 +12,12 @@ namespace seg {
 constexpr int kItems = 32;               // tokens per lane (one bit each in a uint32)
 constexpr int kSegChunk = 32 * kItems;   // tokens per warp chunk
 constexpr int kCuCap = 128;              // cu_seqlens entries staged per warp
+constexpr int kCountChunks = 8;          // chunks per warp in action_count_kernel
+
+// CTAs (of 8 warps) of action_count_kernel for nchunks chunks.
+__host__ __device__ constexpr unsigned action_count_grid(int nchunks) {
+  return unsigned((nchunks + 8 * kCountChunks - 1) / (8 * kCountChunks));
+}
 
 // cu_seqlens entries [blo, blo + n) of one chunk, read from shared memory
 // when the slice fits there, else from global memory.
@@ -70,25 +76,35 @@ __global__ void chunk_first_kernel(const int32_t *cu, int B, int64_t N, int nchu
 }
 
 // Number of action tokens per trajectory; nact must start at zero. One warp
-// per chunk, 8 warps per CTA; in each 512-token window of the chunk lane l
-// reads tokens 16l .. 16l+15 (one contiguous 512-byte warp load), and each
-// lane's trajectory walk only moves forward.
+// per kCountChunks consecutive chunks, 8 warps per CTA (grid:
+// action_count_grid); in each 512-token window lane l reads tokens
+// 16l .. 16l+15 (one contiguous 512-byte warp load). A 16-token vector inside
+// the lane's current trajectory is counted with 4 byte-wise popcounts; only
+// vectors that cross a trajectory end take the per-token walk, which only
+// moves forward.
 __global__ void __launch_bounds__(256) action_count_kernel(const uint8_t *m, const int32_t *cu_g, int B, int64_t N,
                                                            int nchunks, const int *chunk_first, int *nact) {
   __shared__ int32_t s_cu_all[8][kCuCap];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int q = blockIdx.x * 8 + warp;
-  if (q >= nchunks) return;
-  int blo, bhi;
-  const CuView cu = stage_chunk(cu_g, B, nchunks, chunk_first, q, lane, s_cu_all[warp], blo, bhi);
-  const int64_t c0 = int64_t(q) * kSegChunk;
+  const int q0 = (blockIdx.x * 8 + warp) * kCountChunks;
+  if (q0 >= nchunks) return;
+  const int q1 = q0 + kCountChunks < nchunks ? q0 + kCountChunks : nchunks;
+  const int blo = __ldg(chunk_first + q0);
+  const int bhi = q1 < nchunks ? __ldg(chunk_first + q1) : B - 1;
+  const int ncu = bhi - blo + 2;  // cu[blo .. bhi + 1]
+  const CuView cu{cu_g, s_cu_all[warp], blo, ncu <= kCuCap};
+  if (cu.in_smem)
+    for (int i = lane; i < ncu; i += 32) s_cu_all[warp][i] = __ldg(cu_g + blo + i);
+  __syncwarp();
+  const int64_t c0 = int64_t(q0) * kSegChunk;
+  const int64_t c1 = int64_t(q1) * kSegChunk < N ? int64_t(q1) * kSegChunk : N;
   int b = blo;
   int64_t next_end = cu[b + 1];
   int cnt = 0;
   const bool aligned = (reinterpret_cast<uintptr_t>(m) & 15u) == 0;
 #pragma unroll 1
-  for (int g = 0; g < kSegChunk / 512; ++g) {
-    const int64_t t0 = c0 + int64_t(g) * 512 + int64_t(lane) * 16;
+  for (int64_t w0 = c0; w0 < c1; w0 += 512) {
+    const int64_t t0 = w0 + int64_t(lane) * 16;
     if (t0 >= N) break;
     uint32_t w[4] = {0u, 0u, 0u, 0u};
     if (aligned && t0 + 16 <= N) {
@@ -102,6 +118,11 @@ __global__ void __launch_bounds__(256) action_count_kernel(const uint8_t *m, con
         const int64_t t = t0 + k;
         if (t < N && m[t] != 0) w[k >> 2] |= 1u << (8 * (k & 3));
       }
+    }
+    if (t0 + 16 <= next_end) {  // all 16 tokens in trajectory b (t0 >= cu[b]: the walk is behind)
+#pragma unroll
+      for (int k = 0; k < 4; ++k) cnt += __popc(((w[k] & 0x7f7f7f7fu) + 0x7f7f7f7fu | w[k]) & 0x80808080u);
+      continue;
     }
 #pragma unroll
     for (int k = 0; k < 16; ++k) {
@@ -124,6 +145,57 @@ __global__ void __launch_bounds__(256) action_count_kernel(const uint8_t *m, con
   const unsigned peers = __match_any_sync(0xffffffffu, b);
   const int tot = __reduce_add_sync(peers, cnt);
   if (lane == __ffs(peers) - 1 && tot) atomicAdd(nact + b, tot);
+}
+
+// adv[t] = a_traj[b] on the action tokens of trajectory b, 0 on every other
+// token; every token below N is written (cu_seqlens covers [0, N)). Same
+// grid as action_count_kernel: kCountChunks chunks per warp; in 128-token
+// groups lane l takes 4 tokens (a 4-byte mask load, a float4 store); a group
+// inside the lane's current trajectory takes no per-token work.
+__global__ void __launch_bounds__(256) traj_broadcast_kernel(const float *a_traj, const uint8_t *m,
+                                                             const int32_t *cu_g, int B, int64_t N, int nchunks,
+                                                             const int *chunk_first, float *adv) {
+  __shared__ int32_t s_cu_all[8][kCuCap];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int q0 = (blockIdx.x * 8 + warp) * kCountChunks;
+  if (q0 >= nchunks) return;
+  const int q1 = q0 + kCountChunks < nchunks ? q0 + kCountChunks : nchunks;
+  const int blo = __ldg(chunk_first + q0);
+  const int bhi = q1 < nchunks ? __ldg(chunk_first + q1) : B - 1;
+  const int ncu = bhi - blo + 2;  // cu[blo .. bhi + 1]
+  const CuView cu{cu_g, s_cu_all[warp], blo, ncu <= kCuCap};
+  if (cu.in_smem)
+    for (int i = lane; i < ncu; i += 32) s_cu_all[warp][i] = __ldg(cu_g + blo + i);
+  __syncwarp();
+  const int64_t c0 = int64_t(q0) * kSegChunk;
+  const int64_t c1 = int64_t(q1) * kSegChunk < N ? int64_t(q1) * kSegChunk : N;
+  int b = blo;
+  int64_t next_end = cu[b + 1];
+  float v = __ldg(a_traj + b);
+  const bool aligned = ((reinterpret_cast<uintptr_t>(m) | reinterpret_cast<uintptr_t>(adv)) & 15u) == 0;
+  // 128-token groups: lane l takes tokens 4l .. 4l+3, so each warp load reads
+  // 128 contiguous bytes and each warp store writes 512
+#pragma unroll 1
+  for (int64_t t0 = c0 + int64_t(lane) * 4; t0 < c1; t0 += 128) {
+    if (aligned && t0 + 4 <= N && t0 + 4 <= next_end) {  // all 4 tokens in trajectory b
+      const uint32_t u = __ldg(reinterpret_cast<const uint32_t *>(m + t0));
+      __stcs(reinterpret_cast<float4 *>(adv + t0), make_float4((u & 0xffu) ? v : 0.f, (u & 0xff00u) ? v : 0.f,
+                                                               (u & 0xff0000u) ? v : 0.f, (u & 0xff000000u) ? v : 0.f));
+      continue;
+    }
+    for (int k = 0; k < 4; ++k) {
+      const int64_t t = t0 + k;
+      if (t >= N) break;
+      if (t >= next_end) {
+        while (b < bhi && t >= next_end) {
+          ++b;
+          next_end = cu[b + 1];
+        }
+        v = __ldg(a_traj + b);
+      }
+      adv[t] = m[t] ? v : 0.f;
+    }
+  }
 }
 
 }  // namespace
