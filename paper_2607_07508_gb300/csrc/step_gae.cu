@@ -15,7 +15,8 @@
 //      scan combines the maps, each lane replays its block (double-float; the
 //      length-adaptive lambda is counted in steps);
 //   4. every token reads its step's advantage, value target and value-loss
-//      flag (coalesced, one pass; non-action tokens get zeros).
+//      flag (coalesced, one pass; non-action tokens get zeros), its step
+//      index recounted from the flags, so no per-token index is stored.
 #include <stdint.h>
 
 #include "sao_common.cuh"
@@ -110,11 +111,10 @@ __global__ void __launch_bounds__(1024) step_scan_kernel(int *block_count, int n
   if (threadIdx.x == 1023) *total = sh[1023];
 }
 
-// Ordered step list with each step's first and one-past-last token, and every
-// token's step (-1 for non-action tokens).
+// Ordered step list with each step's first and one-past-last token.
 __global__ void __launch_bounds__(kThreads) step_scatter_kernel(const uint8_t *m, const uint8_t *ts, int64_t N,
                                                                 const int *block_offset, int *step_first,
-                                                                int *step_end, int *step_id) {
+                                                                int *step_end) {
   const int64_t t0 = int64_t(blockIdx.x) * kRowsPerBlock + int64_t(threadIdx.x) * 16;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   uint32_t act = 0, st = 0, tst = 0;
@@ -146,20 +146,10 @@ __global__ void __launch_bounds__(kThreads) step_scatter_kernel(const uint8_t *m
   const int base = block_offset[blockIdx.x] + before + x - c;  // steps opened before token t0
   if (t0 >= N) return;
   int k = base;
-  int ids[16];
 #pragma unroll
   for (int i = 0; i < 16; ++i) {
     if ((st >> i) & 1u) step_first[k++] = int(t0 + i);
-    ids[i] = ((act >> i) & 1u) ? k - 1 : -1;
     if ((last >> i) & 1u) step_end[k - 1] = int(t0 + i + 1);
-  }
-  if (t0 + 16 <= N && (reinterpret_cast<uintptr_t>(step_id) & 15u) == 0) {
-    int4 *d = reinterpret_cast<int4 *>(step_id + t0);
-#pragma unroll
-    for (int q = 0; q < 4; ++q) d[q] = make_int4(ids[4 * q], ids[4 * q + 1], ids[4 * q + 2], ids[4 * q + 3]);
-  } else {
-    for (int i = 0; i < 16; ++i)
-      if (t0 + i < N) step_id[t0 + i] = ids[i];
   }
 }
 
@@ -224,7 +214,9 @@ __device__ __forceinline__ float2 acc_mean(const Acc2 &a, int n) {
 // A warp takes 32 consecutive steps, one per lane: a lane sums its own step
 // when it is short (4 independent loads at a time), the warp sums the long
 // ones together. Step ranges come from the scatter pass, so no load waits on
-// another.
+// another. (Copying the warp's span of values into shared memory first, for
+// contiguous loads, measured 3x slower: the copy exposes a load latency per 32
+// values, while the steps' own loads already fall in a few nearby lines.)
 __global__ void __launch_bounds__(kThreads) step_reduce_kernel(const float *values, const int *step_first,
                                                                const int *step_end, const int *nsteps, int mode,
                                                                float2 *sv) {
@@ -288,6 +280,9 @@ __device__ __forceinline__ dd dd_shfl_down(dd x, int d) {
 // maps for the policy (a = gamma*lambda_b) and the critic (a = gamma*lambda_c),
 // a shuffle scan gives each lane the advantages to the right of its block, and
 // the lane replays its block.
+// kCrit false: gamma = lambda_critic = 1, where the critic's return telescopes
+// to the trajectory's reward R on every step, so only the policy recursion runs.
+template <bool kCrit>
 __global__ void __launch_bounds__(128) step_gae_kernel(const float *rewards, const int32_t *cu, int B,
                                                        const int *step_first, const int *nsteps, const float2 *sv,
                                                        float gamma, float lam, float lam_c, float alpha,
@@ -345,7 +340,7 @@ __global__ void __launch_bounds__(128) step_gae_kernel(const float *rewards, con
       const dd v = value(i);
       const dd d = delta(i, v, v_next);
       mp = {dd_mul(ap, mp.p), dd_add(dd_mul(ap, mp.c), d)};
-      mc = {dd_mul(ac, mc.p), dd_add(dd_mul(ac, mc.c), d)};
+      if constexpr (kCrit) mc = {dd_mul(ac, mc.p), dd_add(dd_mul(ac, mc.c), d)};
       v_next = v;
     }
   }
@@ -354,21 +349,26 @@ __global__ void __launch_bounds__(128) step_gae_kernel(const float *rewards, con
 #pragma unroll
   for (int d = 1; d < 32; d <<= 1) {
     const StepMap op{dd_shfl_down(sp.p, d), dd_shfl_down(sp.c, d)};
-    const StepMap oc{dd_shfl_down(sc.p, d), dd_shfl_down(sc.c, d)};
-    if (lane + d < 32) {
-      sp = compose_steps(sp, op);
-      sc = compose_steps(sc, oc);
+    if (lane + d < 32) sp = compose_steps(sp, op);
+    if constexpr (kCrit) {
+      const StepMap oc{dd_shfl_down(sc.p, d), dd_shfl_down(sc.c, d)};
+      if (lane + d < 32) sc = compose_steps(sc, oc);
     }
   }
-  dd Ap = dd_shfl_down(sp.c, 1), Ac = dd_shfl_down(sc.c, 1);  // advantages of the step right of the block
+  dd Ap = dd_shfl_down(sp.c, 1), Ac = zero;  // advantages of the step right of the block
+  if constexpr (kCrit) Ac = dd_shfl_down(sc.c, 1);
   if (lane == 31) Ap = Ac = zero;
   dd v_next = v_after;
   for (int i = a1 - 1; i >= a0; --i) {
     const dd v = value(i);
     const dd d = delta(i, v, v_next);
     Ap = dd_add(dd_mul(ap, Ap), d);
-    Ac = dd_add(dd_mul(ac, Ac), d);
-    out[i] = make_float2(dd_round(Ap), dd_round(dd_add(Ac, v)));
+    float r = R;
+    if constexpr (kCrit) {
+      Ac = dd_add(dd_mul(ac, Ac), d);
+      r = dd_round(dd_add(Ac, v));
+    }
+    out[i] = make_float2(dd_round(Ap), r);
     v_next = v;
   }
 }
@@ -387,32 +387,91 @@ __device__ __forceinline__ void step_result(int s, int64_t t, const int *step_en
   }
 }
 
-__global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const int *step_id, const int *step_end,
-                                                                  const float2 *out, int64_t N, int mode,
-                                                                  float *adv, float *ret, uint8_t *vmask) {
-  const int64_t stride = int64_t(gridDim.x) * kThreads * 4;
-  const bool vec = ((reinterpret_cast<uintptr_t>(step_id) | reinterpret_cast<uintptr_t>(adv) |
-                     reinterpret_cast<uintptr_t>(ret)) & 15u) == 0 &&
-                   (reinterpret_cast<uintptr_t>(vmask) & 3u) == 0;
-  for (int64_t t = (int64_t(blockIdx.x) * kThreads + threadIdx.x) * 4; t < N; t += stride) {
-    if (vec && t + 4 <= N) {
-      const int4 s4 = *reinterpret_cast<const int4 *>(step_id + t);
-      const int sv[4] = {s4.x, s4.y, s4.z, s4.w};
-      float a[4], r[4];
-      uint8_t k[4];
+// Action flags and trajectory-start flags of the 4 tokens t0 .. t0+3 (bits),
+// zero past N.
+__device__ __forceinline__ void flags4(const uint8_t *m, const uint8_t *ts, int64_t N, int64_t t0, bool vec,
+                                      uint32_t &M, uint32_t &T) {
+  if (vec && t0 + 4 <= N) {
+    M = nz4(__ldg(reinterpret_cast<const uint32_t *>(m + t0)));
+    T = nz4(__ldg(reinterpret_cast<const uint32_t *>(ts + t0)));
+  } else {
+    M = T = 0;
+    for (int i = 0; i < 4; ++i)
+      if (t0 + i < N) {
+        M |= uint32_t(m[t0 + i] != 0) << i;
+        T |= uint32_t(ts[t0 + i] != 0) << i;
+      }
+  }
+}
+
+// Every token gets its step's results (non-action tokens get zeros). A CTA
+// takes a 4096-token block, as the count pass did, and a warp 512 tokens as
+// four 128-token groups with 4 tokens per lane, so every load and store of
+// the warp is contiguous. Step indices are recounted from the step starts:
+// the block's offset from the scan, the warps before this one through shared
+// memory, the lanes before this one by a warp scan.
+__global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const uint8_t *m, const uint8_t *ts, int64_t N,
+                                                                  const int *block_offset, const int *step_end,
+                                                                  const float2 *out, int mode, float *adv, float *ret,
+                                                                  uint8_t *vmask) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t wbase = int64_t(blockIdx.x) * kRowsPerBlock + int64_t(warp) * 512;
+  const bool vin = ((reinterpret_cast<uintptr_t>(m) | reinterpret_cast<uintptr_t>(ts)) & 3u) == 0;
+  const bool vout = ((reinterpret_cast<uintptr_t>(adv) | reinterpret_cast<uintptr_t>(ret)) & 15u) == 0 &&
+                    (reinterpret_cast<uintptr_t>(vmask) & 3u) == 0;
+  uint32_t act[4], st[4];
+  int x[4], tot[4];  // inclusive lane prefix and warp total of each group's step starts
+  // does the token before the warp's first token act?
+  uint32_t carry = (lane == 0 && wbase > 0 && wbase - 1 < N && m[wbase - 1] != 0) ? 1u : 0u;
+  carry = __shfl_sync(0xffffffffu, carry, 0);
+  int wtot = 0;
 #pragma unroll
-      for (int i = 0; i < 4; ++i) step_result(sv[i], t + i, step_end, out, mode, a[i], r[i], k[i]);
-      *reinterpret_cast<float4 *>(adv + t) = make_float4(a[0], a[1], a[2], a[3]);
-      *reinterpret_cast<float4 *>(ret + t) = make_float4(r[0], r[1], r[2], r[3]);
-      if (vmask) *reinterpret_cast<uchar4 *>(vmask + t) = make_uchar4(k[0], k[1], k[2], k[3]);
+  for (int g = 0; g < 4; ++g) {
+    uint32_t M, T;
+    flags4(m, ts, N, wbase + g * 128 + lane * 4, vin, M, T);
+    const uint32_t up = __shfl_up_sync(0xffffffffu, M, 1);
+    const uint32_t prevbit = lane == 0 ? carry : (up >> 3) & 1u;
+    const uint32_t prev = ((M << 1) | prevbit) & 15u;  // bit i: token i-1 acts
+    act[g] = M;
+    st[g] = M & (T | ~prev) & 15u;
+    carry = __shfl_sync(0xffffffffu, M >> 3, 31) & 1u;
+    int v = __popc(st[g]);
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, v, o);
+      if (lane >= o) v += y;
+    }
+    x[g] = v;
+    tot[g] = __shfl_sync(0xffffffffu, v, 31);
+    wtot += tot[g];
+  }
+  __shared__ int sh[kThreads / 32];
+  if (lane == 0) sh[warp] = wtot;
+  __syncthreads();
+  int run = block_offset[blockIdx.x];
+  for (int w = 0; w < warp; ++w) run += sh[w];
+#pragma unroll
+  for (int g = 0; g < 4; ++g) {
+    const int64_t t0 = wbase + g * 128 + lane * 4;
+    const int before = run + x[g] - __popc(st[g]);  // steps opened before token t0
+    run += tot[g];
+    if (t0 >= N) continue;
+    float a[4], r[4];
+    uint8_t k[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int sid = ((act[g] >> i) & 1u) ? before + __popc(st[g] & ((2u << i) - 1u)) - 1 : -1;
+      step_result(sid, t0 + i, step_end, out, mode, a[i], r[i], k[i]);
+    }
+    if (vout && t0 + 4 <= N) {
+      __stcs(reinterpret_cast<float4 *>(adv + t0), make_float4(a[0], a[1], a[2], a[3]));
+      __stcs(reinterpret_cast<float4 *>(ret + t0), make_float4(r[0], r[1], r[2], r[3]));
+      if (vmask) *reinterpret_cast<uchar4 *>(vmask + t0) = make_uchar4(k[0], k[1], k[2], k[3]);
     } else {
-      for (int64_t u = t; u < t + 4 && u < N; ++u) {
-        float a, r;
-        uint8_t k;
-        step_result(step_id[u], u, step_end, out, mode, a, r, k);
-        adv[u] = a;
-        ret[u] = r;
-        if (vmask) vmask[u] = k;
+      for (int i = 0; i < 4 && t0 + i < N; ++i) {
+        adv[t0 + i] = a[i];
+        ret[t0 + i] = r[i];
+        if (vmask) vmask[t0 + i] = k[i];
       }
     }
   }
@@ -424,7 +483,7 @@ size_t step_gae_ws_bytes(int64_t N, int64_t B) {
   (void)B;
   const int64_t nblocks = (N + kRowsPerBlock - 1) / kRowsPerBlock;
   return round256(size_t(N)) + round256(sizeof(int) * (nblocks + 1)) + round256(sizeof(int) * 4) +
-         round256(sizeof(int) * N) + round256(sizeof(int) * N) + round256(sizeof(int) * N) + round256(sizeof(float2) * N) +
+         round256(sizeof(int) * N) + round256(sizeof(int) * N) + round256(sizeof(float2) * N) +
          round256(sizeof(float2) * N);
 }
 
@@ -438,7 +497,6 @@ sao_status step_gae_launch(const float *values, const float *rewards, const uint
   int *block = c.take<int>(size_t(nblocks) + 1);
   int *nsteps = c.take<int>(4);
   int *step_first = c.take<int>(size_t(N));
-  int *step_id = c.take<int>(size_t(N));
   int *step_end = c.take<int>(size_t(N));
   float2 *sv = c.take<float2>(size_t(N));
   float2 *out = c.take<float2>(size_t(N));
@@ -450,18 +508,20 @@ sao_status step_gae_launch(const float *values, const float *rewards, const uint
   mark_traj_starts<<<unsigned((B + 255) / 256), 256, 0, s>>>(cu, B, N, ts);
   step_count_kernel<<<unsigned(nblocks), kThreads, 0, s>>>(m, ts, N, block);
   step_scan_kernel<<<1, 1024, 0, s>>>(block, int(nblocks), nsteps);
-  step_scatter_kernel<<<unsigned(nblocks), kThreads, 0, s>>>(m, ts, N, block, step_first, step_end, step_id);
+  step_scatter_kernel<<<unsigned(nblocks), kThreads, 0, s>>>(m, ts, N, block, step_first, step_end);
   SAO_TRY(launch_end(slot, s));
   const unsigned warps_grid = unsigned(di.sm_count * 8);
   slot = launch_begin("step_gae_reduce", s);
   step_reduce_kernel<<<warps_grid, kThreads, 0, s>>>(values, step_first, step_end, nsteps, mode, sv);
   SAO_TRY(launch_end(slot, s));
   slot = launch_begin("step_gae_scan", s);
-  step_gae_kernel<<<unsigned((int64_t(B) * 32 + 127) / 128), 128, 0, s>>>(rewards, cu, B, step_first, nsteps, sv,
-                                                                          gamma, lam, lam_c, alpha, out);
+  auto scan = (gamma == 1.f && lam_c == 1.f) ? step_gae_kernel<false> : step_gae_kernel<true>;
+  scan<<<unsigned((int64_t(B) * 32 + 127) / 128), 128, 0, s>>>(rewards, cu, B, step_first, nsteps, sv, gamma, lam,
+                                                               lam_c, alpha, out);
   SAO_TRY(launch_end(slot, s));
   slot = launch_begin("step_gae_broadcast", s);
-  step_broadcast_kernel<<<warps_grid, kThreads, 0, s>>>(step_id, step_end, out, N, mode, adv, ret, vmask);
+  step_broadcast_kernel<<<unsigned(nblocks), kThreads, 0, s>>>(m, ts, N, block, step_end, out, mode, adv, ret,
+                                                                vmask);
   return launch_end(slot, s);
 }
 
