@@ -243,25 +243,52 @@ __global__ void __launch_bounds__(kThreads) clip_loss_kernel(ClipArgs a) {
   }
 }
 
-__global__ void __launch_bounds__(256) clip_finalize_kernel(const float2 *part_loss, const int *part_cnt, int n,
-                                                            const Norms *norms, float *loss, int64_t *counts) {
+// One CTA of 1024 threads sums the per-CTA partials in a fixed order: thread i
+// takes partials i, i + 1024, ... (eight loads in flight), then the warps and
+// the CTA combine theirs in lane and warp order.
+constexpr int kFinThreads = 1024;
+
+__global__ void __launch_bounds__(kFinThreads) clip_finalize_kernel(const float2 *part_loss, const int *part_cnt,
+                                                                    int n, const Norms *norms, float *loss,
+                                                                    int64_t *counts) {
   Sum2 acc;
   long long l = 0, h = 0, f = 0;
-  for (int i = threadIdx.x; i < n; i += 256) {
+  constexpr int kU = 8;
+  int i = threadIdx.x;
+  for (; i + (kU - 1) * kFinThreads < n; i += kU * kFinThreads) {
+    float2 p[kU];
+    int c0[kU], c1[kU], c2[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int j = i + u * kFinThreads;
+      p[u] = part_loss[j];
+      c0[u] = part_cnt[j];
+      c1[u] = part_cnt[n + j];
+      c2[u] = part_cnt[2 * n + j];
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      acc.merge(p[u].x, p[u].y);
+      l += c0[u];
+      h += c1[u];
+      f += c2[u];
+    }
+  }
+  for (; i < n; i += kFinThreads) {
     acc.merge(part_loss[i].x, part_loss[i].y);
     l += part_cnt[i];
     h += part_cnt[n + i];
     f += part_cnt[2 * n + i];
   }
-  __shared__ float2 sd[8];
-  __shared__ long long sl[3][8];
+  __shared__ float2 sd[kFinThreads / 32];
+  __shared__ long long sl[3][kFinThreads / 32];
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    const float ohi = __shfl_xor_sync(0xffffffffu, acc.hi, o), olo = __shfl_xor_sync(0xffffffffu, acc.lo, o);
+    const float ohi = __shfl_down_sync(0xffffffffu, acc.hi, o), olo = __shfl_down_sync(0xffffffffu, acc.lo, o);
     acc.merge(ohi, olo);
-    l += __shfl_xor_sync(0xffffffffu, l, o);
-    h += __shfl_xor_sync(0xffffffffu, h, o);
-    f += __shfl_xor_sync(0xffffffffu, f, o);
+    l += __shfl_down_sync(0xffffffffu, l, o);
+    h += __shfl_down_sync(0xffffffffu, h, o);
+    f += __shfl_down_sync(0xffffffffu, f, o);
   }
   const int w = threadIdx.x >> 5;
   if ((threadIdx.x & 31) == 0) {
@@ -274,7 +301,7 @@ __global__ void __launch_bounds__(256) clip_finalize_kernel(const float2 *part_l
   if (threadIdx.x == 0) {
     Sum2 T;
     long long L = 0, Hh = 0, F = 0;
-    for (int k = 0; k < 8; ++k) {
+    for (int k = 0; k < kFinThreads / 32; ++k) {
       T.merge(sd[k].x, sd[k].y);
       L += sl[0][k];
       Hh += sl[1][k];
@@ -509,7 +536,7 @@ sao_status clip_loss_launch(const float *logp, const float *old, const float *ad
   clip_loss_kernel<false><<<grid, kThreads, 0, s>>>(a);
   SAO_TRY(launch_end(slot, s));
   slot = launch_begin("clip_loss_finalize", s);
-  clip_finalize_kernel<<<1, 256, 0, s>>>(part_loss, part_cnt, int(grid), norms, loss, counts);
+  clip_finalize_kernel<<<1, kFinThreads, 0, s>>>(part_loss, part_cnt, int(grid), norms, loss, counts);
   return launch_end(slot, s);
 }
 
