@@ -54,6 +54,26 @@ def test_step_advantages_edge_layouts(lengths, mode):
     _check_step(wl, 1.0, 0.9, 1.0, 0.0, mode)
 
 
+def test_step_advantages_misaligned_outputs():
+    """Outputs and inputs one element past a 16-byte boundary: the scalar paths
+    of the count, scatter and broadcast passes give the same results."""
+    wl = S.make_custom([3, 0, 4100, 1, 900], 8, 16, "f32", seed=21, dense=False, obs_frac=0.4)
+    N = wl.N
+    mis = lambda t: torch.cat([t[:1], t])[1:]
+    adv = mis(torch.full((N,), float("nan"), device="cuda"))
+    ret = mis(torch.full((N,), float("nan"), device="cuda"))
+    vm = mis(torch.full((N,), 7, dtype=torch.uint8, device="cuda"))
+    for mode in (sao.SAO_STEP_AVERAGE, sao.SAO_STEP_LAST):
+        sao.sao_step_advantages(mis(cuda(wl.values)), cuda(wl.rewards), mis(cuda(wl.loss_mask)), cuda(wl.cu_seqlens),
+                                1.0, f32(0.95), 1.0, 0.0, mode, adv, ret, sao.workspace(N), value_mask=vm)
+        torch.cuda.synchronize()
+        wa, wr, wv = O.step_advantages(wl.values, wl.rewards, wl.loss_mask, wl.cu_seqlens, 1.0, f32(0.95), 1.0, 0.0,
+                                       mode)
+        assert rel_err_floor(adv.cpu().numpy(), wa, 1e-3).max() <= ADV_TOL
+        assert rel_err_floor(ret.cpu().numpy(), wr, 1e-3).max() <= ADV_TOL
+        assert np.array_equal(vm.cpu().numpy(), wv)
+
+
 def test_step_advantages_no_action_tokens():
     wl = S.make_custom([10, 300], 8, 16, "f32", seed=4, dense=False)
     wl.loss_mask[:] = 0
@@ -149,6 +169,48 @@ def test_running_mean_advantages_match_oracle():
             torch.cuda.synchronize()
             want, hist_o, seen_o = O.running_mean_advantages(wl.rewards, pid, wl.loss_mask, wl.cu_seqlens, hist_o,
                                                              seen_o, window)
+            assert rel_err_floor(adv.cpu().numpy(), want, 1e-3).max() <= 1e-5
+            assert np.array_equal(seen_d.cpu().numpy(), seen_o)
+            assert np.allclose(hist_d.cpu().numpy(), hist_o)
+
+
+def _misaligned(t):
+    """The same values one element past a 16-byte boundary (scalar paths)."""
+    pad = torch.empty(t.numel() + 1, dtype=t.dtype, device=t.device)
+    pad[1:] = t
+    return pad[1:]
+
+
+def test_group_and_running_mean_edge_layouts():
+    """5,003 trajectories (several shared-memory tiles, a partly filled last
+    CTA), empty and one-token trajectories, ragged lengths, a misaligned mask
+    and output (the broadcast's scalar path), and for the running mean two
+    batches with per-prompt windows of 8 and one window of 128."""
+    rng = np.random.default_rng(11)
+    lengths = rng.integers(0, 40, size=5003)
+    lengths[:3] = [0, 1, 0]
+    lengths[-2:] = [0, 1]
+    wl = S.make_custom(lengths.tolist(), 8, 16, "f32", seed=12, dense=False, obs_frac=0.3)
+    m_d, cu_d, R_d = _misaligned(cuda(wl.loss_mask)), cuda(wl.cu_seqlens), cuda(wl.rewards)
+    gid = rng.integers(-5, 600, size=wl.B).astype(np.int32)
+    adv = _misaligned(torch.full((wl.N,), float("nan"), device="cuda"))
+    sao.sao_group_advantages(R_d, cuda(gid), m_d, cu_d, 1e-6, adv, sao.workspace(wl.N))
+    torch.cuda.synchronize()
+    want = O.group_advantages(wl.rewards, gid, wl.loss_mask, wl.cu_seqlens, f32(1e-6))
+    assert rel_err_floor(adv.cpu().numpy(), want, 1e-3).max() <= 1e-5
+    for P, window in ((37, 8), (1, 128)):
+        hist_d = torch.zeros(P, window, device="cuda")
+        seen_d = torch.zeros(P, dtype=torch.int64, device="cuda")
+        hist_o, seen_o = np.zeros((P, window)), np.zeros(P, np.int64)
+        for batch in range(2):
+            pid = rng.integers(0, P, size=wl.B).astype(np.int32)
+            R = (wl.rewards + batch).astype(np.float32)
+            adv = _misaligned(torch.full((wl.N,), float("nan"), device="cuda"))
+            sao.sao_running_mean_advantages(cuda(R), cuda(pid), hist_d, seen_d, m_d, cu_d, adv,
+                                            sao.workspace(wl.N))
+            torch.cuda.synchronize()
+            want, hist_o, seen_o = O.running_mean_advantages(R, pid, wl.loss_mask, wl.cu_seqlens, hist_o, seen_o,
+                                                             window)
             assert rel_err_floor(adv.cpu().numpy(), want, 1e-3).max() <= 1e-5
             assert np.array_equal(seen_d.cpu().numpy(), seen_o)
             assert np.allclose(hist_d.cpu().numpy(), hist_o)
