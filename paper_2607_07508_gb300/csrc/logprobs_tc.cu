@@ -101,10 +101,23 @@ __device__ __forceinline__ void tile_coords(int L, const GemmParams &p, int nM, 
   n = within / gm;
 }
 
-template <int kEpi, bool kAMN, bool kBMN>
+// kMT = 2 (the long-K backward products, plain store epilogues): a CTA tile
+// is two 128-row M tiles sharing every B stage, one per TMEM accumulator, so
+// each B tile feeds two MMAs and W (or H) is read once per wave of 2 x 152
+// row tiles instead of 152; the stages (A 32 KB + B 32 KB) shrink to 3. The
+// tile's epilogue then waits for both accumulators, which costs little when
+// K spans thousands of blocks.
+template <int kEpi, bool kAMN, bool kBMN, int kMT = 1>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
                    const __grid_constant__ CUtensorMap map_c, const GemmParams p) {
+  static_assert(kMT == 1 || kMT == 2, "one or two M tiles per CTA tile");
+  static_assert(kMT == 1 || kEpi == kStoreF32 || kEpi == kStoreBF16, "two M tiles: plain store epilogues only");
+  constexpr int kStages = kMT == 2 ? 3 : STAGES;
+  constexpr uint32_t kABytes = A_BYTES * kMT;
+  constexpr uint32_t kStageBytes = kABytes + B_BYTES;
+  constexpr int kTM = BM * kMT;  // rows of a CTA tile
+  static_assert(size_t(kStages) * kStageBytes <= size_t(STAGES) * STAGE_BYTES, "same shared-memory layout");
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -119,7 +132,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   if (p.m_count) {
     const int c = *p.m_count;
     rows = c;
-    nM = (c + BM - 1) / BM;
+    nM = (c + kTM - 1) / kTM;
   }
   if (p.k_count) nK = (*p.k_count + BK - 1) / BK;
   const int num_tiles = nM * p.nN;
@@ -169,16 +182,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const uint32_t fb = smem_u32(&ctl->full[stage]);
           issued |= 1u << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-          mbar_arrive_expect_tx(fb, STAGE_BYTES);
-          const uint32_t sa = base + uint32_t(stage) * STAGE_BYTES;
-          const uint32_t sb = sa + A_BYTES;
+          mbar_arrive_expect_tx(fb, kStageBytes);
+          const uint32_t sa = base + uint32_t(stage) * kStageBytes;
+          const uint32_t sb = sa + kABytes;
           const int k0 = kb * BK;
           if (!kAMN) {
-            tma_load_2d(sa, &map_a, fb, k0, p.a_row_off + m * BM);
+#pragma unroll
+            for (int j = 0; j < kMT; ++j) tma_load_2d(sa + j * A_BYTES, &map_a, fb, k0, p.a_row_off + m * kTM + j * BM);
           } else {
 #pragma unroll
-            for (int j = 0; j < BM / 64; ++j)
-              tma_load_2d(sa + j * MN_ATOM_BYTES, &map_a, fb, p.a_row_off + m * BM + 64 * j, k0);
+            for (int j = 0; j < kTM / 64; ++j)
+              tma_load_2d(sa + j * MN_ATOM_BYTES, &map_a, fb, p.a_row_off + m * kTM + 64 * j, k0);
           }
           if (!kBMN) {
             tma_load_2d(sb, &map_b, fb, k0, p.b_row_off + n * BN);
@@ -187,7 +201,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             for (int j = 0; j < BN / 64; ++j)
               tma_load_2d(sb + j * MN_ATOM_BYTES, &map_b, fb, n * BN + 64 * j, p.b_row_off + k0);
           }
-          if (++stage == STAGES) {
+          if (++stage == kStages) {
             stage = 0;
             phase ^= 1u;
           }
@@ -195,7 +209,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
       if (!ok) {
         // let the copies already in flight land before the CTA can exit
-        for (int s = 0; s < STAGES; ++s) {
+        for (int s = 0; s < kStages; ++s) {
           if (!((issued >> s) & 1u)) continue;
           const uint32_t par = (issued_phase >> s) & 1u;
           const uint64_t t0 = globaltimer_ns();
@@ -213,8 +227,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       int local = 0;
       bool ok = true;
       for (int L = blockIdx.x; L < num_tiles && ok; L += gridDim.x, ++local) {
-        const int acc = local & 1;
-        const uint32_t acc_phase = uint32_t(local >> 1) & 1u;
+        // kMT == 2: both accumulators serve one tile, tracked as accumulator 0
+        const int acc = kMT == 2 ? 0 : (local & 1);
+        const uint32_t acc_phase = kMT == 2 ? (uint32_t(local) & 1u) : (uint32_t(local >> 1) & 1u);
         if (!mbar_wait(smem_u32(&ctl->acc_empty[acc]), acc_phase ^ 1u, abort, p.err)) break;
         fence_after_sync();
         const uint32_t d_tmem = tmem_base + uint32_t(acc) * BN;
@@ -224,18 +239,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             break;
           }
           fence_after_sync();
-          const uint32_t sa = base + uint32_t(stage) * STAGE_BYTES;
-          const uint32_t sb = sa + A_BYTES;
+          const uint32_t sa = base + uint32_t(stage) * kStageBytes;
+          const uint32_t sb = sa + kABytes;
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk) {
-            const uint64_t ad = kAMN ? sdesc_sw128(sa + kk * 2048u, MN_ATOM_BYTES, 1024u)
-                                     : sdesc_sw128(sa + kk * 32u, 16u, 1024u);
             const uint64_t bd = kBMN ? sdesc_sw128(sb + kk * 2048u, MN_ATOM_BYTES, 1024u)
                                      : sdesc_sw128(sb + kk * 32u, 16u, 1024u);
-            mma_bf16(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+#pragma unroll
+            for (int j = 0; j < kMT; ++j) {  // A tile j (rows j*128 ..) into accumulator acc + j
+              const uint32_t aj = sa + uint32_t(j) * A_BYTES;
+              const uint64_t ad = kAMN ? sdesc_sw128(aj + kk * 2048u, MN_ATOM_BYTES, 1024u)
+                                       : sdesc_sw128(aj + kk * 32u, 16u, 1024u);
+              mma_bf16(d_tmem + uint32_t(j) * BN, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+            }
           }
           mma_commit(smem_u32(&ctl->empty[stage]));
-          if (++stage == STAGES) {
+          if (++stage == kStages) {
             stage = 0;
             phase ^= 1u;
           }
@@ -252,8 +271,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     for (int L = blockIdx.x; L < num_tiles; L += gridDim.x, ++local) {
       int m, n;
       tile_coords(L, p, nM, m, n);
-      const int acc = local & 1;
-      const uint32_t acc_phase = uint32_t(local >> 1) & 1u;
+      const int acc = kMT == 2 ? 0 : (local & 1);
+      const uint32_t acc_phase = kMT == 2 ? (uint32_t(local) & 1u) : (uint32_t(local >> 1) & 1u);
       bool ok = mbar_wait(smem_u32(&ctl->acc_full[acc]), acc_phase, abort, p.err);
       // The dlogits epilogue synchronises its 4 warps with named barriers, so
       // they must agree on whether this tile goes ahead.
@@ -261,7 +280,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (!ok) break;
       fence_after_sync();
       const uint32_t taddr = tmem_base + (uint32_t(quad * 32) << 16) + uint32_t(acc) * BN;
-      const int64_t row = int64_t(m) * BM + r;
+      const int64_t row = int64_t(m) * kTM + r;
       const bool row_ok = row < rows;
       const int64_t orig = (row_ok && p.row_idx) ? int64_t(__ldg(p.row_idx + row)) : row;
 
@@ -440,19 +459,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
         }
       } else {
-        // kStoreF32 / kStoreBF16: plain tile store (optionally accumulating)
-        const int64_t orow = p.c_row_off + orig;
+        // kStoreF32 / kStoreBF16: plain tile store (optionally accumulating); with
+        // kMT == 2 the second M tile comes from the second accumulator
+#pragma unroll 1
+        for (int j = 0; j < kMT; ++j) {
+        const int64_t rowj = row + int64_t(j) * BM;
+        const bool okj = rowj < rows;
+        const int64_t origj = j == 0 ? orig : ((okj && p.row_idx) ? int64_t(__ldg(p.row_idx + rowj)) : rowj);
+        const int64_t orow = p.c_row_off + origj;
 #pragma unroll 1
         for (int c = 0; c < BN / 32; ++c) {
           uint32_t u[32];
-          tmem_ld32(taddr + c * 32, u);
+          tmem_ld32(taddr + uint32_t(j) * BN + c * 32, u);
           tmem_wait_ld();
           if (kzero) {
 #pragma unroll
             for (int j = 0; j < 32; ++j) u[j] = 0u;
           }
           const int col = n * BN + c * 32;
-          if (!row_ok || col >= p.cols) continue;
+          if (!okj || col >= p.cols) continue;
           const bool full = col + 32 <= p.cols;
           if constexpr (kEpi == kStoreF32) {
             float *dst = p.cf + orow * p.ldc + col;
@@ -494,6 +519,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 if (col + j < p.cols) dst[j] = __float2bfloat16_rn(__uint_as_float(u[j]));
             }
           }
+        }
         }
         fence_before_sync();
         mbar_arrive(smem_u32(&ctl->acc_empty[acc]));
@@ -638,10 +664,10 @@ sao_status make_map(CUtensorMap *m, const void *ptr, uint64_t inner, uint64_t ou
   return SAO_OK;
 }
 
-template <int kEpi, bool kAMN, bool kBMN>
+template <int kEpi, bool kAMN, bool kBMN, int kMT = 1>
 sao_status launch_gemm(const char *name, const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &mc,
                        const GemmParams &p, cudaStream_t s) {
-  auto kern = tc_gemm_kernel<kEpi, kAMN, kBMN>;
+  auto kern = tc_gemm_kernel<kEpi, kAMN, kBMN, kMT>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [&] {
@@ -797,9 +823,9 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
       p.row_idx = cr.idx;
       SAO_TRY((launch_gemm<kDLogits, false, false>("tc_dlogits", mHc_K, mW_K, mZ_K, p, s)));
     }
-    {  // dH (+)= dZ W[v0:v0+vc]
+    {  // dH (+)= dZ W[v0:v0+vc]: two 128-row tiles per CTA tile share each W stage
       GemmParams p{};
-      p.nM = nMt;
+      p.nM = int((N + 2 * BM - 1) / (2 * BM));
       p.nN = (h + BN - 1) / BN;
       p.nK = (vc + BK - 1) / BK;
       p.group_m = 1;
@@ -812,16 +838,16 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
       if (multi) {
         p.cf = dh_acc;  // compacted rows
         p.accumulate = first ? 0 : 1;
-        SAO_TRY((launch_gemm<kStoreF32, false, true>("tc_dH_gemm", mZ_K, mW_MN, mZ_K, p, s)));
+        SAO_TRY((launch_gemm<kStoreF32, false, true, 2>("tc_dH_gemm", mZ_K, mW_MN, mZ_K, p, s)));
       } else {
         p.cb = static_cast<__nv_bfloat16 *>(dH);
         p.row_idx = cr.idx;  // scatter to the original rows
-        SAO_TRY((launch_gemm<kStoreBF16, false, true>("tc_dH_gemm", mZ_K, mW_MN, mZ_K, p, s)));
+        SAO_TRY((launch_gemm<kStoreBF16, false, true, 2>("tc_dH_gemm", mZ_K, mW_MN, mZ_K, p, s)));
       }
     }
-    {  // dW[v0:v0+vc] (+)= dZ^T H over the compacted tokens
+    {  // dW[v0:v0+vc] (+)= dZ^T H over the compacted tokens: two 128-row vocabulary tiles per CTA tile
       GemmParams p{};
-      p.nM = (vc + BM - 1) / BM;
+      p.nM = (vc + 2 * BM - 1) / (2 * BM);
       p.nN = (h + BN - 1) / BN;
       p.nK = int((N + BK - 1) / BK);
       p.group_m = 1;
@@ -833,7 +859,7 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
       p.accumulate = accumulate;
       p.err = err;
       p.k_count = cr.count;
-      SAO_TRY((launch_gemm<kStoreF32, true, true>("tc_dW_gemm", mZ_MN, mHc_MN, mZ_MN, p, s)));
+      SAO_TRY((launch_gemm<kStoreF32, true, true, 2>("tc_dW_gemm", mZ_MN, mHc_MN, mZ_MN, p, s)));
     }
     if (multi && last)
       SAO_TRY(scatter_rows_to_bf16(dh_acc, h, cr.pos, N, static_cast<__nv_bfloat16 *>(dH), s));
