@@ -3,6 +3,7 @@ per-kernel launch counts, total time and share. Usage:
     python -m paper_2607_07508_gb300.ncu_summary launches.csv [name-filter ...]"""
 import collections
 import csv
+import re
 import io
 import sys
 
@@ -20,12 +21,17 @@ def summarize(path, only=None):
         short = name.split("(")[0].replace("void ", "")
         if "sao::" in short:
             short = short.split("::")[-1]
-        short = short.replace("tc_gemm_kernel<0, 0, 0>", "tc_gemm<softmax> (logits lse fwd)")
-        short = short.replace("tc_gemm_kernel<4, 0, 0>", "tc_gemm<softmax+store> (logits lse fwd, stores bf16 e)")
-        short = short.replace("tc_gemm_kernel<1, 0, 0>", "tc_gemm<dlogits> (bwd recompute + dZ)")
-        short = short.replace("tc_gemm_kernel<3, 0, 1>", "tc_gemm<store bf16> (dH = dZ W)")
-        short = short.replace("tc_gemm_kernel<2, 0, 1>", "tc_gemm<store f32> (dH accumulate)")
-        short = short.replace("tc_gemm_kernel<2, 1, 1>", "tc_gemm<store f32> (dW = dZ^T H)")
+        mt = re.match(r"tc_gemm_kernel<(\d), (\d), (\d)(?:, (\d))?>", short)
+        if mt:
+            label = {("0", "0", "0"): "tc_gemm<softmax> (logits lse fwd)",
+                     ("4", "0", "0"): "tc_gemm<softmax+store> (logits lse fwd, stores bf16 e)",
+                     ("1", "0", "0"): "tc_gemm<dlogits> (bwd recompute + dZ)",
+                     ("3", "0", "1"): "tc_gemm<store bf16> (dH = dZ W)",
+                     ("2", "0", "1"): "tc_gemm<store f32> (dH accumulate)",
+                     ("2", "1", "1"): "tc_gemm<store f32> (dW = dZ^T H)"}.get(mt.groups()[:3], short)
+            if mt.group(4) == "2":
+                label += ", 2 M tiles per CTA tile"
+            short = label
         if only and not any(o in name for o in only):
             continue
         v = float(r["Metric Value"].replace(",", "")) * scale[r["Metric Unit"]]
