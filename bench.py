@@ -574,8 +574,13 @@ def main():
         host["mask"].copy_(step.mask)
         host["cu"].copy_(step.cu)
         out = torch.empty(1 + 1 + 4 * 2, dtype=torch.float32, pin_memory=True)
-        dst = {"H": step.H, "y": step.y, "old": step.old, "values": step.values, "rewards": step.rewards,
-               "mask": step.mask, "cu": step.cu}
+        # Two device input sets: step i+1's inputs are copied on a second
+        # stream into one set while step i runs on the other.
+        names = ("H", "y", "old", "values", "rewards", "mask", "cu")
+        sets = [{k: getattr(step, k) for k in names}, {k: torch.empty_like(getattr(step, k)) for k in names}]
+        copy_stream = torch.cuda.Stream(device=dev)
+        copied = [torch.cuda.Event(), torch.cuda.Event()]  # set j holds the next inputs
+        freed = [torch.cuda.Event(), torch.cuda.Event()]   # the step that read set j is done
         h2d = sum(t.numel() * t.element_size() for t in host.values())
         d2h = out.numel() * out.element_size()
         res = torch.empty(10, dtype=torch.float32, device=dev)
@@ -584,11 +589,25 @@ def main():
         e2 = torch.cuda.Event(enable_timing=True)
         e3 = torch.cuda.Event(enable_timing=True)
         t_wall = time.perf_counter()
+
+        def stage(i):
+            j = i % 2
+            with torch.cuda.stream(copy_stream):
+                copy_stream.wait_event(e2 if i == 0 else freed[j])  # i = 1: freed[1] not yet recorded
+                for k in names:
+                    sets[j][k].copy_(host[k], non_blocking=True)
+                copied[j].record(copy_stream)
+
         e2.record(stream)
-        for _ in range(args.steps):
-            for k, t in host.items():
-                dst[k].copy_(t, non_blocking=True)
+        stage(0)
+        for i in range(args.steps):
+            if i + 1 < args.steps:
+                stage(i + 1)
+            stream.wait_event(copied[i % 2])
+            for k in names:
+                setattr(step, k, sets[i % 2][k])
             step.run()
+            freed[i % 2].record(stream)
             res[0:1].copy_(step.loss)
             res[1:2].copy_(step.vloss)
             res[2:10].copy_(step.counts.view(torch.float32))
@@ -596,6 +615,8 @@ def main():
         e3.record(stream)
         torch.cuda.synchronize()
         barrier()
+        for k in names:
+            setattr(step, k, sets[0][k])
         ms_e2e = e2.elapsed_time(e3) / args.steps
         if world > 1:
             t = torch.tensor([ms_e2e], device=dev)
@@ -604,7 +625,9 @@ def main():
         e2e = {"value": total_tokens / (ms_e2e / 1000.0), "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e,
                "note": "pinned host H, token ids, rollout log-probs, values, rewards, mask and cu_seqlens copied in, "
-                       "loss, value loss and counts copied out, every step; W stays resident (model weight)"}
+                       "loss, value loss and counts copied out, every step; W stays resident (model weight); "
+                       "the inputs of step i+1 are copied on a second stream into a second buffer set while step "
+                       "i runs"}
 
     # ---- CPU baseline (rank 0, single GPU only) ---------------------------------
     cpu = None
