@@ -180,6 +180,57 @@ def test_cached_moe_bench_configuration_sampled_rows():
     assert rel_l2(got_dW, want_dW) <= GRAD_TOL
 
 
+@pytest.mark.parametrize("cached", [True, False])
+def test_two_m_tile_gemms_with_ragged_tiles(cached):
+    """A shape at which both backward GEMMs take two 128-row M tiles per CTA
+    tile (at least four waves of paired tiles on the GPU): 20,100 rows and
+    20,168 vocabulary rows, so the last paired tile of dW has a full first and
+    a 72-row second tile, and dH's last pair a partial first tile only.
+    logp, dH on sampled rows and dW on sampled vocabulary rows (the last 72
+    included) against the oracle."""
+    N, h, V = 20100, 2048, 20168
+    wl = S.make_custom([N], h, V, "bf16", seed=77, device="cuda")
+    H, W, y = wl.H, wl.W, torch.as_tensor(wl.y).cuda()
+    ws = sao.workspace(N, h, V, H.dtype)
+    logp = torch.empty(N, device="cuda")
+    lse = torch.empty(N, device="cuda")
+    rng = np.random.default_rng(78)
+    G = rng.normal(size=N).astype(np.float32)
+    G[rng.random(N) < 0.01] = 0.0
+    Gd = torch.as_tensor(G).cuda()
+    dH = torch.full_like(H, float("nan"))
+    dW = torch.full((V, h), float("nan"), device="cuda")
+    if cached:
+        cache = sao.logprob_cache(N, V)
+        sao.sao_token_logprobs_fwd_cached(H, W, y, logp, lse, cache, ws)
+        sao.sao_token_logprobs_bwd_cached(H, W, y, lse, Gd, dH, dW, cache, ws)
+    else:
+        sao.sao_token_logprobs_fwd(H, W, y, logp, lse, ws)
+        sao.sao_token_logprobs_bwd(H, W, y, lse, Gd, dH, dW, ws)
+    torch.cuda.synchronize()
+    rows = np.sort(np.concatenate([rng.choice(N, size=24, replace=False), [N - 1]]))
+    H_cpu, W_cpu = H[torch.as_tensor(rows).cuda()].cpu(), W.cpu()
+    want_lp, want_lse = O.token_logprobs(H_cpu, W_cpu, wl.y[rows])
+    assert np.abs(logp.cpu().numpy()[rows] - want_lp).max() <= LOGP_TOL
+    want_dH, _ = O.token_logprobs_bwd(H_cpu, W_cpu, wl.y[rows], want_lse, G[rows])
+    assert rel_l2(dH.float().cpu().numpy()[rows], want_dH) <= GRAD_TOL
+    # dW rows: every token contributes; the GPU lse (checked on the sampled rows) stands in for the
+    # full-vocabulary lse of all 20,100 rows
+    vrows = np.unique(np.concatenate([rng.choice(V, size=48, replace=False), np.arange(V - 72, V)]))
+    Hd = O._f64(H.cpu())
+    Z = Hd @ O._f64(W_cpu[torch.as_tensor(vrows)]).T                       # [N, |vrows|]
+    lse_gpu = lse.cpu().numpy().astype(np.float64)                           # the forward's lse (checked above)
+    dZ = -G.astype(np.float64)[:, None] * np.exp(Z - lse_gpu[:, None])
+    pos = {int(v): i for i, v in enumerate(vrows)}
+    for t in range(N):
+        j = pos.get(int(wl.y[t]), -1)
+        if j >= 0:
+            dZ[t, j] += G[t]
+    want_dW = dZ.T @ Hd
+    got_dW = dW[torch.as_tensor(vrows).cuda()].cpu().numpy()
+    assert rel_l2(got_dW, want_dW) <= GRAD_TOL
+
+
 def test_cached_argument_errors():
     wl, H, W, y = _case(64, 64, 300, seed=3)
     logp = torch.empty(64, device="cuda")
