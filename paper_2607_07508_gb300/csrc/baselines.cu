@@ -319,8 +319,8 @@ __global__ void __launch_bounds__(kFinThreads) clip_finalize_kernel(const float2
 // trajectory, 8 per CTA sharing shared-memory tiles of the group ids and
 // rewards; lane l takes entries l, l + 32, ... of each tile in batch order
 // (compensated fp32), the lanes' partial sums are combined down to lane 0 in
-// a fixed order, and the final moments are taken in fp64. Two passes: the
-// mean, then the centred second moment.
+// a fixed order, and the final moments are taken in fp64: the mean, then the
+// centred second moment.
 constexpr int kTile = 2048;
 
 // Lane 0's total of the 32 lanes' compensated partials (fixed tree order).
@@ -343,12 +343,46 @@ __global__ void __launch_bounds__(256) group_norm_kernel(const float *R, const i
   Sum2 s, s2;
   int n = 0;
   float mu = 0.f;
-  for (int pass = 0; pass < 2; ++pass) {
-    if (pass) {  // the group's mean, from lane 0 to every lane
-      const Sum2 t = warp_total(s);
-      const int nt = __reduce_add_sync(0xffffffffu, n);
-      mu = __shfl_sync(0xffffffffu, float(t.value() / double(nt > 0 ? nt : 1)), 0);
+  // A lane meets its members (entries lane, lane + 32, ...) in batch order;
+  // up to 4 of their rewards stay in registers, so when no lane of the CTA has
+  // more (groups of tens of trajectories) the second moment needs no second
+  // sweep, and it adds the same values in the same order.
+  float r0 = 0.f, r1 = 0.f, r2 = 0.f, r3 = 0.f;
+  for (int t0 = 0; t0 < B; t0 += kTile) {
+    const int len = min(kTile, B - t0);
+    __syncthreads();
+    for (int k = threadIdx.x; k < len; k += blockDim.x) {
+      sg[k] = gid[t0 + k];
+      sr[k] = R[t0 + k];
     }
+    __syncthreads();
+    if (b >= B) continue;
+    for (int k = lane; k < len; k += 32) {
+      if (sg[k] != g) continue;
+      const float r = sr[k];
+      s.add(r);
+      r0 = n == 0 ? r : r0;
+      r1 = n == 1 ? r : r1;
+      r2 = n == 2 ? r : r2;
+      r3 = n == 3 ? r : r3;
+      ++n;
+    }
+  }
+  if (b < B) {  // the group's mean, from lane 0 to every lane
+    const Sum2 t = warp_total(s);
+    const int nt = __reduce_add_sync(0xffffffffu, n);
+    mu = __shfl_sync(0xffffffffu, float(t.value() / double(nt > 0 ? nt : 1)), 0);
+  }
+  const bool sweep = __syncthreads_or(b < B && n > 4);
+  if (!sweep) {
+    const float rr[4] = {r0, r1, r2, r3};
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (i < n) {
+        const float d = __fsub_rn(rr[i], mu);
+        s2.add(__fmul_rn(d, d));
+      }
+  } else {
     for (int t0 = 0; t0 < B; t0 += kTile) {
       const int len = min(kTile, B - t0);
       __syncthreads();
@@ -360,13 +394,8 @@ __global__ void __launch_bounds__(256) group_norm_kernel(const float *R, const i
       if (b >= B) continue;
       for (int k = lane; k < len; k += 32) {
         if (sg[k] != g) continue;
-        if (pass == 0) {
-          s.add(sr[k]);
-          ++n;
-        } else {
-          const float d = __fsub_rn(sr[k], mu);
-          s2.add(__fmul_rn(d, d));
-        }
+        const float d = __fsub_rn(sr[k], mu);
+        s2.add(__fmul_rn(d, d));
       }
     }
   }
