@@ -425,37 +425,79 @@ __device__ __forceinline__ double warp_total_f64(double x) {
   return x;  // lane 0
 }
 
-__global__ void __launch_bounds__(256) running_mean_kernel(const float *R, const int32_t *pid, int B,
-                                                           const float *history, const long long *seen, int window,
-                                                           float *a_traj, long long *rec) {
-  __shared__ int32_t sp[kTile];
-  __shared__ float sR[kTile];
+// In-batch ranks for dense prompt ids (P <= kRankMaxPrompts): counts of each
+// prompt per block of kRankBlock trajectories, then their exclusive prefix over
+// the blocks (row nblk: each prompt's total), so the rank of b is
+// table[b / kRankBlock][p] plus the trajectories of p in b's block before b.
+constexpr int kRankBlock = 1024;
+constexpr int kRankMaxPrompts = 4096;
+
+__global__ void __launch_bounds__(256) rank_count_kernel(const int32_t *pid, int B, int P, int *table) {
+  __shared__ int cnt[kRankMaxPrompts];
+  for (int q = threadIdx.x; q < P; q += blockDim.x) cnt[q] = 0;
+  __syncthreads();
+  const int b0 = blockIdx.x * kRankBlock;
+  for (int i = threadIdx.x; i < kRankBlock && b0 + i < B; i += blockDim.x) {
+    const int q = pid[b0 + i];
+    if (q >= 0 && q < P) atomicAdd(&cnt[q], 1);  // ids outside [0, P) are the caller's error: skipped
+  }
+  __syncthreads();
+  for (int q = threadIdx.x; q < P; q += blockDim.x) table[int64_t(blockIdx.x) * P + q] = cnt[q];
+}
+
+__global__ void rank_scan_kernel(int *table, int nblk, int P) {
+  const int q = blockIdx.x * blockDim.x + threadIdx.x;
+  if (q >= P) return;
+  int run = 0;
+  for (int k = 0; k < nblk; ++k) {
+    const int v = table[int64_t(k) * P + q];
+    table[int64_t(k) * P + q] = run;
+    run += v;
+  }
+  table[int64_t(nblk) * P + q] = run;
+}
+
+// One warp per trajectory b of prompt p: the sum of the rewards of the most
+// recent min(k, window) in-batch trajectories of p before b, walking down from
+// b - 1 32 entries at a time (lane l takes b - 1 - 32 j - l; a ballot ranks
+// the hits, newest first), and k, their number. With the rank table the walk
+// stops at the window-th hit and k comes from the table; without it the walk
+// runs to the start of the batch. Either way the same hits are summed in the
+// same order.
+__global__ void __launch_bounds__(256) running_mean_kernel(const float *R, const int32_t *pid, int B, int P,
+                                                           const int *table, const float *history,
+                                                           const long long *seen, int window, float *a_traj,
+                                                           long long *rec, int *rank) {
   const int lane = threadIdx.x & 31;
   const int b = blockIdx.x * 8 + (threadIdx.x >> 5);
-  const int p = b < B ? pid[b] : -1;
-  double sum = 0.0;  // this lane's share
-  int k = 0;         // in-batch trajectories of p before b (warp-uniform)
-  // tiles of the batch, newest first, down from the block's last trajectory
-  const int bend = min(B, int(blockIdx.x + 1) * 8);
-  for (int t1 = bend; t1 > 0; t1 -= kTile) {
-    const int t0 = max(0, t1 - kTile), len = t1 - t0;
-    __syncthreads();
-    for (int i = threadIdx.x; i < len; i += blockDim.x) {
-      sp[i] = pid[t0 + i];
-      sR[i] = R[t0 + i];
+  if (b >= B) return;
+  const int p = pid[b];
+  if (p < 0 || p >= P) {  // outside [0, num_prompts): no window to read, advantage 0
+    if (lane == 0) {
+      a_traj[b] = 0.f;
+      rec[b] = -1;
     }
-    __syncthreads();
-    if (b >= B) continue;
-    // entries i = top - lane for top = min(len, b - t0) - 1, top - 32, ...
-    for (int top = min(len, b - t0) - 1; top >= 0; top -= 32) {
-      const int i = top - lane;
-      const bool hit = i >= 0 && sp[i] == p;
-      const unsigned mask = __ballot_sync(0xffffffffu, hit);
-      if (hit && k + __popc(mask & ((1u << lane) - 1u)) < window) sum += double(sR[i]);
-      k += __popc(mask);
+    return;
+  }
+  double sum = 0.0;  // this lane's share
+  int hits = 0;      // warp-uniform
+  for (int top = b - 1; top >= 0; top -= 32) {
+    const int i = top - lane;
+    const bool hit = i >= 0 && __ldg(pid + i) == p;
+    const unsigned mask = __ballot_sync(0xffffffffu, hit);
+    if (hit && hits + __popc(mask & ((1u << lane) - 1u)) < window) sum += double(__ldg(R + i));
+    hits += __popc(mask);
+    if (table && hits >= window) break;
+  }
+  int k = hits;
+  if (table) {  // rank of b: earlier blocks from the table, then b's own block
+    const int b0 = b / kRankBlock * kRankBlock;
+    k = __ldg(table + int64_t(b / kRankBlock) * P + p);
+    for (int i0 = b0; i0 < b; i0 += 32) {
+      const int i = i0 + lane;
+      k += __popc(__ballot_sync(0xffffffffu, i < b && __ldg(pid + i) == p));
     }
   }
-  if (b >= B) return;
   const long long c = seen[p];
   // old slots still holding rewards: the first min(c, window) slots, except the
   // k (cyclic) slots c % window, ..., (c + k - 1) % window written since
@@ -472,15 +514,18 @@ __global__ void __launch_bounds__(256) running_mean_kernel(const float *R, const
     const long long n = (c + k) < window ? (c + k) : window;
     a_traj[b] = float(double(R[b]) - (n > 0 ? sum / double(n) : 0.0));
     rec[b] = c + k;  // b's position in its prompt's reward sequence
+    if (rank) rank[b] = k;
   }
 }
 
 // Records the batch: the last `window` rewards of each prompt go to their ring
 // slots (distinct slots), and the prompt's last trajectory advances its count.
-// Positions come from the first pass, so this pass never reads `seen`. One
-// warp per trajectory counts the later trajectories of its prompt, stopping
-// once there are `window` of them.
-__global__ void __launch_bounds__(256) running_mean_record_kernel(const float *R, const int32_t *pid, int B,
+// Positions come from the first pass, so this pass never reads `seen`. The
+// number of later trajectories of b's prompt is its total minus b's rank when
+// the rank table exists; otherwise one warp per trajectory counts them,
+// stopping once there are `window` of them.
+__global__ void __launch_bounds__(256) running_mean_record_kernel(const float *R, const int32_t *pid, int B, int P,
+                                                                  const int *totals, const int *rank,
                                                                   const long long *rec, float *history,
                                                                   long long *seen, int window) {
   __shared__ int32_t sp[kTile];
@@ -488,16 +533,20 @@ __global__ void __launch_bounds__(256) running_mean_record_kernel(const float *R
   const int b = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int p = b < B ? pid[b] : -1;
   int after = 0;
-  for (int t0 = int(blockIdx.x) * 8 + 1; t0 < B; t0 += kTile) {
-    const int len = min(kTile, B - t0);
-    __syncthreads();
-    for (int i = threadIdx.x; i < len; i += blockDim.x) sp[i] = pid[t0 + i];
-    __syncthreads();
-    if (b >= B || after >= window) continue;
-    for (int i = max(0, b + 1 - t0) + lane; i - lane < len && after < window; i += 32)
-      after += __popc(__ballot_sync(0xffffffffu, i < len && sp[i] == p));
+  if (totals) {
+    if (b < B && p >= 0 && p < P) after = totals[p] - 1 - rank[b];
+  } else {
+    for (int t0 = int(blockIdx.x) * 8 + 1; t0 < B; t0 += kTile) {
+      const int len = min(kTile, B - t0);
+      __syncthreads();
+      for (int i = threadIdx.x; i < len; i += blockDim.x) sp[i] = pid[t0 + i];
+      __syncthreads();
+      if (b >= B || after >= window) continue;
+      for (int i = max(0, b + 1 - t0) + lane; i - lane < len && after < window; i += 32)
+        after += __popc(__ballot_sync(0xffffffffu, i < len && sp[i] == p));
+    }
   }
-  if (b >= B || lane != 0) return;
+  if (b >= B || lane != 0 || rec[b] < 0) return;  // rec < 0: a prompt id outside [0, num_prompts)
   if (after < window) history[int64_t(p) * window + int(rec[b] % window)] = R[b];
   if (after == 0) seen[p] = rec[b] + 1;
 }
@@ -597,9 +646,9 @@ sao_status group_adv_launch(const float *rewards, const int32_t *gid, int32_t B,
   return broadcast_launch(a_traj, m, cu, B, N, chunk_first, adv, s);
 }
 
-sao_status running_mean_launch(const float *rewards, const int32_t *pid, int32_t B, float *history, int64_t *seen,
-                               int32_t window, const uint8_t *m, const int32_t *cu, int64_t N, float *adv,
-                               void *ws_body, size_t body_bytes, cudaStream_t s) {
+sao_status running_mean_launch(const float *rewards, const int32_t *pid, int32_t B, int32_t P, float *history,
+                               int64_t *seen, int32_t window, const uint8_t *m, const int32_t *cu, int64_t N,
+                               float *adv, void *ws_body, size_t body_bytes, cudaStream_t s) {
   Carver c(ws_body, body_bytes);
   float *a_traj = c.take<float>(size_t(B) + 1);
   long long *rec = c.take<long long>(size_t(B) + 1);
@@ -609,12 +658,28 @@ sao_status running_mean_launch(const float *rewards, const int32_t *pid, int32_t
     if (N > 0) SAO_CUDA_TRY(cudaMemsetAsync(adv, 0, sizeof(float) * size_t(N), s));
     return SAO_OK;
   }
+  // the rank table, when the prompt ids are few enough and it fits in the rest of the workspace
+  const int nblk = (B + kRankBlock - 1) / kRankBlock;
+  int *table = nullptr, *rank = nullptr;
+  if (P <= kRankMaxPrompts) {
+    Carver t = c;
+    int *tab = t.take<int>(size_t(nblk + 1) * size_t(P));
+    int *rk = t.take<int>(size_t(B));
+    if (t.ok()) {
+      table = tab;
+      rank = rk;
+    }
+  }
   int slot = launch_begin("running_mean_advantages", s);
+  if (table) {
+    rank_count_kernel<<<unsigned(nblk), 256, 0, s>>>(pid, B, P, table);
+    rank_scan_kernel<<<unsigned((P + 255) / 256), 256, 0, s>>>(table, nblk, P);
+  }
   const unsigned g = unsigned((B + 7) / 8);  // a warp per trajectory
-  running_mean_kernel<<<g, 256, 0, s>>>(rewards, pid, B, history, reinterpret_cast<const long long *>(seen), window,
-                                        a_traj, rec);
-  running_mean_record_kernel<<<g, 256, 0, s>>>(rewards, pid, B, rec, history, reinterpret_cast<long long *>(seen),
-                                               window);
+  running_mean_kernel<<<g, 256, 0, s>>>(rewards, pid, B, P, table, history,
+                                        reinterpret_cast<const long long *>(seen), window, a_traj, rec, rank);
+  running_mean_record_kernel<<<g, 256, 0, s>>>(rewards, pid, B, P, table ? table + int64_t(nblk) * P : nullptr,
+                                               rank, rec, history, reinterpret_cast<long long *>(seen), window);
   SAO_TRY(launch_end(slot, s));
   return broadcast_launch(a_traj, m, cu, B, N, chunk_first, adv, s);
 }

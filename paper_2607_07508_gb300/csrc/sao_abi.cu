@@ -452,8 +452,8 @@ sao_status sao_running_mean_advantages(const float *rewards, const int32_t *prom
   SAO_TRY(take_ws(ws, ws_bytes, baselines_ws_bytes(N, B), &w));
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   SAO_TRY(begin_call(ws, s));
-  SAO_TRY(running_mean_launch(rewards, prompt_ids, B, history, seen, window, loss_mask, cu_seqlens, N, adv, w.body,
-                              w.body_bytes, s));
+  SAO_TRY(running_mean_launch(rewards, prompt_ids, B, num_prompts, history, seen, window, loss_mask, cu_seqlens, N,
+                              adv, w.body, w.body_bytes, s));
   return finish_call(ws, s);
 }
 

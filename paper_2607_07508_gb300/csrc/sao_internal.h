@@ -44,9 +44,9 @@ sao_status clip_loss_launch(const float *logp, const float *old, const float *ad
                             int32_t B, int64_t N, float eps_low, float eps_high, int norm, float *loss, float *coef,
                             uint8_t *flags, int64_t *counts, const float *grad_loss, void *ws_body,
                             size_t body_bytes, cudaStream_t s);
-sao_status running_mean_launch(const float *rewards, const int32_t *pid, int32_t B, float *history, int64_t *seen,
-                               int32_t window, const uint8_t *m, const int32_t *cu, int64_t N, float *adv,
-                               void *ws_body, size_t body_bytes, cudaStream_t s);
+sao_status running_mean_launch(const float *rewards, const int32_t *pid, int32_t B, int32_t P, float *history,
+                               int64_t *seen, int32_t window, const uint8_t *m, const int32_t *cu, int64_t N,
+                               float *adv, void *ws_body, size_t body_bytes, cudaStream_t s);
 sao_status group_adv_launch(const float *rewards, const int32_t *gid, int32_t B, const uint8_t *m, const int32_t *cu,
                             int64_t N, float eps, float *adv, void *ws_body, size_t body_bytes, cudaStream_t s);
 

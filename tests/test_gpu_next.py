@@ -185,7 +185,8 @@ def test_group_and_running_mean_edge_layouts():
     """5,003 trajectories (several shared-memory tiles, a partly filled last
     CTA), empty and one-token trajectories, ragged lengths, a misaligned mask
     and output (the broadcast's scalar path), and for the running mean two
-    batches with per-prompt windows of 8 and one window of 128."""
+    batches with per-prompt windows of 8, one window of 128, and 5,000 prompts
+    (the walk without the rank table)."""
     rng = np.random.default_rng(11)
     lengths = rng.integers(0, 40, size=5003)
     lengths[:3] = [0, 1, 0]
@@ -198,7 +199,7 @@ def test_group_and_running_mean_edge_layouts():
     torch.cuda.synchronize()
     want = O.group_advantages(wl.rewards, gid, wl.loss_mask, wl.cu_seqlens, f32(1e-6))
     assert rel_err_floor(adv.cpu().numpy(), want, 1e-3).max() <= 1e-5
-    for P, window in ((37, 8), (1, 128)):
+    for P, window in ((37, 8), (1, 128), (5000, 8)):  # 5000 prompts: more than the rank table takes
         hist_d = torch.zeros(P, window, device="cuda")
         seen_d = torch.zeros(P, dtype=torch.int64, device="cuda")
         hist_o, seen_o = np.zeros((P, window)), np.zeros(P, np.int64)
