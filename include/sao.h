@@ -269,7 +269,9 @@ SAO_API sao_status sao_group_advantages(const float *rewards, const int32_t *gro
  *   history [num_prompts, window] fp32 and seen [num_prompts] int64: the
  *   windows (ring buffers indexed by seen % window) and the number of rewards
  *   recorded per prompt; caller-owned device state, updated in place (zero
- *   both before the first batch). prompt_ids in [0, num_prompts).
+ *   both before the first batch). prompt_ids in [0, num_prompts); a
+ *   trajectory with an id outside that range gets advantage 0 and is not
+ *   recorded.
  */
 SAO_API sao_status sao_running_mean_advantages(const float *rewards, const int32_t *prompt_ids, int32_t B,
                                                int32_t num_prompts, float *history, int64_t *seen, int32_t window,
