@@ -142,3 +142,25 @@ def test_logprobs_backward_all_zero_gradient(dt):
     torch.cuda.synchronize()
     assert not dH.float().abs().max().item() and not dW.abs().max().item()
     assert torch.equal(dW2, prev)
+
+
+def test_logprobs_backward_all_zero_gradient_paired_tiles():
+    """The same with h = 2048 and V = 20,000, where the dW GEMM takes two M
+    tiles per CTA tile: the empty contraction writes zeros to both tiles, or
+    leaves dW unchanged when accumulating; on both log-prob paths."""
+    wl, H, W, y = _case(300, 2048, 20000, "bf16", seed=4)
+    logp, lse = _fwd(H, W, y)
+    G = torch.zeros(300, device="cuda")
+    dH, dW = _bwd(H, W, y, lse, G)
+    prev = torch.randn(20000, 2048, device="cuda")
+    _, dW2 = _bwd(H, W, y, lse, G, accumulate=prev)
+    cache = sao.logprob_cache(300, 20000)
+    ws = sao.workspace(300, 2048, 20000, H.dtype)
+    sao.sao_token_logprobs_fwd_cached(H, W, y, logp, lse, cache, ws)
+    dH3 = torch.full_like(H, float("nan"))
+    dW3 = torch.full((20000, 2048), float("nan"), device="cuda")
+    sao.sao_token_logprobs_bwd_cached(H, W, y, lse, G, dH3, dW3, cache, ws)
+    torch.cuda.synchronize()
+    assert not dH.float().abs().max().item() and not dW.abs().max().item()
+    assert torch.equal(dW2, prev)
+    assert not dH3.float().abs().max().item() and not dW3.abs().max().item()
