@@ -180,12 +180,14 @@ def test_cached_moe_bench_configuration_sampled_rows():
     assert rel_l2(got_dW, want_dW) <= GRAD_TOL
 
 
-@pytest.mark.parametrize("cached", [True, False])
-def test_two_m_tile_gemms_with_ragged_tiles(cached):
+@pytest.mark.parametrize("cached,chunked", [(True, False), (False, False), (True, True)])
+def test_two_m_tile_gemms_with_ragged_tiles(cached, chunked):
     """A shape at which both backward GEMMs take two 128-row M tiles per CTA
     tile (at least four waves of paired tiles on the GPU): 20,100 rows and
     20,168 vocabulary rows, so the last paired tile of dW has a full first and
-    a 72-row second tile, and dH's last pair a partial first tile only.
+    a 72-row second tile, and dH's last pair a partial first tile only. With
+    `chunked` a small dZ budget splits the vocabulary into chunks, so dH
+    accumulates in fp32 (the other store epilogue) and is scattered at the end.
     logp, dH on sampled rows and dW on sampled vocabulary rows (the last 72
     included) against the oracle."""
     N, h, V = 20100, 2048, 20168
@@ -200,14 +202,20 @@ def test_two_m_tile_gemms_with_ragged_tiles(cached):
     Gd = torch.as_tensor(G).cuda()
     dH = torch.full_like(H, float("nan"))
     dW = torch.full((V, h), float("nan"), device="cuda")
-    if cached:
-        cache = sao.logprob_cache(N, V)
-        sao.sao_token_logprobs_fwd_cached(H, W, y, logp, lse, cache, ws)
-        sao.sao_token_logprobs_bwd_cached(H, W, y, lse, Gd, dH, dW, cache, ws)
-    else:
-        sao.sao_token_logprobs_fwd(H, W, y, logp, lse, ws)
-        sao.sao_token_logprobs_bwd(H, W, y, lse, Gd, dH, dW, ws)
-    torch.cuda.synchronize()
+    if chunked:
+        sao.sao_set_dz_budget_bytes(N * 5120 * 2)       # Vc = 5120 -> 4 chunks, the last one ragged
+    try:
+        if cached:
+            cache = sao.logprob_cache(N, V)
+            sao.sao_token_logprobs_fwd_cached(H, W, y, logp, lse, cache, ws)
+            sao.sao_token_logprobs_bwd_cached(H, W, y, lse, Gd, dH, dW, cache, ws)
+        else:
+            sao.sao_token_logprobs_fwd(H, W, y, logp, lse, ws)
+            sao.sao_token_logprobs_bwd(H, W, y, lse, Gd, dH, dW, ws)
+        torch.cuda.synchronize()
+    finally:
+        if chunked:
+            sao.sao_set_dz_budget_bytes(24 << 30)
     rows = np.sort(np.concatenate([rng.choice(N, size=24, replace=False), [N - 1]]))
     H_cpu, W_cpu = H[torch.as_tensor(rows).cuda()].cpu(), W.cpu()
     want_lp, want_lse = O.token_logprobs(H_cpu, W_cpu, wl.y[rows])
