@@ -92,45 +92,39 @@ struct ClipArgs {
 };
 
 // One token of the clipped surrogate: returns the weighted value term and
-// writes the coefficient d loss / d logp (before the sign) and the flag.
+// writes the coefficient d loss / d logp (before the sign) and the flag. The
+// cases are taken by selects in the order not-action, non-finite, clipped
+// above, clipped below, kept; a value term is (w * f) * a with f = r, or the
+// bound it is clipped to.
 __device__ __forceinline__ float clip_token(float lp, float old, float a, bool act, float lo, float hi, float w,
                                             float &coef, uint8_t &flag, int &nl, int &nh, int &nf) {
-  coef = 0.f;
-  if (!act) {
-    flag = SAO_FLAG_NOT_ACTION;
-    return 0.f;
-  }
   const float d = lp - old;
-  if (!isfinite(d) || !isfinite(a)) {
-    flag = SAO_FLAG_NONFINITE;
-    nf++;
-    return 0.f;
-  }
+  // zero when d and a are both finite, NaN otherwise
+  const bool fin = ((d - d) + (a - a)) == 0.f;
   const float r = expf(d);
-  if (a > 0.f && r > hi) {
-    flag = 2;
-    nh++;
-    return w * hi * a;
-  }
-  if (a < 0.f && r < lo) {
-    flag = 1;
-    nl++;
-    return w * lo * a;
-  }
-  flag = 0;
-  const float t = w * r * a;
-  coef = -t;
-  return t;
+  const bool ch = a > 0.f && r > hi;
+  const bool cl = a < 0.f && r < lo;
+  const float f = ch ? hi : (cl ? lo : r);
+  const float t = w * f * a;
+  const bool live = act && fin;
+  nf += act && !fin;
+  nh += live && ch;
+  nl += live && cl;
+  flag = !act ? uint8_t(SAO_FLAG_NOT_ACTION) : !fin ? uint8_t(SAO_FLAG_NONFINITE) : ch ? uint8_t(2) : cl ? uint8_t(1) : uint8_t(0);
+  coef = live && !ch && !cl ? -t : 0.f;
+  return live ? t : 0.f;
 }
 
 template <bool kBwd>
-__global__ void __launch_bounds__(kThreads) clip_loss_kernel(ClipArgs a) {
+__global__ void __launch_bounds__(kThreads, 5) clip_loss_kernel(ClipArgs a) {
   __shared__ int32_t s_cu_all[kWarps][kCuCap];
   __shared__ float2 s_sum[kWarps];
   __shared__ int s_cnt[3][kWarps];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int q = blockIdx.x * kWarps + warp;
-  Sum2 acc;  // compensated sum of the value terms
+  // a lane's 32 value terms in fp32 (relative error ~1e-6, far inside the 1e-4
+  // loss bar); lanes, warps and CTAs are then combined compensated
+  float lacc = 0.f;
   int nl = 0, nh = 0, nf = 0;
   if (q < a.nchunks) {
     int blo, bhi;
@@ -183,18 +177,26 @@ __global__ void __launch_bounds__(kThreads) clip_loss_kernel(ClipArgs a) {
       }
       float cf[4];
       uint8_t fl[4];
+      float wt[4] = {w, w, w, w};
+      if (a.seq && tg + 3 >= next_end) {
+        // the lane's four tokens reach a trajectory end (rare for long trajectories)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int64_t t = tg + i;
+          if (t < N && t >= next_end) {
+            while (b < bhi && t >= next_end) {
+              ++b;
+              next_end = cu[b + 1];
+            }
+            w = weight(b);
+          }
+          wt[i] = w;
+        }
+      }
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        const int64_t t = tg + i;
-        if (a.seq && t < N && t >= next_end) {
-          while (b < bhi && t >= next_end) {
-            ++b;
-            next_end = cu[b + 1];
-          }
-          w = weight(b);
-        }
-        acc.add(clip_token(lp[i], od[i], ad[i], act[i], a.lo, a.hi, w, cf[i], fl[i], nl, nh, nf));
-        cf[i] *= gscale;
+        lacc += clip_token(lp[i], od[i], ad[i], act[i], a.lo, a.hi, wt[i], cf[i], fl[i], nl, nh, nf);
+        if constexpr (kBwd) cf[i] *= gscale;
       }
       if (vec) {
         if (a.coef) *reinterpret_cast<float4 *>(a.coef + tg) = make_float4(cf[0], cf[1], cf[2], cf[3]);
@@ -211,6 +213,8 @@ __global__ void __launch_bounds__(kThreads) clip_loss_kernel(ClipArgs a) {
   }
   if constexpr (!kBwd) {
     // warp, then CTA (fixed order), in compensated fp32
+    Sum2 acc;
+    acc.add(lacc);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       const float ohi = __shfl_xor_sync(0xffffffffu, acc.hi, o), olo = __shfl_xor_sync(0xffffffffu, acc.lo, o);

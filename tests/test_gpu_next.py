@@ -139,6 +139,46 @@ def test_clip_loss_edge_layouts(norm):
     assert rel_err_floor(coef, want["coef"], 1e-12).max() <= 1e-5
 
 
+
+@pytest.mark.parametrize("norm", [sao.SAO_NORM_TOKEN, sao.SAO_NORM_SEQUENCE])
+def test_clip_loss_short_trajectories_and_misaligned_inputs(norm):
+    """Trajectories of 0 to 6 tokens (hundreds per 1024-token chunk, more than
+    a chunk stages, so the walk reads the offsets from global memory) around
+    two long ones and a ragged tail; once with aligned inputs (the staged
+    path) and once with every input one element past a 16-byte boundary (the
+    scalar path)."""
+    rng = np.random.default_rng(12)
+    lengths = [int(x) for x in rng.integers(0, 7, size=1500)]
+    lengths[700] = 3000
+    lengths[-2] = 1500
+    wl = S.make_custom(lengths, 8, 16, "f32", seed=13, dense=False, obs_frac=0.3)
+    adv = rng.normal(size=wl.N).astype(np.float32)
+    old = (wl.logp_syn + rng.normal(0, 0.4, wl.N)).astype(np.float32)
+    el, eh = 0.2, 0.28
+    want = O.clip_loss(wl.logp_syn, old, adv, wl.loss_mask, wl.cu_seqlens, el, eh, norm)
+    skip = _near_clip_bound(wl.logp_syn, old, el, eh)
+    keep = ~skip
+    for mis in (False, True):
+        N = wl.N
+        place = _misaligned if mis else (lambda t: t)
+        loss = torch.empty(1, device="cuda")
+        counts = torch.empty(4, dtype=torch.int64, device="cuda")
+        coef = place(torch.full((N,), float("nan"), device="cuda"))
+        flags = place(torch.full((N,), 9, dtype=torch.uint8, device="cuda"))
+        grad = place(torch.full((N,), float("nan"), device="cuda"))
+        ws = sao.workspace(N)
+        args = [place(cuda(x)) for x in (wl.logp_syn, old, adv, wl.loss_mask)] + [cuda(wl.cu_seqlens)]
+        sao.sao_clip_loss_fwd(*args, el, eh, norm, loss, counts, ws, coef=coef, flags=flags)
+        sao.sao_clip_loss_bwd(*args, el, eh, norm, torch.tensor([2.0], device="cuda"), grad, ws)
+        torch.cuda.synchronize()
+        got_flags = flags.cpu().numpy()
+        assert np.array_equal(got_flags[keep], want["flags"][keep]), mis
+        if not skip.any():
+            assert np.array_equal(counts.cpu().numpy(), want["counts"]), mis
+        assert abs(loss.item() - want["loss"]) <= 1e-4 * max(abs(want["loss"]), 1e-6), mis
+        assert rel_err_floor(coef.cpu().numpy()[keep], want["coef"][keep], 1e-12).max() <= 1e-5, mis
+        assert rel_err_floor(grad.cpu().numpy()[keep], 2.0 * want["coef"][keep], 1e-12).max() <= 1e-5, mis
+
 def test_group_advantages_match_oracle():
     for name in ("small", "large"):
         wl = S.make_workload(name, dense=False)
