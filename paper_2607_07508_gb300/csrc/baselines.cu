@@ -44,14 +44,31 @@ struct Norms {
   long long n_seq;     // trajectories with at least one action token
 };
 
-// Sums the per-trajectory action counts (one CTA, fixed order).
-__global__ void __launch_bounds__(256) norms_kernel(const int *nact, int B, Norms *out) {
+// Sums the per-trajectory action counts: one CTA of 1024 threads, thread i
+// taking entries i, i + 1024, ... with eight loads in flight (integer sums,
+// so the order does not matter).
+constexpr int kNormThreads = 1024;
+
+__global__ void __launch_bounds__(kNormThreads) norms_kernel(const int *nact, int B, Norms *out) {
   long long n = 0, s = 0;
-  for (int b = threadIdx.x; b < B; b += 256) {
-    n += nact[b];
-    s += nact[b] > 0;
+  constexpr int kU = 8;
+  int b = threadIdx.x;
+  for (; b + (kU - 1) * kNormThreads < B; b += kU * kNormThreads) {
+    int v[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) v[u] = __ldg(nact + b + u * kNormThreads);
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      n += v[u];
+      s += v[u] > 0;
+    }
   }
-  __shared__ long long sh[2][8];
+  for (; b < B; b += kNormThreads) {
+    const int v = __ldg(nact + b);
+    n += v;
+    s += v > 0;
+  }
+  __shared__ long long sh[2][kNormThreads / 32];
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     n += __shfl_xor_sync(0xffffffffu, n, o);
@@ -64,7 +81,7 @@ __global__ void __launch_bounds__(256) norms_kernel(const int *nact, int B, Norm
   __syncthreads();
   if (threadIdx.x == 0) {
     Norms r{0, 0};
-    for (int w = 0; w < 8; ++w) {
+    for (int w = 0; w < kNormThreads / 32; ++w) {
       r.n_action += sh[0][w];
       r.n_seq += sh[1][w];
     }
@@ -584,10 +601,11 @@ sao_status clip_loss_launch(const float *logp, const float *old, const float *ad
   SAO_CUDA_TRY(cudaMemsetAsync(nact, 0, sizeof(int) * size_t(B), s));
   const unsigned grid = unsigned((nchunks + kWarps - 1) / kWarps);
   int slot = launch_begin("clip_loss_counts", s);
-  seg::chunk_first_kernel<<<unsigned((nchunks + 255) / 256), 256, 0, s>>>(cu, B, N, int(nchunks), chunk_first);
+  seg::chunk_first_kernel<<<seg::chunk_first_grid(int(nchunks)), seg::kChunkFirstThreads, 0, s>>>(
+      cu, B, N, int(nchunks), chunk_first);
   seg::action_count_kernel<<<seg::action_count_grid(int(nchunks)), 256, 0, s>>>(m, cu, B, N, int(nchunks),
                                                                                 chunk_first, nact);
-  norms_kernel<<<1, 256, 0, s>>>(nact, B, norms);
+  norms_kernel<<<1, kNormThreads, 0, s>>>(nact, B, norms);
   SAO_TRY(launch_end(slot, s));
   ClipArgs a;
   a.logp = logp;
@@ -628,7 +646,8 @@ static sao_status broadcast_launch(const float *a_traj, const uint8_t *m, const 
   if (N == 0) return SAO_OK;
   const int64_t nchunks = (N + kSegChunk - 1) / kSegChunk;
   int slot = launch_begin("adv_broadcast", s);
-  seg::chunk_first_kernel<<<unsigned((nchunks + 255) / 256), 256, 0, s>>>(cu, B, N, int(nchunks), chunk_first);
+  seg::chunk_first_kernel<<<seg::chunk_first_grid(int(nchunks)), seg::kChunkFirstThreads, 0, s>>>(
+      cu, B, N, int(nchunks), chunk_first);
   seg::traj_broadcast_kernel<<<seg::action_count_grid(int(nchunks)), 256, 0, s>>>(a_traj, m, cu, B, N,
                                                                                   int(nchunks), chunk_first, adv);
   return launch_end(slot, s);

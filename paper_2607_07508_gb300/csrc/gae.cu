@@ -852,7 +852,8 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   }
   {
     int slot = launch_begin("gae_chunk_first", s);
-    seg::chunk_first_kernel<<<unsigned((nchunks + 255) / 256), 256, 0, s>>>(cu, B, N, int(nchunks), chunk_first);
+    seg::chunk_first_kernel<<<seg::chunk_first_grid(int(nchunks)), seg::kChunkFirstThreads, 0, s>>>(
+      cu, B, N, int(nchunks), chunk_first);
     SAO_TRY(launch_end(slot, s));
   }
   if (alpha > 0.f) {

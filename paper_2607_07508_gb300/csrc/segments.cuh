@@ -14,6 +14,14 @@ constexpr int kSegChunk = 32 * kItems;   // tokens per warp chunk
 constexpr int kCuCap = 128;              // cu_seqlens entries staged per warp
 constexpr int kCountChunks = 8;          // chunks per warp in action_count_kernel
 
+// chunk_first_kernel: one chunk per thread, 1024 threads per CTA, and a
+// sample of every ceil(B / 4096)-th cu_seqlens entry in shared memory.
+constexpr int kChunkFirstThreads = 1024;
+constexpr int kChunkFirstSample = 4096;
+__host__ __device__ constexpr unsigned chunk_first_grid(int nchunks) {
+  return unsigned((nchunks + kChunkFirstThreads - 1) / kChunkFirstThreads);
+}
+
 // CTAs (of 8 warps) of action_count_kernel for nchunks chunks.
 __host__ __device__ constexpr unsigned action_count_grid(int nchunks) {
   return unsigned((nchunks + 8 * kCountChunks - 1) / (8 * kCountChunks));
@@ -38,17 +46,6 @@ struct CuView {
   }
 };
 
-// Largest b in [0, B-1] with cu[b] <= t (the trajectory holding token t).
-__device__ __forceinline__ int find_traj(const int32_t *cu, int B, int64_t t) {
-  int lo = 0, hi = B - 1;
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (int64_t(__ldg(cu + mid)) <= t) lo = mid;
-    else hi = mid - 1;
-  }
-  return lo;
-}
-
 // Stages the cu_seqlens slice of warp chunk q into `s_cu` (kCuCap entries) and
 // returns the view; blo/bhi are the first/last trajectories the chunk can touch.
 __device__ __forceinline__ CuView stage_chunk(const int32_t *cu, int B, int nchunks, const int *chunk_first, int q,
@@ -67,12 +64,37 @@ __device__ __forceinline__ CuView stage_chunk(const int32_t *cu, int B, int nchu
 // includes this header launches its own copy.
 namespace {
 
-// First trajectory of every warp chunk (one binary search per chunk).
-__global__ void chunk_first_kernel(const int32_t *cu, int B, int64_t N, int nchunks, int *chunk_first) {
-  const int q = blockIdx.x * blockDim.x + threadIdx.x;
+// First trajectory of every warp chunk: the largest b with cu[b] <= t for the
+// chunk's first token t. The CTA stages the samples cu[k S] (S = ceil(B /
+// 4096)); a thread's search over them gives the k with cu[k S] <= t <
+// cu[(k + 1) S], so the answer lies in [k S, (k + 1) S) and only that short
+// range is searched in global memory. Grid: chunk_first_grid, block
+// kChunkFirstThreads.
+__global__ void __launch_bounds__(kChunkFirstThreads) chunk_first_kernel(const int32_t *cu, int B, int64_t N,
+                                                                        int nchunks, int *chunk_first) {
+  __shared__ int32_t samp[kChunkFirstSample];
+  const int S = B > kChunkFirstSample ? (B + kChunkFirstSample - 1) / kChunkFirstSample : 1;
+  const int ns = (B + S - 1) / S;  // samples k S < B
+  for (int k = threadIdx.x; k < ns; k += kChunkFirstThreads) samp[k] = __ldg(cu + int64_t(k) * S);
+  __syncthreads();
+  const int q = blockIdx.x * kChunkFirstThreads + threadIdx.x;
   if (q >= nchunks) return;
-  const int64_t t = int64_t(q) * kSegChunk;
-  chunk_first[q] = find_traj(cu, B, t < N ? t : N - 1);
+  int64_t t = int64_t(q) * kSegChunk;
+  if (t >= N) t = N - 1;
+  int lo = 0, hi = ns - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (int64_t(samp[mid]) <= t) lo = mid;
+    else hi = mid - 1;
+  }
+  int blo = lo * S;
+  int bhi = blo + S - 1 < B - 1 ? blo + S - 1 : B - 1;
+  while (blo < bhi) {
+    const int mid = (blo + bhi + 1) >> 1;
+    if (int64_t(__ldg(cu + mid)) <= t) blo = mid;
+    else bhi = mid - 1;
+  }
+  chunk_first[q] = blo;
 }
 
 // Number of action tokens per trajectory; nact must start at zero. One warp

@@ -86,29 +86,69 @@ __global__ void __launch_bounds__(kThreads) step_count_kernel(const uint8_t *m, 
 }
 static_assert(kRowsPerBlock == kThreads * 16, "16 tokens per thread");
 
-__global__ void __launch_bounds__(1024) step_scan_kernel(int *block_count, int nblocks, int *total) {
-  __shared__ int sh[1024];
-  const int per = (nblocks + 1023) / 1024;
-  const int b0 = threadIdx.x * per;
-  int s = 0;
-  for (int i = 0; i < per; ++i)
-    if (b0 + i < nblocks) s += block_count[b0 + i];
-  sh[threadIdx.x] = s;
-  __syncthreads();
-  for (int o = 1; o < 1024; o <<= 1) {
-    const int v = threadIdx.x >= o ? sh[threadIdx.x - o] : 0;
-    __syncthreads();
-    sh[threadIdx.x] += v;
-    __syncthreads();
+// Exclusive scan of the per-block step counts in place (one CTA of 1024
+// threads). Thread i owns a run of `per` consecutive counts, `per` a multiple
+// of 8, so each 8-count piece is two aligned 16-byte loads and a thread's
+// pieces are all in flight at once; warp shuffles and one shared-memory row
+// of warp totals scan the thread sums.
+constexpr int kScanPiece = 8;
+
+__device__ __forceinline__ void load_piece(const int *p, int b, int nblocks, int (&v)[kScanPiece]) {
+  if (b + kScanPiece <= nblocks && (reinterpret_cast<uintptr_t>(p) & 15u) == 0) {
+    const int4 x = *reinterpret_cast<const int4 *>(p + b);
+    const int4 y = *reinterpret_cast<const int4 *>(p + b + 4);
+    v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
+    v[4] = y.x; v[5] = y.y; v[6] = y.z; v[7] = y.w;
+  } else {
+#pragma unroll
+    for (int k = 0; k < kScanPiece; ++k) v[k] = b + k < nblocks ? p[b + k] : 0;
   }
-  int run = threadIdx.x ? sh[threadIdx.x - 1] : 0;
-  for (int i = 0; i < per; ++i)
-    if (b0 + i < nblocks) {
-      const int c = block_count[b0 + i];
-      block_count[b0 + i] = run;
-      run += c;
+}
+
+__global__ void __launch_bounds__(1024) step_scan_kernel(int *block_count, int nblocks, int *total) {
+  __shared__ int sh[32];
+  const int per = ((nblocks + 1023) / 1024 + kScanPiece - 1) / kScanPiece * kScanPiece;
+  const int b0 = threadIdx.x * per;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int s = 0;
+#pragma unroll 4
+  for (int i = 0; i < per; i += kScanPiece) {
+    int v[kScanPiece];
+    load_piece(block_count, b0 + i, nblocks, v);
+#pragma unroll
+    for (int k = 0; k < kScanPiece; ++k) s += v[k];
+  }
+  int x = s;  // inclusive scan of the thread sums within the warp
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) sh[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = sh[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
     }
-  if (threadIdx.x == 1023) *total = sh[1023];
+    sh[lane] = w;  // inclusive over warps
+  }
+  __syncthreads();
+  int run = (warp ? sh[warp - 1] : 0) + x - s;
+#pragma unroll 4
+  for (int i = 0; i < per; i += kScanPiece) {
+    int v[kScanPiece];
+    load_piece(block_count, b0 + i, nblocks, v);
+#pragma unroll
+    for (int k = 0; k < kScanPiece; ++k) {
+      const int b = b0 + i + k;
+      if (b < nblocks) block_count[b] = run;
+      run += v[k];
+    }
+  }
+  if (threadIdx.x == 1023) *total = sh[31];
 }
 
 // Ordered step list with each step's first and one-past-last token.
@@ -223,11 +263,19 @@ __global__ void __launch_bounds__(kThreads) step_reduce_kernel(const float *valu
   const int lane = threadIdx.x & 31;
   const int S = *nsteps;
   const int nwarps = (gridDim.x * kThreads) >> 5;
-  for (int g = (blockIdx.x * kThreads + threadIdx.x) >> 5; g * 32 < S; g += nwarps) {
+  // the next group's step ranges are loaded while this group is summed
+  int g = (blockIdx.x * kThreads + threadIdx.x) >> 5;
+  int nfirst = g * 32 + lane < S ? step_first[g * 32 + lane] : 0;
+  int nend = g * 32 + lane < S ? step_end[g * 32 + lane] : 0;
+  for (; g * 32 < S; g += nwarps) {
     const int s = g * 32 + lane;
     const bool own = s < S;
-    const int first = own ? step_first[s] : 0;
-    const int end = own ? step_end[s] : 0;
+    const int first = nfirst, end = nend;
+    const int sn = (g + nwarps) * 32 + lane;
+    if (sn < S) {
+      nfirst = step_first[sn];
+      nend = step_end[sn];
+    }
     if (mode == SAO_STEP_LAST) {  // the value of the step's last token
       if (own) sv[s] = make_float2(values[end - 1], 0.f);
       continue;
@@ -251,7 +299,15 @@ __global__ void __launch_bounds__(kThreads) step_reduce_kernel(const float *valu
       longs &= longs - 1;
       const int f = __shfl_sync(0xffffffffu, first, src), e = __shfl_sync(0xffffffffu, end, src);
       Acc2 part;
-      for (int t = f + lane; t < e; t += 32) part.add(values[t]);
+      // a lane's tokens f + lane, f + lane + 32, ... in order, four loads at a time
+      for (int t = f + lane; t < e; t += 128) {
+        float x[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) x[k] = t + 32 * k < e ? values[t + 32 * k] : 0.f;
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          if (t + 32 * k < e) part.add(x[k]);
+      }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
         Acc2 other;
@@ -276,25 +332,37 @@ __device__ __forceinline__ dd dd_shfl_down(dd x, int d) {
   return {__shfl_down_sync(0xffffffffu, x.hi, d), __shfl_down_sync(0xffffffffu, x.lo, d)};
 }
 
+constexpr int kGaeWarps = 4;  // warps (trajectories) per CTA of step_gae_kernel
+constexpr int kStepGroup = 8; // step values a lane loads ahead of its recursion
+
 // One warp per trajectory: lane l folds steps [s0 + l*c, s0 + (l+1)*c) into
 // maps for the policy (a = gamma*lambda_b) and the critic (a = gamma*lambda_c),
 // a shuffle scan gives each lane the advantages to the right of its block, and
-// the lane replays its block.
+// the lane replays its block. Both passes walk the block backwards in groups
+// of kStepGroup steps whose values are loaded before the group's recursion, so
+// a long trajectory (thousands of steps per lane) waits for one load latency
+// per group, not per step.
 // kCrit false: gamma = lambda_critic = 1, where the critic's return telescopes
 // to the trajectory's reward R on every step, so only the policy recursion runs.
 template <bool kCrit>
-__global__ void __launch_bounds__(128) step_gae_kernel(const float *rewards, const int32_t *cu, int B,
-                                                       const int *step_first, const int *nsteps, const float2 *sv,
-                                                       float gamma, float lam, float lam_c, float alpha,
-                                                       float2 *out /*[S] (adv, ret)*/) {
+__global__ void __launch_bounds__(32 * kGaeWarps) step_gae_kernel(const float *rewards, const int32_t *cu, int B,
+                                                                  int64_t N, const int *step_first,
+                                                                  const int *block_offset, int nblocks,
+                                                                  const int *nsteps, const float2 *sv, float gamma,
+                                                                  float lam, float lam_c, float alpha,
+                                                                  float2 *out /*[S] (adv, ret)*/) {
   const int lane = threadIdx.x & 31;
-  const int b = (blockIdx.x * 128 + threadIdx.x) >> 5;
+  const int b = (blockIdx.x * (32 * kGaeWarps) + threadIdx.x) >> 5;
   if (b >= B) return;
   const int S = *nsteps;
   // steps of trajectory b: those whose first token lies in [cu[b], cu[b+1]);
-  // first step index with step_first >= t by a 33-way warp search
+  // first step index with step_first >= t by a 33-way warp search, starting
+  // from the steps opened before t's 4096-token block and before the next one
   auto lower = [&](int64_t t) {
-    int lo = 0, hi = S;  // the answer lies in [lo, hi]
+    if (t >= N) return S;
+    const int blk = int(t / kRowsPerBlock);
+    int lo = block_offset[blk];
+    int hi = blk + 1 < nblocks ? block_offset[blk + 1] : S;  // the answer lies in [lo, hi]
     while (hi - lo > 32) {
       const int p = lo + int(int64_t(hi - lo) * (lane + 1) / 33);  // 32 rising pivots in [lo, hi)
       const unsigned below = __ballot_sync(0xffffffffu, int64_t(step_first[p]) < t);
@@ -336,13 +404,22 @@ __global__ void __launch_bounds__(128) step_gae_kernel(const float *rewards, con
   StepMap mp{one, zero}, mc{one, zero};
   {
     dd v_next = v_after;
-    for (int i = a1 - 1; i >= a0; --i) {
-      const dd v = value(i);
+    auto fold = [&](int i, float2 vi) {
+      const dd v{vi.x, vi.y};
       const dd d = delta(i, v, v_next);
       mp = {dd_mul(ap, mp.p), dd_add(dd_mul(ap, mp.c), d)};
       if constexpr (kCrit) mc = {dd_mul(ac, mc.p), dd_add(dd_mul(ac, mc.c), d)};
       v_next = v;
+    };
+    int i = a1 - 1;
+    for (; i - (kStepGroup - 1) >= a0; i -= kStepGroup) {
+      float2 vg[kStepGroup];
+#pragma unroll
+      for (int k = 0; k < kStepGroup; ++k) vg[k] = sv[i - k];
+#pragma unroll
+      for (int k = 0; k < kStepGroup; ++k) fold(i - k, vg[k]);
     }
+    for (; i >= a0; --i) fold(i, sv[i]);
   }
   // suffix scan over lanes: the maps of lanes l+1 .. 31 applied to A = 0
   StepMap sp = mp, sc = mc;
@@ -359,8 +436,8 @@ __global__ void __launch_bounds__(128) step_gae_kernel(const float *rewards, con
   if constexpr (kCrit) Ac = dd_shfl_down(sc.c, 1);
   if (lane == 31) Ap = Ac = zero;
   dd v_next = v_after;
-  for (int i = a1 - 1; i >= a0; --i) {
-    const dd v = value(i);
+  auto replay = [&](int i, float2 vi) {
+    const dd v{vi.x, vi.y};
     const dd d = delta(i, v, v_next);
     Ap = dd_add(dd_mul(ap, Ap), d);
     float r = R;
@@ -370,7 +447,16 @@ __global__ void __launch_bounds__(128) step_gae_kernel(const float *rewards, con
     }
     out[i] = make_float2(dd_round(Ap), r);
     v_next = v;
+  };
+  int i = a1 - 1;
+  for (; i - (kStepGroup - 1) >= a0; i -= kStepGroup) {
+    float2 vg[kStepGroup];
+#pragma unroll
+    for (int k = 0; k < kStepGroup; ++k) vg[k] = sv[i - k];
+#pragma unroll
+    for (int k = 0; k < kStepGroup; ++k) replay(i - k, vg[k]);
   }
+  for (; i >= a0; --i) replay(i, sv[i]);
 }
 
 // Every token reads its step's results (non-action tokens get zeros); four
@@ -516,8 +602,8 @@ sao_status step_gae_launch(const float *values, const float *rewards, const uint
   SAO_TRY(launch_end(slot, s));
   slot = launch_begin("step_gae_scan", s);
   auto scan = (gamma == 1.f && lam_c == 1.f) ? step_gae_kernel<false> : step_gae_kernel<true>;
-  scan<<<unsigned((int64_t(B) * 32 + 127) / 128), 128, 0, s>>>(rewards, cu, B, step_first, nsteps, sv, gamma, lam,
-                                                               lam_c, alpha, out);
+  scan<<<unsigned((int64_t(B) + kGaeWarps - 1) / kGaeWarps), 32 * kGaeWarps, 0, s>>>(
+      rewards, cu, B, N, step_first, block, int(nblocks), nsteps, sv, gamma, lam, lam_c, alpha, out);
   SAO_TRY(launch_end(slot, s));
   slot = launch_begin("step_gae_broadcast", s);
   step_broadcast_kernel<<<unsigned(nblocks), kThreads, 0, s>>>(m, ts, N, block, step_end, out, mode, adv, ret,
