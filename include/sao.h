@@ -145,12 +145,16 @@ SAO_API sao_status sao_token_logprobs_bwd(const void *H, const void *W, sao_dtyp
 
 /*
  * The same two calls with the forward's probabilities kept for the backward
- * (bf16 only). The forward additionally stores, for every row it computes,
- * e[t, v] = exp(z[t, v] - m) in bf16, m being the maximum of z[t, .] over the
- * 256-wide vocabulary tile holding v, with those maxima; the backward forms
- * p[t, v] = e[t, v] exp(m - lse[t]) from them, so dZ costs one pass over the
- * stored rows instead of recomputing the logits (2 h V flops per row). The
- * results match sao_token_logprobs_fwd / _bwd within the bf16 rounding of e.
+ * (bf16 only), so the backward needs neither the logits nor dZ in memory.
+ * For every row it computes, the forward takes a shift kappa = z[t, y] + 20
+ * (the sampled token's logit, from a pre-pass) and stores e[t, v] = exp(z[t,
+ * v] - kappa) in bf16; once lse is known, the entry at v = y becomes e[t, y] -
+ * exp(lse - kappa). Then dZ[t, .] = -G[t] exp(kappa - lse[t]) e[t, .], and the
+ * backward is two GEMMs on e: dH = (e W) scaled per row, dW = e^T (s H). A row
+ * with some z[t, v] more than 60 above z[t, y] (p_y below e^-60) would
+ * overflow that range: the forward flags it (its lse and log-prob are still
+ * exact) and the backward recomputes that row's logits. The results match
+ * sao_token_logprobs_fwd / _bwd within the bf16 rounding of e and of s H.
  *   cache        caller-owned device buffer of sao_logprob_cache_bytes(N, V)
  *                bytes (about 2 N V bytes), 256-byte aligned; written by the
  *                forward, read (not modified) by the backward, which must get

@@ -26,14 +26,24 @@ sao_status simt_bwd(const float *H, const float *W, const int32_t *y, const floa
                     int64_t N, int32_t h, int32_t V, float *dH, float *dW, int accumulate, void *ws,
                     size_t ws_bytes, cudaStream_t s);
 
-// The forward's stored probabilities (tensor-core path): e[f, v] =
-// exp(z - max_tile) in bf16 for forward row f, the per-(tile, row) partials
-// (max_tile, sum-exp) and the forward row of every token (-1: not computed).
+// The forward's stored probabilities (tensor-core path). For forward row f
+// (token idx[f]) with shift kappa[f] = z[f, y] + kKappaOffset, where z[f, y]
+// is the sampled token's logit from a pre-pass, e[f, v] = exp(z[f, v] -
+// kappa[f]) in bf16, except at v = y, which holds e[f, y] - exp(lse - kappa)
+// once the forward has lse. Then dZ[f, .] = -G exp(kappa - lse) e[f, .]: the
+// backward is two GEMMs on e with a per-row scale. flag[f] marks a row where
+// some z - kappa exceeded kFlagExponent (its stored values were clamped); the
+// backward recomputes those rows' logits instead.
+constexpr float kKappaOffset = 20.f;
+constexpr float kFlagExponent = 40.f;
 struct LogprobCache {
   __nv_bfloat16 *e;   // [rows, lde]
   int64_t lde, rows;
-  float2 *part;       // [ceil(V/256), N]
-  int *pos;           // [N]
+  int *idx;           // [N] forward row -> token
+  int *pos;           // [N] token -> forward row, or -1 (not computed)
+  int *count;         // device scalar: forward rows
+  float *kappa;       // [N] per forward row
+  uint8_t *flag;      // [N] per forward row
   size_t bytes;       // total size of the cache buffer
 };
 LogprobCache logprob_cache_view(void *base, int64_t N, int32_t V);

@@ -83,6 +83,11 @@ struct GemmParams {
   const int *m_count;
   const int *k_count;
   const int *row_idx;
+  // softmax+store: per-row shift and overflow flags (the cache's); plain
+  // stores: optional per-row scale of the accumulator (GEMM row index)
+  const float *kappa;
+  uint8_t *flag;
+  const float *row_scale;
 };
 
 struct __align__(8) SmemCtl {
@@ -135,6 +140,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     nM = (c + kTM - 1) / kTM;
   }
   if (p.k_count) nK = (*p.k_count + BK - 1) / BK;
+  // an empty contraction added to the output changes nothing: skip the grid
+  if (kEpi == kStoreF32 && p.k_count && nK == 0 && p.accumulate) return;
   const int num_tiles = nM * p.nN;
   const bool kzero = (nK == 0);  // empty contraction: the tile is all zeros
 
@@ -325,26 +332,26 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           if (have) p.zy[row] = zsel;
         }
       } else if constexpr (kEpi == kSoftmaxStore) {
-        // As kSoftmax, but the tile's maximum is taken first (one pass over
-        // TMEM), so the second pass can also store e = exp(z - max_tile) as
-        // bf16: the backward then forms p = e * exp(max_tile - lse) instead of
-        // recomputing the logits. Boxes of 128 rows x 64 columns go out through
-        // two swizzled staging buffers and TMA stores issued by one thread.
+        // As kSoftmax, in one pass over TMEM, and also storing e = exp(z -
+        // kappa) as bf16 with the row's own shift kappa (the sampled token's
+        // logit + kKappaOffset): the backward then needs no per-tile maxima.
+        // The tile's partial is (kappa, sum e). A 32-column chunk holding some
+        // z > kappa + kFlagExponent (a sampled token far below the row's
+        // maximum) flags the row, stores clamped values, and enters the
+        // partial against its own maximum instead. Boxes of 128 rows x 64
+        // columns go out through two swizzled staging buffers and TMA stores
+        // issued by one thread.
         const bool issuer = (warp == 2 && lane == 0);
         const int col0 = n * BN;
         const int yy = row_ok ? __ldg(p.y + orig) : -1;
-        float mx = -INFINITY;
-#pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
-          uint32_t u[32];
-          tmem_ld32(taddr + c * 32, u);
-          tmem_wait_ld();
-          const int valid = p.vocab - (col0 + c * 32);
-#pragma unroll
-          for (int j = 0; j < 32; ++j) mx = (j < valid) ? fmaxf(mx, __uint_as_float(u[j])) : mx;
-        }
-        const float off = -mx * kLog2e;
-        float sm = 0.f, zsel = 0.f;
+        const float kap = row_ok ? __ldg(p.kappa + row) : 0.f;
+        const float off = -kap * kLog2e;
+        // a flagged row's values are clamped to 2^64: its row of e W stays far
+        // from fp32 overflow in the backward, which scales that row by 0
+        constexpr float kClampLog2 = 64.f;
+        float sk = 0.f;                      // sum of e over the unflagged chunks
+        float bm = -INFINITY, bs = 0.f;      // flagged chunks: online (max, sum exp(z - max))
+        float zsel = 0.f;
         bool have = false;
 #pragma unroll 1
         for (int box = 0; box < BN / 64; ++box) {
@@ -364,13 +371,28 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             const int cbase = col0 + c * 32;
             const int valid = p.vocab - cbase;
             uint32_t pk[16];
+            float cs = 0.f, cm = -INFINITY;
 #pragma unroll
             for (int j = 0; j < 32; j += 2) {
-              const float e0 = (j < valid) ? ex2_approx(fmaf(__uint_as_float(u[j]), kLog2e, off)) : 0.f;
-              const float e1 = (j + 1 < valid) ? ex2_approx(fmaf(__uint_as_float(u[j + 1]), kLog2e, off)) : 0.f;
-              sm += e0 + e1;
+              const float z0 = __uint_as_float(u[j]), z1 = __uint_as_float(u[j + 1]);
+              const float e0 = (j < valid) ? ex2_approx(fminf(fmaf(z0, kLog2e, off), kClampLog2)) : 0.f;
+              const float e1 = (j + 1 < valid) ? ex2_approx(fminf(fmaf(z1, kLog2e, off), kClampLog2)) : 0.f;
+              cm = (j < valid) ? fmaxf(cm, z0) : cm;
+              cm = (j + 1 < valid) ? fmaxf(cm, z1) : cm;
+              cs += e0 + e1;
               const __nv_bfloat162 b2 = __floats2bfloat162_rn(e0, e1);
               pk[j / 2] = *reinterpret_cast<const uint32_t *>(&b2);
+            }
+            if (cm - kap > kFlagExponent) {  // rare: redo the chunk's sum against its maximum
+              float s2 = 0.f;
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                s2 += (j < valid) ? ex2_approx((__uint_as_float(u[j]) - cm) * kLog2e) : 0.f;
+              const float mn = fmaxf(bm, cm);
+              bs = fmaf(bs, ex2_approx((bm - mn) * kLog2e), s2 * ex2_approx((cm - mn) * kLog2e));
+              bm = mn;
+            } else {
+              sk += cs;
             }
             const unsigned rel = unsigned(yy - cbase);
             if (rel < 32u) {
@@ -397,7 +419,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
         }
         if (row_ok) {
-          p.part[int64_t(n) * p.rows + row] = make_float2(mx, sm);  // compacted row, stride N
+          float2 part = make_float2(kap, sk);
+          if (bm != -INFINITY) {  // a flagged chunk: merge the two partials
+            const float mn = fmaxf(kap, bm);
+            part = make_float2(mn, fmaf(sk, ex2_approx((kap - mn) * kLog2e), bs * ex2_approx((bm - mn) * kLog2e)));
+            p.flag[row] = 1;
+          }
+          p.part[int64_t(n) * p.rows + row] = part;  // compacted row, stride N
           if (have) p.zy[row] = zsel;
         }
       } else if constexpr (kEpi == kDLogits) {
@@ -467,6 +495,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const bool okj = rowj < rows;
         const int64_t origj = j == 0 ? orig : ((okj && p.row_idx) ? int64_t(__ldg(p.row_idx + rowj)) : rowj);
         const int64_t orow = p.c_row_off + origj;
+        const float rs = (p.row_scale && okj) ? __ldg(p.row_scale + rowj) : 1.f;
 #pragma unroll 1
         for (int c = 0; c < BN / 32; ++c) {
           uint32_t u[32];
@@ -475,6 +504,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           if (kzero) {
 #pragma unroll
             for (int j = 0; j < 32; ++j) u[j] = 0u;
+          }
+          if (p.row_scale) {  // a zero scale gives zeros whatever the accumulator holds
+#pragma unroll
+            for (int j = 0; j < 32; ++j) u[j] = rs == 0.f ? 0u : __float_as_uint(__uint_as_float(u[j]) * rs);
           }
           const int col = n * BN + c * 32;
           if (!okj || col >= p.cols) continue;
@@ -539,93 +572,123 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 }
 
 // ---------------------------------------------------------------------------
-// backward from the forward's stored probabilities
+// the probability cache: row shifts, the sampled token's entry, backward scales
 // ---------------------------------------------------------------------------
-// dZ[i, v - v0] = G_t (1[v == y_t] - e[f, v] exp(max[tile(v), f] - lse_t)) for
-// the compacted backward row i (token t = idx[i], forward row f = pos[t]) and
-// v in [v0, v0 + vc): one CTA per row, 16-byte loads and stores of 8 bf16.
-// Rows from the active count up to the next multiple of 128 are zeroed (the
-// GEMMs read whole 128-row tiles); a token whose forward row was skipped has
-// no stored probabilities: its row is zeroed and SAO_DEVERR_CACHE_ROW raised.
-constexpr int kDzThreads = 256;
+constexpr int kRowWarps = 8;  // rows (one per warp) per CTA of the row kernels
 
-__global__ void __launch_bounds__(kDzThreads) dz_from_cache_kernel(
-    const __nv_bfloat16 *__restrict__ e, int64_t lde, const float2 *__restrict__ part, int64_t N,
-    const int *__restrict__ pos, const int *__restrict__ idx, const int *__restrict__ count,
-    const int32_t *__restrict__ y, const float *__restrict__ lse, const float *__restrict__ G, int v0, int vc,
-    __nv_bfloat16 *__restrict__ dz, int64_t ldz, unsigned int *err) {
-  const int64_t i = blockIdx.x;
-  const int64_t cnt = *count;
-  if (i >= (cnt + BM - 1) / BM * BM) return;
-  __nv_bfloat16 *out = dz + i * ldz;
-  int f = -1;
-  int64_t t = 0;
-  if (i < cnt) {
-    t = __ldg(idx + i);
-    f = __ldg(pos + t);
-    if (f < 0 && threadIdx.x == 0) raise_device_error(err, SAO_DEVERR_CACHE_ROW);
-  }
-  if (f < 0) {
-    for (int k = threadIdx.x * 8; k < vc; k += kDzThreads * 8) {
-      if (k + 8 <= vc)
-        *reinterpret_cast<uint4 *>(out + k) = make_uint4(0u, 0u, 0u, 0u);
-      else
-        for (int j = k; j < vc; ++j) out[j] = __float2bfloat16_rn(0.f);
-    }
-    return;
-  }
-  const float g = __ldg(G + t);
-  const float l2 = __ldg(lse + t) * kLog2e;
-  const int yy = __ldg(y + t) - v0;
-  const __nv_bfloat16 *src = e + int64_t(f) * lde + v0;
-  // the 8 columns of a vector share one 256-wide tile (v0 and k are multiples of 8)
-  auto scale = [&](int k) { return g * ex2_approx(fmaf(__ldg(&part[int64_t((v0 + k) / BN) * N + f].x), kLog2e, -l2)); };
-  auto dz8 = [&](const uint4 q, float gs, int k) {
-    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
-    uint32_t o[4];
+// kappa[f] = H[t] . W[y[t]] + kKappaOffset (fp32 sums of the bf16 products) for
+// forward row f < count, A being the forward GEMM's A operand (row f is token
+// t = idx[f]); flag[f] = 0. One warp per row, 16-byte loads (h % 8 == 0).
+__global__ void __launch_bounds__(32 * kRowWarps) kappa_kernel(const __nv_bfloat16 *A, int h,
+                                                              const __nv_bfloat16 *W, const int32_t *y, int V,
+                                                              const int *idx, const int *count, float *kappa,
+                                                              uint8_t *flag) {
+  const int f = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (f >= *count) return;
+  const int yy = __ldg(y + __ldg(idx + f));
+  float acc = 0.f;
+  if (yy >= 0 && yy < V) {
+    const __nv_bfloat16 *a = A + int64_t(f) * h, *w = W + int64_t(yy) * h;
+    for (int k = lane * 8; k < h; k += 256) {
+      const uint4 av = __ldg(reinterpret_cast<const uint4 *>(a + k));
+      const uint4 wv = __ldg(reinterpret_cast<const uint4 *>(w + k));
+      const uint32_t aw[4] = {av.x, av.y, av.z, av.w}, ww[4] = {wv.x, wv.y, wv.z, wv.w};
 #pragma unroll
-    for (int h2 = 0; h2 < 4; ++h2) {
-      const float2 ev = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[h2]));
-      float d0 = -gs * ev.x, d1 = -gs * ev.y;
-      if (k + 2 * h2 == yy) d0 += g;
-      if (k + 2 * h2 + 1 == yy) d1 += g;
-      const __nv_bfloat162 b2 = __floats2bfloat162_rn(d0, d1);
-      o[h2] = *reinterpret_cast<const uint32_t *>(&b2);
-    }
-    return make_uint4(o[0], o[1], o[2], o[3]);
-  };
-  constexpr int kStep = kDzThreads * 8, kUnroll = 4;
-  int k = threadIdx.x * 8;
-  // kUnroll independent 16-byte loads in flight per thread
-  for (; k + (kUnroll - 1) * kStep + 8 <= vc; k += kUnroll * kStep) {
-    uint4 q[kUnroll];
-    float gs[kUnroll];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      q[u] = __ldcs(reinterpret_cast<const uint4 *>(src + k + u * kStep));
-      gs[u] = scale(k + u * kStep);
-    }
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u)
-      __stcs(reinterpret_cast<uint4 *>(out + k + u * kStep), dz8(q[u], gs[u], k + u * kStep));
-  }
-  for (; k < vc; k += kStep) {
-    const float gs = scale(k);
-    if (k + 8 <= vc) {
-      __stcs(reinterpret_cast<uint4 *>(out + k), dz8(__ldcs(reinterpret_cast<const uint4 *>(src + k)), gs, k));
-    } else {
-      for (int j = k; j < vc; ++j) {
-        float d = -gs * __bfloat162float(src[j]);
-        if (j == yy) d += g;
-        out[j] = __float2bfloat16_rn(d);
+      for (int q = 0; q < 4; ++q) {
+        const float2 x = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&aw[q]));
+        const float2 z = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&ww[q]));
+        acc = fmaf(x.x, z.x, acc);
+        acc = fmaf(x.y, z.y, acc);
       }
     }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  }
+  if (lane == 0) {
+    kappa[f] = acc + kKappaOffset;
+    flag[f] = 0;
   }
 }
 
-__global__ void iota_kernel(int *pos, int64_t N) {
+// Once lse is known: e[f, y] = exp(z_y - kappa) - exp(lse - kappa) =
+// -exp(z_y - kappa) expm1(-logp), for the unflagged rows with a valid token,
+// so that dZ[f, .] = -G exp(kappa - lse) e[f, .] holds at v = y as well.
+__global__ void patch_target_kernel(__nv_bfloat16 *e, int64_t lde, const int *idx, const int *count,
+                                    const int32_t *y, int V, const float *zy, const float *logp,
+                                    const float *kappa, const uint8_t *flag) {
+  const int f = blockIdx.x * blockDim.x + threadIdx.x;
+  if (f >= *count || flag[f]) return;
+  const int t = idx[f];
+  const int yy = y[t];
+  if (yy < 0 || yy >= V) return;
+  const float a = expf(zy[f] - kappa[f]);
+  e[int64_t(f) * lde + yy] = __float2bfloat16_rn(-a * expm1f(-logp[t]));
+}
+
+// Forward rows = tokens (no row was skipped).
+__global__ void cache_identity_kernel(int *idx, int *pos, int *count, int64_t N) {
   const int64_t t = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (t < N) pos[t] = int(t);
+  if (t < N) idx[t] = pos[t] = int(t);
+  if (t == 0) *count = int(N);
+}
+
+// fb[t] = 1 when grad[t] != 0 and the token's forward row is flagged (those
+// rows are recomputed); grad != 0 on a token the forward skipped raises
+// SAO_DEVERR_CACHE_ROW (it contributes nothing).
+__global__ void bwd_token_kernel(const float *G, const int *pos, const uint8_t *flag, int64_t N, uint8_t *fb,
+                                 unsigned int *err) {
+  const int64_t t = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (t >= N) return;
+  uint8_t v = 0;
+  if (G[t] != 0.f) {
+    const int f = pos[t];
+    if (f < 0)
+      raise_device_error(err, SAO_DEVERR_CACHE_ROW);
+    else
+      v = flag[f];
+  }
+  fb[t] = v;
+}
+
+// For forward row f < round_up(count, 128): sc[f] = -G[t] exp(kappa[f] -
+// lse[t]) (0 past count and on flagged rows) and Hs[f] = bf16(sc[f] H[t]),
+// the dW GEMM's B operand. One warp per row, 16-byte loads and stores.
+__global__ void __launch_bounds__(32 * kRowWarps) bwd_scale_kernel(const __nv_bfloat16 *H, int h,
+                                                                  const int *idx, const int *count,
+                                                                  const float *G, const float *lse,
+                                                                  const float *kappa, const uint8_t *flag,
+                                                                  float *sc, __nv_bfloat16 *Hs,
+                                                                  int64_t rows_cap) {
+  const int64_t f = int64_t(blockIdx.x) * kRowWarps + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  const int n = *count;
+  const int64_t pad = (int64_t(n) + BM - 1) / BM * BM;
+  if (f >= pad || f >= rows_cap) return;
+  float sf = 0.f;
+  int t = -1;
+  if (f < n) {
+    t = __ldg(idx + f);
+    if (!flag[f]) sf = -__ldg(G + t) * expf(__ldg(kappa + f) - __ldg(lse + t));
+  }
+  if (lane == 0) sc[f] = sf;
+  __nv_bfloat16 *dst = Hs + f * h;
+  for (int k = lane * 8; k < h; k += 256) {
+    uint4 o = make_uint4(0u, 0u, 0u, 0u);
+    if (sf != 0.f) {
+      const uint4 v = __ldg(reinterpret_cast<const uint4 *>(H + int64_t(t) * h + k));
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+      uint32_t r[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float2 x = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[q]));
+        const __nv_bfloat162 b2 = __floats2bfloat162_rn(sf * x.x, sf * x.y);
+        r[q] = *reinterpret_cast<const uint32_t *>(&b2);
+      }
+      o = make_uint4(r[0], r[1], r[2], r[3]);
+    }
+    *reinterpret_cast<uint4 *>(dst + k) = o;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -700,24 +763,32 @@ int vocab_chunk(int64_t N, int V) {
 
 }  // namespace
 
+// Backward workspace beyond the row compaction: the dZ chunk buffer and the
+// fp32 dH accumulator of the recompute path (which the cached path runs on
+// its flagged rows), and the cached path's row scales, scaled H rows and
+// per-token flags.
 size_t tc_ws_bytes(int64_t N, int32_t h, int32_t V) {
   const int64_t nvt = (int64_t(V) + BN - 1) / BN;
+  const int64_t cap = (N + BM - 1) / BM * BM;
   const size_t fwd = round256(sizeof(float2) * size_t(nvt) * size_t(N)) + round256(sizeof(float) * size_t(N));
   const int vc = vocab_chunk(N, V);
   size_t bwd = round256(size_t(N) * size_t(vc) * 2);
   if (vc < V) bwd += round256(size_t(N) * size_t(h) * sizeof(float));
+  bwd += round256(sizeof(float) * size_t(cap)) + round256(size_t(cap) * size_t(h) * 2) + round256(size_t(N));
   return compact_ws_bytes(N, h) + (fwd > bwd ? fwd : bwd);
 }
 
 LogprobCache logprob_cache_view(void *base, int64_t N, int32_t V) {
-  const int64_t nvt = (int64_t(V) + BN - 1) / BN;
   LogprobCache k;
   k.rows = (N + BM - 1) / BM * BM;
   k.lde = (int64_t(V) + 63) / 64 * 64;
   Carver c(base, ~size_t(0));
   k.e = c.take<__nv_bfloat16>(size_t(k.rows) * size_t(k.lde));
-  k.part = c.take<float2>(size_t(nvt) * size_t(N));
+  k.idx = c.take<int>(size_t(N));
   k.pos = c.take<int>(size_t(N));
+  k.count = c.take<int>(4);
+  k.kappa = c.take<float>(size_t(N));
+  k.flag = c.take<uint8_t>(size_t(N));
   k.bytes = c.off;
   return k;
 }
@@ -730,9 +801,10 @@ sao_status tc_fwd(const void *H, const void *W, const int32_t *y, const uint8_t 
   // Rows with row_mask == 0 are skipped: the GEMM runs on the compacted rows.
   CompactRows cr{};
   if (row_mask) SAO_TRY(compact_rows(row_mask, nullptr, N, static_cast<const __nv_bfloat16 *>(H), h, &cr, c, s));
-  float2 *part = cache ? cache->part : c.take<float2>(size_t(nvt) * size_t(N));
+  float2 *part = c.take<float2>(size_t(nvt) * size_t(N));
   float *zy = c.take<float>(size_t(N));
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the log-prob forward");
+  const void *A = row_mask ? static_cast<const void *>(cr.Hc) : H;
   CUtensorMap ma, mb;
   if (row_mask)
     SAO_TRY(make_map(&ma, cr.Hc, uint64_t(h), uint64_t(cr.cap), uint64_t(h), 64, BM));
@@ -758,36 +830,65 @@ sao_status tc_fwd(const void *H, const void *W, const int32_t *y, const uint8_t 
     p.row_idx = cr.idx;
   }
   if (cache) {
-    // also store e = exp(z - max_tile) and every token's forward row
+    // the forward rows and their tokens, then each row's shift
+    if (row_mask) {
+      SAO_CUDA_TRY(cudaMemcpyAsync(cache->idx, cr.idx, sizeof(int) * size_t(N), cudaMemcpyDeviceToDevice, s));
+      SAO_CUDA_TRY(cudaMemcpyAsync(cache->pos, cr.pos, sizeof(int) * size_t(N), cudaMemcpyDeviceToDevice, s));
+      SAO_CUDA_TRY(cudaMemcpyAsync(cache->count, cr.count, sizeof(int), cudaMemcpyDeviceToDevice, s));
+    } else {
+      int slot = launch_begin("cache_rows", s);
+      cache_identity_kernel<<<unsigned((N + 255) / 256), 256, 0, s>>>(cache->idx, cache->pos, cache->count, N);
+      SAO_TRY(launch_end(slot, s));
+    }
+    int slot = launch_begin("cache_kappa", s);
+    kappa_kernel<<<unsigned((N + kRowWarps - 1) / kRowWarps), 32 * kRowWarps, 0, s>>>(
+        static_cast<const __nv_bfloat16 *>(A), h, static_cast<const __nv_bfloat16 *>(W), y, V, cache->idx,
+        cache->count, cache->kappa, cache->flag);
+    SAO_TRY(launch_end(slot, s));
+    // also store e = exp(z - kappa)
+    p.kappa = cache->kappa;
+    p.flag = cache->flag;
     CUtensorMap me;
     SAO_TRY(make_map(&me, cache->e, uint64_t(V), uint64_t(cache->rows), uint64_t(cache->lde), 64, BM));
     SAO_TRY((launch_gemm<kSoftmaxStore, false, false>("tc_logits_lse_fwd", ma, mb, me, p, s)));
-    if (row_mask) {
-      SAO_CUDA_TRY(cudaMemcpyAsync(cache->pos, cr.pos, sizeof(int) * size_t(N), cudaMemcpyDeviceToDevice, s));
-    } else {
-      int slot = launch_begin("iota_pos", s);
-      iota_kernel<<<unsigned((N + 255) / 256), 256, 0, s>>>(cache->pos, N);
-      SAO_TRY(launch_end(slot, s));
-    }
   } else {
     SAO_TRY((launch_gemm<kSoftmax, false, false>("tc_logits_lse_fwd", ma, mb, ma, p, s)));
   }
-  return lse_merge_launch(part, nvt, zy, y, nullptr, row_mask ? cr.pos : nullptr, N, V, logp, lse, err, s);
+  SAO_TRY(lse_merge_launch(part, nvt, zy, y, nullptr, row_mask ? cr.pos : nullptr, N, V, logp, lse, err, s));
+  if (cache) {
+    int slot = launch_begin("cache_patch", s);
+    patch_target_kernel<<<unsigned((N + 255) / 256), 256, 0, s>>>(cache->e, cache->lde, cache->idx, cache->count, y,
+                                                                   V, zy, logp, cache->kappa, cache->flag);
+    SAO_TRY(launch_end(slot, s));
+  }
+  return SAO_OK;
 }
 
-sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *lse, const float *G, int64_t N,
-                  int32_t h, int32_t V, void *dH, float *dW, int accumulate, unsigned int *err, void *ws,
-                  size_t ws_bytes, const LogprobCache *cache, cudaStream_t s) {
+namespace {
+
+// The backward with the logits recomputed, on the rows with mask[t] != 0
+// (mask given) or G[t] != 0: dZ per vocabulary chunk by the dlogits GEMM, then
+// dH and dW. overwrite_dH: dH is written on every row (zeros on inactive
+// ones); otherwise only the active rows of dH are written. `names` label the
+// three GEMMs' launches for the library's timers.
+struct BwdNames {
+  const char *dlogits, *dH, *dW;
+};
+constexpr BwdNames kBwdNames{"tc_dlogits", "tc_dH_gemm", "tc_dW_gemm"};
+constexpr BwdNames kFlaggedNames{"flagged_dlogits", "flagged_dH_gemm", "flagged_dW_gemm"};
+
+sao_status bwd_recompute(const void *H, const void *W, const int32_t *y, const float *lse, const float *G,
+                         const uint8_t *mask, int64_t N, int32_t h, int32_t V, void *dH, float *dW, int accumulate,
+                         bool overwrite_dH, const BwdNames &names, unsigned int *err, Carver &c, cudaStream_t s) {
   const int Vc = vocab_chunk(N, V);
   const bool multi = Vc < V;
-  Carver c(ws, ws_bytes);
   // Rows whose incoming gradient is zero contribute nothing: compact the rest.
   CompactRows cr{};
-  SAO_TRY(compact_rows(nullptr, G, N, static_cast<const __nv_bfloat16 *>(H), h, &cr, c, s));
+  SAO_TRY(compact_rows(mask, mask ? nullptr : G, N, static_cast<const __nv_bfloat16 *>(H), h, &cr, c, s));
   __nv_bfloat16 *dz = c.take<__nv_bfloat16>(size_t(N) * size_t(Vc));
   float *dh_acc = multi ? c.take<float>(size_t(N) * size_t(h)) : nullptr;
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the log-prob backward");
-  if (!multi) SAO_CUDA_TRY(cudaMemsetAsync(dH, 0, size_t(N) * size_t(h) * 2, s));
+  if (!multi && overwrite_dH) SAO_CUDA_TRY(cudaMemsetAsync(dH, 0, size_t(N) * size_t(h) * 2, s));
 
   CUtensorMap mHc_K, mW_K, mHc_MN, mW_MN;
   SAO_TRY(make_map(&mHc_K, cr.Hc, uint64_t(h), uint64_t(cr.cap), uint64_t(h), 64, BM));
@@ -805,12 +906,7 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
     CUtensorMap mZ_K, mZ_MN;
     SAO_TRY(make_map(&mZ_K, dz, uint64_t(vc), uint64_t(N), uint64_t(Vc), 64, BM));
     SAO_TRY(make_map(&mZ_MN, dz, uint64_t(vc), uint64_t(N), uint64_t(Vc), 64, 64));
-    if (cache) {  // dZ from the stored probabilities, compacted rows
-      int slot = launch_begin("dz_from_cache", s);
-      dz_from_cache_kernel<<<unsigned(N), kDzThreads, 0, s>>>(cache->e, cache->lde, cache->part, N, cache->pos,
-                                                               cr.idx, cr.count, y, lse, G, v0, vc, dz, Vc, err);
-      SAO_TRY(launch_end(slot, s));
-    } else {  // dZ for vocabulary [v0, v0 + vc), compacted rows: recompute the logits
+    {  // dZ for vocabulary [v0, v0 + vc), compacted rows: recompute the logits
       GemmParams p{};
       p.nM = nMt;
       p.nN = (vc + BN - 1) / BN;
@@ -829,7 +925,7 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
       p.err = err;
       p.m_count = cr.count;
       p.row_idx = cr.idx;
-      SAO_TRY((launch_gemm<kDLogits, false, false>("tc_dlogits", mHc_K, mW_K, mZ_K, p, s)));
+      SAO_TRY((launch_gemm<kDLogits, false, false>(names.dlogits, mHc_K, mW_K, mZ_K, p, s)));
     }
     {  // dH (+)= dZ W[v0:v0+vc]: two 128-row tiles per CTA tile share each W stage when enough tiles remain
       GemmParams p{};
@@ -847,13 +943,13 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
       if (multi) {
         p.cf = dh_acc;  // compacted rows
         p.accumulate = first ? 0 : 1;
-        SAO_TRY((pair ? launch_gemm<kStoreF32, false, true, 2>("tc_dH_gemm", mZ_K, mW_MN, mZ_K, p, s)
-                      : launch_gemm<kStoreF32, false, true, 1>("tc_dH_gemm", mZ_K, mW_MN, mZ_K, p, s)));
+        SAO_TRY((pair ? launch_gemm<kStoreF32, false, true, 2>(names.dH, mZ_K, mW_MN, mZ_K, p, s)
+                      : launch_gemm<kStoreF32, false, true, 1>(names.dH, mZ_K, mW_MN, mZ_K, p, s)));
       } else {
         p.cb = static_cast<__nv_bfloat16 *>(dH);
         p.row_idx = cr.idx;  // scatter to the original rows
-        SAO_TRY((pair ? launch_gemm<kStoreBF16, false, true, 2>("tc_dH_gemm", mZ_K, mW_MN, mZ_K, p, s)
-                      : launch_gemm<kStoreBF16, false, true, 1>("tc_dH_gemm", mZ_K, mW_MN, mZ_K, p, s)));
+        SAO_TRY((pair ? launch_gemm<kStoreBF16, false, true, 2>(names.dH, mZ_K, mW_MN, mZ_K, p, s)
+                      : launch_gemm<kStoreBF16, false, true, 1>(names.dH, mZ_K, mW_MN, mZ_K, p, s)));
       }
     }
     {  // dW[v0:v0+vc] (+)= dZ^T H over the compacted tokens: two 128-row vocabulary tiles per CTA tile
@@ -871,13 +967,86 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
       p.accumulate = accumulate;
       p.err = err;
       p.k_count = cr.count;
-      SAO_TRY((pair ? launch_gemm<kStoreF32, true, true, 2>("tc_dW_gemm", mZ_MN, mHc_MN, mZ_MN, p, s)
-                    : launch_gemm<kStoreF32, true, true, 1>("tc_dW_gemm", mZ_MN, mHc_MN, mZ_MN, p, s)));
+      SAO_TRY((pair ? launch_gemm<kStoreF32, true, true, 2>(names.dW, mZ_MN, mHc_MN, mZ_MN, p, s)
+                    : launch_gemm<kStoreF32, true, true, 1>(names.dW, mZ_MN, mHc_MN, mZ_MN, p, s)));
     }
     if (multi && last)
-      SAO_TRY(scatter_rows_to_bf16(dh_acc, h, cr.pos, N, static_cast<__nv_bfloat16 *>(dH), s));
+      SAO_TRY(scatter_rows_to_bf16(dh_acc, h, cr.pos, N, static_cast<__nv_bfloat16 *>(dH), overwrite_dH, s));
   }
   return SAO_OK;
+}
+
+}  // namespace
+
+sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *lse, const float *G, int64_t N,
+                  int32_t h, int32_t V, void *dH, float *dW, int accumulate, unsigned int *err, void *ws,
+                  size_t ws_bytes, const LogprobCache *cache, cudaStream_t s) {
+  Carver c(ws, ws_bytes);
+  if (!cache) return bwd_recompute(H, W, y, lse, G, nullptr, N, h, V, dH, dW, accumulate, true, kBwdNames, err, c, s);
+
+  // From the stored probabilities: dZ[f, .] = sc[f] e[f, .] with sc[f] =
+  // -G exp(kappa - lse), so dH[t] = sc[f] (e W)[f] (row scale in the GEMM's
+  // epilogue) and dW = e^T (sc H) over the forward rows.
+  const int64_t cap = cache->rows;
+  float *sc = c.take<float>(size_t(cap));
+  __nv_bfloat16 *Hs = c.take<__nv_bfloat16>(size_t(cap) * size_t(h));
+  uint8_t *fb = c.take<uint8_t>(size_t(N));
+  if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the log-prob backward");
+  SAO_CUDA_TRY(cudaMemsetAsync(dH, 0, size_t(N) * size_t(h) * 2, s));
+  int slot = launch_begin("cache_scales", s);
+  bwd_token_kernel<<<unsigned((N + 255) / 256), 256, 0, s>>>(G, cache->pos, cache->flag, N, fb, err);
+  bwd_scale_kernel<<<unsigned((cap + kRowWarps - 1) / kRowWarps), 32 * kRowWarps, 0, s>>>(
+      static_cast<const __nv_bfloat16 *>(H), h, cache->idx, cache->count, G, lse, cache->kappa, cache->flag, sc, Hs,
+      cap);
+  SAO_TRY(launch_end(slot, s));
+
+  CUtensorMap mE_K, mE_MN, mW_MN, mHs_MN;
+  SAO_TRY(make_map(&mE_K, cache->e, uint64_t(V), uint64_t(cap), uint64_t(cache->lde), 64, BM));
+  SAO_TRY(make_map(&mE_MN, cache->e, uint64_t(V), uint64_t(cap), uint64_t(cache->lde), 64, 64));
+  SAO_TRY(make_map(&mW_MN, W, uint64_t(h), uint64_t(V), uint64_t(h), 64, 64));
+  SAO_TRY(make_map(&mHs_MN, Hs, uint64_t(h), uint64_t(cap), uint64_t(h), 64, 64));
+  DeviceInfo di;
+  SAO_TRY(device_info(&di));
+  const int sms = di.sm_count;
+  {  // dH[t] = sc[f] (e W)[f], scattered to the tokens: two 128-row tiles per CTA tile share each W stage
+    GemmParams p{};
+    const bool pair = pair_tiles(int((N + 2 * BM - 1) / (2 * BM)) * ((h + BN - 1) / BN), sms);
+    p.nM = pair ? int((N + 2 * BM - 1) / (2 * BM)) : int((N + BM - 1) / BM);
+    p.nN = (h + BN - 1) / BN;
+    p.nK = (V + BK - 1) / BK;
+    p.group_m = 1;
+    p.rows = N;
+    p.cols = h;
+    p.ldc = h;
+    p.err = err;
+    p.m_count = cache->count;
+    p.row_idx = cache->idx;
+    p.row_scale = sc;
+    p.cb = static_cast<__nv_bfloat16 *>(dH);
+    SAO_TRY((pair ? launch_gemm<kStoreBF16, false, true, 2>("tc_dH_gemm", mE_K, mW_MN, mE_K, p, s)
+                  : launch_gemm<kStoreBF16, false, true, 1>("tc_dH_gemm", mE_K, mW_MN, mE_K, p, s)));
+  }
+  {  // dW (+)= e^T (sc H) over the forward rows: two 128-row vocabulary tiles per CTA tile
+    GemmParams p{};
+    const bool pair = pair_tiles((V + 2 * BM - 1) / (2 * BM) * ((h + BN - 1) / BN), sms);
+    p.nM = pair ? (V + 2 * BM - 1) / (2 * BM) : (V + BM - 1) / BM;
+    p.nN = (h + BN - 1) / BN;
+    p.nK = int((N + BK - 1) / BK);
+    p.group_m = 1;
+    p.rows = V;
+    p.cols = h;
+    p.cf = dW;
+    p.ldc = h;
+    p.accumulate = accumulate;
+    p.err = err;
+    p.k_count = cache->count;
+    SAO_TRY((pair ? launch_gemm<kStoreF32, true, true, 2>("tc_dW_gemm", mE_MN, mHs_MN, mE_MN, p, s)
+                  : launch_gemm<kStoreF32, true, true, 1>("tc_dW_gemm", mE_MN, mHs_MN, mE_MN, p, s)));
+  }
+  // Flagged rows (a sampled token more than kFlagExponent - kKappaOffset nats
+  // below its row's maximum) got sc = 0 above: recompute their logits, write
+  // their dH rows and add their dW. With none, these GEMMs find no rows.
+  return bwd_recompute(H, W, y, lse, G, fb, N, h, V, dH, dW, 1, false, kFlaggedNames, err, c, s);
 }
 
 }  // namespace sao

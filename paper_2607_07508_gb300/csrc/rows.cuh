@@ -23,7 +23,9 @@ size_t compact_ws_bytes(int64_t N, int32_t h);
 sao_status compact_rows(const uint8_t *mask, const float *g, int64_t N, const __nv_bfloat16 *H, int32_t h,
                         CompactRows *out, Carver &c, cudaStream_t s);
 
+// dH[t] = bf16(acc[pos[t]]) on the active rows; inactive rows get zeros when
+// all_rows, else keep their contents.
 sao_status scatter_rows_to_bf16(const float *acc, int32_t h, const int *pos, int64_t N, __nv_bfloat16 *dH,
-                                cudaStream_t s);
+                                bool all_rows, cudaStream_t s);
 
 }  // namespace sao

@@ -1,9 +1,10 @@
 """GPU parity of the cached log-prob path (sao_token_logprobs_fwd_cached /
-_bwd_cached: the forward stores bf16 e = exp(z - tile max), the backward forms
-dZ from it instead of recomputing the logits) with the fp64 oracle, through the
-C ABI: small shapes with ragged tiles checked in full, the moe shape in the
-launch configuration bench.py times checked on sampled rows, row masks,
-vocabulary chunking, accumulation and the argument errors."""
+_bwd_cached: the forward stores bf16 e = exp(z - kappa) with one shift per row,
+the backward runs its two GEMMs on e with per-row scales instead of recomputing
+the logits) with the fp64 oracle, through the C ABI: small shapes with ragged
+tiles checked in full, the moe shape in the launch configuration bench.py
+times checked on sampled rows, row masks, vocabulary chunking, accumulation,
+rows beyond the stored range and the argument errors."""
 import numpy as np
 import pytest
 import torch
@@ -256,3 +257,44 @@ def test_cached_argument_errors():
     with pytest.raises(sao.SaoError) as e:
         sao.sao_token_logprobs_fwd_cached(Hf, Wf, y, logp, lse, big, sao.workspace(64, 64, 300, torch.float32))
     assert e.value.status == 4
+
+
+def test_cached_rows_far_below_their_maximum_are_recomputed():
+    """Rows whose sampled token's logit lies 64 nats below another logit of the
+    row exceed the stored range (e relative to the sampled token's logit):
+    the forward flags them and still returns their exact lse and log-prob,
+    and the backward recomputes their logits. One flagged row has a zero
+    gradient (nothing to recompute), one unflagged row shares its token."""
+    N, h, V = 300, 64, 1000
+    wl, H, W, y = _case(N, h, V, seed=41)
+    H, W = H.clone(), W.clone()
+    yv = wl.y.copy()
+    jstar = 7
+    far = [5, 130, 299, 200]
+    for r in far:
+        yv[r] = 11 + r
+        H[r].zero_()
+        H[r, 0] = 8.0
+        W[11 + r].zero_()
+        W[11 + r, 0] = -4.0   # z[r, y] = -32
+    W[jstar].zero_()
+    W[jstar, 0] = 4.0         # z[r, jstar] = +32: 64 nats above the sampled token
+    yv[17] = 11 + 5           # an ordinary row sampling the same token
+    y = torch.as_tensor(yv).cuda()
+    cache = sao.logprob_cache(N, V)
+    logp, lse = _fwd(H, W, y, cache)
+    G = np.random.default_rng(43).normal(size=N).astype(np.float32)
+    G[200] = 0.0
+    dH, dW = _bwd(H, W, y, lse, torch.as_tensor(G).cuda(), cache)
+    torch.cuda.synchronize()
+    want_lp, want_lse = O.token_logprobs(H.cpu(), W.cpu(), yv)
+    assert want_lp[far].max() < -60.0
+    assert np.abs(logp.cpu().numpy() - want_lp).max() <= LOGP_TOL
+    assert np.abs(lse.cpu().numpy() - want_lse).max() <= LOGP_TOL
+    want_dH, want_dW = O.token_logprobs_bwd(H.cpu(), W.cpu(), yv, want_lse, G)
+    got_dH = dH.float().cpu().numpy()
+    assert rel_l2(got_dH, want_dH) <= GRAD_TOL
+    for r in far:
+        assert rel_l2(got_dH[r], want_dH[r]) <= GRAD_TOL or (G[r] == 0 and np.all(got_dH[r] == 0))
+    assert rel_l2(dW.cpu().numpy(), want_dW) <= GRAD_TOL
+    assert np.all(np.isfinite(dW.cpu().numpy()))
