@@ -524,9 +524,11 @@ def main():
     avg_ms = dom_ms / dom_n
     fl = kernel_flops(dom_name, wl.h, wl.V, rows_fwd, rows_bwd)
     peak_t = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    cached = step.cache is not None
     if fl is not None:
         achieved = fl / (avg_ms / 1000.0) / 1e12
-        dom_rows = rows_fwd if dom_name == "tc_logits_lse_fwd" else rows_bwd
+        # the cached backward's GEMMs run over the forward rows (zero-gradient rows scaled by 0)
+        dom_rows = rows_fwd if (dom_name == "tc_logits_lse_fwd" or cached) else rows_bwd
         roofline = {"bound": "tensor", "kernel": dom_name, "achieved": achieved, "peak": peak_t,
                     "unit": "TFLOP/s", "frac": achieved / peak_t, "traffic": stored_traffic(dom_name, dom_rows, wl.name),
                     "traffic_unit": "bytes per launch (dram read + write, ncu, scaled by active rows)",
@@ -535,9 +537,8 @@ def main():
     else:
         roofline = {"bound": "hbm", "kernel": dom_name, "achieved": None, "peak": peaks.get("hbm_gbs"),
                     "unit": "GB/s", "frac": None, "traffic": None}
-    cached = step.cache is not None
     step_alg = 2.0 * wl.h * wl.V * (rows_fwd + 2 * rows_bwd)
-    step_exec = 2.0 * wl.h * wl.V * (rows_fwd + (2 if cached else 3) * rows_bwd)
+    step_exec = 2.0 * wl.h * wl.V * (3 * rows_fwd if cached else rows_fwd + 3 * rows_bwd)
     burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
     step_roof = {"algorithmic_tflops": step_alg / (ms / 1000) / 1e12,
                  "frac_of_burst_peak": step_alg / (ms / 1000) / 1e12 / burst,
@@ -546,8 +547,10 @@ def main():
                  "algorithmic_flops_per_step": f"2hV per forward row ({rows_fwd} action tokens) + 4hV per row "
                                                f"with a non-zero gradient ({rows_bwd}); 6*N*h*V = "
                                                f"{6.0 * wl.N * wl.h * wl.V:.4g} if no row were skipped",
-                 "executed_flops_per_step": ("algorithmic (the backward reads the forward's stored bf16 "
-                                             "probabilities: no logit recompute)" if cached else
+                 "executed_flops_per_step": ("2hV per forward row, three times: the backward's two GEMMs read "
+                                             "the forward's stored bf16 probabilities (no logit recompute) and "
+                                             "run over the forward rows, a zero-gradient row scaled by 0"
+                                             if cached else
                                              "algorithmic + 2hV per backward row (the logits are recomputed)"),
                  "logprob_path": "cached" if cached else "recompute",
                  "rows_forward": rows_fwd, "rows_backward": rows_bwd,

@@ -26,9 +26,9 @@ def summarize(path, only=None):
             label = {("0", "0", "0"): "tc_gemm<softmax> (logits lse fwd)",
                      ("4", "0", "0"): "tc_gemm<softmax+store> (logits lse fwd, stores bf16 e)",
                      ("1", "0", "0"): "tc_gemm<dlogits> (bwd recompute + dZ)",
-                     ("3", "0", "1"): "tc_gemm<store bf16> (dH = dZ W)",
+                     ("3", "0", "1"): "tc_gemm<store bf16> (dH = row-scaled e W, or dZ W)",
                      ("2", "0", "1"): "tc_gemm<store f32> (dH accumulate)",
-                     ("2", "1", "1"): "tc_gemm<store f32> (dW = dZ^T H)"}.get(mt.groups()[:3], short)
+                     ("2", "1", "1"): "tc_gemm<store f32> (dW = e^T (s H), or dZ^T H)"}.get(mt.groups()[:3], short)
             if mt.group(4) == "2":
                 label += ", 2 M tiles per CTA tile"
             short = label
