@@ -259,12 +259,17 @@ def test_cached_argument_errors():
     assert e.value.status == 4
 
 
-def test_cached_rows_far_below_their_maximum_are_recomputed():
+@pytest.mark.parametrize("chunked,masked", [(False, False), (True, True), (False, True)])
+def test_cached_rows_far_below_their_maximum_are_recomputed(chunked, masked):
     """Rows whose sampled token's logit lies 64 nats below another logit of the
     row exceed the stored range (e relative to the sampled token's logit):
     the forward flags them and still returns their exact lse and log-prob,
     and the backward recomputes their logits. One flagged row has a zero
-    gradient (nothing to recompute), one unflagged row shares its token."""
+    gradient (nothing to recompute), one unflagged row shares its token.
+    chunked: a small dZ budget makes the recompute run in vocabulary chunks
+    (fp32 dH accumulator, then a scatter of the flagged rows only) and dW
+    accumulates onto given contents; masked: a row mask skips some rows, so
+    forward rows and tokens are numbered differently."""
     N, h, V = 300, 64, 1000
     wl, H, W, y = _case(N, h, V, seed=41)
     H, W = H.clone(), W.clone()
@@ -281,20 +286,41 @@ def test_cached_rows_far_below_their_maximum_are_recomputed():
     W[jstar, 0] = 4.0         # z[r, jstar] = +32: 64 nats above the sampled token
     yv[17] = 11 + 5           # an ordinary row sampling the same token
     y = torch.as_tensor(yv).cuda()
-    cache = sao.logprob_cache(N, V)
-    logp, lse = _fwd(H, W, y, cache)
-    G = np.random.default_rng(43).normal(size=N).astype(np.float32)
+    rng = np.random.default_rng(43)
+    G = rng.normal(size=N).astype(np.float32)
     G[200] = 0.0
-    dH, dW = _bwd(H, W, y, lse, torch.as_tensor(G).cuda(), cache)
-    torch.cuda.synchronize()
+    mask = None
+    if masked:
+        m = (rng.random(N) < 0.7).astype(np.uint8)
+        m[far] = 1
+        m[17] = 1
+        G[m == 0] = 0.0
+        mask = torch.as_tensor(m).cuda()
+    cache = sao.logprob_cache(N, V)
+    logp, lse = _fwd(H, W, y, cache, row_mask=mask)
+    prev = torch.randn(V, h, device="cuda") if chunked else None
+    if chunked:
+        sao.sao_set_dz_budget_bytes(N * 256 * 2)     # Vc = 256 -> 4 chunks, the last ragged
+    try:
+        dH, dW = _bwd(H, W, y, lse, torch.as_tensor(G).cuda(), cache, accumulate=prev)
+        torch.cuda.synchronize()
+    finally:
+        sao.sao_set_dz_budget_bytes(24 << 30)
     want_lp, want_lse = O.token_logprobs(H.cpu(), W.cpu(), yv)
     assert want_lp[far].max() < -60.0
-    assert np.abs(logp.cpu().numpy() - want_lp).max() <= LOGP_TOL
-    assert np.abs(lse.cpu().numpy() - want_lse).max() <= LOGP_TOL
+    got_lp, got_lse = logp.cpu().numpy(), lse.cpu().numpy()
+    keep = np.ones(N, bool) if mask is None else mask.cpu().numpy() != 0
+    assert np.abs(got_lp[keep] - want_lp[keep]).max() <= LOGP_TOL
+    assert np.abs(got_lse[keep] - want_lse[keep]).max() <= LOGP_TOL
     want_dH, want_dW = O.token_logprobs_bwd(H.cpu(), W.cpu(), yv, want_lse, G)
     got_dH = dH.float().cpu().numpy()
+    got_dW = dW.cpu().numpy() - (prev.cpu().numpy() if chunked else 0.0)
     assert rel_l2(got_dH, want_dH) <= GRAD_TOL
     for r in far:
-        assert rel_l2(got_dH[r], want_dH[r]) <= GRAD_TOL or (G[r] == 0 and np.all(got_dH[r] == 0))
-    assert rel_l2(dW.cpu().numpy(), want_dW) <= GRAD_TOL
-    assert np.all(np.isfinite(dW.cpu().numpy()))
+        if G[r] == 0:
+            assert np.all(got_dH[r] == 0)
+        else:
+            assert rel_l2(got_dH[r], want_dH[r]) <= GRAD_TOL
+    assert np.all(got_dH[G == 0] == 0)
+    assert rel_l2(got_dW, want_dW) <= GRAD_TOL
+    assert np.all(np.isfinite(got_dW))
