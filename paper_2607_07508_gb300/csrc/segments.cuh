@@ -196,26 +196,40 @@ __global__ void __launch_bounds__(256) traj_broadcast_kernel(const float *a_traj
   float v = __ldg(a_traj + b);
   const bool aligned = ((reinterpret_cast<uintptr_t>(m) | reinterpret_cast<uintptr_t>(adv)) & 15u) == 0;
   // 128-token groups: lane l takes tokens 4l .. 4l+3, so each warp load reads
-  // 128 contiguous bytes and each warp store writes 512
+  // 128 contiguous bytes and each warp store writes 512; the mask words of 8
+  // groups are loaded together, so a warp waits for one load latency per
+  // 1024 tokens instead of one per group
 #pragma unroll 1
-  for (int64_t t0 = c0 + int64_t(lane) * 4; t0 < c1; t0 += 128) {
-    if (aligned && t0 + 4 <= N && t0 + 4 <= next_end) {  // all 4 tokens in trajectory b
-      const uint32_t u = __ldg(reinterpret_cast<const uint32_t *>(m + t0));
-      __stcs(reinterpret_cast<float4 *>(adv + t0), make_float4((u & 0xffu) ? v : 0.f, (u & 0xff00u) ? v : 0.f,
-                                                               (u & 0xff0000u) ? v : 0.f, (u & 0xff000000u) ? v : 0.f));
-      continue;
+  for (int64_t base = c0; base < c1; base += 8 * 128) {
+    uint32_t u[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int64_t t0 = base + j * 128 + int64_t(lane) * 4;
+      u[j] = (aligned && t0 + 4 <= c1) ? __ldg(reinterpret_cast<const uint32_t *>(m + t0)) : 0u;
     }
-    for (int k = 0; k < 4; ++k) {
-      const int64_t t = t0 + k;
-      if (t >= N) break;
-      if (t >= next_end) {
-        while (b < bhi && t >= next_end) {
-          ++b;
-          next_end = cu[b + 1];
-        }
-        v = __ldg(a_traj + b);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int64_t t0 = base + j * 128 + int64_t(lane) * 4;
+      if (t0 >= c1) break;
+      if (aligned && t0 + 4 <= c1 && t0 + 4 <= next_end) {  // all 4 tokens in trajectory b
+        const uint32_t w = u[j];
+        __stcs(reinterpret_cast<float4 *>(adv + t0), make_float4((w & 0xffu) ? v : 0.f, (w & 0xff00u) ? v : 0.f,
+                                                                 (w & 0xff0000u) ? v : 0.f,
+                                                                 (w & 0xff000000u) ? v : 0.f));
+        continue;
       }
-      adv[t] = m[t] ? v : 0.f;
+      for (int k = 0; k < 4; ++k) {
+        const int64_t t = t0 + k;
+        if (t >= c1) break;
+        if (t >= next_end) {
+          while (b < bhi && t >= next_end) {
+            ++b;
+            next_end = cu[b + 1];
+          }
+          v = __ldg(a_traj + b);
+        }
+        adv[t] = m[t] ? v : 0.f;
+      }
     }
   }
 }
