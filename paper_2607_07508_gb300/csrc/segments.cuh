@@ -99,11 +99,11 @@ __global__ void __launch_bounds__(kChunkFirstThreads) chunk_first_kernel(const i
 
 // Number of action tokens per trajectory; nact must start at zero. One warp
 // per kCountChunks consecutive chunks, 8 warps per CTA (grid:
-// action_count_grid); in each 512-token window lane l reads tokens
-// 16l .. 16l+15 (one contiguous 512-byte warp load). A 16-token vector inside
-// the lane's current trajectory is counted with 4 byte-wise popcounts; only
-// vectors that cross a trajectory end take the per-token walk, which only
-// moves forward.
+// action_count_grid). A lane's 4 tokens inside its current trajectory are
+// counted with one byte-wise popcount; only groups that cross a trajectory
+// end take the per-token walk. Each lane adds its count to a trajectory's
+// total when it leaves it, and the lanes that end in the same trajectory add
+// theirs together.
 __global__ void __launch_bounds__(256) action_count_kernel(const uint8_t *m, const int32_t *cu_g, int B, int64_t N,
                                                            int nchunks, const int *chunk_first, int *nact) {
   __shared__ int32_t s_cu_all[8][kCuCap];
@@ -123,45 +123,43 @@ __global__ void __launch_bounds__(256) action_count_kernel(const uint8_t *m, con
   int b = blo;
   int64_t next_end = cu[b + 1];
   int cnt = 0;
-  const bool aligned = (reinterpret_cast<uintptr_t>(m) & 15u) == 0;
+  const bool aligned = (reinterpret_cast<uintptr_t>(m) & 3u) == 0;
+  // 128-token groups, lane l taking tokens 4l .. 4l+3 (each warp load reads 128
+  // contiguous bytes); the mask words of 8 groups are loaded together, so a
+  // warp waits for one load latency per 1024 tokens; a lane's tokens only
+  // increase, so its walk only moves forward
 #pragma unroll 1
-  for (int64_t w0 = c0; w0 < c1; w0 += 512) {
-    const int64_t t0 = w0 + int64_t(lane) * 16;
-    if (t0 >= N) break;
-    uint32_t w[4] = {0u, 0u, 0u, 0u};
-    if (aligned && t0 + 16 <= N) {
-      const uint4 x = __ldg(reinterpret_cast<const uint4 *>(m + t0));
-      w[0] = x.x;
-      w[1] = x.y;
-      w[2] = x.z;
-      w[3] = x.w;
-    } else {
-      for (int k = 0; k < 16; ++k) {
+  for (int64_t base = c0; base < c1; base += 8 * 128) {
+    uint32_t u[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int64_t t0 = base + j * 128 + int64_t(lane) * 4;
+      u[j] = (aligned && t0 + 4 <= c1) ? __ldg(reinterpret_cast<const uint32_t *>(m + t0)) : 0u;
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int64_t t0 = base + j * 128 + int64_t(lane) * 4;
+      if (t0 >= c1) break;
+      if (aligned && t0 + 4 <= c1 && t0 + 4 <= next_end) {  // all 4 tokens in trajectory b
+        cnt += __popc(((u[j] & 0x7f7f7f7fu) + 0x7f7f7f7fu | u[j]) & 0x80808080u);
+        continue;
+      }
+      for (int k = 0; k < 4; ++k) {
         const int64_t t = t0 + k;
-        if (t < N && m[t] != 0) w[k >> 2] |= 1u << (8 * (k & 3));
-      }
-    }
-    if (t0 + 16 <= next_end) {  // all 16 tokens in trajectory b (t0 >= cu[b]: the walk is behind)
-#pragma unroll
-      for (int k = 0; k < 4; ++k) cnt += __popc(((w[k] & 0x7f7f7f7fu) + 0x7f7f7f7fu | w[k]) & 0x80808080u);
-      continue;
-    }
-#pragma unroll
-    for (int k = 0; k < 16; ++k) {
-      const int64_t t = t0 + k;
-      if (t >= N) break;
-      if (t >= next_end) {
-        const int nb0 = b;
-        while (b < bhi && t >= next_end) {
-          ++b;
-          next_end = cu[b + 1];
+        if (t >= c1) break;
+        if (t >= next_end) {
+          const int nb0 = b;
+          while (b < bhi && t >= next_end) {
+            ++b;
+            next_end = cu[b + 1];
+          }
+          if (b != nb0 && cnt) {
+            atomicAdd(nact + nb0, cnt);
+            cnt = 0;
+          }
         }
-        if (b != nb0 && cnt) {
-          atomicAdd(nact + nb0, cnt);
-          cnt = 0;
-        }
+        cnt += m[t] != 0;
       }
-      cnt += ((w[k >> 2] >> (8 * (k & 3))) & 0xffu) != 0u;
     }
   }
   const unsigned peers = __match_any_sync(0xffffffffu, b);
