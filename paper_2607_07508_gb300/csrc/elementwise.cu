@@ -59,17 +59,24 @@ __global__ void __launch_bounds__(kThreads) count_mask_kernel(const uint8_t *__r
   if (vec) {
     const int64_t n16 = N / 16;
     const uint4 *m16 = reinterpret_cast<const uint4 *>(m);
-    for (int64_t i = tid; i < n16; i += stride) {
-      uint4 q = __ldg(m16 + i);
-      // a mask byte is 0 or non-zero; count non-zero bytes
-      uint32_t w[4] = {q.x, q.y, q.z, q.w};
+    // a mask byte is 0 or non-zero; count non-zero bytes
+    auto count16 = [](const uint4 q) {
+      const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+      int n = 0;
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        uint32_t x = w[k];
-        uint32_t nz = ((x & 0x7f7f7f7fu) + 0x7f7f7f7fu | x) & 0x80808080u;
-        c += __popc(nz);
-      }
+      for (int k = 0; k < 4; ++k) n += __popc(((w[k] & 0x7f7f7f7fu) + 0x7f7f7f7fu | w[k]) & 0x80808080u);
+      return n;
+    };
+    int64_t i = tid;
+    // four independent 16-byte loads in flight per thread
+    for (; i + 3 * stride < n16; i += 4 * stride) {
+      uint4 q[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) q[u] = __ldg(m16 + i + u * stride);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) c += count16(q[u]);
     }
+    for (; i < n16; i += stride) c += count16(__ldg(m16 + i));
     done = n16 * 16;
   }
   for (int64_t i = done + tid; i < N; i += stride) c += (m[i] != 0);
