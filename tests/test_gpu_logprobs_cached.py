@@ -121,6 +121,25 @@ def test_cached_row_mask_and_skipped_rows():
         sao.sao_set_checked(False)
 
 
+def test_cached_forward_with_every_row_skipped():
+    """A row mask of zeros leaves no forward row: log-probs are 0, and a
+    backward with a zero gradient writes zeros to dH and dW, or leaves an
+    accumulated dW as it was."""
+    wl, H, W, y = _case(300, 64, 1000, seed=23)
+    mask = torch.zeros(300, dtype=torch.uint8, device="cuda")
+    cache = sao.logprob_cache(300, 1000)
+    logp, lse = _fwd(H, W, y, cache, row_mask=mask)
+    G = torch.zeros(300, device="cuda")
+    dH, dW = _bwd(H, W, y, lse, G, cache)
+    prev = torch.randn(1000, 64, device="cuda")
+    dH2, dW2 = _bwd(H, W, y, lse, G, cache, accumulate=prev)
+    torch.cuda.synchronize()
+    assert not logp.cpu().numpy().any() and not lse.cpu().numpy().any()
+    assert not dH.float().cpu().numpy().any() and not dW.cpu().numpy().any()
+    assert not dH2.float().cpu().numpy().any()
+    assert torch.equal(dW2, prev)
+
+
 def test_cached_backward_chunked_and_accumulate():
     """A small dZ budget forces several vocabulary chunks (the last one ragged,
     not a multiple of 8 columns); accumulate_dW adds to dW."""
