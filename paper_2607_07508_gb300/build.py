@@ -45,13 +45,23 @@ def _stamp(srcs) -> str:
     return h.hexdigest()
 
 
+def _code_only(text: str) -> str:
+    """The source without comments and with whitespace collapsed (the sources
+    hold no string literal with a comment marker in it)."""
+    import re
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return " ".join(text.split())
+
+
 def kernel_source_hash(names=("logprobs_tc.cu", "tc_ptx.cuh", "rows.cu", "rows.cuh")) -> str:
-    """Short hash of the sources that define the tensor-core kernels, used to
-    tell whether stored profiler counters still describe the current kernels."""
+    """Short hash of the code (comments and layout ignored) of the sources that
+    define the tensor-core kernels, used to tell whether stored profiler
+    counters still describe the current kernels."""
     h = hashlib.sha256()
     for n in names:
-        with open(os.path.join(CSRC, n), "rb") as f:
-            h.update(f.read())
+        with open(os.path.join(CSRC, n)) as f:
+            h.update(_code_only(f.read()).encode())
     return h.hexdigest()[:16]
 
 

@@ -6,10 +6,15 @@
 //
 //   forward   Z = H W^T          -> online (max, sum-exp) per row over each
 //                                   256-wide vocabulary tile + gather of z[y]
+//                                   (cached: also e = exp(z - kappa) in bf16,
+//                                   one shift kappa per row)
 //   backward  Z = H W^T (again)  -> dZ = G (1[v == y] - exp(z - lse)), bf16,
 //                                   into a [N, Vc] chunk buffer
 //             dH (+)= dZ W_chunk    (A K-major, B = W MN-major)
 //             dW_chunk = dZ^T H     (A = dZ MN-major, B = H MN-major)
+//   cached backward (dZ = s e row by row, s = -G exp(kappa - lse)):
+//             dH = s (e W)          (A = e K-major, row scale in the epilogue)
+//             dW = e^T (s H)        (A = e MN-major, B = s H MN-major)
 //
 // CTA layout (192 threads): warp 0 issues TMA loads of 128x64 A and 256x64 B
 // bf16 tiles (128-byte swizzle) into a 4-stage shared-memory ring; warp 1
