@@ -109,3 +109,13 @@ def test_cached_logprobs_argument_errors_without_gpu(lib):
     st = lib.sao_token_logprobs_bwd_cached(P(16), P(16), 0, P(16), P(16), P(16), 8, 8, 10, P(16), P(16), 0,
                                            P(256), 1 << 20, None, 0, None)
     assert st == 4
+
+
+def test_kernel_source_hash_ignores_comments_and_layout_only():
+    """The hash that keys the stored ncu traffic counters: comments and
+    whitespace do not change it, any code token does."""
+    from paper_2607_07508_gb300.build import _code_only
+    base = "int f(int x) {\n  return x + 1;  // add one\n}\n"
+    assert _code_only(base) == _code_only("/* doc */ int f(int x)\n{ return x + 1; }")
+    assert _code_only(base) != _code_only(base.replace("x + 1", "x + 2"))
+    assert _code_only("a /* multi\nline */ b // tail\nc") == "a b c"
