@@ -253,18 +253,21 @@ def cpu_baseline(wl, rows: int, H_cpu=None, W_cpu=None):
                        f"log-prob fwd + policy loss + log-prob bwd on {rows} sampled tokens over the full "
                        f"vocabulary ({t_gemm:.2f} s), extrapolated linearly to {wl.N} tokens; BLAS threads = "
                        f"host cores"),
-            "measured_s": t_on + t_gemm, "_pl": pl["loss"]}
+            "measured_s": t_on + t_gemm, "_pl": pl["loss"], "_idx": idx}
 
 
-def choose_rows(wl, H_cpu, W_cpu, budget_s=15.0):
-    from oracle import sao_oracle as O
-    r = 8
-    t0 = time.perf_counter()
-    lp, lse = O.token_logprobs(H_cpu[:r], W_cpu, wl.y[:r])
-    O.token_logprobs_bwd(H_cpu[:r], W_cpu, wl.y[:r], lse, np.ones(r))
-    dt = time.perf_counter() - t0
-    rows = int(max(8, min(512, r * budget_s / max(dt, 1e-3))))
-    return rows
+def sized_cpu_baseline(wl, H_cpu, W_cpu, budget_s=15.0, first_rows=256):
+    """The oracle on a sample sized for about `budget_s` of work: a first run
+    on `first_rows` sampled tokens; if it took less than half the budget, one
+    more run with the sample scaled to the budget (its per-call part, the fp64
+    copy of W, makes the estimate err on the short side), which is reported."""
+    cb = cpu_baseline(wl, first_rows, H_cpu, W_cpu)
+    t = cb["measured_s"]
+    if t < 0.5 * budget_s:
+        rows = int(min(4096, first_rows * budget_s / max(t, 1e-3)))
+        if rows > first_rows:
+            cb = cpu_baseline(wl, rows, H_cpu, W_cpu)
+    return cb
 
 
 # ---------------------------------------------------------------------------
@@ -283,9 +286,8 @@ def run_reference(args):
     import torch
     wl = S.make_workload(args.config, device="cpu")
     H_cpu, W_cpu = wl.H, wl.W
-    rows = max(8, choose_rows(wl, H_cpu, W_cpu, budget_s=8.0) // 2)
-    for _ in range(args.warmup if args.warmup < 1 else 1):
-        cpu_baseline(wl, 8, H_cpu, W_cpu)
+    # each step is a bounded sample: the row count a 4-second budget gives
+    rows = len(sized_cpu_baseline(wl, H_cpu, W_cpu, budget_s=4.0, first_rows=64)["_idx"])
     vals = []
     cb = None
     for _ in range(args.steps):
@@ -636,9 +638,9 @@ def main():
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         H_cpu, W_cpu = step.H.cpu(), step.W.cpu()
-        rows = choose_rows(wl, H_cpu, W_cpu)
-        cpu = cpu_baseline(wl, rows, H_cpu, W_cpu)
+        cpu = sized_cpu_baseline(wl, H_cpu, W_cpu)
         cpu.pop("_pl", None)
+        cpu.pop("_idx", None)
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
