@@ -591,6 +591,45 @@ def test_group_advantages_are_standardised():
     assert np.all(single == 0)
 
 
+def test_group_advantages_two_members_closed_form():
+    """A group {0, 1} interleaved with another in the batch, eps 0: population
+    variance 1/4, so the advantages are exactly -1 and +1 (a sample variance
+    would give -/+ 1/sqrt(2)); observation tokens get 0. A group of equal
+    rewards gets 0 once eps > 0 (with eps 0 it is 0/0: eps sits under the
+    square root for this case)."""
+    R = np.array([0.0, 3.0, 1.0, 5.0], np.float32)
+    gid = np.array([7, 9, 7, 9])
+    cu = np.array([0, 3, 5, 9, 10])
+    m = np.array([1, 0, 1, 1, 1, 0, 1, 1, 0, 1], np.uint8)
+    adv = O.group_advantages(R, gid, m, cu, 0.0)
+    want = np.array([-1, 0, -1, -1, -1, 0, 1, 1, 0, 1], np.float64)
+    assert np.array_equal(adv, want)
+    R[3] = 3.0
+    adv = O.group_advantages(R, gid, m, cu, 1e-6)
+    assert np.all(adv[3:5] == 0) and adv[9] == 0
+
+
+def test_running_mean_window_one_and_ring_wrap():
+    """Window 1: the baseline is the prompt's previous reward. Window 3 over
+    rewards 1..7 of one prompt: the baseline of reward k is the mean of the
+    (up to) three before it, across two batches, with the ring wrapping."""
+    R = np.array([2.0, 5.0, 1.0], np.float32)
+    pid = np.zeros(3, np.int64)
+    cu = np.arange(4)
+    m = np.ones(3, np.uint8)
+    adv, _, _ = O.running_mean_advantages(R, pid, m, cu, np.zeros((1, 1)), np.zeros(1, np.int64), 1)
+    assert np.allclose(adv, [2.0, 3.0, -4.0])
+    hist, seen = np.zeros((1, 3)), np.zeros(1, np.int64)
+    got = []
+    for batch in (np.arange(1, 5), np.arange(5, 8)):
+        a, hist, seen = O.running_mean_advantages(batch.astype(np.float32), np.zeros(len(batch), np.int64),
+                                                  np.ones(len(batch), np.uint8), np.arange(len(batch) + 1),
+                                                  hist, seen, 3)
+        got.extend(a)
+    want = [1.0, 2.0 - 1.0, 3.0 - 1.5, 4.0 - 2.0, 5.0 - 3.0, 6.0 - 4.0, 7.0 - 5.0]
+    assert np.allclose(got, want) and int(seen[0]) == 7
+
+
 def test_running_mean_baseline_window():
     """Window 2 for prompt 0 over rewards 1, 0, 1, 1: baselines 0 (empty), 1,
     mean(1, 0), mean(0, 1); prompt 1 keeps its own window."""
