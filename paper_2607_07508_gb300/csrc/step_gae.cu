@@ -283,15 +283,16 @@ __global__ void __launch_bounds__(kThreads) step_reduce_kernel(const float *valu
     const bool shortstep = own && end - first <= kShortStep;
     Acc2 acc;
     if (shortstep) {
-      int t = first;
-      for (; t + 4 <= end; t += 4) {
-        const float a0 = values[t], a1 = values[t + 1], a2 = values[t + 2], a3 = values[t + 3];
-        acc.add(a0);
-        acc.add(a1);
-        acc.add(a2);
-        acc.add(a3);
+      // 4 tokens at a time, the loads of a group (the ragged last one too)
+      // issued before its adds, which keep the token order
+      for (int t = first; t < end; t += 4) {
+        float x[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) x[k] = t + k < end ? values[t + k] : 0.f;
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          if (t + k < end) acc.add(x[k]);
       }
-      for (; t < end; ++t) acc.add(values[t]);
     }
     unsigned longs = __ballot_sync(0xffffffffu, own && !shortstep);
     while (longs) {
