@@ -493,6 +493,23 @@ def test_step_gae_telescopes_and_broadcasts():
     assert list(np.flatnonzero(vm_last)) == [3, 7, 9]
 
 
+def test_step_gae_steps_stop_at_trajectory_ends():
+    """Action runs that touch across a trajectory boundary are two steps, one
+    per trajectory, each with its own reward; an empty trajectory and one with
+    only observation tokens get nothing. gamma = lambda = 1: a step's
+    advantage is its trajectory's reward minus the step value."""
+    m = np.array([1, 1, 1, 1, 1, 0, 0], np.uint8)
+    v = np.array([0.2, 0.4, 0.1, 0.3, 0.5, 9.0, 9.0])
+    cu = np.array([0, 2, 2, 5, 7])                     # [0,2) | empty | [2,5) | [5,7) observations
+    R = np.array([1.0, 7.0, 0.0, 3.0])
+    a, r, vm = O.step_advantages(v, R, m, cu, 1.0, 1.0, 1.0, 0.0, O.STEP_AVERAGE)
+    assert np.allclose(a[:2], 1.0 - 0.3) and np.allclose(a[2:5], 0.0 - 0.3)
+    assert np.all(a[5:] == 0) and np.all(r[5:] == 0) and np.array_equal(vm, m)
+    a, _, vm = O.step_advantages(v, R, m, cu, 1.0, 1.0, 1.0, 0.0, O.STEP_LAST)
+    assert np.allclose(a[:2], 1.0 - 0.4) and np.allclose(a[2:5], 0.0 - 0.5)
+    assert list(np.flatnonzero(vm)) == [1, 4]
+
+
 def test_step_gae_explicit_sum_and_step_count_lambda():
     """Step advantages follow the explicit GAE sum over steps, with the
     length-adaptive lambda counted in steps (App. A.1)."""
