@@ -536,6 +536,31 @@ def test_clip_loss_no_bounds_equals_dis_without_bounds():
     assert abs(a["loss"] - b["loss"]) < 1e-12 and np.allclose(a["coef"], b["coef"], atol=1e-15)
 
 
+def test_clip_loss_clipping_is_strict_and_sign_dependent():
+    """A ratio exactly at a bound gives min(rA, clip(r)A) = rA with both terms
+    equal: not counted as clipped; one representable step outward is. A ratio
+    above 1+eps_high with A < 0 (or below 1-eps_low with A > 0) is never
+    clipped: the min takes the unclipped term."""
+    for d in (np.float32(0.25), np.float32(0.6)):
+        r = np.float32(np.exp(d))
+        eps_h = float(r - np.float32(1.0))                # exact (Sterbenz)
+        assert np.float32(1.0) + np.float32(eps_h) == r
+        assert O.clip_flags([d], [0.0], [1.0], [1], 0.5, eps_h)[0] == O.CLIP_NONE
+        d_out = np.nextafter(d, np.float32(1.0))
+        if np.float32(np.exp(d_out)) > r:
+            assert O.clip_flags([d_out], [0.0], [1.0], [1], 0.5, eps_h)[0] == O.CLIP_HIGH
+        assert O.clip_flags([d_out], [0.0], [-1.0], [1], 0.5, eps_h)[0] == O.CLIP_NONE
+    for d in (np.float32(-0.25), np.float32(-0.6)):
+        r = np.float32(np.exp(d))
+        eps_l = float(np.float32(1.0) - r)
+        assert np.float32(1.0) - np.float32(eps_l) == r
+        assert O.clip_flags([d], [0.0], [-1.0], [1], eps_l, 0.5)[0] == O.CLIP_NONE
+        d_out = np.nextafter(d, np.float32(-1.0))
+        if np.float32(np.exp(d_out)) < r:
+            assert O.clip_flags([d_out], [0.0], [-1.0], [1], eps_l, 0.5)[0] == O.CLIP_LOW
+        assert O.clip_flags([d_out], [0.0], [1.0], [1], eps_l, 0.5)[0] == O.CLIP_NONE
+
+
 def test_clip_loss_hand_example():
     """A > 0 above 1+eps_high and A < 0 below 1-eps_low are clipped (value at the
     bound, zero gradient); A > 0 below 1-eps_low and A < 0 above 1+eps_high are
