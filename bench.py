@@ -143,7 +143,7 @@ class ClockSampler:
 class LossHeadStep:
     """Device buffers and the six ABI calls of one loss-head step."""
 
-    def __init__(self, wl, device, torch, cached=True):
+    def __init__(self, wl, device, torch, cached=False):
         from paper_2607_07508_gb300 import sao
         self.sao = sao
         self.torch = torch
@@ -178,15 +178,15 @@ class LossHeadStep:
         # workload's staleness noise (prepared once, outside any timing).
         sao.sao_token_logprobs_fwd(self.H, self.W, self.y, self.logp, self.lse, self.ws)
         self.old = (self.logp + torch.as_tensor(wl.xi).to(dev)).contiguous()
-        # The forward keeps its probabilities (bf16, about 2*N*V bytes) for the
-        # backward when they fit next to everything else; else the backward
-        # recomputes the logits.
+        # The default path is vocabulary-chunked with the logits recomputed in
+        # the backward: no [N, V] buffer of any dtype exists. Only on request
+        # (cached=True) does the forward keep its bf16 probabilities (about
+        # 2*N*V bytes) for the backward.
         self.cache = None
-        if cached and self.H.dtype == torch.bfloat16:
-            need = sao.sao_logprob_cache_bytes(N, V)
-            free, _ = torch.cuda.mem_get_info(dev)
-            if need + (4 << 30) < free:
-                self.cache = sao.logprob_cache(N, V, device=dev)
+        if cached:
+            if self.H.dtype != torch.bfloat16:
+                raise ValueError("the probability cache is for bf16 workloads only")
+            self.cache = sao.logprob_cache(N, V, device=dev)
 
     def run(self):
         s, wl = self.sao, self.wl
@@ -224,15 +224,28 @@ def kernel_flops(name, h, V, rows_fwd, rows_bwd):
 # ---------------------------------------------------------------------------
 # CPU baseline: the fp64 oracle on a bounded sample of the same workload
 # ---------------------------------------------------------------------------
-def cpu_baseline(wl, rows: int, H_cpu=None, W_cpu=None):
+POOL_ROWS = 4096
+
+
+def sample_pool(wl, H_cpu):
+    """A seeded pool of up to POOL_ROWS token rows (random order) and their
+    hidden states: every CPU-baseline sample is a prefix of it."""
+    rng = np.random.default_rng(0)
+    pool = rng.choice(wl.N, size=min(POOL_ROWS, wl.N), replace=False)
+    import torch
+    return pool, H_cpu[torch.as_tensor(pool)]
+
+
+def cpu_baseline(wl, rows: int, pool, H_pool, W_cpu, threads_note: str):
     """Times the oracle on `rows` sampled tokens (all three GEMMs over the full
     vocabulary) and on all N tokens for the O(N) parts; returns tokens/s
     extrapolated to the N-token step."""
     from oracle import sao_oracle as O
-    rng = np.random.default_rng(0)
-    idx = np.sort(rng.choice(wl.N, size=rows, replace=False))
-    Hs = (H_cpu if H_cpu is not None else wl.H.cpu())[idx]
-    Wc = W_cpu if W_cpu is not None else wl.W.cpu()
+    rows = min(rows, len(pool))
+    order = np.argsort(pool[:rows])
+    idx = pool[:rows][order]
+    import torch
+    Hs = H_pool[:rows][torch.as_tensor(order)]
     ys = wl.y[idx]
     t0 = time.perf_counter()
     adv, ret = O.advantages(wl.values, wl.rewards, wl.loss_mask, wl.cu_seqlens, wl.gamma, wl.lam, wl.lam_critic,
@@ -240,34 +253,94 @@ def cpu_baseline(wl, rows: int, H_cpu=None, W_cpu=None):
     O.value_loss(wl.values, ret, wl.loss_mask)
     t_on = time.perf_counter() - t0
     t1 = time.perf_counter()
-    logp, lse = O.token_logprobs(Hs, Wc, ys)
+    logp, lse = O.token_logprobs(Hs, W_cpu, ys)
     old = logp + wl.xi[idx]
-    pl = O.policy_loss(logp, old, adv[idx], wl.loss_mask[idx], wl.eps_low, wl.eps_high)
+    O.policy_loss(logp, old, adv[idx], wl.loss_mask[idx], wl.eps_low, wl.eps_high)
     G = O.policy_loss_bwd(logp, old, adv[idx], wl.loss_mask[idx], wl.eps_low, wl.eps_high, 0, 1.0)
-    O.token_logprobs_bwd(Hs, Wc, ys, lse, G)
+    O.token_logprobs_bwd(Hs, W_cpu, ys, lse, G)
     t_gemm = time.perf_counter() - t1
     t_step = t_on + t_gemm * (wl.N / rows)
-    cores = os.cpu_count() or 1
-    return {"value": wl.N / t_step, "unit": UNIT, "cores": cores, "kind": "oracle",
+    return {"value": wl.N / t_step, "unit": UNIT, "kind": "oracle",
             "sample": (f"fp64 numpy oracle: advantages + value loss on all {wl.N} tokens ({t_on:.2f} s), "
                        f"log-prob fwd + policy loss + log-prob bwd on {rows} sampled tokens over the full "
-                       f"vocabulary ({t_gemm:.2f} s), extrapolated linearly to {wl.N} tokens; BLAS threads = "
-                       f"host cores"),
-            "measured_s": t_on + t_gemm, "_pl": pl["loss"], "_idx": idx}
+                       f"vocabulary ({t_gemm:.2f} s), extrapolated linearly to {wl.N} tokens; {threads_note}"),
+            "measured_s": t_on + t_gemm, "rows": rows, "t_on": t_on, "t_gemm": t_gemm, "threads_note": threads_note}
 
 
-def sized_cpu_baseline(wl, H_cpu, W_cpu, budget_s=15.0, first_rows=256):
-    """The oracle on a sample sized for about `budget_s` of work: a first run
-    on `first_rows` sampled tokens; if it took less than half the budget, one
-    more run with the sample scaled to the budget (its per-call part, the fp64
-    copy of W, makes the estimate err on the short side), which is reported."""
-    cb = cpu_baseline(wl, first_rows, H_cpu, W_cpu)
-    t = cb["measured_s"]
-    if t < 0.5 * budget_s:
-        rows = int(min(4096, first_rows * budget_s / max(t, 1e-3)))
-        if rows > first_rows:
-            cb = cpu_baseline(wl, rows, H_cpu, W_cpu)
-    return cb
+def two_point(wl, a, b):
+    """Whole-step tokens/s from two sample sizes: the GEMM part's time as a
+    fixed part (the oracle's per-call fp64 copy of W) plus a per-row part, fit
+    through both samples, then extrapolated to all N rows."""
+    per_row = (b["t_gemm"] - a["t_gemm"]) / (b["rows"] - a["rows"])
+    if per_row <= 0:
+        return b
+    fixed = max(0.0, a["t_gemm"] - per_row * a["rows"])
+    t_step = b["t_on"] + fixed + per_row * wl.N
+    out = dict(b)
+    out["value"] = wl.N / t_step
+    out["sample"] = (f"fp64 numpy oracle: advantages + value loss on all {wl.N} tokens ({b['t_on']:.2f} s), "
+                     f"log-prob fwd + policy loss + log-prob bwd on {a['rows']} and {b['rows']} sampled tokens "
+                     f"over the full vocabulary ({a['t_gemm']:.2f} s, {b['t_gemm']:.2f} s), fit as {fixed:.2f} s "
+                     f"per call + {1e3 * per_row:.2f} ms per token and extrapolated to {wl.N} tokens; "
+                     f"{b['threads_note']}")
+    return out
+
+
+def sized_cpu_baseline(wl, pool, H_pool, W_cpu, threads_note, budget_s=15.0, first_rows=64):
+    """The oracle on samples of 4x more tokens each time until one takes at
+    least 40 % of `budget_s` (or the pool is used up); the last two samples
+    give the fixed and per-token parts of the time (two_point)."""
+    prev, cur = None, cpu_baseline(wl, first_rows, pool, H_pool, W_cpu, threads_note)
+    while cur["measured_s"] < 0.4 * budget_s and cur["rows"] < len(pool):
+        prev, cur = cur, cpu_baseline(wl, min(len(pool), 4 * cur["rows"]), pool, H_pool, W_cpu, threads_note)
+    return two_point(wl, prev, cur) if prev is not None else cur
+
+
+def cpu_baseline_child(args):
+    """--cpu-baseline-child FILE: the oracle on the sample the parent saved,
+    in a process whose BLAS thread count the parent fixed through the
+    environment before numpy loaded; prints one JSON object."""
+    import torch
+    from paper_2607_07508_gb300 import synthetic as S
+    d = torch.load(args.cpu_baseline_child)
+    wl = S.make_workload(d["config"], dense=False, seed=d["seed"], N_override=d["N_override"])
+    note = f"BLAS threads = {d['threads']} (OPENBLAS/OMP/MKL_NUM_THREADS)"
+    cb = sized_cpu_baseline(wl, d["pool"].numpy(), d["H_pool"], d["W"], note, budget_s=d["budget_s"], first_rows=8)
+    print(json.dumps({k: cb[k] for k in ("value", "unit", "kind", "sample", "rows")}))
+    return 0
+
+
+def cpu_baselines(wl, H_cpu, W_cpu, config, seed, N_override, budget_s=12.0):
+    """The oracle timed on the host cores twice: with numpy's BLAS on every
+    core (in this process) and on one thread (a child process started with
+    the BLAS thread count fixed, since it cannot change once numpy is
+    loaded). Reported: all-cores value as `value`, both figures by name."""
+    import tempfile
+    import torch
+    pool, H_pool = sample_pool(wl, H_cpu)
+    cores = os.cpu_count() or 1
+    allc = sized_cpu_baseline(wl, pool, H_pool, W_cpu, f"BLAS threads = host cores ({cores})", budget_s=budget_s)
+    one = None
+    fd, path = tempfile.mkstemp(suffix=".pt", prefix="sao_cpu_baseline_")
+    os.close(fd)
+    try:
+        torch.save({"config": config, "seed": seed, "N_override": N_override, "pool": torch.as_tensor(pool),
+                    "H_pool": H_pool,
+                    "W": W_cpu, "threads": 1, "budget_s": budget_s}, path)
+        env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1")
+        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--cpu-baseline-child", path], env=env,
+                           capture_output=True, text=True, timeout=600)
+        if r.returncode == 0 and r.stdout.strip():
+            one = json.loads(r.stdout.strip().splitlines()[-1])
+    except (subprocess.TimeoutExpired, OSError, ValueError):
+        one = None
+    finally:
+        os.unlink(path)
+    out = {"value": allc["value"], "unit": UNIT, "cores": cores, "kind": "oracle", "sample": allc["sample"],
+           "sample_rows": allc["rows"],
+           "value_all_cores": allc["value"], "cores_all": cores,
+           "value_1thread": one["value"] if one else None, "sample_1thread": one["sample"] if one else None}
+    return out
 
 
 # ---------------------------------------------------------------------------
@@ -283,35 +356,48 @@ def run_reference(args):
     if rank != 0:
         return 0
     from paper_2607_07508_gb300 import synthetic as S
-    import torch
     wl = S.make_workload(args.config, device="cpu")
     H_cpu, W_cpu = wl.H, wl.W
+    pool, H_pool = sample_pool(wl, H_cpu)
+    cores = os.cpu_count() or 1
+    note = f"BLAS threads = host cores ({cores})"
     # each step is a bounded sample: the row count a 4-second budget gives
-    rows = len(sized_cpu_baseline(wl, H_cpu, W_cpu, budget_s=4.0, first_rows=64)["_idx"])
-    vals = []
+    rows = sized_cpu_baseline(wl, pool, H_pool, W_cpu, note, budget_s=4.0, first_rows=16)["rows"]
+    vals, walls = [], []
     cb = None
     for _ in range(args.steps):
-        cb = cpu_baseline(wl, rows, H_cpu, W_cpu)
+        cb = cpu_baseline(wl, rows, pool, H_pool, W_cpu, note)
         vals.append(cb["value"])
+        walls.append(cb["measured_s"])
     value = statistics.median(vals)
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * wl.N / value,
+            "steps": args.steps, "warmup": args.warmup,
+            # the time each bounded sample step took; `value` extrapolates it to the whole batch
+            "ms_per_step": 1000.0 * statistics.median(walls),
+            "ms_per_step_is": f"wall time of one bounded sample step ({rows} sampled tokens for the GEMMs, all "
+                              f"{wl.N} for the O(N) parts)",
+            "ms_per_step_extrapolated": 1000.0 * wl.N / value,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "config": workload_config(wl),
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cb["cores"], "kind": "oracle",
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": cb["sample"]},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
     return 0
 
 
-def workload_config(wl):
+def workload_config(wl, cached=False):
     if wl.name == "moe":
         what = (f"moe: MoE-policy head, {wl.N} packed tokens in {wl.B} single-rollout agentic trajectories "
                 f"(lognormal lengths, median 4k, max 32k), 25% observation tokens")
     else:
         what = f"{wl.name}: {wl.N} packed tokens in {wl.B} trajectories; {wl.recipe}"
-    return {"workload": what,
+    if cached:
+        what += ("; VARIANT: the forward stores bf16 probabilities of every computed row over the whole "
+                 "vocabulary (2*N*V bytes) for the backward")
+    else:
+        what += "; log-probs vocabulary-chunked, logits recomputed in the backward (no [N, V] buffer)"
+    return {"workload": what, "logprob_path": "cached" if cached else "recompute",
             "tokens": wl.N, "trajectories": wl.B, "hidden": wl.h, "vocab": wl.V, "dtype": wl.dtype,
             "gamma": wl.gamma, "lambda": wl.lam, "eps_low": wl.eps_low, "eps_high": wl.eps_high,
             "l2": (f"inputs larger than L2 (H {wl.N * wl.h * 2 / 1e6:.0f} MB + W {wl.V * wl.h * 2 / 1e6:.0f} MB per step, "
@@ -454,11 +540,18 @@ def main():
                     help="override the packed token count (smaller cases for profiling captures)")
     ap.add_argument("--config", default=WORKLOAD, choices=["tiny", "small", "moe", "long", "large"],
                     help="workload (the metric is quoted on moe; the others are the parity configurations)")
-    ap.add_argument("--recompute", action="store_true",
-                    help="backward recomputes the logits instead of reading the forward's stored probabilities")
+    ap.add_argument("--cached", action="store_true",
+                    help="time the variant whose forward stores bf16 probabilities for all computed rows "
+                         "(2*N*V bytes) instead of the default vocabulary-chunked recompute path")
+    ap.add_argument("--recompute", action="store_true", help="the default path (kept for older command lines)")
+    ap.add_argument("--dz-budget-gib", type=float, default=None,
+                    help="bound on the backward's bf16 dZ buffer (default: the library's, 4 GiB)")
+    ap.add_argument("--cpu-baseline-child", default=None, help=argparse.SUPPRESS)
     ap.add_argument("--bandwidth-study", action="store_true",
                     help="time the O(N) kernels alone on the 2^27-token bandwidth workload")
     args = ap.parse_args()
+    if args.cpu_baseline_child:
+        return cpu_baseline_child(args)
     if args.impl == "reference":
         return run_reference(args)
     if args.bandwidth_study:
@@ -475,10 +568,12 @@ def main():
         dist.init_process_group("nccl", device_id=dev)
     sao.load()
     peaks, peak_src = load_peaks()
+    if args.dz_budget_gib is not None:
+        sao.sao_set_dz_budget_bytes(int(args.dz_budget_gib * (1 << 30)))
 
-    wl = S.make_workload(args.config, device=dev, seed=S.SEED_BASE + S.CONFIG_NAMES.index(args.config) + 97 * rank,
-                         N_override=args.tokens)
-    step = LossHeadStep(wl, dev, torch, cached=not args.recompute)
+    seed = S.SEED_BASE + S.CONFIG_NAMES.index(args.config) + 97 * rank
+    wl = S.make_workload(args.config, device=dev, seed=seed, N_override=args.tokens)
+    step = LossHeadStep(wl, dev, torch, cached=args.cached)
     stream = torch.cuda.current_stream()
     for _ in range(max(3, args.warmup)):
         step.run()
@@ -525,27 +620,37 @@ def main():
     dom_name, (dom_n, dom_ms) = dom
     avg_ms = dom_ms / dom_n
     fl = kernel_flops(dom_name, wl.h, wl.V, rows_fwd, rows_bwd)
-    peak_t = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+    sustained = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    peak_mhz = (peaks.get("clocks_under_load") or {}).get("sm_mhz_median")
+    bench_mhz = clk.get("sm_mhz")
     cached = step.cache is not None
     if fl is not None:
         achieved = fl / (avg_ms / 1000.0) / 1e12
         # the cached backward's GEMMs run over the forward rows (zero-gradient rows scaled by 0)
         dom_rows = rows_fwd if (dom_name == "tc_logits_lse_fwd" or cached) else rows_bwd
-        roofline = {"bound": "tensor", "kernel": dom_name, "achieved": achieved, "peak": peak_t,
-                    "unit": "TFLOP/s", "frac": achieved / peak_t, "traffic": stored_traffic(dom_name, dom_rows, wl.name),
+        roofline = {"bound": "tensor", "kernel": dom_name, "achieved": achieved, "peak": burst,
+                    "unit": "TFLOP/s", "frac": achieved / burst,
+                    "traffic": stored_traffic(dom_name, dom_rows, wl.name),
                     "traffic_unit": "bytes per launch (dram read + write, ncu, scaled by active rows)",
                     "algorithmic_per_launch": f"2*rows*h*V = {fl:.4g} flop", "avg_launch_ms": avg_ms,
-                    "peak_source": f"{peak_src} bf16_tflops_sustained (kernel timed inside a long step)"}
+                    "peak_source": f"{peak_src} bf16_tflops (burst)",
+                    "frac_of_sustained_peak": achieved / sustained}
     else:
         roofline = {"bound": "hbm", "kernel": dom_name, "achieved": None, "peak": peaks.get("hbm_gbs"),
                     "unit": "GB/s", "frac": None, "traffic": None}
     step_alg = 2.0 * wl.h * wl.V * (rows_fwd + 2 * rows_bwd)
     step_exec = 2.0 * wl.h * wl.V * (3 * rows_fwd if cached else rows_fwd + 3 * rows_bwd)
-    burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
-    step_roof = {"algorithmic_tflops": step_alg / (ms / 1000) / 1e12,
-                 "frac_of_burst_peak": step_alg / (ms / 1000) / 1e12 / burst,
-                 "executed_tflops": step_exec / (ms / 1000) / 1e12,
-                 "executed_frac_of_sustained_peak": step_exec / (ms / 1000) / 1e12 / peak_t,
+    alg_t = step_alg / (ms / 1000) / 1e12
+    exe_t = step_exec / (ms / 1000) / 1e12
+    step_roof = {"algorithmic_tflops": alg_t,
+                 "frac_of_burst_peak": alg_t / burst,
+                 "executed_tflops": exe_t,
+                 "executed_frac_of_burst_peak": exe_t / burst,
+                 # the sustained peak was taken at its own clocks: compare flops per SM clock
+                 "executed_frac_of_sustained_peak_per_clock": (
+                     (exe_t / bench_mhz) / (sustained / peak_mhz) if bench_mhz and peak_mhz else None),
+                 "clocks_mhz": {"this_step_median": bench_mhz, "sustained_peak_run_median": peak_mhz},
                  "algorithmic_flops_per_step": f"2hV per forward row ({rows_fwd} action tokens) + 4hV per row "
                                                f"with a non-zero gradient ({rows_bwd}); 6*N*h*V = "
                                                f"{6.0 * wl.N * wl.h * wl.V:.4g} if no row were skipped",
@@ -555,6 +660,10 @@ def main():
                                              if cached else
                                              "algorithmic + 2hV per backward row (the logits are recomputed)"),
                  "logprob_path": "cached" if cached else "recompute",
+                 "largest_logit_buffer": (f"[{rows_fwd}, {wl.V}] bf16 probabilities ({2.0 * rows_fwd * wl.V / 1e9:.1f} GB)"
+                                          if cached else
+                                          f"bf16 dZ of one row block x vocabulary chunk, at most "
+                                          f"{sao.sao_get_dz_budget_bytes() / 2**30:.2f} GiB"),
                  "rows_forward": rows_fwd, "rows_backward": rows_bwd,
                  "peak_source": peak_src}
     kernels = {k: {"launches": n, "avg_ms": t / n} for k, (n, t) in sorted(prof.items(), key=lambda kv: -kv[1][1])}
@@ -637,15 +746,13 @@ def main():
     # ---- CPU baseline (rank 0, single GPU only) ---------------------------------
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        H_cpu, W_cpu = step.H.cpu(), step.W.cpu()
-        cpu = sized_cpu_baseline(wl, H_cpu, W_cpu)
-        cpu.pop("_pl", None)
-        cpu.pop("_idx", None)
+        cpu = cpu_baselines(wl, step.H.cpu(), step.W.cpu(), args.config, seed, args.tokens)
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
                 "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
-                "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": workload_config(wl),
+                "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+                "config": workload_config(wl, cached=step.cache is not None),
                 "roofline": roofline, "step_roofline": step_roof, "cpu_baseline": cpu, "e2e": e2e,
                 "clocks": clk, "gpu_launches": launches * 1, "gpu_launches_per_step": launches / args.steps,
                 "kernels": kernels}

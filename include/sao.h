@@ -93,10 +93,16 @@ SAO_API const char *sao_last_error_string(void);
 SAO_API void sao_set_checked(int on);
 SAO_API int sao_get_checked(void);
 
-/* Upper bound on the bf16 dZ chunk buffer of sao_token_logprobs_bwd
- * (default 24 GiB). Smaller budgets split the vocabulary into more chunks and
- * add an fp32 dH accumulator. Affects sao_workspace_bytes. Process-wide. */
+/* Upper bound on the bf16 dZ buffer of sao_token_logprobs_bwd (default
+ * 4 GiB, at least 1 MiB). The backward never holds dZ for all N x V logits:
+ * it works on blocks of rows times chunks of the vocabulary whose bf16 dZ fits
+ * the budget (one block and one chunk when N x V does), choosing the split
+ * with the least extra traffic (an fp32 dH accumulator read and written once
+ * per extra vocabulary chunk; dW added to once per extra row block). Affects
+ * sao_workspace_bytes. Process-wide. */
 SAO_API void sao_set_dz_budget_bytes(size_t bytes);
+/* The current bound (bytes) set by sao_set_dz_budget_bytes or the default. */
+SAO_API size_t sao_get_dz_budget_bytes(void);
 
 /*
  * Test hooks of the advantage scan (process-wide; defaults restored by
@@ -212,7 +218,9 @@ SAO_API sao_status sao_advantages(const float *values, const float *rewards, con
  * Every token of step i receives adv = A_i and ret = GAE(lambda_critic)_i +
  * V(S_i); other tokens get 0. value_mask (nullable, [N] uint8) marks the
  * tokens the value loss keeps: all step tokens (SAO_STEP_AVERAGE) or the last
- * token of each step (SAO_STEP_LAST). Per-step arithmetic is fp64.
+ * token of each step (SAO_STEP_LAST). Per-step sums are compensated fp32
+ * pairs and the step recursion runs in double-float (about 48 bits each; the
+ * fp64 pipe is not used), then each result is rounded once to fp32.
  * Arguments otherwise as sao_advantages; workspace from sao_workspace_bytes.
  */
 SAO_API sao_status sao_step_advantages(const float *values, const float *rewards, const uint8_t *loss_mask,
@@ -254,7 +262,8 @@ SAO_API sao_status sao_clip_loss_bwd(const float *logp, const float *old_logp, c
 /*
  * GRPO's group-normalised advantage (Preliminaries): for trajectory b in
  * group g = group_ids[b], A_b = (R_b - mean_g R) / sqrt(var_g R + eps_stab)
- * (population variance over the group's trajectories, fp64), broadcast to b's
+ * (population variance over the group's trajectories: sums in compensated
+ * fp32, about 48 bits, the final moments in fp64), broadcast to b's
  * action tokens; every other token gets 0. Cost O(B^2 / SMs) for the group
  * statistics (deterministic), then O(N).
  */

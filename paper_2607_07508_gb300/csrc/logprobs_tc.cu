@@ -757,30 +757,67 @@ sao_status launch_gemm(const char *name, const CUtensorMap &ma, const CUtensorMa
 // (at 8k tokens dH has 176 paired tiles on 152 SMs and runs 15 % slower).
 bool pair_tiles(int64_t paired_tiles, int sms) { return paired_tiles >= 4 * int64_t(sms); }
 
-int vocab_chunk(int64_t N, int V) {
+// Rows per block (a multiple of 128, or N) and vocabulary columns per chunk (a
+// multiple of 256, or V rounded up to 256) of the recompute backward.
+struct BwdPlan {
+  int64_t rows;
+  int vc;
+};
+
+// The recompute backward holds dZ for one block of rows and one chunk of the
+// vocabulary at a time, at most dz_budget() bytes of bf16 whatever N and V.
+// Several vocabulary chunks add an fp32 dH accumulator that the dH GEMM reads
+// and writes once per extra chunk; several row blocks make the dW GEMM add
+// into dW once per extra block. The plan takes the split with the least of
+// that extra traffic (plus a fixed cost per block and chunk for the launches
+// and the partial last wave).
+BwdPlan bwd_plan(int64_t N, int32_t h, int32_t V) {
   const int64_t vpad = (int64_t(V) + BN - 1) / BN * BN;
-  int64_t vc = int64_t(dz_budget() / (size_t(N > 0 ? N : 1) * 2));
-  vc = vc / BN * BN;
-  if (vc < BN) vc = BN;
-  if (vc > vpad) vc = vpad;
-  return int(vc);
+  const double budget = double(dz_budget());
+  BwdPlan best{N > 0 ? N : 1, int(vpad)};
+  if (N <= 0 || double(N) * double(vpad) * 2.0 <= budget) return best;
+  double best_cost = -1.0;
+  const int64_t max_blocks = (N + BM - 1) / BM;
+  for (int64_t nb = 1; nb <= max_blocks && nb <= 4096; ++nb) {
+    int64_t rows = (N + nb - 1) / nb;
+    rows = (rows + BM - 1) / BM * BM;
+    if (rows > N) rows = N;
+    const int64_t blocks = (N + rows - 1) / rows;
+    if (blocks != nb) continue;  // the same split as a smaller nb
+    int64_t vc = int64_t(budget / (2.0 * double(rows))) / BN * BN;
+    if (vc < BN) vc = BN;
+    if (vc > vpad) vc = vpad;
+    const int64_t chunks = (V + vc - 1) / vc;
+    const double nh = double(N) * double(h), vh = double(V) * double(h);
+    double cost = double(chunks - 1) * nh * 8.0 + (chunks > 1 ? nh * 6.0 : 0.0) + double(blocks - 1) * vh * 8.0 +
+                  double(blocks * chunks) * double(256 << 20);
+    if (best_cost < 0.0 || cost < best_cost) {
+      best_cost = cost;
+      best = BwdPlan{rows, int(vc)};
+    }
+  }
+  return best;
 }
 
 }  // namespace
 
-// Backward workspace beyond the row compaction: the dZ chunk buffer and the
-// fp32 dH accumulator of the recompute path (which the cached path runs on
-// its flagged rows), and the cached path's row scales, scaled H rows and
-// per-token flags.
+// Workspace of the log-prob calls: the forward's row compaction, tile
+// partials and gathered logits; the backward's row compaction of one row
+// block, its dZ chunk buffer and fp32 dH accumulator (recompute path; the
+// cached path runs it on its flagged rows), after the cached path's row
+// scales, scaled H rows and per-token flags.
 size_t tc_ws_bytes(int64_t N, int32_t h, int32_t V) {
   const int64_t nvt = (int64_t(V) + BN - 1) / BN;
   const int64_t cap = (N + BM - 1) / BM * BM;
-  const size_t fwd = round256(sizeof(float2) * size_t(nvt) * size_t(N)) + round256(sizeof(float) * size_t(N));
-  const int vc = vocab_chunk(N, V);
-  size_t bwd = round256(size_t(N) * size_t(vc) * 2);
-  if (vc < V) bwd += round256(size_t(N) * size_t(h) * sizeof(float));
-  bwd += round256(sizeof(float) * size_t(cap)) + round256(size_t(cap) * size_t(h) * 2) + round256(size_t(N));
-  return compact_ws_bytes(N, h) + (fwd > bwd ? fwd : bwd);
+  const size_t fwd = compact_ws_bytes(N, h) + round256(sizeof(float2) * size_t(nvt) * size_t(N)) +
+                     round256(sizeof(float) * size_t(N));
+  const BwdPlan pl = bwd_plan(N, h, V);
+  size_t rec = compact_ws_bytes(pl.rows, h) + round256(size_t(pl.rows) * size_t(pl.vc) * 2);
+  if (pl.vc < V) rec += round256(size_t(pl.rows) * size_t(h) * sizeof(float));
+  const size_t cached = round256(sizeof(float) * size_t(cap)) + round256(size_t(cap) * size_t(h) * 2) +
+                        round256(size_t(N));
+  const size_t bwd = cached + rec;
+  return fwd > bwd ? fwd : bwd;
 }
 
 LogprobCache logprob_cache_view(void *base, int64_t N, int32_t V) {
@@ -882,10 +919,10 @@ struct BwdNames {
 constexpr BwdNames kBwdNames{"tc_dlogits", "tc_dH_gemm", "tc_dW_gemm"};
 constexpr BwdNames kFlaggedNames{"flagged_dlogits", "flagged_dH_gemm", "flagged_dW_gemm"};
 
-sao_status bwd_recompute(const void *H, const void *W, const int32_t *y, const float *lse, const float *G,
-                         const uint8_t *mask, int64_t N, int32_t h, int32_t V, void *dH, float *dW, int accumulate,
-                         bool overwrite_dH, const BwdNames &names, unsigned int *err, Carver &c, cudaStream_t s) {
-  const int Vc = vocab_chunk(N, V);
+sao_status bwd_recompute_block(const void *H, const void *W, const int32_t *y, const float *lse, const float *G,
+                               const uint8_t *mask, int64_t N, int32_t h, int32_t V, int Vc, void *dH, float *dW,
+                               int accumulate, bool overwrite_dH, const BwdNames &names, unsigned int *err, Carver &c,
+                               cudaStream_t s) {
   const bool multi = Vc < V;
   // Rows whose incoming gradient is zero contribute nothing: compact the rest.
   CompactRows cr{};
@@ -976,7 +1013,27 @@ sao_status bwd_recompute(const void *H, const void *W, const int32_t *y, const f
                     : launch_gemm<kStoreF32, true, true, 1>(names.dW, mZ_MN, mHc_MN, mZ_MN, p, s)));
     }
     if (multi && last)
-      SAO_TRY(scatter_rows_to_bf16(dh_acc, h, cr.pos, N, static_cast<__nv_bfloat16 *>(dH), overwrite_dH, s));
+      SAO_TRY(scatter_rows_to_bf16(dh_acc, h, cr.pos, cr.idx, cr.count, N, static_cast<__nv_bfloat16 *>(dH),
+                                   overwrite_dH, s));
+  }
+  return SAO_OK;
+}
+
+// The whole backward: one bwd_recompute_block per block of rows of the plan,
+// each on its own slice of H, y, lse, G, the mask and dH, all adding into dW
+// after the first; the blocks reuse the same scratch in stream order.
+sao_status bwd_recompute(const void *H, const void *W, const int32_t *y, const float *lse, const float *G,
+                         const uint8_t *mask, int64_t N, int32_t h, int32_t V, void *dH, float *dW, int accumulate,
+                         bool overwrite_dH, const BwdNames &names, unsigned int *err, Carver &c, cudaStream_t s) {
+  const BwdPlan pl = bwd_plan(N, h, V);
+  const __nv_bfloat16 *Hb = static_cast<const __nv_bfloat16 *>(H);
+  __nv_bfloat16 *dHb = static_cast<__nv_bfloat16 *>(dH);
+  for (int64_t r0 = 0; r0 < N; r0 += pl.rows) {
+    const int64_t nr = (N - r0) < pl.rows ? (N - r0) : pl.rows;
+    Carver cb = c;
+    SAO_TRY(bwd_recompute_block(Hb + r0 * h, W, y + r0, lse + r0, G + r0, mask ? mask + r0 : nullptr, nr, h, V,
+                                pl.vc, dHb + r0 * h, dW, r0 == 0 ? accumulate : 1, overwrite_dH, names, err, cb,
+                                s));
   }
   return SAO_OK;
 }

@@ -114,17 +114,15 @@ __global__ void gather_rows_kernel(const __nv_bfloat16 *H, int h, const int *idx
   }
 }
 
-// dH[t] = bf16(acc[pos[t]]) for active rows; the others get 0 (all_rows) or
-// are left as they are.
+// dH[t] = bf16(acc[pos[t]]) for active rows; the others get 0.
 __global__ void scatter_rows_f32_to_bf16_kernel(const float *acc, int h, const int *pos, int64_t N,
-                                                __nv_bfloat16 *dH, bool all_rows) {
+                                                __nv_bfloat16 *dH) {
   const int vec = h / 4;
   const int64_t total = N * vec;
   for (int64_t e = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; e < total; e += int64_t(gridDim.x) * blockDim.x) {
     const int64_t t = e / vec;
     const int v = int(e - t * vec);
     const int i = pos[t];
-    if (i < 0 && !all_rows) continue;
     float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
     if (i >= 0) x = reinterpret_cast<const float4 *>(acc + int64_t(i) * h)[v];
     const __nv_bfloat162 a = __floats2bfloat162_rn(x.x, x.y), b = __floats2bfloat162_rn(x.z, x.w);
@@ -132,6 +130,23 @@ __global__ void scatter_rows_f32_to_bf16_kernel(const float *acc, int h, const i
     w.x = *reinterpret_cast<const uint32_t *>(&a);
     w.y = *reinterpret_cast<const uint32_t *>(&b);
     reinterpret_cast<uint2 *>(dH + t * h)[v] = w;
+  }
+}
+
+// dH[idx[i]] = bf16(acc[i]) for the active rows i < count only.
+__global__ void scatter_active_f32_to_bf16_kernel(const float *acc, int h, const int *idx, const int *count,
+                                                  __nv_bfloat16 *dH) {
+  const int vec = h / 4;
+  const int64_t total = int64_t(*count) * vec;
+  for (int64_t e = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; e < total; e += int64_t(gridDim.x) * blockDim.x) {
+    const int64_t i = e / vec;
+    const int v = int(e - i * vec);
+    const float4 x = reinterpret_cast<const float4 *>(acc + i * h)[v];
+    const __nv_bfloat162 a = __floats2bfloat162_rn(x.x, x.y), b = __floats2bfloat162_rn(x.z, x.w);
+    uint2 w;
+    w.x = *reinterpret_cast<const uint32_t *>(&a);
+    w.y = *reinterpret_cast<const uint32_t *>(&b);
+    reinterpret_cast<uint2 *>(dH + int64_t(idx[i]) * h)[v] = w;
   }
 }
 
@@ -172,12 +187,15 @@ sao_status compact_rows(const uint8_t *mask, const float *g, int64_t N, const __
   return launch_end(slot, s);
 }
 
-sao_status scatter_rows_to_bf16(const float *acc, int32_t h, const int *pos, int64_t N, __nv_bfloat16 *dH,
-                                bool all_rows, cudaStream_t s) {
+sao_status scatter_rows_to_bf16(const float *acc, int32_t h, const int *pos, const int *idx, const int *count,
+                                int64_t N, __nv_bfloat16 *dH, bool all_rows, cudaStream_t s) {
   DeviceInfo di;
   SAO_TRY(device_info(&di));
   int slot = launch_begin("scatter_dH", s);
-  scatter_rows_f32_to_bf16_kernel<<<unsigned(di.sm_count * 8), 256, 0, s>>>(acc, h, pos, N, dH, all_rows);
+  if (all_rows)
+    scatter_rows_f32_to_bf16_kernel<<<unsigned(di.sm_count * 8), 256, 0, s>>>(acc, h, pos, N, dH);
+  else
+    scatter_active_f32_to_bf16_kernel<<<unsigned(di.sm_count * 8), 256, 0, s>>>(acc, h, idx, count, dH);
   return launch_end(slot, s);
 }
 

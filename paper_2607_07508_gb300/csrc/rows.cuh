@@ -24,8 +24,9 @@ sao_status compact_rows(const uint8_t *mask, const float *g, int64_t N, const __
                         CompactRows *out, Carver &c, cudaStream_t s);
 
 // dH[t] = bf16(acc[pos[t]]) on the active rows; inactive rows get zeros when
-// all_rows, else keep their contents.
-sao_status scatter_rows_to_bf16(const float *acc, int32_t h, const int *pos, int64_t N, __nv_bfloat16 *dH,
-                                bool all_rows, cudaStream_t s);
+// all_rows (a sweep over all N rows), else keep their contents (a sweep over
+// the `*count` active rows idx[0..count) only).
+sao_status scatter_rows_to_bf16(const float *acc, int32_t h, const int *pos, const int *idx, const int *count,
+                                int64_t N, __nv_bfloat16 *dH, bool all_rows, cudaStream_t s);
 
 }  // namespace sao

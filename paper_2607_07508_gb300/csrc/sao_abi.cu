@@ -13,7 +13,7 @@
 
 namespace sao {
 
-static std::atomic<size_t> g_dz_budget{size_t(24) << 30};
+static std::atomic<size_t> g_dz_budget{size_t(4) << 30};
 void set_dz_budget(size_t bytes) { g_dz_budget.store(bytes < (size_t(1) << 20) ? (size_t(1) << 20) : bytes); }
 size_t dz_budget() { return g_dz_budget.load(); }
 
@@ -104,6 +104,7 @@ void sao_set_checked(int on) { set_checked(on); }
 int sao_get_checked(void) { return checked_mode() ? 1 : 0; }
 
 void sao_set_dz_budget_bytes(size_t bytes) { set_dz_budget(bytes); }
+size_t sao_get_dz_budget_bytes(void) { return dz_budget(); }
 
 void sao_debug_set_scan_hooks(uint64_t wait_ns, int32_t skip_chunks) {
   g_scan_wait_ns.store(wait_ns == 0 ? kWaitLimitNs : (wait_ns > kWaitLimitNs ? kWaitLimitNs : wait_ns));

@@ -119,3 +119,24 @@ def test_kernel_source_hash_ignores_comments_and_layout_only():
     assert _code_only(base) == _code_only("/* doc */ int f(int x)\n{ return x + 1; }")
     assert _code_only(base) != _code_only(base.replace("x + 1", "x + 2"))
     assert _code_only("a /* multi\nline */ b // tail\nc") == "a b c"
+
+
+def test_backward_never_sizes_a_buffer_by_n_times_v(lib):
+    """The recompute backward's dZ lives in row blocks x vocabulary chunks
+    bounded by the dZ budget (default 4 GiB): quadrupling V at a fixed N grows
+    the workspace only by the forward's per-256-column tile partials (8 bytes
+    per row per 256 columns), never by 2 bytes per logit."""
+    from paper_2607_07508_gb300 import sao
+    assert sao.sao_get_dz_budget_bytes() == 4 << 30
+    for N, h, V in ((65536, 2048, 151936), (524288, 4096, 151936), (262144, 6144, 154880)):
+        w1 = sao.sao_workspace_bytes(N, h, V)
+        w4 = sao.sao_workspace_bytes(N, h, 4 * V)
+        assert w4 - w1 <= 8 * N * (3 * V // 256 + 4) + (1 << 20)
+        assert w1 < 2 * N * V          # smaller than one bf16 copy of the logits
+    sao.sao_set_dz_budget_bytes(1 << 30)
+    try:
+        assert sao.sao_get_dz_budget_bytes() == 1 << 30
+        small_budget = sao.sao_workspace_bytes(65536, 2048, 151936)
+    finally:
+        sao.sao_set_dz_budget_bytes(4 << 30)
+    assert small_budget < sao.sao_workspace_bytes(65536, 2048, 151936)

@@ -17,6 +17,7 @@ pytestmark = pytest.mark.gpu
 
 LOGP_TOL = 2e-3     # absolute
 GRAD_TOL = 2e-2     # relative L2
+DEFAULT_DZ_BUDGET = 4 << 30   # the library's default bound on the backward's dZ buffer
 
 
 def _fwd(H, W, y, cache, row_mask=None):
@@ -148,12 +149,12 @@ def test_cached_backward_chunked_and_accumulate():
     logp, lse = _fwd(H, W, y, cache)
     G = np.random.default_rng(3).normal(size=700).astype(np.float32)
     prev = torch.randn(3003, 128, device="cuda")
-    sao.sao_set_dz_budget_bytes(700 * 512 * 2)       # Vc = 512 -> 6 chunks
+    sao.sao_set_dz_budget_bytes(700 * 512 * 2)       # one row block, Vc = 512: 6 vocabulary chunks
     try:
         dH, dW = _bwd(H, W, y, lse, torch.as_tensor(G).cuda(), cache, accumulate=prev)
         torch.cuda.synchronize()
     finally:
-        sao.sao_set_dz_budget_bytes(24 << 30)
+        sao.sao_set_dz_budget_bytes(DEFAULT_DZ_BUDGET)
     _, want_lse = O.token_logprobs(H.cpu(), W.cpu(), wl.y)
     want_dH, want_dW = O.token_logprobs_bwd(H.cpu(), W.cpu(), wl.y, want_lse, G)
     assert rel_l2(dH.float().cpu().numpy(), want_dH) <= GRAD_TOL
@@ -223,7 +224,7 @@ def test_two_m_tile_gemms_with_ragged_tiles(cached, chunked):
     dH = torch.full_like(H, float("nan"))
     dW = torch.full((V, h), float("nan"), device="cuda")
     if chunked:
-        sao.sao_set_dz_budget_bytes(N * 5120 * 2)       # Vc = 5120 -> 4 chunks, the last one ragged
+        sao.sao_set_dz_budget_bytes(N * 5120 * 2)       # several vocabulary chunks, the last one ragged
     try:
         if cached:
             cache = sao.logprob_cache(N, V)
@@ -235,7 +236,7 @@ def test_two_m_tile_gemms_with_ragged_tiles(cached, chunked):
         torch.cuda.synchronize()
     finally:
         if chunked:
-            sao.sao_set_dz_budget_bytes(24 << 30)
+            sao.sao_set_dz_budget_bytes(DEFAULT_DZ_BUDGET)
     rows = np.sort(np.concatenate([rng.choice(N, size=24, replace=False), [N - 1]]))
     H_cpu, W_cpu = H[torch.as_tensor(rows).cuda()].cpu(), W.cpu()
     want_lp, want_lse = O.token_logprobs(H_cpu, W_cpu, wl.y[rows])
@@ -319,12 +320,12 @@ def test_cached_rows_far_below_their_maximum_are_recomputed(chunked, masked):
     logp, lse = _fwd(H, W, y, cache, row_mask=mask)
     prev = torch.randn(V, h, device="cuda") if chunked else None
     if chunked:
-        sao.sao_set_dz_budget_bytes(N * 256 * 2)     # Vc = 256 -> 4 chunks, the last ragged
+        sao.sao_set_dz_budget_bytes(N * 256 * 2)     # several vocabulary chunks, the last ragged
     try:
         dH, dW = _bwd(H, W, y, lse, torch.as_tensor(G).cuda(), cache, accumulate=prev)
         torch.cuda.synchronize()
     finally:
-        sao.sao_set_dz_budget_bytes(24 << 30)
+        sao.sao_set_dz_budget_bytes(DEFAULT_DZ_BUDGET)
     want_lp, want_lse = O.token_logprobs(H.cpu(), W.cpu(), yv)
     assert want_lp[far].max() < -60.0
     got_lp, got_lse = logp.cpu().numpy(), lse.cpu().numpy()

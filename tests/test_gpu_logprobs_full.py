@@ -1,15 +1,19 @@
 """Full-size parity of the tensor-core log-prob path, in the launch
-configuration bench.py times (persistent grid, many tiles per CTA).
+configuration bench.py times (persistent grid, many tiles per CTA; the
+backward in row blocks x vocabulary chunks under the default 4 GiB dZ bound).
 
 The oracle cannot redo 2*N*h*V fp64 flops at these sizes, so:
-  * logp and lse are checked on a seeded sample of rows, each over the whole
-    vocabulary (the oracle's own forward on those rows);
-  * with the incoming gradient non-zero only on sampled rows, dH is checked on
-    those rows (and must be exactly zero elsewhere) and dW on a seeded sample
-    of vocabulary rows that includes the sampled tokens (the oracle's own lse);
-  * with a dense gradient, dH is checked on sampled rows, and dW against the
-    linearity property dW(G) = dW(G on S) + dW(G off S) plus the column sums
-    sum_v dW[v, :] = 0 that every softmax gradient satisfies.
+  * logp and lse are checked on a seeded sample of 1024 rows, each over the
+    whole vocabulary (the oracle's own forward on those rows);
+  * dH is checked on 1024 sampled rows (the incoming gradient is local to each
+    row, so the oracle's backward on those rows alone is exact);
+  * dW is checked on a seeded sample of vocabulary rows that includes sampled
+    tokens, summed over every row with a non-zero gradient (the oracle's
+    backward over row chunks against the sampled W rows plus one spare row
+    that stands for every token outside the sample; the GPU's lse is the
+    input there, itself checked on the sampled rows);
+  * with a dense gradient, dW is also checked against the linearity property
+    dW(G) = dW(G on S) + dW(G off S) and the column sums sum_v dW[v, :] = 0.
 """
 import numpy as np
 import pytest
@@ -17,12 +21,13 @@ import torch
 
 from oracle import sao_oracle as O
 from paper_2607_07508_gb300 import sao, synthetic as S
-from tests._util import rel_l2
+from tests._util import near_bound, rel_err_floor, rel_l2
 
 pytestmark = pytest.mark.gpu
 
 LOGP_TOL = 2e-3
 GRAD_TOL = 2e-2
+SAMPLE_ROWS = 1024
 
 
 def _run(wl, G=None, ws=None):
@@ -40,18 +45,32 @@ def _run(wl, G=None, ws=None):
     return logp, lse, dH, dW, ws
 
 
-def _oracle_dW_rows(Hs, W_cpu, ys, lse_s, Gs, vrows):
-    """dW restricted to vocabulary rows `vrows` for the sampled token rows."""
-    Wsub = W_cpu[torch.as_tensor(vrows)]
-    pos = {int(v): i for i, v in enumerate(vrows)}
-    ysub = np.array([pos.get(int(t), -1) for t in ys])
-    Hd = O._f64(Hs)
-    Z = Hd @ O._f64(Wsub).T
-    dZ = -Gs[:, None] * np.exp(Z - lse_s[:, None])
-    for i, j in enumerate(ysub):
-        if j >= 0:
-            dZ[i, j] += Gs[i]
-    return dZ.T @ Hd
+def _rows_cpu(H, rows):
+    return H[torch.as_tensor(rows).cuda()].cpu()
+
+
+def oracle_dW_sample(H, W_cpu, y, lse, G, vrows, chunk=16384):
+    """dW[vrows] = sum over the rows t with G[t] != 0, from the oracle's
+    backward on row chunks against W[vrows] plus one spare vocabulary row that
+    every token outside vrows points at: a column of dZ depends only on its
+    own logit, the row's lse and G, and whether it is the sampled token, so the
+    sampled columns come out exact and the spare column is dropped."""
+    vrows = np.asarray(vrows)
+    spare = int(np.setdiff1d(np.arange(len(vrows) + 1), vrows)[0])
+    Wsub = W_cpu[torch.as_tensor(np.concatenate([vrows, [spare]]))]
+    pos = np.full(W_cpu.shape[0], len(vrows), np.int64)
+    pos[vrows] = np.arange(len(vrows))
+    active = np.flatnonzero(G != 0)
+    acc = np.zeros((len(vrows), W_cpu.shape[1]), np.float64)
+    for c0 in range(0, len(active), chunk):
+        rows = active[c0:c0 + chunk]
+        _, dWc = O.token_logprobs_bwd(_rows_cpu(H, rows), Wsub, pos[y[rows]], lse[rows], G[rows])
+        acc += dWc[:len(vrows)]
+    return acc
+
+
+def _vocab_sample(rng, V, tokens, k=256):
+    return np.unique(np.concatenate([rng.choice(V, size=k, replace=False), tokens, [V - 1]]))
 
 
 @pytest.mark.parametrize("name", ["small", "moe", "long", "large"])
@@ -59,27 +78,134 @@ def test_full_size_sampled_rows(name):
     torch.manual_seed(0)
     wl = S.make_workload(name, device="cuda")
     rng = np.random.default_rng(11)
-    rows = np.sort(rng.choice(wl.N, size=32, replace=False))
+    rows = np.sort(rng.choice(wl.N, size=SAMPLE_ROWS, replace=False))
     G = np.zeros(wl.N, np.float32)
     G[rows] = rng.normal(size=len(rows)).astype(np.float32)
     logp, lse, dH, dW, ws = _run(wl, torch.as_tensor(G).cuda())
     torch.cuda.synchronize()
-    H_cpu, W_cpu = wl.H[torch.as_tensor(rows).cuda()].cpu(), wl.W.cpu()
+    H_cpu, W_cpu = _rows_cpu(wl.H, rows), wl.W.cpu()
     want_lp, want_lse = O.token_logprobs(H_cpu, W_cpu, wl.y[rows])
     assert np.abs(logp.cpu().numpy()[rows] - want_lp).max() <= LOGP_TOL
     assert np.abs(lse.cpu().numpy()[rows] - want_lse).max() <= LOGP_TOL
     # dH on the sampled rows, exact zeros elsewhere
     want_dH, _ = O.token_logprobs_bwd(H_cpu, W_cpu, wl.y[rows], want_lse, G[rows])
-    got_dH = dH.float().cpu().numpy()
-    assert rel_l2(got_dH[rows], want_dH) <= GRAD_TOL
-    others = np.ones(wl.N, bool)
-    others[rows] = False
-    assert not np.any(got_dH[others])
-    # dW on a vocabulary sample that includes the sampled tokens
-    vrows = np.unique(np.concatenate([rng.choice(wl.V, size=512, replace=False), wl.y[rows], [wl.V - 1]]))
-    want_dW = _oracle_dW_rows(H_cpu, W_cpu, wl.y[rows], want_lse, G[rows].astype(np.float64), vrows)
+    assert rel_l2(_rows_cpu(dH, rows).float().numpy(), want_dH) <= GRAD_TOL
+    others = torch.ones(wl.N, dtype=torch.bool, device="cuda")
+    others[torch.as_tensor(rows).cuda()] = False
+    assert dH[others].abs().max().item() == 0
+    # dW on a vocabulary sample that includes some sampled tokens
+    vrows = _vocab_sample(rng, wl.V, wl.y[rows[:64]])
+    want_dW = oracle_dW_sample(wl.H, W_cpu, wl.y, lse.cpu().numpy().astype(np.float64), G.astype(np.float64),
+                               vrows)
     got_dW = dW[torch.as_tensor(vrows).cuda()].cpu().numpy()
     assert rel_l2(got_dW, want_dW) <= GRAD_TOL
+
+
+@pytest.mark.parametrize("name", ["moe", "long", "large"])
+def test_bench_step_path(name):
+    """The calls bench.py times, in its order and launch configuration: the
+    forward on the action rows only (row_mask = loss mask), the policy loss
+    against the workload's stale log-probs, its gradient, and the recompute
+    backward on the dense gradient (row blocks x vocabulary chunks at long and
+    large). logp and dH on 1024 sampled action rows, the loss, flags, counts
+    and gradient on every token, dW on sampled vocabulary rows over all rows."""
+    wl = S.make_workload(name, device="cuda")
+    N, h, V = wl.N, wl.h, wl.V
+    assert sao.sao_get_dz_budget_bytes() == 4 << 30
+    y = torch.as_tensor(wl.y).cuda()
+    mask = torch.as_tensor(wl.loss_mask).cuda()
+    ws = sao.workspace(N, h, V, wl.H.dtype)
+    logp = torch.empty(N, device="cuda")
+    lse = torch.empty(N, device="cuda")
+    sao.sao_token_logprobs_fwd(wl.H, wl.W, y, logp, lse, ws, row_mask=mask)
+    old = (logp + torch.as_tensor(wl.xi).cuda()).contiguous()
+    adv = torch.as_tensor(np.random.default_rng(3).normal(size=N).astype(np.float32)).cuda()
+    loss = torch.empty(1, device="cuda")
+    counts = torch.empty(4, dtype=torch.int64, device="cuda")
+    coef = torch.empty(N, device="cuda")
+    flags = torch.empty(N, dtype=torch.uint8, device="cuda")
+    sao.sao_policy_loss_fwd(logp, old, adv, mask, wl.eps_low, wl.eps_high, loss, counts, ws, coef=coef, flags=flags)
+    G = torch.empty(N, device="cuda")
+    sao.sao_policy_loss_bwd(logp, old, adv, mask, wl.eps_low, wl.eps_high, torch.ones(1, device="cuda"), G, ws)
+    dH = torch.full_like(wl.H, float("nan"))
+    dW = torch.full((V, h), float("nan"), device="cuda")
+    sao.sao_token_logprobs_bwd(wl.H, wl.W, y, lse, G, dH, dW, ws)
+    torch.cuda.synchronize()
+
+    m = wl.loss_mask.astype(bool)
+    lp, ol, ad, g = (t.cpu().numpy() for t in (logp, old, adv, G))
+    # the loss on every token, decided on the GPU's fp32 log-probs (same floats on both sides)
+    pl = O.policy_loss(lp, ol, ad, wl.loss_mask, wl.eps_low, wl.eps_high)
+    ok = ~near_bound(lp, ol, wl.eps_low, wl.eps_high)
+    assert np.array_equal(flags.cpu().numpy()[ok], pl["flags"][ok])
+    if ok.all():
+        assert list(counts.cpu().numpy()) == list(pl["counts"])
+    assert abs(loss.item() - pl["loss"]) <= 1e-4 * abs(pl["loss"])
+    assert rel_err_floor(g[ok], pl["coef"][ok], 1e-12).max() <= 1e-5
+    # log-probs and dH on sampled action rows
+    rng = np.random.default_rng(21)
+    rows = np.sort(rng.choice(np.flatnonzero(m), size=SAMPLE_ROWS, replace=False))
+    H_cpu, W_cpu = _rows_cpu(wl.H, rows), wl.W.cpu()
+    want_lp, want_lse = O.token_logprobs(H_cpu, W_cpu, wl.y[rows])
+    assert np.abs(lp[rows] - want_lp).max() <= LOGP_TOL
+    assert np.all(lp[~m] == 0)
+    want_dH, _ = O.token_logprobs_bwd(H_cpu, W_cpu, wl.y[rows], want_lse, g[rows])
+    assert rel_l2(_rows_cpu(dH, rows).float().numpy(), want_dH) <= GRAD_TOL
+    assert dH[G == 0].abs().max().item() == 0
+    assert torch.isfinite(dH).all().item()
+    # dW on 256 sampled vocabulary rows (plus a few sampled tokens), over every row
+    vrows = _vocab_sample(rng, V, wl.y[rows[:32]])
+    want_dW = oracle_dW_sample(wl.H, W_cpu, wl.y, lse.cpu().numpy().astype(np.float64), g.astype(np.float64),
+                               vrows)
+    got_dW = dW[torch.as_tensor(vrows).cuda()].cpu().numpy()
+    assert rel_l2(got_dW, want_dW) <= GRAD_TOL
+    assert torch.isfinite(dW).all().item()
+
+
+@pytest.mark.parametrize("cached", [False, True])
+def test_peaked_logits_moe_shape(cached):
+    """The moe shape with W ~ N(0, 0.2): logits with a standard deviation near
+    9 (ten times the workload's), so the online maximum moves across tiles,
+    the exponentials span the fp32 range, and, on the cached path, rows whose
+    sampled token lies more than 60 nats below the row's maximum are flagged
+    and recomputed. The sample holds the rows with the lowest log-probs."""
+    wl = S.make_workload("moe", device="cuda")
+    N, h, V = wl.N, wl.h, wl.V
+    W = (wl.W.float() * 10.0).to(torch.bfloat16)
+    y = torch.as_tensor(wl.y).cuda()
+    ws = sao.workspace(N, h, V, wl.H.dtype)
+    logp = torch.empty(N, device="cuda")
+    lse = torch.empty(N, device="cuda")
+    rng = np.random.default_rng(41)
+    G = (rng.normal(size=N) * 1e-3).astype(np.float32)
+    Gt = torch.as_tensor(G).cuda()
+    dH = torch.empty_like(wl.H)
+    dW = torch.empty(V, h, device="cuda")
+    if cached:
+        cache = sao.logprob_cache(N, V)
+        sao.sao_token_logprobs_fwd_cached(wl.H, W, y, logp, lse, cache, ws)
+        sao.sao_token_logprobs_bwd_cached(wl.H, W, y, lse, Gt, dH, dW, cache, ws)
+    else:
+        sao.sao_token_logprobs_fwd(wl.H, W, y, logp, lse, ws)
+        sao.sao_token_logprobs_bwd(wl.H, W, y, lse, Gt, dH, dW, ws)
+    torch.cuda.synchronize()
+    lp = logp.cpu().numpy()
+    lowest = np.argsort(lp)[:64]
+    rows = np.unique(np.concatenate([lowest, rng.choice(N, size=SAMPLE_ROWS - 64, replace=False)]))
+    H_cpu, W_cpu = _rows_cpu(wl.H, rows), W.cpu()
+    want_lp, want_lse = O.token_logprobs(H_cpu, W_cpu, wl.y[rows])
+    assert want_lp.min() < -60.0          # the flagged-row case is in the sample
+    assert np.abs(lp[rows] - want_lp).max() <= LOGP_TOL
+    assert np.abs(lse.cpu().numpy()[rows] - want_lse).max() <= LOGP_TOL
+    want_dH, _ = O.token_logprobs_bwd(H_cpu, W_cpu, wl.y[rows], want_lse, G[rows])
+    got_dH = dH.float().cpu().numpy()[rows]
+    assert rel_l2(got_dH, want_dH) <= GRAD_TOL
+    low = np.isin(rows, lowest)
+    assert rel_l2(got_dH[low], want_dH[low]) <= GRAD_TOL
+    vrows = _vocab_sample(rng, V, wl.y[lowest[:16]])
+    want_dW = oracle_dW_sample(wl.H, W_cpu, wl.y, lse.cpu().numpy().astype(np.float64), G.astype(np.float64),
+                               vrows)
+    assert rel_l2(dW[torch.as_tensor(vrows).cuda()].cpu().numpy(), want_dW) <= GRAD_TOL
 
 
 @pytest.mark.parametrize("name", ["moe", "large"])
@@ -88,11 +214,11 @@ def test_full_size_dense_gradient(name):
     rng = np.random.default_rng(12)
     G = (rng.normal(size=wl.N) * 1e-4).astype(np.float32)
     G[wl.loss_mask == 0] = 0.0
-    rows = np.sort(rng.choice(np.flatnonzero(G), size=24, replace=False))
+    rows = np.sort(rng.choice(np.flatnonzero(G), size=256, replace=False))
     Gt = torch.as_tensor(G).cuda()
     logp, lse, dH, dW, ws = _run(wl, Gt)
     torch.cuda.synchronize()
-    H_cpu, W_cpu = wl.H[torch.as_tensor(rows).cuda()].cpu(), wl.W.cpu()
+    H_cpu, W_cpu = _rows_cpu(wl.H, rows), wl.W.cpu()
     _, want_lse = O.token_logprobs(H_cpu, W_cpu, wl.y[rows])
     want_dH, _ = O.token_logprobs_bwd(H_cpu, W_cpu, wl.y[rows], want_lse, G[rows])
     assert rel_l2(dH.float().cpu().numpy()[rows], want_dH) <= GRAD_TOL
@@ -110,6 +236,32 @@ def test_full_size_dense_gradient(name):
     assert diff <= 1e-2
     colsum = dW.sum(dim=0).abs().max().item()
     assert colsum <= 1e-2 * dW.abs().sum(dim=0).max().item()
+
+
+def test_budget_splits_agree():
+    """The same backward under dZ bounds that give one block and one chunk, one
+    block and several chunks, and several blocks and chunks: dH and dW agree
+    within the bf16 rounding of dZ (the sums are grouped differently)."""
+    wl = S.make_custom([6000, 3000, 1200], 256, 20000, "bf16", seed=91, device="cuda")
+    G = torch.as_tensor(np.random.default_rng(9).normal(size=wl.N).astype(np.float32)).cuda()
+    outs = []
+    try:
+        for budget in (1 << 30, wl.N * 4096 * 2, 1 << 20):
+            sao.sao_set_dz_budget_bytes(budget)
+            _, _, dH, dW, _ = _run(wl, G)
+            outs.append((dH.float().cpu().numpy(), dW.cpu().numpy()))
+    finally:
+        sao.sao_set_dz_budget_bytes(4 << 30)
+    torch.cuda.synchronize()
+    for dH, dW in outs[1:]:
+        assert rel_l2(dH, outs[0][0]) <= 1e-2
+        assert rel_l2(dW, outs[0][1]) <= 1e-2
+    H_cpu, W_cpu = wl.H.cpu(), wl.W.cpu()
+    _, want_lse = O.token_logprobs(H_cpu, W_cpu, wl.y)
+    want_dH, want_dW = O.token_logprobs_bwd(H_cpu, W_cpu, wl.y, want_lse, G.cpu().numpy())
+    for dH, dW in outs:
+        assert rel_l2(dH, want_dH) <= GRAD_TOL
+        assert rel_l2(dW, want_dW) <= GRAD_TOL
 
 
 def test_many_tiles_per_cta_full_oracle():
@@ -146,6 +298,6 @@ def test_full_size_row_mask_forward():
     got = logp.cpu().numpy()
     assert np.all(got[~m] == 0) and np.all(lse.cpu().numpy()[~m] == 0)
     assert np.array_equal(got[m], full_lp.cpu().numpy()[m])
-    rows = np.sort(np.random.default_rng(13).choice(np.flatnonzero(m), size=16, replace=False))
-    want, _ = O.token_logprobs(wl.H[torch.as_tensor(rows).cuda()].cpu(), wl.W.cpu(), wl.y[rows])
+    rows = np.sort(np.random.default_rng(13).choice(np.flatnonzero(m), size=256, replace=False))
+    want, _ = O.token_logprobs(_rows_cpu(wl.H, rows), wl.W.cpu(), wl.y[rows])
     assert np.abs(got[rows] - want).max() <= LOGP_TOL

@@ -276,6 +276,38 @@ def test_policy_loss_eps_low_one_disables_lower_mask():
     assert list(out["flags"]) == [0, 0]
 
 
+def test_clip_ratio_hand_counts_and_empty_batch():
+    """§4.4's clip ratio: the share of action tokens that f masks by a bound.
+    The hand example above masks one token low and one high out of four;
+    non-finite tokens are masked but not clipped; no action token gives 0."""
+    logp = np.array([-1.0, -0.7, -1.3, -0.8], np.float32)
+    old = np.full(4, -1.0, np.float32)
+    out = O.policy_loss(logp, old, np.array([0.5, 2.0, -1.0, -0.25], np.float32), np.ones(4, np.uint8), 0.2, 0.28)
+    assert O.clip_ratio(out["counts"]) == 0.5
+    assert O.clip_ratio([4, 0, 0, 3]) == 0.0
+    assert O.clip_ratio([7, 2, 0, 5]) == 2 / 7
+    assert O.clip_ratio([0, 0, 0, 0]) == 0.0
+    assert O.clip_ratio(np.zeros(4, np.int64)) == 0.0
+
+
+def test_clip_ratio_brute_force():
+    """Counted token by token in fp64 on ratios kept 1e-3 away from both
+    bounds: clipped action tokens over all action tokens."""
+    r = _rng(31)
+    N = 400
+    ratio = np.exp(r.normal(0.0, 0.5, size=N))
+    el, eh = 0.3, 0.4
+    keep = (np.abs(ratio - (1 - el)) > 1e-3) & (np.abs(ratio - (1 + eh)) > 1e-3)
+    ratio = ratio[keep]
+    old = np.zeros(len(ratio), np.float32)
+    logp = np.log(ratio).astype(np.float32)
+    m = (r.random(len(ratio)) < 0.8).astype(np.uint8)
+    out = O.policy_loss(logp, old, np.ones(len(ratio), np.float32), m, el, eh)
+    clipped = sum(1 for t in range(len(ratio)) if m[t] and (ratio[t] <= 1 - el or ratio[t] >= 1 + eh))
+    assert 0 < clipped < m.sum()
+    assert O.clip_ratio(out["counts"]) == clipped / int(m.sum())
+
+
 def test_policy_loss_paper_bounds():
     hp = json.load(open(GOLDEN))
     for key in ("clip_reasoning", "clip_coding"):
