@@ -36,24 +36,24 @@ WORKLOAD = "moe"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
-def stored_traffic(kernel: str, rows: int, workload: str = "moe"):
-    """DRAM bytes per launch of `kernel` from the committed ncu capture
-    (profiles/dram_traffic_moe.txt, taken on the moe shape), scaled to `rows`
-    active rows, or None for another shape, a missing capture, or kernel
-    sources changed since it was taken."""
-    if workload != "moe":
-        return None
+def stored_traffic(kernel: str, rows: int, cols: float):
+    """DRAM bytes per launch of `kernel` from the committed small-case ncu
+    capture (profiles/dram_traffic_tc_gemm_moe8k.txt: the moe shape at 8,192
+    tokens), scaled by rows x vocabulary columns per launch to a launch of
+    `rows` rows and `cols` columns (the dZ writes and operand reads dominate
+    and grow with both), or None for a missing capture or kernel sources
+    changed since it was taken."""
     from paper_2607_07508_gb300.build import kernel_source_hash
-    path = os.path.join(ROOT, "profiles", "dram_traffic_moe.txt")
+    path = os.path.join(ROOT, "profiles", "dram_traffic_tc_gemm_moe8k.txt")
     try:
         lines = [l.split() for l in open(path) if l.strip() and not l.startswith("#")]
     except OSError:
         return None
     src = kernel_source_hash()
     for f in lines:
-        if len(f) == 5 and f[0] == kernel and f[1] == src:
-            cap_rows, rd, wr = int(f[2]), float(f[3]), float(f[4])
-            return (rd + wr) * rows / cap_rows
+        if len(f) == 6 and f[0] == kernel and f[1] == src:
+            cap_rows, cap_cols, rd, wr = int(f[2]), int(f[3]), float(f[4]), float(f[5])
+            return (rd + wr) * (rows * cols) / (cap_rows * cap_cols)
     return None
 
 
@@ -210,9 +210,10 @@ class LossHeadStep:
             s.sao_token_logprobs_bwd(self.H, self.W, self.y, self.lse, self.G, self.dH, self.dW, self.ws)
 
 
-# Algorithmic work per launch of each tensor-core kernel, in flops: the
-# forward computes the rows with loss_mask = 1, the backward kernels the rows
-# with a non-zero incoming gradient.
+# Algorithmic work per step of each tensor-core kernel, in flops: the forward
+# computes the rows with loss_mask = 1, the backward kernels the rows with a
+# non-zero incoming gradient (over all vocabulary chunks and row blocks of the
+# step; a launch does its share of it).
 def kernel_flops(name, h, V, rows_fwd, rows_bwd):
     if name == "tc_logits_lse_fwd":
         return 2.0 * rows_fwd * h * V
@@ -546,6 +547,8 @@ def main():
     ap.add_argument("--recompute", action="store_true", help="the default path (kept for older command lines)")
     ap.add_argument("--dz-budget-gib", type=float, default=None,
                     help="bound on the backward's bf16 dZ buffer (default: the library's, 4 GiB)")
+    ap.add_argument("--cta-pairs", type=int, choices=[0, 1], default=None,
+                    help="tile the tensor-core GEMMs over CTA pairs (1) or single CTAs (0); default: the library's")
     ap.add_argument("--cpu-baseline-child", default=None, help=argparse.SUPPRESS)
     ap.add_argument("--bandwidth-study", action="store_true",
                     help="time the O(N) kernels alone on the 2^27-token bandwidth workload")
@@ -570,6 +573,8 @@ def main():
     peaks, peak_src = load_peaks()
     if args.dz_budget_gib is not None:
         sao.sao_set_dz_budget_bytes(int(args.dz_budget_gib * (1 << 30)))
+    if args.cta_pairs is not None:
+        sao.sao_set_cta_pairs(bool(args.cta_pairs))
 
     seed = S.SEED_BASE + S.CONFIG_NAMES.index(args.config) + 97 * rank
     wl = S.make_workload(args.config, device=dev, seed=seed, N_override=args.tokens)
@@ -619,7 +624,9 @@ def main():
     dom = max(prof.items(), key=lambda kv: kv[1][1])
     dom_name, (dom_n, dom_ms) = dom
     avg_ms = dom_ms / dom_n
-    fl = kernel_flops(dom_name, wl.h, wl.V, rows_fwd, rows_bwd)
+    fl_step = kernel_flops(dom_name, wl.h, wl.V, rows_fwd, rows_bwd)
+    per_step = dom_n / args.steps
+    fl = fl_step / per_step if fl_step is not None else None
     burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
     sustained = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
     peak_mhz = (peaks.get("clocks_under_load") or {}).get("sm_mhz_median")
@@ -631,9 +638,13 @@ def main():
         dom_rows = rows_fwd if (dom_name == "tc_logits_lse_fwd" or cached) else rows_bwd
         roofline = {"bound": "tensor", "kernel": dom_name, "achieved": achieved, "peak": burst,
                     "unit": "TFLOP/s", "frac": achieved / burst,
-                    "traffic": stored_traffic(dom_name, dom_rows, wl.name),
-                    "traffic_unit": "bytes per launch (dram read + write, ncu, scaled by active rows)",
-                    "algorithmic_per_launch": f"2*rows*h*V = {fl:.4g} flop", "avg_launch_ms": avg_ms,
+                    "traffic": (stored_traffic(dom_name, dom_rows, wl.V / per_step)
+                                if wl.name == "moe" and args.tokens is None else None),
+                    "traffic_unit": ("bytes per launch (dram read + write from the 8k-token ncu capture, scaled by "
+                                     "rows x vocabulary columns per launch)"),
+                    "algorithmic_per_launch": (f"2*rows*h*V = {fl_step:.4g} flop per step over {per_step:g} "
+                                               f"launches = {fl:.4g} flop per launch"),
+                    "avg_launch_ms": avg_ms, "launches_per_step": per_step,
                     "peak_source": f"{peak_src} bf16_tflops (burst)",
                     "frac_of_sustained_peak": achieved / sustained}
     else:
@@ -660,6 +671,8 @@ def main():
                                              if cached else
                                              "algorithmic + 2hV per backward row (the logits are recomputed)"),
                  "logprob_path": "cached" if cached else "recompute",
+                 "gemm_tiling": "CTA pairs (tcgen05 cta_group::2, M = 256)" if sao.sao_get_cta_pairs()
+                                else "single CTAs (M = 128)",
                  "largest_logit_buffer": (f"[{rows_fwd}, {wl.V}] bf16 probabilities ({2.0 * rows_fwd * wl.V / 1e9:.1f} GB)"
                                           if cached else
                                           f"bf16 dZ of one row block x vocabulary chunk, at most "

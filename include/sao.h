@@ -104,6 +104,16 @@ SAO_API void sao_set_dz_budget_bytes(size_t bytes);
 /* The current bound (bytes) set by sao_set_dz_budget_bytes or the default. */
 SAO_API size_t sao_get_dz_budget_bytes(void);
 
+/* Tiling of the bf16 tensor-core GEMMs (process-wide; default 0). on = 1:
+ * CTA pairs, clusters of 2 CTAs sharing each tcgen05.mma.cta_group::2 of
+ * M = 256 (each CTA loads its own 128 rows of A and half of the B tile); on =
+ * 0: single CTAs with M = 128 MMAs. Results agree to within the fp32
+ * accumulation order. On one GB300 under its power cap the pairs do about 3 %
+ * more work per SM clock but run at a lower clock, and the moe step takes
+ * 2.5 % longer, hence the default. Affects later calls only. */
+SAO_API void sao_set_cta_pairs(int on);
+SAO_API int sao_get_cta_pairs(void);
+
 /*
  * Test hooks of the advantage scan (process-wide; defaults restored by
  * (0, 0)): every look-back wait gives up after wait_ns nanoseconds (0: the

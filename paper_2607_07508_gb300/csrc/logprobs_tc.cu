@@ -95,8 +95,10 @@ struct GemmParams {
   const float *row_scale;
 };
 
+constexpr int kMaxStages = 6;  // CTA pairs hold half a B tile per stage: 6 stages in the same bytes
+
 struct __align__(8) SmemCtl {
-  uint64_t full[STAGES], empty[STAGES], acc_full[2], acc_empty[2];
+  uint64_t full[kMaxStages], empty[kMaxStages], acc_full[2], acc_empty[2];
   uint32_t tmem_base;
   int abort;
 };
@@ -117,16 +119,30 @@ __device__ __forceinline__ void tile_coords(int L, const GemmParams &p, int nM, 
 // row tiles instead of 152; the stages (A 32 KB + B 32 KB) shrink to 3. The
 // tile's epilogue then waits for both accumulators, which costs little when
 // K spans thousands of blocks.
-template <int kEpi, bool kAMN, bool kBMN, int kMT = 1>
+//
+// kCG = 2: the grid is made of CTA pairs (clusters of 2) and every MMA is a
+// tcgen05.mma.cta_group::2 of M = 256 over the pair. Each CTA loads its own
+// 128 rows of A and its half (128 columns) of the B tile into its own shared
+// memory, so a pair moves 3/4 of the operand bytes two single CTAs would for
+// the same flops, and accumulates its own 128 rows x 256 columns in its own
+// TMEM. The even CTA's producer counts both CTAs' copies on its full barrier
+// (the odd CTA's copies signal it across the pair), its one MMA thread issues
+// for the pair and commits to both CTAs' empty and accumulator barriers, and
+// both CTAs' epilogue threads release an accumulator on the even CTA's
+// barrier. The stages hold half a B tile: 6 (or 4 with kMT = 2).
+template <int kEpi, bool kAMN, bool kBMN, int kMT = 1, int kCG = 1>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
                    const __grid_constant__ CUtensorMap map_c, const GemmParams p) {
   static_assert(kMT == 1 || kMT == 2, "one or two M tiles per CTA tile");
+  static_assert(kCG == 1 || kCG == 2, "single CTAs or CTA pairs");
   static_assert(kMT == 1 || kEpi == kStoreF32 || kEpi == kStoreBF16, "two M tiles: plain store epilogues only");
-  constexpr int kStages = kMT == 2 ? 3 : STAGES;
   constexpr uint32_t kABytes = A_BYTES * kMT;
-  constexpr uint32_t kStageBytes = kABytes + B_BYTES;
-  constexpr int kTM = BM * kMT;  // rows of a CTA tile
+  constexpr uint32_t kBBytes = B_BYTES / kCG;  // this CTA's part of a B stage
+  constexpr uint32_t kStageBytes = kABytes + kBBytes;
+  constexpr int kStages = int(size_t(STAGES) * STAGE_BYTES / kStageBytes);
+  constexpr int kTM = BM * kMT * kCG;  // rows of a tile (of the pair's tile for kCG = 2)
+  static_assert(kStages <= kMaxStages, "barrier arrays");
   static_assert(size_t(kStages) * kStageBytes <= size_t(STAGES) * STAGE_BYTES, "same shared-memory layout");
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -137,6 +153,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   volatile int *abort = &ctl->abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // CTA pairs: rank in the pair, the pair's index and the number of pairs
+  const uint32_t rank = kCG == 2 ? cluster_ctarank() : 0u;
+  const int cl = int(blockIdx.x) / kCG, ncl = int(gridDim.x) / kCG;
   int nM = p.nM, nK = p.nK;
   int64_t rows = p.rows;
   if (p.m_count) {
@@ -151,20 +170,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const bool kzero = (nK == 0);  // empty contraction: the tile is all zeros
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < kStages; ++s) {
       mbar_init(smem_u32(&ctl->full[s]), 1);
       mbar_init(smem_u32(&ctl->empty[s]), 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&ctl->acc_full[a]), 1);
-      mbar_init(smem_u32(&ctl->acc_empty[a]), 4 * 32);
+      mbar_init(smem_u32(&ctl->acc_empty[a]), 4 * 32 * kCG);
     }
     ctl->abort = 0;
     fence_barrier_init();
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(&ctl->tmem_base), TMEM_COLS);
-    tmem_relinquish();
+    if constexpr (kCG == 2) {
+      tmem_alloc_pair(smem_u32(&ctl->tmem_base), TMEM_COLS);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(smem_u32(&ctl->tmem_base), TMEM_COLS);
+      tmem_relinquish();
+    }
   }
   if (warp == 0 && lane == 0) {
     tma_prefetch_map(&map_a);
@@ -172,8 +196,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
   fence_before_sync();
   __syncthreads();
+  // both CTAs' barriers exist before either CTA's copies, commits or arrivals reach them
+  if constexpr (kCG == 2) cluster_sync();
   fence_after_sync();
   const uint32_t tmem_base = ctl->tmem_base;
+  // releases an accumulator: on this CTA's barrier, or the even CTA's for a pair
+  auto release_acc = [&](int a) {
+    const uint32_t bar = smem_u32(&ctl->acc_empty[a]);
+    if (kCG == 2 && rank != 0u)
+      mbar_arrive_cluster(mapa_shared(bar, 0u));
+    else
+      mbar_arrive(bar);
+  };
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -183,7 +217,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       bool ok = true;
       uint32_t issued = 0;  // bit s: stage s has a load whose full-barrier phase is phase_of(s)
       uint32_t issued_phase = 0;
-      for (int L = blockIdx.x; L < num_tiles && ok; L += gridDim.x) {
+      // a load lands in this CTA's shared memory; its bytes are counted on
+      // this CTA's full barrier, or on the even CTA's for a pair
+      auto load = [&](uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y) {
+        if constexpr (kCG == 2)
+          tma_load_2d_pair(dst, map, bar, x, y);
+        else
+          tma_load_2d(dst, map, bar, x, y);
+      };
+      for (int L = cl; L < num_tiles && ok; L += ncl) {
         int m, n;
         tile_coords(L, p, nM, m, n);
         for (int kb = 0; kb < nK; ++kb) {
@@ -191,27 +233,30 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             ok = false;
             break;
           }
-          const uint32_t fb = smem_u32(&ctl->full[stage]);
+          const uint32_t fb_own = smem_u32(&ctl->full[stage]);
+          const uint32_t fb = kCG == 2 ? mapa_shared(fb_own, 0u) : fb_own;
           issued |= 1u << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-          mbar_arrive_expect_tx(fb, kStageBytes);
+          if (rank == 0u) mbar_arrive_expect_tx(fb_own, kStageBytes * kCG);
           const uint32_t sa = base + uint32_t(stage) * kStageBytes;
           const uint32_t sb = sa + kABytes;
           const int k0 = kb * BK;
-          if (!kAMN) {
 #pragma unroll
-            for (int j = 0; j < kMT; ++j) tma_load_2d(sa + j * A_BYTES, &map_a, fb, k0, p.a_row_off + m * kTM + j * BM);
-          } else {
+          for (int j = 0; j < kMT; ++j) {  // this CTA's 128 rows of M tile j
+            const int row = p.a_row_off + m * kTM + j * BM * kCG + int(rank) * BM;
+            if (!kAMN) {
+              load(sa + j * A_BYTES, &map_a, fb, k0, row);
+            } else {
 #pragma unroll
-            for (int j = 0; j < kTM / 64; ++j)
-              tma_load_2d(sa + j * MN_ATOM_BYTES, &map_a, fb, p.a_row_off + m * kTM + 64 * j, k0);
+              for (int jj = 0; jj < BM / 64; ++jj) load(sa + j * A_BYTES + jj * MN_ATOM_BYTES, &map_a, fb, row + 64 * jj, k0);
+            }
           }
+          const int ncol = n * BN + int(rank) * (BN / kCG);  // this CTA's columns of the B tile
           if (!kBMN) {
-            tma_load_2d(sb, &map_b, fb, k0, p.b_row_off + n * BN);
+            load(sb, &map_b, fb, k0, p.b_row_off + ncol);
           } else {
 #pragma unroll
-            for (int j = 0; j < BN / 64; ++j)
-              tma_load_2d(sb + j * MN_ATOM_BYTES, &map_b, fb, n * BN + 64 * j, p.b_row_off + k0);
+            for (int j = 0; j < BN / kCG / 64; ++j) load(sb + j * MN_ATOM_BYTES, &map_b, fb, ncol + 64 * j, p.b_row_off + k0);
           }
           if (++stage == kStages) {
             stage = 0;
@@ -219,8 +264,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
         }
       }
-      if (!ok) {
-        // let the copies already in flight land before the CTA can exit
+      if (!ok && rank == 0u) {
+        // let the copies already in flight land before the CTA can exit (a
+        // pair's full barriers, in the even CTA, count both CTAs' copies)
         for (int s = 0; s < kStages; ++s) {
           if (!((issued >> s) & 1u)) continue;
           const uint32_t par = (issued_phase >> s) & 1u;
@@ -232,13 +278,26 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16(BM, BN, kAMN, kBMN);
+    // a pair's MMAs are all issued by the even CTA
+    if (lane == 0 && rank == 0u) {
+      constexpr uint32_t idesc = idesc_bf16(BM * kCG, BN, kAMN, kBMN);
       int stage = 0;
       uint32_t phase = 0;
       int local = 0;
       bool ok = true;
-      for (int L = blockIdx.x; L < num_tiles && ok; L += gridDim.x, ++local) {
+      auto commit = [&](uint32_t bar) {
+        if constexpr (kCG == 2)
+          mma_commit_pair(bar, uint16_t(0x3));
+        else
+          mma_commit(bar);
+      };
+      auto mma = [&](uint32_t d, uint64_t ad, uint64_t bd, uint32_t accum) {
+        if constexpr (kCG == 2)
+          mma_bf16_pair(d, ad, bd, idesc, accum);
+        else
+          mma_bf16(d, ad, bd, idesc, accum);
+      };
+      for (int L = cl; L < num_tiles && ok; L += ncl, ++local) {
         // kMT == 2: both accumulators serve one tile, tracked as accumulator 0
         const int acc = kMT == 2 ? 0 : (local & 1);
         const uint32_t acc_phase = kMT == 2 ? (uint32_t(local) & 1u) : (uint32_t(local >> 1) & 1u);
@@ -262,17 +321,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
               const uint32_t aj = sa + uint32_t(j) * A_BYTES;
               const uint64_t ad = kAMN ? sdesc_sw128(aj + kk * 2048u, MN_ATOM_BYTES, 1024u)
                                        : sdesc_sw128(aj + kk * 32u, 16u, 1024u);
-              mma_bf16(d_tmem + uint32_t(j) * BN, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+              mma(d_tmem + uint32_t(j) * BN, ad, bd, (kb | kk) != 0 ? 1u : 0u);
             }
           }
-          mma_commit(smem_u32(&ctl->empty[stage]));
+          commit(smem_u32(&ctl->empty[stage]));
           if (++stage == kStages) {
             stage = 0;
             phase ^= 1u;
           }
         }
         if (!ok) break;
-        mma_commit(smem_u32(&ctl->acc_full[acc]));
+        commit(smem_u32(&ctl->acc_full[acc]));
       }
     }
   } else {
@@ -280,7 +339,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int quad = warp & 3;  // TMEM lane quadrant this warp may access
     const int r = quad * 32 + lane;
     int local = 0;
-    for (int L = blockIdx.x; L < num_tiles; L += gridDim.x, ++local) {
+    for (int L = cl; L < num_tiles; L += ncl, ++local) {
       int m, n;
       tile_coords(L, p, nM, m, n);
       const int acc = kMT == 2 ? 0 : (local & 1);
@@ -292,7 +351,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (!ok) break;
       fence_after_sync();
       const uint32_t taddr = tmem_base + (uint32_t(quad * 32) << 16) + uint32_t(acc) * BN;
-      const int64_t row = int64_t(m) * kTM + r;
+      // this CTA's first row of the tile (M tile 0); M tile j starts BM * kCG rows further
+      const int64_t row0 = int64_t(m) * kTM + int64_t(rank) * BM;
+      const int64_t row = row0 + r;
       const bool row_ok = row < rows;
       const int64_t orig = (row_ok && p.row_idx) ? int64_t(__ldg(p.row_idx + row)) : row;
 
@@ -331,7 +392,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
         }
         fence_before_sync();
-        mbar_arrive(smem_u32(&ctl->acc_empty[acc]));
+        release_acc(acc);
         if (row_ok) {
           p.part[int64_t(n) * p.rows + row] = make_float2(mx, sm);  // compacted row, stride N
           if (have) p.zy[row] = zsel;
@@ -371,7 +432,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             tmem_wait_ld();
             if (c == BN / 32 - 1) {
               fence_before_sync();
-              mbar_arrive(smem_u32(&ctl->acc_empty[acc]));
+              release_acc(acc);
             }
             const int cbase = col0 + c * 32;
             const int valid = p.vocab - cbase;
@@ -418,8 +479,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
           fence_proxy_async_smem();
           named_barrier(EPI_BARRIER, 128);
-          if (issuer) {  // e is read again only by the backward: evict it first from L2
-            tma_store_2d_hint(&map_c, buf, col0 + box * 64, m * BM, l2_evict_first());
+          // (the odd CTA of a pair may hold no row of the last tile: nothing to store)
+          if (issuer && row0 < rows) {  // e is read again only by the backward: evict it first from L2
+            tma_store_2d_hint(&map_c, buf, col0 + box * 64, int(row0), l2_evict_first());
             bulk_commit_group();
           }
         }
@@ -458,7 +520,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             tmem_wait_ld();
             if (c == BN / 32 - 1) {
               fence_before_sync();
-              mbar_arrive(smem_u32(&ctl->acc_empty[acc]));
+              release_acc(acc);
             }
             const int lc = lc0 + c * 32;
             uint32_t pk[16];
@@ -486,8 +548,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
           fence_proxy_async_smem();
           named_barrier(EPI_BARRIER, 128);
-          if (issuer) {
-            tma_store_2d(&map_c, buf, lc0 + box * 64, m * BM);
+          if (issuer && row0 < rows) {
+            tma_store_2d(&map_c, buf, lc0 + box * 64, int(row0));
             bulk_commit_group();
           }
         }
@@ -496,7 +558,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // kMT == 2 the second M tile comes from the second accumulator
 #pragma unroll 1
         for (int j = 0; j < kMT; ++j) {
-        const int64_t rowj = row + int64_t(j) * BM;
+        const int64_t rowj = row + int64_t(j) * BM * kCG;
         const bool okj = rowj < rows;
         const int64_t origj = j == 0 ? orig : ((okj && p.row_idx) ? int64_t(__ldg(p.row_idx + rowj)) : rowj);
         const int64_t orow = p.c_row_off + origj;
@@ -560,7 +622,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         }
         fence_before_sync();
-        mbar_arrive(smem_u32(&ctl->acc_empty[acc]));
+        release_acc(acc);
       }
     }
   }
@@ -570,9 +632,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
   fence_before_sync();
   __syncthreads();
+  // neither CTA of a pair frees its TMEM or exits while the other may still
+  // reach its shared memory (copies counted on the even CTA's barriers,
+  // releases of its accumulators, commits to the odd CTA's barriers)
+  if constexpr (kCG == 2) cluster_sync();
   if (warp == 1) {
     fence_after_sync();
-    tmem_dealloc(tmem_base, TMEM_COLS);
+    if constexpr (kCG == 2)
+      tmem_dealloc_pair(tmem_base, TMEM_COLS);
+    else
+      tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
 
@@ -732,30 +801,94 @@ sao_status make_map(CUtensorMap *m, const void *ptr, uint64_t inner, uint64_t ou
   return SAO_OK;
 }
 
-template <int kEpi, bool kAMN, bool kBMN, int kMT = 1>
+template <int kEpi, bool kAMN, bool kBMN, int kMT = 1, int kCG = 1>
 sao_status launch_gemm(const char *name, const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &mc,
                        const GemmParams &p, cudaStream_t s) {
-  auto kern = tc_gemm_kernel<kEpi, kAMN, kBMN, kMT>;
+  auto kern = tc_gemm_kernel<kEpi, kAMN, kBMN, kMT, kCG>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
+  static int max_pairs = 0;  // CTA pairs that fit on the device at once
   std::call_once(once, [&] {
     attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(SMEM_BYTES));
+    if (attr_err == cudaSuccess && kCG == 2) {
+      cudaLaunchAttribute at[1];
+      at[0].id = cudaLaunchAttributeClusterDimension;
+      at[0].val.clusterDim.x = 2;
+      at[0].val.clusterDim.y = 1;
+      at[0].val.clusterDim.z = 1;
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(2);
+      cfg.blockDim = dim3(NUM_THREADS);
+      cfg.dynamicSmemBytes = SMEM_BYTES;
+      cfg.attrs = at;
+      cfg.numAttrs = 1;
+      attr_err = cudaOccupancyMaxActiveClusters(&max_pairs, kern, &cfg);
+    }
   });
-  if (attr_err != cudaSuccess) return fail(SAO_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(attr_err));
+  if (attr_err != cudaSuccess) return fail(SAO_ERR_CUDA, "kernel set-up: %s", cudaGetErrorString(attr_err));
   DeviceInfo di;
   SAO_TRY(device_info(&di));
   const int tiles = p.nM * p.nN;
   if (tiles == 0 || p.nK == 0) return SAO_OK;
-  const int grid = tiles < di.sm_count ? tiles : di.sm_count;
-  int slot = launch_begin(name, s);
-  kern<<<grid, NUM_THREADS, SMEM_BYTES, s>>>(ma, mb, mc, p);
-  return launch_end(slot, s);
+  if constexpr (kCG == 2) {
+    if (max_pairs < 1) return fail(SAO_ERR_UNSUPPORTED, "no CTA pair of the GEMM kernel fits on this device");
+    const int pairs = tiles < max_pairs ? tiles : max_pairs;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(2 * pairs));
+    cfg.blockDim = dim3(NUM_THREADS);
+    cfg.dynamicSmemBytes = SMEM_BYTES;
+    cfg.stream = s;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int slot = launch_begin(name, s);
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, ma, mb, mc, p);
+    if (e != cudaSuccess) return fail(SAO_ERR_CUDA, "cudaLaunchKernelEx (%s): %s", name, cudaGetErrorString(e));
+    return launch_end(slot, s);
+  } else {
+    const int grid = tiles < di.sm_count ? tiles : di.sm_count;
+    int slot = launch_begin(name, s);
+    kern<<<grid, NUM_THREADS, SMEM_BYTES, s>>>(ma, mb, mc, p);
+    return launch_end(slot, s);
+  }
+}
+
+// The same GEMM with kmt M tiles per CTA tile (plain store epilogues may take
+// two) on single CTAs (cg = 1) or CTA pairs (cg = 2).
+template <int kEpi, bool kAMN, bool kBMN>
+sao_status launch_gemm_cfg(const char *name, int kmt, int cg, const CUtensorMap &ma, const CUtensorMap &mb,
+                           const CUtensorMap &mc, const GemmParams &p, cudaStream_t s) {
+  if constexpr (kEpi == kStoreF32 || kEpi == kStoreBF16) {
+    if (kmt == 2)
+      return cg == 2 ? launch_gemm<kEpi, kAMN, kBMN, 2, 2>(name, ma, mb, mc, p, s)
+                     : launch_gemm<kEpi, kAMN, kBMN, 2, 1>(name, ma, mb, mc, p, s);
+  }
+  return cg == 2 ? launch_gemm<kEpi, kAMN, kBMN, 1, 2>(name, ma, mb, mc, p, s)
+                 : launch_gemm<kEpi, kAMN, kBMN, 1, 1>(name, ma, mb, mc, p, s);
 }
 
 // Two M tiles per CTA tile halve the re-reads of the shared operand but also
 // the number of tiles: worth it while at least four waves of tiles remain
 // (at 8k tokens dH has 176 paired tiles on 152 SMs and runs 15 % slower).
-bool pair_tiles(int64_t paired_tiles, int sms) { return paired_tiles >= 4 * int64_t(sms); }
+// `workers` = SMs, or SM pairs for CTA pairs.
+bool pair_tiles(int64_t paired_tiles, int workers) { return paired_tiles >= 4 * int64_t(workers); }
+
+// M tiles per CTA tile (1 or 2) for a long-K product with `rows` output rows
+// and `cols` output columns, and the tiles along M that gives.
+struct MTiles {
+  int kmt, nM;
+};
+MTiles m_tiles(int64_t rows, int cols, int cg, int sms) {
+  const int64_t per = int64_t(BM) * cg;
+  const int64_t nN = (cols + BN - 1) / BN;
+  const int64_t two = (rows + 2 * per - 1) / (2 * per);
+  if (pair_tiles(two * nN, sms / cg)) return MTiles{2, int(two)};
+  return MTiles{1, int((rows + per - 1) / per)};
+}
 
 // Rows per block (a multiple of 128, or N) and vocabulary columns per chunk (a
 // multiple of 256, or V rounded up to 256) of the recompute backward.
@@ -852,9 +985,11 @@ sao_status tc_fwd(const void *H, const void *W, const int32_t *y, const uint8_t 
     SAO_TRY(make_map(&ma, cr.Hc, uint64_t(h), uint64_t(cr.cap), uint64_t(h), 64, BM));
   else
     SAO_TRY(make_map(&ma, H, uint64_t(h), uint64_t(N), uint64_t(h), 64, BM));
-  SAO_TRY(make_map(&mb, W, uint64_t(h), uint64_t(V), uint64_t(h), 64, BN));
+  // CTA pairs: each CTA of a pair loads half of the 256-row W tile
+  const int cg = cta_group();
+  SAO_TRY(make_map(&mb, W, uint64_t(h), uint64_t(V), uint64_t(h), 64, BN / cg));
   GemmParams p{};
-  p.nM = int((N + BM - 1) / BM);
+  p.nM = int((N + BM * cg - 1) / (BM * cg));
   p.nN = nvt;
   p.nK = (h + BK - 1) / BK;
   // 64 row tiles per raster group (32 MB of H) stay in L2 while W streams: W is
@@ -892,9 +1027,9 @@ sao_status tc_fwd(const void *H, const void *W, const int32_t *y, const uint8_t 
     p.flag = cache->flag;
     CUtensorMap me;
     SAO_TRY(make_map(&me, cache->e, uint64_t(V), uint64_t(cache->rows), uint64_t(cache->lde), 64, BM));
-    SAO_TRY((launch_gemm<kSoftmaxStore, false, false>("tc_logits_lse_fwd", ma, mb, me, p, s)));
+    SAO_TRY((launch_gemm_cfg<kSoftmaxStore, false, false>("tc_logits_lse_fwd", 1, cg, ma, mb, me, p, s)));
   } else {
-    SAO_TRY((launch_gemm<kSoftmax, false, false>("tc_logits_lse_fwd", ma, mb, ma, p, s)));
+    SAO_TRY((launch_gemm_cfg<kSoftmax, false, false>("tc_logits_lse_fwd", 1, cg, ma, mb, ma, p, s)));
   }
   SAO_TRY(lse_merge_launch(part, nvt, zy, y, nullptr, row_mask ? cr.pos : nullptr, N, V, logp, lse, err, s));
   if (cache) {
@@ -934,10 +1069,10 @@ sao_status bwd_recompute_block(const void *H, const void *W, const int32_t *y, c
 
   CUtensorMap mHc_K, mW_K, mHc_MN, mW_MN;
   SAO_TRY(make_map(&mHc_K, cr.Hc, uint64_t(h), uint64_t(cr.cap), uint64_t(h), 64, BM));
-  SAO_TRY(make_map(&mW_K, W, uint64_t(h), uint64_t(V), uint64_t(h), 64, BN));
+  const int cg = cta_group();
+  SAO_TRY(make_map(&mW_K, W, uint64_t(h), uint64_t(V), uint64_t(h), 64, BN / cg));
   SAO_TRY(make_map(&mHc_MN, cr.Hc, uint64_t(h), uint64_t(cr.cap), uint64_t(h), 64, 64));
   SAO_TRY(make_map(&mW_MN, W, uint64_t(h), uint64_t(V), uint64_t(h), 64, 64));
-  const int nMt = int((N + BM - 1) / BM);
   DeviceInfo di;
   SAO_TRY(device_info(&di));
   const int sms = di.sm_count;
@@ -950,7 +1085,7 @@ sao_status bwd_recompute_block(const void *H, const void *W, const int32_t *y, c
     SAO_TRY(make_map(&mZ_MN, dz, uint64_t(vc), uint64_t(N), uint64_t(Vc), 64, 64));
     {  // dZ for vocabulary [v0, v0 + vc), compacted rows: recompute the logits
       GemmParams p{};
-      p.nM = nMt;
+      p.nM = int((N + BM * cg - 1) / (BM * cg));
       p.nN = (vc + BN - 1) / BN;
       p.nK = (h + BK - 1) / BK;
       p.group_m = 64;  // as the forward
@@ -967,12 +1102,12 @@ sao_status bwd_recompute_block(const void *H, const void *W, const int32_t *y, c
       p.err = err;
       p.m_count = cr.count;
       p.row_idx = cr.idx;
-      SAO_TRY((launch_gemm<kDLogits, false, false>(names.dlogits, mHc_K, mW_K, mZ_K, p, s)));
+      SAO_TRY((launch_gemm_cfg<kDLogits, false, false>(names.dlogits, 1, cg, mHc_K, mW_K, mZ_K, p, s)));
     }
     {  // dH (+)= dZ W[v0:v0+vc]: two 128-row tiles per CTA tile share each W stage when enough tiles remain
       GemmParams p{};
-      const bool pair = pair_tiles(int((N + 2 * BM - 1) / (2 * BM)) * ((h + BN - 1) / BN), sms);
-      p.nM = pair ? int((N + 2 * BM - 1) / (2 * BM)) : nMt;
+      const MTiles mt = m_tiles(N, h, cg, sms);
+      p.nM = mt.nM;
       p.nN = (h + BN - 1) / BN;
       p.nK = (vc + BK - 1) / BK;
       p.group_m = 1;
@@ -985,19 +1120,17 @@ sao_status bwd_recompute_block(const void *H, const void *W, const int32_t *y, c
       if (multi) {
         p.cf = dh_acc;  // compacted rows
         p.accumulate = first ? 0 : 1;
-        SAO_TRY((pair ? launch_gemm<kStoreF32, false, true, 2>(names.dH, mZ_K, mW_MN, mZ_K, p, s)
-                      : launch_gemm<kStoreF32, false, true, 1>(names.dH, mZ_K, mW_MN, mZ_K, p, s)));
+        SAO_TRY((launch_gemm_cfg<kStoreF32, false, true>(names.dH, mt.kmt, cg, mZ_K, mW_MN, mZ_K, p, s)));
       } else {
         p.cb = static_cast<__nv_bfloat16 *>(dH);
         p.row_idx = cr.idx;  // scatter to the original rows
-        SAO_TRY((pair ? launch_gemm<kStoreBF16, false, true, 2>(names.dH, mZ_K, mW_MN, mZ_K, p, s)
-                      : launch_gemm<kStoreBF16, false, true, 1>(names.dH, mZ_K, mW_MN, mZ_K, p, s)));
+        SAO_TRY((launch_gemm_cfg<kStoreBF16, false, true>(names.dH, mt.kmt, cg, mZ_K, mW_MN, mZ_K, p, s)));
       }
     }
     {  // dW[v0:v0+vc] (+)= dZ^T H over the compacted tokens: two 128-row vocabulary tiles per CTA tile
       GemmParams p{};
-      const bool pair = pair_tiles((vc + 2 * BM - 1) / (2 * BM) * ((h + BN - 1) / BN), sms);
-      p.nM = pair ? (vc + 2 * BM - 1) / (2 * BM) : (vc + BM - 1) / BM;
+      const MTiles mt = m_tiles(vc, h, cg, sms);
+      p.nM = mt.nM;
       p.nN = (h + BN - 1) / BN;
       p.nK = int((N + BK - 1) / BK);
       p.group_m = 1;
@@ -1009,8 +1142,7 @@ sao_status bwd_recompute_block(const void *H, const void *W, const int32_t *y, c
       p.accumulate = accumulate;
       p.err = err;
       p.k_count = cr.count;
-      SAO_TRY((pair ? launch_gemm<kStoreF32, true, true, 2>(names.dW, mZ_MN, mHc_MN, mZ_MN, p, s)
-                    : launch_gemm<kStoreF32, true, true, 1>(names.dW, mZ_MN, mHc_MN, mZ_MN, p, s)));
+      SAO_TRY((launch_gemm_cfg<kStoreF32, true, true>(names.dW, mt.kmt, cg, mZ_MN, mHc_MN, mZ_MN, p, s)));
     }
     if (multi && last)
       SAO_TRY(scatter_rows_to_bf16(dh_acc, h, cr.pos, cr.idx, cr.count, N, static_cast<__nv_bfloat16 *>(dH),
@@ -1070,10 +1202,11 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
   DeviceInfo di;
   SAO_TRY(device_info(&di));
   const int sms = di.sm_count;
+  const int cg = cta_group();
   {  // dH[t] = sc[f] (e W)[f], scattered to the tokens: two 128-row tiles per CTA tile share each W stage
     GemmParams p{};
-    const bool pair = pair_tiles(int((N + 2 * BM - 1) / (2 * BM)) * ((h + BN - 1) / BN), sms);
-    p.nM = pair ? int((N + 2 * BM - 1) / (2 * BM)) : int((N + BM - 1) / BM);
+    const MTiles mt = m_tiles(N, h, cg, sms);
+    p.nM = mt.nM;
     p.nN = (h + BN - 1) / BN;
     p.nK = (V + BK - 1) / BK;
     p.group_m = 1;
@@ -1085,13 +1218,12 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
     p.row_idx = cache->idx;
     p.row_scale = sc;
     p.cb = static_cast<__nv_bfloat16 *>(dH);
-    SAO_TRY((pair ? launch_gemm<kStoreBF16, false, true, 2>("tc_dH_gemm", mE_K, mW_MN, mE_K, p, s)
-                  : launch_gemm<kStoreBF16, false, true, 1>("tc_dH_gemm", mE_K, mW_MN, mE_K, p, s)));
+    SAO_TRY((launch_gemm_cfg<kStoreBF16, false, true>("tc_dH_gemm", mt.kmt, cg, mE_K, mW_MN, mE_K, p, s)));
   }
   {  // dW (+)= e^T (sc H) over the forward rows: two 128-row vocabulary tiles per CTA tile
     GemmParams p{};
-    const bool pair = pair_tiles((V + 2 * BM - 1) / (2 * BM) * ((h + BN - 1) / BN), sms);
-    p.nM = pair ? (V + 2 * BM - 1) / (2 * BM) : (V + BM - 1) / BM;
+    const MTiles mt = m_tiles(V, h, cg, sms);
+    p.nM = mt.nM;
     p.nN = (h + BN - 1) / BN;
     p.nK = int((N + BK - 1) / BK);
     p.group_m = 1;
@@ -1102,8 +1234,7 @@ sao_status tc_bwd(const void *H, const void *W, const int32_t *y, const float *l
     p.accumulate = accumulate;
     p.err = err;
     p.k_count = cache->count;
-    SAO_TRY((pair ? launch_gemm<kStoreF32, true, true, 2>("tc_dW_gemm", mE_MN, mHs_MN, mE_MN, p, s)
-                  : launch_gemm<kStoreF32, true, true, 1>("tc_dW_gemm", mE_MN, mHs_MN, mE_MN, p, s)));
+    SAO_TRY((launch_gemm_cfg<kStoreF32, true, true>("tc_dW_gemm", mt.kmt, cg, mE_MN, mHs_MN, mE_MN, p, s)));
   }
   // Flagged rows (a sampled token more than kFlagExponent - kKappaOffset nats
   // below its row's maximum) got sc = 0 above: recompute their logits, write

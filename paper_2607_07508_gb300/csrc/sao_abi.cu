@@ -17,6 +17,10 @@ static std::atomic<size_t> g_dz_budget{size_t(4) << 30};
 void set_dz_budget(size_t bytes) { g_dz_budget.store(bytes < (size_t(1) << 20) ? (size_t(1) << 20) : bytes); }
 size_t dz_budget() { return g_dz_budget.load(); }
 
+static std::atomic<int> g_cta_pairs{0};
+void set_cta_pairs(int on) { g_cta_pairs.store(on ? 1 : 0); }
+int cta_group() { return g_cta_pairs.load() ? 2 : 1; }
+
 static std::atomic<uint64_t> g_scan_wait_ns{kWaitLimitNs};
 static std::atomic<int> g_scan_skip{0};
 uint64_t scan_wait_ns() { return g_scan_wait_ns.load(); }
@@ -105,6 +109,9 @@ int sao_get_checked(void) { return checked_mode() ? 1 : 0; }
 
 void sao_set_dz_budget_bytes(size_t bytes) { set_dz_budget(bytes); }
 size_t sao_get_dz_budget_bytes(void) { return dz_budget(); }
+
+void sao_set_cta_pairs(int on) { set_cta_pairs(on); }
+int sao_get_cta_pairs(void) { return cta_group() == 2 ? 1 : 0; }
 
 void sao_debug_set_scan_hooks(uint64_t wait_ns, int32_t skip_chunks) {
   g_scan_wait_ns.store(wait_ns == 0 ? kWaitLimitNs : (wait_ns > kWaitLimitNs ? kWaitLimitNs : wait_ns));

@@ -63,6 +63,9 @@ sao_status logprobs_bwd_launch(const void *H, const void *W, sao_dtype dt, const
 
 void set_dz_budget(size_t bytes);
 size_t dz_budget();
+// GEMM tiling of the tensor-core path: 1 = single CTAs, 2 = CTA pairs.
+void set_cta_pairs(int on);
+int cta_group();
 
 // Test hooks of the advantage scan (see sao_debug_set_scan_hooks in sao.h).
 uint64_t scan_wait_ns();

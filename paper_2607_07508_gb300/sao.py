@@ -26,7 +26,8 @@ FLAG_IN, FLAG_LOW, FLAG_HIGH, FLAG_NONFINITE, FLAG_NOT_ACTION = 0, 1, 2, 3, 4
 FLAG_MISMATCH_LOW, FLAG_MISMATCH_HIGH = 5, 6
 
 EXPORTS = ("sao_version", "sao_last_error_string", "sao_set_checked", "sao_get_checked",
-           "sao_set_dz_budget_bytes", "sao_get_dz_budget_bytes", "sao_debug_set_scan_hooks", "sao_workspace_bytes", "sao_token_logprobs_fwd",
+           "sao_set_dz_budget_bytes", "sao_get_dz_budget_bytes", "sao_set_cta_pairs", "sao_get_cta_pairs",
+           "sao_debug_set_scan_hooks", "sao_workspace_bytes", "sao_token_logprobs_fwd",
            "sao_token_logprobs_bwd", "sao_advantages", "sao_advantages_noalloc", "sao_step_advantages",
            "sao_policy_loss_fwd", "sao_policy_loss_bwd", "sao_clip_loss_fwd", "sao_clip_loss_bwd",
            "sao_group_advantages", "sao_running_mean_advantages", "sao_decoupled_loss_fwd",
@@ -62,6 +63,8 @@ def load(path: Optional[str] = None):
         "sao_get_checked": (ctypes.c_int, []),
         "sao_set_dz_budget_bytes": (None, [SZ]),
         "sao_get_dz_budget_bytes": (SZ, []),
+        "sao_set_cta_pairs": (None, [ctypes.c_int]),
+        "sao_get_cta_pairs": (ctypes.c_int, []),
         "sao_debug_set_scan_hooks": (None, [ctypes.c_uint64, I32]),
         "sao_workspace_bytes": (SZ, [I64, I32, I32, ctypes.c_int]),
         "sao_logprob_cache_bytes": (SZ, [I64, I32]),
@@ -156,6 +159,14 @@ def sao_set_dz_budget_bytes(nbytes: int):
 
 def sao_get_dz_budget_bytes() -> int:
     return int(load().sao_get_dz_budget_bytes())
+
+
+def sao_set_cta_pairs(on: bool):
+    load().sao_set_cta_pairs(1 if on else 0)
+
+
+def sao_get_cta_pairs() -> bool:
+    return bool(load().sao_get_cta_pairs())
 
 
 def sao_debug_set_scan_hooks(wait_ns: int = 0, skip_chunks: int = 0):
