@@ -406,7 +406,7 @@ def workload_config(wl, cached=False):
 
 
 # Algorithmic bytes per token of each O(N) kernel (reads + writes).
-ON_BYTES = {"gae_scan": 13, "policy_loss_fwd": 18, "policy_loss_bwd": 17, "value_loss": 13, "count_mask": 1,
+ON_BYTES = {"gae_scan": 13, "gae_telescoped": 13, "policy_loss_fwd": 18, "policy_loss_bwd": 17, "value_loss": 13, "count_mask": 1,
             "gae_count": 1, "decoupled_loss_fwd": 22, "decoupled_loss_bwd": 21}
 
 
@@ -461,6 +461,8 @@ def bandwidth_study(args):
     whole = {
         "sao_advantages": (13, lambda: sao.sao_advantages(v, R, m, cu, wl.gamma, wl.lam, wl.lam_critic, 0.0,
                                                           adv, ret, ws)),
+        "sao_advantages (gamma = lambda = 1)": (13, lambda: sao.sao_advantages(v, R, m, cu, 1.0, 1.0, 1.0, 0.0,
+                                                                               adv, ret, ws)),
         "sao_step_advantages": (14, lambda: sao.sao_step_advantages(v, R, m, cu, wl.gamma, wl.lam, wl.lam_critic,
                                                                     0.0, sao.SAO_STEP_AVERAGE, adv, ret, ws,
                                                                     value_mask=vm)),

@@ -355,9 +355,12 @@ SAO_API sao_status sao_decoupled_loss_bwd(const float *logp, const float *prox_l
  * fit (for example 2^25 tokens with up to 65,536 trajectories); larger
  * inputs return SAO_ERR_SHAPE with the bytes needed. Nothing is allocated
  * and nothing is freed.
- * The first call on each device looks up the array's device address (with
- * that device current) and caches it; make that first call before any stream
- * capture. Every call on a device shares the one array, so calls that overlap
+ * Each call made outside stream capture looks up the array's device address
+ * (with the calling thread's current device) and remembers it for that
+ * device, so a device reset or a new primary context is picked up; a call
+ * under stream capture uses the remembered address and returns
+ * SAO_ERR_INVALID_ARG if no call on that device came before the capture.
+ * Every call on a device shares the one array, so calls that overlap
  * on the GPU (two streams, or two threads) race and corrupt each other's
  * results; serialise them. Each call clears the parts of the array that must
  * start at zero, so stale contents from a previous call do no harm.

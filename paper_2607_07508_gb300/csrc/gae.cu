@@ -856,6 +856,19 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
       cu, B, N, int(nchunks), chunk_first);
     SAO_TRY(launch_end(slot, s));
   }
+  if (gamma == 1.0f && lam == 1.0f && lam_c == 1.0f && !(alpha > 0.f)) {
+    // gamma = lambda = 1: every delta telescopes, A = R_b - V on the action
+    // tokens and the return is R_b, exactly what the scan would produce (its
+    // double-float lambda-return is R_b itself): one streaming pass, after
+    // the coefficient kernel's check of cu_seqlens
+    int slot = launch_begin("gae_coef", s);
+    gae_coef_kernel<<<(B + 127) / 128, 128, 0, s>>>(cu, B, N, gamma, lam, lam_c, alpha, nact, coef, err);
+    SAO_TRY(launch_end(slot, s));
+    slot = launch_begin("gae_telescoped", s);
+    seg::traj_broadcast_kernel<true><<<seg::action_count_grid(int(nchunks)), 256, 0, s>>>(
+        rewards, m, cu, B, N, int(nchunks), chunk_first, adv, values, ret);
+    return launch_end(slot, s);
+  }
   if (alpha > 0.f) {
     int slot = launch_begin("gae_count", s);
     seg::action_count_kernel<<<seg::action_count_grid(int(nchunks)), 256, 0, s>>>(m, cu, B, N, int(nchunks),

@@ -25,22 +25,38 @@ std::mutex g_scratch_mu;
 std::vector<DeviceScratch> g_scratch_ptrs;
 
 // Device address of g_noalloc_scratch on the current device. Host code only
-// sees a host-side stand-in for the array's name, so the address is looked up
-// once per device (with that device current) and cached.
-sao_status scratch_address(void **out) {
+// sees a host-side stand-in for the array's name, so the address comes from
+// cudaGetSymbolAddress with the device current. Outside stream capture it is
+// looked up again on every call (a device reset or a new primary context
+// reloads the module and can move the array) and remembered per device;
+// under capture the remembered address is used, so the first call on a
+// device must come before any capture.
+sao_status scratch_address(cudaStream_t stream, void **out) {
   int dev = 0;
   SAO_CUDA_TRY(cudaGetDevice(&dev));
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  SAO_CUDA_TRY(cudaStreamIsCapturing(stream, &cs));
   std::lock_guard<std::mutex> lk(g_scratch_mu);
-  for (const auto &d : g_scratch_ptrs)
-    if (d.device == dev) {
-      *out = d.ptr;
-      return SAO_OK;
-    }
+  DeviceScratch *known = nullptr;
+  for (auto &d : g_scratch_ptrs)
+    if (d.device == dev) known = &d;
+  if (cs != cudaStreamCaptureStatusNone) {
+    if (!known)
+      return fail(SAO_ERR_INVALID_ARG,
+                  "sao_advantages_noalloc: the first call on device %d is under stream capture; make one call "
+                  "before capturing",
+                  dev);
+    *out = known->ptr;
+    return SAO_OK;
+  }
   void *p = nullptr;
   const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
   if (e != cudaSuccess || p == nullptr)
     return fail(SAO_ERR_CUDA, "cudaGetSymbolAddress of the static scratch failed: %s", cudaGetErrorString(e));
-  g_scratch_ptrs.push_back({dev, p});
+  if (known)
+    known->ptr = p;
+  else
+    g_scratch_ptrs.push_back({dev, p});
   *out = p;
   return SAO_OK;
 }
@@ -65,7 +81,7 @@ extern "C" sao_status sao_advantages_noalloc(const float *values, const float *r
   if (N == 0) return sao_advantages(values, rewards, loss_mask, cu_seqlens, B, N, gamma, lambda_policy,
                                     lambda_critic, len_adaptive_alpha, adv, ret, nullptr, 0, stream);
   void *scratch = nullptr;
-  SAO_TRY(scratch_address(&scratch));
+  SAO_TRY(scratch_address(reinterpret_cast<cudaStream_t>(stream), &scratch));
   return sao_advantages(values, rewards, loss_mask, cu_seqlens, B, N, gamma, lambda_policy, lambda_critic,
                         len_adaptive_alpha, adv, ret, scratch, kNoAllocScratchBytes, stream);
 }

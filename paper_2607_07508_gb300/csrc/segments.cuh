@@ -172,9 +172,15 @@ __global__ void __launch_bounds__(256) action_count_kernel(const uint8_t *m, con
 // grid as action_count_kernel: kCountChunks chunks per warp; in 128-token
 // groups lane l takes 4 tokens (a 4-byte mask load, a float4 store); a group
 // inside the lane's current trajectory takes no per-token work.
+// kValues: also ret[t] = a_traj[b] and adv[t] = a_traj[b] - values[t] on the
+// action tokens (0 elsewhere): the GAE of a trajectory whose recursion
+// telescopes (gamma = lambda = 1: the advantage is its reward minus the
+// value, the return its reward), with the values read by float4 as well.
+template <bool kValues>
 __global__ void __launch_bounds__(256) traj_broadcast_kernel(const float *a_traj, const uint8_t *m,
                                                              const int32_t *cu_g, int B, int64_t N, int nchunks,
-                                                             const int *chunk_first, float *adv) {
+                                                             const int *chunk_first, float *adv,
+                                                             const float *values, float *ret) {
   __shared__ int32_t s_cu_all[8][kCuCap];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int q0 = (blockIdx.x * 8 + warp) * kCountChunks;
@@ -192,7 +198,9 @@ __global__ void __launch_bounds__(256) traj_broadcast_kernel(const float *a_traj
   int b = blo;
   int64_t next_end = cu[b + 1];
   float v = __ldg(a_traj + b);
-  const bool aligned = ((reinterpret_cast<uintptr_t>(m) | reinterpret_cast<uintptr_t>(adv)) & 15u) == 0;
+  uintptr_t al = reinterpret_cast<uintptr_t>(m) | reinterpret_cast<uintptr_t>(adv);
+  if (kValues) al |= reinterpret_cast<uintptr_t>(values) | reinterpret_cast<uintptr_t>(ret);
+  const bool aligned = (al & 15u) == 0;
   // 128-token groups: lane l takes tokens 4l .. 4l+3, so each warp load reads
   // 128 contiguous bytes and each warp store writes 512; the mask words of 8
   // groups are loaded together, so a warp waits for one load latency per
@@ -200,10 +208,13 @@ __global__ void __launch_bounds__(256) traj_broadcast_kernel(const float *a_traj
 #pragma unroll 1
   for (int64_t base = c0; base < c1; base += 8 * 128) {
     uint32_t u[8];
+    float4 x[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const int64_t t0 = base + j * 128 + int64_t(lane) * 4;
-      u[j] = (aligned && t0 + 4 <= c1) ? __ldg(reinterpret_cast<const uint32_t *>(m + t0)) : 0u;
+      const bool full = aligned && t0 + 4 <= c1;
+      u[j] = full ? __ldg(reinterpret_cast<const uint32_t *>(m + t0)) : 0u;
+      if (kValues) x[j] = full ? __ldcs(reinterpret_cast<const float4 *>(values + t0)) : make_float4(0.f, 0.f, 0.f, 0.f);
     }
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
@@ -211,9 +222,18 @@ __global__ void __launch_bounds__(256) traj_broadcast_kernel(const float *a_traj
       if (t0 >= c1) break;
       if (aligned && t0 + 4 <= c1 && t0 + 4 <= next_end) {  // all 4 tokens in trajectory b
         const uint32_t w = u[j];
-        __stcs(reinterpret_cast<float4 *>(adv + t0), make_float4((w & 0xffu) ? v : 0.f, (w & 0xff00u) ? v : 0.f,
-                                                                 (w & 0xff0000u) ? v : 0.f,
-                                                                 (w & 0xff000000u) ? v : 0.f));
+        const bool a0 = (w & 0xffu) != 0u, a1 = (w & 0xff00u) != 0u, a2 = (w & 0xff0000u) != 0u,
+                   a3 = (w & 0xff000000u) != 0u;
+        if (kValues) {
+          __stcs(reinterpret_cast<float4 *>(adv + t0),
+                 make_float4(a0 ? __fsub_rn(v, x[j].x) : 0.f, a1 ? __fsub_rn(v, x[j].y) : 0.f,
+                             a2 ? __fsub_rn(v, x[j].z) : 0.f, a3 ? __fsub_rn(v, x[j].w) : 0.f));
+          __stcs(reinterpret_cast<float4 *>(ret + t0), make_float4(a0 ? v : 0.f, a1 ? v : 0.f, a2 ? v : 0.f,
+                                                                   a3 ? v : 0.f));
+        } else {
+          __stcs(reinterpret_cast<float4 *>(adv + t0), make_float4(a0 ? v : 0.f, a1 ? v : 0.f, a2 ? v : 0.f,
+                                                                   a3 ? v : 0.f));
+        }
         continue;
       }
       for (int k = 0; k < 4; ++k) {
@@ -226,7 +246,13 @@ __global__ void __launch_bounds__(256) traj_broadcast_kernel(const float *a_traj
           }
           v = __ldg(a_traj + b);
         }
-        adv[t] = m[t] ? v : 0.f;
+        const bool act = m[t] != 0;
+        if (kValues) {
+          adv[t] = act ? __fsub_rn(v, values[t]) : 0.f;
+          ret[t] = act ? v : 0.f;
+        } else {
+          adv[t] = act ? v : 0.f;
+        }
       }
     }
   }

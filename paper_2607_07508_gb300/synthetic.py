@@ -310,11 +310,17 @@ def bandwidth_workload(N: int = 1 << 27, B: int = 1 << 14, seed: int = SEED_BASE
     med = max(16, N // B // 2)
     lengths = lognormal_lengths(rng, N, med, max(64, 16 * med))
     B = len(lengths)
-    # cheap vectorised turn mask: flip between action/observation every ~256 tokens
-    flips = rng.random(N) < (1.0 / 256.0)
-    phase = np.cumsum(flips) & 1
-    obs = (phase == 1) & (rng.random(N) < 2.0 / 3.0)
-    mask = (~obs).astype(np.uint8)
+    # alternating action / observation turns as in the five configurations
+    # (geometric spans, action mean 256 tokens, observation mean 128: one
+    # third observation tokens), drawn vectorised over the whole batch
+    n_turns = 2 * (N // 384 + 64)
+    spans = np.empty(n_turns, np.int64)
+    spans[0::2] = rng.geometric(1.0 / 256.0, size=n_turns // 2)
+    spans[1::2] = rng.geometric(1.0 / 128.0, size=n_turns // 2)
+    while spans.sum() < N:
+        spans = np.concatenate([spans, spans])
+    kind = np.tile(np.array([1, 0], np.uint8), len(spans) // 2)
+    mask = np.repeat(kind, spans)[:N]
     values = rng.standard_normal(N, dtype=np.float32) * np.float32(0.2) + np.float32(0.4)
     rewards = (rng.random(B) < 0.4).astype(np.float32)
     xi = rng.standard_normal(N, dtype=np.float32) * np.float32(0.1)

@@ -71,6 +71,33 @@ def test_advantages_edge_layouts(lengths):
     assert rel_err_floor(ret, want_r, 1e-3).max() <= ADV_TOL
 
 
+@pytest.mark.parametrize("lengths", [[1], [5, 0, 0, 7], [0, 4096, 1, 4095, 0], [4097, 13, 8190],
+                                     [3] * 2000, [70001], [0, 0, 17, 0]])
+@pytest.mark.parametrize("offset", [0, 1])
+def test_advantages_telescoped_edge_layouts(lengths, offset):
+    """gamma = lambda = lambda_critic = 1 (no length-adaptive lambda) takes the
+    one-pass telescoped kernel: ragged layouts, empty trajectories and
+    trajectories without action tokens, with 16-byte aligned and misaligned
+    (one element off) inputs and outputs."""
+    wl = S.make_custom(lengths, 8, 16, "f32", seed=sum(lengths) + 7 * len(lengths), dense=False, obs_frac=0.4)
+    wl.loss_mask[::97] = 0
+    N = wl.N
+
+    def shifted(a, dtype):
+        t = torch.zeros(N + offset, dtype=dtype, device="cuda")
+        t[offset:] = torch.as_tensor(a).to(dtype).cuda()
+        return t[offset:]
+
+    v, m = shifted(wl.values, torch.float32), shifted(wl.loss_mask, torch.uint8)
+    adv = torch.full((N + offset,), float("nan"), device="cuda")[offset:]
+    ret = torch.full((N + offset,), float("nan"), device="cuda")[offset:]
+    sao.sao_advantages(v, cuda(wl.rewards), m, cuda(wl.cu_seqlens), 1.0, 1.0, 1.0, 0.0, adv, ret, sao.workspace(N))
+    torch.cuda.synchronize()
+    want_a, want_r = O.advantages(wl.values, wl.rewards, wl.loss_mask, wl.cu_seqlens, 1.0, 1.0, 1.0, 0.0)
+    assert rel_err_floor(adv.cpu().numpy(), want_a, 1e-3).max() <= ADV_TOL
+    assert rel_err_floor(ret.cpu().numpy(), want_r, 1e-3).max() <= ADV_TOL
+
+
 def test_advantages_no_action_tokens_and_empty():
     wl = S.make_custom([10, 0, 300], 8, 16, "f32", seed=3, dense=False)
     wl.loss_mask[:] = 0
