@@ -343,9 +343,11 @@ struct GaeArgs {
   const int32_t *cu;
   int B;
   int64_t N;
-  int nchunks;
+  int nchunks;             // scan chunks of 32 lanes x seg tokens
+  int pieces;              // 32-token pieces per lane segment (1, 2, 4 or 8)
+  int nsub;                // 1024-token sub-chunks, the units of chunk_first
   const float4 *coef;      // [B][2]
-  const int *chunk_first;  // [nchunks] trajectory of each chunk's first token
+  const int *chunk_first;  // [nsub] trajectory of each 1024-token sub-chunk's first token
   int *ticket;
   uint64_t *agg;           // [nchunks][kMapWords]: map of the whole chunk
   uint64_t *incl;          // [nchunks][kStateWords]: state at the chunk's left edge
@@ -407,71 +409,94 @@ __device__ GState look_back(const GaeArgs &a, int q, int lane) {
 // ---------------------------------------------------------------------------
 // per-warp staging in shared memory
 // ---------------------------------------------------------------------------
-// Row r holds lane r's 32 tokens. val/ret rows are 8 granules of 16 bytes,
-// granule j stored at 8r + (j ^ (r & 7)); msk rows are 2 granules, granule j
-// at 2r + (j ^ ((r >> 2) & 1)). A quarter-warp (8 lanes) then touches 8
-// distinct bank groups both when it copies 8 consecutive granules of the chunk
-// and when 8 lanes read the same granule of their own rows.
-// A warp keeps two chunks: the one it folds and the one waiting for its
-// look-back; values arrive in val[buf] and leave as advantages.
+// A scan chunk is 32 lane segments of seg = 32 * pieces consecutive tokens;
+// lane r's segment starts at chunk offset r * seg. The segments stream
+// through shared memory one 32-token piece at a time (right to left): row r
+// of a staged piece holds lane r's 32 tokens of that piece. val/ret rows are
+// 8 granules of 16 bytes, granule j stored at 8r + (j ^ (r & 7)); msk rows are
+// 2 granules, granule j at 2r + (j ^ ((r >> 2) & 1)). A quarter-warp (8
+// lanes) then touches 8 distinct bank groups both when it copies the 8
+// granules (128 contiguous bytes of global memory) of one row and when 8 lanes
+// read the same granule of their own rows. With one piece per segment the
+// two value buffers hold two chunks, the one folded last and the one waiting
+// for its look-back and replay (values in, advantages out). With several, they
+// hold the piece being worked on and the next one, copied meanwhile, and the
+// replay copies its chunk's pieces again (a chunk no longer fits).
 struct __align__(16) WarpBuf {
-  float val[2][kChunk];  // values in, advantages out
-  float ret[kChunk];     // returns of the chunk being replayed
-  uint8_t msk[kChunk];   // action flags of the chunk being folded
+  float val[2][kChunk];  // values in, advantages out (two pieces)
+  float ret[kChunk];     // returns of the piece being replayed
+  uint8_t msk[kChunk];   // action flags of the next piece
   int32_t cu[kCuCap];    // cu_seqlens slice of the chunk being folded
 };
 __device__ __forceinline__ int fgran(int r, int j) { return 8 * r + (j ^ (r & 7)); }
 __device__ __forceinline__ int mgran(int r, int j) { return 2 * r + (j ^ ((r >> 2) & 1)); }
 
-__device__ __forceinline__ void cp_async16(void *smem, const void *gmem) {
+// 16-byte copy global -> shared through L2 only, with an L2 eviction policy
+__device__ __forceinline__ void cp_async16(void *smem, const void *gmem, uint64_t policy) {
   const unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(s), "l"(gmem) : "memory");
+  asm volatile("cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2;" ::"r"(s), "l"(gmem), "l"(policy)
+               : "memory");
+}
+// The fold's copy keeps its lines in L2 for the replay's copy of the same
+// chunk (issued about two chunk-times later), which drops them.
+__device__ __forceinline__ uint64_t l2_policy(bool keep) {
+  uint64_t p;
+  if (keep)
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  else
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
 }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
-// Starts the copy of the chunk's values and flags (asynchronous for a full,
-// aligned chunk; element by element, zero-filled past N, otherwise).
-__device__ __forceinline__ void stage_in(const GaeArgs &a, int64_t c0, int lane, float *val, uint8_t *msk) {
+// Starts the copy of piece k of the chunk at c0 (lane r's tokens c0 + r * seg
+// + 32k ..): asynchronous when the piece lies below N for every lane and the
+// inputs are 16-byte aligned, element by element (zero past N) otherwise.
+__device__ __forceinline__ void stage_in(const GaeArgs &a, int64_t c0, int seg, int k, int lane, float *val,
+                                         uint8_t *msk, uint64_t policy) {
   const int64_t N = a.N;
-  if (c0 + kChunk <= N && aligned16_dev(a.values) && aligned16_dev(a.m)) {
+  const int64_t off = c0 + 32 * int64_t(k);
+  if (off + 31 * int64_t(seg) + 32 <= N && aligned16_dev(a.values) && aligned16_dev(a.m)) {
 #pragma unroll
     for (int it = 0; it < 8; ++it) {
-      const int G = it * 32 + lane;
-      cp_async16(&val[4 * fgran(G >> 3, G & 7)], a.values + c0 + 4 * G);
+      const int G = it * 32 + lane, r = G >> 3, j = G & 7;
+      cp_async16(&val[4 * fgran(r, j)], a.values + off + int64_t(r) * seg + 4 * j, policy);
     }
 #pragma unroll
     for (int it = 0; it < 2; ++it) {
-      const int G = it * 32 + lane;
-      cp_async16(&msk[16 * mgran(G >> 1, G & 1)], a.m + c0 + 16 * G);
+      const int G = it * 32 + lane, r = G >> 1, j = G & 1;
+      cp_async16(&msk[16 * mgran(r, j)], a.m + off + int64_t(r) * seg + 16 * j, policy);
     }
   } else {
     for (int i = lane; i < kChunk; i += 32) {
-      const int64_t t = c0 + i;
-      const int r = i >> 5, k = i & 31;
-      val[4 * fgran(r, k >> 2) + (k & 3)] = t < N ? a.values[t] : 0.f;
-      msk[16 * mgran(r, k >> 4) + (k & 15)] = (t < N && a.m[t] != 0) ? 1 : 0;
+      const int r = i >> 5, kk = i & 31;
+      const int64_t t = off + int64_t(r) * seg + kk;
+      val[4 * fgran(r, kk >> 2) + (kk & 3)] = t < N ? a.values[t] : 0.f;
+      msk[16 * mgran(r, kk >> 4) + (kk & 15)] = (t < N && a.m[t] != 0) ? 1 : 0;
     }
   }
 }
 
-__device__ __forceinline__ void stage_out(const GaeArgs &a, int64_t c0, int lane, const float *val,
+__device__ __forceinline__ void stage_out(const GaeArgs &a, int64_t c0, int seg, int k, int lane, const float *val,
                                           const float *ret) {
   const int64_t N = a.N;
-  if (c0 + kChunk <= N && aligned16_dev(a.adv) && aligned16_dev(a.ret)) {
+  const int64_t off = c0 + 32 * int64_t(k);
+  if (off + 31 * int64_t(seg) + 32 <= N && aligned16_dev(a.adv) && aligned16_dev(a.ret)) {
 #pragma unroll
     for (int it = 0; it < 8; ++it) {
-      const int G = it * 32 + lane;
-      const int p = 4 * fgran(G >> 3, G & 7);
-      __stcs(reinterpret_cast<float4 *>(a.adv + c0) + G, *reinterpret_cast<const float4 *>(&val[p]));
-      __stcs(reinterpret_cast<float4 *>(a.ret + c0) + G, *reinterpret_cast<const float4 *>(&ret[p]));
+      const int G = it * 32 + lane, r = G >> 3, j = G & 7;
+      const int p = 4 * fgran(r, j);
+      const int64_t t = off + int64_t(r) * seg + 4 * j;
+      __stcs(reinterpret_cast<float4 *>(a.adv + t), *reinterpret_cast<const float4 *>(&val[p]));
+      __stcs(reinterpret_cast<float4 *>(a.ret + t), *reinterpret_cast<const float4 *>(&ret[p]));
     }
   } else {
     for (int i = lane; i < kChunk; i += 32) {
-      const int64_t t = c0 + i;
-      const int r = i >> 5, k = i & 31;
+      const int r = i >> 5, kk = i & 31;
+      const int64_t t = off + int64_t(r) * seg + kk;
       if (t < N) {
-        a.adv[t] = val[4 * fgran(r, k >> 2) + (k & 3)];
-        a.ret[t] = ret[4 * fgran(r, k >> 2) + (k & 3)];
+        a.adv[t] = val[4 * fgran(r, kk >> 2) + (kk & 3)];
+        a.ret[t] = ret[4 * fgran(r, kk >> 2) + (kk & 3)];
       }
     }
   }
@@ -483,12 +508,41 @@ __device__ __forceinline__ uint32_t nonzero_bytes(uint32_t x) {
   return (h * 0x00204081u) >> 28;
 }
 
+// Action-token bits of the lane's staged row (bit k: token k of the piece).
+__device__ __forceinline__ uint32_t row_actions(const uint8_t *msk, int lane) {
+  const uint4 m0 = *reinterpret_cast<const uint4 *>(&msk[16 * mgran(lane, 0)]);
+  const uint4 m1 = *reinterpret_cast<const uint4 *>(&msk[16 * mgran(lane, 1)]);
+  return nonzero_bytes(m0.x) | nonzero_bytes(m0.y) << 4 | nonzero_bytes(m0.z) << 8 | nonzero_bytes(m0.w) << 12 |
+         nonzero_bytes(m1.x) << 16 | nonzero_bytes(m1.y) << 20 | nonzero_bytes(m1.z) << 24 |
+         nonzero_bytes(m1.w) << 28;
+}
+
+// Trajectory ends among the 32 tokens from t0 (bit e: token t0 + e is the last
+// token of its trajectory), by a forward walk over cu_seqlens; b_last is the
+// trajectory of the last of those tokens below N. No bits past N.
+__device__ __forceinline__ uint32_t piece_ends(const GaeArgs &a, const CuView &cu, int blo, int bhi, int64_t t0,
+                                               int &b_last) {
+  uint32_t ends = 0;
+  b_last = blo;
+  if (t0 >= a.N) return 0;
+  const int64_t tl = (t0 + kItems <= a.N ? int64_t(kItems) : a.N - t0) - 1;  // last token, relative to t0
+  int b = cu.find(blo, bhi, t0);
+  for (;;) {
+    const int64_t e = cu[b + 1] - 1 - t0;  // last token of trajectory b, relative to t0
+    if (e >= 0 && e <= tl) ends |= 1u << e;
+    if (e >= tl || b >= bhi) break;  // b holds the piece's last token (or cu_seqlens is malformed)
+    ++b;
+  }
+  b_last = b;
+  return ends;
+}
+
 // ---------------------------------------------------------------------------
 // per-lane fold and replay
 // ---------------------------------------------------------------------------
-// The lane's tokens are t0 .. t0+31; bit k of `act` / `ends`: token t0+k is an
+// A piece's tokens are t0 .. t0+31; bit k of `act` / `ends`: token t0+k is an
 // action token / the last token of its trajectory; b_last is the trajectory of
-// the lane's last token below N.
+// the piece's last token below N.
 
 // The token loops below take 4 tokens at a time. A group in which no lane of
 // the warp holds a trajectory end or a waiting reward (the common case: turns
@@ -496,14 +550,25 @@ __device__ __forceinline__ uint32_t nonzero_bytes(uint32_t x) {
 // double-float a*B + g*V per token with the action flag applied by selects;
 // otherwise the warp takes the general path for that group.
 
-// Map of the lane's 32 tokens.
+// A lane's fold of its segment so far (the pieces right of the current one):
+// the lambda-returns with a zero state at the segment's right edge, the value
+// of the leftmost action token folded, the reward still waiting, the map
+// flags and the number of action tokens.
 template <bool kCrit>
-__device__ GMap<kCrit> fold_lane(const GaeArgs &a, const float *val, int lane, uint32_t act, uint32_t ends,
-                                 int64_t t0, const CuView &cu, int blo, int b_last) {
-  Coefs<kCrit> k = load_coefs<kCrit>(a.coef, b_last);
-  df Bp = {0.f, 0.f}, Bc = {0.f, 0.f};
-  float Vn = 0.f, P = 0.f;
-  int fl = 0, n = 0;
+struct FoldState {
+  Coefs<kCrit> k;
+  df Bp, Bc;
+  float Vn, P;
+  int fl, nact;
+};
+
+template <bool kCrit>
+__device__ void fold_piece(const GaeArgs &a, const float *val, int lane, uint32_t act, uint32_t ends, int64_t t0,
+                           const CuView &cu, int blo, int b_last, FoldState<kCrit> &f) {
+  Coefs<kCrit> k = f.k;
+  df Bp = f.Bp, Bc = f.Bc;
+  float Vn = f.Vn, P = f.P;
+  int fl = f.fl;
   const int sw = lane & 7;
 #pragma unroll 1
   for (int g = 7; g >= 0; --g) {
@@ -544,19 +609,29 @@ __device__ GMap<kCrit> fold_lane(const GaeArgs &a, const float *val, int lane, u
       fl |= a4 ? 2 : 0;
     }
   }
-  // act tokens left of the leftmost end (all of them when there is none)
-  const int lead = ends ? __clz(__brev(ends)) : 32;  // index of the lowest end bit
-  n = __popc(act & (lead >= 32 ? 0xffffffffu : ((1u << lead) - 1u)));
+  f.k = k;
+  f.Bp = Bp;
+  f.Bc = Bc;
+  f.Vn = Vn;
+  f.P = P;
+  f.fl = fl;
+  f.nact += __popc(act);
+}
+
+// The map of the lane's whole segment from its fold.
+template <bool kCrit>
+__device__ GMap<kCrit> lane_map(const FoldState<kCrit> &f) {
   GMap<kCrit> m;
-  m.fl = fl;
-  m.vp = (fl & 2) ? Vn : P;
-  m.cp = Bp;
-  m.kp = k.p;
-  m.ap = fl == 2 ? df_pow(k.p.a, n - 1) : df{0.f, 0.f};
+  m.fl = f.fl;
+  m.vp = (f.fl & 2) ? f.Vn : f.P;
+  m.cp = f.Bp;
+  m.kp = f.k.p;
+  // with no trajectory end every action token of the segment is in one trajectory
+  m.ap = f.fl == 2 ? df_pow(f.k.p.a, f.nact - 1) : df{0.f, 0.f};
   if constexpr (kCrit) {
-    m.cc = Bc;
-    m.kc = k.c;
-    m.ac = fl == 2 ? df_pow(k.c.a, n - 1) : df{0.f, 0.f};
+    m.cc = f.Bc;
+    m.kc = f.k.c;
+    m.ac = f.fl == 2 ? df_pow(f.k.c.a, f.nact - 1) : df{0.f, 0.f};
   }
   return m;
 }
@@ -566,13 +641,23 @@ __device__ GMap<kCrit> fold_lane(const GaeArgs &a, const float *val, int lane, u
 // A is small against V), and otherwise already within half an ulp of A.
 __device__ __forceinline__ float adv_round(df B, float v) { return __fadd_rn(__fsub_rn(B.hi, v), B.lo); }
 
-// Replays the lane's tokens from the state at its right edge; advantages
-// overwrite the values in the lane's row, returns go to the ret row.
+// A lane's replay state: the state at the right edge of the current piece and
+// the coefficients and reward of the trajectory there.
 template <bool kCrit>
-__device__ void replay_lane(const GaeArgs &a, float *val, float *ret, int lane, uint32_t act, uint32_t ends,
-                            int64_t t0, const CuView &cu, int blo, int b_last, GState st) {
-  Coefs<kCrit> k = load_coefs<kCrit>(a.coef, b_last);
-  float R = __ldg(a.rewards + b_last);
+struct ReplayState {
+  GState st;
+  Coefs<kCrit> k;
+  float R;
+};
+
+// Replays one piece; advantages overwrite the values in the lane's row,
+// returns go to the ret row.
+template <bool kCrit>
+__device__ void replay_piece(const GaeArgs &a, float *val, float *ret, int lane, uint32_t act, uint32_t ends,
+                             int64_t t0, const CuView &cu, int blo, int b_last, ReplayState<kCrit> &rs) {
+  Coefs<kCrit> k = rs.k;
+  float R = rs.R;
+  GState st = rs.st;
   const int sw = lane & 7;
 #pragma unroll 1
   for (int g = 7; g >= 0; --g) {
@@ -624,16 +709,19 @@ __device__ void replay_lane(const GaeArgs &a, float *val, float *ret, int lane, 
     *vp = make_float4(ov[0], ov[1], ov[2], ov[3]);
     *rp = make_float4(orr[0], orr[1], orr[2], orr[3]);
   }
+  rs.k = k;
+  rs.R = R;
+  rs.st = st;
 }
 
 // What a lane keeps about a folded chunk until its look-back is done.
 template <bool kCrit>
 struct Pending {
   int q;           // chunk index
-  int buf;         // val buffer holding the chunk
-  bool active;     // the lane's first token is below N
-  uint32_t act, ends;
-  int blo, b_last;
+  int buf;         // one piece per segment: the value buffer holding the chunk
+  uint32_t act;    // one piece per segment: the lane's action bits
+  int blo, bhi;    // trajectories the chunk can touch
+  int b_seg;       // trajectory of the lane's last token below N
   GMap<kCrit> E;   // maps of the lanes to the right within the chunk
   GMap<kCrit> S;   // lane 0: map of the whole chunk
 };
@@ -644,56 +732,58 @@ __device__ __forceinline__ int take_chunk(const GaeArgs &a, int lane) {
   return a.nchunks - 1 - __shfl_sync(0xffffffffu, t, 0);
 }
 
-// Copies chunk q into val[buf], folds each lane's tokens, scans the lane maps
-// and publishes the chunk's map (or, when it ignores its right neighbour, its
+// Folds each lane's segment of chunk q piece by piece (right to left, the
+// next piece copied while the current one is folded), scans the lane maps and
+// publishes the chunk's map (or, when it ignores its right neighbour, its
 // left-edge state). Nothing here waits on another warp.
 template <bool kCrit>
 __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, int lane, int q, int buf, Pending<kCrit> &p) {
-  const int64_t c0 = int64_t(q) * kChunk;
-  const int64_t t0 = c0 + int64_t(lane) * kItems;
+  const int seg = 32 * a.pieces;
+  const bool one = a.pieces == 1;  // the chunk stays in val[buf] until its replay
+  const int64_t c0 = int64_t(q) * kChunk * a.pieces;
+  const int64_t s0 = c0 + int64_t(lane) * seg;  // the lane's segment
   const int64_t N = a.N;
-  stage_in(a, c0, lane, w.val[buf], w.msk);
+  const uint64_t keep = l2_policy(true);
+  stage_in(a, c0, seg, a.pieces - 1, lane, w.val[one ? buf : 0], w.msk, keep);
 
   // This chunk's slice of cu_seqlens, in shared memory when it fits.
-  const int blo = __ldg(a.chunk_first + q);
-  const int bhi = q + 1 < a.nchunks ? __ldg(a.chunk_first + q + 1) : a.B - 1;
+  const int sub0 = q * a.pieces, sub1 = (q + 1) * a.pieces;
+  const int blo = __ldg(a.chunk_first + sub0);
+  const int bhi = sub1 < a.nsub ? __ldg(a.chunk_first + sub1) : a.B - 1;
   const int ncu = bhi - blo + 2;  // cu[blo .. bhi + 1]
   const CuView cu{a.cu, w.cu, blo, ncu <= kCuCap};
   if (cu.in_smem)
     for (int i = lane; i < ncu; i += 32) w.cu[i] = __ldg(a.cu + blo + i);
   __syncwarp();
 
-  // trajectory ends among the lane's tokens (forward walk over cu_seqlens)
-  const bool active = t0 < N;
-  uint32_t ends = 0;
-  int b_last = blo;
-  if (active) {
-    const int64_t tl = (t0 + kItems <= N ? int64_t(kItems) : N - t0) - 1;  // last token, relative to t0
-    int b = cu.find(blo, bhi, t0);
-    for (;;) {
-      const int64_t e = cu[b + 1] - 1 - t0;  // last token of trajectory b, relative to t0
-      if (e >= 0 && e <= tl) ends |= 1u << e;
-      if (e >= tl || b >= bhi) break;  // b holds the lane's last token (or cu_seqlens is malformed)
-      ++b;
-    }
-    b_last = b;
+  // the trajectory of the lane's last token below N gives its first coefficients
+  const int64_t s_end = (s0 + seg < N ? s0 + seg : N) - 1;
+  const int b_seg = s0 < N ? cu.find(blo, bhi, s_end) : blo;
+  FoldState<kCrit> f;
+  f.k = load_coefs<kCrit>(a.coef, b_seg);
+  f.Bp = f.Bc = {0.f, 0.f};
+  f.Vn = f.P = 0.f;
+  f.fl = 0;
+  f.nact = 0;
+  uint32_t act = 0;
+#pragma unroll 1
+  for (int k = a.pieces - 1; k >= 0; --k) {
+    const int cur = one ? buf : (a.pieces - 1 - k) & 1;
+    cp_async_wait_all();
+    __syncwarp();
+    act = row_actions(w.msk, lane);
+    __syncwarp();  // every lane has read the flags and finished the previous piece
+    if (k > 0) stage_in(a, c0, seg, k - 1, lane, w.val[cur ^ 1], w.msk, keep);
+    const int64_t t0 = s0 + 32 * int64_t(k);
+    int b_last;
+    const uint32_t ends = piece_ends(a, cu, blo, bhi, t0, b_last);
+    // every lane folds (the token loops vote across the warp); a lane past N
+    // has no flags and keeps its state
+    fold_piece<kCrit>(a, w.val[cur], lane, act, ends, t0, cu, blo, b_last, f);
   }
 
-  cp_async_wait_all();
-  __syncwarp();
-  uint32_t act;
-  {
-    const uint4 m0 = *reinterpret_cast<const uint4 *>(&w.msk[16 * mgran(lane, 0)]);
-    const uint4 m1 = *reinterpret_cast<const uint4 *>(&w.msk[16 * mgran(lane, 1)]);
-    act = nonzero_bytes(m0.x) | nonzero_bytes(m0.y) << 4 | nonzero_bytes(m0.z) << 8 | nonzero_bytes(m0.w) << 12 |
-          nonzero_bytes(m1.x) << 16 | nonzero_bytes(m1.y) << 20 | nonzero_bytes(m1.z) << 24 |
-          nonzero_bytes(m1.w) << 28;
-  }
-
-  // fold the lane's tokens, then the suffix scan of the warp's 32 maps
-  // every lane folds (the token loops vote across the warp); a lane past N
-  // has no flags and yields the identity map
-  GMap<kCrit> S = fold_lane<kCrit>(a, w.val[buf], lane, act, ends, t0, cu, blo, b_last);
+  // the suffix scan of the warp's 32 lane maps
+  GMap<kCrit> S = lane_map<kCrit>(f);
 #pragma unroll 1
   for (int d = 1; d < 32; d <<= 1) {
     const GMap<kCrit> o = shfl_down_map<kCrit>(S, d);
@@ -712,37 +802,58 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, int lane, int q, int bu
   }
   p.q = q;
   p.buf = buf;
-  p.active = active;
   p.act = act;
-  p.ends = ends;
   p.blo = blo;
-  p.b_last = b_last;
+  p.bhi = bhi;
+  p.b_seg = b_seg;
   p.E = E;
   p.S = S;
+  __syncwarp();  // the staging buffers are free for the replay of the previous chunk
 }
 
 // Looks back for the state at the chunk's right edge, publishes its left-edge
-// state, replays the tokens and stores advantages and returns.
+// state, then re-stages the chunk piece by piece (right to left), replays the
+// tokens and stores advantages and returns.
 template <bool kCrit>
 __device__ void finish_chunk(const GaeArgs &a, WarpBuf &w, int lane, const Pending<kCrit> &p) {
+  const int seg = 32 * a.pieces;
+  const int64_t c0 = int64_t(p.q) * kChunk * a.pieces;
+  const int64_t s0 = c0 + int64_t(lane) * seg;
+  const bool one = a.pieces == 1;  // the chunk is still in val[p.buf]
+  const uint64_t drop = l2_policy(false);
+  if (!one) stage_in(a, c0, seg, a.pieces - 1, lane, w.val[0], w.msk, drop);  // lands while the look-back runs
   const bool last = (p.q == a.nchunks - 1);
   const bool reset = __shfl_sync(0xffffffffu, p.S.fl & 1, 0) != 0;  // lane 0 holds the chunk's map
   GState right = zero_state();
   if (!last) right = look_back<kCrit>(a, p.q, lane);
   if (lane == 0 && !reset && !last)
     publish_state<kCrit>(a.incl + size_t(p.q) * kStateWords<kCrit>, apply<kCrit>(p.S, right));
-  const int64_t c0 = int64_t(p.q) * kChunk;
-  {
-    // every lane replays (the token loops vote across the warp); rows past N
-    // are never stored
-    const GState in = apply<kCrit>(p.E, right);
-    const CuView cu{a.cu, nullptr, p.blo, false};  // ends are rare: read cu_seqlens from global memory
-    const int64_t t0 = c0 + int64_t(lane) * kItems;
-    replay_lane<kCrit>(a, w.val[p.buf], w.ret, lane, p.act, p.ends, t0, cu, p.blo, p.b_last, in);
+  // every lane replays (the token loops vote across the warp); rows past N
+  // are never stored
+  const CuView cu{a.cu, nullptr, p.blo, false};  // ends are rare: read cu_seqlens from global memory
+  ReplayState<kCrit> rs;
+  rs.st = apply<kCrit>(p.E, right);
+  rs.k = load_coefs<kCrit>(a.coef, p.b_seg);
+  rs.R = __ldg(a.rewards + p.b_seg);
+#pragma unroll 1
+  for (int k = a.pieces - 1; k >= 0; --k) {
+    const int cur = one ? p.buf : (a.pieces - 1 - k) & 1;
+    uint32_t act = p.act;
+    if (!one) {
+      cp_async_wait_all();
+      __syncwarp();
+      act = row_actions(w.msk, lane);
+      __syncwarp();  // every lane has read the flags; the other buffer's piece is stored
+      if (k > 0) stage_in(a, c0, seg, k - 1, lane, w.val[cur ^ 1], w.msk, drop);
+    }
+    const int64_t t0 = s0 + 32 * int64_t(k);
+    int b_last;
+    const uint32_t ends = piece_ends(a, cu, p.blo, p.bhi, t0, b_last);
+    replay_piece<kCrit>(a, w.val[cur], w.ret, lane, act, ends, t0, cu, p.blo, b_last, rs);
+    __syncwarp();
+    stage_out(a, c0, seg, k, lane, w.val[cur], w.ret);
+    __syncwarp();
   }
-  __syncwarp();
-  stage_out(a, c0, lane, w.val[p.buf], w.ret);
-  __syncwarp();
 }
 
 // Persistent warps, software-pipelined: a warp takes a chunk (ticket), folds
@@ -829,8 +940,16 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
                       int32_t B, int64_t N, float gamma, float lam, float lam_c, float alpha, float *adv,
                       float *ret, unsigned int *err, void *ws_body, size_t body_bytes, cudaStream_t s) {
   if (N == 0) return SAO_OK;
+  // 1024-token sub-chunks (the units of chunk_first and of the count and
+  // broadcast passes) and the scan's chunks of 32 lane segments of
+  // 32 * pieces tokens: longer segments spread the warp scan and look-back of
+  // a chunk over more tokens, as long as the scan keeps about 16k chunks to
+  // share out (pieces from N alone, so every device gives the same bits)
   const int64_t nchunks = (N + kChunk - 1) / kChunk;
   if (nchunks > (int64_t(1) << 30)) return fail(SAO_ERR_SHAPE, "too many tokens for the advantage scan");
+  int pieces = 1;
+  while (pieces < 8 && (N >> 24) >= 2 * pieces) pieces *= 2;
+  const int64_t nscan = (N + int64_t(kChunk) * pieces - 1) / (int64_t(kChunk) * pieces);
   const bool crit_trivial = (gamma == 1.0f && lam_c == 1.0f);
   const size_t map_words = crit_trivial ? kMapWords<false> : kMapWords<true>;
   const size_t state_words = crit_trivial ? kStateWords<false> : kStateWords<true>;
@@ -887,7 +1006,9 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   a.cu = cu;
   a.B = B;
   a.N = N;
-  a.nchunks = int(nchunks);
+  a.nchunks = int(nscan);
+  a.pieces = pieces;
+  a.nsub = int(nchunks);
   a.coef = coef;
   a.chunk_first = chunk_first;
   a.ticket = ticket;
@@ -902,7 +1023,7 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   auto kern = crit_trivial ? gae_scan_kernel<false> : gae_scan_kernel<true>;
   SAO_TRY(set_scan_smem(kern, crit_trivial ? 0 : 1, di.device));
   // persistent: as many warps as fit on the GPU, never more than chunks
-  const int64_t ctas = (nchunks + kWarps - 1) / kWarps;
+  const int64_t ctas = (nscan + kWarps - 1) / kWarps;
   const int64_t resident = int64_t(di.sm_count) * kMinBlocks;
   const unsigned grid = unsigned(ctas < resident ? ctas : resident);
   int slot = launch_begin("gae_scan", s);

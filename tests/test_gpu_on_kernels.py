@@ -126,6 +126,25 @@ def test_advantages_bandwidth_size_properties():
         assert rel_err_floor(ret[lo:hi], r, 1e-3).max() <= ADV_TOL
 
 
+@pytest.mark.parametrize("N", [1 << 25, (1 << 26) + 12345])
+def test_advantages_long_lane_segments(N):
+    """From 2^25 tokens on, the scan's lanes own 64-256-token segments streamed
+    in 32-token pieces: 64 sampled trajectories and the last two (the ragged
+    tail) against the oracle, with lambda = 0.95 and with the length-adaptive
+    lambda and lambda_critic < 1."""
+    wl = S.bandwidth_workload(N=N, B=max(1, N >> 13))
+    rng = np.random.default_rng(N % 1000)
+    picks = np.concatenate([rng.choice(wl.B, size=64, replace=False), [wl.B - 2, wl.B - 1]])
+    for coefs in ((1.0, 0.95, 1.0, 0.0), (0.99, 1.0, 0.97, 1.5)):
+        adv, ret, g = _gae_gpu(wl, gamma=coefs[0], lam=coefs[1], lam_c=coefs[2], alpha=coefs[3])
+        for b in picks:
+            lo, hi = wl.cu_seqlens[b], wl.cu_seqlens[b + 1]
+            a, r = O.advantages(wl.values[lo:hi], wl.rewards[b:b + 1], wl.loss_mask[lo:hi], np.array([0, hi - lo]),
+                                g["gamma"], g["lam"], g["lam_c"], g["alpha"])
+            assert rel_err_floor(adv[lo:hi], a, 1e-3).max() <= ADV_TOL
+            assert rel_err_floor(ret[lo:hi], r, 1e-3).max() <= ADV_TOL
+
+
 def test_advantages_checked_mode_reports_bad_cu_seqlens():
     wl = S.make_custom([10, 20], 8, 16, "f32", seed=5, dense=False)
     bad = wl.cu_seqlens.copy()
