@@ -11,6 +11,7 @@
 
 #include "sao_common.cuh"
 #include "sao_internal.h"
+#include "dfloat.cuh"
 #include "segments.cuh"
 
 namespace sao {
@@ -147,8 +148,9 @@ __global__ void __launch_bounds__(kThreads, 5) clip_loss_kernel(ClipArgs a) {
     int blo, bhi;
     const CuView cu = seg::stage_chunk(a.cu, a.B, a.nchunks, a.chunk_first, q, lane, s_cu_all[warp], blo, bhi);
     const Norms nm = *a.norms;
-    const float w_tok = nm.n_action > 0 ? float(1.0 / double(nm.n_action)) : 0.f;
-    const double inv_seq = nm.n_seq > 0 ? 1.0 / double(nm.n_seq) : 0.0;
+    // fp32 weights (one rounding each, far inside the 1e-5 coefficient bar)
+    const float w_tok = nm.n_action > 0 ? __fdiv_rn(1.f, float(nm.n_action)) : 0.f;
+    const float inv_seq = nm.n_seq > 0 ? __fdiv_rn(1.f, float(nm.n_seq)) : 0.f;
     const float gscale = kBwd ? __ldg(a.grad_scale) : 1.f;
     // window-major: in each 128-token window of the chunk, lane l takes tokens
     // 4l .. 4l+3, so every warp load and store is one contiguous 512 (or 128)
@@ -160,7 +162,7 @@ __global__ void __launch_bounds__(kThreads, 5) clip_loss_kernel(ClipArgs a) {
     auto weight = [&](int bb) {
       if (!a.seq) return w_tok;
       const int L = __ldg(a.nact + bb);
-      return L > 0 ? float(inv_seq / double(L)) : 0.f;
+      return L > 0 ? __fdiv_rn(inv_seq, float(L)) : 0.f;
     };
     float w = weight(b);
     const bool aligned = aligned16_dev(a.logp) && aligned16_dev(a.old) && aligned16_dev(a.adv) &&
@@ -354,13 +356,52 @@ __device__ __forceinline__ Sum2 warp_total(Sum2 s) {
   return s;
 }
 
+// flag = 0 when some group id is larger than the next one (the flag starts at
+// 1): with non-decreasing ids every group is one contiguous run of the batch.
+__global__ void group_sorted_kernel(const int32_t *gid, int B, int *flag) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b + 1 < B && __ldg(gid + b) > __ldg(gid + b + 1)) *flag = 0;
+}
+
+// First index of the run of group id g that holds index b (dir = -1), or one
+// past its last index (dir = +1), for sorted ids; a warp walks 32 entries per
+// step.
+__device__ int run_edge(const int32_t *gid, int B, int b, int g, int dir, int lane) {
+  int edge = b;
+  for (;;) {
+    const int i = edge + dir * (1 + lane);
+    const bool in = i >= 0 && i < B && __ldg(gid + i) == g;
+    const unsigned out = __ballot_sync(0xffffffffu, !in);
+    if (out) return edge + dir * (__ffs(out) - 1) + (dir > 0 ? 1 : 0);
+    edge += 32 * dir;
+  }
+}
+
 __global__ void __launch_bounds__(256) group_norm_kernel(const float *R, const int32_t *gid, int B, float eps,
-                                                         float *a_traj) {
+                                                         const int *sorted, float *a_traj) {
   __shared__ int32_t sg[kTile];
   __shared__ float sr[kTile];
+  __shared__ int s_range[2];
   const int lane = threadIdx.x & 31;
   const int b = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int g = b < B ? gid[b] : 0;
+  // The entries to visit: the whole batch, or with non-decreasing ids the runs
+  // of this CTA's groups (the same members in the same lane order, so the same
+  // sums either way).
+  if (threadIdx.x < 32) {
+    int lo = 0, hi = B;
+    if (*sorted) {
+      const int b0 = blockIdx.x * 8, b1 = min(B, b0 + 8) - 1;
+      lo = run_edge(gid, B, b0, __ldg(gid + b0), -1, lane);
+      hi = run_edge(gid, B, b1, __ldg(gid + b1), +1, lane);
+    }
+    if (lane == 0) {
+      s_range[0] = lo;
+      s_range[1] = hi;
+    }
+  }
+  __syncthreads();
+  const int lo = s_range[0], hi = s_range[1];
   Sum2 s, s2;
   int n = 0;
   float mu = 0.f;
@@ -369,16 +410,16 @@ __global__ void __launch_bounds__(256) group_norm_kernel(const float *R, const i
   // more (groups of tens of trajectories) the second moment needs no second
   // sweep, and it adds the same values in the same order.
   float r0 = 0.f, r1 = 0.f, r2 = 0.f, r3 = 0.f;
-  for (int t0 = 0; t0 < B; t0 += kTile) {
-    const int len = min(kTile, B - t0);
+  for (int t0 = lo / kTile * kTile; t0 < hi; t0 += kTile) {
+    const int klo = max(lo - t0, 0), khi = min(kTile, hi - t0);
     __syncthreads();
-    for (int k = threadIdx.x; k < len; k += blockDim.x) {
+    for (int k = klo + int(threadIdx.x); k < khi; k += blockDim.x) {
       sg[k] = gid[t0 + k];
       sr[k] = R[t0 + k];
     }
     __syncthreads();
     if (b >= B) continue;
-    for (int k = lane; k < len; k += 32) {
+    for (int k = klo + ((lane - klo) & 31); k < khi; k += 32) {
       if (sg[k] != g) continue;
       const float r = sr[k];
       s.add(r);
@@ -392,7 +433,7 @@ __global__ void __launch_bounds__(256) group_norm_kernel(const float *R, const i
   if (b < B) {  // the group's mean, from lane 0 to every lane
     const Sum2 t = warp_total(s);
     const int nt = __reduce_add_sync(0xffffffffu, n);
-    mu = __shfl_sync(0xffffffffu, float(t.value() / double(nt > 0 ? nt : 1)), 0);
+    mu = __shfl_sync(0xffffffffu, dfl::round(dfl::div_int(dfl::norm(t.hi, t.lo), nt > 0 ? nt : 1)), 0);
   }
   const bool sweep = __syncthreads_or(b < B && n > 4);
   if (!sweep) {
@@ -404,16 +445,16 @@ __global__ void __launch_bounds__(256) group_norm_kernel(const float *R, const i
         s2.add(__fmul_rn(d, d));
       }
   } else {
-    for (int t0 = 0; t0 < B; t0 += kTile) {
-      const int len = min(kTile, B - t0);
+    for (int t0 = lo / kTile * kTile; t0 < hi; t0 += kTile) {
+      const int klo = max(lo - t0, 0), khi = min(kTile, hi - t0);
       __syncthreads();
-      for (int k = threadIdx.x; k < len; k += blockDim.x) {
+      for (int k = klo + int(threadIdx.x); k < khi; k += blockDim.x) {
         sg[k] = gid[t0 + k];
         sr[k] = R[t0 + k];
       }
       __syncthreads();
       if (b >= B) continue;
-      for (int k = lane; k < len; k += 32) {
+      for (int k = klo + ((lane - klo) & 31); k < khi; k += 32) {
         if (sg[k] != g) continue;
         const float d = __fsub_rn(sr[k], mu);
         s2.add(__fmul_rn(d, d));
@@ -424,11 +465,14 @@ __global__ void __launch_bounds__(256) group_norm_kernel(const float *R, const i
   const Sum2 t = warp_total(s), t2 = warp_total(s2);
   const int nt = __reduce_add_sync(0xffffffffu, n);
   if (lane == 0) {
-    // exact mean correction for the rounded mu: var = E[(r - mu)^2] - (mean - mu)^2
-    const double mean = t.value() / double(nt);
-    const double dm = mean - double(mu);
-    const double var = t2.value() / double(nt) - dm * dm;
-    a_traj[b] = float((double(R[b]) - mean) / sqrt((var > 0.0 ? var : 0.0) + double(eps)));
+    // exact mean correction for the rounded mu: var = E[(r - mu)^2] - (mean - mu)^2,
+    // in double-float; then (R - mean) rounded once and divided in fp32
+    const dfl::F2 mean = dfl::div_int(dfl::norm(t.hi, t.lo), nt);
+    const dfl::F2 dm = dfl::sub(mean, dfl::F2{mu, 0.f});
+    const dfl::F2 var = dfl::sub(dfl::div_int(dfl::norm(t2.hi, t2.lo), nt), dfl::mul(dm, dm));
+    const float v = fmaxf(dfl::round(var), 0.f);
+    const float num = dfl::round(dfl::sub(dfl::F2{R[b], 0.f}, mean));
+    a_traj[b] = __fdiv_rn(num, __fsqrt_rn(__fadd_rn(v, eps)));
   }
 }
 
@@ -438,13 +482,9 @@ __global__ void __launch_bounds__(256) group_norm_kernel(const float *R, const i
 // those k writes have not overwritten. So every trajectory is independent:
 // one warp per trajectory walks the batch backwards from b (most recent
 // first, 32 entries per step: a ballot ranks the matches), then the ring
-// buffers are updated in a second pass. Sums are fp64, combined in a fixed
-// order.
-__device__ __forceinline__ double warp_total_f64(double x) {
-#pragma unroll
-  for (int d = 16; d >= 1; d >>= 1) x += __shfl_down_sync(0xffffffffu, x, d);
-  return x;  // lane 0
-}
+// buffers are updated in a second pass. Sums are compensated fp32 (about 48
+// bits), combined in a fixed order; the mean and the advantage in
+// double-float.
 
 // In-batch ranks for dense prompt ids (P <= kRankMaxPrompts): counts of each
 // prompt per block of kRankBlock trajectories, then their exclusive prefix over
@@ -500,13 +540,13 @@ __global__ void __launch_bounds__(256) running_mean_kernel(const float *R, const
     }
     return;
   }
-  double sum = 0.0;  // this lane's share
-  int hits = 0;      // warp-uniform
+  Sum2 sum;      // this lane's share, compensated fp32
+  int hits = 0;  // warp-uniform
   for (int top = b - 1; top >= 0; top -= 32) {
     const int i = top - lane;
     const bool hit = i >= 0 && __ldg(pid + i) == p;
     const unsigned mask = __ballot_sync(0xffffffffu, hit);
-    if (hit && hits + __popc(mask & ((1u << lane) - 1u)) < window) sum += double(__ldg(R + i));
+    if (hit && hits + __popc(mask & ((1u << lane) - 1u)) < window) sum.add(__ldg(R + i));
     hits += __popc(mask);
     if (table && hits >= window) break;
   }
@@ -527,13 +567,14 @@ __global__ void __launch_bounds__(256) running_mean_kernel(const float *R, const
     const float *h = history + int64_t(p) * window;
     for (int q = lane; q < valid_old; q += 32) {
       const int since = int(((long long)q - c % window + window) % window);  // write order of slot q after c
-      if (since >= k) sum += double(h[q]);
+      if (since >= k) sum.add(h[q]);
     }
   }
-  sum = warp_total_f64(sum);
+  sum = warp_total(sum);
   if (lane == 0) {
     const long long n = (c + k) < window ? (c + k) : window;
-    a_traj[b] = float(double(R[b]) - (n > 0 ? sum / double(n) : 0.0));
+    const dfl::F2 mean = n > 0 ? dfl::div_int(dfl::norm(sum.hi, sum.lo), int(n)) : dfl::F2{0.f, 0.f};
+    a_traj[b] = dfl::round(dfl::sub(dfl::F2{R[b], 0.f}, mean));
     rec[b] = c + k;  // b's position in its prompt's reward sequence
     if (rank) rank[b] = k;
   }
@@ -658,13 +699,17 @@ sao_status group_adv_launch(const float *rewards, const int32_t *gid, int32_t B,
   Carver c(ws_body, body_bytes);
   float *a_traj = c.take<float>(size_t(B) + 1);
   int *chunk_first = c.take<int>(size_t((N + kSegChunk - 1) / kSegChunk) + 1);
+  int *sorted = c.take<int>(1);
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the group advantages");
   if (B == 0) {
     if (N > 0) SAO_CUDA_TRY(cudaMemsetAsync(adv, 0, sizeof(float) * size_t(N), s));
     return SAO_OK;
   }
+  SAO_CUDA_TRY(cudaMemsetAsync(sorted, 0, sizeof(int), s));
+  SAO_CUDA_TRY(cudaMemsetAsync(sorted, 1, 1, s));  // the int 1
   int slot = launch_begin("group_advantages", s);
-  group_norm_kernel<<<unsigned((B + 7) / 8), 256, 0, s>>>(rewards, gid, B, eps, a_traj);
+  group_sorted_kernel<<<unsigned((B + 255) / 256), 256, 0, s>>>(gid, B, sorted);
+  group_norm_kernel<<<unsigned((B + 7) / 8), 256, 0, s>>>(rewards, gid, B, eps, sorted, a_traj);
   SAO_TRY(launch_end(slot, s));
   return broadcast_launch(a_traj, m, cu, B, N, chunk_first, adv, s);
 }

@@ -193,6 +193,33 @@ def test_group_advantages_match_oracle():
         assert rel_err_floor(adv.cpu().numpy(), want, 1e-3).max() <= 1e-5
 
 
+@pytest.mark.parametrize("seed", [0, 1])
+def test_group_advantages_sorted_ids_same_bits(seed):
+    """Non-decreasing group ids (a prompt's rollouts adjacent) take the path
+    that visits only each CTA's runs: groups of 1 to 3,000 trajectories, runs
+    across the 2,048-entry tiles, negative ids. Against the oracle, and bit
+    for bit against the same partition under ids relabelled out of order
+    (which takes the whole-batch scan)."""
+    rng = np.random.default_rng(seed)
+    sizes = np.concatenate([[1, 2, 3000, 8, 1], rng.integers(1, 60, size=300), [2500, 5]])
+    B = int(sizes.sum())
+    lengths = rng.integers(0, 40, size=B)
+    wl = S.make_custom(lengths.tolist(), 8, 16, "f32", seed=21 + seed, dense=False, obs_frac=0.3)
+    gid = (np.repeat(np.arange(len(sizes)), sizes) - 3).astype(np.int32)
+    relabel = ((gid.astype(np.int64) + 3) * 7919 % 100003).astype(np.int32)
+    assert np.any(np.diff(relabel) < 0) and np.all(np.diff(gid) >= 0)
+    outs = []
+    for ids in (gid, relabel):
+        adv = torch.empty(wl.N, device="cuda")
+        sao.sao_group_advantages(cuda(wl.rewards), cuda(ids), cuda(wl.loss_mask), cuda(wl.cu_seqlens), 1e-6, adv,
+                                 sao.workspace(wl.N))
+        torch.cuda.synchronize()
+        outs.append(adv.cpu().numpy())
+    assert np.array_equal(outs[0], outs[1])
+    want = O.group_advantages(wl.rewards, gid, wl.loss_mask, wl.cu_seqlens, f32(1e-6))
+    assert rel_err_floor(outs[0], want, 1e-3).max() <= 1e-5
+
+
 def test_running_mean_advantages_match_oracle():
     """Two batches in a row with per-prompt windows of 8 (§4.3) and one global
     window of 128 (§4.5); the windows persist between calls."""
