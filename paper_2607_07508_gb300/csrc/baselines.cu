@@ -506,16 +506,26 @@ __global__ void __launch_bounds__(256) rank_count_kernel(const int32_t *pid, int
   for (int q = threadIdx.x; q < P; q += blockDim.x) table[int64_t(blockIdx.x) * P + q] = cnt[q];
 }
 
-__global__ void rank_scan_kernel(int *table, int nblk, int P) {
-  const int q = blockIdx.x * blockDim.x + threadIdx.x;
+// One warp per prompt: exclusive prefix of its per-block counts, 32 blocks at
+// a time by a shuffle scan.
+__global__ void __launch_bounds__(256) rank_scan_kernel(int *table, int nblk, int P) {
+  const int q = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
   if (q >= P) return;
   int run = 0;
-  for (int k = 0; k < nblk; ++k) {
-    const int v = table[int64_t(k) * P + q];
-    table[int64_t(k) * P + q] = run;
-    run += v;
+  for (int k0 = 0; k0 < nblk; k0 += 32) {
+    const int k = k0 + lane;
+    const int v = k < nblk ? table[int64_t(k) * P + q] : 0;
+    int inc = v;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      const int o = __shfl_up_sync(0xffffffffu, inc, d);
+      if (lane >= d) inc += o;
+    }
+    if (k < nblk) table[int64_t(k) * P + q] = run + inc - v;
+    run += __shfl_sync(0xffffffffu, inc, 31);
   }
-  table[int64_t(nblk) * P + q] = run;
+  if (lane == 0) table[int64_t(nblk) * P + q] = run;
 }
 
 // One warp per trajectory b of prompt p: the sum of the rewards of the most
@@ -542,21 +552,43 @@ __global__ void __launch_bounds__(256) running_mean_kernel(const float *R, const
   }
   Sum2 sum;      // this lane's share, compensated fp32
   int hits = 0;  // warp-uniform
-  for (int top = b - 1; top >= 0; top -= 32) {
-    const int i = top - lane;
-    const bool hit = i >= 0 && __ldg(pid + i) == p;
-    const unsigned mask = __ballot_sync(0xffffffffu, hit);
-    if (hit && hits + __popc(mask & ((1u << lane) - 1u)) < window) sum.add(__ldg(R + i));
-    hits += __popc(mask);
-    if (table && hits >= window) break;
+  // four 32-entry slices per step: their ids, then the hit rewards, loaded
+  // together; the hits are then taken slice by slice as one slice at a time
+  // would (same sums in the same order)
+  bool done = false;
+  for (int top = b - 1; top >= 0 && !done; top -= 128) {
+    int ids[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = top - 32 * u - lane;
+      ids[u] = i >= 0 ? __ldg(pid + i) : -1;
+    }
+    float rw[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) rw[u] = ids[u] == p ? __ldg(R + (top - 32 * u - lane)) : 0.f;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (done) break;
+      const bool hit = ids[u] == p;
+      const unsigned mask = __ballot_sync(0xffffffffu, hit);
+      if (hit && hits + __popc(mask & ((1u << lane) - 1u)) < window) sum.add(rw[u]);
+      hits += __popc(mask);
+      if (table && hits >= window) done = true;
+    }
   }
   int k = hits;
   if (table) {  // rank of b: earlier blocks from the table, then b's own block
     const int b0 = b / kRankBlock * kRankBlock;
     k = __ldg(table + int64_t(b / kRankBlock) * P + p);
-    for (int i0 = b0; i0 < b; i0 += 32) {
-      const int i = i0 + lane;
-      k += __popc(__ballot_sync(0xffffffffu, i < b && __ldg(pid + i) == p));
+    for (int i0 = b0; i0 < b; i0 += 128) {
+      int ids[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + 32 * u + lane;
+        ids[u] = i < b ? __ldg(pid + i) : -1;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) k += __popc(__ballot_sync(0xffffffffu, ids[u] == p));
     }
   }
   const long long c = seen[p];
@@ -741,7 +773,7 @@ sao_status running_mean_launch(const float *rewards, const int32_t *pid, int32_t
   int slot = launch_begin("running_mean_advantages", s);
   if (table) {
     rank_count_kernel<<<unsigned(nblk), 256, 0, s>>>(pid, B, P, table);
-    rank_scan_kernel<<<unsigned((P + 255) / 256), 256, 0, s>>>(table, nblk, P);
+    rank_scan_kernel<<<unsigned((P + 7) / 8), 256, 0, s>>>(table, nblk, P);
   }
   const unsigned g = unsigned((B + 7) / 8);  // a warp per trajectory
   running_mean_kernel<<<g, 256, 0, s>>>(rewards, pid, B, P, table, history,

@@ -12,7 +12,7 @@ namespace seg {
 constexpr int kItems = 32;               // tokens per lane (one bit each in a uint32)
 constexpr int kSegChunk = 32 * kItems;   // tokens per warp chunk
 constexpr int kCuCap = 128;              // cu_seqlens entries staged per warp
-constexpr int kCountChunks = 8;          // chunks per warp in action_count_kernel
+constexpr int kCountChunks = 2;          // chunks per warp in action_count_kernel
 
 // chunk_first_kernel: one chunk per thread, 1024 threads per CTA, and a
 // sample of every ceil(B / 4096)-th cu_seqlens entry in shared memory.
