@@ -98,6 +98,23 @@ __device__ __forceinline__ df df_axpby(df a, df x, df g, float v) {
   lo = __fadd_rn(lo, s.lo);
   return quick_two_sum(s.hi, lo);
 }
+// The same a*x + g*v with the result left unnormalised: (s, lo) with lo a few
+// ulps of s, which the next step's products take as they are. The
+// branch-free token loops renormalise once per 4-token group, so the pair
+// never drifts (its low part stays within a few ulps of the high one).
+__device__ __forceinline__ df df_axpby_u(df a, df x, df g, float v) {
+  const float p1 = __fmul_rn(a.hi, x.hi);
+  const float e1 = __fmaf_rn(a.hi, x.hi, -p1);
+  const float p2 = __fmul_rn(g.hi, v);
+  const float e2 = __fmaf_rn(g.hi, v, -p2);
+  const df s = two_sum(p1, p2);
+  float lo = __fmaf_rn(a.hi, x.lo, e1);
+  lo = __fmaf_rn(a.lo, x.hi, lo);
+  lo = __fmaf_rn(g.lo, v, lo);
+  lo = __fadd_rn(lo, e2);
+  return {s.hi, __fadd_rn(lo, s.lo)};
+}
+__device__ __forceinline__ df df_renorm(df x) { return two_sum(x.hi, x.lo); }
 // x^e for 0 <= e < 32 by squaring.
 __device__ df df_pow(df x, int e) {
   df r = {1.f, 0.f};
@@ -598,14 +615,16 @@ __device__ void fold_piece(const GaeArgs &a, const float *val, int lane, uint32_
 #pragma unroll
       for (int i = 3; i >= 0; --i) {
         const bool on = (a4 >> i) & 1u;
-        const df np = df_axpby(k.p.a, Bp, k.p.g, Vn);
+        const df np = df_axpby_u(k.p.a, Bp, k.p.g, Vn);
         Bp = on ? np : Bp;
         if constexpr (kCrit) {
-          const df nc = df_axpby(k.c.a, Bc, k.c.g, Vn);
+          const df nc = df_axpby_u(k.c.a, Bc, k.c.g, Vn);
           Bc = on ? nc : Bc;
         }
         Vn = on ? vv[i] : Vn;
       }
+      Bp = df_renorm(Bp);
+      if constexpr (kCrit) Bc = df_renorm(Bc);
       fl |= a4 ? 2 : 0;
     }
   }
@@ -693,11 +712,11 @@ __device__ void replay_piece(const GaeArgs &a, float *val, float *ret, int lane,
 #pragma unroll
       for (int i = 3; i >= 0; --i) {
         const bool on = (a4 >> i) & 1u;
-        const df np = df_axpby(k.p.a, st.Bp, k.p.g, st.Vn);
+        const df np = df_axpby_u(k.p.a, st.Bp, k.p.g, st.Vn);
         ov[i] = on ? adv_round(np, vv[i]) : 0.f;
         st.Bp = on ? np : st.Bp;
         if constexpr (kCrit) {
-          const df nc = df_axpby(k.c.a, st.Bc, k.c.g, st.Vn);
+          const df nc = df_axpby_u(k.c.a, st.Bc, k.c.g, st.Vn);
           orr[i] = on ? df_round(nc) : 0.f;
           st.Bc = on ? nc : st.Bc;
         } else {
@@ -705,6 +724,8 @@ __device__ void replay_piece(const GaeArgs &a, float *val, float *ret, int lane,
         }
         st.Vn = on ? vv[i] : st.Vn;
       }
+      st.Bp = df_renorm(st.Bp);
+      if constexpr (kCrit) st.Bc = df_renorm(st.Bc);
     }
     *vp = make_float4(ov[0], ov[1], ov[2], ov[3]);
     *rp = make_float4(orr[0], orr[1], orr[2], orr[3]);
