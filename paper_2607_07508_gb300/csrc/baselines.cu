@@ -721,7 +721,7 @@ static sao_status broadcast_launch(const float *a_traj, const uint8_t *m, const 
   int slot = launch_begin("adv_broadcast", s);
   seg::chunk_first_kernel<<<seg::chunk_first_grid(int(nchunks)), seg::kChunkFirstThreads, 0, s>>>(
       cu, B, N, int(nchunks), chunk_first);
-  seg::traj_broadcast_kernel<false><<<seg::action_count_grid(int(nchunks)), 256, 0, s>>>(
+  seg::traj_broadcast_kernel<false><<<seg::broadcast_grid(int(nchunks)), 256, 0, s>>>(
       a_traj, m, cu, B, N, int(nchunks), chunk_first, adv, nullptr, nullptr);
   return launch_end(slot, s);
 }

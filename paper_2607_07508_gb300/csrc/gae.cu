@@ -1005,7 +1005,7 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
     gae_coef_kernel<<<(B + 127) / 128, 128, 0, s>>>(cu, B, N, gamma, lam, lam_c, alpha, nact, coef, err);
     SAO_TRY(launch_end(slot, s));
     slot = launch_begin("gae_telescoped", s);
-    seg::traj_broadcast_kernel<true><<<seg::action_count_grid(int(nchunks)), 256, 0, s>>>(
+    seg::traj_broadcast_kernel<true><<<seg::broadcast_grid(int(nchunks)), 256, 0, s>>>(
         rewards, m, cu, B, N, int(nchunks), chunk_first, adv, values, ret);
     return launch_end(slot, s);
   }

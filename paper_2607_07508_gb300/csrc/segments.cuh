@@ -12,7 +12,8 @@ namespace seg {
 constexpr int kItems = 32;               // tokens per lane (one bit each in a uint32)
 constexpr int kSegChunk = 32 * kItems;   // tokens per warp chunk
 constexpr int kCuCap = 128;              // cu_seqlens entries staged per warp
-constexpr int kCountChunks = 2;          // chunks per warp in action_count_kernel
+constexpr int kCountChunks = 8;          // chunks per warp in action_count_kernel
+constexpr int kCastChunks = 2;           // chunks per warp in traj_broadcast_kernel
 
 // chunk_first_kernel: one chunk per thread, 1024 threads per CTA, and a
 // sample of every ceil(B / 4096)-th cu_seqlens entry in shared memory.
@@ -25,6 +26,10 @@ __host__ __device__ constexpr unsigned chunk_first_grid(int nchunks) {
 // CTAs (of 8 warps) of action_count_kernel for nchunks chunks.
 __host__ __device__ constexpr unsigned action_count_grid(int nchunks) {
   return unsigned((nchunks + 8 * kCountChunks - 1) / (8 * kCountChunks));
+}
+// CTAs (of 8 warps) of traj_broadcast_kernel for nchunks chunks.
+__host__ __device__ constexpr unsigned broadcast_grid(int nchunks) {
+  return unsigned((nchunks + 8 * kCastChunks - 1) / (8 * kCastChunks));
 }
 
 // cu_seqlens entries [blo, blo + n) of one chunk, read from shared memory
@@ -168,8 +173,9 @@ __global__ void __launch_bounds__(256) action_count_kernel(const uint8_t *m, con
 }
 
 // adv[t] = a_traj[b] on the action tokens of trajectory b, 0 on every other
-// token; every token below N is written (cu_seqlens covers [0, N)). Same
-// grid as action_count_kernel: kCountChunks chunks per warp; in 128-token
+// token; every token below N is written (cu_seqlens covers [0, N)). Grid:
+// broadcast_grid, kCastChunks chunks per warp (its stores run in one short
+// wave per chunk pair, so small units keep the SMs busy to the end); in 128-token
 // groups lane l takes 4 tokens (a 4-byte mask load, a float4 store); a group
 // inside the lane's current trajectory takes no per-token work.
 // kValues: also ret[t] = a_traj[b] and adv[t] = a_traj[b] - values[t] on the
@@ -183,9 +189,9 @@ __global__ void __launch_bounds__(256) traj_broadcast_kernel(const float *a_traj
                                                              const float *values, float *ret) {
   __shared__ int32_t s_cu_all[8][kCuCap];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int q0 = (blockIdx.x * 8 + warp) * kCountChunks;
+  const int q0 = (blockIdx.x * 8 + warp) * kCastChunks;
   if (q0 >= nchunks) return;
-  const int q1 = q0 + kCountChunks < nchunks ? q0 + kCountChunks : nchunks;
+  const int q1 = q0 + kCastChunks < nchunks ? q0 + kCastChunks : nchunks;
   const int blo = __ldg(chunk_first + q0);
   const int bhi = q1 < nchunks ? __ldg(chunk_first + q1) : B - 1;
   const int ncu = bhi - blo + 2;  // cu[blo .. bhi + 1]
