@@ -214,6 +214,21 @@ class LossHeadStep:
 # computes the rows with loss_mask = 1, the backward kernels the rows with a
 # non-zero incoming gradient (over all vocabulary chunks and row blocks of the
 # step; a launch does its share of it).
+def kernel_bytes(name, h, rows, cols):
+    """Bytes one launch of a log-prob GEMM must move at least (operands read
+    once, outputs written once) for `rows` token rows and `cols` vocabulary
+    columns: the yardstick for its DRAM traffic."""
+    if name == "tc_logits_lse_fwd":  # H_c, W, per-tile (max, sum) partials
+        return 2 * rows * h + 2 * cols * h + 8 * rows * -(-cols // 256)
+    if name == "tc_dlogits":  # H_c, W chunk -> bf16 dZ chunk
+        return 2 * rows * h + 2 * cols * h + 2 * rows * cols
+    if name == "tc_dH_gemm":  # dZ chunk, W chunk -> fp32 dH
+        return 2 * rows * cols + 2 * cols * h + 4 * rows * h
+    if name == "tc_dW_gemm":  # dZ chunk, H_c -> fp32 dW rows of the chunk
+        return 2 * rows * cols + 2 * rows * h + 4 * cols * h
+    return None
+
+
 def kernel_flops(name, h, V, rows_fwd, rows_bwd):
     if name == "tc_logits_lse_fwd":
         return 2.0 * rows_fwd * h * V
@@ -642,6 +657,7 @@ def main():
                     "unit": "TFLOP/s", "frac": achieved / burst,
                     "traffic": (stored_traffic(dom_name, dom_rows, wl.V / per_step)
                                 if wl.name == "moe" and args.tokens is None else None),
+                    "algorithmic_bytes_per_launch": kernel_bytes(dom_name, wl.h, dom_rows, wl.V / per_step),
                     "traffic_unit": ("bytes per launch (dram read + write from the 8k-token ncu capture, scaled by "
                                      "rows x vocabulary columns per launch)"),
                     "algorithmic_per_launch": (f"2*rows*h*V = {fl_step:.4g} flop per step over {per_step:g} "
