@@ -44,13 +44,16 @@
 #include "sao_common.cuh"
 #include "sao_internal.h"
 #include "segments.cuh"
+#include "tc_ptx.cuh"
 
 namespace sao {
 namespace {
 
 constexpr int kThreads = 128;
 constexpr int kWarps = kThreads / 32;
-constexpr int kMinBlocks = 4;             // 16 warps per SM (shared memory bound)
+constexpr int kMinBlocks = 4;             // 16 warps per SM (shared memory and TMEM bound)
+constexpr int kMaxPieces = 4;             // 32-token pieces per lane segment, at most
+constexpr int kTmemCols = 32 * kMaxPieces;  // TMEM columns per CTA: 4 CTAs fill an SM's 512
 constexpr int kItems = seg::kItems;       // tokens per lane (one bit each)
 constexpr int kChunk = seg::kSegChunk;    // tokens per warp chunk
 static_assert(kItems == 32 && kChunk == 1024, "the staging layout assumes 32 x 32 tokens per warp");
@@ -361,7 +364,7 @@ struct GaeArgs {
   int B;
   int64_t N;
   int nchunks;             // scan chunks of 32 lanes x seg tokens
-  int pieces;              // 32-token pieces per lane segment (1, 2, 4 or 8)
+  int pieces;              // 32-token pieces per lane segment (1, 2 or 4)
   int nsub;                // 1024-token sub-chunks, the units of chunk_first
   const float4 *coef;      // [B][2]
   const int *chunk_first;  // [nsub] trajectory of each 1024-token sub-chunk's first token
@@ -374,7 +377,7 @@ struct GaeArgs {
 };
 
 using seg::CuView;
-using seg::kCuCap;
+
 
 
 // State at the right edge of chunk q, from the chunks to its right. The warp
@@ -427,23 +430,29 @@ __device__ GState look_back(const GaeArgs &a, int q, int lane) {
 // per-warp staging in shared memory
 // ---------------------------------------------------------------------------
 // A scan chunk is 32 lane segments of seg = 32 * pieces consecutive tokens;
-// lane r's segment starts at chunk offset r * seg. The segments stream
-// through shared memory one 32-token piece at a time (right to left): row r
-// of a staged piece holds lane r's 32 tokens of that piece. val/ret rows are
-// 8 granules of 16 bytes, granule j stored at 8r + (j ^ (r & 7)); msk rows are
-// 2 granules, granule j at 2r + (j ^ ((r >> 2) & 1)). A quarter-warp (8
-// lanes) then touches 8 distinct bank groups both when it copies the 8
-// granules (128 contiguous bytes of global memory) of one row and when 8 lanes
-// read the same granule of their own rows. With one piece per segment the
-// two value buffers hold two chunks, the one folded last and the one waiting
-// for its look-back and replay (values in, advantages out). With several, they
-// hold the piece being worked on and the next one, copied meanwhile, and the
-// replay copies its chunk's pieces again (a chunk no longer fits).
+// lane r's segment starts at chunk offset r * seg. The fold streams the
+// segments through shared memory one 32-token piece at a time (right to
+// left): row r of a staged piece holds lane r's 32 tokens of that piece.
+// val/ret rows are 8 granules of 16 bytes, granule j stored at
+// 8r + (j ^ (r & 7)); msk rows are 2 granules, granule j at
+// 2r + (j ^ ((r >> 2) & 1)). A quarter-warp (8 lanes) then touches 8 distinct
+// bank groups both when it copies the 8 granules (128 contiguous bytes of
+// global memory) of one row and when 8 lanes read the same granule of their
+// own rows. The two value buffers hold the piece being folded and the next
+// one, copied meanwhile. Each lane also stores its values into its own TMEM
+// lane (the warp's 32 lanes of the CTA's allocation, column 32k + i for token
+// i of piece k) and its action bits into `act`, so that the replay, after the
+// look-back, reads the chunk from the SM instead of from DRAM a second time;
+// the replay writes advantages into val[0] and returns into ret, which the
+// warp then stores coalesced.
+constexpr int kScanCuCap = 120;  // cu_seqlens entries staged per warp
 struct __align__(16) WarpBuf {
-  float val[2][kChunk];  // values in, advantages out (two pieces)
-  float ret[kChunk];     // returns of the piece being replayed
-  uint8_t msk[kChunk];   // action flags of the next piece
-  int32_t cu[kCuCap];    // cu_seqlens slice of the chunk being folded
+  float val[2][kChunk];           // values of two pieces (fold); advantages of one (replay)
+  float ret[kChunk];              // returns of the piece being replayed
+  uint8_t msk[kChunk];            // action flags of the piece being copied
+  uint32_t act[kMaxPieces][32];   // per piece, each lane's action bits
+  int32_t cu[kScanCuCap];         // cu_seqlens slice of the chunk being folded
+  uint32_t tmem;                  // TMEM address of the CTA's allocation (warp 0's buffer)
 };
 __device__ __forceinline__ int fgran(int r, int j) { return 8 * r + (j ^ (r & 7)); }
 __device__ __forceinline__ int mgran(int r, int j) { return 2 * r + (j ^ ((r >> 2) & 1)); }
@@ -454,15 +463,32 @@ __device__ __forceinline__ void cp_async16(void *smem, const void *gmem, uint64_
   asm volatile("cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2;" ::"r"(s), "l"(gmem), "l"(policy)
                : "memory");
 }
-// The fold's copy keeps its lines in L2 for the replay's copy of the same
-// chunk (issued about two chunk-times later), which drops them.
-__device__ __forceinline__ uint64_t l2_policy(bool keep) {
+// Every input line is read once: the copies leave L2 first.
+__device__ __forceinline__ uint64_t l2_evict_first() {
   uint64_t p;
-  if (keep)
-    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-  else
-    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
   return p;
+}
+
+// The lane's 4 TMEM columns from `taddr` (lane field: the warp's TMEM lanes).
+__device__ __forceinline__ void tmem_st4(uint32_t taddr, float4 v) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr),
+               "r"(__float_as_uint(v.x)), "r"(__float_as_uint(v.y)), "r"(__float_as_uint(v.z)),
+               "r"(__float_as_uint(v.w))
+               : "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+// Starts the load of 4 TMEM columns; the registers hold them only after
+// tmem_wait_ld4 on the same registers (which the compiler then cannot read
+// earlier).
+__device__ __forceinline__ void tmem_ld4(uint32_t taddr, uint32_t (&r)[4]) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(taddr)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_wait_ld4(uint32_t (&r)[4]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3])::"memory");
 }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
@@ -580,8 +606,8 @@ struct FoldState {
 };
 
 template <bool kCrit>
-__device__ void fold_piece(const GaeArgs &a, const float *val, int lane, uint32_t act, uint32_t ends, int64_t t0,
-                           const CuView &cu, int blo, int b_last, FoldState<kCrit> &f) {
+__device__ void fold_piece(const GaeArgs &a, const float *val, uint32_t tcol, int lane, uint32_t act, uint32_t ends,
+                           int64_t t0, const CuView &cu, int blo, int b_last, FoldState<kCrit> &f) {
   Coefs<kCrit> k = f.k;
   df Bp = f.Bp, Bc = f.Bc;
   float Vn = f.Vn, P = f.P;
@@ -590,6 +616,7 @@ __device__ void fold_piece(const GaeArgs &a, const float *val, int lane, uint32_
 #pragma unroll 1
   for (int g = 7; g >= 0; --g) {
     const float4 v4 = *reinterpret_cast<const float4 *>(&val[4 * (8 * lane + (g ^ sw))]);
+    tmem_st4(tcol + 4 * g, v4);  // kept for the replay
     const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
     const uint32_t a4 = (act >> (4 * g)) & 15u, e4 = (ends >> (4 * g)) & 15u;
     if (__any_sync(0xffffffffu, e4 != 0u || P != 0.f)) {
@@ -669,21 +696,27 @@ struct ReplayState {
   float R;
 };
 
-// Replays one piece; advantages overwrite the values in the lane's row,
-// returns go to the ret row.
+// Replays one piece from the values the fold left in TMEM (the next group's
+// load in flight while a group is replayed); advantages go to the lane's row
+// of `adv`, returns to its row of `ret`.
 template <bool kCrit>
-__device__ void replay_piece(const GaeArgs &a, float *val, float *ret, int lane, uint32_t act, uint32_t ends,
-                             int64_t t0, const CuView &cu, int blo, int b_last, ReplayState<kCrit> &rs) {
+__device__ void replay_piece(const GaeArgs &a, uint32_t tcol, float *adv, float *ret, int lane, uint32_t act,
+                             uint32_t ends, int64_t t0, const CuView &cu, int blo, int b_last,
+                             ReplayState<kCrit> &rs) {
   Coefs<kCrit> k = rs.k;
   float R = rs.R;
   GState st = rs.st;
   const int sw = lane & 7;
+  uint32_t nx[4];
+  tmem_ld4(tcol + 28, nx);
+  tmem_wait_ld4(nx);
 #pragma unroll 1
   for (int g = 7; g >= 0; --g) {
-    float4 *vp = reinterpret_cast<float4 *>(&val[4 * (8 * lane + (g ^ sw))]);
+    float4 *vp = reinterpret_cast<float4 *>(&adv[4 * (8 * lane + (g ^ sw))]);
     float4 *rp = reinterpret_cast<float4 *>(&ret[4 * (8 * lane + (g ^ sw))]);
-    const float4 v4 = *vp;
-    const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
+    const float vv[4] = {__uint_as_float(nx[0]), __uint_as_float(nx[1]), __uint_as_float(nx[2]),
+                         __uint_as_float(nx[3])};
+    if (g > 0) tmem_ld4(tcol + 4 * (g - 1), nx);
     float ov[4], orr[4];
     const uint32_t a4 = (act >> (4 * g)) & 15u, e4 = (ends >> (4 * g)) & 15u;
     if (__any_sync(0xffffffffu, e4 != 0u || st.P != 0.f)) {
@@ -729,18 +762,17 @@ __device__ void replay_piece(const GaeArgs &a, float *val, float *ret, int lane,
     }
     *vp = make_float4(ov[0], ov[1], ov[2], ov[3]);
     *rp = make_float4(orr[0], orr[1], orr[2], orr[3]);
+    if (g > 0) tmem_wait_ld4(nx);
   }
   rs.k = k;
   rs.R = R;
   rs.st = st;
 }
 
-// What a lane keeps about a folded chunk until its look-back is done.
+// What a lane keeps about a folded chunk for its look-back and replay.
 template <bool kCrit>
 struct Pending {
   int q;           // chunk index
-  int buf;         // one piece per segment: the value buffer holding the chunk
-  uint32_t act;    // one piece per segment: the lane's action bits
   int blo, bhi;    // trajectories the chunk can touch
   int b_seg;       // trajectory of the lane's last token below N
   GMap<kCrit> E;   // maps of the lanes to the right within the chunk
@@ -754,25 +786,25 @@ __device__ __forceinline__ int take_chunk(const GaeArgs &a, int lane) {
 }
 
 // Folds each lane's segment of chunk q piece by piece (right to left, the
-// next piece copied while the current one is folded), scans the lane maps and
-// publishes the chunk's map (or, when it ignores its right neighbour, its
-// left-edge state). Nothing here waits on another warp.
+// next piece copied while the current one is folded and its values kept in
+// TMEM), scans the lane maps and publishes the chunk's map (or, when it
+// ignores its right neighbour, its left-edge state). Nothing here waits on
+// another warp.
 template <bool kCrit>
-__device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, int lane, int q, int buf, Pending<kCrit> &p) {
+__device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane, int q, Pending<kCrit> &p) {
   const int seg = 32 * a.pieces;
-  const bool one = a.pieces == 1;  // the chunk stays in val[buf] until its replay
   const int64_t c0 = int64_t(q) * kChunk * a.pieces;
   const int64_t s0 = c0 + int64_t(lane) * seg;  // the lane's segment
   const int64_t N = a.N;
-  const uint64_t keep = l2_policy(true);
-  stage_in(a, c0, seg, a.pieces - 1, lane, w.val[one ? buf : 0], w.msk, keep);
+  const uint64_t pol = l2_evict_first();
+  stage_in(a, c0, seg, a.pieces - 1, lane, w.val[0], w.msk, pol);
 
   // This chunk's slice of cu_seqlens, in shared memory when it fits.
   const int sub0 = q * a.pieces, sub1 = (q + 1) * a.pieces;
   const int blo = __ldg(a.chunk_first + sub0);
   const int bhi = sub1 < a.nsub ? __ldg(a.chunk_first + sub1) : a.B - 1;
   const int ncu = bhi - blo + 2;  // cu[blo .. bhi + 1]
-  const CuView cu{a.cu, w.cu, blo, ncu <= kCuCap};
+  const CuView cu{a.cu, w.cu, blo, ncu <= kScanCuCap};
   if (cu.in_smem)
     for (int i = lane; i < ncu; i += 32) w.cu[i] = __ldg(a.cu + blo + i);
   __syncwarp();
@@ -786,22 +818,23 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, int lane, int q, int bu
   f.Vn = f.P = 0.f;
   f.fl = 0;
   f.nact = 0;
-  uint32_t act = 0;
 #pragma unroll 1
   for (int k = a.pieces - 1; k >= 0; --k) {
-    const int cur = one ? buf : (a.pieces - 1 - k) & 1;
+    const int cur = (a.pieces - 1 - k) & 1;
     cp_async_wait_all();
     __syncwarp();
-    act = row_actions(w.msk, lane);
+    const uint32_t act = row_actions(w.msk, lane);
+    w.act[k][lane] = act;
     __syncwarp();  // every lane has read the flags and finished the previous piece
-    if (k > 0) stage_in(a, c0, seg, k - 1, lane, w.val[cur ^ 1], w.msk, keep);
+    if (k > 0) stage_in(a, c0, seg, k - 1, lane, w.val[cur ^ 1], w.msk, pol);
     const int64_t t0 = s0 + 32 * int64_t(k);
     int b_last;
     const uint32_t ends = piece_ends(a, cu, blo, bhi, t0, b_last);
     // every lane folds (the token loops vote across the warp); a lane past N
     // has no flags and keeps its state
-    fold_piece<kCrit>(a, w.val[cur], lane, act, ends, t0, cu, blo, b_last, f);
+    fold_piece<kCrit>(a, w.val[cur], tmem + 32 * k, lane, act, ends, t0, cu, blo, b_last, f);
   }
+  tmem_wait_st();  // the values are in TMEM before the replay reads them
 
   // the suffix scan of the warp's 32 lane maps
   GMap<kCrit> S = lane_map<kCrit>(f);
@@ -822,27 +855,21 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, int lane, int q, int bu
       publish_map<kCrit>(a.agg + size_t(q) * kMapWords<kCrit>, S);
   }
   p.q = q;
-  p.buf = buf;
-  p.act = act;
   p.blo = blo;
   p.bhi = bhi;
   p.b_seg = b_seg;
   p.E = E;
   p.S = S;
-  __syncwarp();  // the staging buffers are free for the replay of the previous chunk
 }
 
 // Looks back for the state at the chunk's right edge, publishes its left-edge
-// state, then re-stages the chunk piece by piece (right to left), replays the
-// tokens and stores advantages and returns.
+// state, then replays the tokens piece by piece (right to left) from TMEM and
+// stores advantages and returns.
 template <bool kCrit>
-__device__ void finish_chunk(const GaeArgs &a, WarpBuf &w, int lane, const Pending<kCrit> &p) {
+__device__ void replay_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane, const Pending<kCrit> &p) {
   const int seg = 32 * a.pieces;
   const int64_t c0 = int64_t(p.q) * kChunk * a.pieces;
   const int64_t s0 = c0 + int64_t(lane) * seg;
-  const bool one = a.pieces == 1;  // the chunk is still in val[p.buf]
-  const uint64_t drop = l2_policy(false);
-  if (!one) stage_in(a, c0, seg, a.pieces - 1, lane, w.val[0], w.msk, drop);  // lands while the look-back runs
   const bool last = (p.q == a.nchunks - 1);
   const bool reset = __shfl_sync(0xffffffffu, p.S.fl & 1, 0) != 0;  // lane 0 holds the chunk's map
   GState right = zero_state();
@@ -858,48 +885,48 @@ __device__ void finish_chunk(const GaeArgs &a, WarpBuf &w, int lane, const Pendi
   rs.R = __ldg(a.rewards + p.b_seg);
 #pragma unroll 1
   for (int k = a.pieces - 1; k >= 0; --k) {
-    const int cur = one ? p.buf : (a.pieces - 1 - k) & 1;
-    uint32_t act = p.act;
-    if (!one) {
-      cp_async_wait_all();
-      __syncwarp();
-      act = row_actions(w.msk, lane);
-      __syncwarp();  // every lane has read the flags; the other buffer's piece is stored
-      if (k > 0) stage_in(a, c0, seg, k - 1, lane, w.val[cur ^ 1], w.msk, drop);
-    }
+    const uint32_t act = w.act[k][lane];
     const int64_t t0 = s0 + 32 * int64_t(k);
     int b_last;
     const uint32_t ends = piece_ends(a, cu, p.blo, p.bhi, t0, b_last);
-    replay_piece<kCrit>(a, w.val[cur], w.ret, lane, act, ends, t0, cu, p.blo, b_last, rs);
+    replay_piece<kCrit>(a, tmem + 32 * k, w.val[0], w.ret, lane, act, ends, t0, cu, p.blo, b_last, rs);
     __syncwarp();
-    stage_out(a, c0, seg, k, lane, w.val[cur], w.ret);
-    __syncwarp();
+    stage_out(a, c0, seg, k, lane, w.val[0], w.ret);
+    __syncwarp();  // every lane has read its granules before the next piece overwrites them
   }
 }
 
-// Persistent warps, software-pipelined: a warp takes a chunk (ticket), folds
-// and publishes it, and only then looks back for the chunk it took before, so
-// the chunks it waits on have had a whole fold to publish. Tickets keep the
-// decoupled look-back safe: a warp waits only on chunks taken before its own,
-// and every taken chunk is published before its warp waits on anything.
+// Persistent warps: a warp takes a chunk (ticket), folds and publishes it,
+// looks back and replays it, and takes the next. Tickets keep the decoupled
+// look-back safe: a warp waits only on chunks taken before its own, and every
+// taken chunk is folded and published at once, before its warp waits on
+// anything. Each CTA holds kTmemCols TMEM columns for the whole launch (four
+// CTAs per SM take all 512, so the allocation never waits on this kernel).
 template <bool kCrit>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) gae_scan_kernel(GaeArgs a) {
   extern __shared__ __align__(16) unsigned char s_raw[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  WarpBuf &w = reinterpret_cast<WarpBuf *>(s_raw)[warp];
-  int q = take_chunk(a, lane);
-  if (q < 0) return;
-  Pending<kCrit> p;
-  int buf = 0;
-  fold_chunk<kCrit>(a, w, lane, q, buf, p);
-  for (;;) {
-    const int qn = take_chunk(a, lane);
-    Pending<kCrit> n;
-    if (qn >= 0) fold_chunk<kCrit>(a, w, lane, qn, buf ^ 1, n);
-    finish_chunk<kCrit>(a, w, lane, p);
-    if (qn < 0) break;
-    p = n;
-    buf ^= 1;
+  WarpBuf *wb = reinterpret_cast<WarpBuf *>(s_raw);
+  WarpBuf &w = wb[warp];
+  if (warp == 0) {
+    tc::tmem_alloc(static_cast<uint32_t>(__cvta_generic_to_shared(&wb[0].tmem)), kTmemCols);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = wb[0].tmem + (uint32_t(32 * warp) << 16);  // the warp's TMEM lanes
+#pragma unroll 1
+  for (int q = take_chunk(a, lane); q >= 0; q = take_chunk(a, lane)) {
+    Pending<kCrit> p;
+    fold_chunk<kCrit>(a, w, tmem, lane, q, p);
+    replay_chunk<kCrit>(a, w, tmem, lane, p);
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(wb[0].tmem, kTmemCols);
   }
 }
 
@@ -969,7 +996,7 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   const int64_t nchunks = (N + kChunk - 1) / kChunk;
   if (nchunks > (int64_t(1) << 30)) return fail(SAO_ERR_SHAPE, "too many tokens for the advantage scan");
   int pieces = 1;
-  while (pieces < 8 && (N >> 24) >= 2 * pieces) pieces *= 2;
+  while (pieces < kMaxPieces && (N >> 24) >= 2 * pieces) pieces *= 2;
   const int64_t nscan = (N + int64_t(kChunk) * pieces - 1) / (int64_t(kChunk) * pieces);
   const bool crit_trivial = (gamma == 1.0f && lam_c == 1.0f);
   const size_t map_words = crit_trivial ? kMapWords<false> : kMapWords<true>;
