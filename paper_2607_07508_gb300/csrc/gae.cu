@@ -872,17 +872,20 @@ __device__ void replay_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int la
   const int64_t s0 = c0 + int64_t(lane) * seg;
   const bool last = (p.q == a.nchunks - 1);
   const bool reset = __shfl_sync(0xffffffffu, p.S.fl & 1, 0) != 0;  // lane 0 holds the chunk's map
+  // the coefficients and reward of the lane's last trajectory, loaded while
+  // the look-back runs
+  ReplayState<kCrit> rs;
+  rs.k = load_coefs<kCrit>(a.coef, p.b_seg);
+  rs.R = __ldg(a.rewards + p.b_seg);
   GState right = zero_state();
   if (!last) right = look_back<kCrit>(a, p.q, lane);
   if (lane == 0 && !reset && !last)
     publish_state<kCrit>(a.incl + size_t(p.q) * kStateWords<kCrit>, apply<kCrit>(p.S, right));
   // every lane replays (the token loops vote across the warp); rows past N
-  // are never stored
-  const CuView cu{a.cu, nullptr, p.blo, false};  // ends are rare: read cu_seqlens from global memory
-  ReplayState<kCrit> rs;
+  // are never stored. The fold's copy of the chunk's cu_seqlens slice is
+  // still in shared memory.
+  const CuView cu{a.cu, w.cu, p.blo, p.bhi - p.blo + 2 <= kScanCuCap};
   rs.st = apply<kCrit>(p.E, right);
-  rs.k = load_coefs<kCrit>(a.coef, p.b_seg);
-  rs.R = __ldg(a.rewards + p.b_seg);
 #pragma unroll 1
   for (int k = a.pieces - 1; k >= 0; --k) {
     const uint32_t act = w.act[k][lane];
