@@ -18,24 +18,27 @@
 // leaves, where B = Vn = 0). Each action token maps S affinely
 // (B' = a B + g Vn + P, Vn' = V, P' = 0); the last token of a trajectory
 // resets S to (0, 0, 0, R_b). Maps compose associatively, so:
-//   * a warp owns a 1024-token chunk, each lane 32 consecutive tokens; the
-//     chunk is copied into shared memory with cp.async (16-byte granules,
-//     rows XOR-swizzled so that both the coalesced copies and the lane-major
-//     row reads are free of bank conflicts),
-//   * each lane folds its 32 tokens into one map, driven by two bit masks
+//   * a warp owns a chunk of 32 lane segments, each lane 32 * pieces
+//     consecutive tokens (pieces = 1, 2 or 4, from N); the segments stream
+//     through shared memory one 32-token piece at a time with cp.async
+//     (16-byte granules, rows XOR-swizzled so that both the coalesced copies
+//     and the lane-major row reads are free of bank conflicts),
+//   * each lane folds its segment into one map, driven by two bit masks
 //     (action tokens, trajectory ends) so the common token costs one fused
-//     double-float a*B + g*V, a few selects and no index arithmetic,
+//     double-float a*B + g*V, a few selects and no index arithmetic, and
+//     keeps its values in its own TMEM lane for the replay (the scan issues
+//     no MMA, so the SM's 256 KB of TMEM is free: 4 CTAs x 128 columns),
 //   * a warp-shuffle suffix scan combines the 32 maps of the chunk,
-//   * warps chain their chunks right-to-left by decoupled look-back: each CTA
-//     takes one ticket and its warps work on the chunks below it, so a warp
-//     only ever waits on chunks whose warps started before it; the look-back
-//     polls 32 predecessors at once and carries the nearest known state
-//     through the maps before it one by one (so results do not depend on
-//     timing); maps and states are published as tagged 8-byte words, so
-//     neither side needs a fence; every wait is bounded and a time-out raises
-//     SAO_DEVERR_SCAN_TIMEOUT,
-//   * each lane then replays its tokens from its incoming state, writing A
-//     and the return into shared memory, and the warp stores both coalesced.
+//   * warps chain their chunks right-to-left by decoupled look-back: chunks
+//     are taken by ticket, so a warp only ever waits on chunks taken before
+//     its own; the look-back polls 32 predecessors at once and carries the
+//     nearest known state through the maps before it one by one (so results
+//     do not depend on timing); maps and states are published as tagged
+//     8-byte words, so neither side needs a fence; every wait is bounded and
+//     a time-out raises SAO_DEVERR_SCAN_TIMEOUT,
+//   * each lane then replays its tokens from TMEM, starting from its incoming
+//     state, writing A and the return into shared memory, and the warp
+//     stores both coalesced.
 // Traffic: values 4 B + mask 1 B read, adv 4 B + ret 4 B written per token.
 #include <stdint.h>
 
