@@ -26,14 +26,25 @@ namespace sao {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kRowsPerBlock = 4096;
+constexpr int kRowsPerBlock = 4096;       // tokens per block: the unit of the step offsets and of the broadcast
+constexpr int kCountRows = 16384;         // tokens per CTA of the count and scatter passes (4 blocks)
+constexpr int kTokensPerThread = kCountRows / kThreads;  // 64: four 16-byte loads in flight
+constexpr int kSubBlocks = kCountRows / kRowsPerBlock;
+constexpr int kWarpsPerBlock = kRowsPerBlock / kTokensPerThread / 32;  // 2
 constexpr int kShortStep = 32;  // a step this long or shorter is summed by one lane
 
-__global__ void mark_traj_starts(const int32_t *cu, int B, int64_t N, uint8_t *traj_start) {
+// Trajectory starts as a bit mask over the tokens (bit t & 31 of word t >> 5).
+__global__ void mark_traj_starts(const int32_t *cu, int B, int64_t N, uint32_t *tsb) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
   const int64_t t = cu[b];
-  if (t >= 0 && t < N && cu[b + 1] > t) traj_start[t] = 1;
+  if (t >= 0 && t < N && cu[b + 1] > t) atomicOr(tsb + (t >> 5), 1u << (t & 31));
+}
+// Trajectory-start bits of the n (32, 4 or 1) tokens from t0, a multiple of
+// n (zero past N).
+__device__ __forceinline__ uint32_t ts_bits(const uint32_t *tsb, int64_t N, int64_t t0, int n) {
+  const uint32_t mask = n >= 32 ? 0xFFFFFFFFu : (1u << n) - 1u;
+  return t0 < N ? (__ldg(tsb + (t0 >> 5)) >> (t0 & 31)) & mask : 0u;
 }
 
 // Bit i set when byte i of x is non-zero (i = 0..3).
@@ -42,37 +53,38 @@ __device__ __forceinline__ uint32_t nz4(uint32_t x) {
   return (h * 0x00204081u) >> 28;
 }
 
-// Step starts among the 16 tokens t0 .. t0+15 (bit i: token t0+i opens a
-// step: an action token that opens a trajectory or follows a non-action
-// token), and their action flags. 16-byte loads when the run is in range and
-// aligned, byte loads otherwise.
-__device__ __forceinline__ uint32_t step_starts16(const uint8_t *m, const uint8_t *ts, int64_t N, int64_t t0,
-                                                  uint32_t &act, uint32_t &tstart) {
-  uint32_t M = 0, T = 0;
-  if (t0 + 16 <= N && ((reinterpret_cast<uintptr_t>(m) | reinterpret_cast<uintptr_t>(ts)) & 15u) == 0) {
-    const uint4 mv = __ldg(reinterpret_cast<const uint4 *>(m + t0));
-    const uint4 tv = __ldg(reinterpret_cast<const uint4 *>(ts + t0));
-    M = nz4(mv.x) | nz4(mv.y) << 4 | nz4(mv.z) << 8 | nz4(mv.w) << 12;
-    T = nz4(tv.x) | nz4(tv.y) << 4 | nz4(tv.z) << 8 | nz4(tv.w) << 12;
+// Step starts among the 64 tokens t0 .. t0+63, t0 a multiple of 64 (bit i:
+// token t0+i opens a step: an action token that opens a trajectory or
+// follows a non-action token), their action flags and trajectory starts.
+// Four 16-byte loads in flight when the run is in range and aligned, byte
+// loads otherwise.
+__device__ __forceinline__ uint64_t step_starts64(const uint8_t *m, const uint32_t *tsb, int64_t N, int64_t t0,
+                                                  uint64_t &act, uint64_t &tstart) {
+  uint64_t M = 0;
+  const uint64_t T = uint64_t(ts_bits(tsb, N, t0, 32)) | uint64_t(ts_bits(tsb, N, t0 + 32, 32)) << 32;
+  if (t0 + 64 <= N && (reinterpret_cast<uintptr_t>(m) & 15u) == 0) {
+    uint4 mv[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) mv[k] = __ldg(reinterpret_cast<const uint4 *>(m + t0) + k);
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      M |= uint64_t(nz4(mv[k].x) | nz4(mv[k].y) << 4 | nz4(mv[k].z) << 8 | nz4(mv[k].w) << 12) << (16 * k);
   } else {
-    for (int i = 0; i < 16; ++i)
-      if (t0 + i < N) {
-        M |= uint32_t(m[t0 + i] != 0) << i;
-        T |= uint32_t(ts[t0 + i] != 0) << i;
-      }
+    for (int i = 0; i < 64; ++i)
+      if (t0 + i < N) M |= uint64_t(m[t0 + i] != 0) << i;
   }
-  const uint32_t prev = (M << 1) | uint32_t(t0 > 0 && t0 - 1 < N && m[t0 - 1] != 0);  // bit i: token t0+i-1 acts
+  const uint64_t prev = (M << 1) | uint64_t(t0 > 0 && t0 - 1 < N && m[t0 - 1] != 0);  // bit i: token t0+i-1 acts
   act = M;
   tstart = T;
-  return M & (T | ~prev) & 0xFFFFu;
+  return M & (T | ~prev);
 }
 
-// Step starts per 4096-token block (each thread 16 consecutive tokens).
-__global__ void __launch_bounds__(kThreads) step_count_kernel(const uint8_t *m, const uint8_t *ts, int64_t N,
-                                                              int *block_count) {
-  const int64_t t0 = int64_t(blockIdx.x) * kRowsPerBlock + int64_t(threadIdx.x) * 16;
-  uint32_t act, tst;
-  int c = t0 < N ? __popc(step_starts16(m, ts, N, t0, act, tst)) : 0;
+// Step starts per CTA of kCountRows tokens, each thread 64 consecutive tokens.
+__global__ void __launch_bounds__(kThreads) step_count_kernel(const uint8_t *m, const uint32_t *ts, int64_t N,
+                                                              int *cta_count) {
+  const int64_t t0 = int64_t(blockIdx.x) * kCountRows + int64_t(threadIdx.x) * kTokensPerThread;
+  uint64_t act, tst;
+  int c = t0 < N ? __popcll(step_starts64(m, ts, N, t0, act, tst)) : 0;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
   __shared__ int sh[kThreads / 32];
@@ -81,10 +93,11 @@ __global__ void __launch_bounds__(kThreads) step_count_kernel(const uint8_t *m, 
   if (threadIdx.x == 0) {
     int s = 0;
     for (int w = 0; w < kThreads / 32; ++w) s += sh[w];
-    block_count[blockIdx.x] = s;
+    cta_count[blockIdx.x] = s;
   }
 }
-static_assert(kRowsPerBlock == kThreads * 16, "16 tokens per thread");
+static_assert(kTokensPerThread == 64 && kWarpsPerBlock * 32 * kTokensPerThread == kRowsPerBlock,
+              "64 tokens per thread, whole warps per block");
 
 // Exclusive scan of the per-block step counts in place (one CTA of 1024
 // threads). Thread i owns a run of `per` consecutive counts, `per` a multiple
@@ -152,25 +165,29 @@ __global__ void __launch_bounds__(1024) step_scan_kernel(int *block_count, int n
 }
 
 // Ordered step list with each step's first and one-past-last token.
-__global__ void __launch_bounds__(kThreads) step_scatter_kernel(const uint8_t *m, const uint8_t *ts, int64_t N,
-                                                                const int *block_offset, int *step_first,
+// Also writes, per block of kRowsPerBlock tokens, the steps opened before it
+// (the offsets the step search and the broadcast use).
+__global__ void __launch_bounds__(kThreads) step_scatter_kernel(const uint8_t *m, const uint32_t *ts, int64_t N,
+                                                                const int *cta_offset, int nblocks,
+                                                                int *block_offset, int *step_first,
                                                                 int *step_end) {
-  const int64_t t0 = int64_t(blockIdx.x) * kRowsPerBlock + int64_t(threadIdx.x) * 16;
+  const int64_t t0 = int64_t(blockIdx.x) * kCountRows + int64_t(threadIdx.x) * kTokensPerThread;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  uint32_t act = 0, st = 0, tst = 0;
-  if (t0 < N) st = step_starts16(m, ts, N, t0, act, tst);
-  // does token t0+16 continue a step? (an action token that opens no trajectory)
-  uint32_t nact = __shfl_down_sync(0xffffffffu, act, 1), ntst = __shfl_down_sync(0xffffffffu, tst, 1);
+  uint64_t act = 0, st = 0, tst = 0;
+  if (t0 < N) st = step_starts64(m, ts, N, t0, act, tst);
+  // does token t0+64 continue a step? (an action token that opens no trajectory)
+  const uint32_t lo_act = uint32_t(act), lo_tst = uint32_t(tst);
+  uint32_t nact = __shfl_down_sync(0xffffffffu, lo_act, 1), ntst = __shfl_down_sync(0xffffffffu, lo_tst, 1);
   if (lane == 31) {
-    const int64_t u = t0 + 16;
+    const int64_t u = t0 + kTokensPerThread;
     nact = (u < N && m[u] != 0) ? 1u : 0u;
-    ntst = (u < N && ts[u] != 0) ? 1u : 0u;
+    ntst = ts_bits(ts, N, u, 1);
   }
-  const uint32_t cont_next = (nact & ~ntst) & 1u;
+  const uint64_t cont_next = (nact & ~ntst) & 1u;
   // bit i: token t0+i+1 continues the step; last: token t0+i is a step's last token
-  const uint32_t cont = ((act & ~tst) >> 1) | (cont_next << 15);
-  const uint32_t last = act & ~cont & 0xFFFFu;
-  const int c = __popc(st);
+  const uint64_t cont = ((act & ~tst) >> 1) | (cont_next << 63);
+  const uint64_t last = act & ~cont;
+  const int c = __popcll(st);
   // exclusive prefix of the counts over the block
   int x = c;
 #pragma unroll
@@ -181,13 +198,22 @@ __global__ void __launch_bounds__(kThreads) step_scatter_kernel(const uint8_t *m
   __shared__ int sh[kThreads / 32];
   if (lane == 31) sh[warp] = x;
   __syncthreads();
+  const int cta0 = cta_offset[blockIdx.x];
+  if (threadIdx.x < kSubBlocks) {
+    const int blk = blockIdx.x * kSubBlocks + threadIdx.x;
+    int o = cta0;
+    for (int w = 0; w < threadIdx.x * kWarpsPerBlock; ++w) o += sh[w];
+    if (blk < nblocks) block_offset[blk] = o;
+  }
+  if (t0 >= N) return;
   int before = 0;
   for (int w = 0; w < warp; ++w) before += sh[w];
-  const int base = block_offset[blockIdx.x] + before + x - c;  // steps opened before token t0
-  if (t0 >= N) return;
+  const int base = cta0 + before + x - c;  // steps opened before token t0
   int k = base;
-#pragma unroll
-  for (int i = 0; i < 16; ++i) {
+  uint64_t bits = st | last;
+  while (bits) {
+    const int i = __ffsll(static_cast<long long>(bits)) - 1;
+    bits &= bits - 1;
     if ((st >> i) & 1u) step_first[k++] = int(t0 + i);
     if ((last >> i) & 1u) step_end[k - 1] = int(t0 + i + 1);
   }
@@ -283,14 +309,14 @@ __global__ void __launch_bounds__(kThreads) step_reduce_kernel(const float *valu
     const bool shortstep = own && end - first <= kShortStep;
     Acc2 acc;
     if (shortstep) {
-      // 4 tokens at a time, the loads of a group (the ragged last one too)
+      // 8 tokens at a time, the loads of a group (the ragged last one too)
       // issued before its adds, which keep the token order
-      for (int t = first; t < end; t += 4) {
-        float x[4];
+      for (int t = first; t < end; t += 8) {
+        float x[8];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) x[k] = t + k < end ? values[t + k] : 0.f;
+        for (int k = 0; k < 8; ++k) x[k] = t + k < end ? values[t + k] : 0.f;
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
+        for (int k = 0; k < 8; ++k)
           if (t + k < end) acc.add(x[k]);
       }
     }
@@ -300,13 +326,13 @@ __global__ void __launch_bounds__(kThreads) step_reduce_kernel(const float *valu
       longs &= longs - 1;
       const int f = __shfl_sync(0xffffffffu, first, src), e = __shfl_sync(0xffffffffu, end, src);
       Acc2 part;
-      // a lane's tokens f + lane, f + lane + 32, ... in order, four loads at a time
-      for (int t = f + lane; t < e; t += 128) {
-        float x[4];
+      // a lane's tokens f + lane, f + lane + 32, ... in order, eight loads at a time
+      for (int t = f + lane; t < e; t += 256) {
+        float x[8];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) x[k] = t + 32 * k < e ? values[t + 32 * k] : 0.f;
+        for (int k = 0; k < 8; ++k) x[k] = t + 32 * k < e ? values[t + 32 * k] : 0.f;
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
+        for (int k = 0; k < 8; ++k)
           if (t + 32 * k < e) part.add(x[k]);
       }
 #pragma unroll
@@ -476,34 +502,31 @@ __device__ __forceinline__ void step_result(int s, int64_t t, const int *step_en
 
 // Action flags and trajectory-start flags of the 4 tokens t0 .. t0+3 (bits),
 // zero past N.
-__device__ __forceinline__ void flags4(const uint8_t *m, const uint8_t *ts, int64_t N, int64_t t0, bool vec,
+__device__ __forceinline__ void flags4(const uint8_t *m, const uint32_t *ts, int64_t N, int64_t t0, bool vec,
                                       uint32_t &M, uint32_t &T) {
+  T = ts_bits(ts, N, t0, 4);
   if (vec && t0 + 4 <= N) {
     M = nz4(__ldg(reinterpret_cast<const uint32_t *>(m + t0)));
-    T = nz4(__ldg(reinterpret_cast<const uint32_t *>(ts + t0)));
   } else {
-    M = T = 0;
+    M = 0;
     for (int i = 0; i < 4; ++i)
-      if (t0 + i < N) {
-        M |= uint32_t(m[t0 + i] != 0) << i;
-        T |= uint32_t(ts[t0 + i] != 0) << i;
-      }
+      if (t0 + i < N) M |= uint32_t(m[t0 + i] != 0) << i;
   }
 }
 
 // Every token gets its step's results (non-action tokens get zeros). A CTA
-// takes a 4096-token block, as the count pass did, and a warp 512 tokens as
-// four 128-token groups with 4 tokens per lane, so every load and store of
-// the warp is contiguous. Step indices are recounted from the step starts:
-// the block's offset from the scan, the warps before this one through shared
+// takes a block of kRowsPerBlock tokens and a warp 512 tokens as four
+// 128-token groups with 4 tokens per lane, so every load and store of the
+// warp is contiguous. Step indices are recounted from the step starts: the
+// block's offset from the scan, the warps before this one through shared
 // memory, the lanes before this one by a warp scan.
-__global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const uint8_t *m, const uint8_t *ts, int64_t N,
+__global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const uint8_t *m, const uint32_t *ts, int64_t N,
                                                                   const int *block_offset, const int *step_end,
                                                                   const float2 *out, int mode, float *adv, float *ret,
                                                                   uint8_t *vmask) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t wbase = int64_t(blockIdx.x) * kRowsPerBlock + int64_t(warp) * 512;
-  const bool vin = ((reinterpret_cast<uintptr_t>(m) | reinterpret_cast<uintptr_t>(ts)) & 3u) == 0;
+  const bool vin = (reinterpret_cast<uintptr_t>(m) & 3u) == 0;
   const bool vout = ((reinterpret_cast<uintptr_t>(adv) | reinterpret_cast<uintptr_t>(ret)) & 15u) == 0 &&
                     (reinterpret_cast<uintptr_t>(vmask) & 3u) == 0;
   uint32_t act[4], st[4];
@@ -569,7 +592,9 @@ __global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const uint8_t 
 size_t step_gae_ws_bytes(int64_t N, int64_t B) {
   (void)B;
   const int64_t nblocks = (N + kRowsPerBlock - 1) / kRowsPerBlock;
-  return round256(size_t(N)) + round256(sizeof(int) * (nblocks + 1)) + round256(sizeof(int) * 4) +
+  const int64_t nctas = (N + kCountRows - 1) / kCountRows;
+  return round256(sizeof(uint32_t) * size_t((N + 31) / 32)) + round256(sizeof(int) * (nctas + 1)) +
+         round256(sizeof(int) * (nblocks + 1)) + round256(sizeof(int) * 4) +
          round256(sizeof(int) * N) + round256(sizeof(int) * N) + round256(sizeof(float2) * N) +
          round256(sizeof(float2) * N);
 }
@@ -580,7 +605,10 @@ sao_status step_gae_launch(const float *values, const float *rewards, const uint
   if (N == 0) return SAO_OK;
   const int64_t nblocks = (N + kRowsPerBlock - 1) / kRowsPerBlock;
   Carver c(ws_body, body_bytes);
-  uint8_t *ts = c.take<uint8_t>(size_t(N));
+  const size_t ts_words = size_t((N + 31) / 32);
+  uint32_t *ts = c.take<uint32_t>(ts_words);
+  const int64_t nctas = (N + kCountRows - 1) / kCountRows;
+  int *cta = c.take<int>(size_t(nctas) + 1);
   int *block = c.take<int>(size_t(nblocks) + 1);
   int *nsteps = c.take<int>(4);
   int *step_first = c.take<int>(size_t(N));
@@ -590,12 +618,13 @@ sao_status step_gae_launch(const float *values, const float *rewards, const uint
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the step-level advantages");
   DeviceInfo di;
   SAO_TRY(device_info(&di));
-  SAO_CUDA_TRY(cudaMemsetAsync(ts, 0, size_t(N), s));
+  SAO_CUDA_TRY(cudaMemsetAsync(ts, 0, sizeof(uint32_t) * ts_words, s));
   int slot = launch_begin("step_gae_segments", s);
   mark_traj_starts<<<unsigned((B + 255) / 256), 256, 0, s>>>(cu, B, N, ts);
-  step_count_kernel<<<unsigned(nblocks), kThreads, 0, s>>>(m, ts, N, block);
-  step_scan_kernel<<<1, 1024, 0, s>>>(block, int(nblocks), nsteps);
-  step_scatter_kernel<<<unsigned(nblocks), kThreads, 0, s>>>(m, ts, N, block, step_first, step_end);
+  const unsigned count_grid = unsigned((N + kCountRows - 1) / kCountRows);
+  step_count_kernel<<<count_grid, kThreads, 0, s>>>(m, ts, N, cta);
+  step_scan_kernel<<<1, 1024, 0, s>>>(cta, int(nctas), nsteps);
+  step_scatter_kernel<<<count_grid, kThreads, 0, s>>>(m, ts, N, cta, int(nblocks), block, step_first, step_end);
   SAO_TRY(launch_end(slot, s));
   const unsigned warps_grid = unsigned(di.sm_count * 8);
   slot = launch_begin("step_gae_reduce", s);
