@@ -472,6 +472,7 @@ def bandwidth_study(args):
     hist = torch.zeros(64, 8, dtype=torch.float32, device=dev)
     seen = torch.zeros(64, dtype=torch.int64, device=dev)
 
+    n_act = int(wl.loss_mask.astype(np.int64).sum())
     # whole calls with their algorithmic bytes per token (reads + writes)
     whole = {
         "sao_advantages": (13, lambda: sao.sao_advantages(v, R, m, cu, wl.gamma, wl.lam, wl.lam_critic, 0.0,
@@ -483,6 +484,10 @@ def bandwidth_study(args):
                                                                     value_mask=vm)),
         "sao_policy_loss_fwd": (18, lambda: sao.sao_policy_loss_fwd(lp, old, adv, m, wl.eps_low, wl.eps_high, loss,
                                                                     counts, ws, coef=coef, flags=flags)),
+        # a trainer that knows its normaliser (the data-parallel action-token
+        # total) passes it: the forward then needs no count pass
+        "sao_policy_loss_fwd (n_norm given)": (18, lambda: sao.sao_policy_loss_fwd(
+            lp, old, adv, m, wl.eps_low, wl.eps_high, loss, counts, ws, coef=coef, flags=flags, n_norm=n_act)),
         "sao_value_loss": (13, lambda: sao.sao_value_loss(v, ret, m, loss, dV, ws, ev_sums=ev)),
         "sao_clip_loss_fwd": (18, lambda: sao.sao_clip_loss_fwd(lp, old, adv, m, cu, 0.2, 0.28,
                                                                 sao.SAO_NORM_SEQUENCE, loss, counts, ws, coef=coef,
@@ -492,6 +497,8 @@ def bandwidth_study(args):
         "sao_decoupled_loss_fwd": (22, lambda: sao.sao_decoupled_loss_fwd(lp, old, roll, adv, m, 0.2, 0.28, 0.5,
                                                                           2.0, loss, counts6, ws, coef=coef,
                                                                           flags=flags)),
+        "sao_decoupled_loss_fwd (n_norm given)": (22, lambda: sao.sao_decoupled_loss_fwd(
+            lp, old, roll, adv, m, 0.2, 0.28, 0.5, 2.0, loss, counts6, ws, coef=coef, flags=flags, n_norm=n_act)),
         "sao_group_advantages": (5, lambda: sao.sao_group_advantages(R, gid, m, cu, 1e-6, adv, ws)),
         "sao_running_mean_advantages": (5, lambda: sao.sao_running_mean_advantages(R, pid, hist, seen, m, cu, adv,
                                                                                    ws)),

@@ -140,12 +140,17 @@ struct PLArgs {
   int64_t n_norm;
   const long long *cnt_partial;
   int n_cnt;
+  long long *act_out;  // fwd with n_norm > 0: per-CTA action-token counts (no count pass ran)
   float *coef;       // may be null
   uint8_t *flags;    // may be null
   const float *grad_scale;  // bwd: device scalar; fwd: null
   double *loss_partial;
   long long *cnt3_partial;  // [3][grid]
 };
+
+__device__ __forceinline__ int nonzero4(uchar4 m) {
+  return (m.x != 0) + (m.y != 0) + (m.z != 0) + (m.w != 0);
+}
 
 template <bool kBwd>
 __global__ void __launch_bounds__(kThreads) policy_loss_kernel(PLArgs a) {
@@ -154,7 +159,7 @@ __global__ void __launch_bounds__(kThreads) policy_loss_kernel(PLArgs a) {
   const float inv_n = n > 0 ? float(1.0 / double(n)) : 0.f;
   const float gscale = kBwd ? __ldg(a.grad_scale) : 1.f;
   double acc = 0.0;
-  int n_low = 0, n_high = 0, n_nonfin = 0;
+  int n_low = 0, n_high = 0, n_nonfin = 0, n_act = 0;
 
   const int64_t tid = int64_t(blockIdx.x) * kThreads + threadIdx.x;
   const int64_t stride = int64_t(gridDim.x) * kThreads;
@@ -170,6 +175,7 @@ __global__ void __launch_bounds__(kThreads) policy_loss_kernel(PLArgs a) {
       const float4 od = __ldg(reinterpret_cast<const float4 *>(a.old) + i);
       const float4 ad = __ldg(reinterpret_cast<const float4 *>(a.adv) + i);
       const uchar4 mk = __ldg(reinterpret_cast<const uchar4 *>(a.m) + i);
+      if (!kBwd) n_act += nonzero4(mk);
       float contrib = 0.f;
       PLToken t0 = pl_token(lp.x, od.x, ad.x, mk.x, a.lo, a.hi, inv_n, contrib, n_low, n_high, n_nonfin);
       PLToken t1 = pl_token(lp.y, od.y, ad.y, mk.y, a.lo, a.hi, inv_n, contrib, n_low, n_high, n_nonfin);
@@ -185,7 +191,9 @@ __global__ void __launch_bounds__(kThreads) policy_loss_kernel(PLArgs a) {
   }
   for (int64_t i = done + tid; i < a.N; i += stride) {
     float contrib = 0.f;
-    PLToken t = pl_token(__ldg(a.logp + i), __ldg(a.old + i), __ldg(a.adv + i), __ldg(a.m + i), a.lo,
+    const uint8_t mi = __ldg(a.m + i);
+    if (!kBwd) n_act += mi != 0;
+    PLToken t = pl_token(__ldg(a.logp + i), __ldg(a.old + i), __ldg(a.adv + i), mi, a.lo,
                          a.hi, inv_n, contrib, n_low, n_high, n_nonfin);
     acc += double(contrib);
     if (a.coef) a.coef[i] = t.coef * gscale;
@@ -196,7 +204,9 @@ __global__ void __launch_bounds__(kThreads) policy_loss_kernel(PLArgs a) {
   long long l = block_sum((long long)n_low);
   long long h = block_sum((long long)n_high);
   long long f = block_sum((long long)n_nonfin);
+  const long long na = a.act_out ? block_sum((long long)n_act) : 0;
   if (threadIdx.x == 0) {
+    if (a.act_out) a.act_out[blockIdx.x] = na;
     a.loss_partial[blockIdx.x] = acc;
     a.cnt3_partial[blockIdx.x] = l;
     a.cnt3_partial[gridDim.x + blockIdx.x] = h;
@@ -243,6 +253,7 @@ struct DLArgs {
   int64_t n_norm;
   const long long *cnt_partial;
   int n_cnt;
+  long long *act_out;  // fwd with n_norm > 0: per-CTA action-token counts (no count pass ran)
   float *coef;              // may be null
   uint8_t *flags;           // may be null
   const float *grad_scale;  // bwd: device scalar; fwd: null
@@ -304,6 +315,7 @@ __global__ void __launch_bounds__(kThreads) decoupled_loss_kernel(DLArgs a) {
   const float gscale = kBwd ? __ldg(a.grad_scale) : 1.f;
   double acc = 0.0;
   DLCounts c;
+  int n_act = 0;
   const int64_t tid = int64_t(blockIdx.x) * kThreads + threadIdx.x;
   const int64_t stride = int64_t(gridDim.x) * kThreads;
   const bool vec = aligned16_dev(a.logp) && aligned16_dev(a.prox) && aligned16_dev(a.roll) &&
@@ -319,6 +331,7 @@ __global__ void __launch_bounds__(kThreads) decoupled_loss_kernel(DLArgs a) {
       const float4 ro = __ldcs(reinterpret_cast<const float4 *>(a.roll) + i);
       const float4 ad = __ldcs(reinterpret_cast<const float4 *>(a.adv) + i);
       const uchar4 mk = __ldcs(reinterpret_cast<const uchar4 *>(a.m) + i);
+      if (!kBwd) n_act += nonzero4(mk);
       float contrib = 0.f;
       const PLToken t0 = dl_token(lp.x, px.x, ro.x, ad.x, mk.x, a, inv_n, contrib, c);
       const PLToken t1 = dl_token(lp.y, px.y, ro.y, ad.y, mk.y, a, inv_n, contrib, c);
@@ -334,8 +347,10 @@ __global__ void __launch_bounds__(kThreads) decoupled_loss_kernel(DLArgs a) {
   }
   for (int64_t i = done + tid; i < a.N; i += stride) {
     float contrib = 0.f;
+    const uint8_t mi = __ldg(a.m + i);
+    if (!kBwd) n_act += mi != 0;
     const PLToken t = dl_token(__ldg(a.logp + i), __ldg(a.prox + i), __ldg(a.roll + i), __ldg(a.adv + i),
-                               __ldg(a.m + i), a, inv_n, contrib, c);
+                               mi, a, inv_n, contrib, c);
     acc += double(contrib);
     if (a.coef) a.coef[i] = t.coef * gscale;
     if (a.flags) a.flags[i] = t.flag;
@@ -345,8 +360,10 @@ __global__ void __launch_bounds__(kThreads) decoupled_loss_kernel(DLArgs a) {
   const long long k0 = block_sum((long long)c.low), k1 = block_sum((long long)c.high);
   const long long k2 = block_sum((long long)c.nonfin), k3 = block_sum((long long)c.wlow);
   const long long k4 = block_sum((long long)c.whigh);
+  const long long na = a.act_out ? block_sum((long long)n_act) : 0;
   if (threadIdx.x == 0) {
     const int g = gridDim.x, b = blockIdx.x;
+    if (a.act_out) a.act_out[b] = na;
     a.loss_partial[b] = acc;
     a.cnt5_partial[b] = k0;
     a.cnt5_partial[g + b] = k1;
@@ -543,7 +560,9 @@ sao_status policy_loss_launch(const float *logp, const float *old, const float *
   double *lossp = c.take<double>(grid);
   long long *cnt3 = c.take<long long>(3 * size_t(grid));
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the policy loss");
-  const bool need_count = (n_norm <= 0) || (grad_loss == nullptr);
+  // the normaliser must be known before the token pass; with n_norm given,
+  // the forward counts the action tokens for `counts` itself
+  const bool need_count = n_norm <= 0;
   if (need_count) SAO_TRY(launch_count(m, N, cnt, grid, s));
   PLArgs a;
   a.logp = logp;
@@ -556,6 +575,7 @@ sao_status policy_loss_launch(const float *logp, const float *old, const float *
   a.n_norm = n_norm;
   a.cnt_partial = cnt;
   a.n_cnt = need_count ? grid : 0;
+  a.act_out = (!need_count && grad_loss == nullptr) ? cnt : nullptr;
   a.coef = coef;
   a.flags = flags;
   a.grad_scale = grad_loss;
@@ -586,7 +606,7 @@ sao_status decoupled_loss_launch(const float *logp, const float *prox, const flo
   double *lossp = c.take<double>(grid);
   long long *cnt5 = c.take<long long>(5 * size_t(grid));
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the decoupled loss");
-  const bool need_count = (n_norm <= 0) || (grad_loss == nullptr);
+  const bool need_count = n_norm <= 0;
   if (need_count) SAO_TRY(launch_count(m, N, cnt, grid, s));
   DLArgs a;
   a.logp = logp;
@@ -602,6 +622,7 @@ sao_status decoupled_loss_launch(const float *logp, const float *prox, const flo
   a.n_norm = n_norm;
   a.cnt_partial = cnt;
   a.n_cnt = need_count ? grid : 0;
+  a.act_out = (!need_count && grad_loss == nullptr) ? cnt : nullptr;
   a.coef = coef;
   a.flags = flags;
   a.grad_scale = grad_loss;

@@ -228,6 +228,7 @@ def test_policy_loss_edge_cases():
         _check_pl(logp, old, adv, mask, 0.2, 0.28)
         _check_pl(logp, old, adv, mask, 0.3, 5.0, n_norm=12345)
         _check_pl(logp, old, adv, mask, 0.8, 3.0, offset=1)     # misaligned: scalar path
+        _check_pl(logp, old, adv, mask, 0.8, 3.0, n_norm=777, offset=1)  # forward counts the action tokens
     # non-finite inputs, masked tokens, exact-bound ratios, eps_low >= 1
     logp = np.array([-1, -1, -1, -1, -1, -30, -1, -1], np.float32)
     old = np.array([-np.inf, -1, np.nan, -1, -1, 0, -1.5, -1], np.float32)
@@ -247,6 +248,8 @@ def test_policy_loss_bandwidth_size():
     wl = S.bandwidth_workload()
     adv = (np.random.default_rng(1).standard_normal(wl.N, dtype=np.float32))
     _check_pl(wl.logp_syn, wl.old_logp_syn, adv, wl.loss_mask, wl.eps_low, wl.eps_high)
+    # with the normaliser given, the forward counts the action tokens itself
+    _check_pl(wl.logp_syn, wl.old_logp_syn, adv, wl.loss_mask, wl.eps_low, wl.eps_high, n_norm=int(wl.N))
 
 
 # ---------------------------------------------------------------------------
