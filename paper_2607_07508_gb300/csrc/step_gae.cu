@@ -486,102 +486,87 @@ __global__ void __launch_bounds__(32 * kGaeWarps) step_gae_kernel(const float *r
   for (; i >= a0; --i) replay(i, sv[i]);
 }
 
-// Every token reads its step's results (non-action tokens get zeros); four
-// consecutive tokens per thread.
-__device__ __forceinline__ void step_result(int s, int64_t t, const int *step_end, const float2 *out, int mode,
-                                            float &a, float &r, uint8_t &k) {
-  a = r = 0.f;
-  k = 0;
-  if (s >= 0) {
-    const float2 o = out[s];
-    a = o.x;
-    r = o.y;
-    k = (mode == SAO_STEP_AVERAGE || t == int64_t(step_end[s]) - 1) ? 1 : 0;
+// Every token gets its step's results (non-action tokens get zeros), step by
+// step: a warp takes 32 consecutive steps (one per lane: first token, end,
+// results) and writes the tokens from its first step's first token to the
+// next group's (the steps and the observation tokens after each), in
+// 128-token windows with 4 tokens per lane, so every store of the warp is
+// contiguous. A lane finds the step of its tokens by a binary search over the
+// 32 first tokens held in the warp's lanes; the first group also writes the
+// tokens before the first step. Neither the mask nor the flags are read again.
+__device__ __forceinline__ int steps_at_or_before(int F, int t) {  // #{j : F_j <= t}, F_j rising over the lanes
+  int pos = 0;
+#pragma unroll
+  for (int b = 16; b >= 1; b >>= 1) {
+    const int f = __shfl_sync(0xffffffffu, F, pos + b - 1);
+    if (f <= t) pos += b;
   }
+  const int f31 = __shfl_sync(0xffffffffu, F, 31);
+  return (pos == 31 && f31 <= t) ? 32 : pos;
 }
 
-// Action flags and trajectory-start flags of the 4 tokens t0 .. t0+3 (bits),
-// zero past N.
-__device__ __forceinline__ void flags4(const uint8_t *m, const uint32_t *ts, int64_t N, int64_t t0, bool vec,
-                                      uint32_t &M, uint32_t &T) {
-  T = ts_bits(ts, N, t0, 4);
-  if (vec && t0 + 4 <= N) {
-    M = nz4(__ldg(reinterpret_cast<const uint32_t *>(m + t0)));
-  } else {
-    M = 0;
-    for (int i = 0; i < 4; ++i)
-      if (t0 + i < N) M |= uint32_t(m[t0 + i] != 0) << i;
-  }
-}
-
-// Every token gets its step's results (non-action tokens get zeros). A CTA
-// takes a block of kRowsPerBlock tokens and a warp 512 tokens as four
-// 128-token groups with 4 tokens per lane, so every load and store of the
-// warp is contiguous. Step indices are recounted from the step starts: the
-// block's offset from the scan, the warps before this one through shared
-// memory, the lanes before this one by a warp scan.
-__global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const uint8_t *m, const uint32_t *ts, int64_t N,
-                                                                  const int *block_offset, const int *step_end,
-                                                                  const float2 *out, int mode, float *adv, float *ret,
-                                                                  uint8_t *vmask) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int64_t wbase = int64_t(blockIdx.x) * kRowsPerBlock + int64_t(warp) * 512;
-  const bool vin = (reinterpret_cast<uintptr_t>(m) & 3u) == 0;
+__global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const int *nsteps, const int *step_first,
+                                                                  const int *step_end, const float2 *out, int mode,
+                                                                  int64_t N, float *adv, float *ret, uint8_t *vmask) {
+  const int lane = threadIdx.x & 31;
+  const int S = *nsteps;
+  const int ngroups = S > 0 ? (S + 31) / 32 : 1;
+  const int nwarps = (gridDim.x * kThreads) >> 5;
   const bool vout = ((reinterpret_cast<uintptr_t>(adv) | reinterpret_cast<uintptr_t>(ret)) & 15u) == 0 &&
                     (reinterpret_cast<uintptr_t>(vmask) & 3u) == 0;
-  uint32_t act[4], st[4];
-  int x[4], tot[4];  // inclusive lane prefix and warp total of each group's step starts
-  // does the token before the warp's first token act?
-  uint32_t carry = (lane == 0 && wbase > 0 && wbase - 1 < N && m[wbase - 1] != 0) ? 1u : 0u;
-  carry = __shfl_sync(0xffffffffu, carry, 0);
-  int wtot = 0;
+  const bool last_mode = mode != SAO_STEP_AVERAGE;
+  for (int g = (blockIdx.x * kThreads + threadIdx.x) >> 5; g < ngroups; g += nwarps) {
+    const int s = g * 32 + lane;
+    const bool has = s < S;
+    const int F = has ? step_first[s] : INT_MAX;
+    const int E = has ? step_end[s] : 0;
+    const float2 o = has ? out[s] : make_float2(0.f, 0.f);
+    const int lo = g == 0 ? 0 : __shfl_sync(0xffffffffu, F, 0);
+    const int hi = (g + 1) * 32 < S ? step_first[(g + 1) * 32] : int(N);  // the group writes [lo, hi)
+    for (int c = lo & ~3; c < hi; c += 128) {
+      const int t4 = c + 4 * lane;
+      float a[4], r[4];
+      uint8_t k[4];
+      const int j0 = steps_at_or_before(F, t4) - 1;  // step of token t4 in the group (-1: before it)
+      const int fn = __shfl_sync(0xffffffffu, F, j0 + 1 < 32 ? j0 + 1 : 31);
+      const int next = j0 + 1 < 32 ? fn : INT_MAX;  // first token of the step after j0 in the group
+      if (__all_sync(0xffffffffu, next > t4 + 3)) {
+        // the lane's 4 tokens lie in one step's tokens and the gap after them
+        const int src = j0 < 0 ? 0 : j0;
+        const float sa = __shfl_sync(0xffffffffu, o.x, src), sr = __shfl_sync(0xffffffffu, o.y, src);
+        const int se = __shfl_sync(0xffffffffu, E, src);
 #pragma unroll
-  for (int g = 0; g < 4; ++g) {
-    uint32_t M, T;
-    flags4(m, ts, N, wbase + g * 128 + lane * 4, vin, M, T);
-    const uint32_t up = __shfl_up_sync(0xffffffffu, M, 1);
-    const uint32_t prevbit = lane == 0 ? carry : (up >> 3) & 1u;
-    const uint32_t prev = ((M << 1) | prevbit) & 15u;  // bit i: token i-1 acts
-    act[g] = M;
-    st[g] = M & (T | ~prev) & 15u;
-    carry = __shfl_sync(0xffffffffu, M >> 3, 31) & 1u;
-    int v = __popc(st[g]);
+        for (int i = 0; i < 4; ++i) {
+          const bool in = j0 >= 0 && t4 + i < se;
+          a[i] = in ? sa : 0.f;
+          r[i] = in ? sr : 0.f;
+          k[i] = (in && (!last_mode || t4 + i == se - 1)) ? 1 : 0;
+        }
+      } else {
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, v, o);
-      if (lane >= o) v += y;
-    }
-    x[g] = v;
-    tot[g] = __shfl_sync(0xffffffffu, v, 31);
-    wtot += tot[g];
-  }
-  __shared__ int sh[kThreads / 32];
-  if (lane == 0) sh[warp] = wtot;
-  __syncthreads();
-  int run = block_offset[blockIdx.x];
-  for (int w = 0; w < warp; ++w) run += sh[w];
-#pragma unroll
-  for (int g = 0; g < 4; ++g) {
-    const int64_t t0 = wbase + g * 128 + lane * 4;
-    const int before = run + x[g] - __popc(st[g]);  // steps opened before token t0
-    run += tot[g];
-    if (t0 >= N) continue;
-    float a[4], r[4];
-    uint8_t k[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int sid = ((act[g] >> i) & 1u) ? before + __popc(st[g] & ((2u << i) - 1u)) - 1 : -1;
-      step_result(sid, t0 + i, step_end, out, mode, a[i], r[i], k[i]);
-    }
-    if (vout && t0 + 4 <= N) {
-      __stcs(reinterpret_cast<float4 *>(adv + t0), make_float4(a[0], a[1], a[2], a[3]));
-      __stcs(reinterpret_cast<float4 *>(ret + t0), make_float4(r[0], r[1], r[2], r[3]));
-      if (vmask) *reinterpret_cast<uchar4 *>(vmask + t0) = make_uchar4(k[0], k[1], k[2], k[3]);
-    } else {
-      for (int i = 0; i < 4 && t0 + i < N; ++i) {
-        adv[t0 + i] = a[i];
-        ret[t0 + i] = r[i];
-        if (vmask) vmask[t0 + i] = k[i];
+        for (int i = 0; i < 4; ++i) {
+          const int j = steps_at_or_before(F, t4 + i) - 1;
+          const int src = j < 0 ? 0 : j;
+          const float sa = __shfl_sync(0xffffffffu, o.x, src), sr = __shfl_sync(0xffffffffu, o.y, src);
+          const int se = __shfl_sync(0xffffffffu, E, src);
+          const bool in = j >= 0 && t4 + i < se;
+          a[i] = in ? sa : 0.f;
+          r[i] = in ? sr : 0.f;
+          k[i] = (in && (!last_mode || t4 + i == se - 1)) ? 1 : 0;
+        }
+      }
+      if (vout && t4 >= lo && t4 + 3 < hi) {
+        __stcs(reinterpret_cast<float4 *>(adv + t4), make_float4(a[0], a[1], a[2], a[3]));
+        __stcs(reinterpret_cast<float4 *>(ret + t4), make_float4(r[0], r[1], r[2], r[3]));
+        if (vmask) *reinterpret_cast<uchar4 *>(vmask + t4) = make_uchar4(k[0], k[1], k[2], k[3]);
+      } else {
+        for (int i = 0; i < 4; ++i) {
+          const int t = t4 + i;
+          if (t < lo || t >= hi) continue;
+          adv[t] = a[i];
+          ret[t] = r[i];
+          if (vmask) vmask[t] = k[i];
+        }
       }
     }
   }
@@ -603,6 +588,8 @@ sao_status step_gae_launch(const float *values, const float *rewards, const uint
                            int64_t N, float gamma, float lam, float lam_c, float alpha, int mode, float *adv,
                            float *ret, uint8_t *vmask, void *ws_body, size_t body_bytes, cudaStream_t s) {
   if (N == 0) return SAO_OK;
+  // token indices are int32 here, with room for a 128-token window past N
+  if (N > int64_t(INT_MAX) - 256) return fail(SAO_ERR_SHAPE, "too many tokens for the step-level advantages");
   const int64_t nblocks = (N + kRowsPerBlock - 1) / kRowsPerBlock;
   Carver c(ws_body, body_bytes);
   const size_t ts_words = size_t((N + 31) / 32);
@@ -636,8 +623,7 @@ sao_status step_gae_launch(const float *values, const float *rewards, const uint
       rewards, cu, B, N, step_first, block, int(nblocks), nsteps, sv, gamma, lam, lam_c, alpha, out);
   SAO_TRY(launch_end(slot, s));
   slot = launch_begin("step_gae_broadcast", s);
-  step_broadcast_kernel<<<unsigned(nblocks), kThreads, 0, s>>>(m, ts, N, block, step_end, out, mode, adv, ret,
-                                                                vmask);
+  step_broadcast_kernel<<<warps_grid, kThreads, 0, s>>>(nsteps, step_first, step_end, out, mode, N, adv, ret, vmask);
   return launch_end(slot, s);
 }
 
