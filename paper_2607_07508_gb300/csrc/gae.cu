@@ -776,6 +776,7 @@ __device__ void replay_piece(const GaeArgs &a, uint32_t tcol, float *adv, float 
 template <bool kCrit>
 struct Pending {
   int q;           // chunk index
+  int slot;        // TMEM columns from 32 * slot and act rows from slot hold the chunk
   int blo, bhi;    // trajectories the chunk can touch
   int b_seg;       // trajectory of the lane's last token below N
   GMap<kCrit> E;   // maps of the lanes to the right within the chunk
@@ -794,7 +795,7 @@ __device__ __forceinline__ int take_chunk(const GaeArgs &a, int lane) {
 // ignores its right neighbour, its left-edge state). Nothing here waits on
 // another warp.
 template <bool kCrit>
-__device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane, int q, Pending<kCrit> &p) {
+__device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane, int q, int slot, Pending<kCrit> &p) {
   const int seg = 32 * a.pieces;
   const int64_t c0 = int64_t(q) * kChunk * a.pieces;
   const int64_t s0 = c0 + int64_t(lane) * seg;  // the lane's segment
@@ -827,7 +828,7 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane
     cp_async_wait_all();
     __syncwarp();
     const uint32_t act = row_actions(w.msk, lane);
-    w.act[k][lane] = act;
+    w.act[slot + k][lane] = act;
     __syncwarp();  // every lane has read the flags and finished the previous piece
     if (k > 0) stage_in(a, c0, seg, k - 1, lane, w.val[cur ^ 1], w.msk, pol);
     const int64_t t0 = s0 + 32 * int64_t(k);
@@ -835,7 +836,7 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane
     const uint32_t ends = piece_ends(a, cu, blo, bhi, t0, b_last);
     // every lane folds (the token loops vote across the warp); a lane past N
     // has no flags and keeps its state
-    fold_piece<kCrit>(a, w.val[cur], tmem + 32 * k, lane, act, ends, t0, cu, blo, b_last, f);
+    fold_piece<kCrit>(a, w.val[cur], tmem + 32 * (slot + k), lane, act, ends, t0, cu, blo, b_last, f);
   }
   tmem_wait_st();  // the values are in TMEM before the replay reads them
 
@@ -858,6 +859,7 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane
       publish_map<kCrit>(a.agg + size_t(q) * kMapWords<kCrit>, S);
   }
   p.q = q;
+  p.slot = slot;
   p.blo = blo;
   p.bhi = bhi;
   p.b_seg = b_seg;
@@ -869,7 +871,8 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane
 // state, then replays the tokens piece by piece (right to left) from TMEM and
 // stores advantages and returns.
 template <bool kCrit>
-__device__ void replay_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane, const Pending<kCrit> &p) {
+__device__ void replay_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane, const Pending<kCrit> &p,
+                             bool pipelined) {
   const int seg = 32 * a.pieces;
   const int64_t c0 = int64_t(p.q) * kChunk * a.pieces;
   const int64_t s0 = c0 + int64_t(lane) * seg;
@@ -885,17 +888,17 @@ __device__ void replay_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int la
   if (lane == 0 && !reset && !last)
     publish_state<kCrit>(a.incl + size_t(p.q) * kStateWords<kCrit>, apply<kCrit>(p.S, right));
   // every lane replays (the token loops vote across the warp); rows past N
-  // are never stored. The fold's copy of the chunk's cu_seqlens slice is
-  // still in shared memory.
-  const CuView cu{a.cu, w.cu, p.blo, p.bhi - p.blo + 2 <= kScanCuCap};
+  // are never stored. Unless the next chunk has been folded since, the
+  // fold's copy of the chunk's cu_seqlens slice is still in shared memory.
+  const CuView cu{a.cu, w.cu, p.blo, !pipelined && p.bhi - p.blo + 2 <= kScanCuCap};
   rs.st = apply<kCrit>(p.E, right);
 #pragma unroll 1
   for (int k = a.pieces - 1; k >= 0; --k) {
-    const uint32_t act = w.act[k][lane];
+    const uint32_t act = w.act[p.slot + k][lane];
     const int64_t t0 = s0 + 32 * int64_t(k);
     int b_last;
     const uint32_t ends = piece_ends(a, cu, p.blo, p.bhi, t0, b_last);
-    replay_piece<kCrit>(a, tmem + 32 * k, w.val[0], w.ret, lane, act, ends, t0, cu, p.blo, b_last, rs);
+    replay_piece<kCrit>(a, tmem + 32 * (p.slot + k), w.val[0], w.ret, lane, act, ends, t0, cu, p.blo, b_last, rs);
     __syncwarp();
     stage_out(a, c0, seg, k, lane, w.val[0], w.ret);
     __syncwarp();  // every lane has read its granules before the next piece overwrites them
@@ -903,12 +906,11 @@ __device__ void replay_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int la
 }
 
 // Persistent warps: a warp takes a chunk (ticket), folds and publishes it,
-// looks back and replays it, and takes the next. Tickets keep the decoupled
-// look-back safe: a warp waits only on chunks taken before its own, and every
-// taken chunk is folded and published at once, before its warp waits on
-// anything. Each CTA holds kTmemCols TMEM columns for the whole launch (four
+// looks back and replays it. Tickets keep the decoupled look-back safe: a
+// warp waits only on chunks taken before its own, and every taken chunk is
+// folded and published at once, before its warp waits on anything. Each CTA holds kTmemCols TMEM columns for the whole launch (four
 // CTAs per SM take all 512, so the allocation never waits on this kernel).
-template <bool kCrit>
+template <bool kCrit, bool kPipe>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) gae_scan_kernel(GaeArgs a) {
   extern __shared__ __align__(16) unsigned char s_raw[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -922,11 +924,38 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) gae_scan_kernel(GaeArgs 
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = wb[0].tmem + (uint32_t(32 * warp) << 16);  // the warp's TMEM lanes
+  if constexpr (kPipe) {
+    // short segments: two chunks in flight, one per half of the warp's TMEM
+    // columns; the warp folds a chunk before it looks back for the one it
+    // folded before, so the chunks it waits on have had a whole fold to
+    // publish (with one chunk at a time that wait is exposed, and at these
+    // chunk sizes it dominates)
+    int q = take_chunk(a, lane);
+    if (q >= 0) {
+      Pending<kCrit> p;
+      int half = 0;
+      fold_chunk<kCrit>(a, w, tmem, lane, q, 0, p);
 #pragma unroll 1
-  for (int q = take_chunk(a, lane); q >= 0; q = take_chunk(a, lane)) {
-    Pending<kCrit> p;
-    fold_chunk<kCrit>(a, w, tmem, lane, q, p);
-    replay_chunk<kCrit>(a, w, tmem, lane, p);
+      for (;;) {
+        const int qn = take_chunk(a, lane);
+        Pending<kCrit> n;
+        if (qn >= 0) fold_chunk<kCrit>(a, w, tmem, lane, qn, (half ^ 1) * (kMaxPieces / 2), n);
+        replay_chunk<kCrit>(a, w, tmem, lane, p, true);
+        if (qn < 0) break;
+        p = n;
+        half ^= 1;
+      }
+    }
+  } else {
+    // long segments: one chunk at a time in all of the warp's columns (the
+    // per-chunk scan, look-back and set-up spread over 4096 tokens cost less
+    // than the exposed wait)
+#pragma unroll 1
+    for (int q = take_chunk(a, lane); q >= 0; q = take_chunk(a, lane)) {
+      Pending<kCrit> p;
+      fold_chunk<kCrit>(a, w, tmem, lane, q, 0, p);
+      replay_chunk<kCrit>(a, w, tmem, lane, p, false);
+    }
   }
   tc::fence_before_sync();
   __syncthreads();
@@ -969,8 +998,8 @@ constexpr size_t kScanSmem = sizeof(WarpBuf) * kWarps;
 // and device.
 sao_status set_scan_smem(void (*kern)(GaeArgs), int which, int device) {
   constexpr int kMaxDevices = 64;
-  static std::once_flag once[2][kMaxDevices];
-  static cudaError_t err[2][kMaxDevices];
+  static std::once_flag once[4][kMaxDevices];
+  static cudaError_t err[4][kMaxDevices];
   if (device < 0 || device >= kMaxDevices) return fail(SAO_ERR_CUDA, "device %d out of range", device);
   std::call_once(once[which][device], [&] {
     err[which][device] = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kScanSmem));
@@ -1074,8 +1103,11 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   a.wait_ns = scan_wait_ns();
   DeviceInfo di;
   SAO_TRY(device_info(&di));
-  auto kern = crit_trivial ? gae_scan_kernel<false> : gae_scan_kernel<true>;
-  SAO_TRY(set_scan_smem(kern, crit_trivial ? 0 : 1, di.device));
+  // segments of 1 or 2 pieces: two chunks in flight per warp
+  const bool pipe = pieces <= kMaxPieces / 2;
+  auto kern = crit_trivial ? (pipe ? gae_scan_kernel<false, true> : gae_scan_kernel<false, false>)
+                           : (pipe ? gae_scan_kernel<true, true> : gae_scan_kernel<true, false>);
+  SAO_TRY(set_scan_smem(kern, (crit_trivial ? 0 : 2) + (pipe ? 1 : 0), di.device));
   // persistent: as many warps as fit on the GPU, never more than chunks
   const int64_t ctas = (nscan + kWarps - 1) / kWarps;
   const int64_t resident = int64_t(di.sm_count) * kMinBlocks;
