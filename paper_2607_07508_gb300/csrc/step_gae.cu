@@ -32,6 +32,7 @@ constexpr int kTokensPerThread = kCountRows / kThreads;  // 64: four 16-byte loa
 constexpr int kSubBlocks = kCountRows / kRowsPerBlock;
 constexpr int kWarpsPerBlock = kRowsPerBlock / kTokensPerThread / 32;  // 2
 constexpr int kShortStep = 32;  // a step this long or shorter is summed by one lane
+constexpr int64_t kWarpPerStepBelow = int64_t(1) << 25;  // fewer tokens than this: one warp per step
 
 // Trajectory starts as a bit mask over the tokens (bit t & 31 of word t >> 5).
 __global__ void mark_traj_starts(const int32_t *cu, int B, int64_t N, uint32_t *tsb) {
@@ -278,17 +279,44 @@ __device__ __forceinline__ float2 acc_mean(const Acc2 &a, int n) {
 }
 
 // A warp takes 32 consecutive steps, one per lane: a lane sums its own step
-// when it is short (4 independent loads at a time), the warp sums the long
-// ones together. Step ranges come from the scatter pass, so no load waits on
-// another. (Copying the warp's span of values into shared memory first, for
-// contiguous loads, measured 3x slower: the copy exposes a load latency per 32
-// values, while the steps' own loads already fall in a few nearby lines.)
+// when it is short (8 independent loads at a time), the warp sums the long
+// ones together; below kWarpPerStepBelow tokens, a warp takes one step. Step
+// ranges come from the scatter pass, so no load waits on another. (Copying
+// the warp's span of values into shared memory first, for contiguous loads,
+// measured 3x slower: the copy exposes a load latency per 32 values, while
+// the steps' own loads already fall in a few nearby lines.)
+template <bool kWarpPerStep>
 __global__ void __launch_bounds__(kThreads) step_reduce_kernel(const float *values, const int *step_first,
                                                                const int *step_end, const int *nsteps, int mode,
                                                                float2 *sv) {
   const int lane = threadIdx.x & 31;
   const int S = *nsteps;
   const int nwarps = (gridDim.x * kThreads) >> 5;
+  if (kWarpPerStep && mode != SAO_STEP_LAST) {
+    // few steps: one warp per step, so every SM has work (the mode depends
+    // on N alone, so every device gives the same bits)
+    for (int s = (blockIdx.x * kThreads + threadIdx.x) >> 5; s < S; s += nwarps) {
+      const int f = step_first[s], e = step_end[s];
+      Acc2 part;
+      for (int t = f + lane; t < e; t += 256) {
+        float x[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) x[k] = t + 32 * k < e ? values[t + 32 * k] : 0.f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          if (t + 32 * k < e) part.add(x[k]);
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        Acc2 other;
+        other.hi = __shfl_xor_sync(0xffffffffu, part.hi, o);
+        other.lo = __shfl_xor_sync(0xffffffffu, part.lo, o);
+        part.add(other);
+      }
+      if (lane == 0) sv[s] = acc_mean(part, e - f);
+    }
+    return;
+  }
   // the next group's step ranges are loaded while this group is summed
   int g = (blockIdx.x * kThreads + threadIdx.x) >> 5;
   int nfirst = g * 32 + lane < S ? step_first[g * 32 + lane] : 0;
@@ -489,9 +517,9 @@ __global__ void __launch_bounds__(32 * kGaeWarps) step_gae_kernel(const float *r
 // Every token gets its step's results (non-action tokens get zeros), step by
 // step: a warp takes 32 consecutive steps (one per lane: first token, end,
 // results) and writes the tokens from its first step's first token to the
-// next group's (the steps and the observation tokens after each), in
-// 128-token windows with 4 tokens per lane, so every store of the warp is
-// contiguous. A lane finds the step of its tokens by a binary search over the
+// next group's (the steps and the observation tokens after each), or a share
+// of those windows when there are fewer groups than warps, in 128-token
+// windows with 4 tokens per lane, so every store of the warp is contiguous. A lane finds the step of its tokens by a binary search over the
 // 32 first tokens held in the warp's lanes; the first group also writes the
 // tokens before the first step. Neither the mask nor the flags are read again.
 __device__ __forceinline__ int steps_at_or_before(int F, int t) {  // #{j : F_j <= t}, F_j rising over the lanes
@@ -512,10 +540,14 @@ __global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const int *nst
   const int S = *nsteps;
   const int ngroups = S > 0 ? (S + 31) / 32 : 1;
   const int nwarps = (gridDim.x * kThreads) >> 5;
+  // with fewer groups than warps, each group's windows are shared out over
+  // up to 64 warps
+  const int parts = max(1, min(64, nwarps / ngroups));
   const bool vout = ((reinterpret_cast<uintptr_t>(adv) | reinterpret_cast<uintptr_t>(ret)) & 15u) == 0 &&
                     (reinterpret_cast<uintptr_t>(vmask) & 3u) == 0;
   const bool last_mode = mode != SAO_STEP_AVERAGE;
-  for (int g = (blockIdx.x * kThreads + threadIdx.x) >> 5; g < ngroups; g += nwarps) {
+  for (int u = (blockIdx.x * kThreads + threadIdx.x) >> 5; u < ngroups * parts; u += nwarps) {
+    const int g = u / parts, part = u % parts;
     const int s = g * 32 + lane;
     const bool has = s < S;
     const int F = has ? step_first[s] : INT_MAX;
@@ -523,8 +555,11 @@ __global__ void __launch_bounds__(kThreads) step_broadcast_kernel(const int *nst
     const float2 o = has ? out[s] : make_float2(0.f, 0.f);
     const int lo = g == 0 ? 0 : __shfl_sync(0xffffffffu, F, 0);
     const int hi = (g + 1) * 32 < S ? step_first[(g + 1) * 32] : int(N);  // the group writes [lo, hi)
-    for (int c = lo & ~3; c < hi; c += 128) {
-      const int t4 = c + 4 * lane;
+    const int c0 = lo & ~3;
+    const int nwin = (hi - c0 + 127) / 128, per = (nwin + parts - 1) / parts;
+    const int w1 = min(nwin, (part + 1) * per);
+    for (int win = part * per; win < w1; ++win) {
+      const int t4 = c0 + 128 * win + 4 * lane;
       float a[4], r[4];
       uint8_t k[4];
       const int j0 = steps_at_or_before(F, t4) - 1;  // step of token t4 in the group (-1: before it)
@@ -615,7 +650,8 @@ sao_status step_gae_launch(const float *values, const float *rewards, const uint
   SAO_TRY(launch_end(slot, s));
   const unsigned warps_grid = unsigned(di.sm_count * 8);
   slot = launch_begin("step_gae_reduce", s);
-  step_reduce_kernel<<<warps_grid, kThreads, 0, s>>>(values, step_first, step_end, nsteps, mode, sv);
+  auto reduce = N < kWarpPerStepBelow ? step_reduce_kernel<true> : step_reduce_kernel<false>;
+  reduce<<<warps_grid, kThreads, 0, s>>>(values, step_first, step_end, nsteps, mode, sv);
   SAO_TRY(launch_end(slot, s));
   slot = launch_begin("step_gae_scan", s);
   auto scan = (gamma == 1.f && lam_c == 1.f) ? step_gae_kernel<false> : step_gae_kernel<true>;
