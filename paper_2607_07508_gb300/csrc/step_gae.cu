@@ -2,21 +2,22 @@
 // conversation turn = a maximal run of action tokens inside a trajectory) and
 // broadcast to the step's tokens.
 //
-//   1. flag trajectory starts, then step starts (an action token that opens a
-//      trajectory or follows a non-action token); a block-level scan gives the
-//      ordered step list with each step's token range (count on the device)
-//      and every action token's step;
+//   1. flag trajectory starts (a bit mask), then step starts (an action token
+//      that opens a trajectory or follows a non-action token); a count pass,
+//      a scan and a scatter pass give the ordered step list with each step's
+//      token range (count on the device) and per-block step offsets;
 //   2. a warp takes 32 consecutive steps, one per lane: a lane sums its own
 //      step when it is short (most turns), the warp sums the long ones
-//      together; sums are compensated fp32 pairs (~48 bits), so GB300's slow
-//      fp64 pipe is not on this path;
+//      together (below 2^25 tokens, one warp per step); sums are compensated
+//      fp32 pairs (~48 bits), so GB300's slow fp64 pipe is not on this path;
 //   3. one warp per trajectory runs the backward GAE over its steps: each
 //      lane folds a contiguous block of steps into an affine map, a shuffle
 //      scan combines the maps, each lane replays its block (double-float; the
 //      length-adaptive lambda is counted in steps);
-//   4. every token reads its step's advantage, value target and value-loss
-//      flag (coalesced, one pass; non-action tokens get zeros), its step
-//      index recounted from the flags, so no per-token index is stored.
+//   4. step by step, every token gets its step's advantage, value target and
+//      value-loss flag (non-action tokens get zeros): a warp writes the token
+//      spans of 32 consecutive steps, so no per-token index is stored and the
+//      mask is not read again.
 #include <stdint.h>
 
 #include "sao_common.cuh"
