@@ -296,8 +296,12 @@ def advantages(values, rewards, loss_mask, cu_seqlens, gamma: float, lam: float,
 # value loss (Preliminaries, PPO) and explained variance (§4.4)
 # ---------------------------------------------------------------------------
 
-def value_loss(values, ret, loss_mask) -> Tuple[float, np.ndarray, np.ndarray]:
-    """L_v = (1/n) sum_t m_t (V_t - ret_t)^2 over the n action tokens.
+def value_loss(values, ret, loss_mask, n_norm: int = 0) -> Tuple[float, np.ndarray, np.ndarray]:
+    """L_v = (1/n) sum_t m_t (V_t - ret_t)^2 over the action tokens
+    (Preliminaries, the PPO value error), with n = n_norm if n_norm > 0, else
+    the number of action tokens: the batch mean of the unsplit batch when
+    data-parallel ranks share the batch's action-token count, as the policy
+    loss's normaliser does.
 
     Returns (loss, dL/dV, ev_sums) with ev_sums = [sum m(R-V), sum m(R-V)^2,
     sum m R, sum m R^2] (R = ret) for the explained variance.
@@ -305,7 +309,7 @@ def value_loss(values, ret, loss_mask) -> Tuple[float, np.ndarray, np.ndarray]:
     V = _f64(values)
     R = _f64(ret)
     m = np.asarray(loss_mask).astype(bool)
-    n = int(m.sum())
+    n = int(n_norm) if n_norm > 0 else int(m.sum())
     d = np.where(m, V - R, 0.0)
     loss = float((d * d).sum() / n) if n > 0 else 0.0
     grad = 2.0 * d / n if n > 0 else np.zeros_like(d)
