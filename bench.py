@@ -489,6 +489,8 @@ def bandwidth_study(args):
         "sao_policy_loss_fwd (n_norm given)": (18, lambda: sao.sao_policy_loss_fwd(
             lp, old, adv, m, wl.eps_low, wl.eps_high, loss, counts, ws, coef=coef, flags=flags, n_norm=n_act)),
         "sao_value_loss": (13, lambda: sao.sao_value_loss(v, ret, m, loss, dV, ws, ev_sums=ev)),
+        "sao_value_loss (n_norm given)": (13, lambda: sao.sao_value_loss(v, ret, m, loss, dV, ws, ev_sums=ev,
+                                                                         n_norm=n_act)),
         "sao_clip_loss_fwd": (18, lambda: sao.sao_clip_loss_fwd(lp, old, adv, m, cu, 0.2, 0.28,
                                                                 sao.SAO_NORM_SEQUENCE, loss, counts, ws, coef=coef,
                                                                 flags=flags)),

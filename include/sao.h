@@ -398,16 +398,21 @@ SAO_API sao_status sao_policy_loss_bwd(const float *logp, const float *old_logp,
                                size_t ws_bytes, sao_stream_t stream);
 
 /*
- * Value loss (Preliminaries, PPO): over the n action tokens,
+ * Value loss (Preliminaries, PPO): over the action tokens, with n = n_norm if
+ * n_norm > 0, else the number of action tokens,
  *   loss = (1/n) sum_t (V_t - ret_t)^2           [1] fp32 output
  *   grad_values[t] = 2 (V_t - ret_t) / n, 0 on non-action tokens   [N] fp32
  *   ev_sums = {sum (R-V), sum (R-V)^2, sum R, sum R^2} over action tokens
  *             ([4] fp64, may be NULL), from which explained variance
  *             EV = 1 - Var(R - V) / Var(R) (§4.4) follows.
+ * n_norm is the normaliser shared by data-parallel ranks (the action tokens
+ * of the whole batch), as for the policy loss: the ranks' losses and
+ * gradients then add up to those of the unsplit batch. With n_norm > 0 the
+ * call makes one pass over the tokens; otherwise it counts them first.
  */
 SAO_API sao_status sao_value_loss(const float *values, const float *ret, const uint8_t *loss_mask,
-                          int64_t N, float *loss, float *grad_values, double *ev_sums, void *ws,
-                          size_t ws_bytes, sao_stream_t stream);
+                          int64_t N, int64_t n_norm, float *loss, float *grad_values, double *ev_sums,
+                          void *ws, size_t ws_bytes, sao_stream_t stream);
 
 /*
  * Kernel timing for profiling. When enabled, every kernel the library

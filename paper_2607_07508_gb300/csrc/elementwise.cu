@@ -417,6 +417,7 @@ struct VLArgs {
   const float *v, *ret;
   const uint8_t *m;
   int64_t N;
+  int64_t n_norm;
   const long long *cnt_partial;
   int n_cnt;
   float *grad;
@@ -424,7 +425,7 @@ struct VLArgs {
 };
 
 __global__ void __launch_bounds__(kThreads) value_loss_kernel(VLArgs a) {
-  const long long n = total_of(a.cnt_partial, a.n_cnt);
+  const long long n = a.n_norm > 0 ? a.n_norm : total_of(a.cnt_partial, a.n_cnt);
   const float two_over_n = n > 0 ? float(2.0 / double(n)) : 0.f;
   Acc2 a_d2, a_e, a_e2, a_r, a_r2;
   const int64_t tid = int64_t(blockIdx.x) * kThreads + threadIdx.x;
@@ -495,8 +496,8 @@ __global__ void __launch_bounds__(kThreads) value_loss_kernel(VLArgs a) {
 
 __global__ void __launch_bounds__(kThreads) value_loss_finalize(const double *sums, int grid,
                                                                 const long long *cnt_partial, int n_cnt,
-                                                                float *loss, double *ev) {
-  const long long n = total_of(cnt_partial, n_cnt);
+                                                                int64_t n_norm, float *loss, double *ev) {
+  const long long n = n_norm > 0 ? n_norm : total_of(cnt_partial, n_cnt);
   double s[5] = {0, 0, 0, 0, 0};
   for (int i = threadIdx.x; i < grid; i += kThreads)
 #pragma unroll
@@ -641,20 +642,22 @@ sao_status decoupled_loss_launch(const float *logp, const float *prox, const flo
   return launch_end(slot, s);
 }
 
-sao_status value_loss_launch(const float *v, const float *ret, const uint8_t *m, int64_t N, float *loss,
-                             float *grad, double *ev, void *ws_body, size_t body_bytes, cudaStream_t s) {
+sao_status value_loss_launch(const float *v, const float *ret, const uint8_t *m, int64_t N, int64_t n_norm,
+                             float *loss, float *grad, double *ev, void *ws_body, size_t body_bytes,
+                             cudaStream_t s) {
   const int grid = stream_grid(N, value_loss_kernel);
   Carver c(ws_body, body_bytes);
   long long *cnt = c.take<long long>(grid);
   double *sums = c.take<double>(5 * size_t(grid));
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the value loss");
-  SAO_TRY(launch_count(m, N, cnt, grid, s));
-  VLArgs a{v, ret, m, N, cnt, grid, grad, sums};
+  const bool need_count = n_norm <= 0;  // the normaliser must be known before the token pass
+  if (need_count) SAO_TRY(launch_count(m, N, cnt, grid, s));
+  VLArgs a{v, ret, m, N, n_norm, cnt, need_count ? grid : 0, grad, sums};
   int slot = launch_begin("value_loss", s);
   value_loss_kernel<<<grid, kThreads, 0, s>>>(a);
   SAO_TRY(launch_end(slot, s));
   slot = launch_begin("value_loss_finalize", s);
-  value_loss_finalize<<<1, kThreads, 0, s>>>(sums, grid, cnt, grid, loss, ev);
+  value_loss_finalize<<<1, kThreads, 0, s>>>(sums, grid, cnt, need_count ? grid : 0, n_norm, loss, ev);
   return launch_end(slot, s);
 }
 

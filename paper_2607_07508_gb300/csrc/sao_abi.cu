@@ -371,8 +371,9 @@ sao_status sao_decoupled_loss_bwd(const float *logp, const float *prox_logp, con
   return finish_call(ws, s);
 }
 
-sao_status sao_value_loss(const float *values, const float *ret, const uint8_t *loss_mask, int64_t N, float *loss,
-                          float *grad_values, double *ev_sums, void *ws, size_t ws_bytes, sao_stream_t stream) {
+sao_status sao_value_loss(const float *values, const float *ret, const uint8_t *loss_mask, int64_t N, int64_t n_norm,
+                          float *loss, float *grad_values, double *ev_sums, void *ws, size_t ws_bytes,
+                          sao_stream_t stream) {
   SAO_RANGE();
   if (N < 0) return fail(SAO_ERR_SHAPE, "N < 0");
   if (!loss) return fail(SAO_ERR_INVALID_ARG, "NULL loss");
@@ -381,7 +382,7 @@ sao_status sao_value_loss(const float *values, const float *ret, const uint8_t *
   SAO_TRY(take_ws(ws, ws_bytes, elementwise_ws_bytes(N, 0), &w));
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   SAO_TRY(begin_call(ws, s));
-  SAO_TRY(value_loss_launch(values, ret, loss_mask, N, loss, grad_values, ev_sums, w.body, w.body_bytes, s));
+  SAO_TRY(value_loss_launch(values, ret, loss_mask, N, n_norm, loss, grad_values, ev_sums, w.body, w.body_bytes, s));
   return finish_call(ws, s);
 }
 

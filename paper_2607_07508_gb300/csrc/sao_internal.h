@@ -18,7 +18,7 @@ sao_status policy_loss_launch(const float *logp, const float *old, const float *
                               int64_t N, float eps_low, float eps_high, int64_t n_norm, float *loss,
                               float *coef, uint8_t *flags, int64_t *counts, const float *grad_loss,
                               void *ws_body, size_t body_bytes, cudaStream_t s);
-sao_status value_loss_launch(const float *v, const float *ret, const uint8_t *m, int64_t N, float *loss,
+sao_status value_loss_launch(const float *v, const float *ret, const uint8_t *m, int64_t N, int64_t n_norm, float *loss,
                              float *grad, double *ev, void *ws_body, size_t body_bytes, cudaStream_t s);
 sao_status decoupled_loss_launch(const float *logp, const float *prox, const float *roll, const float *adv,
                                  const uint8_t *m, int64_t N, float eps_low, float eps_high, float w_low,

@@ -4,8 +4,9 @@ The loss head is row-independent except inside one trajectory (the advantage
 scan), so a batch shards by whole trajectories with no exchange on the data
 path. The only cross-rank quantity is the denominator of the token mean (the
 number of action tokens of the whole batch): each rank passes the all-reduced
-count as ``n_norm`` to the policy-loss calls, after which the per-rank losses
-and weight gradients simply add up (the trainer's usual gradient all-reduce).
+count as ``n_norm`` to the policy-loss and value-loss calls, after which the
+per-rank losses and weight gradients simply add up (the trainer's usual
+gradient all-reduce).
 """
 from __future__ import annotations
 

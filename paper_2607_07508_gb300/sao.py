@@ -82,7 +82,7 @@ def load(path: Optional[str] = None):
         "sao_policy_loss_bwd": (ctypes.c_int, [P, P, P, P, I64, F, F, I64, P, P, P, SZ, P]),
         "sao_decoupled_loss_fwd": (ctypes.c_int, [P, P, P, P, P, I64, F, F, F, F, I64, P, P, P, P, P, SZ, P]),
         "sao_decoupled_loss_bwd": (ctypes.c_int, [P, P, P, P, P, I64, F, F, F, F, I64, P, P, P, SZ, P]),
-        "sao_value_loss": (ctypes.c_int, [P, P, P, I64, P, P, P, P, SZ, P]),
+        "sao_value_loss": (ctypes.c_int, [P, P, P, I64, I64, P, P, P, P, SZ, P]),
         "sao_clip_loss_fwd": (ctypes.c_int, [P, P, P, P, P, I32, I64, F, F, ctypes.c_int, P, P, P, P, P, SZ, P]),
         "sao_clip_loss_bwd": (ctypes.c_int, [P, P, P, P, P, I32, I64, F, F, ctypes.c_int, P, P, P, SZ, P]),
         "sao_group_advantages": (ctypes.c_int, [P, P, I32, P, P, I64, F, P, P, SZ, P]),
@@ -363,7 +363,7 @@ def sao_decoupled_loss_bwd(logp, prox_logp, rollout_logp, adv, loss_mask, eps_lo
                                          ws.numel(), _stream(stream)))
 
 
-def sao_value_loss(values, ret, loss_mask, loss, grad_values, ws, ev_sums=None, stream=None):
+def sao_value_loss(values, ret, loss_mask, loss, grad_values, ws, ev_sums=None, n_norm=0, stream=None):
     N = values.numel()
     _expect(values, torch.float32, N, "values")
     _expect(ret, torch.float32, N, "ret")
@@ -371,8 +371,8 @@ def sao_value_loss(values, ret, loss_mask, loss, grad_values, ws, ev_sums=None, 
     _expect(grad_values, torch.float32, N, "grad_values")
     _expect(loss, torch.float32, 1, "loss")
     _expect(ev_sums, torch.float64, 4, "ev_sums")
-    _check(load().sao_value_loss(_ptr(values), _ptr(ret), _ptr(loss_mask), N, _ptr(loss), _ptr(grad_values),
-                                 _ptr(ev_sums), _ptr(ws), ws.numel(), _stream(stream)))
+    _check(load().sao_value_loss(_ptr(values), _ptr(ret), _ptr(loss_mask), N, int(n_norm), _ptr(loss),
+                                 _ptr(grad_values), _ptr(ev_sums), _ptr(ws), ws.numel(), _stream(stream)))
 
 
 def sao_clip_loss_fwd(logp, old_logp, adv, loss_mask, cu_seqlens, eps_low, eps_high, norm, loss, counts, ws,

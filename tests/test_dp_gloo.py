@@ -1,6 +1,7 @@
 """Data-parallel contract of the loss head, checked with two gloo ranks on CPU:
 sharding by trajectory plus one all-reduced action-token count (n_norm) makes
-the sum of the per-rank losses and weight gradients equal the unsplit batch.
+the sum of the per-rank policy and value losses and of the weight gradients
+equal the unsplit batch, and the value gradients its slices.
 The arithmetic on each rank is the fp64 oracle (no GPU here)."""
 import os
 import socket
@@ -37,16 +38,25 @@ def _rank_main(rank, world, port, out):
         n_norm = dp.global_action_count(int(loc["mask_tok"].sum()))
         pl = O.policy_loss(logp, old, adv, loc["mask_tok"], 0.2, 0.28, n_norm=n_norm)
         _, dW = O.token_logprobs_bwd(loc["H_tok"], wl.W, loc["y_tok"], lse, pl["coef"])
+        ret_loc = loc["values_tok"] + 0.5 * loc["xi_tok"]
+        vl, vg, _ = O.value_loss(loc["values_tok"], ret_loc, loc["mask_tok"], n_norm=n_norm)
         t_loss = torch.tensor([pl["loss"]], dtype=torch.float64)
+        t_vloss = torch.tensor([vl], dtype=torch.float64)
         t_dW = torch.tensor(dW)
         dist.all_reduce(t_loss)
+        dist.all_reduce(t_vloss)
         dist.all_reduce(t_dW)
+        # each rank's value gradient is its slice of the unsplit batch's
+        t0, t1 = int(wl.cu_seqlens[shard[0]]), int(wl.cu_seqlens[shard[1]])
+        _, vg_f, _ = O.value_loss(wl.values, wl.values + 0.5 * wl.xi, wl.loss_mask)
+        out[f"vgrad{rank}"] = float(np.abs(vg - vg_f[t0:t1]).max())
         if rank == 0:
             adv_f, _ = O.advantages(wl.values, wl.rewards, wl.loss_mask, wl.cu_seqlens, 1.0, 0.95, 1.0)
             lp_f, lse_f = O.token_logprobs(wl.H, wl.W, wl.y)
             pl_f = O.policy_loss(lp_f, lp_f + wl.xi, adv_f, wl.loss_mask, 0.2, 0.28)
             _, dW_f = O.token_logprobs_bwd(wl.H, wl.W, wl.y, lse_f, pl_f["coef"])
             out["loss"] = (float(t_loss.item()), pl_f["loss"])
+            out["vloss"] = (float(t_vloss.item()), O.value_loss(wl.values, wl.values + 0.5 * wl.xi, wl.loss_mask)[0])
             out["dW"] = float(np.abs(t_dW.numpy() - dW_f).max()), float(np.abs(dW_f).max())
             out["n_norm"] = (n_norm, int(wl.loss_mask.sum()))
     finally:
@@ -78,3 +88,6 @@ def test_two_gloo_ranks_match_unsplit_batch():
     err, scale = out["dW"]
     assert err <= 1e-12 * max(1.0, scale)
     assert out["n_norm"][0] == out["n_norm"][1]
+    got, want = out["vloss"]
+    assert abs(got - want) <= 1e-12 * max(1.0, abs(want))
+    assert out["vgrad0"] <= 1e-15 and out["vgrad1"] <= 1e-15

@@ -256,12 +256,12 @@ def test_policy_loss_bandwidth_size():
 # value loss
 # ---------------------------------------------------------------------------
 
-def _vl_gpu(v, r, m):
+def _vl_gpu(v, r, m, n_norm=0):
     N = len(v)
     loss = torch.empty(1, device="cuda")
     grad = torch.empty(N, device="cuda")
     ev = torch.empty(4, dtype=torch.float64, device="cuda")
-    sao.sao_value_loss(cuda(v), cuda(r), cuda(m), loss, grad, sao.workspace(N), ev_sums=ev)
+    sao.sao_value_loss(cuda(v), cuda(r), cuda(m), loss, grad, sao.workspace(N), ev_sums=ev, n_norm=n_norm)
     torch.cuda.synchronize()
     return float(loss.item()), grad.cpu().numpy(), ev.cpu().numpy()
 
@@ -271,12 +271,13 @@ def test_value_loss_match_oracle(name):
     wl = S.bandwidth_workload() if name == "bandwidth" else S.make_workload(name, dense=False)
     rng = np.random.default_rng(2)
     ret = (wl.values + rng.normal(0, 0.3, wl.N)).astype(np.float32)
-    loss, grad, ev = _vl_gpu(wl.values, ret, wl.loss_mask)
-    wl_, wg, wev = O.value_loss(wl.values, ret, wl.loss_mask)
-    assert abs(loss - wl_) <= LOSS_TOL * abs(wl_)
-    assert rel_err_floor(grad, wg, 1e-12).max() <= 1e-5
-    # fp32 per-token products, compensated fp32 accumulation: ~1e-7 relative
-    assert np.allclose(ev, wev, rtol=1e-6, atol=1e-6 * np.abs(wev).max())
+    for n_norm in (0, 3 * int(wl.loss_mask.sum()) + 1):  # counted, or given (one pass)
+        loss, grad, ev = _vl_gpu(wl.values, ret, wl.loss_mask, n_norm)
+        wl_, wg, wev = O.value_loss(wl.values, ret, wl.loss_mask, n_norm)
+        assert abs(loss - wl_) <= LOSS_TOL * abs(wl_)
+        assert rel_err_floor(grad, wg, 1e-12).max() <= 1e-5
+        # fp32 per-token products, compensated fp32 accumulation: ~1e-7 relative
+        assert np.allclose(ev, wev, rtol=1e-6, atol=1e-6 * np.abs(wev).max())
 
 
 def test_value_loss_zero_and_empty():

@@ -479,6 +479,23 @@ def test_value_loss_finite_differences_and_mean():
         assert abs(num - g[t]) < 1e-8
 
 
+def test_value_loss_external_normaliser_scales_loss_and_grad():
+    # a batch split in two with the whole batch's count as the normaliser:
+    # the halves' losses and gradients are the whole batch's, split
+    r = _rng(53)
+    v = r.normal(size=30)
+    R = r.normal(size=30)
+    m = (r.random(30) < 0.7).astype(np.uint8)
+    n = int(m.sum())
+    loss, g, _ = O.value_loss(v, R, m)
+    l1, g1, _ = O.value_loss(v[:11], R[:11], m[:11], n_norm=n)
+    l2, g2, _ = O.value_loss(v[11:], R[11:], m[11:], n_norm=n)
+    assert abs(l1 + l2 - loss) < 1e-14
+    assert np.array_equal(np.concatenate([g1, g2]), g)
+    l3, g3, _ = O.value_loss(v, R, m, n_norm=4 * n)
+    assert abs(4 * l3 - loss) < 1e-14 and np.allclose(4 * g3, g, rtol=1e-15, atol=0)
+
+
 def test_explained_variance_matches_numpy_var():
     r = _rng(52)
     v = r.normal(size=100)
