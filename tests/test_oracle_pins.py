@@ -830,3 +830,39 @@ def test_decoupled_loss_nonfinite_tokens_are_masked():
     out = O.decoupled_loss(logp, prox, roll, adv, m, 0.2, 0.28, 0.5, 2.0)
     assert all(out["flags"][t] == O.FLAG_NONFINITE for t in (3, 5, 7))
     assert out["counts"][3] == 3 and out["counts"][0] == 30 and np.isfinite(out["loss"])
+
+
+# ---------------------------------------------------------------------------
+# helpers the entry points build on, pinned directly
+# ---------------------------------------------------------------------------
+
+def test_trajectory_lambda_hand_values():
+    # lambda = 1 - 1/(alpha * l), clamped to [0, 1]; alpha <= 0 keeps the fixed lambda (§4.1)
+    assert O.trajectory_lambda(0.95, 0.0, 10) == 0.95
+    assert abs(O.trajectory_lambda(0.95, 1.5, 3) - (1.0 - 1.0 / 4.5)) < 1e-15
+    assert O.trajectory_lambda(0.95, 1.5, 0) == 0.0
+    assert O.trajectory_lambda(0.95, 0.5, 1) == 0.0          # 1 - 1/0.5 < 0
+    assert abs(O.trajectory_lambda(0.95, 1.5, 128_000) - (1.0 - 1.0 / 192_000)) < 1e-15
+
+
+def test_step_spans_hand_cases():
+    m = np.array([1, 1, 0, 1, 0, 0, 1, 1, 1], np.uint8)
+    assert O.step_spans(m, 0, 9) == [(0, 2), (3, 4), (6, 9)]
+    assert O.step_spans(m, 1, 7) == [(1, 2), (3, 4), (6, 7)]   # clipped at the trajectory's bounds
+    assert O.step_spans(np.zeros(5, np.uint8), 0, 5) == []
+    assert O.step_spans(np.ones(4, np.uint8), 0, 4) == [(0, 4)]
+
+
+def test_decoupled_flags_hand_cases():
+    # r = pi_theta / pi_old, w = pi_old / pi_rollout; band (w_low, w_high) = (0.5, 2.0), eps 0.2 / 0.28
+    ln = np.log
+    logp = np.array([0.0, ln(1.5), ln(0.5), 0.0, 0.0, 0.0, np.nan, 0.0], np.float32)
+    prox = np.zeros(8, np.float32)
+    roll = np.array([0.0, 0.0, 0.0, ln(4.0), -ln(3.0), 0.0, 0.0, 0.0], np.float32)
+    adv = np.array([1.0, 1.0, -1.0, 1.0, 1.0, -1.0, 1.0, 1.0], np.float32)
+    m = np.array([1, 1, 1, 1, 1, 1, 1, 0], np.uint8)
+    f = O.decoupled_flags(logp, prox, roll, adv, m, 0.2, 0.28, 0.5, 2.0)
+    # kept; r = 1.5 > 1.28 with A > 0: clip high; r = 0.5 < 0.8 with A < 0: clip low;
+    # w = 1/4 <= 0.5: mismatch low; w = 3 >= 2: mismatch high; kept (A < 0, r = 1);
+    # non-finite log-ratio; not an action token
+    assert list(f) == [0, 2, 1, 5, 6, 0, 3, 4]
