@@ -21,7 +21,7 @@ def summarize(path, only=None):
         short = name.split("(")[0].replace("void ", "")
         if "sao::" in short:
             short = short.split("::")[-1]
-        mt = re.match(r"tc_gemm_kernel<(\d), (\d), (\d)(?:, (\d))?>", short)
+        mt = re.match(r"tc_gemm_kernel<(\d), (\d), (\d)(?:, (\d))?(?:, (\d))?>", short)
         if mt:
             label = {("0", "0", "0"): "tc_gemm<softmax> (logits lse fwd)",
                      ("4", "0", "0"): "tc_gemm<softmax+store> (logits lse fwd, stores bf16 e)",
@@ -31,6 +31,8 @@ def summarize(path, only=None):
                      ("2", "1", "1"): "tc_gemm<store f32> (dW = e^T (s H), or dZ^T H)"}.get(mt.groups()[:3], short)
             if mt.group(4) == "2":
                 label += ", 2 M tiles per CTA tile"
+            if mt.group(5) == "2":
+                label += ", CTA pairs"
             short = label
         if only and not any(o in name for o in only):
             continue
