@@ -74,6 +74,27 @@ def test_step_advantages_misaligned_outputs():
         assert np.array_equal(vm.cpu().numpy(), wv)
 
 
+@pytest.mark.parametrize("mode", [sao.SAO_STEP_AVERAGE, sao.SAO_STEP_LAST])
+def test_step_advantages_large_batch(mode):
+    """2^25 + 4,321 tokens of turn-length steps: from 2^25 tokens the per-step
+    sums take 32 steps per warp, and the broadcast's groups are not split; 48
+    sampled trajectories and the last two (the ragged tail) against the oracle
+    on their own slices."""
+    N = (1 << 25) + 4321
+    wl = S.bandwidth_workload(N=N, B=max(1, N >> 13))
+    g, lam, lc, al = f32(0.99), f32(0.95), f32(0.97), f32(1.5)
+    adv, ret, vm = _step_gpu(wl, g, lam, lc, al, mode)
+    rng = np.random.default_rng(mode + 5)
+    picks = np.concatenate([rng.choice(wl.B, size=48, replace=False), [wl.B - 2, wl.B - 1]])
+    for b in picks:
+        lo, hi = wl.cu_seqlens[b], wl.cu_seqlens[b + 1]
+        wa, wr, wv = O.step_advantages(wl.values[lo:hi], wl.rewards[b:b + 1], wl.loss_mask[lo:hi],
+                                       np.array([0, hi - lo]), g, lam, lc, al, mode)
+        assert rel_err_floor(adv[lo:hi], wa, 1e-3).max() <= ADV_TOL
+        assert rel_err_floor(ret[lo:hi], wr, 1e-3).max() <= ADV_TOL
+        assert np.array_equal(vm[lo:hi], wv)
+
+
 def test_step_advantages_no_action_tokens():
     wl = S.make_custom([10, 300], 8, 16, "f32", seed=4, dense=False)
     wl.loss_mask[:] = 0
