@@ -424,27 +424,41 @@ struct VLArgs {
   double *sums;  // [5][grid]: sum d^2, sum e, sum e^2, sum R, sum R^2
 };
 
+// Per-token terms of the value loss and the EV sums, exact up to the final
+// additions: d = V - R as an fp32 pair (two-sum), its square and R^2 as a
+// rounded product plus the product's remainder (fused multiply-add), so the
+// sums are fp64-grade although every operation is fp32.
+struct VLTerms {
+  Acc2 d2, e, r, r2;  // sum d^2 (= sum (R - V)^2), sum (R - V), sum R, sum R^2: leading parts
+  float d2_lo = 0.f, e_lo = 0.f, r2_lo = 0.f;  // their small remainders, summed plainly
+  __device__ __forceinline__ void add(float v, float rt) {
+    const float dh = __fsub_rn(v, rt);
+    const float bb = __fsub_rn(dh, v);
+    const float dl = __fsub_rn(__fsub_rn(v, __fsub_rn(dh, bb)), __fadd_rn(rt, bb));  // v - rt = dh + dl exactly
+    const float p = __fmul_rn(dh, dh);
+    d2.add(p);
+    d2_lo = __fadd_rn(d2_lo, __fmaf_rn(2.f * dh, dl, __fmaf_rn(dh, dh, -p)));
+    e.add(-dh);
+    e_lo = __fsub_rn(e_lo, dl);
+    r.add(rt);
+    const float q = __fmul_rn(rt, rt);
+    r2.add(q);
+    r2_lo = __fadd_rn(r2_lo, __fmaf_rn(rt, rt, -q));
+  }
+};
+
 __global__ void __launch_bounds__(kThreads) value_loss_kernel(VLArgs a) {
   const long long n = a.n_norm > 0 ? a.n_norm : total_of(a.cnt_partial, a.n_cnt);
   const float two_over_n = n > 0 ? float(2.0 / double(n)) : 0.f;
-  Acc2 a_d2, a_e, a_e2, a_r, a_r2;
+  VLTerms acc;
   const int64_t tid = int64_t(blockIdx.x) * kThreads + threadIdx.x;
   const int64_t stride = int64_t(gridDim.x) * kThreads;
   const bool vec = aligned16_dev(a.v) && aligned16_dev(a.ret) && aligned16_dev(a.grad) &&
                    ((reinterpret_cast<uintptr_t>(a.m) & 3u) == 0);
-  auto one = [&](float v, float r, uint8_t m, float &g, float &d2, float &e, float &e2, float &rr,
-                 float &rr2) {
-    if (!m) {
-      g = 0.f;
-      return;
-    }
-    const float d = v - r;
-    g = two_over_n * d;
-    d2 = fmaf(d, d, d2);
-    e -= d;
-    e2 = fmaf(d, d, e2);
-    rr += r;
-    rr2 = fmaf(r, r, rr2);
+  auto one = [&](float v, float r, uint8_t m) {
+    if (!m) return 0.f;
+    acc.add(v, r);
+    return two_over_n * (v - r);
   };
   int64_t done = 0;
   if (vec) {
@@ -454,41 +468,27 @@ __global__ void __launch_bounds__(kThreads) value_loss_kernel(VLArgs a) {
       const float4 r = __ldg(reinterpret_cast<const float4 *>(a.ret) + i);
       const uchar4 m = __ldg(reinterpret_cast<const uchar4 *>(a.m) + i);
       float4 g;
-      float d2 = 0, e = 0, e2 = 0, rr = 0, rr2 = 0;
-      one(v.x, r.x, m.x, g.x, d2, e, e2, rr, rr2);
-      one(v.y, r.y, m.y, g.y, d2, e, e2, rr, rr2);
-      one(v.z, r.z, m.z, g.z, d2, e, e2, rr, rr2);
-      one(v.w, r.w, m.w, g.w, d2, e, e2, rr, rr2);
+      g.x = one(v.x, r.x, m.x);
+      g.y = one(v.y, r.y, m.y);
+      g.z = one(v.z, r.z, m.z);
+      g.w = one(v.w, r.w, m.w);
       reinterpret_cast<float4 *>(a.grad)[i] = g;
-      a_d2.add(d2);
-      a_e.add(e);
-      a_e2.add(e2);
-      a_r.add(rr);
-      a_r2.add(rr2);
     }
     done = n4 * 4;
   }
-  for (int64_t i = done + tid; i < a.N; i += stride) {
-    float g, d2 = 0, e = 0, e2 = 0, rr = 0, rr2 = 0;
-    one(__ldg(a.v + i), __ldg(a.ret + i), __ldg(a.m + i), g, d2, e, e2, rr, rr2);
-    a.grad[i] = g;
-    a_d2.add(d2);
-    a_e.add(e);
-    a_e2.add(e2);
-    a_r.add(rr);
-    a_r2.add(rr2);
-  }
-  double s_d2 = a_d2.value(), s_e = a_e.value(), s_e2 = a_e2.value(), s_r = a_r.value(), s_r2 = a_r2.value();
+  for (int64_t i = done + tid; i < a.N; i += stride)
+    a.grad[i] = one(__ldg(a.v + i), __ldg(a.ret + i), __ldg(a.m + i));
+  double s_d2 = acc.d2.value() + double(acc.d2_lo), s_e = acc.e.value() + double(acc.e_lo);
+  double s_r = acc.r.value(), s_r2 = acc.r2.value() + double(acc.r2_lo);
   s_d2 = block_sum(s_d2);
   s_e = block_sum(s_e);
-  s_e2 = block_sum(s_e2);
   s_r = block_sum(s_r);
   s_r2 = block_sum(s_r2);
   if (threadIdx.x == 0) {
     const int g = gridDim.x, b = blockIdx.x;
     a.sums[b] = s_d2;
     a.sums[g + b] = s_e;
-    a.sums[2 * g + b] = s_e2;
+    a.sums[2 * g + b] = s_d2;  // sum (R - V)^2 = sum d^2
     a.sums[3 * g + b] = s_r;
     a.sums[4 * g + b] = s_r2;
   }
