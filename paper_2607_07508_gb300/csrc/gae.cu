@@ -443,11 +443,12 @@ __device__ GState look_back(const GaeArgs &a, int q, int lane) {
 // global memory) of one row and when 8 lanes read the same granule of their
 // own rows. The two value buffers hold the piece being folded and the next
 // one, copied meanwhile. Each lane also stores its values into its own TMEM
-// lane (the warp's 32 lanes of the CTA's allocation, column 32k + i for token
-// i of piece k) and its action bits into `act`, so that the replay, after the
-// look-back, reads the chunk from the SM instead of from DRAM a second time;
-// the replay writes advantages into val[0] and returns into ret, which the
-// warp then stores coalesced.
+// lane (the warp's 32 lanes of the CTA's allocation, column 32 (s + k) + i for
+// token i of piece k, where the slot s is 0, or 2 for the second of two
+// 2-piece chunks in flight) and its action bits into act[s + k], so that the
+// replay, after the look-back, reads the chunk from the SM instead of from
+// DRAM a second time; the replay writes advantages into val[0] and returns
+// into ret, which the warp then stores coalesced.
 constexpr int kScanCuCap = 120;  // cu_seqlens entries staged per warp
 struct __align__(16) WarpBuf {
   float val[2][kChunk];           // values of two pieces (fold); advantages of one (replay)
@@ -908,8 +909,9 @@ __device__ void replay_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int la
 // Persistent warps: a warp takes a chunk (ticket), folds and publishes it,
 // looks back and replays it. Tickets keep the decoupled look-back safe: a
 // warp waits only on chunks taken before its own, and every taken chunk is
-// folded and published at once, before its warp waits on anything. Each CTA holds kTmemCols TMEM columns for the whole launch (four
-// CTAs per SM take all 512, so the allocation never waits on this kernel).
+// folded and published at once, before its warp waits on anything. Each CTA
+// holds kTmemCols TMEM columns for the whole launch (four CTAs per SM take all
+// 512, so the allocation never waits on this kernel).
 template <bool kCrit, bool kPipe>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) gae_scan_kernel(GaeArgs a) {
   extern __shared__ __align__(16) unsigned char s_raw[];
