@@ -207,6 +207,11 @@ SAO_API sao_status sao_token_logprobs_bwd_cached(const void *H, const void *W, s
  *   cu_seqlens [B+1] int32 with 0 = cu[0] <= ... <= cu[B] = N
  *   adv, ret [N] fp32 outputs
  * Scalars: 0 <= gamma, lambda_policy, lambda_critic <= 1.
+ * The scan keeps each chunk's values in TMEM between its two passes: while it
+ * runs, each SM's 512 TMEM columns are held by its CTAs, so a kernel on
+ * another stream that allocates TMEM on the same SM waits for them (and the
+ * scan waits for such a kernel's columns); neither depends on the other's
+ * progress, so the wait always ends.
  */
 SAO_API sao_status sao_advantages(const float *values, const float *rewards, const uint8_t *loss_mask,
                           const int32_t *cu_seqlens, int32_t B, int64_t N, float gamma,
