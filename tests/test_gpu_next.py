@@ -95,6 +95,28 @@ def test_step_advantages_large_batch(mode):
         assert np.array_equal(vm[lo:hi], wv)
 
 
+@pytest.mark.parametrize("N", [(1 << 20) + 3, (1 << 25) + 777])
+def test_step_advantages_short_steps(N):
+    """Token-by-token random masks: steps of 1-3 tokens, several inside one
+    lane's 4 tokens (the broadcast's per-token search), one lane per short step
+    in the per-step sums, millions of steps; sampled trajectories and the
+    ragged tail against the oracle on their own slices, both value modes."""
+    wl = S.bandwidth_workload(N=N, B=max(1, N >> 13))
+    rng = np.random.default_rng(N % 997)
+    wl.loss_mask = (rng.random(N) < 0.6).astype(np.uint8)
+    g, lam, lc = f32(1.0), f32(0.95), f32(1.0)
+    picks = np.concatenate([rng.choice(wl.B, size=24, replace=False), [wl.B - 2, wl.B - 1]])
+    for mode in (sao.SAO_STEP_AVERAGE, sao.SAO_STEP_LAST):
+        adv, ret, vm = _step_gpu(wl, g, lam, lc, 0.0, mode)
+        for b in picks:
+            lo, hi = wl.cu_seqlens[b], wl.cu_seqlens[b + 1]
+            wa, wr, wv = O.step_advantages(wl.values[lo:hi], wl.rewards[b:b + 1], wl.loss_mask[lo:hi],
+                                           np.array([0, hi - lo]), g, lam, lc, 0.0, mode)
+            assert rel_err_floor(adv[lo:hi], wa, 1e-3).max() <= ADV_TOL
+            assert rel_err_floor(ret[lo:hi], wr, 1e-3).max() <= ADV_TOL
+            assert np.array_equal(vm[lo:hi], wv)
+
+
 def test_step_advantages_no_action_tokens():
     wl = S.make_custom([10, 300], 8, 16, "f32", seed=4, dense=False)
     wl.loss_mask[:] = 0
