@@ -145,6 +145,27 @@ def test_advantages_long_lane_segments(N):
             assert rel_err_floor(ret[lo:hi], r, 1e-3).max() <= ADV_TOL
 
 
+def test_advantages_short_trajectories_random_masks():
+    """4-piece lane segments (2^26 tokens and more, one chunk per warp in all
+    of its TMEM columns) with ~512-token trajectories and token-by-token random
+    masks: many trajectory ends inside each piece (the per-token path) and
+    mixed 4-token groups; sampled trajectories and the ragged tail against the
+    oracle."""
+    N = (1 << 26) + 999
+    wl = S.bandwidth_workload(N=N, B=N >> 9)
+    rng = np.random.default_rng(26)
+    wl.loss_mask = (rng.random(N) < 0.6).astype(np.uint8)
+    picks = np.concatenate([rng.choice(wl.B, size=64, replace=False), [wl.B - 2, wl.B - 1]])
+    for coefs in ((1.0, 0.95, 1.0, 0.0), (0.99, 1.0, 0.97, 1.5)):
+        adv, ret, g = _gae_gpu(wl, gamma=coefs[0], lam=coefs[1], lam_c=coefs[2], alpha=coefs[3])
+        for b in picks:
+            lo, hi = wl.cu_seqlens[b], wl.cu_seqlens[b + 1]
+            a, r = O.advantages(wl.values[lo:hi], wl.rewards[b:b + 1], wl.loss_mask[lo:hi], np.array([0, hi - lo]),
+                                g["gamma"], g["lam"], g["lam_c"], g["alpha"])
+            assert rel_err_floor(adv[lo:hi], a, 1e-3).max() <= ADV_TOL
+            assert rel_err_floor(ret[lo:hi], r, 1e-3).max() <= ADV_TOL
+
+
 def test_advantages_checked_mode_reports_bad_cu_seqlens():
     wl = S.make_custom([10, 20], 8, 16, "f32", seed=5, dense=False)
     bad = wl.cu_seqlens.copy()
