@@ -570,7 +570,6 @@ def main():
     ap.add_argument("--cached", action="store_true",
                     help="time the variant whose forward stores bf16 probabilities for all computed rows "
                          "(2*N*V bytes) instead of the default vocabulary-chunked recompute path")
-    ap.add_argument("--recompute", action="store_true", help="the default path (kept for older command lines)")
     ap.add_argument("--dz-budget-gib", type=float, default=None,
                     help="bound on the backward's bf16 dZ buffer (default: the library's, 4 GiB)")
     ap.add_argument("--cta-pairs", type=int, choices=[0, 1], default=None,
