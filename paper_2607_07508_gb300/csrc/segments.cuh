@@ -141,6 +141,12 @@ __global__ void __launch_bounds__(256) action_count_kernel(const uint8_t *m, con
       const int64_t t0 = base + j * 128 + int64_t(lane) * 4;
       u[j] = (aligned && t0 + 4 <= c1) ? __ldg(reinterpret_cast<const uint32_t *>(m + t0)) : 0u;
     }
+    if (aligned && base + 8 * 128 <= c1 && base + 8 * 128 <= next_end) {
+      // the whole window inside the lane's current trajectory (the common case)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) cnt += __popc(((u[j] & 0x7f7f7f7fu) + 0x7f7f7f7fu | u[j]) & 0x80808080u);
+      continue;
+    }
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const int64_t t0 = base + j * 128 + int64_t(lane) * 4;
