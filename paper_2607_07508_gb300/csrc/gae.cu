@@ -515,6 +515,7 @@ __device__ __forceinline__ void stage_in(const GaeArgs &a, int64_t c0, int seg, 
       cp_async16(&msk[16 * mgran(r, j)], a.m + off + int64_t(r) * seg + 16 * j, policy);
     }
   } else {
+#pragma unroll 1
     for (int i = lane; i < kChunk; i += 32) {
       const int r = i >> 5, kk = i & 31;
       const int64_t t = off + int64_t(r) * seg + kk;
@@ -538,6 +539,7 @@ __device__ __forceinline__ void stage_out(const GaeArgs &a, int64_t c0, int seg,
       __stcs(reinterpret_cast<float4 *>(a.ret + t), *reinterpret_cast<const float4 *>(&ret[p]));
     }
   } else {
+#pragma unroll 1
     for (int i = lane; i < kChunk; i += 32) {
       const int r = i >> 5, kk = i & 31;
       const int64_t t = off + int64_t(r) * seg + kk;
@@ -592,10 +594,14 @@ __device__ __forceinline__ uint32_t piece_ends(const GaeArgs &a, const CuView &c
 // the piece's last token below N.
 
 // The token loops below take 4 tokens at a time. A group in which no lane of
-// the warp holds a trajectory end or a waiting reward (the common case: turns
-// and trajectories span hundreds of tokens) runs branch-free, one fused
-// double-float a*B + g*V per token with the action flag applied by selects;
-// otherwise the warp takes the general path for that group.
+// the warp holds a trajectory end (the common case: trajectories span
+// thousands of tokens) runs branch-free, one fused double-float a*B + g*V per
+// token with the action flag applied by selects; otherwise the warp takes the
+// general path for that group. A reward still waiting for its action token
+// (observation tokens after a trajectory's last action token) rides along on
+// the branch-free path: there B = Vn = 0, the step's products and sums are
+// exactly 0, and adding the reward to the high part gives the (R, 0) of the
+// general path's step.
 
 // A lane's fold of its segment so far (the pieces right of the current one):
 // the lambda-returns with a zero state at the segment's right edge, the value
@@ -623,7 +629,7 @@ __device__ void fold_piece(const GaeArgs &a, const float *val, uint32_t tcol, in
     tmem_st4(tcol + 4 * g, v4);  // kept for the replay
     const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
     const uint32_t a4 = (act >> (4 * g)) & 15u, e4 = (ends >> (4 * g)) & 15u;
-    if (__any_sync(0xffffffffu, e4 != 0u || P != 0.f)) {
+    if (__any_sync(0xffffffffu, e4 != 0u)) {
 #pragma unroll
       for (int i = 3; i >= 0; --i) {
         if ((e4 >> i) & 1u) {  // last token of a trajectory: reset
@@ -646,13 +652,16 @@ __device__ void fold_piece(const GaeArgs &a, const float *val, uint32_t tcol, in
 #pragma unroll
       for (int i = 3; i >= 0; --i) {
         const bool on = (a4 >> i) & 1u;
-        const df np = df_axpby_u(k.p.a, Bp, k.p.g, Vn);
+        df np = df_axpby_u(k.p.a, Bp, k.p.g, Vn);
+        np.hi = __fadd_rn(np.hi, P);
         Bp = on ? np : Bp;
         if constexpr (kCrit) {
-          const df nc = df_axpby_u(k.c.a, Bc, k.c.g, Vn);
+          df nc = df_axpby_u(k.c.a, Bc, k.c.g, Vn);
+          nc.hi = __fadd_rn(nc.hi, P);
           Bc = on ? nc : Bc;
         }
         Vn = on ? vv[i] : Vn;
+        P = on ? 0.f : P;
       }
       Bp = df_renorm(Bp);
       if constexpr (kCrit) Bc = df_renorm(Bc);
@@ -723,7 +732,7 @@ __device__ void replay_piece(const GaeArgs &a, uint32_t tcol, float *adv, float 
     if (g > 0) tmem_ld4(tcol + 4 * (g - 1), nx);
     float ov[4], orr[4];
     const uint32_t a4 = (act >> (4 * g)) & 15u, e4 = (ends >> (4 * g)) & 15u;
-    if (__any_sync(0xffffffffu, e4 != 0u || st.P != 0.f)) {
+    if (__any_sync(0xffffffffu, e4 != 0u)) {
 #pragma unroll
       for (int i = 3; i >= 0; --i) {
         ov[i] = orr[i] = 0.f;
@@ -749,17 +758,20 @@ __device__ void replay_piece(const GaeArgs &a, uint32_t tcol, float *adv, float 
 #pragma unroll
       for (int i = 3; i >= 0; --i) {
         const bool on = (a4 >> i) & 1u;
-        const df np = df_axpby_u(k.p.a, st.Bp, k.p.g, st.Vn);
+        df np = df_axpby_u(k.p.a, st.Bp, k.p.g, st.Vn);
+        np.hi = __fadd_rn(np.hi, st.P);
         ov[i] = on ? adv_round(np, vv[i]) : 0.f;
         st.Bp = on ? np : st.Bp;
         if constexpr (kCrit) {
-          const df nc = df_axpby_u(k.c.a, st.Bc, k.c.g, st.Vn);
+          df nc = df_axpby_u(k.c.a, st.Bc, k.c.g, st.Vn);
+          nc.hi = __fadd_rn(nc.hi, st.P);
           orr[i] = on ? df_round(nc) : 0.f;
           st.Bc = on ? nc : st.Bc;
         } else {
           orr[i] = on ? R : 0.f;
         }
         st.Vn = on ? vv[i] : st.Vn;
+        st.P = on ? 0.f : st.P;
       }
       st.Bp = df_renorm(st.Bp);
       if constexpr (kCrit) st.Bc = df_renorm(st.Bc);
@@ -932,21 +944,20 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) gae_scan_kernel(GaeArgs 
     // folded before, so the chunks it waits on have had a whole fold to
     // publish (with one chunk at a time that wait is exposed, and at these
     // chunk sizes it dominates)
-    int q = take_chunk(a, lane);
-    if (q >= 0) {
-      Pending<kCrit> p;
-      int half = 0;
-      fold_chunk<kCrit>(a, w, tmem, lane, q, 0, p);
+    // (one call site each for the fold and the replay: the kernel's code
+    // stays small enough for the instruction cache)
+    Pending<kCrit> p;
+    bool have = false;
+    int half = 0;
 #pragma unroll 1
-      for (;;) {
-        const int qn = take_chunk(a, lane);
-        Pending<kCrit> n;
-        if (qn >= 0) fold_chunk<kCrit>(a, w, tmem, lane, qn, (half ^ 1) * (kMaxPieces / 2), n);
-        replay_chunk<kCrit>(a, w, tmem, lane, p, true);
-        if (qn < 0) break;
-        p = n;
-        half ^= 1;
-      }
+    for (int q = take_chunk(a, lane);; q = take_chunk(a, lane)) {
+      Pending<kCrit> n;
+      if (q >= 0) fold_chunk<kCrit>(a, w, tmem, lane, q, half * (kMaxPieces / 2), n);
+      if (have) replay_chunk<kCrit>(a, w, tmem, lane, p, true);
+      if (q < 0) break;
+      p = n;
+      have = true;
+      half ^= 1;
     }
   } else {
     // long segments: one chunk at a time in all of the warp's columns (the
