@@ -124,6 +124,7 @@ __device__ __forceinline__ df df_renorm(df x) { return two_sum(x.hi, x.lo); }
 // x^e for 0 <= e < 32 by squaring.
 __device__ df df_pow(df x, int e) {
   df r = {1.f, 0.f};
+#pragma unroll 1
   while (e) {
     if (e & 1) r = df_mul(r, x);
     e >>= 1;
@@ -630,8 +631,9 @@ __device__ void fold_piece(const GaeArgs &a, const float *val, uint32_t tcol, in
     const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
     const uint32_t a4 = (act >> (4 * g)) & 15u, e4 = (ends >> (4 * g)) & 15u;
     if (__any_sync(0xffffffffu, e4 != 0u)) {
-#pragma unroll
+#pragma unroll 1
       for (int i = 3; i >= 0; --i) {
+        const float v = i == 3 ? vv[3] : (i == 2 ? vv[2] : (i == 1 ? vv[1] : vv[0]));
         if ((e4 >> i) & 1u) {  // last token of a trajectory: reset
           const int b = cu.find(blo, b_last, t0 + 4 * g + i);
           k = load_coefs<kCrit>(a.coef, b);
@@ -643,7 +645,7 @@ __device__ void fold_piece(const GaeArgs &a, const float *val, uint32_t tcol, in
         if ((a4 >> i) & 1u) {
           Bp = step_return(k.p, Bp, Vn, P);
           if constexpr (kCrit) Bc = step_return(k.c, Bc, Vn, P);
-          Vn = vv[i];
+          Vn = v;
           P = 0.f;
           fl |= 2;
         }
@@ -733,9 +735,10 @@ __device__ void replay_piece(const GaeArgs &a, uint32_t tcol, float *adv, float 
     float ov[4], orr[4];
     const uint32_t a4 = (act >> (4 * g)) & 15u, e4 = (ends >> (4 * g)) & 15u;
     if (__any_sync(0xffffffffu, e4 != 0u)) {
-#pragma unroll
+#pragma unroll 1
       for (int i = 3; i >= 0; --i) {
-        ov[i] = orr[i] = 0.f;
+        const float v = i == 3 ? vv[3] : (i == 2 ? vv[2] : (i == 1 ? vv[1] : vv[0]));
+        float o = 0.f, orv = 0.f;
         if ((e4 >> i) & 1u) {
           const int b = cu.find(blo, b_last, t0 + 4 * g + i);
           k = load_coefs<kCrit>(a.coef, b);
@@ -747,11 +750,16 @@ __device__ void replay_piece(const GaeArgs &a, uint32_t tcol, float *adv, float 
         if ((a4 >> i) & 1u) {
           st.Bp = step_return(k.p, st.Bp, st.Vn, st.P);
           if constexpr (kCrit) st.Bc = step_return(k.c, st.Bc, st.Vn, st.P);
-          ov[i] = adv_round(st.Bp, vv[i]);
+          o = adv_round(st.Bp, v);
           // gamma = lambda_critic = 1: the critic's return is the trajectory's reward
-          orr[i] = kCrit ? df_round(st.Bc) : R;
-          st.Vn = vv[i];
+          orv = kCrit ? df_round(st.Bc) : R;
+          st.Vn = v;
           st.P = 0.f;
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          ov[j] = j == i ? o : ov[j];
+          orr[j] = j == i ? orv : orr[j];
         }
       }
     } else {
