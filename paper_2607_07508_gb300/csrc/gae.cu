@@ -437,7 +437,7 @@ __device__ GState look_back(const GaeArgs &a, int q, int lane) {
 // lane r's segment starts at chunk offset r * seg. The fold streams the
 // segments through shared memory one 32-token piece at a time (right to
 // left): row r of a staged piece holds lane r's 32 tokens of that piece.
-// val/ret rows are 8 granules of 16 bytes, granule j stored at
+// val rows are 8 granules of 16 bytes, granule j stored at
 // 8r + (j ^ (r & 7)); msk rows are 2 granules, granule j at
 // 2r + (j ^ ((r >> 2) & 1)). A quarter-warp (8 lanes) then touches 8 distinct
 // bank groups both when it copies the 8 granules (128 contiguous bytes of
@@ -446,16 +446,17 @@ __device__ GState look_back(const GaeArgs &a, int q, int lane) {
 // one, copied meanwhile. Each lane also stores its values into its own TMEM
 // lane (the warp's 32 lanes of the CTA's allocation, column 32 (s + k) + i for
 // token i of piece k, where the slot s is 0, or 2 for the second of two
-// 2-piece chunks in flight) and its action bits into act[s + k], so that the
-// replay, after the look-back, reads the chunk from the SM instead of from
-// DRAM a second time; the replay writes advantages into val[0] and returns
-// into ret, which the warp then stores coalesced.
+// 2-piece chunks in flight) and its action bits into act[s + k] (the chunk's
+// trajectory-end bits are in ends[s + k]), so that the replay, after the
+// look-back, reads the chunk from the SM instead of from DRAM a second time;
+// the replay writes advantages into val[0] and returns into val[1], which the
+// warp then stores coalesced.
 constexpr int kScanCuCap = 120;  // cu_seqlens entries staged per warp
 struct __align__(16) WarpBuf {
-  float val[2][kChunk];           // values of two pieces (fold); advantages of one (replay)
-  float ret[kChunk];              // returns of the piece being replayed
+  float val[2][kChunk];           // values of two pieces (fold); advantages and returns of one (replay)
   uint8_t msk[kChunk];            // action flags of the piece being copied
   uint32_t act[kMaxPieces][32];   // per piece, each lane's action bits
+  uint32_t ends[kMaxPieces][32];  // per piece, each lane's trajectory-end bits
   int32_t cu[kScanCuCap];         // cu_seqlens slice of the chunk being folded
   uint32_t tmem;                  // TMEM address of the CTA's allocation (warp 0's buffer)
 };
@@ -567,32 +568,33 @@ __device__ __forceinline__ uint32_t row_actions(const uint8_t *msk, int lane) {
          nonzero_bytes(m1.w) << 28;
 }
 
-// Trajectory ends among the 32 tokens from t0 (bit e: token t0 + e is the last
-// token of its trajectory), by a forward walk over cu_seqlens; b_last is the
-// trajectory of the last of those tokens below N. No bits past N.
-__device__ __forceinline__ uint32_t piece_ends(const GaeArgs &a, const CuView &cu, int blo, int bhi, int64_t t0,
-                                               int &b_last) {
-  uint32_t ends = 0;
-  b_last = blo;
-  if (t0 >= a.N) return 0;
-  const int64_t tl = (t0 + kItems <= a.N ? int64_t(kItems) : a.N - t0) - 1;  // last token, relative to t0
-  int b = cu.find(blo, bhi, t0);
-  for (;;) {
-    const int64_t e = cu[b + 1] - 1 - t0;  // last token of trajectory b, relative to t0
-    if (e >= 0 && e <= tl) ends |= 1u << e;
-    if (e >= tl || b >= bhi) break;  // b holds the piece's last token (or cu_seqlens is malformed)
-    ++b;
+// The trajectory ends of the chunk at c0 (pieces pieces in `slot`), as bits:
+// every end e = cu[b + 1] - 1 inside the chunk sets bit u mod 32 of
+// ends[slot + u / 32][r], where r = (e - c0) / seg and u = (e - c0) mod seg.
+__device__ __forceinline__ void mark_ends(const CuView &cu, int blo, int bhi, int64_t c0, int seg, int pieces,
+                                          int slot, int lane, WarpBuf &w) {
+#pragma unroll 1
+  for (int i = lane; i < 32 * pieces; i += 32) w.ends[slot + (i >> 5)][i & 31] = 0u;
+  __syncwarp();
+  const int64_t c1 = c0 + 32 * int64_t(seg);
+  const int lseg = 31 - __clz(seg);  // seg is a power of two
+#pragma unroll 1
+  for (int b = blo + lane; b <= bhi; b += 32) {
+    const int64_t e = cu[b + 1] - 1;
+    if (e >= c0 && e < c1) {
+      const int off = int(e - c0), u = off & (seg - 1);
+      atomicOr(&w.ends[slot + (u >> 5)][off >> lseg], 1u << (u & 31));
+    }
   }
-  b_last = b;
-  return ends;
+  __syncwarp();
 }
 
 // ---------------------------------------------------------------------------
 // per-lane fold and replay
 // ---------------------------------------------------------------------------
 // A piece's tokens are t0 .. t0+31; bit k of `act` / `ends`: token t0+k is an
-// action token / the last token of its trajectory; b_last is the trajectory of
-// the piece's last token below N.
+// action token / the last token of its trajectory; blo .. bhi bound the
+// trajectories the chunk can touch.
 
 // The token loops below take 4 tokens at a time. A group in which no lane of
 // the warp holds a trajectory end (the common case: trajectories span
@@ -618,24 +620,25 @@ struct FoldState {
 
 template <bool kCrit>
 __device__ void fold_piece(const GaeArgs &a, const float *val, uint32_t tcol, int lane, uint32_t act, uint32_t ends,
-                           int64_t t0, const CuView &cu, int blo, int b_last, FoldState<kCrit> &f) {
+                           int64_t t0, const CuView &cu, int blo, int bhi, FoldState<kCrit> &f) {
   Coefs<kCrit> k = f.k;
   df Bp = f.Bp, Bc = f.Bc;
   float Vn = f.Vn, P = f.P;
   int fl = f.fl;
   const int sw = lane & 7;
+  const bool any_end = __any_sync(0xffffffffu, ends != 0u);  // else no group needs the general path
 #pragma unroll 1
   for (int g = 7; g >= 0; --g) {
     const float4 v4 = *reinterpret_cast<const float4 *>(&val[4 * (8 * lane + (g ^ sw))]);
     tmem_st4(tcol + 4 * g, v4);  // kept for the replay
     const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
     const uint32_t a4 = (act >> (4 * g)) & 15u, e4 = (ends >> (4 * g)) & 15u;
-    if (__any_sync(0xffffffffu, e4 != 0u)) {
+    if (any_end && __any_sync(0xffffffffu, e4 != 0u)) {
 #pragma unroll 1
       for (int i = 3; i >= 0; --i) {
         const float v = i == 3 ? vv[3] : (i == 2 ? vv[2] : (i == 1 ? vv[1] : vv[0]));
         if ((e4 >> i) & 1u) {  // last token of a trajectory: reset
-          const int b = cu.find(blo, b_last, t0 + 4 * g + i);
+          const int b = cu.find(blo, bhi, t0 + 4 * g + i);
           k = load_coefs<kCrit>(a.coef, b);
           P = __ldg(a.rewards + b);
           Bp = Bc = {0.f, 0.f};
@@ -716,12 +719,13 @@ struct ReplayState {
 // of `adv`, returns to its row of `ret`.
 template <bool kCrit>
 __device__ void replay_piece(const GaeArgs &a, uint32_t tcol, float *adv, float *ret, int lane, uint32_t act,
-                             uint32_t ends, int64_t t0, const CuView &cu, int blo, int b_last,
+                             uint32_t ends, int64_t t0, const CuView &cu, int blo, int bhi,
                              ReplayState<kCrit> &rs) {
   Coefs<kCrit> k = rs.k;
   float R = rs.R;
   GState st = rs.st;
   const int sw = lane & 7;
+  const bool any_end = __any_sync(0xffffffffu, ends != 0u);  // else no group needs the general path
   uint32_t nx[4];
   tmem_ld4(tcol + 28, nx);
   tmem_wait_ld4(nx);
@@ -734,13 +738,13 @@ __device__ void replay_piece(const GaeArgs &a, uint32_t tcol, float *adv, float 
     if (g > 0) tmem_ld4(tcol + 4 * (g - 1), nx);
     float ov[4], orr[4];
     const uint32_t a4 = (act >> (4 * g)) & 15u, e4 = (ends >> (4 * g)) & 15u;
-    if (__any_sync(0xffffffffu, e4 != 0u)) {
+    if (any_end && __any_sync(0xffffffffu, e4 != 0u)) {
 #pragma unroll 1
       for (int i = 3; i >= 0; --i) {
         const float v = i == 3 ? vv[3] : (i == 2 ? vv[2] : (i == 1 ? vv[1] : vv[0]));
         float o = 0.f, orv = 0.f;
         if ((e4 >> i) & 1u) {
-          const int b = cu.find(blo, b_last, t0 + 4 * g + i);
+          const int b = cu.find(blo, bhi, t0 + 4 * g + i);
           k = load_coefs<kCrit>(a.coef, b);
           R = __ldg(a.rewards + b);
           st.Bp = st.Bc = {0.f, 0.f};
@@ -833,6 +837,7 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane
   if (cu.in_smem)
     for (int i = lane; i < ncu; i += 32) w.cu[i] = __ldg(a.cu + blo + i);
   __syncwarp();
+  mark_ends(cu, blo, bhi, c0, seg, a.pieces, slot, lane, w);
 
   // the trajectory of the lane's last token below N gives its first coefficients
   const int64_t s_end = (s0 + seg < N ? s0 + seg : N) - 1;
@@ -853,11 +858,9 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane
     __syncwarp();  // every lane has read the flags and finished the previous piece
     if (k > 0) stage_in(a, c0, seg, k - 1, lane, w.val[cur ^ 1], w.msk, pol);
     const int64_t t0 = s0 + 32 * int64_t(k);
-    int b_last;
-    const uint32_t ends = piece_ends(a, cu, blo, bhi, t0, b_last);
     // every lane folds (the token loops vote across the warp); a lane past N
     // has no flags and keeps its state
-    fold_piece<kCrit>(a, w.val[cur], tmem + 32 * (slot + k), lane, act, ends, t0, cu, blo, b_last, f);
+    fold_piece<kCrit>(a, w.val[cur], tmem + 32 * (slot + k), lane, act, w.ends[slot + k][lane], t0, cu, blo, bhi, f);
   }
   tmem_wait_st();  // the values are in TMEM before the replay reads them
 
@@ -917,11 +920,10 @@ __device__ void replay_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int la
   for (int k = a.pieces - 1; k >= 0; --k) {
     const uint32_t act = w.act[p.slot + k][lane];
     const int64_t t0 = s0 + 32 * int64_t(k);
-    int b_last;
-    const uint32_t ends = piece_ends(a, cu, p.blo, p.bhi, t0, b_last);
-    replay_piece<kCrit>(a, tmem + 32 * (p.slot + k), w.val[0], w.ret, lane, act, ends, t0, cu, p.blo, b_last, rs);
+    replay_piece<kCrit>(a, tmem + 32 * (p.slot + k), w.val[0], w.val[1], lane, act, w.ends[p.slot + k][lane], t0,
+                        cu, p.blo, p.bhi, rs);
     __syncwarp();
-    stage_out(a, c0, seg, k, lane, w.val[0], w.ret);
+    stage_out(a, c0, seg, k, lane, w.val[0], w.val[1]);
     __syncwarp();  // every lane has read its granules before the next piece overwrites them
   }
 }
