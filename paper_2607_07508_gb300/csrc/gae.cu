@@ -20,14 +20,16 @@
 // resets S to (0, 0, 0, R_b). Maps compose associatively, so:
 //   * a warp owns a chunk of 32 lane segments, each lane 32 * pieces
 //     consecutive tokens (pieces = 1, 2 or 4, from N); the segments stream
-//     through shared memory one 32-token piece at a time with cp.async
-//     (16-byte granules, rows XOR-swizzled so that both the coalesced copies
-//     and the lane-major row reads are free of bank conflicts),
+//     through shared memory one 32-token piece at a time, one TMA tensor
+//     copy for the values and one for the mask (the arrays seen as a row per
+//     lane segment, rows swizzled so that the lane-major row reads are free
+//     of bank conflicts), and the results leave the same way,
 //   * each lane folds its segment into one map, driven by two bit masks
-//     (action tokens, trajectory ends) so the common token costs one fused
-//     double-float a*B + g*V, a few selects and no index arithmetic, and
-//     keeps its values in its own TMEM lane for the replay (the scan issues
-//     no MMA, so the SM's 256 KB of TMEM is free: 4 CTAs x 128 columns),
+//     (action tokens; trajectory ends, marked once per chunk from its
+//     cu_seqlens slice) so the common token costs one fused double-float
+//     a*B + g*V, a few selects and no index arithmetic, and keeps its values
+//     in its own TMEM lane for the replay (the scan issues no MMA, so the
+//     SM's 256 KB of TMEM is free: 4 CTAs x 128 columns),
 //   * a warp-shuffle suffix scan combines the 32 maps of the chunk,
 //   * warps chain their chunks right-to-left by decoupled look-back: chunks
 //     are taken by ticket, so a warp only ever waits on chunks taken before
@@ -37,8 +39,8 @@
 //     8-byte words, so neither side needs a fence; every wait is bounded and
 //     a time-out raises SAO_DEVERR_SCAN_TIMEOUT,
 //   * each lane then replays its tokens from TMEM, starting from its incoming
-//     state, writing A and the return into shared memory, and the warp
-//     stores both coalesced.
+//     state, writing A and the return into shared memory, from where one
+//     tensor store each takes them out.
 // Traffic: values 4 B + mask 1 B read, adv 4 B + ret 4 B written per token.
 #include <stdint.h>
 
@@ -104,10 +106,12 @@ __device__ __forceinline__ df df_axpby(df a, df x, df g, float v) {
   lo = __fadd_rn(lo, s.lo);
   return quick_two_sum(s.hi, lo);
 }
-// The same a*x + g*v with the result left unnormalised: (s, lo) with lo a few
-// ulps of s, which the next step's products take as they are. The
-// branch-free token loops renormalise once per 4-token group, so the pair
-// never drifts (its low part stays within a few ulps of the high one).
+// The same a*x + g*v with the result left unnormalised: (s, lo), which the
+// next step's products take as they are (every term of lo is carried, none
+// dropped). Each step adds a few ulps of s to lo, so over the 32 tokens
+// between the renormalisations of the branch-free loops (once per piece) lo
+// stays within about a hundred ulps of s, and its own fp32 roundings stay
+// near 2^-40 of the value.
 __device__ __forceinline__ df df_axpby_u(df a, df x, df g, float v) {
   const float p1 = __fmul_rn(a.hi, x.hi);
   const float e1 = __fmaf_rn(a.hi, x.hi, -p1);
@@ -260,20 +264,27 @@ __device__ GState apply(const GMap<kCrit> &m, const GState &s) {
   return r;
 }
 
-template <bool kCrit>
+// The map of lane + d. compose reads the coefficients of its left operand
+// only, so the scan's rounds leave them out (kCoefs = false: r's are the
+// caller's own).
+template <bool kCrit, bool kCoefs = true>
 __device__ __forceinline__ GMap<kCrit> shfl_down_map(const GMap<kCrit> &m, int d) {
-  GMap<kCrit> r;
+  GMap<kCrit> r = m;
   r.fl = __shfl_down_sync(0xffffffffu, m.fl, d);
   r.vp = __shfl_down_sync(0xffffffffu, m.vp, d);
   r.ap = df_shfl_down(m.ap, d);
   r.cp = df_shfl_down(m.cp, d);
-  r.kp.a = df_shfl_down(m.kp.a, d);
-  r.kp.g = df_shfl_down(m.kp.g, d);
+  if constexpr (kCoefs) {
+    r.kp.a = df_shfl_down(m.kp.a, d);
+    r.kp.g = df_shfl_down(m.kp.g, d);
+  }
   if constexpr (kCrit) {
     r.ac = df_shfl_down(m.ac, d);
     r.cc = df_shfl_down(m.cc, d);
-    r.kc.a = df_shfl_down(m.kc.a, d);
-    r.kc.g = df_shfl_down(m.kc.g, d);
+    if constexpr (kCoefs) {
+      r.kc.a = df_shfl_down(m.kc.a, d);
+      r.kc.g = df_shfl_down(m.kc.g, d);
+    }
   }
   return r;
 }
@@ -378,6 +389,15 @@ struct GaeArgs {
   float *adv, *ret;
   unsigned int *err;
   uint64_t wait_ns;        // bound of every look-back wait
+  int64_t tma_rows;        // lane-segment rows the tensor maps cover (0: no maps)
+};
+
+// The per-token arrays viewed as [tma_rows][seg] (a row per lane segment),
+// box 32 x 32 (one piece of one chunk), swizzled as the staging layout below:
+// values, advantages and returns in 128-byte rows by row mod 8, the mask in
+// 32-byte rows by bit 2 of the row.
+struct ScanMaps {
+  CUtensorMap v, m, adv, ret;
 };
 
 using seg::CuView;
@@ -438,43 +458,60 @@ __device__ GState look_back(const GaeArgs &a, int q, int lane) {
 // segments through shared memory one 32-token piece at a time (right to
 // left): row r of a staged piece holds lane r's 32 tokens of that piece.
 // val rows are 8 granules of 16 bytes, granule j stored at
-// 8r + (j ^ (r & 7)); msk rows are 2 granules, granule j at
-// 2r + (j ^ ((r >> 2) & 1)). A quarter-warp (8 lanes) then touches 8 distinct
-// bank groups both when it copies the 8 granules (128 contiguous bytes of
-// global memory) of one row and when 8 lanes read the same granule of their
-// own rows. The two value buffers hold the piece being folded and the next
-// one, copied meanwhile. Each lane also stores its values into its own TMEM
+// 8r + (j ^ (r & 7)) (the tensor copies' 128-byte swizzle, buffers 1024-byte
+// aligned); msk rows are 2 granules, granule j at 2r + (j ^ ((r >> 2) & 1))
+// (their 32-byte swizzle). 8 lanes reading the same granule of their own
+// rows then touch 8 distinct bank groups. The two value buffers hold the
+// piece being folded and the next one, copied meanwhile; chunks the tensor
+// maps do not cover (the ragged end, unaligned arrays) are staged element by
+// element in the same layout. Each lane also stores its values into its own TMEM
 // lane (the warp's 32 lanes of the CTA's allocation, column 32 (s + k) + i for
 // token i of piece k, where the slot s is 0, or 2 for the second of two
 // 2-piece chunks in flight) and its action bits into act[s + k] (the chunk's
 // trajectory-end bits are in ends[s + k]), so that the replay, after the
 // look-back, reads the chunk from the SM instead of from DRAM a second time;
-// the replay writes advantages into val[0] and returns into val[1], which the
-// warp then stores coalesced.
-constexpr int kScanCuCap = 120;  // cu_seqlens entries staged per warp
+// the replay writes advantages into val[0] and returns into val[1], which two
+// tensor stores take out.
+constexpr int kScanCuCap = 120;   // cu_seqlens entries staged per warp
+constexpr int kScanTrajCap = 32;  // trajectories whose coefficients and reward are staged per warp
 struct __align__(16) WarpBuf {
   float val[2][kChunk];           // values of two pieces (fold); advantages and returns of one (replay)
   uint8_t msk[kChunk];            // action flags of the piece being copied
   uint32_t act[kMaxPieces][32];   // per piece, each lane's action bits
   uint32_t ends[kMaxPieces][32];  // per piece, each lane's trajectory-end bits
   int32_t cu[kScanCuCap];         // cu_seqlens slice of the chunk being folded
+  float4 coef[kScanTrajCap][2];   // its trajectories' coefficient rows
+  float rew[kScanTrajCap];        // and rewards
+  uint64_t bar[2];                // completion of the tensor copies into val[0] / val[1]
+  int abort;                      // a copy did not complete in time
   uint32_t tmem;                  // TMEM address of the CTA's allocation (warp 0's buffer)
+};
+// Each warp's buffer starts 1024-byte aligned (the 128-byte swizzle's period)
+constexpr size_t kWarpBufBytes = (sizeof(WarpBuf) + 1023) / 1024 * 1024;
+__device__ __forceinline__ TC coef_row(float4 u) { return {{u.x, u.y}, {u.z, u.w}}; }
+
+// Coefficients and reward of trajectory b: from the warp's staged copy when
+// the chunk's trajectories fit, else from global memory.
+struct TrajView {
+  const float4 *gcoef;
+  const float *grew;
+  const float4 (*scoef)[2];
+  const float *srew;
+  int blo;
+  bool in_smem;
+  template <bool kCrit>
+  __device__ __forceinline__ Coefs<kCrit> coefs(int b) const {
+    if (!in_smem) return load_coefs<kCrit>(gcoef, b);
+    Coefs<kCrit> k;
+    k.p = coef_row(scoef[b - blo][0]);
+    if constexpr (kCrit) k.c = coef_row(scoef[b - blo][1]);
+    return k;
+  }
+  __device__ __forceinline__ float reward(int b) const { return in_smem ? srew[b - blo] : __ldg(grew + b); }
 };
 __device__ __forceinline__ int fgran(int r, int j) { return 8 * r + (j ^ (r & 7)); }
 __device__ __forceinline__ int mgran(int r, int j) { return 2 * r + (j ^ ((r >> 2) & 1)); }
 
-// 16-byte copy global -> shared through L2 only, with an L2 eviction policy
-__device__ __forceinline__ void cp_async16(void *smem, const void *gmem, uint64_t policy) {
-  const unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
-  asm volatile("cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2;" ::"r"(s), "l"(gmem), "l"(policy)
-               : "memory");
-}
-// Every input line is read once: the copies leave L2 first.
-__device__ __forceinline__ uint64_t l2_evict_first() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
 
 // The lane's 4 TMEM columns from `taddr` (lane field: the warp's TMEM lanes).
 __device__ __forceinline__ void tmem_st4(uint32_t taddr, float4 v) {
@@ -496,61 +533,83 @@ __device__ __forceinline__ void tmem_ld4(uint32_t taddr, uint32_t (&r)[4]) {
 __device__ __forceinline__ void tmem_wait_ld4(uint32_t (&r)[4]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3])::"memory");
 }
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
 
-// Starts the copy of piece k of the chunk at c0 (lane r's tokens c0 + r * seg
-// + 32k ..): asynchronous when the piece lies below N for every lane and the
-// inputs are 16-byte aligned, element by element (zero past N) otherwise.
-__device__ __forceinline__ void stage_in(const GaeArgs &a, int64_t c0, int seg, int k, int lane, float *val,
-                                         uint8_t *msk, uint64_t policy) {
+// The tensor copies of a piece, with an L2 policy (every input line is read
+// once: the copies leave L2 first).
+__device__ __forceinline__ void tma_load_hint(uint32_t dst, const CUtensorMap *map, uint32_t bar, int32_t x, int32_t y,
+                                              uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1, {%3, "
+      "%4}], [%2], %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y), "l"(policy)
+      : "memory");
+}
+
+// Whether chunk q lies in the rows the tensor maps cover.
+__device__ __forceinline__ bool chunk_tma(const GaeArgs &a, int q) { return 32 * (int64_t(q) + 1) <= a.tma_rows; }
+
+// Starts the copy of piece k of chunk q (first token c0) into val and msk:
+// one tensor copy each when the chunk has them (completion on `bar`),
+// element by element otherwise (zero past N).
+__device__ __forceinline__ void stage_in(const GaeArgs &a, const ScanMaps &mp, bool tma, int q, int64_t c0, int seg,
+                                         int k, int lane, float *val, uint8_t *msk, uint32_t bar, uint64_t policy) {
+  if (tma) {
+    if (lane == 0) {
+      tc::mbar_arrive_expect_tx(bar, uint32_t(kChunk * (sizeof(float) + 1)));
+      tma_load_hint(tc::smem_u32(val), &mp.v, bar, 32 * k, 32 * q, policy);
+      tma_load_hint(tc::smem_u32(msk), &mp.m, bar, 32 * k, 32 * q, policy);
+    }
+    return;
+  }
   const int64_t N = a.N;
   const int64_t off = c0 + 32 * int64_t(k);
-  if (off + 31 * int64_t(seg) + 32 <= N && aligned16_dev(a.values) && aligned16_dev(a.m)) {
-#pragma unroll
-    for (int it = 0; it < 8; ++it) {
-      const int G = it * 32 + lane, r = G >> 3, j = G & 7;
-      cp_async16(&val[4 * fgran(r, j)], a.values + off + int64_t(r) * seg + 4 * j, policy);
-    }
-#pragma unroll
-    for (int it = 0; it < 2; ++it) {
-      const int G = it * 32 + lane, r = G >> 1, j = G & 1;
-      cp_async16(&msk[16 * mgran(r, j)], a.m + off + int64_t(r) * seg + 16 * j, policy);
-    }
-  } else {
 #pragma unroll 1
-    for (int i = lane; i < kChunk; i += 32) {
-      const int r = i >> 5, kk = i & 31;
-      const int64_t t = off + int64_t(r) * seg + kk;
-      val[4 * fgran(r, kk >> 2) + (kk & 3)] = t < N ? a.values[t] : 0.f;
-      msk[16 * mgran(r, kk >> 4) + (kk & 15)] = (t < N && a.m[t] != 0) ? 1 : 0;
-    }
+  for (int i = lane; i < kChunk; i += 32) {
+    const int r = i >> 5, kk = i & 31;
+    const int64_t t = off + int64_t(r) * seg + kk;
+    val[4 * fgran(r, kk >> 2) + (kk & 3)] = t < N ? a.values[t] : 0.f;
+    msk[16 * mgran(r, kk >> 4) + (kk & 15)] = (t < N && a.m[t] != 0) ? 1 : 0;
   }
 }
 
-__device__ __forceinline__ void stage_out(const GaeArgs &a, int64_t c0, int seg, int k, int lane, const float *val,
-                                          const float *ret) {
+// Waits for the piece staged into buffer `buf` (parity bit buf of `phases`).
+__device__ __forceinline__ void stage_wait(const GaeArgs &a, bool tma, WarpBuf &w, int buf, uint32_t &phases) {
+  if (tma) {
+    tc::mbar_wait(tc::smem_u32(&w.bar[buf]), (phases >> buf) & 1u, &w.abort, a.err);
+    phases ^= 1u << buf;
+  }
+  __syncwarp();
+}
+
+// Stores piece k of chunk q from val (advantages) and ret (returns); on
+// return the buffers may be written again.
+__device__ __forceinline__ void stage_out(const GaeArgs &a, const ScanMaps &mp, bool tma, int q, int64_t c0, int seg,
+                                          int k, int lane, const float *val, const float *ret, uint64_t policy) {
+  if (tma) {
+    tc::fence_proxy_async_smem();  // this lane's writes, visible to the tensor copy
+    __syncwarp();
+    if (lane == 0) {
+      tc::tma_store_2d_hint(&mp.adv, tc::smem_u32(val), 32 * k, 32 * q, policy);
+      tc::tma_store_2d_hint(&mp.ret, tc::smem_u32(ret), 32 * k, 32 * q, policy);
+      tc::bulk_commit_group();
+      tc::bulk_wait_group_read<0>();
+    }
+    __syncwarp();
+    return;
+  }
   const int64_t N = a.N;
   const int64_t off = c0 + 32 * int64_t(k);
-  if (off + 31 * int64_t(seg) + 32 <= N && aligned16_dev(a.adv) && aligned16_dev(a.ret)) {
-#pragma unroll
-    for (int it = 0; it < 8; ++it) {
-      const int G = it * 32 + lane, r = G >> 3, j = G & 7;
-      const int p = 4 * fgran(r, j);
-      const int64_t t = off + int64_t(r) * seg + 4 * j;
-      __stcs(reinterpret_cast<float4 *>(a.adv + t), *reinterpret_cast<const float4 *>(&val[p]));
-      __stcs(reinterpret_cast<float4 *>(a.ret + t), *reinterpret_cast<const float4 *>(&ret[p]));
-    }
-  } else {
 #pragma unroll 1
-    for (int i = lane; i < kChunk; i += 32) {
-      const int r = i >> 5, kk = i & 31;
-      const int64_t t = off + int64_t(r) * seg + kk;
-      if (t < N) {
-        a.adv[t] = val[4 * fgran(r, kk >> 2) + (kk & 3)];
-        a.ret[t] = ret[4 * fgran(r, kk >> 2) + (kk & 3)];
-      }
+  for (int i = lane; i < kChunk; i += 32) {
+    const int r = i >> 5, kk = i & 31;
+    const int64_t t = off + int64_t(r) * seg + kk;
+    if (t < N) {
+      a.adv[t] = val[4 * fgran(r, kk >> 2) + (kk & 3)];
+      a.ret[t] = ret[4 * fgran(r, kk >> 2) + (kk & 3)];
     }
   }
+  tc::fence_proxy_async_smem();  // these reads before a later tensor copy into the buffers
+  __syncwarp();
 }
 
 // Bit i set when byte i of x is non-zero (i = 0..3).
@@ -620,7 +679,8 @@ struct FoldState {
 
 template <bool kCrit>
 __device__ void fold_piece(const GaeArgs &a, const float *val, uint32_t tcol, int lane, uint32_t act, uint32_t ends,
-                           int64_t t0, const CuView &cu, int blo, int bhi, FoldState<kCrit> &f) {
+                           int64_t t0, const CuView &cu, const TrajView &tv, int blo, int bhi,
+                           FoldState<kCrit> &f) {
   Coefs<kCrit> k = f.k;
   df Bp = f.Bp, Bc = f.Bc;
   float Vn = f.Vn, P = f.P;
@@ -639,8 +699,8 @@ __device__ void fold_piece(const GaeArgs &a, const float *val, uint32_t tcol, in
         const float v = i == 3 ? vv[3] : (i == 2 ? vv[2] : (i == 1 ? vv[1] : vv[0]));
         if ((e4 >> i) & 1u) {  // last token of a trajectory: reset
           const int b = cu.find(blo, bhi, t0 + 4 * g + i);
-          k = load_coefs<kCrit>(a.coef, b);
-          P = __ldg(a.rewards + b);
+          k = tv.coefs<kCrit>(b);
+          P = tv.reward(b);
           Bp = Bc = {0.f, 0.f};
           Vn = 0.f;
           fl = 1;
@@ -668,13 +728,12 @@ __device__ void fold_piece(const GaeArgs &a, const float *val, uint32_t tcol, in
         Vn = on ? vv[i] : Vn;
         P = on ? 0.f : P;
       }
-      Bp = df_renorm(Bp);
-      if constexpr (kCrit) Bc = df_renorm(Bc);
       fl |= a4 ? 2 : 0;
     }
   }
   f.k = k;
-  f.Bp = Bp;
+  f.Bp = df_renorm(Bp);
+  if constexpr (kCrit) Bc = df_renorm(Bc);
   f.Bc = Bc;
   f.Vn = Vn;
   f.P = P;
@@ -719,7 +778,7 @@ struct ReplayState {
 // of `adv`, returns to its row of `ret`.
 template <bool kCrit>
 __device__ void replay_piece(const GaeArgs &a, uint32_t tcol, float *adv, float *ret, int lane, uint32_t act,
-                             uint32_t ends, int64_t t0, const CuView &cu, int blo, int bhi,
+                             uint32_t ends, int64_t t0, const CuView &cu, const TrajView &tv, int blo, int bhi,
                              ReplayState<kCrit> &rs) {
   Coefs<kCrit> k = rs.k;
   float R = rs.R;
@@ -745,8 +804,8 @@ __device__ void replay_piece(const GaeArgs &a, uint32_t tcol, float *adv, float 
         float o = 0.f, orv = 0.f;
         if ((e4 >> i) & 1u) {
           const int b = cu.find(blo, bhi, t0 + 4 * g + i);
-          k = load_coefs<kCrit>(a.coef, b);
-          R = __ldg(a.rewards + b);
+          k = tv.coefs<kCrit>(b);
+          R = tv.reward(b);
           st.Bp = st.Bc = {0.f, 0.f};
           st.Vn = 0.f;
           st.P = R;
@@ -785,8 +844,6 @@ __device__ void replay_piece(const GaeArgs &a, uint32_t tcol, float *adv, float 
         st.Vn = on ? vv[i] : st.Vn;
         st.P = on ? 0.f : st.P;
       }
-      st.Bp = df_renorm(st.Bp);
-      if constexpr (kCrit) st.Bc = df_renorm(st.Bc);
     }
     *vp = make_float4(ov[0], ov[1], ov[2], ov[3]);
     *rp = make_float4(orr[0], orr[1], orr[2], orr[3]);
@@ -794,6 +851,8 @@ __device__ void replay_piece(const GaeArgs &a, uint32_t tcol, float *adv, float 
   }
   rs.k = k;
   rs.R = R;
+  st.Bp = df_renorm(st.Bp);
+  if constexpr (kCrit) st.Bc = df_renorm(st.Bc);
   rs.st = st;
 }
 
@@ -820,13 +879,17 @@ __device__ __forceinline__ int take_chunk(const GaeArgs &a, int lane) {
 // ignores its right neighbour, its left-edge state). Nothing here waits on
 // another warp.
 template <bool kCrit>
-__device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane, int q, int slot, Pending<kCrit> &p) {
+__device__ void fold_chunk(const GaeArgs &a, const ScanMaps &mp, WarpBuf &w, uint32_t tmem, int lane, int q, int slot,
+                           uint32_t &phases, Pending<kCrit> &p) {
   const int seg = 32 * a.pieces;
   const int64_t c0 = int64_t(q) * kChunk * a.pieces;
   const int64_t s0 = c0 + int64_t(lane) * seg;  // the lane's segment
   const int64_t N = a.N;
-  const uint64_t pol = l2_evict_first();
-  stage_in(a, c0, seg, a.pieces - 1, lane, w.val[0], w.msk, pol);
+  const bool tma = chunk_tma(a, q);
+  const uint64_t pol = tc::l2_evict_first();
+  tc::fence_proxy_async_smem();  // this lane's reads of val and msk before the copies refill them
+  __syncwarp();
+  stage_in(a, mp, tma, q, c0, seg, a.pieces - 1, lane, w.val[0], w.msk, tc::smem_u32(&w.bar[0]), pol);
 
   // This chunk's slice of cu_seqlens, in shared memory when it fits.
   const int sub0 = q * a.pieces, sub1 = (q + 1) * a.pieces;
@@ -834,8 +897,14 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane
   const int bhi = sub1 < a.nsub ? __ldg(a.chunk_first + sub1) : a.B - 1;
   const int ncu = bhi - blo + 2;  // cu[blo .. bhi + 1]
   const CuView cu{a.cu, w.cu, blo, ncu <= kScanCuCap};
+  const TrajView tv{a.coef, a.rewards, w.coef, w.rew, blo, ncu - 1 <= kScanTrajCap};
   if (cu.in_smem)
     for (int i = lane; i < ncu; i += 32) w.cu[i] = __ldg(a.cu + blo + i);
+  if (tv.in_smem && lane < ncu - 1) {  // with the cu_seqlens slice, in one round trip
+    w.coef[lane][0] = __ldg(a.coef + 2 * (blo + lane));
+    if constexpr (kCrit) w.coef[lane][1] = __ldg(a.coef + 2 * (blo + lane) + 1);
+    w.rew[lane] = __ldg(a.rewards + blo + lane);
+  }
   __syncwarp();
   mark_ends(cu, blo, bhi, c0, seg, a.pieces, slot, lane, w);
 
@@ -843,7 +912,7 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane
   const int64_t s_end = (s0 + seg < N ? s0 + seg : N) - 1;
   const int b_seg = s0 < N ? cu.find(blo, bhi, s_end) : blo;
   FoldState<kCrit> f;
-  f.k = load_coefs<kCrit>(a.coef, b_seg);
+  f.k = tv.coefs<kCrit>(b_seg);
   f.Bp = f.Bc = {0.f, 0.f};
   f.Vn = f.P = 0.f;
   f.fl = 0;
@@ -851,16 +920,18 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane
 #pragma unroll 1
   for (int k = a.pieces - 1; k >= 0; --k) {
     const int cur = (a.pieces - 1 - k) & 1;
-    cp_async_wait_all();
-    __syncwarp();
+    stage_wait(a, tma, w, cur, phases);
     const uint32_t act = row_actions(w.msk, lane);
     w.act[slot + k][lane] = act;
+    tc::fence_proxy_async_smem();  // the reads of msk and of the other value buffer before the next copy
     __syncwarp();  // every lane has read the flags and finished the previous piece
-    if (k > 0) stage_in(a, c0, seg, k - 1, lane, w.val[cur ^ 1], w.msk, pol);
+    if (k > 0)
+      stage_in(a, mp, tma, q, c0, seg, k - 1, lane, w.val[cur ^ 1], w.msk, tc::smem_u32(&w.bar[cur ^ 1]), pol);
     const int64_t t0 = s0 + 32 * int64_t(k);
     // every lane folds (the token loops vote across the warp); a lane past N
     // has no flags and keeps its state
-    fold_piece<kCrit>(a, w.val[cur], tmem + 32 * (slot + k), lane, act, w.ends[slot + k][lane], t0, cu, blo, bhi, f);
+    fold_piece<kCrit>(a, w.val[cur], tmem + 32 * (slot + k), lane, act, w.ends[slot + k][lane], t0, cu, tv, blo, bhi,
+                      f);
   }
   tmem_wait_st();  // the values are in TMEM before the replay reads them
 
@@ -868,7 +939,7 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane
   GMap<kCrit> S = lane_map<kCrit>(f);
 #pragma unroll 1
   for (int d = 1; d < 32; d <<= 1) {
-    const GMap<kCrit> o = shfl_down_map<kCrit>(S, d);
+    const GMap<kCrit> o = shfl_down_map<kCrit, false>(S, d);
     if (lane + d < 32) S = compose<kCrit>(S, o);
   }
   GMap<kCrit> E = shfl_down_map<kCrit>(S, 1);  // lanes to my right within the chunk
@@ -895,8 +966,8 @@ __device__ void fold_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane
 // state, then replays the tokens piece by piece (right to left) from TMEM and
 // stores advantages and returns.
 template <bool kCrit>
-__device__ void replay_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int lane, const Pending<kCrit> &p,
-                             bool pipelined) {
+__device__ int replay_chunk(const GaeArgs &a, const ScanMaps &mp, WarpBuf &w, uint32_t tmem, int lane,
+                            const Pending<kCrit> &p, bool pipelined) {
   const int seg = 32 * a.pieces;
   const int64_t c0 = int64_t(p.q) * kChunk * a.pieces;
   const int64_t s0 = c0 + int64_t(lane) * seg;
@@ -904,28 +975,38 @@ __device__ void replay_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int la
   const bool reset = __shfl_sync(0xffffffffu, p.S.fl & 1, 0) != 0;  // lane 0 holds the chunk's map
   // the coefficients and reward of the lane's last trajectory, loaded while
   // the look-back runs
+  // Unless the next chunk has been folded since, the fold's copies of the
+  // chunk's cu_seqlens slice and trajectory table are still in shared memory.
+  const CuView cu{a.cu, w.cu, p.blo, !pipelined && p.bhi - p.blo + 2 <= kScanCuCap};
+  const TrajView tv{a.coef, a.rewards, w.coef, w.rew, p.blo, !pipelined && p.bhi - p.blo + 1 <= kScanTrajCap};
   ReplayState<kCrit> rs;
-  rs.k = load_coefs<kCrit>(a.coef, p.b_seg);
-  rs.R = __ldg(a.rewards + p.b_seg);
+  rs.k = tv.coefs<kCrit>(p.b_seg);
+  rs.R = tv.reward(p.b_seg);
   GState right = zero_state();
   if (!last) right = look_back<kCrit>(a, p.q, lane);
   if (lane == 0 && !reset && !last)
     publish_state<kCrit>(a.incl + size_t(p.q) * kStateWords<kCrit>, apply<kCrit>(p.S, right));
   // every lane replays (the token loops vote across the warp); rows past N
-  // are never stored. Unless the next chunk has been folded since, the
-  // fold's copy of the chunk's cu_seqlens slice is still in shared memory.
-  const CuView cu{a.cu, w.cu, p.blo, !pipelined && p.bhi - p.blo + 2 <= kScanCuCap};
+  // are never stored
   rs.st = apply<kCrit>(p.E, right);
+  const bool tma = chunk_tma(a, p.q);
+  const uint64_t pol = tc::l2_evict_first();
+  int t = 0;
 #pragma unroll 1
   for (int k = a.pieces - 1; k >= 0; --k) {
+    // one chunk at a time: the next ticket is taken before the last piece so
+    // that its round trip overlaps the piece. The chunk is folded right after
+    // this replay, which waits on nothing, so the tickets still only wait on
+    // chunks that are folded without waiting.
+    if (!pipelined && k == 0 && lane == 0) t = atomicAdd(a.ticket, 1);
     const uint32_t act = w.act[p.slot + k][lane];
     const int64_t t0 = s0 + 32 * int64_t(k);
     replay_piece<kCrit>(a, tmem + 32 * (p.slot + k), w.val[0], w.val[1], lane, act, w.ends[p.slot + k][lane], t0,
-                        cu, p.blo, p.bhi, rs);
+                        cu, tv, p.blo, p.bhi, rs);
     __syncwarp();
-    stage_out(a, c0, seg, k, lane, w.val[0], w.val[1]);
-    __syncwarp();  // every lane has read its granules before the next piece overwrites them
+    stage_out(a, mp, tma, p.q, c0, seg, k, lane, w.val[0], w.val[1], pol);
   }
+  return pipelined ? -1 : a.nchunks - 1 - __shfl_sync(0xffffffffu, t, 0);
 }
 
 // Persistent warps: a warp takes a chunk (ticket), folds and publishes it,
@@ -935,19 +1016,29 @@ __device__ void replay_chunk(const GaeArgs &a, WarpBuf &w, uint32_t tmem, int la
 // holds kTmemCols TMEM columns for the whole launch (four CTAs per SM take all
 // 512, so the allocation never waits on this kernel).
 template <bool kCrit, bool kPipe>
-__global__ void __launch_bounds__(kThreads, kMinBlocks) gae_scan_kernel(GaeArgs a) {
-  extern __shared__ __align__(16) unsigned char s_raw[];
+__global__ void __launch_bounds__(kThreads, kMinBlocks)
+    gae_scan_kernel(GaeArgs a, const __grid_constant__ ScanMaps mp) {
+  extern __shared__ __align__(1024) unsigned char s_raw[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  WarpBuf *wb = reinterpret_cast<WarpBuf *>(s_raw);
-  WarpBuf &w = wb[warp];
+  const uint32_t raw = tc::smem_u32(s_raw);
+  unsigned char *base = s_raw + (((raw + 1023u) & ~1023u) - raw);
+  WarpBuf &w = *reinterpret_cast<WarpBuf *>(base + size_t(warp) * kWarpBufBytes);
+  WarpBuf &w0 = *reinterpret_cast<WarpBuf *>(base);
+  if (lane == 0) {
+    tc::mbar_init(tc::smem_u32(&w.bar[0]), 1);
+    tc::mbar_init(tc::smem_u32(&w.bar[1]), 1);
+    w.abort = 0;
+    tc::fence_barrier_init();
+  }
+  uint32_t phases = 0;
   if (warp == 0) {
-    tc::tmem_alloc(static_cast<uint32_t>(__cvta_generic_to_shared(&wb[0].tmem)), kTmemCols);
+    tc::tmem_alloc(tc::smem_u32(&w0.tmem), kTmemCols);
     tc::tmem_relinquish();
   }
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
-  const uint32_t tmem = wb[0].tmem + (uint32_t(32 * warp) << 16);  // the warp's TMEM lanes
+  const uint32_t tmem = w0.tmem + (uint32_t(32 * warp) << 16);  // the warp's TMEM lanes
   if constexpr (kPipe) {
     // short segments: two chunks in flight, one per half of the warp's TMEM
     // columns; the warp folds a chunk before it looks back for the one it
@@ -962,8 +1053,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) gae_scan_kernel(GaeArgs 
 #pragma unroll 1
     for (int q = take_chunk(a, lane);; q = take_chunk(a, lane)) {
       Pending<kCrit> n;
-      if (q >= 0) fold_chunk<kCrit>(a, w, tmem, lane, q, half * (kMaxPieces / 2), n);
-      if (have) replay_chunk<kCrit>(a, w, tmem, lane, p, true);
+      if (q >= 0) fold_chunk<kCrit>(a, mp, w, tmem, lane, q, half * (kMaxPieces / 2), phases, n);
+      if (have) replay_chunk<kCrit>(a, mp, w, tmem, lane, p, true);
       if (q < 0) break;
       p = n;
       have = true;
@@ -974,17 +1065,18 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) gae_scan_kernel(GaeArgs 
     // per-chunk scan, look-back and set-up spread over 4096 tokens cost less
     // than the exposed wait)
 #pragma unroll 1
-    for (int q = take_chunk(a, lane); q >= 0; q = take_chunk(a, lane)) {
+    for (int q = take_chunk(a, lane); q >= 0;) {
       Pending<kCrit> p;
-      fold_chunk<kCrit>(a, w, tmem, lane, q, 0, p);
-      replay_chunk<kCrit>(a, w, tmem, lane, p, false);
+      fold_chunk<kCrit>(a, mp, w, tmem, lane, q, 0, phases, p);
+      q = replay_chunk<kCrit>(a, mp, w, tmem, lane, p, false);  // takes the next ticket
     }
   }
+  if (lane == 0) tc::bulk_wait_group<0>();  // the last stores are done
   tc::fence_before_sync();
   __syncthreads();
   if (warp == 0) {
     tc::fence_after_sync();
-    tc::tmem_dealloc(wb[0].tmem, kTmemCols);
+    tc::tmem_dealloc(w0.tmem, kTmemCols);
   }
 }
 
@@ -1015,11 +1107,11 @@ __global__ void gae_coef_kernel(const int32_t *cu, int B, int64_t N, float gamma
   coef[2 * b + 1] = make_float4(Ac.hi, Ac.lo, Gc.hi, Gc.lo);
 }
 
-constexpr size_t kScanSmem = sizeof(WarpBuf) * kWarps;
+constexpr size_t kScanSmem = kWarpBufBytes * kWarps + 1024;  // + alignment slack
 
 // The scan's shared memory exceeds the default 48 KB: opt in once per kernel
 // and device.
-sao_status set_scan_smem(void (*kern)(GaeArgs), int which, int device) {
+sao_status set_scan_smem(void (*kern)(GaeArgs, ScanMaps), int which, int device) {
   constexpr int kMaxDevices = 64;
   static std::once_flag once[4][kMaxDevices];
   static cudaError_t err[4][kMaxDevices];
@@ -1030,6 +1122,33 @@ sao_status set_scan_smem(void (*kern)(GaeArgs), int which, int device) {
   if (err[which][device] != cudaSuccess)
     return fail(SAO_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(err[which][device]));
   return SAO_OK;
+}
+
+// One map of a per-token array as [rows][seg] elements, box 32 x 32.
+bool scan_map(CUtensorMap *map, const void *ptr, CUtensorMapDataType type, size_t esize, int64_t rows, int seg,
+              CUtensorMapSwizzle swizzle) {
+  auto fn = tensor_map_encoder();
+  if (!fn || (reinterpret_cast<uintptr_t>(ptr) & 15u) != 0) return false;
+  cuuint64_t dims[2] = {cuuint64_t(seg), cuuint64_t(rows)};
+  cuuint64_t strides[1] = {cuuint64_t(seg) * esize};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, type, 2, const_cast<void *>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
+            CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// The tensor maps of the scan's per-token arrays over their N / seg whole
+// lane-segment rows; 0 rows (every piece staged element by element) when an
+// array is not 16-byte aligned or there is not one whole chunk.
+int64_t scan_maps(const float *values, const uint8_t *m, const float *adv, const float *ret, int64_t N, int seg,
+                  ScanMaps *maps) {
+  const int64_t rows = N / seg;
+  if (rows < 32) return 0;
+  const bool ok = scan_map(&maps->v, values, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, rows, seg, CU_TENSOR_MAP_SWIZZLE_128B) &&
+                  scan_map(&maps->m, m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, rows, seg, CU_TENSOR_MAP_SWIZZLE_32B) &&
+                  scan_map(&maps->adv, adv, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, rows, seg, CU_TENSOR_MAP_SWIZZLE_128B) &&
+                  scan_map(&maps->ret, ret, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, rows, seg, CU_TENSOR_MAP_SWIZZLE_128B);
+  return ok ? rows : 0;
 }
 
 }  // namespace
@@ -1124,6 +1243,8 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   a.ret = ret;
   a.err = err;
   a.wait_ns = scan_wait_ns();
+  ScanMaps maps;
+  a.tma_rows = scan_maps(values, m, adv, ret, N, 32 * pieces, &maps);
   DeviceInfo di;
   SAO_TRY(device_info(&di));
   // segments of 1 or 2 pieces: two chunks in flight per warp
@@ -1136,7 +1257,7 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   const int64_t resident = int64_t(di.sm_count) * kMinBlocks;
   const unsigned grid = unsigned(ctas < resident ? ctas : resident);
   int slot = launch_begin("gae_scan", s);
-  kern<<<grid, kThreads, kScanSmem, s>>>(a);
+  kern<<<grid, kThreads, kScanSmem, s>>>(a, maps);
   return launch_end(slot, s);
 }
 

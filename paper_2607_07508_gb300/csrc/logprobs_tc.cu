@@ -934,6 +934,8 @@ BwdPlan bwd_plan(int64_t N, int32_t h, int32_t V) {
 
 }  // namespace
 
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() { return encode_fn(); }
+
 // Workspace of the log-prob calls: the forward's row compaction, tile
 // partials and gathered logits; the backward's row compaction of one row
 // block, its dZ chunk buffer and fp32 dH accumulator (recompute path; the

@@ -1,6 +1,8 @@
 // Internal launcher interface between the C-ABI layer and the kernel files.
 #pragma once
 
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -25,6 +27,10 @@ sao_status decoupled_loss_launch(const float *logp, const float *prox, const flo
                                  float w_high, int64_t n_norm, float *loss, float *coef, uint8_t *flags,
                                  int64_t *counts, const float *grad_loss, void *ws_body, size_t body_bytes,
                                  cudaStream_t s);
+
+// logprobs_tc.cu: the driver's tensor-map encoder (null when the driver has
+// none), shared by every kernel that stages tiles with TMA
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder();
 
 // gae.cu ----------------------------------------------------------------------
 size_t gae_ws_bytes(int64_t N, int64_t B);
