@@ -1087,9 +1087,9 @@ __global__ void preset_ticket_kernel(int *ticket, int skip) { *ticket = skip; }
 
 // Per-trajectory coefficients (fp64 then split to double-float) and a check of
 // cu_seqlens: 0 = cu[0] <= cu[1] <= ... <= cu[B] = N.
-__global__ void gae_coef_kernel(const int32_t *cu, int B, int64_t N, float gamma, float lam, float lam_c,
-                                float alpha, const int *nact, float4 *coef, unsigned int *err) {
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+__device__ __forceinline__ void gae_coef_one(int b, const int32_t *cu, int B, int64_t N, float gamma, float lam,
+                                             float lam_c, float alpha, const int *nact, float4 *coef,
+                                             unsigned int *err) {
   if (b >= B) return;
   if ((b == 0 && cu[0] != 0) || cu[b + 1] < cu[b] || (b == B - 1 && int64_t(cu[B]) != N))
     raise_device_error(err, SAO_DEVERR_CU_SEQLENS);
@@ -1105,6 +1105,23 @@ __global__ void gae_coef_kernel(const int32_t *cu, int B, int64_t N, float gamma
   const df Ac = df_from_double(ac), Gc = df_from_double(g - ac);
   coef[2 * b] = make_float4(Ap.hi, Ap.lo, Gp.hi, Gp.lo);
   coef[2 * b + 1] = make_float4(Ac.hi, Ac.lo, Gc.hi, Gc.lo);
+}
+__global__ void gae_coef_kernel(const int32_t *cu, int B, int64_t N, float gamma, float lam, float lam_c,
+                                float alpha, const int *nact, float4 *coef, unsigned int *err) {
+  gae_coef_one(blockIdx.x * blockDim.x + threadIdx.x, cu, B, N, gamma, lam, lam_c, alpha, nact, coef, err);
+}
+// Both set-up passes in one launch when lambda does not depend on the action
+// counts (alpha = 0): CTAs [0, nfirst) find the first trajectory of every
+// 1024-token sub-chunk, the others compute the coefficients.
+__global__ void __launch_bounds__(seg::kChunkFirstThreads)
+    gae_prep_kernel(const int32_t *cu, int B, int64_t N, int nsub, int *chunk_first, unsigned nfirst, float gamma,
+                    float lam, float lam_c, float4 *coef, unsigned int *err) {
+  if (blockIdx.x < nfirst) {
+    seg::chunk_first_block(cu, B, N, nsub, chunk_first, int(blockIdx.x));
+    return;
+  }
+  gae_coef_one(int(blockIdx.x - nfirst) * seg::kChunkFirstThreads + threadIdx.x, cu, B, N, gamma, lam, lam_c, 0.f,
+               nullptr, coef, err);
 }
 
 constexpr size_t kScanSmem = kWarpBufBytes * kWarps + 1024;  // + alignment slack
@@ -1183,8 +1200,8 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   char *zero_begin = c.base + c.off;
   int *ticket = c.take<int>(1);
   int *nact = c.take<int>(size_t(B) + 1);
-  uint64_t *agg = c.take<uint64_t>(map_words * size_t(nchunks));
-  uint64_t *incl = c.take<uint64_t>(state_words * size_t(nchunks));
+  uint64_t *agg = c.take<uint64_t>(map_words * size_t(nscan));
+  uint64_t *incl = c.take<uint64_t>(state_words * size_t(nscan));
   char *zero_end = c.base + c.off;
   float4 *coef = c.take<float4>(2 * (size_t(B) + 1));
   int *chunk_first = c.take<int>(size_t(nchunks) + 1);
@@ -1194,35 +1211,37 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
     preset_ticket_kernel<<<1, 1, 0, s>>>(ticket, skip);
     SAO_CUDA_TRY(cudaGetLastError());
   }
-  {
+  if (alpha > 0.f) {
+    // lambda from each trajectory's action count: chunk_first, the count,
+    // then the coefficients
     int slot = launch_begin("gae_chunk_first", s);
     seg::chunk_first_kernel<<<seg::chunk_first_grid(int(nchunks)), seg::kChunkFirstThreads, 0, s>>>(
       cu, B, N, int(nchunks), chunk_first);
+    SAO_TRY(launch_end(slot, s));
+    slot = launch_begin("gae_count", s);
+    seg::action_count_kernel<<<seg::action_count_grid(int(nchunks)), 256, 0, s>>>(m, cu, B, N, int(nchunks),
+                                                                                    chunk_first, nact);
+    SAO_TRY(launch_end(slot, s));
+    slot = launch_begin("gae_coef", s);
+    gae_coef_kernel<<<(B + 127) / 128, 128, 0, s>>>(cu, B, N, gamma, lam, lam_c, alpha, nact, coef, err);
+    SAO_TRY(launch_end(slot, s));
+  } else {
+    const unsigned nfirst = seg::chunk_first_grid(int(nchunks));
+    const unsigned ncoef = unsigned((int64_t(B) + seg::kChunkFirstThreads - 1) / seg::kChunkFirstThreads);
+    int slot = launch_begin("gae_prep", s);
+    gae_prep_kernel<<<nfirst + ncoef, seg::kChunkFirstThreads, 0, s>>>(cu, B, N, int(nchunks), chunk_first, nfirst,
+                                                                       gamma, lam, lam_c, coef, err);
     SAO_TRY(launch_end(slot, s));
   }
   if (gamma == 1.0f && lam == 1.0f && lam_c == 1.0f && !(alpha > 0.f)) {
     // gamma = lambda = 1: every delta telescopes, A = R_b - V on the action
     // tokens and the return is R_b, exactly what the scan would produce (its
     // double-float lambda-return is R_b itself): one streaming pass, after
-    // the coefficient kernel's check of cu_seqlens
-    int slot = launch_begin("gae_coef", s);
-    gae_coef_kernel<<<(B + 127) / 128, 128, 0, s>>>(cu, B, N, gamma, lam, lam_c, alpha, nact, coef, err);
-    SAO_TRY(launch_end(slot, s));
-    slot = launch_begin("gae_telescoped", s);
+    // the set-up kernel's check of cu_seqlens
+    int slot = launch_begin("gae_telescoped", s);
     seg::traj_broadcast_kernel<true><<<seg::broadcast_grid(int(nchunks)), 256, 0, s>>>(
         rewards, m, cu, B, N, int(nchunks), chunk_first, adv, values, ret);
     return launch_end(slot, s);
-  }
-  if (alpha > 0.f) {
-    int slot = launch_begin("gae_count", s);
-    seg::action_count_kernel<<<seg::action_count_grid(int(nchunks)), 256, 0, s>>>(m, cu, B, N, int(nchunks),
-                                                                                    chunk_first, nact);
-    SAO_TRY(launch_end(slot, s));
-  }
-  {
-    int slot = launch_begin("gae_coef", s);
-    gae_coef_kernel<<<(B + 127) / 128, 128, 0, s>>>(cu, B, N, gamma, lam, lam_c, alpha, nact, coef, err);
-    SAO_TRY(launch_end(slot, s));
   }
   GaeArgs a;
   a.values = values;

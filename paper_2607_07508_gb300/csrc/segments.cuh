@@ -73,16 +73,16 @@ namespace {
 // chunk's first token t. The CTA stages the samples cu[k S] (S = ceil(B /
 // 4096)); a thread's search over them gives the k with cu[k S] <= t <
 // cu[(k + 1) S], so the answer lies in [k S, (k + 1) S) and only that short
-// range is searched in global memory. Grid: chunk_first_grid, block
-// kChunkFirstThreads.
-__global__ void __launch_bounds__(kChunkFirstThreads) chunk_first_kernel(const int32_t *cu, int B, int64_t N,
-                                                                        int nchunks, int *chunk_first) {
+// range is searched in global memory. `block` takes the chunks from
+// block * kChunkFirstThreads, one per thread of a kChunkFirstThreads CTA.
+__device__ __forceinline__ void chunk_first_block(const int32_t *cu, int B, int64_t N, int nchunks, int *chunk_first,
+                                                  int block) {
   __shared__ int32_t samp[kChunkFirstSample];
   const int S = B > kChunkFirstSample ? (B + kChunkFirstSample - 1) / kChunkFirstSample : 1;
   const int ns = (B + S - 1) / S;  // samples k S < B
   for (int k = threadIdx.x; k < ns; k += kChunkFirstThreads) samp[k] = __ldg(cu + int64_t(k) * S);
   __syncthreads();
-  const int q = blockIdx.x * kChunkFirstThreads + threadIdx.x;
+  const int q = block * kChunkFirstThreads + threadIdx.x;
   if (q >= nchunks) return;
   int64_t t = int64_t(q) * kSegChunk;
   if (t >= N) t = N - 1;
@@ -100,6 +100,11 @@ __global__ void __launch_bounds__(kChunkFirstThreads) chunk_first_kernel(const i
     else bhi = mid - 1;
   }
   chunk_first[q] = blo;
+}
+// Grid: chunk_first_grid, block kChunkFirstThreads.
+__global__ void __launch_bounds__(kChunkFirstThreads) chunk_first_kernel(const int32_t *cu, int B, int64_t N,
+                                                                        int nchunks, int *chunk_first) {
+  chunk_first_block(cu, B, N, nchunks, chunk_first, blockIdx.x);
 }
 
 // Number of action tokens per trajectory; nact must start at zero. One warp
