@@ -1111,17 +1111,24 @@ __global__ void gae_coef_kernel(const int32_t *cu, int B, int64_t N, float gamma
   gae_coef_one(blockIdx.x * blockDim.x + threadIdx.x, cu, B, N, gamma, lam, lam_c, alpha, nact, coef, err);
 }
 // Both set-up passes in one launch when lambda does not depend on the action
-// counts (alpha = 0): CTAs [0, nfirst) find the first trajectory of every
-// 1024-token sub-chunk, the others compute the coefficients.
-__global__ void __launch_bounds__(seg::kChunkFirstThreads)
-    gae_prep_kernel(const int32_t *cu, int B, int64_t N, int nsub, int *chunk_first, unsigned nfirst, float gamma,
-                    float lam, float lam_c, float4 *coef, unsigned int *err) {
-  if (blockIdx.x < nfirst) {
-    seg::chunk_first_block(cu, B, N, nsub, chunk_first, int(blockIdx.x));
-    return;
-  }
-  gae_coef_one(int(blockIdx.x - nfirst) * seg::kChunkFirstThreads + threadIdx.x, cu, B, N, gamma, lam, lam_c, 0.f,
-               nullptr, coef, err);
+// counts (alpha = 0), one thread per trajectory b: its coefficients and the
+// check of cu_seqlens, and the first trajectory of every 1024-token
+// sub-chunk that starts inside it (chunk_first[q] = b for cu[b] <= 1024 q <
+// cu[b + 1]: with a valid cu_seqlens every sub-chunk is written once).
+// chunk_first starts zeroed, so a malformed cu_seqlens (flagged here) still
+// leaves every entry a trajectory index.
+__global__ void __launch_bounds__(256) gae_prep_kernel(const int32_t *cu, int B, int64_t N, int nsub,
+                                                       int *chunk_first, float gamma, float lam, float lam_c,
+                                                       float4 *coef, unsigned int *err) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  gae_coef_one(b, cu, B, N, gamma, lam, lam_c, 0.f, nullptr, coef, err);
+  int64_t t0 = cu[b], t1 = cu[b + 1];
+  t0 = t0 < 0 ? 0 : (t0 > N ? N : t0);
+  t1 = t1 < 0 ? 0 : (t1 > N ? N : t1);
+  const int64_t q0 = (t0 + kChunk - 1) / kChunk, q1 = (t1 + kChunk - 1) / kChunk;
+#pragma unroll 1
+  for (int64_t q = q0; q < q1 && q < nsub; ++q) chunk_first[q] = b;
 }
 
 constexpr size_t kScanSmem = kWarpBufBytes * kWarps + 1024;  // + alignment slack
@@ -1196,15 +1203,15 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   const size_t map_words = crit_trivial ? kMapWords<false> : kMapWords<true>;
   const size_t state_words = crit_trivial ? kStateWords<false> : kStateWords<true>;
   Carver c(ws_body, body_bytes);
-  // ticket, action counts and the publication arrays start at zero
+  // ticket, action counts, the publication arrays and chunk_first start at zero
   char *zero_begin = c.base + c.off;
   int *ticket = c.take<int>(1);
   int *nact = c.take<int>(size_t(B) + 1);
   uint64_t *agg = c.take<uint64_t>(map_words * size_t(nscan));
   uint64_t *incl = c.take<uint64_t>(state_words * size_t(nscan));
+  int *chunk_first = c.take<int>(size_t(nchunks) + 1);
   char *zero_end = c.base + c.off;
   float4 *coef = c.take<float4>(2 * (size_t(B) + 1));
-  int *chunk_first = c.take<int>(size_t(nchunks) + 1);
   if (!c.ok()) return fail(SAO_ERR_WORKSPACE, "workspace too small for the advantage scan");
   SAO_CUDA_TRY(cudaMemsetAsync(zero_begin, 0, size_t(zero_end - zero_begin), s));
   if (const int skip = scan_skip(); skip > 0) {
@@ -1226,11 +1233,9 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
     gae_coef_kernel<<<(B + 127) / 128, 128, 0, s>>>(cu, B, N, gamma, lam, lam_c, alpha, nact, coef, err);
     SAO_TRY(launch_end(slot, s));
   } else {
-    const unsigned nfirst = seg::chunk_first_grid(int(nchunks));
-    const unsigned ncoef = unsigned((int64_t(B) + seg::kChunkFirstThreads - 1) / seg::kChunkFirstThreads);
     int slot = launch_begin("gae_prep", s);
-    gae_prep_kernel<<<nfirst + ncoef, seg::kChunkFirstThreads, 0, s>>>(cu, B, N, int(nchunks), chunk_first, nfirst,
-                                                                       gamma, lam, lam_c, coef, err);
+    gae_prep_kernel<<<(B + 255) / 256, 256, 0, s>>>(cu, B, N, int(nchunks), chunk_first, gamma, lam, lam_c, coef,
+                                                    err);
     SAO_TRY(launch_end(slot, s));
   }
   if (gamma == 1.0f && lam == 1.0f && lam_c == 1.0f && !(alpha > 0.f)) {
