@@ -98,6 +98,37 @@ def test_advantages_telescoped_edge_layouts(lengths, offset):
     assert rel_err_floor(ret.cpu().numpy(), want_r, 1e-3).max() <= ADV_TOL
 
 
+@pytest.mark.parametrize("lengths", [[1], [5, 0, 0, 7], [0, 4096, 1, 4095, 0], [4097, 13, 8190],
+                                     [3] * 2000, [70001], [0, 0, 17, 0], [0] * 3 + [300000, 0, 77777, 1] + [0] * 2])
+@pytest.mark.parametrize("offset", [0, 1])
+@pytest.mark.parametrize("gamma,lam,lam_c", [(1.0, 0.95, 1.0), (0.99, 0.9, 0.97)])
+def test_advantages_fixed_lambda_layouts(lengths, offset, gamma, lam, lam_c):
+    """A fixed lambda (alpha = 0) takes the one-launch set-up (a thread per
+    trajectory writes the chunk_first entries of the sub-chunks starting
+    inside it, so empty trajectories write none) and the scan; aligned inputs
+    take the tensor copies for whole chunks and plain loads for the ragged
+    end, inputs and outputs one element off 16-byte alignment take plain loads
+    and stores everywhere."""
+    wl = S.make_custom(lengths, 8, 16, "f32", seed=sum(lengths) + 11 * len(lengths), dense=False, obs_frac=0.4)
+    wl.loss_mask[::97] = 0
+    N = wl.N
+
+    def shifted(a, dtype):
+        t = torch.zeros(N + offset, dtype=dtype, device="cuda")
+        t[offset:] = torch.as_tensor(a).to(dtype).cuda()
+        return t[offset:]
+
+    v, m = shifted(wl.values, torch.float32), shifted(wl.loss_mask, torch.uint8)
+    adv = torch.full((N + offset,), float("nan"), device="cuda")[offset:]
+    ret = torch.full((N + offset,), float("nan"), device="cuda")[offset:]
+    g, l, lc = f32(gamma), f32(lam), f32(lam_c)
+    sao.sao_advantages(v, cuda(wl.rewards), m, cuda(wl.cu_seqlens), g, l, lc, 0.0, adv, ret, sao.workspace(N))
+    torch.cuda.synchronize()
+    want_a, want_r = O.advantages(wl.values, wl.rewards, wl.loss_mask, wl.cu_seqlens, g, l, lc, 0.0)
+    assert rel_err_floor(adv.cpu().numpy(), want_a, 1e-3).max() <= ADV_TOL
+    assert rel_err_floor(ret.cpu().numpy(), want_r, 1e-3).max() <= ADV_TOL
+
+
 def test_advantages_no_action_tokens_and_empty():
     wl = S.make_custom([10, 0, 300], 8, 16, "f32", seed=3, dense=False)
     wl.loss_mask[:] = 0
@@ -143,6 +174,37 @@ def test_advantages_long_lane_segments(N):
                                 g["gamma"], g["lam"], g["lam_c"], g["alpha"])
             assert rel_err_floor(adv[lo:hi], a, 1e-3).max() <= ADV_TOL
             assert rel_err_floor(ret[lo:hi], r, 1e-3).max() <= ADV_TOL
+
+
+def test_advantages_misaligned_4_piece_mode():
+    """2^26 + 999 tokens (4-piece lane segments, one chunk per warp) with
+    values, mask and outputs one element off 16-byte alignment: no tensor
+    maps, every piece staged with plain loads and stored with plain stores;
+    sampled trajectories and the ragged tail against the oracle."""
+    N = (1 << 26) + 999
+    wl = S.bandwidth_workload(N=N, B=N >> 13)
+    off = 1
+
+    def shifted(a, dtype):
+        t = torch.zeros(N + off, dtype=dtype, device="cuda")
+        t[off:] = torch.as_tensor(a).to(dtype).cuda()
+        return t[off:]
+
+    v, m = shifted(wl.values, torch.float32), shifted(wl.loss_mask, torch.uint8)
+    adv = torch.full((N + off,), float("nan"), device="cuda")[off:]
+    ret = torch.full((N + off,), float("nan"), device="cuda")[off:]
+    g, l = f32(1.0), f32(0.95)
+    sao.sao_advantages(v, cuda(wl.rewards), m, cuda(wl.cu_seqlens), g, l, 1.0, 0.0, adv, ret, sao.workspace(N))
+    torch.cuda.synchronize()
+    adv, ret = adv.cpu().numpy(), ret.cpu().numpy()
+    rng = np.random.default_rng(7)
+    picks = np.concatenate([rng.choice(wl.B, size=32, replace=False), [wl.B - 2, wl.B - 1]])
+    for b in picks:
+        lo, hi = wl.cu_seqlens[b], wl.cu_seqlens[b + 1]
+        a, r = O.advantages(wl.values[lo:hi], wl.rewards[b:b + 1], wl.loss_mask[lo:hi], np.array([0, hi - lo]),
+                            g, l, 1.0, 0.0)
+        assert rel_err_floor(adv[lo:hi], a, 1e-3).max() <= ADV_TOL
+        assert rel_err_floor(ret[lo:hi], r, 1e-3).max() <= ADV_TOL
 
 
 def test_advantages_short_trajectories_random_masks():
