@@ -118,7 +118,8 @@ SAO_API int sao_get_cta_pairs(void);
  * Test hooks of the advantage scan (process-wide; defaults restored by
  * (0, 0)): every look-back wait gives up after wait_ns nanoseconds (0: the
  * default 2 s; longer values are capped at it), and the scan's top
- * skip_chunks 1024-token chunks are never processed, so the chunks below them
+ * skip_chunks chunks (of 1024, 2048 or 4096 tokens, chosen from N) are never
+ * processed, so the chunks below them
  * wait for a carry that never comes. Failure-detection tests use them to make
  * the bounded wait run out: the call still completes, the context stays
  * usable, and checked mode reports SAO_DEVERR_SCAN_TIMEOUT. Not for
@@ -207,6 +208,8 @@ SAO_API sao_status sao_token_logprobs_bwd_cached(const void *H, const void *W, s
  *   cu_seqlens [B+1] int32 with 0 = cu[0] <= ... <= cu[B] = N
  *   adv, ret [N] fp32 outputs
  * Scalars: 0 <= gamma, lambda_policy, lambda_critic <= 1.
+ * Arrays that start 16-byte aligned move by TMA tensor copies; other
+ * alignments are staged element by element (same results, slower).
  * The scan keeps each chunk's values in TMEM between its two passes: while it
  * runs, each SM's 512 TMEM columns are held by its CTAs, so a kernel on
  * another stream that allocates TMEM on the same SM waits for them (and the
