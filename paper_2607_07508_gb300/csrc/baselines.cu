@@ -378,12 +378,14 @@ __device__ int run_edge(const int32_t *gid, int B, int b, int g, int dir, int la
 }
 
 __global__ void __launch_bounds__(256) group_norm_kernel(const float *R, const int32_t *gid, int B, float eps,
-                                                         const int *sorted, float *a_traj) {
+                                                         const int *sorted, float *a_traj, const int32_t *cu,
+                                                         int64_t N, int nchunks, int *chunk_first) {
   __shared__ int32_t sg[kTile];
   __shared__ float sr[kTile];
   __shared__ int s_range[2];
   const int lane = threadIdx.x & 31;
   const int b = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (b < B) seg::chunk_first_of(cu, b, N, nchunks, chunk_first, lane, 32);  // for the broadcast
   const int g = b < B ? gid[b] : 0;
   // The entries to visit: the whole batch, or with non-decreasing ids the runs
   // of this CTA's groups (the same members in the same lane order, so the same
@@ -538,10 +540,12 @@ __global__ void __launch_bounds__(256) rank_scan_kernel(int *table, int nblk, in
 __global__ void __launch_bounds__(256) running_mean_kernel(const float *R, const int32_t *pid, int B, int P,
                                                            const int *table, const float *history,
                                                            const long long *seen, int window, float *a_traj,
-                                                           long long *rec, int *rank) {
+                                                           long long *rec, int *rank, const int32_t *cu, int64_t N,
+                                                           int nchunks, int *chunk_first) {
   const int lane = threadIdx.x & 31;
   const int b = blockIdx.x * 8 + (threadIdx.x >> 5);
   if (b >= B) return;
+  seg::chunk_first_of(cu, b, N, nchunks, chunk_first, lane, 32);  // for the broadcast
   const int p = pid[b];
   if (p < 0 || p >= P) {  // outside [0, num_prompts): no window to read, advantage 0
     if (lane == 0) {
@@ -671,11 +675,12 @@ sao_status clip_loss_launch(const float *logp, const float *old, const float *ad
     if (counts) SAO_CUDA_TRY(cudaMemsetAsync(counts, 0, 4 * sizeof(int64_t), s));
     return SAO_OK;
   }
-  SAO_CUDA_TRY(cudaMemsetAsync(nact, 0, sizeof(int) * size_t(B), s));
+  // chunk_first and nact start at zero (one memset: nact follows chunk_first)
+  SAO_CUDA_TRY(cudaMemsetAsync(chunk_first, 0, size_t(reinterpret_cast<char *>(nact + B) -
+                                                       reinterpret_cast<char *>(chunk_first)), s));
   const unsigned grid = unsigned((nchunks + kWarps - 1) / kWarps);
   int slot = launch_begin("clip_loss_counts", s);
-  seg::chunk_first_kernel<<<seg::chunk_first_grid(int(nchunks)), seg::kChunkFirstThreads, 0, s>>>(
-      cu, B, N, int(nchunks), chunk_first);
+  seg::chunk_first_kernel<<<seg::chunk_first_grid(B), 256, 0, s>>>(cu, B, N, int(nchunks), chunk_first);
   seg::action_count_kernel<<<seg::action_count_grid(int(nchunks)), 256, 0, s>>>(m, cu, B, N, int(nchunks),
                                                                                 chunk_first, nact);
   norms_kernel<<<1, kNormThreads, 0, s>>>(nact, B, norms);
@@ -713,14 +718,13 @@ sao_status clip_loss_launch(const float *logp, const float *old, const float *ad
   return launch_end(slot, s);
 }
 
-// adv[t] = a_traj[trajectory of t] on action tokens, 0 elsewhere, all N tokens.
+// adv[t] = a_traj[trajectory of t] on action tokens, 0 elsewhere, all N tokens
+// (chunk_first written by the per-trajectory pass before it).
 static sao_status broadcast_launch(const float *a_traj, const uint8_t *m, const int32_t *cu, int32_t B, int64_t N,
-                                   int *chunk_first, float *adv, cudaStream_t s) {
+                                   const int *chunk_first, float *adv, cudaStream_t s) {
   if (N == 0) return SAO_OK;
   const int64_t nchunks = (N + kSegChunk - 1) / kSegChunk;
   int slot = launch_begin("adv_broadcast", s);
-  seg::chunk_first_kernel<<<seg::chunk_first_grid(int(nchunks)), seg::kChunkFirstThreads, 0, s>>>(
-      cu, B, N, int(nchunks), chunk_first);
   seg::traj_broadcast_kernel<false><<<seg::broadcast_grid(int(nchunks)), 256, 0, s>>>(
       a_traj, m, cu, B, N, int(nchunks), chunk_first, adv, nullptr, nullptr);
   return launch_end(slot, s);
@@ -737,11 +741,16 @@ sao_status group_adv_launch(const float *rewards, const int32_t *gid, int32_t B,
     if (N > 0) SAO_CUDA_TRY(cudaMemsetAsync(adv, 0, sizeof(float) * size_t(N), s));
     return SAO_OK;
   }
-  SAO_CUDA_TRY(cudaMemsetAsync(sorted, 0, sizeof(int), s));
+  // chunk_first (written by the group pass for the broadcast) and the flag
+  // start at zero, then the flag is set to 1 (sorted until shown otherwise)
+  SAO_CUDA_TRY(cudaMemsetAsync(chunk_first, 0, size_t(reinterpret_cast<char *>(sorted + 1) -
+                                                       reinterpret_cast<char *>(chunk_first)), s));
   SAO_CUDA_TRY(cudaMemsetAsync(sorted, 1, 1, s));  // the int 1
+  const int nchunks = int((N + kSegChunk - 1) / kSegChunk);
   int slot = launch_begin("group_advantages", s);
   group_sorted_kernel<<<unsigned((B + 255) / 256), 256, 0, s>>>(gid, B, sorted);
-  group_norm_kernel<<<unsigned((B + 7) / 8), 256, 0, s>>>(rewards, gid, B, eps, sorted, a_traj);
+  group_norm_kernel<<<unsigned((B + 7) / 8), 256, 0, s>>>(rewards, gid, B, eps, sorted, a_traj, cu, N, nchunks,
+                                                          chunk_first);
   SAO_TRY(launch_end(slot, s));
   return broadcast_launch(a_traj, m, cu, B, N, chunk_first, adv, s);
 }
@@ -770,6 +779,9 @@ sao_status running_mean_launch(const float *rewards, const int32_t *pid, int32_t
       rank = rk;
     }
   }
+  const int nchunks = int((N + kSegChunk - 1) / kSegChunk);
+  // chunk_first (written by the per-trajectory pass for the broadcast) starts at zero
+  SAO_CUDA_TRY(cudaMemsetAsync(chunk_first, 0, sizeof(int) * (size_t(nchunks) + 1), s));
   int slot = launch_begin("running_mean_advantages", s);
   if (table) {
     rank_count_kernel<<<unsigned(nblk), 256, 0, s>>>(pid, B, P, table);
@@ -777,7 +789,8 @@ sao_status running_mean_launch(const float *rewards, const int32_t *pid, int32_t
   }
   const unsigned g = unsigned((B + 7) / 8);  // a warp per trajectory
   running_mean_kernel<<<g, 256, 0, s>>>(rewards, pid, B, P, table, history,
-                                        reinterpret_cast<const long long *>(seen), window, a_traj, rec, rank);
+                                        reinterpret_cast<const long long *>(seen), window, a_traj, rec, rank, cu,
+                                        N, nchunks, chunk_first);
   running_mean_record_kernel<<<g, 256, 0, s>>>(rewards, pid, B, P, table ? table + int64_t(nblk) * P : nullptr,
                                                rank, rec, history, reinterpret_cast<long long *>(seen), window);
   SAO_TRY(launch_end(slot, s));

@@ -1123,12 +1123,7 @@ __global__ void __launch_bounds__(256) gae_prep_kernel(const int32_t *cu, int B,
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
   gae_coef_one(b, cu, B, N, gamma, lam, lam_c, 0.f, nullptr, coef, err);
-  int64_t t0 = cu[b], t1 = cu[b + 1];
-  t0 = t0 < 0 ? 0 : (t0 > N ? N : t0);
-  t1 = t1 < 0 ? 0 : (t1 > N ? N : t1);
-  const int64_t q0 = (t0 + kChunk - 1) / kChunk, q1 = (t1 + kChunk - 1) / kChunk;
-#pragma unroll 1
-  for (int64_t q = q0; q < q1 && q < nsub; ++q) chunk_first[q] = b;
+  seg::chunk_first_of(cu, b, N, nsub, chunk_first);
 }
 
 constexpr size_t kScanSmem = kWarpBufBytes * kWarps + 1024;  // + alignment slack
@@ -1222,8 +1217,7 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
     // lambda from each trajectory's action count: chunk_first, the count,
     // then the coefficients
     int slot = launch_begin("gae_chunk_first", s);
-    seg::chunk_first_kernel<<<seg::chunk_first_grid(int(nchunks)), seg::kChunkFirstThreads, 0, s>>>(
-      cu, B, N, int(nchunks), chunk_first);
+    seg::chunk_first_kernel<<<seg::chunk_first_grid(B), 256, 0, s>>>(cu, B, N, int(nchunks), chunk_first);
     SAO_TRY(launch_end(slot, s));
     slot = launch_begin("gae_count", s);
     seg::action_count_kernel<<<seg::action_count_grid(int(nchunks)), 256, 0, s>>>(m, cu, B, N, int(nchunks),

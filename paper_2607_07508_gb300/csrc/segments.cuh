@@ -15,14 +15,6 @@ constexpr int kCuCap = 128;              // cu_seqlens entries staged per warp
 constexpr int kCountChunks = 8;          // chunks per warp in action_count_kernel
 constexpr int kCastChunks = 2;           // chunks per warp in traj_broadcast_kernel
 
-// chunk_first_kernel: one chunk per thread, 1024 threads per CTA, and a
-// sample of every ceil(B / 4096)-th cu_seqlens entry in shared memory.
-constexpr int kChunkFirstThreads = 1024;
-constexpr int kChunkFirstSample = 4096;
-__host__ __device__ constexpr unsigned chunk_first_grid(int nchunks) {
-  return unsigned((nchunks + kChunkFirstThreads - 1) / kChunkFirstThreads);
-}
-
 // CTAs (of 8 warps) of action_count_kernel for nchunks chunks.
 __host__ __device__ constexpr unsigned action_count_grid(int nchunks) {
   return unsigned((nchunks + 8 * kCountChunks - 1) / (8 * kCountChunks));
@@ -69,43 +61,30 @@ __device__ __forceinline__ CuView stage_chunk(const int32_t *cu, int B, int nchu
 // includes this header launches its own copy.
 namespace {
 
-// First trajectory of every warp chunk: the largest b with cu[b] <= t for the
-// chunk's first token t. The CTA stages the samples cu[k S] (S = ceil(B /
-// 4096)); a thread's search over them gives the k with cu[k S] <= t <
-// cu[(k + 1) S], so the answer lies in [k S, (k + 1) S) and only that short
-// range is searched in global memory. `block` takes the chunks from
-// block * kChunkFirstThreads, one per thread of a kChunkFirstThreads CTA.
-__device__ __forceinline__ void chunk_first_block(const int32_t *cu, int B, int64_t N, int nchunks, int *chunk_first,
-                                                  int block) {
-  __shared__ int32_t samp[kChunkFirstSample];
-  const int S = B > kChunkFirstSample ? (B + kChunkFirstSample - 1) / kChunkFirstSample : 1;
-  const int ns = (B + S - 1) / S;  // samples k S < B
-  for (int k = threadIdx.x; k < ns; k += kChunkFirstThreads) samp[k] = __ldg(cu + int64_t(k) * S);
-  __syncthreads();
-  const int q = block * kChunkFirstThreads + threadIdx.x;
-  if (q >= nchunks) return;
-  int64_t t = int64_t(q) * kSegChunk;
-  if (t >= N) t = N - 1;
-  int lo = 0, hi = ns - 1;
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (int64_t(samp[mid]) <= t) lo = mid;
-    else hi = mid - 1;
-  }
-  int blo = lo * S;
-  int bhi = blo + S - 1 < B - 1 ? blo + S - 1 : B - 1;
-  while (blo < bhi) {
-    const int mid = (blo + bhi + 1) >> 1;
-    if (int64_t(__ldg(cu + mid)) <= t) blo = mid;
-    else bhi = mid - 1;
-  }
-  chunk_first[q] = blo;
+// First trajectory of every warp chunk, by trajectory: chunk q gets b when
+// its first token lies in b (cu[b] <= q * kSegChunk < cu[b + 1]), so with a
+// valid cu_seqlens every chunk is written once, by the one trajectory holding
+// its first token (empty trajectories write none). chunk_first must start
+// zeroed: a malformed cu_seqlens then still leaves every entry a trajectory
+// index, so the passes that read it stay inside cu_seqlens.
+// `first`, `step`: the entries one thread writes (0, 1 alone; lane, 32 for a
+// warp sharing one trajectory).
+__device__ __forceinline__ void chunk_first_of(const int32_t *cu, int b, int64_t N, int nchunks, int *chunk_first,
+                                               int first = 0, int step = 1) {
+  int64_t t0 = cu[b], t1 = cu[b + 1];
+  t0 = t0 < 0 ? 0 : (t0 > N ? N : t0);
+  t1 = t1 < 0 ? 0 : (t1 > N ? N : t1);
+  const int64_t q0 = (t0 + kSegChunk - 1) / kSegChunk, q1 = (t1 + kSegChunk - 1) / kSegChunk;
+#pragma unroll 1
+  for (int64_t q = q0 + first; q < q1 && q < nchunks; q += step) chunk_first[q] = b;
 }
-// Grid: chunk_first_grid, block kChunkFirstThreads.
-__global__ void __launch_bounds__(kChunkFirstThreads) chunk_first_kernel(const int32_t *cu, int B, int64_t N,
-                                                                        int nchunks, int *chunk_first) {
-  chunk_first_block(cu, B, N, nchunks, chunk_first, blockIdx.x);
+// One thread per trajectory. Grid: (B + 255) / 256 CTAs of 256 threads.
+__global__ void __launch_bounds__(256) chunk_first_kernel(const int32_t *cu, int B, int64_t N, int nchunks,
+                                                          int *chunk_first) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b < B) chunk_first_of(cu, b, N, nchunks, chunk_first);
 }
+__host__ __device__ constexpr unsigned chunk_first_grid(int B) { return unsigned((B + 255) / 256); }
 
 // Number of action tokens per trajectory; nact must start at zero. One warp
 // per kCountChunks consecutive chunks, 8 warps per CTA (grid:
