@@ -512,7 +512,6 @@ struct TrajView {
 __device__ __forceinline__ int fgran(int r, int j) { return 8 * r + (j ^ (r & 7)); }
 __device__ __forceinline__ int mgran(int r, int j) { return 2 * r + (j ^ ((r >> 2) & 1)); }
 
-
 // The lane's 4 TMEM columns from `taddr` (lane field: the warp's TMEM lanes).
 __device__ __forceinline__ void tmem_st4(uint32_t taddr, float4 v) {
   asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr),
