@@ -1186,12 +1186,14 @@ sao_status gae_launch(const float *values, const float *rewards, const uint8_t *
   // 1024-token sub-chunks (the units of chunk_first and of the count and
   // broadcast passes) and the scan's chunks of 32 lane segments of
   // 32 * pieces tokens: longer segments spread the warp scan and look-back of
-  // a chunk over more tokens, as long as the scan keeps about 16k chunks to
-  // share out (pieces from N alone, so every device gives the same bits)
+  // a chunk over more tokens, as long as the scan keeps enough chunks to
+  // share out: 2 pieces from 2^23 tokens (4,096 chunks of 2,048), 4 from 2^25
+  // (8,192 of 4,096); measured at 2^23 / 2^24 tokens, 1 piece 49 / 82 us,
+  // 2 pieces 39 / 62 us, 4 pieces - / 64 us. Pieces come from N alone, so
+  // every device gives the same bits.
   const int64_t nchunks = (N + kChunk - 1) / kChunk;
   if (nchunks > (int64_t(1) << 30)) return fail(SAO_ERR_SHAPE, "too many tokens for the advantage scan");
-  int pieces = 1;
-  while (pieces < kMaxPieces && (N >> 24) >= 2 * pieces) pieces *= 2;
+  const int pieces = N >= (int64_t(1) << 25) ? 4 : (N >= (int64_t(1) << 23) ? 2 : 1);
   const int64_t nscan = (N + int64_t(kChunk) * pieces - 1) / (int64_t(kChunk) * pieces);
   const bool crit_trivial = (gamma == 1.0f && lam_c == 1.0f);
   const size_t map_words = crit_trivial ? kMapWords<false> : kMapWords<true>;

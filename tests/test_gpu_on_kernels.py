@@ -157,12 +157,13 @@ def test_advantages_bandwidth_size_properties():
         assert rel_err_floor(ret[lo:hi], r, 1e-3).max() <= ADV_TOL
 
 
-@pytest.mark.parametrize("N", [1 << 25, (1 << 26) + 12345])
+@pytest.mark.parametrize("N", [(1 << 23) + 4321, (1 << 24) + 77, 1 << 25, (1 << 26) + 12345])
 def test_advantages_long_lane_segments(N):
-    """From 2^25 tokens on, the scan's lanes own 64-256-token segments streamed
-    in 32-token pieces: 64 sampled trajectories and the last two (the ragged
-    tail) against the oracle, with lambda = 0.95 and with the length-adaptive
-    lambda and lambda_critic < 1."""
+    """From 2^23 tokens on, the scan's lanes own 64-token segments (two chunks
+    in flight per warp), from 2^25 on 128-token segments (one chunk at a
+    time), streamed in 32-token pieces: 64 sampled trajectories and the last
+    two (the ragged tail) against the oracle, with lambda = 0.95 and with the
+    length-adaptive lambda and lambda_critic < 1."""
     wl = S.bandwidth_workload(N=N, B=max(1, N >> 13))
     rng = np.random.default_rng(N % 1000)
     picks = np.concatenate([rng.choice(wl.B, size=64, replace=False), [wl.B - 2, wl.B - 1]])
@@ -208,7 +209,7 @@ def test_advantages_misaligned_4_piece_mode():
 
 
 def test_advantages_short_trajectories_random_masks():
-    """4-piece lane segments (2^26 tokens and more, one chunk per warp in all
+    """4-piece lane segments (2^25 tokens and more, one chunk per warp in all
     of its TMEM columns) with ~512-token trajectories and token-by-token random
     masks: many trajectory ends inside each piece (the per-token path) and
     mixed 4-token groups; sampled trajectories and the ragged tail against the
