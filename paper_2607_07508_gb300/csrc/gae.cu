@@ -972,12 +972,12 @@ __device__ int replay_chunk(const GaeArgs &a, const ScanMaps &mp, WarpBuf &w, ui
   const int64_t s0 = c0 + int64_t(lane) * seg;
   const bool last = (p.q == a.nchunks - 1);
   const bool reset = __shfl_sync(0xffffffffu, p.S.fl & 1, 0) != 0;  // lane 0 holds the chunk's map
-  // the coefficients and reward of the lane's last trajectory, loaded while
-  // the look-back runs
   // Unless the next chunk has been folded since, the fold's copies of the
   // chunk's cu_seqlens slice and trajectory table are still in shared memory.
   const CuView cu{a.cu, w.cu, p.blo, !pipelined && p.bhi - p.blo + 2 <= kScanCuCap};
   const TrajView tv{a.coef, a.rewards, w.coef, w.rew, p.blo, !pipelined && p.bhi - p.blo + 1 <= kScanTrajCap};
+  // the coefficients and reward of the lane's last trajectory, loaded while
+  // the look-back runs
   ReplayState<kCrit> rs;
   rs.k = tv.coefs<kCrit>(p.b_seg);
   rs.R = tv.reward(p.b_seg);
